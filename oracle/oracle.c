@@ -1,0 +1,189 @@
+/*
+ * ORACLE — TEST INFRASTRUCTURE ONLY.
+ *
+ * A plain, slow, fp64 CPU statement of the embedding-adapter visual-memory build of
+ * "Just MLPs: Efficient Visual State Reconstruction for Multimodal Language Models"
+ * (delta-Vision). Only the tests, the smoke check and the benchmark's CPU-baseline leg
+ * may load it. It shares no code, header, table or helper with the CUDA path.
+ *
+ * What it computes, for every visual token row x = E_i (a row of the initial visual
+ * embeddings, Sec. 2 Eq. 1) and every layer l, in this order:
+ *   z = x D_l                          Sec. 3.1 Eq. 4: D_l in R^{d x r}; stored [r][d]
+ *   h = phi(z), phi = SiLU             Sec. 3.1 Eq. 4: phi(u) = u / (1 + exp(-u))
+ *   m = x + h U_l                      Sec. 3.1 Eqs. 4-5: M_l = E + Delta_l(E); U_l in
+ *                                      R^{r x d}, stored [d][r]
+ *   n = gamma_l * m / sqrt(mean(m^2) + eps)
+ *                                      Sec. 3.2 Eq. 7 applies the frozen input norm LN_l;
+ *                                      App. K names it RMSNorm (learnable gain, no centring)
+ *   k = W_K,l n (+ b_K,l), v = W_V,l n (+ b_V,l)
+ *                                      Sec. 3.2 Eq. 7: K^v_l = W_K,l LN_l(M_l), same for V;
+ *                                      W stored [kv][d]; the bias is the backbone's, if any
+ *   k <- RoPE(k, positions of token i) Sec. 3.2 keeps the original causal attention and
+ *                                      Sec. 1 / App. H keep the visual positions, so the
+ *                                      backbone's rotary embedding is applied to visual keys
+ *                                      at their original positions; V is not rotated.
+ * RoPE reading: rotate-half pairs (j, j + D_h/2) of each head, inverse frequency
+ * theta^(-2j/D_h); the angle of pair j is p * theta^(-2j/D_h), where p is the 1-D
+ * position, or for M-RoPE the (t, h, w) position selected by the contiguous section
+ * that j falls in (sections s0, s1, s2 with s0 + s1 + s2 = D_h / 2).
+ *
+ * Every input is a bf16 bit pattern widened exactly to double; every step runs in double.
+ * Tokens are independent of each other (every step above acts on one row), so the only
+ * parallelism is an OpenMP loop over the requested tokens.
+ */
+#include <math.h>
+#include <omp.h>
+#include <stdint.h>
+#include <stdlib.h>
+#include <string.h>
+
+typedef struct {
+  int d;               /* hidden size */
+  int n_layers;        /* L */
+  int n_kv_heads;      /* H_kv */
+  int head_dim;        /* D_h */
+  int rank;            /* r */
+  int rope;            /* 0: 1-D RoPE, 1: M-RoPE (t, h, w) */
+  double rope_theta;
+  int mrope_section[3];
+  double rms_eps;
+} oracle_cfg;
+
+static double bf16_to_f64(uint16_t b) {
+  uint32_t u = ((uint32_t)b) << 16;
+  float f;
+  memcpy(&f, &u, 4);
+  return (double)f;
+}
+
+/* phi of Sec. 3.1 Eq. 4: SiLU(u) = u * sigmoid(u) = u / (1 + e^-u). */
+double oracle_silu(double u) { return u / (1.0 + exp(-u)); }
+
+/* Adapter of Sec. 3.1 Eqs. 4-5 for one token row and one layer.
+ * x[d] in; Dl = D_l stored [r][d]; Ul = U_l stored [d][r]; z[r], h[r], m[d] out. */
+void oracle_adapter_row(int d, int r, const double* x, const uint16_t* Dl, const uint16_t* Ul,
+                        double* z, double* h, double* m) {
+  for (int k = 0; k < r; ++k) {
+    double s = 0.0;
+    for (int j = 0; j < d; ++j) s += x[j] * bf16_to_f64(Dl[(int64_t)k * d + j]);
+    z[k] = s;
+    h[k] = oracle_silu(s);
+  }
+  for (int j = 0; j < d; ++j) {
+    double s = 0.0;
+    for (int k = 0; k < r; ++k) s += h[k] * bf16_to_f64(Ul[(int64_t)j * r + k]);
+    m[j] = x[j] + s;
+  }
+}
+
+/* RMSNorm with gain (LN_l of Sec. 3.2 Eq. 7; RMSNorm per App. K):
+ * n_j = gamma_j * m_j / sqrt((1/d) sum_i m_i^2 + eps). */
+void oracle_rmsnorm_row(int d, const double* m, const double* gamma, double eps, double* n) {
+  double ss = 0.0;
+  for (int j = 0; j < d; ++j) ss += m[j] * m[j];
+  double inv = 1.0 / sqrt(ss / (double)d + eps);
+  for (int j = 0; j < d; ++j) n[j] = gamma[j] * m[j] * inv;
+}
+
+/* One projection of Sec. 3.2 Eq. 7: out = W n (+ b), W stored [kv][d], b [kv] or NULL. */
+void oracle_project_row(int d, int kv, const uint16_t* W, const uint16_t* b, const double* n,
+                        double* out) {
+  for (int c = 0; c < kv; ++c) {
+    double s = 0.0;
+    for (int j = 0; j < d; ++j) s += bf16_to_f64(W[(int64_t)c * d + j]) * n[j];
+    out[c] = s + (b ? bf16_to_f64(b[c]) : 0.0);
+  }
+}
+
+/* Rotary position embedding of one head (rotate-half pairs (j, j + D/2)).
+ * pos3 holds the position of each axis: pos3[0] for 1-D RoPE; (t, h, w) for M-RoPE,
+ * where pair j takes the axis whose contiguous section contains j. */
+void oracle_rope_head(int head_dim, double theta, int mrope, const int* section,
+                      const double* pos3, double* x) {
+  int half = head_dim / 2;
+  for (int j = 0; j < half; ++j) {
+    double p = pos3[0];
+    if (mrope) {
+      if (j >= section[0] + section[1]) p = pos3[2];
+      else if (j >= section[0]) p = pos3[1];
+    }
+    double a = p * pow(theta, -2.0 * (double)j / (double)head_dim);
+    double c = cos(a), s = sin(a);
+    double x1 = x[j], x2 = x[j + half];
+    x[j] = x1 * c - x2 * s;
+    x[j + half] = x2 * c + x1 * s;
+  }
+}
+
+/*
+ * The whole build for a list of tokens.
+ *   x0    bf16 [B][n_vis][d];   pos int32 [B][P][n_vis], P = 1 (1-D) or 3 (M-RoPE)
+ *   D [L][r][d], U [L][d][r], gamma [L][d], Wk/Wv [L][kv][d], bk/bv [L][kv] or NULL
+ *   tokens: flat token ids t = b * n_vis + i;  n_tokens of them
+ * Outputs (each may be NULL), indexed by the position q of the token in `tokens`:
+ *   k_out, v_out [q][L][kv];  m_out [q][L][d];  h_out [q][L][r];  n_out [q][L][d]
+ * Returns 0, or -1 on a bad argument.
+ */
+int oracle_build_tokens(const oracle_cfg* c, const uint16_t* x0, int n_vis, const int32_t* pos,
+                        const uint16_t* D, const uint16_t* U, const uint16_t* gamma,
+                        const uint16_t* Wk, const uint16_t* Wv, const uint16_t* bk,
+                        const uint16_t* bv, const int64_t* tokens, int64_t n_tokens,
+                        double* k_out, double* v_out, double* m_out, double* h_out,
+                        double* n_out) {
+  if (!c || !x0 || !pos || !D || !U || !gamma || !Wk || !Wv || !tokens) return -1;
+  const int d = c->d, L = c->n_layers, r = c->rank, Dh = c->head_dim;
+  const int kv = c->n_kv_heads * Dh;
+  const int P = c->rope ? 3 : 1;
+  if (d <= 0 || L <= 0 || r <= 0 || Dh <= 0 || (Dh & 1) || n_vis <= 0) return -1;
+  if (c->rope && c->mrope_section[0] + c->mrope_section[1] + c->mrope_section[2] != Dh / 2)
+    return -1;
+#pragma omp parallel
+  {
+    double* x = malloc(sizeof(double) * d);
+    double* m = malloc(sizeof(double) * d);
+    double* n = malloc(sizeof(double) * d);
+    double* g = malloc(sizeof(double) * d);
+    double* z = malloc(sizeof(double) * r);
+    double* h = malloc(sizeof(double) * r);
+    double* kk = malloc(sizeof(double) * kv);
+    double* vv = malloc(sizeof(double) * kv);
+#pragma omp for schedule(dynamic, 1) collapse(2)
+    for (int64_t q = 0; q < n_tokens; ++q) {
+      for (int l = 0; l < L; ++l) {
+        const int64_t t = tokens[q];
+        const int64_t b = t / n_vis, i = t % n_vis;
+        for (int j = 0; j < d; ++j) x[j] = bf16_to_f64(x0[t * d + j]);
+        oracle_adapter_row(d, r, x, D + (int64_t)l * r * d, U + (int64_t)l * d * r, z, h, m);
+        for (int j = 0; j < d; ++j) g[j] = bf16_to_f64(gamma[(int64_t)l * d + j]);
+        oracle_rmsnorm_row(d, m, g, c->rms_eps, n);
+        oracle_project_row(d, kv, Wk + (int64_t)l * kv * d, bk ? bk + (int64_t)l * kv : NULL,
+                           n, kk);
+        oracle_project_row(d, kv, Wv + (int64_t)l * kv * d, bv ? bv + (int64_t)l * kv : NULL,
+                           n, vv);
+        double p3[3];
+        for (int a = 0; a < P; ++a) p3[a] = (double)pos[(b * P + a) * n_vis + i];
+        for (int hh = 0; hh < c->n_kv_heads; ++hh)
+          oracle_rope_head(Dh, c->rope_theta, c->rope, c->mrope_section, p3, kk + hh * Dh);
+        const int64_t o = q * L + l;
+        if (k_out) memcpy(k_out + o * kv, kk, sizeof(double) * kv);
+        if (v_out) memcpy(v_out + o * kv, vv, sizeof(double) * kv);
+        if (m_out) memcpy(m_out + o * d, m, sizeof(double) * d);
+        if (n_out) memcpy(n_out + o * d, n, sizeof(double) * d);
+        if (h_out) memcpy(h_out + o * r, h, sizeof(double) * r);
+      }
+    }
+    free(x); free(m); free(n); free(g); free(z); free(h); free(kk); free(vv);
+  }
+  return 0;
+}
+
+/* Number of threads the OpenMP runtime will use (reported beside oracle timings). */
+int oracle_num_threads(void) {
+  int nt = 1;
+#pragma omp parallel
+  {
+#pragma omp single
+    nt = omp_get_num_threads();
+  }
+  return nt;
+}

@@ -1,0 +1,52 @@
+"""The oracle's pins catch plausible mistakes.
+
+Each case plants one mistake in a copy of ``oracle/oracle.c`` (on the CPU), builds it, and
+runs the pin suite against that build in a child process; the suite must fail. A case whose
+mistake the pins no longer detect fails here.
+"""
+import os
+import subprocess
+import sys
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+SRC = os.path.join(ROOT, "oracle", "oracle.c")
+
+MUTANTS = {
+    "silu_is_sigmoid": ("return u / (1.0 + exp(-u));", "return 1.0 / (1.0 + exp(-u));"),
+    "silu_wrong_sign": ("return u / (1.0 + exp(-u));", "return u / (1.0 + exp(u));"),
+    "down_transposed": ("Dl[(int64_t)k * d + j]", "Dl[(int64_t)j * r + k]"),
+    "up_transposed": ("Ul[(int64_t)j * r + k]", "Ul[(int64_t)k * d + j]"),
+    "residual_dropped": ("m[j] = x[j] + s;", "m[j] = s;"),
+    "norm_sum_not_mean": ("sqrt(ss / (double)d + eps)", "sqrt(ss + eps)"),
+    "eps_outside_sqrt": ("sqrt(ss / (double)d + eps)", "(sqrt(ss / (double)d) + eps)"),
+    "gain_dropped": ("n[j] = gamma[j] * m[j] * inv;", "n[j] = m[j] * inv;"),
+    "projection_transposed": ("bf16_to_f64(W[(int64_t)c * d + j])", "bf16_to_f64(W[(int64_t)j * kv + c])"),
+    "bias_dropped": ("out[c] = s + (b ? bf16_to_f64(b[c]) : 0.0);", "out[c] = s;"),
+    "rope_wrong_direction": ("x[j] = x1 * c - x2 * s;", "x[j] = x1 * c + x2 * s;"),
+    "rope_interleaved_pairs": ("double x1 = x[j], x2 = x[j + half];", "double x1 = x[2 * j], x2 = x[2 * j + 1];"),
+    "rope_frequency_exponent": ("pow(theta, -2.0 * (double)j / (double)head_dim)", "pow(theta, -(double)j / (double)head_dim)"),
+    "mrope_axes_swapped": ("if (j >= section[0] + section[1]) p = pos3[2];", "if (j >= section[0] + section[1]) p = pos3[1];"),
+    "value_rotated": ("oracle_rope_head(Dh, c->rope_theta, c->rope, c->mrope_section, p3, kk + hh * Dh);",
+                      "{ oracle_rope_head(Dh, c->rope_theta, c->rope, c->mrope_section, p3, kk + hh * Dh); "
+                      "oracle_rope_head(Dh, c->rope_theta, c->rope, c->mrope_section, p3, vv + hh * Dh); }"),
+    "position_of_wrong_batch": ("pos[(b * P + a) * n_vis + i]", "pos[a * n_vis + i]"),
+}
+
+
+@pytest.mark.parametrize("name", sorted(MUTANTS))
+def test_pins_reject_mutant(name, tmp_path):
+    old, new = MUTANTS[name]
+    src = open(SRC).read()
+    assert src.count(old) >= 1, f"mutation site for {name} no longer in oracle.c"
+    mutated = tmp_path / "oracle_mut.c"
+    mutated.write_text(src.replace(old, new))
+    lib = tmp_path / "liboracle_mut.so"
+    subprocess.check_call(["gcc", "-O1", "-std=c11", "-fPIC", "-shared", "-fopenmp", str(mutated),
+                           "-o", str(lib), "-lm"])
+    env = dict(os.environ, DV_ORACLE_LIB=str(lib), OMP_NUM_THREADS="2")
+    r = subprocess.run([sys.executable, "-m", "pytest", "-q", "-x", "-p", "no:cacheprovider",
+                        os.path.join(ROOT, "tests", "test_oracle_pins.py")],
+                       cwd=ROOT, env=env, capture_output=True, text=True, timeout=300)
+    assert r.returncode != 0, f"pins did not catch mutant {name}:\n{r.stdout[-2000:]}"
