@@ -1,0 +1,361 @@
+#!/usr/bin/env python
+"""Benchmark of the layer-wise visual KV-memory build (embedding adapter, Sec. 3.1-3.2).
+
+One step = one build of every layer's visual K/V cache entries for one batch of synthetic
+visual embeddings: row statistics, stacked down-projection + SiLU, RMS statistics, and the
+K/V projection with RoPE and the bf16 cache store, all in the library's CUDA kernels.
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--config NAME] [--impl dv|reference]
+
+Prints ONE JSON line on rank 0. Under torchrun (N > 1) every rank builds its own batch of the
+workload (weak scaling, no collective on the data path); timing is the max over ranks.
+``--impl reference`` times the fp64 oracle on the host cores instead (bounded samples).
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import re
+import statistics
+import subprocess
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+METRIC = "visual tokens/sec of layer-wise visual KV-memory build; % of BF16 tensor roofline"
+UNIT = "visual tokens/s"
+DEFAULT_WORKLOAD = "llava15_7b"
+FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+GEMM_SOURCES = ["paper_2609_34972_gb300/csrc/dv_gemm.cu", "paper_2609_34972_gb300/csrc/dv_ptx.cuh",
+                "paper_2609_34972_gb300/csrc/dv_internal.h"]
+
+
+def load_peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(path):
+        with open(path) as f:
+            p = json.load(f)
+        return p, "measured"
+    return dict(FALLBACK_PEAKS), "fallback"
+
+
+def kernel_source_hash() -> str:
+    h = hashlib.sha256()
+    for rel in GEMM_SOURCES:
+        with open(os.path.join(ROOT, rel), "rb") as f:
+            h.update(f.read())
+    return h.hexdigest()[:16]
+
+
+def profiled_traffic(workload: str):
+    """DRAM bytes per launch of the K/V kernel from the committed ncu summary, if that summary
+    was taken on the current kernel source (else None)."""
+    path = os.path.join(ROOT, "profiles", f"kv_proj_rope_store_{workload}.md")
+    if not os.path.exists(path):
+        return None
+    text = open(path).read()
+    m = re.search(r"dram_bytes_per_launch:\s*([0-9.eE+]+)", text)
+    s = re.search(r"kernel_source_sha256_16:\s*([0-9a-f]+)", text)
+    if not m or not s or s.group(1) != kernel_source_hash():
+        return None
+    return float(m.group(1))
+
+
+class ClockSampler:
+    """Samples nvidia-smi clocks and throttle reasons while the timed region runs."""
+
+    FIELDS = ["index", "clocks.sm", "clocks.max.sm", "power.draw", "clocks_event_reasons.active",
+              "clocks_event_reasons.hw_slowdown", "clocks_event_reasons.hw_thermal_slowdown",
+              "clocks_event_reasons.sw_thermal_slowdown", "clocks_event_reasons.sw_power_cap"]
+
+    def __init__(self, gpu_id: str | None):
+        self.proc = None
+        self.gpu_id = gpu_id
+
+    def start(self):
+        cmd = ["nvidia-smi", "--query-gpu=" + ",".join(self.FIELDS), "--format=csv,noheader,nounits",
+               "-lms", "100"]
+        if self.gpu_id:
+            cmd += ["-i", self.gpu_id]
+        try:
+            self.proc = subprocess.Popen(cmd, stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except (OSError, ValueError):
+            self.proc = None
+        time.sleep(0.3)
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        time.sleep(0.15)
+        self.proc.terminate()
+        try:
+            out, _ = self.proc.communicate(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+            out, _ = self.proc.communicate()
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in out.splitlines():
+            parts = [x.strip() for x in line.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                sm.append(float(parts[1]))
+                mx.append(float(parts[2]))
+            except ValueError:
+                continue
+            for n, v in zip(names, parts[5:9]):
+                if v.lower().startswith("active"):
+                    reasons.add(n)
+        if not sm:
+            return None
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx), "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+def dist_env():
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return rank, world, local
+
+
+def time_oracle_sample(inp, budget_s: float, seed: int = 0):
+    """Oracle throughput (tokens/s) on a bounded sample of whole tokens (all layers)."""
+    import numpy as np
+    import oracle
+    cfg = inp.cfg
+    rng = np.random.default_rng(seed)
+    t0 = time.perf_counter()
+    oracle.build_tokens(inp, np.array([0], dtype=np.int64))
+    t1 = time.perf_counter() - t0
+    n = int(max(1, min(cfg.tokens, budget_s / max(t1, 1e-6))))
+    toks = np.sort(rng.choice(cfg.tokens, size=n, replace=False)).astype(np.int64)
+    t0 = time.perf_counter()
+    oracle.build_tokens(inp, toks)
+    dt = time.perf_counter() - t0
+    return {"value": n / dt, "unit": UNIT, "cores": oracle.num_threads(), "kind": "oracle",
+            "sample": f"{n} of {cfg.tokens} tokens (all {cfg.n_layers} layers each) of the "
+                      f"{cfg.name} workload, fp64, {dt:.1f} s"}
+
+
+def run_reference(args):
+    """The oracle as the reference arm: every step is a bounded sample of (token, layer) pairs."""
+    import numpy as np
+    import oracle
+    import synth
+    rank, world, _ = dist_env()
+    if rank != 0:
+        return
+    cfg = synth.CONFIGS[args.config]
+    inp = synth.make_inputs(cfg)
+    rng = np.random.default_rng(0)
+    t0 = time.perf_counter()
+    oracle.build_tokens(inp, np.array([0], dtype=np.int64), layers=[0])
+    t_pair = max(time.perf_counter() - t0, 1e-4)
+    n_steps = args.warmup + args.steps
+    cores = oracle.num_threads()
+    # one random layer per step, evaluated for per_step random tokens (parallel over tokens)
+    per_step = max(1, int(min(cfg.tokens, (args.ref_budget_s / n_steps) / t_pair * cores)))
+    total_t, total_pairs = 0.0, 0
+    for step in range(n_steps):
+        toks = np.sort(rng.choice(cfg.tokens, size=per_step, replace=False)).astype(np.int64)
+        lay = [int(rng.integers(0, cfg.n_layers))]
+        t0 = time.perf_counter()
+        oracle.build_tokens(inp, toks, layers=lay)
+        dt = time.perf_counter() - t0
+        if step >= args.warmup:
+            total_t += dt
+            total_pairs += per_step
+    value = (total_pairs / cfg.n_layers) / total_t
+    out = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": 1000.0 * total_t / args.steps, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": {"workload": cfg.name, "description": cfg.description,
+                   "sample_per_step": f"{per_step} tokens x 1 random layer"},
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": oracle.num_threads(), "kind": "oracle",
+                         "sample": f"{per_step} random tokens at one random layer per step of the "
+                                   f"{cfg.name} workload; tokens/s = (token, layer) pairs/s / "
+                                   f"{cfg.n_layers} layers"},
+        "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(out), flush=True)
+
+
+def run_dv(args):
+    import numpy as np
+    import torch
+    import synth
+    from paper_2609_34972_gb300.build import build_library
+    build_library()
+    import paper_2609_34972_gb300 as dv
+
+    rank, world, local = dist_env()
+    dist = None
+    if world > 1:
+        import torch.distributed as tdist
+        tdist.init_process_group("nccl" if torch.cuda.is_available() else "gloo")
+        dist = tdist
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    cfg = synth.CONFIGS[args.config]
+    peaks, peak_src = load_peaks()
+
+    # ---- inputs (host, seeded) -> device; plan once outside the timing
+    inp = synth.make_inputs(cfg)
+    from tests import gpu_util as gu
+    weights = gu.device_weights(inp, dev)
+    plan = dv.memory_plan(gu.dv_config(cfg), weights)
+    del weights
+    x0 = gu.torch_bf16(inp.x0, dev)
+    pos = torch.from_numpy(np.ascontiguousarray(inp.pos)).to(dev)
+    shape = (cfg.n_layers, cfg.batch, cfg.n_vis, cfg.n_kv_heads, cfg.head_dim)
+    kc = torch.zeros(shape, dtype=torch.bfloat16, device=dev)
+    vc = torch.zeros(shape, dtype=torch.bfloat16, device=dev)
+    stream = torch.cuda.current_stream()
+
+    def barrier():
+        if dist is not None:
+            dist.barrier()
+
+    # ---- warm-up
+    for _ in range(args.warmup):
+        dv.build_visual_memory(plan, x0, pos, kc, vc, stream=stream)
+    torch.cuda.synchronize()
+    st = dv.plan_status(plan)
+    if st != dv.DV_OK:
+        raise RuntimeError(f"device status after warm-up: {dv.error_string(st)}")
+
+    # ---- timed region (device-resident inputs)
+    gpu_id = None
+    try:
+        gpu_id = "GPU-" + str(torch.cuda.get_device_properties(dev).uuid)
+    except Exception:
+        gpu_id = str(local)
+    clocks = ClockSampler(gpu_id)
+    dv.timing_enable(plan, True)
+    barrier()
+    torch.cuda.synchronize()
+    clocks.start()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(args.steps):
+        dv.build_visual_memory(plan, x0, pos, kc, vc, stream=stream)
+    e1.record(stream)
+    torch.cuda.synchronize()
+    clk = clocks.stop()
+    barrier()
+    ms_total = e0.elapsed_time(e1)
+    stage_ms, n_timed = dv.timing_read(plan)
+    dv.timing_enable(plan, False)
+    st = dv.plan_status(plan)
+    if st != dv.DV_OK:
+        raise RuntimeError(f"device status after timed region: {dv.error_string(st)}")
+    if dist is not None:
+        t = torch.tensor([ms_total], dtype=torch.float64, device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms_total = float(t.item())
+    ms_step = ms_total / args.steps
+    value = world * cfg.tokens * args.steps / (ms_total / 1000.0)
+
+    # ---- end to end through host buffers (pinned), copies inside the timed region
+    x0_h = gu.torch_bf16(inp.x0, "cpu").pin_memory()
+    pos_h = torch.from_numpy(np.ascontiguousarray(inp.pos)).pin_memory()
+    k_h = torch.empty(shape, dtype=torch.bfloat16).pin_memory()
+    v_h = torch.empty(shape, dtype=torch.bfloat16).pin_memory()
+    e2e_steps = max(5, min(args.steps, args.e2e_steps))
+    for _ in range(3):
+        dv.build_visual_memory_from_host(plan, x0_h, pos_h, k_h, v_h, x0, pos, kc, vc, stream)
+    torch.cuda.synchronize()
+    barrier()
+    e0.record(stream)
+    for _ in range(e2e_steps):
+        dv.build_visual_memory_from_host(plan, x0_h, pos_h, k_h, v_h, x0, pos, kc, vc, stream)
+    e1.record(stream)
+    torch.cuda.synchronize()
+    barrier()
+    ms_e2e = e0.elapsed_time(e1)
+    if dist is not None:
+        t = torch.tensor([ms_e2e], dtype=torch.float64, device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms_e2e = float(t.item())
+    e2e_value = world * cfg.tokens * e2e_steps / (ms_e2e / 1000.0)
+    h2d = x0_h.numel() * 2 + pos_h.numel() * 4
+    d2h = (k_h.numel() + v_h.numel()) * 2
+
+    # ---- roofline of the dominant kernel (K/V projection + RoPE + store) and of the step
+    kv_ms = stage_ms[3] / max(n_timed, 1)
+    kv_flops = 4.0 * cfg.d * cfg.kv * cfg.tokens * cfg.n_layers
+    peak_tf = peaks["bf16_tflops"]
+    achieved_tf = kv_flops / (kv_ms * 1e-3) / 1e12
+    t_roof_ms = max(cfg.flops() / (peak_tf * 1e12), cfg.min_bytes() / (peaks["hbm_gbs"] * 1e9)) * 1e3
+    traffic = profiled_traffic(cfg.name)
+
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        cpu = time_oracle_sample(inp, args.cpu_budget_s)
+
+    if rank == 0:
+        out = {
+            "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+            "config": {"workload": cfg.name, "description": cfg.description,
+                       "tokens_per_step_per_gpu": cfg.tokens, "layers": cfg.n_layers,
+                       "l2": f"inputs larger than L2: the {cfg.n_layers}-layer weight set "
+                             f"({(cfg.min_bytes() - cfg.tokens * cfg.n_layers * 4 * cfg.kv) / 1e9:.2f} GB "
+                             f"incl. x0) is streamed from HBM every step",
+                       "parallelism": "replicas (weak scaling, no collective)" if world > 1 else "1 GPU"},
+            "clocks": clk,
+            "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": h2d,
+                    "d2h_bytes_per_step": d2h, "steps": e2e_steps,
+                    "ms_per_step": ms_e2e / e2e_steps},
+            "gpu_launches": args.steps * dv.kernels_per_build(plan),
+            "roofline": {"bound": "tensor", "achieved": achieved_tf, "peak": peak_tf,
+                         "unit": "TFLOP/s", "frac": achieved_tf / peak_tf, "traffic": traffic,
+                         "kernel": "dv_gemm_kernel<EPI_KV> (K/V projection + RoPE + cache store)",
+                         "peak_source": f"bf16_tflops (burst) of {peak_src}",
+                         "flops_per_launch": kv_flops, "ms_per_launch": kv_ms},
+            "roofline_step": {"t_roof_ms": t_roof_ms, "frac": t_roof_ms / ms_step,
+                              "frac_sustained": max(cfg.flops() / (peaks["bf16_tflops_sustained"] * 1e12),
+                                                    cfg.min_bytes() / (peaks["hbm_gbs"] * 1e9)) * 1e3 / ms_step,
+                              "plain_flops": cfg.flops(), "min_bytes": cfg.min_bytes()},
+            "stage_ms_per_step": dict(zip(dv.STAGE_NAMES, [s / max(n_timed, 1) for s in stage_ms])),
+            "cpu_baseline": cpu,
+        }
+        print(json.dumps(out), flush=True)
+    dv.free(plan)
+    if dist is not None:
+        dist.destroy_process_group()
+
+
+def main():
+    ap = argparse.ArgumentParser(description=__doc__, formatter_class=argparse.RawDescriptionHelpFormatter)
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=1000)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--config", default=DEFAULT_WORKLOAD)
+    ap.add_argument("--impl", choices=["dv", "reference"], default="dv")
+    ap.add_argument("--e2e-steps", type=int, default=100)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--cpu-budget-s", type=float, default=15.0)
+    ap.add_argument("--ref-budget-s", type=float, default=120.0)
+    args = ap.parse_args()
+    args.warmup = max(args.warmup, 3)   # at least 3 untimed warm-up steps
+    if args.steps > 4096:
+        ap.error("--steps must be <= 4096 (per-stage timing records at most 4096 builds)")
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_dv(args)
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,186 @@
+/*
+ * dv.h — C ABI of the GB300 (sm_103a) visual-memory build for delta-Vision
+ * ("Just MLPs: Efficient Visual State Reconstruction for Multimodal Language Models").
+ *
+ * The library builds, for every visual token and every layer l, the key/value cache entries
+ * that text tokens read:
+ *     M_l = E + SiLU(E D_l) U_l                 (Sec. 3.1, Eqs. 4-5: embedding adapter)
+ *     K_l = RoPE(W_K,l RMSNorm_l(M_l) [+ b_K,l]),  V_l = W_V,l RMSNorm_l(M_l) [+ b_V,l]
+ *                                               (Sec. 3.2, Eq. 7; RMSNorm per App. K; RoPE
+ *                                                at the original visual positions)
+ * and stores them as bf16 into a caller-owned KV cache. Visual tokens get no query,
+ * attention output or feed-forward update (Sec. 3.2), so K/V entries are the only output.
+ *
+ * Conventions for every entry point:
+ *   - Tensor arguments are DEVICE pointers on the current CUDA device, owned by the caller.
+ *   - bf16 tensors are IEEE bfloat16 bit patterns, row-major, innermost index last.
+ *   - Every call returns a dv_status; no exception or abort crosses the ABI. Arguments are
+ *     validated before anything is launched: a call that returns an error launched nothing
+ *     (except DV_ERR_CUDA, which reports a failed launch or allocation).
+ *   - Builds are stream-ordered and asynchronous: they enqueue kernels on `stream` (a
+ *     cudaStream_t passed as void*, NULL = legacy default stream) and never synchronise.
+ */
+#ifndef DV_H
+#define DV_H
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+  DV_OK = 0,
+  DV_ERR_INVALID_ARG = 1,        /* null pointer, negative size, bad enum value */
+  DV_ERR_UNSUPPORTED_SHAPE = 2,  /* a shape outside what the kernels are built for */
+  DV_ERR_ALIGNMENT = 3,          /* a pointer or stride misses its 16-byte alignment */
+  DV_ERR_OOM = 4,                /* device allocation failed */
+  DV_ERR_CUDA = 5,               /* a CUDA runtime or driver call failed */
+  DV_ERR_DEVICE_TIMEOUT = 6,     /* a device-side wait gave up (see dv_plan_status) */
+  DV_ERR_UNSUPPORTED_DEVICE = 7  /* the current device is not an sm_103 GPU */
+} dv_status;
+
+enum { DV_ACT_SILU = 0 };                  /* phi of Sec. 3.1 Eq. 4 */
+enum { DV_ROPE_1D = 0, DV_ROPE_MROPE = 1 };
+
+/* Model shape and build limits. Supported (else DV_ERR_UNSUPPORTED_SHAPE):
+ *   d % 64 == 0, 64 <= d <= 16384;  1 <= rank <= 256;  head_dim in {64, 128};
+ *   1 <= n_kv_heads, n_kv_heads * head_dim <= 8192;  1 <= n_layers <= 256;
+ *   act == DV_ACT_SILU;  rope_theta > 0;  rms_eps >= 0;
+ *   DV_ROPE_MROPE: mrope_section[i] >= 0 and their sum == head_dim / 2 (contiguous sections
+ *   of the frequency index: t first, then h, then w);
+ *   max_batch * max_n_vis >= 1 and <= 2^24 (the tokens one build may carry). */
+typedef struct dv_config {
+  int d;                 /* hidden size of the language model */
+  int n_layers;          /* L: layers that receive visual K/V */
+  int n_kv_heads;        /* H_kv */
+  int head_dim;          /* D_h */
+  int rank;              /* r: adapter bottleneck (Sec. 3.1) */
+  int act;               /* DV_ACT_SILU */
+  int rope;              /* DV_ROPE_1D or DV_ROPE_MROPE */
+  float rope_theta;      /* RoPE base */
+  int mrope_section[3];  /* frequency pairs per axis (t, h, w); DV_ROPE_MROPE only */
+  float rms_eps;         /* epsilon inside the RMSNorm square root */
+  int max_batch;         /* largest batch a build may pass */
+  int max_n_vis;         /* largest number of visual tokens per batch element */
+  int has_kv_bias;       /* 1: weights carry b_K, b_V; 0: no bias */
+} dv_config;
+
+/* Weights of all L layers, bf16, device pointers. Read only during dv_memory_plan: the plan
+ * keeps repacked copies, so the caller may free or change these after it returns.
+ *   D      [L][r][d]    down-projection D_l (Sec. 3.1 Eq. 4) as an nn.Linear weight [out][in]
+ *   U      [L][d][r]    up-projection U_l, nn.Linear layout [out][in]
+ *   gamma  [L][d]       gain of the frozen input RMSNorm LN_l (Sec. 3.2 Eq. 7)
+ *   Wk, Wv [L][kv][d]   frozen key / value projections W_K,l, W_V,l (kv = n_kv_heads*head_dim)
+ *   bk, bv [L][kv]      biases, or NULL when has_kv_bias == 0 */
+typedef struct dv_weights {
+  const void* D;
+  const void* U;
+  const void* gamma;
+  const void* Wk;
+  const void* Wv;
+  const void* bk;
+  const void* bv;
+} dv_weights;
+
+/* Destination KV cache (bf16, caller-owned). Element (layer l, batch b, slot s, head h, j) of
+ * K lives at k[l*s_layer + b*s_batch + s*s_seq + h*s_head + j], j < head_dim contiguous; the
+ * same for V. Strides are in elements and must be multiples of 8 (16 bytes); k and v must be
+ * 16-byte aligned. */
+typedef struct dv_kv_cache {
+  void* k;
+  void* v;
+  long long s_layer;
+  long long s_batch;
+  long long s_seq;
+  long long s_head;
+} dv_kv_cache;
+
+typedef struct dv_plan dv_plan;
+
+/*
+ * dv_memory_plan — validate the configuration, allocate the plan and its workspace on the
+ * current device, and repack the weights for the build kernels (all L down-projections
+ * stacked into one matrix, since every layer reads only E: Sec. 3.1 "conditionally
+ * independent across layers given E"; RMSNorm gain and the rank-r update folded into
+ * the K/V weights).
+ *   cfg     shape and limits (copied)
+ *   w       device weights (read on `stream` before this call returns; not retained)
+ *   stream  cudaStream_t as void*; the repack kernels run on it and this call waits for them
+ *   out     receives the plan; *out is set to NULL on any error
+ * Errors: DV_ERR_INVALID_ARG, DV_ERR_UNSUPPORTED_SHAPE, DV_ERR_UNSUPPORTED_DEVICE,
+ * DV_ERR_OOM, DV_ERR_CUDA. On error nothing stays allocated.
+ */
+int dv_memory_plan(const dv_config* cfg, const dv_weights* w, void* stream, dv_plan** out);
+
+/*
+ * dv_build_visual_memory — the hot path. For batch*n_vis visual tokens writes K^v_l and V^v_l
+ * of every layer (Sec. 3.1 Eqs. 4-5, Sec. 3.2 Eq. 7) into the cache.
+ *   x0     bf16 [batch][n_vis][d]: the visual embeddings E (Sec. 2 Eq. 1); 16-byte aligned
+ *   pos    int32 [batch][P][n_vis], P = 1 (DV_ROPE_1D) or 3 (DV_ROPE_MROPE: t, h, w): the
+ *          original positions of the visual tokens (Sec. 1 and App. H keep them unchanged)
+ *   slot   int32 [batch][n_vis] cache slot of each token, or NULL for slot0 + i
+ *   slot0  first slot when slot == NULL
+ *   out    destination cache; token i of batch element b goes to slot slot[b][i] (or slot0+i)
+ *   stream cudaStream_t as void*
+ * batch*n_vis == 0 is a no-op. Concurrent builds with the same plan must be ordered on one
+ * stream (they share the plan's workspace). The caller keeps slots in range of its cache.
+ * Errors: DV_ERR_INVALID_ARG, DV_ERR_UNSUPPORTED_SHAPE (more tokens than the plan's limit),
+ * DV_ERR_ALIGNMENT, DV_ERR_CUDA.
+ */
+int dv_build_visual_memory(dv_plan* plan, const void* x0, int batch, int n_vis, const int* pos,
+                           const int* slot, int slot0, const dv_kv_cache* out, void* stream);
+
+/*
+ * dv_plan_status — synchronises the device, reads and clears the plan's device status word.
+ * Returns DV_OK, DV_ERR_DEVICE_TIMEOUT when a kernel of an earlier build gave up on a wait
+ * (its outputs are then incomplete), or DV_ERR_INVALID_ARG for a NULL plan.
+ */
+int dv_plan_status(dv_plan* plan);
+
+/* dv_free — release the plan and everything it owns (synchronises the device first).
+ * dv_free(NULL) is a no-op. */
+void dv_free(dv_plan* plan);
+
+/* dv_error_string — static description of a status code (never NULL). */
+const char* dv_error_string(int status);
+
+/*
+ * Per-stage device timing of builds, for measurement. While enabled, each build records
+ * CUDA events around its stages on the build's stream (at most 4096 builds are recorded).
+ *   dv_timing_enable(plan, 1) starts a new record (0 stops recording).
+ *   dv_timing_read(plan, ms, n_stages, n_builds) synchronises on the recorded events and
+ *   writes the summed milliseconds of each stage into ms[0..n_stages-1] (stage order:
+ *   0 row sums of squares of E, 1 stacked down-projection + SiLU, 2 RMS statistics,
+ *   3 K/V projection + RoPE + cache store) and the number of builds into *n_builds.
+ */
+int dv_timing_enable(dv_plan* plan, int on);
+int dv_timing_read(dv_plan* plan, double* ms, int n_stages, int* n_builds);
+
+/* Number of kernels one build launches (for launch accounting). */
+int dv_kernels_per_build(const dv_plan* plan);
+
+/*
+ * dv_debug_wait_timeout — failure-detection self-test. Launches one kernel whose single
+ * thread waits on a shared-memory barrier that nothing will complete, with a limit of
+ * timeout_us microseconds; the wait gives up, the kernel records DV_ERR_DEVICE_TIMEOUT in
+ * the plan's status word and returns normally, so the context stays usable. Read the result
+ * with dv_plan_status. timeout_us must be in [1, 2000000].
+ */
+int dv_debug_wait_timeout(dv_plan* plan, int timeout_us, void* stream);
+
+/*
+ * dv_debug_copy_workspace — copies the intermediate results of the last build on this plan
+ * into caller-owned device buffers (stream-ordered), for stage-wise testing:
+ *   H     bf16 [tokens][n_layers * r_pad]  SiLU(E D_l) of every layer, r_pad = rank rounded
+ *         up to 64 (columns past rank are zero)
+ *   rstd  fp32 [n_layers][tokens]           1 / sqrt(mean(M_l^2) + eps)
+ *   xx    fp32 [tokens]                     sum of squares of each row of E
+ * Any of the three may be NULL. tokens must not exceed the plan's limit; *r_pad_out (if not
+ * NULL) receives r_pad.
+ */
+int dv_debug_copy_workspace(dv_plan* plan, int tokens, void* H, void* rstd, void* xx,
+                            int* r_pad_out, void* stream);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* DV_H */

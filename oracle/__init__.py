@@ -55,7 +55,7 @@ def _load():
         lib.oracle_project_row.argtypes = [i32, i32, vp, vp, vp, vp]
         lib.oracle_rope_head.argtypes = [i32, dbl, i32, vp, vp, vp]
         lib.oracle_build_tokens.argtypes = [ctypes.POINTER(_Cfg), vp, i32, vp, vp, vp, vp, vp,
-                                            vp, vp, vp, vp, i64, vp, vp, vp, vp, vp]
+                                            vp, vp, vp, vp, i64, vp, i32, vp, vp, vp, vp, vp]
         lib.oracle_build_tokens.restype = i32
         lib.oracle_num_threads.restype = i32
         _lib = lib
@@ -117,13 +117,14 @@ def rope_head(x, pos3, theta: float, mrope: bool = False, section=(0, 0, 0)):
     return x
 
 
-def build_tokens(inp, tokens=None, want=("k", "v")):
-    """Run the whole build for the given flat token ids (default: every token).
+def build_tokens(inp, tokens=None, want=("k", "v"), layers=None):
+    """Run the whole build for the given flat token ids (default: every token) and layers
+    (default: all, in order).
 
     ``inp`` carries ``cfg`` (d, n_layers, n_kv_heads, head_dim, rank, rope, rope_theta,
     mrope_section, rms_eps, n_vis) and the bf16-bit arrays x0, D, U, gamma, Wk, Wv, bk, bv
-    and int32 pos [B][P][N_v]. Returns a dict of fp64 arrays: k, v [n][L][kv], m, n [n][L][d],
-    h [n][L][r], for the names in ``want``.
+    and int32 pos [B][P][N_v]. Returns a dict of fp64 arrays: k, v [n][Ls][kv], m, n [n][Ls][d],
+    h [n][Ls][r] (Ls = number of evaluated layers), for the names in ``want``.
     """
     cfg = inp.cfg
     c = _Cfg(cfg.d, cfg.n_layers, cfg.n_kv_heads, cfg.head_dim, cfg.rank,
@@ -133,7 +134,9 @@ def build_tokens(inp, tokens=None, want=("k", "v")):
     if tokens is None:
         tokens = np.arange(B * cfg.n_vis, dtype=np.int64)
     tokens = np.ascontiguousarray(tokens, dtype=np.int64)
-    nt, L, kv = tokens.shape[0], cfg.n_layers, cfg.n_kv_heads * cfg.head_dim
+    lay = None if layers is None else np.ascontiguousarray(layers, dtype=np.int32)
+    nt, kv = tokens.shape[0], cfg.n_kv_heads * cfg.head_dim
+    L = cfg.n_layers if lay is None else lay.shape[0]
     out = {}
     shapes = {"k": (nt, L, kv), "v": (nt, L, kv), "m": (nt, L, cfg.d), "h": (nt, L, cfg.rank),
               "n": (nt, L, cfg.d)}
@@ -144,7 +147,7 @@ def build_tokens(inp, tokens=None, want=("k", "v")):
     rc = _load().oracle_build_tokens(
         ctypes.byref(c), _p(arrs[0]), cfg.n_vis, _p(arrs[1]), _p(arrs[2]), _p(arrs[3]),
         _p(arrs[4]), _p(arrs[5]), _p(arrs[6]), _p(arrs[7]), _p(arrs[8]), _p(tokens), nt,
-        _p(out.get("k")), _p(out.get("v")), _p(out.get("m")), _p(out.get("h")), _p(out.get("n")))
+        _p(lay), 0 if lay is None else int(lay.shape[0]), _p(out.get("k")), _p(out.get("v")), _p(out.get("m")), _p(out.get("h")), _p(out.get("n")))
     if rc != 0:
         raise ValueError("oracle_build_tokens rejected its arguments")
     return out

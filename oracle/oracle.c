@@ -120,14 +120,17 @@ void oracle_rope_head(int head_dim, double theta, int mrope, const int* section,
  *   x0    bf16 [B][n_vis][d];   pos int32 [B][P][n_vis], P = 1 (1-D) or 3 (M-RoPE)
  *   D [L][r][d], U [L][d][r], gamma [L][d], Wk/Wv [L][kv][d], bk/bv [L][kv] or NULL
  *   tokens: flat token ids t = b * n_vis + i;  n_tokens of them
- * Outputs (each may be NULL), indexed by the position q of the token in `tokens`:
- *   k_out, v_out [q][L][kv];  m_out [q][L][d];  h_out [q][L][r];  n_out [q][L][d]
+ *   layers: the layers to evaluate (n_sel_layers of them), or NULL for all L in order
+ * Outputs (each may be NULL), indexed by the position q of the token in `tokens` and the
+ * position s of the layer in `layers` (Ls = number of evaluated layers):
+ *   k_out, v_out [q][Ls][kv];  m_out [q][Ls][d];  h_out [q][Ls][r];  n_out [q][Ls][d]
  * Returns 0, or -1 on a bad argument.
  */
 int oracle_build_tokens(const oracle_cfg* c, const uint16_t* x0, int n_vis, const int32_t* pos,
                         const uint16_t* D, const uint16_t* U, const uint16_t* gamma,
                         const uint16_t* Wk, const uint16_t* Wv, const uint16_t* bk,
                         const uint16_t* bv, const int64_t* tokens, int64_t n_tokens,
+                        const int32_t* layers, int n_sel_layers,
                         double* k_out, double* v_out, double* m_out, double* h_out,
                         double* n_out) {
   if (!c || !x0 || !pos || !D || !U || !gamma || !Wk || !Wv || !tokens) return -1;
@@ -137,6 +140,10 @@ int oracle_build_tokens(const oracle_cfg* c, const uint16_t* x0, int n_vis, cons
   if (d <= 0 || L <= 0 || r <= 0 || Dh <= 0 || (Dh & 1) || n_vis <= 0) return -1;
   if (c->rope && c->mrope_section[0] + c->mrope_section[1] + c->mrope_section[2] != Dh / 2)
     return -1;
+  const int Ls = layers ? n_sel_layers : L;
+  if (Ls <= 0) return -1;
+  for (int s = 0; layers && s < Ls; ++s)
+    if (layers[s] < 0 || layers[s] >= L) return -1;
 #pragma omp parallel
   {
     double* x = malloc(sizeof(double) * d);
@@ -149,7 +156,8 @@ int oracle_build_tokens(const oracle_cfg* c, const uint16_t* x0, int n_vis, cons
     double* vv = malloc(sizeof(double) * kv);
 #pragma omp for schedule(dynamic, 1) collapse(2)
     for (int64_t q = 0; q < n_tokens; ++q) {
-      for (int l = 0; l < L; ++l) {
+      for (int ls = 0; ls < Ls; ++ls) {
+        const int l = layers ? layers[ls] : ls;
         const int64_t t = tokens[q];
         const int64_t b = t / n_vis, i = t % n_vis;
         for (int j = 0; j < d; ++j) x[j] = bf16_to_f64(x0[t * d + j]);
@@ -164,7 +172,7 @@ int oracle_build_tokens(const oracle_cfg* c, const uint16_t* x0, int n_vis, cons
         for (int a = 0; a < P; ++a) p3[a] = (double)pos[(b * P + a) * n_vis + i];
         for (int hh = 0; hh < c->n_kv_heads; ++hh)
           oracle_rope_head(Dh, c->rope_theta, c->rope, c->mrope_section, p3, kk + hh * Dh);
-        const int64_t o = q * L + l;
+        const int64_t o = q * Ls + ls;
         if (k_out) memcpy(k_out + o * kv, kk, sizeof(double) * kv);
         if (v_out) memcpy(v_out + o * kv, vv, sizeof(double) * kv);
         if (m_out) memcpy(m_out + o * d, m, sizeof(double) * d);

@@ -1,0 +1,237 @@
+"""Python binding of the GB300 visual-memory build (``include/dv.h``).
+
+Argument marshalling only: every step of the build runs in the CUDA kernels of ``libdv.so``.
+PyTorch supplies device memory and the CUDA stream. There is no CPU fallback: if the library
+is missing, every call raises.
+
+    plan = memory_plan(cfg, weights)               # once per weight set
+    build_visual_memory(plan, x0, pos, k_cache, v_cache)   # the hot path
+    free(plan)
+
+Tensor layouts (bf16 unless stated, all on the current CUDA device):
+    x0      [B, N_v, d]          visual embeddings E (Sec. 2 Eq. 1)
+    pos     int32 [B, P, N_v]    P = 1 (1-D RoPE) or 3 (M-RoPE t, h, w)
+    weights D [L, r, d], U [L, d, r], gamma [L, d], Wk, Wv [L, kv, d], bk, bv [L, kv] (optional)
+    k/v cache [L, B_c, S, H_kv, D_h] or any strided view with D_h contiguous
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_HERE, "libdv.so")
+
+DV_OK = 0
+DV_ERR_INVALID_ARG = 1
+DV_ERR_UNSUPPORTED_SHAPE = 2
+DV_ERR_ALIGNMENT = 3
+DV_ERR_OOM = 4
+DV_ERR_CUDA = 5
+DV_ERR_DEVICE_TIMEOUT = 6
+DV_ERR_UNSUPPORTED_DEVICE = 7
+DV_ACT_SILU = 0
+DV_ROPE_1D = 0
+DV_ROPE_MROPE = 1
+
+EXPORTED = ["dv_memory_plan", "dv_build_visual_memory", "dv_plan_status", "dv_free",
+            "dv_error_string", "dv_timing_enable", "dv_timing_read", "dv_kernels_per_build",
+            "dv_debug_wait_timeout", "dv_debug_copy_workspace"]
+N_STAGES = 4
+STAGE_NAMES = ["row_sumsq", "down_proj_silu", "rms_stats", "kv_proj_rope_store"]
+
+
+class DvConfig(ctypes.Structure):
+    _fields_ = [("d", ctypes.c_int), ("n_layers", ctypes.c_int), ("n_kv_heads", ctypes.c_int),
+                ("head_dim", ctypes.c_int), ("rank", ctypes.c_int), ("act", ctypes.c_int),
+                ("rope", ctypes.c_int), ("rope_theta", ctypes.c_float),
+                ("mrope_section", ctypes.c_int * 3), ("rms_eps", ctypes.c_float),
+                ("max_batch", ctypes.c_int), ("max_n_vis", ctypes.c_int),
+                ("has_kv_bias", ctypes.c_int)]
+
+
+class DvWeights(ctypes.Structure):
+    _fields_ = [(n, ctypes.c_void_p) for n in ("D", "U", "gamma", "Wk", "Wv", "bk", "bv")]
+
+
+class DvKVCache(ctypes.Structure):
+    _fields_ = [("k", ctypes.c_void_p), ("v", ctypes.c_void_p), ("s_layer", ctypes.c_longlong),
+                ("s_batch", ctypes.c_longlong), ("s_seq", ctypes.c_longlong),
+                ("s_head", ctypes.c_longlong)]
+
+
+_lib = None
+
+
+def lib() -> ctypes.CDLL:
+    """The loaded ``libdv.so``; raises if it has not been built."""
+    global _lib
+    if _lib is None:
+        if not os.path.exists(LIB_PATH):
+            raise RuntimeError(f"CUDA library {LIB_PATH} is missing: run "
+                               "`python -c 'import __graft_entry__ as g; g.build()'` first")
+        L = ctypes.CDLL(LIB_PATH)
+        vp, i32 = ctypes.c_void_p, ctypes.c_int
+        L.dv_memory_plan.argtypes = [ctypes.POINTER(DvConfig), ctypes.POINTER(DvWeights), vp,
+                                     ctypes.POINTER(vp)]
+        L.dv_build_visual_memory.argtypes = [vp, vp, i32, i32, vp, vp, i32,
+                                             ctypes.POINTER(DvKVCache), vp]
+        L.dv_plan_status.argtypes = [vp]
+        L.dv_free.argtypes = [vp]
+        L.dv_free.restype = None
+        L.dv_error_string.argtypes = [i32]
+        L.dv_error_string.restype = ctypes.c_char_p
+        L.dv_timing_enable.argtypes = [vp, i32]
+        L.dv_timing_read.argtypes = [vp, ctypes.POINTER(ctypes.c_double), i32,
+                                     ctypes.POINTER(i32)]
+        L.dv_kernels_per_build.argtypes = [vp]
+        L.dv_debug_wait_timeout.argtypes = [vp, i32, vp]
+        L.dv_debug_copy_workspace.argtypes = [vp, i32, vp, vp, vp, ctypes.POINTER(i32), vp]
+        for name in ("dv_memory_plan", "dv_build_visual_memory", "dv_plan_status",
+                     "dv_timing_enable", "dv_timing_read", "dv_kernels_per_build",
+                     "dv_debug_wait_timeout", "dv_debug_copy_workspace"):
+            getattr(L, name).restype = i32
+        _lib = L
+    return _lib
+
+
+class DvError(RuntimeError):
+    def __init__(self, code: int, where: str):
+        self.code = code
+        super().__init__(f"{where}: {error_string(code)} (status {code})")
+
+
+def error_string(code: int) -> str:
+    return lib().dv_error_string(int(code)).decode()
+
+
+def _check(code: int, where: str):
+    if code != DV_OK:
+        raise DvError(code, where)
+
+
+def _stream_handle(stream):
+    import torch
+    if stream is None:
+        stream = torch.cuda.current_stream()
+    return ctypes.c_void_p(int(stream.cuda_stream))
+
+
+def _ptr(t):
+    return None if t is None else ctypes.c_void_p(t.data_ptr())
+
+
+def make_config(d, n_layers, n_kv_heads, head_dim, rank, rope="1d", rope_theta=10000.0,
+                mrope_section=(0, 0, 0), rms_eps=1e-6, max_batch=1, max_n_vis=1,
+                has_kv_bias=False) -> DvConfig:
+    return DvConfig(int(d), int(n_layers), int(n_kv_heads), int(head_dim), int(rank),
+                    DV_ACT_SILU, DV_ROPE_MROPE if rope == "mrope" else DV_ROPE_1D,
+                    float(rope_theta), (ctypes.c_int * 3)(*mrope_section), float(rms_eps),
+                    int(max_batch), int(max_n_vis), int(bool(has_kv_bias)))
+
+
+class Plan:
+    """Owns a ``dv_plan*``: repacked weights, workspace and TMA descriptors on one device."""
+
+    def __init__(self, handle: ctypes.c_void_p, cfg: DvConfig):
+        self.handle = handle
+        self.cfg = cfg
+
+    @property
+    def alive(self) -> bool:
+        return bool(self.handle and self.handle.value)
+
+    def __del__(self):
+        try:
+            free(self)
+        except Exception:
+            pass
+
+
+def memory_plan(cfg: DvConfig, weights: dict, stream=None) -> Plan:
+    """Plan a build for ``cfg`` from device weights (dict of torch tensors, see module doc)."""
+    w = DvWeights(*[_ptr(weights.get(n)) for n in ("D", "U", "gamma", "Wk", "Wv", "bk", "bv")])
+    h = ctypes.c_void_p()
+    _check(lib().dv_memory_plan(ctypes.byref(cfg), ctypes.byref(w), _stream_handle(stream),
+                                ctypes.byref(h)), "dv_memory_plan")
+    return Plan(h, cfg)
+
+
+def kv_cache_view(k, v) -> DvKVCache:
+    """Describe two [L, B, S, H, D_h] (strided, D_h contiguous) bf16 tensors for the C ABI."""
+    if k.dim() != 5 or v.dim() != 5 or k.stride() != v.stride() or k.stride(4) != 1:
+        raise ValueError("k and v must be 5-D [L, B, S, H, D_h] views with equal strides, D_h contiguous")
+    s = k.stride()
+    return DvKVCache(k.data_ptr(), v.data_ptr(), s[0], s[1], s[2], s[3])
+
+
+def build_visual_memory(plan: Plan, x0, pos, k_cache, v_cache, slot=None, slot0: int = 0,
+                        stream=None) -> None:
+    """Enqueue one build on ``stream`` (default: torch's current stream). Asynchronous."""
+    B, N = int(x0.shape[0]), int(x0.shape[1])
+    kvc = kv_cache_view(k_cache, v_cache)
+    _check(lib().dv_build_visual_memory(plan.handle, _ptr(x0), B, N, _ptr(pos), _ptr(slot),
+                                        int(slot0), ctypes.byref(kvc), _stream_handle(stream)),
+           "dv_build_visual_memory")
+
+
+def plan_status(plan: Plan) -> int:
+    """Synchronise and read (and clear) the plan's device status word."""
+    return int(lib().dv_plan_status(plan.handle))
+
+
+def free(plan: Plan) -> None:
+    if plan is not None and plan.alive:
+        lib().dv_free(plan.handle)
+        plan.handle = ctypes.c_void_p()
+
+
+def kernels_per_build(plan: Plan) -> int:
+    return int(lib().dv_kernels_per_build(plan.handle))
+
+
+def timing_enable(plan: Plan, on: bool = True) -> None:
+    _check(lib().dv_timing_enable(plan.handle, int(bool(on))), "dv_timing_enable")
+
+
+def timing_read(plan: Plan):
+    """(per-stage summed milliseconds, number of builds) since timing_enable."""
+    ms = (ctypes.c_double * N_STAGES)()
+    n = ctypes.c_int()
+    _check(lib().dv_timing_read(plan.handle, ms, N_STAGES, ctypes.byref(n)), "dv_timing_read")
+    return list(ms), n.value
+
+
+def debug_wait_timeout(plan: Plan, timeout_us: int, stream=None) -> None:
+    _check(lib().dv_debug_wait_timeout(plan.handle, int(timeout_us), _stream_handle(stream)),
+           "dv_debug_wait_timeout")
+
+
+def debug_workspace(plan: Plan, tokens: int, stream=None):
+    """(H [tokens, L*r_pad] bf16, rstd [L, tokens] fp32, xx [tokens] fp32) of the last build."""
+    import torch
+    r_pad = ctypes.c_int()
+    _check(lib().dv_debug_copy_workspace(plan.handle, 0, None, None, None, ctypes.byref(r_pad),
+                                         None), "dv_debug_copy_workspace")
+    L = plan.cfg.n_layers
+    H = torch.empty((tokens, L * r_pad.value), dtype=torch.bfloat16, device="cuda")
+    rstd = torch.empty((L, tokens), dtype=torch.float32, device="cuda")
+    xx = torch.empty((tokens,), dtype=torch.float32, device="cuda")
+    _check(lib().dv_debug_copy_workspace(plan.handle, int(tokens), _ptr(H), _ptr(rstd), _ptr(xx),
+                                         None, _stream_handle(stream)), "dv_debug_copy_workspace")
+    return H, rstd, xx, r_pad.value
+
+
+def build_visual_memory_from_host(plan: Plan, x0_host, pos_host, k_host, v_host, x0_dev, pos_dev,
+                                  k_dev, v_dev, stream=None) -> None:
+    """End-to-end build from pinned host buffers: copy E and the positions to the device, build,
+    and copy the written K/V entries back, all on one stream. ``*_dev`` are device buffers of the
+    same shapes the caller keeps across calls. Asynchronous like the device-side call."""
+    import torch
+    s = stream or torch.cuda.current_stream()
+    with torch.cuda.stream(s):
+        x0_dev.copy_(x0_host, non_blocking=True)
+        pos_dev.copy_(pos_host, non_blocking=True)
+        build_visual_memory(plan, x0_dev, pos_dev, k_dev, v_dev, stream=s)
+        k_host.copy_(k_dev, non_blocking=True)
+        v_host.copy_(v_dev, non_blocking=True)

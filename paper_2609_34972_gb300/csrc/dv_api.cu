@@ -1,0 +1,603 @@
+// C ABI of the visual-memory build (include/dv.h): argument validation, the plan (repacked
+// weights, workspace, TMA descriptors) and the per-build launch sequence.
+//
+// Plan-time repacking (once per weight set). With r_pad = r rounded up to 64:
+//   Dst  [L*r_pad][d]         stacked down-projections, zero rows past r
+//   Bn   [L*r_pad][d+r_pad]   row n of layer l: [2 U_l[n,:] | G_l[n,:]], G_l = U_l U_l^T
+//   Wkv  [L*2kv][d+r_pad]     per layer, per head h: 128 (or 64) K rows then V rows, each
+//                             [W[c,:] * gamma_l | (W diag(gamma_l) U_l^T)[c,:]]
+// so that, with A_l = [x0 | h_l] (h_l = SiLU(x0 D_l), Sec. 3.1 Eq. 4):
+//   A_l Bn_l^T   = 2 x0 U_l^T + h_l G_l        -> ||M_l||^2 = ||x0||^2 + h_l . (that)
+//   A_l Wkv_l^T  = (x0 + h_l U_l) diag(gamma_l) W^T = gamma_l * M_l projected (Sec. 3.2 Eq. 7)
+// and K/V = rstd_l * (A_l Wkv_l^T) + b is exactly W RMSNorm(M_l) + b, without M_l ever being
+// formed. Per build: (0) ||x0||^2 per token, (1) H = SiLU(x0 Dst^T), (2) rstd, (3) K/V.
+#include <cmath>
+#include <cstdio>
+#include <cstdlib>
+#include <cstring>
+#include <mutex>
+#include <vector>
+
+#include "../../include/dv.h"
+#include "dv_internal.h"
+#include "dv_ptx.cuh"
+
+using dv::GemmParams;
+
+struct dv_plan {
+  dv_config cfg;
+  int device = 0;
+  int num_sms = 0;
+  int r_pad = 0, kv = 0, k_total = 0, max_tokens = 0;
+  uint16_t* Dst = nullptr;
+  uint16_t* Bn = nullptr;
+  uint16_t* Wkv = nullptr;
+  float* bk = nullptr;
+  float* bv = nullptr;
+  uint16_t* H = nullptr;
+  float* xx = nullptr;
+  float* rstd = nullptr;
+  int* status = nullptr;
+  CUtensorMap tm_Dst[3];  // boxes of 64, 128, 256 rows
+  CUtensorMap tm_Bn, tm_Wkv, tm_H;
+  double inv_freq[dv::kMaxHalfHead];
+  // per-stage timing
+  bool timing = false;
+  std::vector<cudaEvent_t> ev;  // kMaxTimed * kStages1
+  int timed = 0;
+};
+
+namespace {
+
+constexpr int kStages = 4;
+constexpr int kEvPerBuild = kStages + 1;
+constexpr int kMaxTimed = 4096;
+constexpr unsigned long long kTimeoutNs = 2000000000ull;  // 2 s per device-side wait
+
+// ------------------------------------------------------------------------------ driver entry
+
+typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,
+                                  const cuuint64_t*, const cuuint64_t*, const cuuint32_t*,
+                                  const cuuint32_t*, CUtensorMapInterleave, CUtensorMapSwizzle,
+                                  CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiledFn encode_fn() {
+  static EncodeTiledFn fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault,
+                                         &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<EncodeTiledFn>(p);
+  });
+  return fn;
+}
+
+// bf16 2-D tensor [rows][cols] (row stride in elements), 128-byte-swizzled boxes of
+// 64 columns x box_rows rows; out-of-range elements read as zero.
+bool encode_2d(CUtensorMap* map, const void* ptr, uint64_t cols, uint64_t rows, uint64_t ld,
+               uint32_t box_rows) {
+  EncodeTiledFn fn = encode_fn();
+  if (!fn) return false;
+  cuuint64_t dims[2] = {cols, rows};
+  cuuint64_t strides[1] = {ld * 2};
+  cuuint32_t box[2] = {static_cast<cuuint32_t>(dv::kBlockK), box_rows};
+  cuuint32_t estr[2] = {1, 1};
+  return fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(ptr), dims, strides, box,
+            estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+            CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+// ------------------------------------------------------------------------------ small kernels
+
+__device__ __forceinline__ float bf(uint16_t b) { return __uint_as_float(static_cast<uint32_t>(b) << 16); }
+
+__device__ __forceinline__ uint16_t to_bf16(float f) {
+  return static_cast<uint16_t>(dv::pack_bf16x2(f, 0.0f) & 0xFFFFu);
+}
+
+// Dst[l*r_pad + k][j] = D[l][k][j] for k < r, else 0.
+__global__ void k_pack_down(const uint16_t* __restrict__ D, uint16_t* __restrict__ Dst, int L,
+                            int r, int r_pad, int d) {
+  const long long total = static_cast<long long>(L) * r_pad * d;
+  for (long long e = blockIdx.x * static_cast<long long>(blockDim.x) + threadIdx.x; e < total;
+       e += static_cast<long long>(gridDim.x) * blockDim.x) {
+    const int j = static_cast<int>(e % d);
+    const long long row = e / d;
+    const int k = static_cast<int>(row % r_pad), l = static_cast<int>(row / r_pad);
+    Dst[e] = k < r ? D[(static_cast<long long>(l) * r + k) * d + j] : 0;
+  }
+}
+
+// Bn[l*r_pad + n][j] = 2 U[l][j][n] (j < d, n < r), zero for padded rows. The G block is
+// written by k_rank_product.
+__global__ void k_pack_norm_u(const uint16_t* __restrict__ U, uint16_t* __restrict__ Bn, int L,
+                              int r, int r_pad, int d, int k_total) {
+  const long long total = static_cast<long long>(L) * r_pad * k_total;
+  for (long long e = blockIdx.x * static_cast<long long>(blockDim.x) + threadIdx.x; e < total;
+       e += static_cast<long long>(gridDim.x) * blockDim.x) {
+    const int j = static_cast<int>(e % k_total);
+    const long long row = e / k_total;
+    const int n = static_cast<int>(row % r_pad), l = static_cast<int>(row / r_pad);
+    float v = 0.0f;
+    if (j < d && n < r) v = 2.0f * bf(U[(static_cast<long long>(l) * d + j) * r + n]);
+    Bn[e] = to_bf16(v);  // the G columns (j >= d) are zero here and filled afterwards
+  }
+}
+
+// Wkv rows: per layer, per head h, HD rows of K then HD rows of V; columns [0, d) hold
+// W[c][j] * gamma[l][j]; columns [d, k_total) are filled by k_rank_product (zero past r).
+__global__ void k_pack_kv(const uint16_t* __restrict__ Wk, const uint16_t* __restrict__ Wv,
+                          const uint16_t* __restrict__ gamma, uint16_t* __restrict__ Wkv, int L,
+                          int kv, int HD, int d, int k_total) {
+  const long long total = static_cast<long long>(L) * 2 * kv * k_total;
+  for (long long e = blockIdx.x * static_cast<long long>(blockDim.x) + threadIdx.x; e < total;
+       e += static_cast<long long>(gridDim.x) * blockDim.x) {
+    const int j = static_cast<int>(e % k_total);
+    const long long row = e / k_total;
+    const int rl = static_cast<int>(row % (2 * kv)), l = static_cast<int>(row / (2 * kv));
+    const int h = rl / (2 * HD), part = (rl / HD) & 1, jj = rl % HD;
+    const int c = h * HD + jj;
+    float v = 0.0f;
+    if (j < d) {
+      const uint16_t* W = part ? Wv : Wk;
+      v = bf(W[(static_cast<long long>(l) * kv + c) * d + j]) * bf(gamma[static_cast<long long>(l) * d + j]);
+    }
+    Wkv[e] = to_bf16(v);
+  }
+}
+
+// out[l][i][n] = sum_j A(l, i, j) * U[l][j][n] for n < r, accumulated in fp32 over j < d:
+//   MODE 0 (fold):  A(l, i, j) = W_part[l][c][j] * gamma[l][j], i indexes the 2*kv Wkv rows
+//                   of layer l; the result goes to Wkv row (l, i), column d + n
+//   MODE 1 (gram):  A(l, i, j) = U[l][j][i], i < r; the result goes to Bn row l*r_pad + i,
+//                   column d + n
+// 64 x 64 output tile per block, 256 threads with 4 x 4 outputs each, j in steps of 32.
+template <int MODE>
+__global__ void __launch_bounds__(256) k_rank_product(const uint16_t* __restrict__ Wk,
+                                                      const uint16_t* __restrict__ Wv,
+                                                      const uint16_t* __restrict__ gamma,
+                                                      const uint16_t* __restrict__ U,
+                                                      uint16_t* __restrict__ out, int rows, int r,
+                                                      int d, int kv, int HD, int r_pad,
+                                                      int k_total) {
+  __shared__ float As[32][65];
+  __shared__ float Us[32][65];
+  const int l = blockIdx.z;
+  const int i0 = blockIdx.y * 64, n0 = blockIdx.x * 64;
+  const int tx = threadIdx.x & 15, ty = threadIdx.x >> 4;
+  float acc[4][4] = {};
+  const uint16_t* Ul = U + static_cast<long long>(l) * d * r;
+  for (int j0 = 0; j0 < d; j0 += 32) {
+    for (int e = threadIdx.x; e < 64 * 32; e += 256) {
+      const int ii = e / 32, jj = e % 32;
+      const int i = i0 + ii, j = j0 + jj;
+      float a = 0.0f;
+      if (i < rows && j < d) {
+        if (MODE == 0) {
+          const int h = i / (2 * HD), part = (i / HD) & 1, c = h * HD + i % HD;
+          const uint16_t* W = part ? Wv : Wk;
+          a = bf(W[(static_cast<long long>(l) * kv + c) * d + j]) *
+              bf(gamma[static_cast<long long>(l) * d + j]);
+        } else {
+          a = bf(Ul[static_cast<long long>(j) * r + i]);
+        }
+      }
+      As[jj][ii] = a;
+      const int nn = e % 64, jk = e / 64;
+      const int n = n0 + nn, j2 = j0 + jk;
+      Us[jk][nn] = (n < r && j2 < d) ? bf(Ul[static_cast<long long>(j2) * r + n]) : 0.0f;
+    }
+    __syncthreads();
+#pragma unroll 8
+    for (int jj = 0; jj < 32; ++jj) {
+      float a[4], u[4];
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        a[q] = As[jj][ty * 4 + q];
+        u[q] = Us[jj][tx * 4 + q];
+      }
+#pragma unroll
+      for (int q = 0; q < 4; ++q)
+#pragma unroll
+        for (int w = 0; w < 4; ++w) acc[q][w] = fmaf(a[q], u[w], acc[q][w]);
+    }
+    __syncthreads();
+  }
+#pragma unroll
+  for (int q = 0; q < 4; ++q) {
+    const int i = i0 + ty * 4 + q;
+    if (i >= rows) continue;
+    const long long orow = MODE == 0 ? static_cast<long long>(l) * 2 * kv + i
+                                     : static_cast<long long>(l) * r_pad + i;
+#pragma unroll
+    for (int w = 0; w < 4; ++w) {
+      const int n = n0 + tx * 4 + w;
+      if (n < r) out[orow * k_total + d + n] = to_bf16(acc[q][w]);
+    }
+  }
+}
+
+__global__ void k_bias_to_f32(const uint16_t* __restrict__ b, float* __restrict__ out, long long n) {
+  for (long long e = blockIdx.x * static_cast<long long>(blockDim.x) + threadIdx.x; e < n;
+       e += static_cast<long long>(gridDim.x) * blockDim.x)
+    out[e] = bf(b[e]);
+}
+
+// xx[t] = sum_j x0[t][j]^2 (fp32), one warp per token row, 16-byte loads.
+__global__ void k_row_sumsq(const uint16_t* __restrict__ x0, int T, int d, float* __restrict__ xx) {
+  const int warp = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+  const int lane = threadIdx.x & 31;
+  if (warp >= T) return;
+  const uint4* row = reinterpret_cast<const uint4*>(x0 + static_cast<long long>(warp) * d);
+  float s = 0.0f;
+  for (int c = lane; c < d / 8; c += 32) {
+    const uint4 v = row[c];
+    const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+      const float a = __uint_as_float(w[e] << 16), b = __uint_as_float(w[e] & 0xFFFF0000u);
+      s = fmaf(a, a, s);
+      s = fmaf(b, b, s);
+    }
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xFFFFFFFFu, s, o);
+  if (lane == 0) xx[warp] = s;
+}
+
+// Failure-detection self-test: waits on a barrier nothing completes; gives up after the limit.
+__global__ void k_wait_timeout(int* status, unsigned long long timeout_ns) {
+  __shared__ __align__(8) uint64_t bar;
+  __shared__ volatile int abort_flag;
+  if (threadIdx.x != 0) return;
+  const uint32_t b = dv::smem_addr(&bar);
+  dv::mbar_init(b, 1);
+  dv::fence_barrier_init();
+  abort_flag = 0;
+  if (!dv::mbar_wait(b, 0, &abort_flag, timeout_ns)) atomicExch(status, DV_ERR_DEVICE_TIMEOUT);
+}
+
+// ------------------------------------------------------------------------------ host helpers
+
+int grid_for(long long n) {
+  long long g = (n + 255) / 256;
+  if (g > 65535LL * 16) g = 65535LL * 16;
+  return static_cast<int>(g < 1 ? 1 : g);
+}
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+bool aligned2(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 1u) == 0; }
+
+int check_config(const dv_config* c) {
+  if (!c) return DV_ERR_INVALID_ARG;
+  if (c->act != DV_ACT_SILU) return DV_ERR_INVALID_ARG;
+  if (c->rope != DV_ROPE_1D && c->rope != DV_ROPE_MROPE) return DV_ERR_INVALID_ARG;
+  if (c->d <= 0 || c->n_layers <= 0 || c->n_kv_heads <= 0 || c->head_dim <= 0 || c->rank <= 0 ||
+      c->max_batch <= 0 || c->max_n_vis <= 0)
+    return DV_ERR_INVALID_ARG;
+  if (!(c->rope_theta > 0.0f) || !(c->rms_eps >= 0.0f) || !std::isfinite(c->rope_theta) ||
+      !std::isfinite(c->rms_eps))
+    return DV_ERR_INVALID_ARG;
+  if (c->has_kv_bias != 0 && c->has_kv_bias != 1) return DV_ERR_INVALID_ARG;
+  if (c->d % 64 != 0 || c->d > 16384) return DV_ERR_UNSUPPORTED_SHAPE;
+  if (c->rank > 256) return DV_ERR_UNSUPPORTED_SHAPE;
+  if (c->head_dim != 64 && c->head_dim != 128) return DV_ERR_UNSUPPORTED_SHAPE;
+  if (static_cast<long long>(c->n_kv_heads) * c->head_dim > 8192) return DV_ERR_UNSUPPORTED_SHAPE;
+  if (c->n_layers > 256) return DV_ERR_UNSUPPORTED_SHAPE;
+  if (static_cast<long long>(c->max_batch) * c->max_n_vis > (1LL << 24)) return DV_ERR_UNSUPPORTED_SHAPE;
+  if (c->rope == DV_ROPE_MROPE) {
+    const int* s = c->mrope_section;
+    if (s[0] < 0 || s[1] < 0 || s[2] < 0) return DV_ERR_INVALID_ARG;
+    if (s[0] + s[1] + s[2] != c->head_dim / 2) return DV_ERR_UNSUPPORTED_SHAPE;
+  }
+  return DV_OK;
+}
+
+void free_plan_memory(dv_plan* p) {
+  void* ptrs[] = {p->Dst, p->Bn, p->Wkv, p->bk, p->bv, p->H, p->xx, p->rstd, p->status};
+  for (void* q : ptrs)
+    if (q) cudaFree(q);
+  for (cudaEvent_t e : p->ev) cudaEventDestroy(e);
+  p->ev.clear();
+}
+
+template <typename T>
+bool dmalloc(T** out, size_t bytes) {
+  void* q = nullptr;
+  if (cudaMalloc(&q, bytes) != cudaSuccess) {
+    cudaGetLastError();
+    *out = nullptr;
+    return false;
+  }
+  *out = static_cast<T*>(q);
+  return true;
+}
+
+}  // namespace
+
+// ================================================================================== C ABI
+
+extern "C" {
+
+const char* dv_error_string(int s) {
+  switch (s) {
+    case DV_OK: return "ok";
+    case DV_ERR_INVALID_ARG: return "invalid argument";
+    case DV_ERR_UNSUPPORTED_SHAPE: return "unsupported shape";
+    case DV_ERR_ALIGNMENT: return "pointer or stride not 16-byte aligned";
+    case DV_ERR_OOM: return "device out of memory";
+    case DV_ERR_CUDA: return "CUDA call failed";
+    case DV_ERR_DEVICE_TIMEOUT: return "a device-side wait timed out";
+    case DV_ERR_UNSUPPORTED_DEVICE: return "device is not an sm_103 GPU";
+    default: return "unknown status";
+  }
+}
+
+int dv_memory_plan(const dv_config* cfg, const dv_weights* w, void* stream, dv_plan** out) {
+  if (!out) return DV_ERR_INVALID_ARG;
+  *out = nullptr;
+  int rc = check_config(cfg);
+  if (rc != DV_OK) return rc;
+  if (!w || !w->D || !w->U || !w->gamma || !w->Wk || !w->Wv) return DV_ERR_INVALID_ARG;
+  if (cfg->has_kv_bias && (!w->bk || !w->bv)) return DV_ERR_INVALID_ARG;
+  const void* wp[] = {w->D, w->U, w->gamma, w->Wk, w->Wv};
+  for (const void* q : wp)
+    if (!aligned2(q)) return DV_ERR_ALIGNMENT;
+  if (cfg->has_kv_bias && (!aligned2(w->bk) || !aligned2(w->bv))) return DV_ERR_ALIGNMENT;
+
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return DV_ERR_CUDA;
+  cudaDeviceProp prop;
+  if (cudaGetDeviceProperties(&prop, dev) != cudaSuccess) return DV_ERR_CUDA;
+  if (prop.major != 10 || prop.minor != 3) return DV_ERR_UNSUPPORTED_DEVICE;
+  if (!encode_fn()) return DV_ERR_CUDA;
+
+  dv_plan* p = new (std::nothrow) dv_plan();
+  if (!p) return DV_ERR_OOM;
+  p->cfg = *cfg;
+  p->device = dev;
+  p->num_sms = prop.multiProcessorCount;
+  const int L = cfg->n_layers, d = cfg->d, r = cfg->rank, HD = cfg->head_dim;
+  p->r_pad = (r + 63) / 64 * 64;
+  p->kv = cfg->n_kv_heads * HD;
+  p->k_total = d + p->r_pad;
+  p->max_tokens = cfg->max_batch * cfg->max_n_vis;
+  const long long T = p->max_tokens;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+
+  bool ok = dmalloc(&p->Dst, sizeof(uint16_t) * L * p->r_pad * d) &&
+            dmalloc(&p->Bn, sizeof(uint16_t) * L * p->r_pad * p->k_total) &&
+            dmalloc(&p->Wkv, sizeof(uint16_t) * static_cast<size_t>(L) * 2 * p->kv * p->k_total) &&
+            dmalloc(&p->H, sizeof(uint16_t) * T * L * p->r_pad) &&
+            dmalloc(&p->xx, sizeof(float) * T) && dmalloc(&p->rstd, sizeof(float) * T * L) &&
+            dmalloc(&p->status, sizeof(int));
+  if (ok && cfg->has_kv_bias)
+    ok = dmalloc(&p->bk, sizeof(float) * L * p->kv) && dmalloc(&p->bv, sizeof(float) * L * p->kv);
+  if (!ok) {
+    free_plan_memory(p);
+    delete p;
+    return DV_ERR_OOM;
+  }
+
+  const uint16_t* D = static_cast<const uint16_t*>(w->D);
+  const uint16_t* U = static_cast<const uint16_t*>(w->U);
+  const uint16_t* G = static_cast<const uint16_t*>(w->gamma);
+  const uint16_t* Wk = static_cast<const uint16_t*>(w->Wk);
+  const uint16_t* Wv = static_cast<const uint16_t*>(w->Wv);
+  cudaMemsetAsync(p->status, 0, sizeof(int), st);
+  k_pack_down<<<grid_for(1LL * L * p->r_pad * d), 256, 0, st>>>(D, p->Dst, L, r, p->r_pad, d);
+  k_pack_norm_u<<<grid_for(1LL * L * p->r_pad * p->k_total), 256, 0, st>>>(U, p->Bn, L, r, p->r_pad,
+                                                                           d, p->k_total);
+  k_pack_kv<<<grid_for(1LL * L * 2 * p->kv * p->k_total), 256, 0, st>>>(Wk, Wv, G, p->Wkv, L, p->kv,
+                                                                        HD, d, p->k_total);
+  {
+    dim3 g1((r + 63) / 64, (r + 63) / 64, L);
+    k_rank_product<1><<<g1, 256, 0, st>>>(Wk, Wv, G, U, p->Bn, r, r, d, p->kv, HD, p->r_pad,
+                                          p->k_total);
+    dim3 g0((r + 63) / 64, (2 * p->kv + 63) / 64, L);
+    k_rank_product<0><<<g0, 256, 0, st>>>(Wk, Wv, G, U, p->Wkv, 2 * p->kv, r, d, p->kv, HD,
+                                          p->r_pad, p->k_total);
+  }
+  if (cfg->has_kv_bias) {
+    k_bias_to_f32<<<grid_for(1LL * L * p->kv), 256, 0, st>>>(static_cast<const uint16_t*>(w->bk), p->bk, 1LL * L * p->kv);
+    k_bias_to_f32<<<grid_for(1LL * L * p->kv), 256, 0, st>>>(static_cast<const uint16_t*>(w->bv), p->bv, 1LL * L * p->kv);
+  }
+  cudaError_t err = cudaGetLastError();
+  if (err == cudaSuccess) err = cudaStreamSynchronize(st);
+  if (err != cudaSuccess) {
+    free_plan_memory(p);
+    delete p;
+    return DV_ERR_CUDA;
+  }
+
+  bool enc = encode_2d(&p->tm_Dst[0], p->Dst, d, 1ull * L * p->r_pad, d, 64) &&
+             encode_2d(&p->tm_Dst[1], p->Dst, d, 1ull * L * p->r_pad, d, 128) &&
+             encode_2d(&p->tm_Dst[2], p->Dst, d, 1ull * L * p->r_pad, d, 256) &&
+             encode_2d(&p->tm_Bn, p->Bn, p->k_total, 1ull * L * p->r_pad, p->k_total, p->r_pad) &&
+             encode_2d(&p->tm_Wkv, p->Wkv, p->k_total, 1ull * L * 2 * p->kv, p->k_total, 2 * HD) &&
+             encode_2d(&p->tm_H, p->H, 1ull * L * p->r_pad, T, 1ull * L * p->r_pad, dv::kBlockM);
+  if (!enc) {
+    free_plan_memory(p);
+    delete p;
+    return DV_ERR_CUDA;
+  }
+  for (int j = 0; j < HD / 2; ++j)
+    p->inv_freq[j] = std::pow(static_cast<double>(cfg->rope_theta), -2.0 * j / HD);
+  *out = p;
+  return DV_OK;
+}
+
+int dv_kernels_per_build(const dv_plan* p) { return p ? kStages : 0; }
+
+int dv_build_visual_memory(dv_plan* p, const void* x0, int batch, int n_vis, const int* pos,
+                           const int* slot, int slot0, const dv_kv_cache* out, void* stream) {
+  if (!p) return DV_ERR_INVALID_ARG;
+  if (batch < 0 || n_vis < 0 || slot0 < 0) return DV_ERR_INVALID_ARG;
+  const long long T = static_cast<long long>(batch) * n_vis;
+  if (T == 0) return DV_OK;
+  if (!x0 || !pos || !out || !out->k || !out->v) return DV_ERR_INVALID_ARG;
+  if (batch > p->cfg.max_batch || n_vis > p->cfg.max_n_vis || T > p->max_tokens)
+    return DV_ERR_UNSUPPORTED_SHAPE;
+  if (!aligned16(x0) || !aligned16(out->k) || !aligned16(out->v)) return DV_ERR_ALIGNMENT;
+  const long long s[4] = {out->s_layer, out->s_batch, out->s_seq, out->s_head};
+  for (long long v : s) {
+    if (v < 0) return DV_ERR_INVALID_ARG;
+    if (v % 8 != 0) return DV_ERR_ALIGNMENT;
+  }
+  if ((reinterpret_cast<uintptr_t>(pos) & 3u) || (slot && (reinterpret_cast<uintptr_t>(slot) & 3u)))
+    return DV_ERR_ALIGNMENT;
+
+  const dv_config& c = p->cfg;
+  const int L = c.n_layers, d = c.d, HD = c.head_dim;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  CUtensorMap tm_x0;
+  if (!encode_2d(&tm_x0, x0, d, static_cast<uint64_t>(T), d, dv::kBlockM)) return DV_ERR_CUDA;
+
+  cudaEvent_t* ev = nullptr;
+  if (p->timing && p->timed < kMaxTimed) ev = &p->ev[static_cast<size_t>(p->timed++) * kEvPerBuild];
+  auto mark = [&](int i) {
+    if (ev) cudaEventRecord(ev[i], st);
+  };
+
+  GemmParams gp;
+  std::memset(&gp, 0, sizeof(gp));
+  gp.status = p->status;
+  gp.timeout_ns = kTimeoutNs;
+
+  mark(0);
+  k_row_sumsq<<<static_cast<int>((T + 7) / 8), 256, 0, st>>>(static_cast<const uint16_t*>(x0),
+                                                             static_cast<int>(T), d, p->xx);
+  cudaError_t err = cudaGetLastError();
+  mark(1);
+
+  // (1) H = SiLU(x0 [D_1 ... D_L]) — one GEMM over all layers' down-projections.
+  const int n1 = L * p->r_pad;
+  const long long m_tiles = (T + dv::kBlockM - 1) / dv::kBlockM;
+  int bn1 = 64;
+  for (int cand : {256, 128}) {
+    if (n1 % cand == 0 && m_tiles * (n1 / cand) >= p->num_sms) {
+      bn1 = cand;
+      break;
+    }
+  }
+  gp.s = {static_cast<int>(T), 1, n1, d / 64, 0, 0};
+  gp.silu = {p->H, n1};
+  const CUtensorMap& tmD = p->tm_Dst[bn1 == 64 ? 0 : (bn1 == 128 ? 1 : 2)];
+  if (err == cudaSuccess) err = dv::launch_gemm(dv::EPI_SILU, bn1, 0, tm_x0, tm_x0, tmD, gp, p->num_sms, st);
+  mark(2);
+
+  // (2) rstd_l from ||x0||^2 + h_l . ([x0 | h_l] [2 U_l^T ; G_l]).
+  gp.s = {static_cast<int>(T), L, p->r_pad, d / 64, p->r_pad / 64, p->r_pad};
+  gp.norm = {p->H, n1, p->r_pad, p->xx, p->rstd, p->max_tokens, 1.0f / d, c.rms_eps};
+  if (err == cudaSuccess)
+    err = dv::launch_gemm(dv::EPI_NORM, p->r_pad, 0, tm_x0, p->tm_H, p->tm_Bn, gp, p->num_sms, st);
+  mark(3);
+
+  // (3) K/V = rstd_l * ([x0 | h_l] Wkv_l^T) + b, RoPE on K, stored into the cache.
+  gp.s = {static_cast<int>(T), L, 2 * p->kv, d / 64, p->r_pad / 64, p->r_pad};
+  dv::EpiKV& e = gp.kv;
+  e.rstd = p->rstd;
+  e.ld_rstd = p->max_tokens;
+  e.bk = p->bk;
+  e.bv = p->bv;
+  e.kv = p->kv;
+  e.pos = pos;
+  e.slot = slot;
+  e.slot0 = slot0;
+  e.n_vis = n_vis;
+  e.n_pos = c.rope == DV_ROPE_MROPE ? 3 : 1;
+  e.sec0 = c.rope == DV_ROPE_MROPE ? c.mrope_section[0] : HD / 2;
+  e.sec01 = c.rope == DV_ROPE_MROPE ? c.mrope_section[0] + c.mrope_section[1] : HD / 2;
+  e.kc = static_cast<uint16_t*>(out->k);
+  e.vc = static_cast<uint16_t*>(out->v);
+  e.s_layer = out->s_layer;
+  e.s_batch = out->s_batch;
+  e.s_seq = out->s_seq;
+  e.s_head = out->s_head;
+  const double two_pi = 6.283185307179586476925286766559;
+  e.two_pi_hi = static_cast<float>(two_pi);
+  e.two_pi_lo = static_cast<float>(two_pi - static_cast<double>(e.two_pi_hi));
+  e.inv_two_pi = static_cast<float>(1.0 / two_pi);
+  for (int j = 0; j < HD / 2; ++j) {
+    e.inv_freq_hi[j] = static_cast<float>(p->inv_freq[j]);
+    e.inv_freq_lo[j] = static_cast<float>(p->inv_freq[j] - static_cast<double>(e.inv_freq_hi[j]));
+  }
+  if (err == cudaSuccess)
+    err = dv::launch_gemm(dv::EPI_KV, 2 * HD, HD, tm_x0, p->tm_H, p->tm_Wkv, gp, p->num_sms, st);
+  mark(4);
+  return err == cudaSuccess ? DV_OK : DV_ERR_CUDA;
+}
+
+int dv_plan_status(dv_plan* p) {
+  if (!p) return DV_ERR_INVALID_ARG;
+  int s = 0;
+  if (cudaDeviceSynchronize() != cudaSuccess) return DV_ERR_CUDA;
+  if (cudaMemcpy(&s, p->status, sizeof(int), cudaMemcpyDeviceToHost) != cudaSuccess) return DV_ERR_CUDA;
+  if (s != 0 && cudaMemset(p->status, 0, sizeof(int)) != cudaSuccess) return DV_ERR_CUDA;
+  return s;
+}
+
+void dv_free(dv_plan* p) {
+  if (!p) return;
+  cudaDeviceSynchronize();
+  free_plan_memory(p);
+  delete p;
+}
+
+int dv_timing_enable(dv_plan* p, int on) {
+  if (!p) return DV_ERR_INVALID_ARG;
+  p->timing = on != 0;
+  p->timed = 0;
+  if (on && p->ev.empty()) {
+    p->ev.resize(static_cast<size_t>(kMaxTimed) * kEvPerBuild);
+    for (auto& e : p->ev)
+      if (cudaEventCreate(&e) != cudaSuccess) return DV_ERR_CUDA;
+  }
+  return DV_OK;
+}
+
+int dv_timing_read(dv_plan* p, double* ms, int n_stages, int* n_builds) {
+  if (!p || !ms || !n_builds || n_stages < 0 || n_stages > kStages) return DV_ERR_INVALID_ARG;
+  for (int s = 0; s < n_stages; ++s) ms[s] = 0.0;
+  for (int b = 0; b < p->timed; ++b) {
+    cudaEvent_t* ev = &p->ev[static_cast<size_t>(b) * kEvPerBuild];
+    if (cudaEventSynchronize(ev[kStages]) != cudaSuccess) return DV_ERR_CUDA;
+    for (int s = 0; s < n_stages; ++s) {
+      float t = 0.0f;
+      if (cudaEventElapsedTime(&t, ev[s], ev[s + 1]) != cudaSuccess) return DV_ERR_CUDA;
+      ms[s] += t;
+    }
+  }
+  *n_builds = p->timed;
+  return DV_OK;
+}
+
+int dv_debug_wait_timeout(dv_plan* p, int timeout_us, void* stream) {
+  if (!p || timeout_us < 1 || timeout_us > 2000000) return DV_ERR_INVALID_ARG;
+  k_wait_timeout<<<1, 32, 0, static_cast<cudaStream_t>(stream)>>>(
+      p->status, static_cast<unsigned long long>(timeout_us) * 1000ull);
+  return cudaGetLastError() == cudaSuccess ? DV_OK : DV_ERR_CUDA;
+}
+
+int dv_debug_copy_workspace(dv_plan* p, int tokens, void* H, void* rstd, void* xx,
+                            int* r_pad_out, void* stream) {
+  if (!p || tokens < 0 || tokens > p->max_tokens) return DV_ERR_INVALID_ARG;
+  if (r_pad_out) *r_pad_out = p->r_pad;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  const int L = p->cfg.n_layers;
+  const size_t hrow = static_cast<size_t>(L) * p->r_pad;
+  cudaError_t err = cudaSuccess;
+  if (H && tokens > 0)
+    err = cudaMemcpyAsync(H, p->H, sizeof(uint16_t) * hrow * tokens, cudaMemcpyDeviceToDevice, st);
+  if (rstd && tokens > 0 && err == cudaSuccess)
+    err = cudaMemcpy2DAsync(rstd, sizeof(float) * tokens, p->rstd, sizeof(float) * p->max_tokens,
+                            sizeof(float) * tokens, L, cudaMemcpyDeviceToDevice, st);
+  if (xx && tokens > 0 && err == cudaSuccess)
+    err = cudaMemcpyAsync(xx, p->xx, sizeof(float) * tokens, cudaMemcpyDeviceToDevice, st);
+  return err == cudaSuccess ? DV_OK : DV_ERR_CUDA;
+}
+
+}  // extern "C"

@@ -1,0 +1,429 @@
+// Persistent, warp-specialised tcgen05 GEMM for the three contractions of the visual-memory
+// build, each with its own fused epilogue:
+//   EPI_SILU  H   = SiLU(x0 [D_1 ... D_L])          all L down-projections as one GEMM, since
+//                                                    every layer reads only E (Sec. 3.1 Eq. 5)
+//   EPI_NORM  rstd_l = (||M_l||^2 / d + eps)^-1/2    the RMS statistic of M_l = x0 + h_l U_l
+//                                                    (Sec. 3.1 Eq. 4), from [x0 | h_l] times
+//                                                    [2 U_l^T ; U_l U_l^T]
+//   EPI_KV    K_l, V_l = rstd_l * ([x0 | h_l] W~_l) (+ b), RoPE on K, bf16 cache store
+//                                                    (Sec. 3.2 Eq. 7)
+//
+// CTA layout (192 threads, one CTA per SM):
+//   warp 0      TMA producer: one lane streams 64-wide K slabs of A (128 token rows) and B
+//               (BLOCK_N weight rows) into a ring of shared-memory stages
+//   warp 1      owns the TMEM allocation; one lane issues tcgen05.mma (128 x BLOCK_N x 16)
+//               into one of two TMEM accumulators
+//   warps 2-5   epilogue: each thread owns one token row (TMEM lane) of the finished
+//               accumulator, while the MMA warp fills the other accumulator
+// Tiles are visited in (layer, n-block, m-block) order, m fastest, so the CTAs working at the
+// same time share weight tiles through L2.
+#include <cstdio>
+
+#include "dv_internal.h"
+#include "dv_ptx.cuh"
+
+namespace dv {
+
+constexpr int kNumThreads = 192;
+constexpr int kEpiThreads = 128;
+constexpr int kRingBytes = 192 * 1024;
+
+template <int BN>
+struct TileCfg {
+  static constexpr int kABytes = kBlockM * kBlockK * 2;
+  static constexpr int kBBytes = BN * kBlockK * 2;
+  static constexpr int kStageBytes = kABytes + kBBytes;
+  static constexpr int kStagesRaw = kRingBytes / kStageBytes;
+  static constexpr int kStages = kStagesRaw > 8 ? 8 : kStagesRaw;
+  static constexpr int kTmemCols = 2 * BN;
+  static constexpr int kSmemBytes = kStages * kStageBytes + 1024 + 256;
+  static_assert(kStageBytes % 1024 == 0, "stage tiles must stay 1024-byte aligned");
+  static_assert(kTmemCols >= 32 && kTmemCols <= 512 && (kTmemCols & (kTmemCols - 1)) == 0,
+                "TMEM allocation must be a power of two in [32, 512]");
+};
+
+// Wait with a time limit only (used to drain in-flight work after an abort).
+__device__ __forceinline__ bool wait_drain(uint32_t bar, uint32_t parity, uint64_t timeout_ns) {
+  int never = 0;
+  return mbar_wait(bar, parity, &never, timeout_ns);
+}
+
+__device__ __forceinline__ void store_row32(uint16_t* dst, const uint32_t (&pk)[16]) {
+  uint4* d = reinterpret_cast<uint4*>(dst);
+  d[0] = make_uint4(pk[0], pk[1], pk[2], pk[3]);
+  d[1] = make_uint4(pk[4], pk[5], pk[6], pk[7]);
+  d[2] = make_uint4(pk[8], pk[9], pk[10], pk[11]);
+  d[3] = make_uint4(pk[12], pk[13], pk[14], pk[15]);
+}
+
+// ------------------------------------------------------------------------------ epilogues
+
+// H[t, n*BN + c] = bf16(SiLU(z)), SiLU(z) = z / (1 + e^-z)  (phi of Sec. 3.1 Eq. 4).
+template <int BN>
+__device__ __forceinline__ void epi_silu(const GemmParams& p, uint32_t tbase, int n, int t) {
+  const bool valid = t < p.s.M;
+  uint16_t* out = p.silu.H + static_cast<size_t>(valid ? t : 0) * p.silu.ldh +
+                  static_cast<size_t>(n) * BN;
+#pragma unroll 1
+  for (int c = 0; c < BN / 32; ++c) {
+    uint32_t r[32];
+    __syncwarp();
+    tmem_ld32(tbase + c * 32, r);
+    tmem_ld_wait();
+    uint32_t pk[16];
+#pragma unroll
+    for (int u = 0; u < 16; ++u) {
+      const float z0 = __uint_as_float(r[2 * u]), z1 = __uint_as_float(r[2 * u + 1]);
+      pk[u] = pack_bf16x2(z0 / (1.0f + __expf(-z0)), z1 / (1.0f + __expf(-z1)));
+    }
+    if (valid) store_row32(out + c * 32, pk);
+  }
+}
+
+// ||m||^2 = ||x0||^2 + h . (2 x0 U^T + h G) with G = U U^T, so with acc = [x0 | h] [2U^T; G]
+// the statistic of RMSNorm is rstd = 1 / sqrt((xx + h . acc) / d + eps).
+template <int BN>
+__device__ __forceinline__ void epi_norm(const GemmParams& p, uint32_t tbase, int l, int t) {
+  const bool valid = t < p.s.M;
+  const uint16_t* hrow = p.norm.H + static_cast<size_t>(valid ? t : 0) * p.norm.ldh +
+                         static_cast<size_t>(l) * p.norm.r_pad;
+  float dot = 0.0f;
+#pragma unroll 1
+  for (int c = 0; c < BN / 32; ++c) {
+    uint32_t r[32];
+    __syncwarp();
+    tmem_ld32(tbase + c * 32, r);
+    tmem_ld_wait();
+    if (valid) {
+      const uint4* hv = reinterpret_cast<const uint4*>(hrow + c * 32);
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        const uint4 w = hv[q];
+        const uint32_t ws[4] = {w.x, w.y, w.z, w.w};
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          dot = fmaf(bf16_bits_to_float(ws[e] & 0xFFFFu), __uint_as_float(r[q * 8 + 2 * e]), dot);
+          dot = fmaf(bf16_bits_to_float(ws[e] >> 16), __uint_as_float(r[q * 8 + 2 * e + 1]), dot);
+        }
+      }
+    }
+  }
+  if (valid) {
+    const float ss = fmaxf(p.norm.xx[t] + dot, 0.0f);
+    p.norm.rstd[static_cast<size_t>(l) * p.norm.ld_rstd + t] =
+        rsqrtf(fmaf(ss, p.norm.inv_d, p.norm.eps));
+  }
+}
+
+// Angle p * theta^(-2j/D_h) reduced to [-pi, pi] before the sine/cosine: the product is kept
+// as an unevaluated sum of two floats (fma residual), then reduced by Cody-Waite subtraction of
+// k * 2pi with 2pi split into two floats.
+__device__ __forceinline__ void rope_sincos(float pos, float fhi, float flo, const EpiKV& kv,
+                                            float& s, float& c) {
+  const float a_hi = pos * fhi;
+  const float a_lo = fmaf(pos, flo, fmaf(pos, fhi, -a_hi));
+  const float k = rintf(a_hi * kv.inv_two_pi);
+  float r = fmaf(-k, kv.two_pi_hi, a_hi);
+  r = fmaf(-k, kv.two_pi_lo, r) + a_lo;
+  __sincosf(r, &s, &c);
+}
+
+// K/V tile of one head: columns [0, HD) are K head h, [HD, 2HD) are V head h (plan packing).
+// k = rstd * acc + b_K, rotated in rotate-half pairs (j, j + HD/2); v = rstd * acc + b_V.
+template <int HD>
+__device__ __forceinline__ void epi_kv(const GemmParams& p, uint32_t tbase, int l, int h, int t) {
+  constexpr int kHalf = HD / 2;
+  const EpiKV& e = p.kv;
+  const bool valid = t < p.s.M;
+  const int tt = valid ? t : 0;
+  const int b = tt / e.n_vis, i = tt - b * e.n_vis;
+  const float rs = valid ? e.rstd[static_cast<size_t>(l) * e.ld_rstd + tt] : 0.0f;
+  const int slot = e.slot ? e.slot[tt] : e.slot0 + i;
+  const long long off = l * e.s_layer + b * e.s_batch + slot * e.s_seq + h * e.s_head;
+  uint16_t* krow = e.kc + off;
+  uint16_t* vrow = e.vc + off;
+  const int* pp = e.pos + static_cast<size_t>(b) * e.n_pos * e.n_vis + i;
+  const float pt = static_cast<float>(pp[0]);
+  const float ph = e.n_pos == 3 ? static_cast<float>(pp[e.n_vis]) : pt;
+  const float pw = e.n_pos == 3 ? static_cast<float>(pp[2 * e.n_vis]) : pt;
+  const float* bk = e.bk ? e.bk + static_cast<size_t>(l) * e.kv + h * HD : nullptr;
+  const float* bv = e.bv ? e.bv + static_cast<size_t>(l) * e.kv + h * HD : nullptr;
+
+#pragma unroll 1
+  for (int jb = 0; jb < kHalf / 32; ++jb) {
+    uint32_t lo[32], hi[32];
+    __syncwarp();
+    tmem_ld32(tbase + jb * 32, lo);
+    tmem_ld32(tbase + kHalf + jb * 32, hi);
+    tmem_ld_wait();
+    uint32_t plo[16], phi[16];
+#pragma unroll
+    for (int u = 0; u < 32; u += 2) {
+      float y1[2], y2[2];
+#pragma unroll
+      for (int w = 0; w < 2; ++w) {
+        const int j = jb * 32 + u + w;
+        float x1 = __uint_as_float(lo[u + w]) * rs;
+        float x2 = __uint_as_float(hi[u + w]) * rs;
+        if (bk) {
+          x1 += bk[j];
+          x2 += bk[kHalf + j];
+        }
+        const float pj = j < e.sec0 ? pt : (j < e.sec01 ? ph : pw);
+        float s, c;
+        rope_sincos(pj, e.inv_freq_hi[j], e.inv_freq_lo[j], e, s, c);
+        y1[w] = x1 * c - x2 * s;
+        y2[w] = x2 * c + x1 * s;
+      }
+      plo[u / 2] = pack_bf16x2(y1[0], y1[1]);
+      phi[u / 2] = pack_bf16x2(y2[0], y2[1]);
+    }
+    if (valid) {
+      store_row32(krow + jb * 32, plo);
+      store_row32(krow + kHalf + jb * 32, phi);
+    }
+  }
+#pragma unroll 1
+  for (int jb = 0; jb < HD / 32; ++jb) {
+    uint32_t r[32];
+    __syncwarp();
+    tmem_ld32(tbase + HD + jb * 32, r);
+    tmem_ld_wait();
+    uint32_t pk[16];
+#pragma unroll
+    for (int u = 0; u < 16; ++u) {
+      float v0 = __uint_as_float(r[2 * u]) * rs, v1 = __uint_as_float(r[2 * u + 1]) * rs;
+      if (bv) {
+        v0 += bv[jb * 32 + 2 * u];
+        v1 += bv[jb * 32 + 2 * u + 1];
+      }
+      pk[u] = pack_bf16x2(v0, v1);
+    }
+    if (valid) store_row32(vrow + jb * 32, pk);
+  }
+}
+
+// ------------------------------------------------------------------------------ the kernel
+
+template <int EPI, int BN, int HD>
+__global__ void __launch_bounds__(kNumThreads, 1)
+    dv_gemm_kernel(const __grid_constant__ CUtensorMap tmA0, const __grid_constant__ CUtensorMap tmA1,
+                   const __grid_constant__ CUtensorMap tmB, const __grid_constant__ GemmParams p) {
+  using C = TileCfg<BN>;
+  constexpr int S = C::kStages;
+  extern __shared__ uint8_t smem_raw[];
+  const uint32_t raw = smem_addr(smem_raw);
+  const uint32_t ring = (raw + 1023u) & ~1023u;
+  uint8_t* ring_ptr = smem_raw + (ring - raw);
+  uint64_t* bars = reinterpret_cast<uint64_t*>(ring_ptr + S * C::kStageBytes);
+  const uint32_t bar0 = smem_addr(bars);
+  auto full_bar = [&](int s) { return bar0 + 8u * s; };
+  auto empty_bar = [&](int s) { return bar0 + 8u * (S + s); };
+  auto tfull_bar = [&](int a) { return bar0 + 8u * (2 * S + a); };
+  auto tempty_bar = [&](int a) { return bar0 + 8u * (2 * S + 2 + a); };
+  const uint32_t drain_bar = bar0 + 8u * (2 * S + 4);
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 2 * S + 5);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const uint64_t tmo = p.timeout_ns;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < S; ++s) {
+      mbar_init(full_bar(s), 1);
+      mbar_init(empty_bar(s), 1);
+    }
+    for (int a = 0; a < 2; ++a) {
+      mbar_init(tfull_bar(a), 1);
+      mbar_init(tempty_bar(a), kEpiThreads);
+    }
+    mbar_init(drain_bar, 1);
+    *abort_flag = 0;
+    fence_barrier_init();
+  }
+  if (warp == 0 && lane == 0) {
+    tma_prefetch_desc(&tmA0);
+    if (p.s.k1_slabs > 0) tma_prefetch_desc(&tmA1);
+    tma_prefetch_desc(&tmB);
+  }
+  if (warp == 1) {
+    tmem_alloc(smem_addr(tmem_slot), C::kTmemCols);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem_base = *tmem_slot;
+
+  const int m_tiles = (p.s.M + kBlockM - 1) / kBlockM;
+  const int n_tiles = p.s.n_per_layer / BN;
+  const int num_tiles = m_tiles * n_tiles * p.s.n_layers;
+  const int k_slabs = p.s.k0_slabs + p.s.k1_slabs;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      // ---------------------------------------------------------------- TMA producer
+      int stage = 0;
+      uint32_t phase = 0, used = 0, issued_parity = 0;
+      for (int tile = blockIdx.x; tile < num_tiles && !*abort_flag; tile += gridDim.x) {
+        const int m = tile % m_tiles;
+        const int rest = tile / m_tiles;
+        const int n = rest % n_tiles;
+        const int l = rest / n_tiles;
+        const int brow = l * p.s.n_per_layer + n * BN;
+        for (int ks = 0; ks < k_slabs; ++ks) {
+          if (!mbar_wait(empty_bar(stage), phase ^ 1u, abort_flag, tmo)) break;
+          const uint32_t a_dst = ring + stage * C::kStageBytes;
+          const uint32_t b_dst = a_dst + C::kABytes;
+          mbar_arrive_expect_tx(full_bar(stage), C::kStageBytes);
+          if (ks < p.s.k0_slabs) {
+            tma_load_2d(a_dst, &tmA0, full_bar(stage), ks * kBlockK, m * kBlockM);
+          } else {
+            tma_load_2d(a_dst, &tmA1, full_bar(stage),
+                        l * p.s.a1_cols_per_layer + (ks - p.s.k0_slabs) * kBlockK, m * kBlockM);
+          }
+          tma_load_2d(b_dst, &tmB, full_bar(stage), ks * kBlockK, brow);
+          used |= 1u << stage;
+          issued_parity = (issued_parity & ~(1u << stage)) | (phase << stage);
+          if (++stage == S) {
+            stage = 0;
+            phase ^= 1u;
+          }
+        }
+      }
+      if (*abort_flag) {  // let every copy still in flight land before the CTA exits
+        for (int s = 0; s < S; ++s)
+          if (used & (1u << s)) wait_drain(full_bar(s), (issued_parity >> s) & 1u, tmo);
+      }
+    }
+  } else if (warp == 1) {
+    if (lane == 0) {
+      // ---------------------------------------------------------------- MMA issuer
+      const uint32_t idesc = idesc_bf16_f32(kBlockM, BN);
+      int stage = 0, acc = 0;
+      uint32_t phase = 0, acc_phase = 0;
+      bool issued_any = false;
+      for (int tile = blockIdx.x; tile < num_tiles && !*abort_flag; tile += gridDim.x) {
+        if (!mbar_wait(tempty_bar(acc), acc_phase ^ 1u, abort_flag, tmo)) break;
+        tc_fence_after();
+        const uint32_t d_tmem = tmem_base + static_cast<uint32_t>(acc * BN);
+        bool ok = true;
+        for (int ks = 0; ks < k_slabs; ++ks) {
+          if (!mbar_wait(full_bar(stage), phase, abort_flag, tmo)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t a_s = ring + stage * C::kStageBytes;
+          const uint32_t b_s = a_s + C::kABytes;
+#pragma unroll
+          for (int k = 0; k < kBlockK / 16; ++k) {
+            umma_bf16(d_tmem, sdesc_kmajor_sw128(a_s + 32u * k), sdesc_kmajor_sw128(b_s + 32u * k),
+                      idesc, (ks | k) != 0 ? 1u : 0u);
+          }
+          issued_any = true;
+          umma_commit(empty_bar(stage));
+          if (++stage == S) {
+            stage = 0;
+            phase ^= 1u;
+          }
+        }
+        if (!ok) break;
+        umma_commit(tfull_bar(acc));
+        if (++acc == 2) {
+          acc = 0;
+          acc_phase ^= 1u;
+        }
+      }
+      if (*abort_flag && issued_any) {  // no TMEM release while an MMA may still run
+        umma_commit(drain_bar);
+        wait_drain(drain_bar, 0, tmo);
+      }
+    }
+  } else {
+    // ------------------------------------------------------------------ epilogue warps
+    const int q = warp & 3;  // the TMEM lane quarter this warp may access
+    const int row = q * 32 + lane;
+    int acc = 0;
+    uint32_t acc_phase = 0;
+    for (int tile = blockIdx.x; tile < num_tiles; tile += gridDim.x) {
+      const int m = tile % m_tiles;
+      const int rest = tile / m_tiles;
+      const int n = rest % n_tiles;
+      const int l = rest / n_tiles;
+      if (!mbar_wait(tfull_bar(acc), acc_phase, abort_flag, tmo)) break;
+      tc_fence_after();
+      const uint32_t tbase =
+          tmem_base + (static_cast<uint32_t>(q * 32) << 16) + static_cast<uint32_t>(acc * BN);
+      const int t = m * kBlockM + row;
+      if constexpr (EPI == EPI_SILU) {
+        epi_silu<BN>(p, tbase, n, t);
+      } else if constexpr (EPI == EPI_NORM) {
+        epi_norm<BN>(p, tbase, l, t);
+      } else {
+        epi_kv<HD>(p, tbase, l, n, t);
+      }
+      tc_fence_before();
+      mbar_arrive(tempty_bar(acc));
+      if (++acc == 2) {
+        acc = 0;
+        acc_phase ^= 1u;
+      }
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  if (threadIdx.x == 0 && *abort_flag) atomicExch(p.status, 6 /* DV_ERR_DEVICE_TIMEOUT */);
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem_base, C::kTmemCols);
+  }
+}
+
+// ------------------------------------------------------------------------------ launch
+
+template <int EPI, int BN, int HD>
+static cudaError_t launch_t(const CUtensorMap& a0, const CUtensorMap& a1, const CUtensorMap& b,
+                            const GemmParams& p, int num_sms, cudaStream_t stream) {
+  using C = TileCfg<BN>;
+  auto kern = dv_gemm_kernel<EPI, BN, HD>;
+  cudaError_t err =
+      cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, C::kSmemBytes);
+  if (err != cudaSuccess) return err;
+  const long long m_tiles = (p.s.M + kBlockM - 1) / kBlockM;
+  const long long tiles = m_tiles * (p.s.n_per_layer / BN) * p.s.n_layers;
+  if (tiles <= 0) return cudaSuccess;
+  const int grid = static_cast<int>(tiles < num_sms ? tiles : num_sms);
+  kern<<<grid, kNumThreads, C::kSmemBytes, stream>>>(a0, a1, b, p);
+  return cudaGetLastError();
+}
+
+int gemm_smem_bytes(int block_n) {
+  switch (block_n) {
+    case 64: return TileCfg<64>::kSmemBytes;
+    case 128: return TileCfg<128>::kSmemBytes;
+    case 256: return TileCfg<256>::kSmemBytes;
+    default: return -1;
+  }
+}
+
+cudaError_t launch_gemm(int epi, int block_n, int head_dim, const CUtensorMap& a0,
+                        const CUtensorMap& a1, const CUtensorMap& b, const GemmParams& p,
+                        int num_sms, cudaStream_t stream) {
+  if (epi == EPI_SILU) {
+    if (block_n == 64) return launch_t<EPI_SILU, 64, 0>(a0, a1, b, p, num_sms, stream);
+    if (block_n == 128) return launch_t<EPI_SILU, 128, 0>(a0, a1, b, p, num_sms, stream);
+    if (block_n == 256) return launch_t<EPI_SILU, 256, 0>(a0, a1, b, p, num_sms, stream);
+  } else if (epi == EPI_NORM) {
+    if (block_n == 64) return launch_t<EPI_NORM, 64, 0>(a0, a1, b, p, num_sms, stream);
+    if (block_n == 128) return launch_t<EPI_NORM, 128, 0>(a0, a1, b, p, num_sms, stream);
+    if (block_n == 256) return launch_t<EPI_NORM, 256, 0>(a0, a1, b, p, num_sms, stream);
+  } else if (epi == EPI_KV) {
+    if (head_dim == 64 && block_n == 128) return launch_t<EPI_KV, 128, 64>(a0, a1, b, p, num_sms, stream);
+    if (head_dim == 128 && block_n == 256) return launch_t<EPI_KV, 256, 128>(a0, a1, b, p, num_sms, stream);
+  }
+  return cudaErrorInvalidValue;
+}
+
+}  // namespace dv

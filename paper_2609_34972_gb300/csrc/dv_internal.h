@@ -1,0 +1,88 @@
+// Internal interface between the C-ABI / plan code (dv_api.cu) and the tcgen05 GEMM kernels
+// (dv_gemm.cu). Not part of the public ABI.
+#pragma once
+#include <cstdint>
+#include <cuda.h>
+#include <cuda_runtime.h>
+
+namespace dv {
+
+constexpr int kBlockM = 128;         // UMMA M: one TMEM lane per token row
+constexpr int kBlockK = 64;          // bf16 elements per 128-byte swizzled row of a K slab
+constexpr int kMaxHalfHead = 64;     // head_dim <= 128
+
+enum Epilogue : int {
+  EPI_SILU = 0,  // stacked down-projection: H = bf16(SiLU(acc))
+  EPI_NORM = 1,  // RMS statistic: rstd = (||x0||^2 + h . acc) / d + eps) ^ -1/2
+  EPI_KV = 2,    // K/V: rstd * acc + bias, RoPE on K, bf16 store into the cache
+};
+
+// Operand schedule shared by all three GEMMs. The A operand of a tile is the 128-row token
+// block of [x0 | H_l]: k0_slabs 64-wide slabs of x0 (tensor map A0), then k1_slabs slabs of H
+// starting at column layer * a1_cols_per_layer (tensor map A1). B is one stacked weight
+// matrix whose rows for layer l start at l * n_per_layer; its columns follow the same slab
+// order as A.
+struct GemmShape {
+  int M;                  // tokens in this build
+  int n_layers;           // groups (layers)
+  int n_per_layer;        // output columns per layer (multiple of BLOCK_N)
+  int k0_slabs;           // d / 64
+  int k1_slabs;           // r_pad / 64, or 0
+  int a1_cols_per_layer;  // r_pad
+};
+
+struct EpiSilu {
+  uint16_t* H;   // bf16 [M_ld][ldh]
+  int ldh;
+};
+
+struct EpiNorm {
+  const uint16_t* H;  // bf16 [M_ld][ldh], h_l at columns l * r_pad
+  int ldh;
+  int r_pad;
+  const float* xx;    // [M] row sums of squares of x0
+  float* rstd;        // [L][ld_rstd]
+  int ld_rstd;
+  float inv_d;
+  float eps;
+};
+
+struct EpiKV {
+  const float* rstd;  // [L][ld_rstd]
+  int ld_rstd;
+  const float* bk;    // fp32 [L][kv] or null
+  const float* bv;
+  int kv;
+  const int* pos;     // int32 [B][P][n_vis]
+  const int* slot;    // int32 [B][n_vis] or null
+  int slot0;
+  int n_vis;
+  int n_pos;          // 1 or 3
+  int sec0, sec01;    // M-RoPE: pairs [0,sec0) -> t, [sec0,sec01) -> h, rest -> w
+  uint16_t* kc;
+  uint16_t* vc;
+  long long s_layer, s_batch, s_seq, s_head;
+  float two_pi_hi, two_pi_lo, inv_two_pi;
+  float inv_freq_hi[kMaxHalfHead];  // theta^(-2j/D_h) split into two floats
+  float inv_freq_lo[kMaxHalfHead];
+};
+
+struct GemmParams {
+  GemmShape s;
+  EpiSilu silu;
+  EpiNorm norm;
+  EpiKV kv;
+  int* status;              // device status word
+  unsigned long long timeout_ns;
+};
+
+// Launches one persistent warp-specialised tcgen05 GEMM. Returns a cudaError_t value.
+// block_n: 64/128/256 for EPI_SILU and EPI_NORM; 2*head_dim (128 or 256) for EPI_KV.
+cudaError_t launch_gemm(int epi, int block_n, int head_dim, const CUtensorMap& a0,
+                        const CUtensorMap& a1, const CUtensorMap& b, const GemmParams& p,
+                        int num_sms, cudaStream_t stream);
+
+// Shared-memory bytes one CTA of that GEMM asks for (for validation and reporting).
+int gemm_smem_bytes(int block_n);
+
+}  // namespace dv

@@ -1,0 +1,109 @@
+"""Helpers for the GPU tests: move seeded inputs to the device, run the C-ABI build through the
+Python binding, gather cache rows, and apply the parity bar against the oracle.
+
+Parity bar (bf16 inputs, fp32 accumulation): for every K and V element,
+    |gpu - oracle| / max(|oracle|, rms of the oracle's head row) <= 2e-2,
+and per (token, layer) the cosine between the GPU and oracle kv vectors is >= 0.9999,
+separately for K and V.
+"""
+from __future__ import annotations
+
+import numpy as np
+
+import synth
+
+REL_TOL = 2e-2
+COS_TOL = 0.9999
+
+
+def torch_bf16(bits, device):
+    import torch
+    a = np.ascontiguousarray(bits, dtype=np.uint16)
+    return torch.from_numpy(a.view(np.int16)).view(torch.bfloat16).to(device)
+
+
+def device_weights(inp, device="cuda"):
+    w = {n: torch_bf16(getattr(inp, n), device) for n in ("D", "U", "gamma", "Wk", "Wv")}
+    if inp.bk is not None:
+        w["bk"] = torch_bf16(inp.bk, device)
+        w["bv"] = torch_bf16(inp.bv, device)
+    return w
+
+
+def dv_config(cfg, max_batch=None, max_n_vis=None):
+    import paper_2609_34972_gb300 as dv
+    return dv.make_config(cfg.d, cfg.n_layers, cfg.n_kv_heads, cfg.head_dim, cfg.rank,
+                          rope=cfg.rope, rope_theta=cfg.rope_theta,
+                          mrope_section=cfg.mrope_section, rms_eps=cfg.rms_eps,
+                          max_batch=max_batch or cfg.batch, max_n_vis=max_n_vis or cfg.n_vis,
+                          has_kv_bias=cfg.bias_sigma > 0)
+
+
+def run_build(inp, plan=None, seq_len=None, batch_cache=None, slot=None, slot0=0, fill=0.0):
+    """Plan (unless given) and build into a fresh [L, B_c, S, H, D_h] cache; returns (k, v, plan)."""
+    import torch
+    import paper_2609_34972_gb300 as dv
+    cfg = inp.cfg
+    dev = torch.device("cuda")
+    if plan is None:
+        plan = dv.memory_plan(dv_config(cfg), device_weights(inp, dev))
+    S = seq_len or cfg.n_vis
+    Bc = batch_cache or cfg.batch
+    shape = (cfg.n_layers, Bc, S, cfg.n_kv_heads, cfg.head_dim)
+    k = torch.full(shape, fill, dtype=torch.bfloat16, device=dev)
+    v = torch.full(shape, fill, dtype=torch.bfloat16, device=dev)
+    x0 = torch_bf16(inp.x0, dev)
+    pos = torch.from_numpy(np.ascontiguousarray(inp.pos)).to(dev)
+    sl = None if slot is None else torch.from_numpy(np.ascontiguousarray(slot, np.int32)).to(dev)
+    dv.build_visual_memory(plan, x0, pos, k, v, slot=sl, slot0=slot0)
+    torch.cuda.synchronize()
+    assert dv.plan_status(plan) == dv.DV_OK
+    return k, v, plan
+
+
+def gather(cache, cfg, tokens, slot=None, slot0=0):
+    """fp64 [n, L, kv] rows of the cache for flat token ids (b * n_vis + i)."""
+    import torch
+    tokens = np.asarray(tokens)
+    b = tokens // cfg.n_vis
+    i = tokens % cfg.n_vis
+    s = slot.reshape(-1)[tokens] if slot is not None else slot0 + i
+    idx_b = torch.as_tensor(b, device=cache.device)
+    idx_s = torch.as_tensor(s, device=cache.device)
+    rows = cache[:, idx_b, idx_s]                       # [L, n, H, D]
+    return rows.permute(1, 0, 2, 3).reshape(len(tokens), cfg.n_layers, -1).double().cpu().numpy()
+
+
+def parity(g, o, head_dim):
+    """(max scaled error, min cosine) of GPU g against oracle o, both [n, L, kv]."""
+    n, L, kv = o.shape
+    oh = o.reshape(n, L, kv // head_dim, head_dim)
+    gh = g.reshape(n, L, kv // head_dim, head_dim)
+    rms = np.sqrt(np.mean(oh * oh, axis=-1, keepdims=True))
+    err = np.abs(gh - oh) / np.maximum(np.abs(oh), rms)
+    cos = np.sum(g * o, axis=-1) / (np.linalg.norm(g, axis=-1) * np.linalg.norm(o, axis=-1))
+    return float(err.max()), float(cos.min())
+
+
+def assert_parity(gk, gv, ok, ov, head_dim, label=""):
+    ek, ck = parity(gk, ok, head_dim)
+    ev, cv = parity(gv, ov, head_dim)
+    msg = f"{label}: K max err {ek:.3e} min cos {ck:.7f}; V max err {ev:.3e} min cos {cv:.7f}"
+    assert np.all(np.isfinite(gk)) and np.all(np.isfinite(gv)), msg
+    assert ek <= REL_TOL and ev <= REL_TOL, msg
+    assert ck >= COS_TOL and cv >= COS_TOL, msg
+    return ek, ev, ck, cv
+
+
+def sample_tokens(T, n=48, seed=0):
+    """Tokens spread over every 128-row tile, always including both ends and tile borders."""
+    rng = np.random.default_rng(seed)
+    fixed = {0, 1, T - 1, T - 2, min(127, T - 1), min(128, T - 1), (T - 1) // 128 * 128}
+    picks = set(int(x) for x in rng.integers(0, T, size=n)) | fixed
+    return np.array(sorted(p for p in picks if 0 <= p < T), dtype=np.int64)
+
+
+def small_config(name, **kw):
+    base = synth.CONFIGS["tiny"]
+    from dataclasses import replace
+    return replace(base, name=name, **kw)

@@ -1,0 +1,84 @@
+"""The C-ABI library without a GPU: it builds for sm_103a, loads, exports every entry point
+declared in include/dv.h, and rejects bad configurations before touching the device."""
+import ctypes
+import os
+import re
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module")
+def dv():
+    from paper_2609_34972_gb300.build import build_library
+    build_library()
+    import paper_2609_34972_gb300 as dv
+    return dv
+
+
+def _declared():
+    src = open(os.path.join(ROOT, "include", "dv.h")).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    return sorted(set(re.findall(r"\b(dv_[a-z_]+)\s*\(", src)))
+
+
+def test_every_declared_symbol_is_exported(dv):
+    names = _declared()
+    assert "dv_memory_plan" in names and "dv_build_visual_memory" in names and "dv_free" in names
+    lib = dv.lib()
+    for n in names:
+        assert hasattr(lib, n), f"{n} declared in dv.h but not exported"
+    assert sorted(dv.EXPORTED) == names
+
+
+def test_error_strings(dv):
+    for code in range(0, 8):
+        assert dv.error_string(code) and dv.error_string(code) != "unknown status"
+    assert dv.error_string(99) == "unknown status"
+
+
+def test_null_arguments_rejected(dv):
+    lib = dv.lib()
+    assert lib.dv_memory_plan(None, None, None, None) == dv.DV_ERR_INVALID_ARG
+    h = ctypes.c_void_p()
+    assert lib.dv_memory_plan(None, None, None, ctypes.byref(h)) == dv.DV_ERR_INVALID_ARG
+    assert lib.dv_build_visual_memory(None, None, 1, 1, None, None, 0, None, None) == dv.DV_ERR_INVALID_ARG
+    assert lib.dv_plan_status(None) == dv.DV_ERR_INVALID_ARG
+    lib.dv_free(None)  # no-op
+
+
+@pytest.mark.parametrize("field,value,code", [
+    ("d", 100, 2), ("d", 0, 1), ("rank", 0, 1), ("rank", 300, 2), ("head_dim", 96, 2),
+    ("n_layers", -1, 1), ("act", 3, 1), ("rope", 5, 1), ("max_batch", 0, 1),
+    ("rope_theta", -1.0, 1), ("rms_eps", -1e-6, 1), ("n_kv_heads", 129, 2),
+])
+def test_bad_config_rejected_before_device(dv, field, value, code):
+    cfg = dv.make_config(512, 4, 8, 64, 16, max_batch=1, max_n_vis=64)
+    setattr(cfg, field, value)
+    w = dv.DvWeights(*([ctypes.c_void_p(256)] * 5 + [None, None]))
+    h = ctypes.c_void_p()
+    assert dv.lib().dv_memory_plan(ctypes.byref(cfg), ctypes.byref(w), None, ctypes.byref(h)) == code
+    assert not h.value
+
+
+def test_mrope_sections_must_cover_half_head(dv):
+    cfg = dv.make_config(512, 4, 8, 128, 16, rope="mrope", mrope_section=(16, 24, 20),
+                         max_batch=1, max_n_vis=64)
+    w = dv.DvWeights(*([ctypes.c_void_p(256)] * 5 + [None, None]))
+    h = ctypes.c_void_p()
+    assert dv.lib().dv_memory_plan(ctypes.byref(cfg), ctypes.byref(w), None, ctypes.byref(h)) == 2
+
+
+def test_missing_weights_rejected(dv):
+    cfg = dv.make_config(512, 4, 8, 64, 16, max_batch=1, max_n_vis=64, has_kv_bias=True)
+    w = dv.DvWeights(*([ctypes.c_void_p(256)] * 5 + [None, None]))   # bias asked for, not given
+    h = ctypes.c_void_p()
+    assert dv.lib().dv_memory_plan(ctypes.byref(cfg), ctypes.byref(w), None, ctypes.byref(h)) == 1
+
+
+def test_binding_fails_loudly_without_library(dv, monkeypatch):
+    monkeypatch.setattr(dv, "_lib", None)
+    monkeypatch.setattr(dv, "LIB_PATH", "/nonexistent/libdv.so")
+    with pytest.raises(RuntimeError):
+        dv.lib()

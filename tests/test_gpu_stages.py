@@ -1,0 +1,55 @@
+"""Stage-wise GPU checks against the oracle: the stacked down-projection with SiLU (H), the
+row sums of squares of E, and the RMS statistic of M_l, read from the build's workspace."""
+import numpy as np
+import pytest
+
+import oracle
+import synth
+from tests import gpu_util as gu
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _cuda():
+    torch = pytest.importorskip("torch")
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    from paper_2609_34972_gb300.build import build_library
+    build_library()
+
+
+CASES = {
+    "tiny": synth.CONFIGS["tiny"],
+    "ragged": gu.small_config("ragged", d=1024, n_layers=3, n_kv_heads=2, n_heads=4,
+                              head_dim=128, rank=80, n_vis=300, batch=2, x0_sigma=0.5, seed=21),
+}
+
+
+@pytest.mark.parametrize("name", sorted(CASES))
+def test_stage_outputs(name):
+    import torch
+    import paper_2609_34972_gb300 as dv
+    cfg = CASES[name]
+    inp = synth.make_inputs(cfg)
+    k, v, plan = gu.run_build(inp)
+    H, rstd, xx, r_pad = dv.debug_workspace(plan, cfg.tokens)
+    torch.cuda.synchronize()
+    ref = oracle.build_tokens(inp, np.arange(cfg.tokens), want=("h", "m"))
+    x = synth.bf16_to_f32(inp.x0).astype(np.float64).reshape(cfg.tokens, cfg.d)
+    # row sums of squares of E: fp32 accumulation of exact squares
+    np.testing.assert_allclose(xx.double().cpu().numpy(), (x * x).sum(1), rtol=1e-5)
+    # H: SiLU(x D_l) rounded to bf16; padded columns are zero
+    Hn = H.double().cpu().numpy().reshape(cfg.tokens, cfg.n_layers, r_pad)
+    h = ref["h"]
+    assert np.all(Hn[:, :, cfg.rank:] == 0.0)
+    scale = np.sqrt(np.mean(h * h))
+    err = np.abs(Hn[:, :, :cfg.rank] - h)
+    assert err.max() <= 2e-2 * max(scale, 1e-30) + 0.0, f"H max err {err.max():.3e} (rms {scale:.3e})"
+    assert np.max(err / np.maximum(np.abs(h), scale)) <= 1e-2
+    # rstd_l = 1 / sqrt(mean(M_l^2) + eps)
+    m = ref["m"]
+    rs_ref = 1.0 / np.sqrt(np.mean(m * m, axis=2) + cfg.rms_eps)     # [T, L]
+    rs = rstd.double().cpu().numpy().T
+    np.testing.assert_allclose(rs, rs_ref, rtol=5e-3)
+    dv.free(plan)

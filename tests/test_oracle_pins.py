@@ -319,3 +319,11 @@ def test_each_batch_element_uses_its_own_positions():
                 kb = out["k"][b, l, h * Dh:(h + 1) * Dh]
                 np.testing.assert_allclose(oracle.rope_head(ka, 40, cfg.rope_theta), kb,
                                            rtol=1e-9, atol=1e-12)
+
+
+def test_layer_subset_matches_full_run():
+    cfg, inp = _random_inputs(n_vis=6)
+    full = oracle.build_tokens(inp)
+    part = oracle.build_tokens(inp, np.array([4, 1]), layers=[3, 0])
+    assert np.array_equal(part["k"][0, 0], full["k"][4, 3]) and np.array_equal(part["k"][1, 1], full["k"][1, 0])
+    assert np.array_equal(part["v"][0, 1], full["v"][4, 0])
