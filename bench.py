@@ -206,6 +206,8 @@ def run_dv(args):
     torch.cuda.set_device(local)
     dev = torch.device("cuda", local)
     cfg = synth.CONFIGS[args.config]
+    if args.layers:
+        cfg = synth.config(args.config, n_layers=args.layers, name=f"{args.config}_L{args.layers}")
     peaks, peak_src = load_peaks()
 
     # ---- inputs (host, seeded) -> device; plan once outside the timing
@@ -342,6 +344,8 @@ def main():
     ap.add_argument("--steps", type=int, default=1000)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--config", default=DEFAULT_WORKLOAD)
+    ap.add_argument("--layers", type=int, default=0,
+                    help="override the layer count (smaller profiling cases of the same shape)")
     ap.add_argument("--impl", choices=["dv", "reference"], default="dv")
     ap.add_argument("--e2e-steps", type=int, default=100)
     ap.add_argument("--no-cpu-baseline", action="store_true")

@@ -8,6 +8,9 @@ separately for K and V.
 """
 from __future__ import annotations
 
+import json
+import os
+
 import numpy as np
 
 import synth
@@ -89,6 +92,11 @@ def assert_parity(gk, gv, ok, ov, head_dim, label=""):
     ek, ck = parity(gk, ok, head_dim)
     ev, cv = parity(gv, ov, head_dim)
     msg = f"{label}: K max err {ek:.3e} min cos {ck:.7f}; V max err {ev:.3e} min cos {cv:.7f}"
+    log = os.environ.get("DV_PARITY_LOG")
+    if log:
+        with open(log, "a") as f:
+            f.write(json.dumps({"case": label, "k_max_err": ek, "k_min_cos": ck, "v_max_err": ev,
+                                "v_min_cos": cv, "n_tokens": int(ok.shape[0])}) + "\n")
     assert np.all(np.isfinite(gk)) and np.all(np.isfinite(gv)), msg
     assert ek <= REL_TOL and ev <= REL_TOL, msg
     assert ck >= COS_TOL and cv >= COS_TOL, msg

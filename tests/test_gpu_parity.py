@@ -84,7 +84,7 @@ def test_slot_mapping_and_untouched_cache():
     inp = synth.make_inputs(cfg)
     rng = np.random.default_rng(5)
     slot = np.stack([rng.permutation(40) + 7, rng.permutation(40) + 3]).astype(np.int32)
-    (_, _, _), (k, v, _) = _full_check(inp, "slots", seq_len=64, batch_cache=3, slot=slot, fill=-7.0)
+    _, (k, v, _) = _full_check(inp, "slots", seq_len=64, batch_cache=3, slot=slot, fill=-7.0)
     written = torch.zeros(k.shape[1], k.shape[2], dtype=torch.bool)
     for b in range(2):
         written[b, torch.as_tensor(slot[b].astype(np.int64))] = True
