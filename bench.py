@@ -31,8 +31,8 @@ METRIC = "visual tokens/sec of layer-wise visual KV-memory build; % of BF16 tens
 UNIT = "visual tokens/s"
 DEFAULT_WORKLOAD = "llava15_7b"
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
-GEMM_SOURCES = ["paper_2609_34972_gb300/csrc/dv_gemm.cu", "paper_2609_34972_gb300/csrc/dv_ptx.cuh",
-                "paper_2609_34972_gb300/csrc/dv_internal.h"]
+GEMM_SOURCES = ["paper_2609_34972_gb300/csrc/dv_kv2sm.cu", "paper_2609_34972_gb300/csrc/dv_ptx.cuh",
+                "paper_2609_34972_gb300/csrc/dv_epilogue.cuh", "paper_2609_34972_gb300/csrc/dv_internal.h"]
 
 
 def load_peaks():
@@ -207,7 +207,8 @@ def run_dv(args):
     dev = torch.device("cuda", local)
     cfg = synth.CONFIGS[args.config]
     if args.layers:
-        cfg = synth.config(args.config, n_layers=args.layers, name=f"{args.config}_L{args.layers}")
+        from dataclasses import replace
+        cfg = replace(cfg, n_layers=args.layers, name=f"{args.config}_L{args.layers}")
     peaks, peak_src = load_peaks()
 
     # ---- inputs (host, seeded) -> device; plan once outside the timing
@@ -322,7 +323,7 @@ def run_dv(args):
             "gpu_launches": args.steps * dv.kernels_per_build(plan),
             "roofline": {"bound": "tensor", "achieved": achieved_tf, "peak": peak_tf,
                          "unit": "TFLOP/s", "frac": achieved_tf / peak_tf, "traffic": traffic,
-                         "kernel": "dv_gemm_kernel<EPI_KV> (K/V projection + RoPE + cache store)",
+                         "kernel": "dv_kv_pair_kernel (K/V projection + RoPE + cache store, 2-SM UMMA)",
                          "peak_source": f"bf16_tflops (burst) of {peak_src}",
                          "flops_per_launch": kv_flops, "ms_per_launch": kv_ms},
             "roofline_step": {"t_roof_ms": t_roof_ms, "frac": t_roof_ms / ms_step,

@@ -43,7 +43,8 @@ enum { DV_ROPE_1D = 0, DV_ROPE_MROPE = 1 };
 
 /* Model shape and build limits. Supported (else DV_ERR_UNSUPPORTED_SHAPE):
  *   d % 64 == 0, 64 <= d <= 16384;  1 <= rank <= 256;  head_dim in {64, 128};
- *   1 <= n_kv_heads, n_kv_heads * head_dim <= 8192;  1 <= n_layers <= 256;
+ *   1 <= n_kv_heads, n_kv_heads * head_dim <= 8192 and a multiple of 128;
+ *   1 <= n_layers <= 256;
  *   act == DV_ACT_SILU;  rope_theta > 0;  rms_eps >= 0;
  *   DV_ROPE_MROPE: mrope_section[i] >= 0 and their sum == head_dim / 2 (contiguous sections
  *   of the frequency index: t first, then h, then w);

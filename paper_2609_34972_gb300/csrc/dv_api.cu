@@ -4,7 +4,8 @@
 // Plan-time repacking (once per weight set). With r_pad = r rounded up to 64:
 //   Dst  [L*r_pad][d]         stacked down-projections, zero rows past r
 //   Bn   [L*r_pad][d+r_pad]   row n of layer l: [2 U_l[n,:] | G_l[n,:]], G_l = U_l U_l^T
-//   Wkv  [L*2kv][d+r_pad]     per layer, per head h: 128 (or 64) K rows then V rows, each
+//   Wkv  [L*2kv][d+r_pad]     per layer, per group of 128 channels: the 128 K rows, then the
+//                             128 V rows of the same channels, each
 //                             [W[c,:] * gamma_l | (W diag(gamma_l) U_l^T)[c,:]]
 // so that, with A_l = [x0 | h_l] (h_l = SiLU(x0 D_l), Sec. 3.1 Eq. 4):
 //   A_l Bn_l^T   = 2 x0 U_l^T + h_l G_l        -> ||M_l||^2 = ||x0||^2 + h_l . (that)
@@ -127,19 +128,25 @@ __global__ void k_pack_norm_u(const uint16_t* __restrict__ U, uint16_t* __restri
   }
 }
 
-// Wkv rows: per layer, per head h, HD rows of K then HD rows of V; columns [0, d) hold
+// Row rl of layer l in Wkv: group rl / 256 of 128 channels, K (first 128) or V (next 128).
+__device__ __forceinline__ void wkv_row(int rl, int& part, int& c) {
+  part = (rl >> 7) & 1;
+  c = (rl >> 8) * 128 + (rl & 127);
+}
+
+// Wkv rows: per layer, per 128-channel group, 128 K rows then 128 V rows; columns [0, d) hold
 // W[c][j] * gamma[l][j]; columns [d, k_total) are filled by k_rank_product (zero past r).
 __global__ void k_pack_kv(const uint16_t* __restrict__ Wk, const uint16_t* __restrict__ Wv,
                           const uint16_t* __restrict__ gamma, uint16_t* __restrict__ Wkv, int L,
-                          int kv, int HD, int d, int k_total) {
+                          int kv, int d, int k_total) {
   const long long total = static_cast<long long>(L) * 2 * kv * k_total;
   for (long long e = blockIdx.x * static_cast<long long>(blockDim.x) + threadIdx.x; e < total;
        e += static_cast<long long>(gridDim.x) * blockDim.x) {
     const int j = static_cast<int>(e % k_total);
     const long long row = e / k_total;
     const int rl = static_cast<int>(row % (2 * kv)), l = static_cast<int>(row / (2 * kv));
-    const int h = rl / (2 * HD), part = (rl / HD) & 1, jj = rl % HD;
-    const int c = h * HD + jj;
+    int part, c;
+    wkv_row(rl, part, c);
     float v = 0.0f;
     if (j < d) {
       const uint16_t* W = part ? Wv : Wk;
@@ -161,8 +168,7 @@ __global__ void __launch_bounds__(256) k_rank_product(const uint16_t* __restrict
                                                       const uint16_t* __restrict__ gamma,
                                                       const uint16_t* __restrict__ U,
                                                       uint16_t* __restrict__ out, int rows, int r,
-                                                      int d, int kv, int HD, int r_pad,
-                                                      int k_total) {
+                                                      int d, int kv, int r_pad, int k_total) {
   __shared__ float As[32][65];
   __shared__ float Us[32][65];
   const int l = blockIdx.z;
@@ -177,7 +183,8 @@ __global__ void __launch_bounds__(256) k_rank_product(const uint16_t* __restrict
       float a = 0.0f;
       if (i < rows && j < d) {
         if (MODE == 0) {
-          const int h = i / (2 * HD), part = (i / HD) & 1, c = h * HD + i % HD;
+          int part, c;
+          wkv_row(i, part, c);
           const uint16_t* W = part ? Wv : Wk;
           a = bf(W[(static_cast<long long>(l) * kv + c) * d + j]) *
               bf(gamma[static_cast<long long>(l) * d + j]);
@@ -286,6 +293,7 @@ int check_config(const dv_config* c) {
   if (c->rank > 256) return DV_ERR_UNSUPPORTED_SHAPE;
   if (c->head_dim != 64 && c->head_dim != 128) return DV_ERR_UNSUPPORTED_SHAPE;
   if (static_cast<long long>(c->n_kv_heads) * c->head_dim > 8192) return DV_ERR_UNSUPPORTED_SHAPE;
+  if ((c->n_kv_heads * c->head_dim) % 128 != 0) return DV_ERR_UNSUPPORTED_SHAPE;
   if (c->n_layers > 256) return DV_ERR_UNSUPPORTED_SHAPE;
   if (static_cast<long long>(c->max_batch) * c->max_n_vis > (1LL << 24)) return DV_ERR_UNSUPPORTED_SHAPE;
   if (c->rope == DV_ROPE_MROPE) {
@@ -392,13 +400,13 @@ int dv_memory_plan(const dv_config* cfg, const dv_weights* w, void* stream, dv_p
   k_pack_norm_u<<<grid_for(1LL * L * p->r_pad * p->k_total), 256, 0, st>>>(U, p->Bn, L, r, p->r_pad,
                                                                            d, p->k_total);
   k_pack_kv<<<grid_for(1LL * L * 2 * p->kv * p->k_total), 256, 0, st>>>(Wk, Wv, G, p->Wkv, L, p->kv,
-                                                                        HD, d, p->k_total);
+                                                                        d, p->k_total);
   {
     dim3 g1((r + 63) / 64, (r + 63) / 64, L);
-    k_rank_product<1><<<g1, 256, 0, st>>>(Wk, Wv, G, U, p->Bn, r, r, d, p->kv, HD, p->r_pad,
+    k_rank_product<1><<<g1, 256, 0, st>>>(Wk, Wv, G, U, p->Bn, r, r, d, p->kv, p->r_pad,
                                           p->k_total);
     dim3 g0((r + 63) / 64, (2 * p->kv + 63) / 64, L);
-    k_rank_product<0><<<g0, 256, 0, st>>>(Wk, Wv, G, U, p->Wkv, 2 * p->kv, r, d, p->kv, HD,
+    k_rank_product<0><<<g0, 256, 0, st>>>(Wk, Wv, G, U, p->Wkv, 2 * p->kv, r, d, p->kv,
                                           p->r_pad, p->k_total);
   }
   if (cfg->has_kv_bias) {
@@ -417,7 +425,7 @@ int dv_memory_plan(const dv_config* cfg, const dv_weights* w, void* stream, dv_p
              encode_2d(&p->tm_Dst[1], p->Dst, d, 1ull * L * p->r_pad, d, 128) &&
              encode_2d(&p->tm_Dst[2], p->Dst, d, 1ull * L * p->r_pad, d, 256) &&
              encode_2d(&p->tm_Bn, p->Bn, p->k_total, 1ull * L * p->r_pad, p->k_total, p->r_pad) &&
-             encode_2d(&p->tm_Wkv, p->Wkv, p->k_total, 1ull * L * 2 * p->kv, p->k_total, 2 * HD) &&
+             encode_2d(&p->tm_Wkv, p->Wkv, p->k_total, 1ull * L * 2 * p->kv, p->k_total, 128) &&
              encode_2d(&p->tm_H, p->H, 1ull * L * p->r_pad, T, 1ull * L * p->r_pad, dv::kBlockM);
   if (!enc) {
     free_plan_memory(p);
@@ -496,7 +504,14 @@ int dv_build_visual_memory(dv_plan* p, const void* x0, int batch, int n_vis, con
     err = dv::launch_gemm(dv::EPI_NORM, p->r_pad, 0, tm_x0, p->tm_H, p->tm_Bn, gp, p->num_sms, st);
   mark(3);
 
-  // (3) K/V = rstd_l * ([x0 | h_l] Wkv_l^T) + b, RoPE on K, stored into the cache.
+  // (3) K/V = rstd_l * (Wkv_l [x0 | h_l]^T) + b, RoPE on K, stored into the cache, on CTA pairs
+  //     with the weights as the M operand and NT-token blocks as the N operand.
+  const int nt = dv::kv_pair_tile_n(T);
+  CUtensorMap tm_x0_half, tm_H_half;
+  if (err == cudaSuccess &&
+      !(encode_2d(&tm_x0_half, x0, d, static_cast<uint64_t>(T), d, nt / 2) &&
+        encode_2d(&tm_H_half, p->H, 1ull * L * p->r_pad, p->max_tokens, 1ull * L * p->r_pad, nt / 2)))
+    err = cudaErrorInvalidValue;
   gp.s = {static_cast<int>(T), L, 2 * p->kv, d / 64, p->r_pad / 64, p->r_pad};
   dv::EpiKV& e = gp.kv;
   e.rstd = p->rstd;
@@ -526,7 +541,7 @@ int dv_build_visual_memory(dv_plan* p, const void* x0, int batch, int n_vis, con
     e.inv_freq_lo[j] = static_cast<float>(p->inv_freq[j] - static_cast<double>(e.inv_freq_hi[j]));
   }
   if (err == cudaSuccess)
-    err = dv::launch_gemm(dv::EPI_KV, 2 * HD, HD, tm_x0, p->tm_H, p->tm_Wkv, gp, p->num_sms, st);
+    err = dv::launch_kv_pair(HD, nt, p->tm_Wkv, tm_x0_half, tm_H_half, gp, p->num_sms, st);
   mark(4);
   return err == cudaSuccess ? DV_OK : DV_ERR_CUDA;
 }

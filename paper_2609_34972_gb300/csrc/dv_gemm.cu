@@ -1,12 +1,11 @@
-// Persistent, warp-specialised tcgen05 GEMM for the three contractions of the visual-memory
-// build, each with its own fused epilogue:
+// Persistent, warp-specialised 1-SM tcgen05 GEMM for the two rank-r contractions of the
+// visual-memory build, each with its own fused epilogue (the K/V contraction runs on CTA pairs,
+// dv_kv2sm.cu):
 //   EPI_SILU  H   = SiLU(x0 [D_1 ... D_L])          all L down-projections as one GEMM, since
 //                                                    every layer reads only E (Sec. 3.1 Eq. 5)
 //   EPI_NORM  rstd_l = (||M_l||^2 / d + eps)^-1/2    the RMS statistic of M_l = x0 + h_l U_l
 //                                                    (Sec. 3.1 Eq. 4), from [x0 | h_l] times
 //                                                    [2 U_l^T ; U_l U_l^T]
-//   EPI_KV    K_l, V_l = rstd_l * ([x0 | h_l] W~_l) (+ b), RoPE on K, bf16 cache store
-//                                                    (Sec. 3.2 Eq. 7)
 //
 // CTA layout (192 threads, one CTA per SM):
 //   warp 0      TMA producer: one lane streams 64-wide K slabs of A (128 token rows) and B
@@ -19,6 +18,7 @@
 // same time share weight tiles through L2.
 #include <cstdio>
 
+#include "dv_epilogue.cuh"
 #include "dv_internal.h"
 #include "dv_ptx.cuh"
 
@@ -46,14 +46,6 @@ struct TileCfg {
 __device__ __forceinline__ bool wait_drain(uint32_t bar, uint32_t parity, uint64_t timeout_ns) {
   int never = 0;
   return mbar_wait(bar, parity, &never, timeout_ns);
-}
-
-__device__ __forceinline__ void store_row32(uint16_t* dst, const uint32_t (&pk)[16]) {
-  uint4* d = reinterpret_cast<uint4*>(dst);
-  d[0] = make_uint4(pk[0], pk[1], pk[2], pk[3]);
-  d[1] = make_uint4(pk[4], pk[5], pk[6], pk[7]);
-  d[2] = make_uint4(pk[8], pk[9], pk[10], pk[11]);
-  d[3] = make_uint4(pk[12], pk[13], pk[14], pk[15]);
 }
 
 // ------------------------------------------------------------------------------ epilogues
@@ -112,94 +104,6 @@ __device__ __forceinline__ void epi_norm(const GemmParams& p, uint32_t tbase, in
     const float ss = fmaxf(p.norm.xx[t] + dot, 0.0f);
     p.norm.rstd[static_cast<size_t>(l) * p.norm.ld_rstd + t] =
         rsqrtf(fmaf(ss, p.norm.inv_d, p.norm.eps));
-  }
-}
-
-// Angle p * theta^(-2j/D_h) reduced to [-pi, pi] before the sine/cosine: the product is kept
-// as an unevaluated sum of two floats (fma residual), then reduced by Cody-Waite subtraction of
-// k * 2pi with 2pi split into two floats.
-__device__ __forceinline__ void rope_sincos(float pos, float fhi, float flo, const EpiKV& kv,
-                                            float& s, float& c) {
-  const float a_hi = pos * fhi;
-  const float a_lo = fmaf(pos, flo, fmaf(pos, fhi, -a_hi));
-  const float k = rintf(a_hi * kv.inv_two_pi);
-  float r = fmaf(-k, kv.two_pi_hi, a_hi);
-  r = fmaf(-k, kv.two_pi_lo, r) + a_lo;
-  __sincosf(r, &s, &c);
-}
-
-// K/V tile of one head: columns [0, HD) are K head h, [HD, 2HD) are V head h (plan packing).
-// k = rstd * acc + b_K, rotated in rotate-half pairs (j, j + HD/2); v = rstd * acc + b_V.
-template <int HD>
-__device__ __forceinline__ void epi_kv(const GemmParams& p, uint32_t tbase, int l, int h, int t) {
-  constexpr int kHalf = HD / 2;
-  const EpiKV& e = p.kv;
-  const bool valid = t < p.s.M;
-  const int tt = valid ? t : 0;
-  const int b = tt / e.n_vis, i = tt - b * e.n_vis;
-  const float rs = valid ? e.rstd[static_cast<size_t>(l) * e.ld_rstd + tt] : 0.0f;
-  const int slot = e.slot ? e.slot[tt] : e.slot0 + i;
-  const long long off = l * e.s_layer + b * e.s_batch + slot * e.s_seq + h * e.s_head;
-  uint16_t* krow = e.kc + off;
-  uint16_t* vrow = e.vc + off;
-  const int* pp = e.pos + static_cast<size_t>(b) * e.n_pos * e.n_vis + i;
-  const float pt = static_cast<float>(pp[0]);
-  const float ph = e.n_pos == 3 ? static_cast<float>(pp[e.n_vis]) : pt;
-  const float pw = e.n_pos == 3 ? static_cast<float>(pp[2 * e.n_vis]) : pt;
-  const float* bk = e.bk ? e.bk + static_cast<size_t>(l) * e.kv + h * HD : nullptr;
-  const float* bv = e.bv ? e.bv + static_cast<size_t>(l) * e.kv + h * HD : nullptr;
-
-#pragma unroll 1
-  for (int jb = 0; jb < kHalf / 32; ++jb) {
-    uint32_t lo[32], hi[32];
-    __syncwarp();
-    tmem_ld32(tbase + jb * 32, lo);
-    tmem_ld32(tbase + kHalf + jb * 32, hi);
-    tmem_ld_wait();
-    uint32_t plo[16], phi[16];
-#pragma unroll
-    for (int u = 0; u < 32; u += 2) {
-      float y1[2], y2[2];
-#pragma unroll
-      for (int w = 0; w < 2; ++w) {
-        const int j = jb * 32 + u + w;
-        float x1 = __uint_as_float(lo[u + w]) * rs;
-        float x2 = __uint_as_float(hi[u + w]) * rs;
-        if (bk) {
-          x1 += bk[j];
-          x2 += bk[kHalf + j];
-        }
-        const float pj = j < e.sec0 ? pt : (j < e.sec01 ? ph : pw);
-        float s, c;
-        rope_sincos(pj, e.inv_freq_hi[j], e.inv_freq_lo[j], e, s, c);
-        y1[w] = x1 * c - x2 * s;
-        y2[w] = x2 * c + x1 * s;
-      }
-      plo[u / 2] = pack_bf16x2(y1[0], y1[1]);
-      phi[u / 2] = pack_bf16x2(y2[0], y2[1]);
-    }
-    if (valid) {
-      store_row32(krow + jb * 32, plo);
-      store_row32(krow + kHalf + jb * 32, phi);
-    }
-  }
-#pragma unroll 1
-  for (int jb = 0; jb < HD / 32; ++jb) {
-    uint32_t r[32];
-    __syncwarp();
-    tmem_ld32(tbase + HD + jb * 32, r);
-    tmem_ld_wait();
-    uint32_t pk[16];
-#pragma unroll
-    for (int u = 0; u < 16; ++u) {
-      float v0 = __uint_as_float(r[2 * u]) * rs, v1 = __uint_as_float(r[2 * u + 1]) * rs;
-      if (bv) {
-        v0 += bv[jb * 32 + 2 * u];
-        v1 += bv[jb * 32 + 2 * u + 1];
-      }
-      pk[u] = pack_bf16x2(v0, v1);
-    }
-    if (valid) store_row32(vrow + jb * 32, pk);
   }
 }
 
@@ -358,10 +262,8 @@ __global__ void __launch_bounds__(kNumThreads, 1)
       const int t = m * kBlockM + row;
       if constexpr (EPI == EPI_SILU) {
         epi_silu<BN>(p, tbase, n, t);
-      } else if constexpr (EPI == EPI_NORM) {
-        epi_norm<BN>(p, tbase, l, t);
       } else {
-        epi_kv<HD>(p, tbase, l, n, t);
+        epi_norm<BN>(p, tbase, l, t);
       }
       tc_fence_before();
       mbar_arrive(tempty_bar(acc));
@@ -419,9 +321,6 @@ cudaError_t launch_gemm(int epi, int block_n, int head_dim, const CUtensorMap& a
     if (block_n == 64) return launch_t<EPI_NORM, 64, 0>(a0, a1, b, p, num_sms, stream);
     if (block_n == 128) return launch_t<EPI_NORM, 128, 0>(a0, a1, b, p, num_sms, stream);
     if (block_n == 256) return launch_t<EPI_NORM, 256, 0>(a0, a1, b, p, num_sms, stream);
-  } else if (epi == EPI_KV) {
-    if (head_dim == 64 && block_n == 128) return launch_t<EPI_KV, 128, 64>(a0, a1, b, p, num_sms, stream);
-    if (head_dim == 128 && block_n == 256) return launch_t<EPI_KV, 256, 128>(a0, a1, b, p, num_sms, stream);
   }
   return cudaErrorInvalidValue;
 }

@@ -14,7 +14,6 @@ constexpr int kMaxHalfHead = 64;     // head_dim <= 128
 enum Epilogue : int {
   EPI_SILU = 0,  // stacked down-projection: H = bf16(SiLU(acc))
   EPI_NORM = 1,  // RMS statistic: rstd = (||x0||^2 + h . acc) / d + eps) ^ -1/2
-  EPI_KV = 2,    // K/V: rstd * acc + bias, RoPE on K, bf16 store into the cache
 };
 
 // Operand schedule shared by all three GEMMs. The A operand of a tile is the 128-row token
@@ -76,13 +75,23 @@ struct GemmParams {
   unsigned long long timeout_ns;
 };
 
-// Launches one persistent warp-specialised tcgen05 GEMM. Returns a cudaError_t value.
-// block_n: 64/128/256 for EPI_SILU and EPI_NORM; 2*head_dim (128 or 256) for EPI_KV.
+// Launches one persistent warp-specialised 1-SM tcgen05 GEMM (EPI_SILU or EPI_NORM,
+// block_n 64/128/256). Returns a cudaError_t value.
 cudaError_t launch_gemm(int epi, int block_n, int head_dim, const CUtensorMap& a0,
                         const CUtensorMap& a1, const CUtensorMap& b, const GemmParams& p,
                         int num_sms, cudaStream_t stream);
 
 // Shared-memory bytes one CTA of that GEMM asks for (for validation and reporting).
 int gemm_smem_bytes(int block_n);
+
+// K/V projection + RoPE + cache store on CTA pairs (2-SM UMMA). w: Wkv with 128-row boxes;
+// x / h: x0 and H with boxes of nt/2 token rows. nt from kv_pair_tile_n.
+cudaError_t launch_kv_pair(int head_dim, int nt, const CUtensorMap& w, const CUtensorMap& x,
+                           const CUtensorMap& h, const GemmParams& p, int num_sms,
+                           cudaStream_t stream);
+
+// Token tile (64, 128, 192 or 256) of the pair kernel for a build of `tokens` tokens.
+int kv_pair_tile_n(long long tokens);
+int kv_pair_smem_bytes(int nt);
 
 }  // namespace dv

@@ -1,0 +1,410 @@
+// K/V projection, RoPE and KV-cache store (Sec. 3.2 Eq. 7) as a 2-SM tcgen05 GEMM.
+//
+//   [K_l | V_l]^T = Wkv_l [x0 | h_l]^T,  then rstd_l * (.) + b, RoPE on K, bf16 into the cache
+//
+// The weights are the M operand and the tokens the N operand ("swap AB"), so the token count
+// only has to be a multiple of the N tile (64..256 in steps of 64), not of 128 or 256 rows.
+// One CTA pair (cluster of 2) computes a 256 x NT tile: 256 weight rows = the 128 K channels
+// of a 128-channel group (leader CTA, TMEM lanes 0..127) and the same 128 V channels (peer
+// CTA), times NT tokens. Each CTA stages only its own half of both operands (128 weight rows,
+// NT/2 token rows), which halves the shared-memory traffic per MMA against a 1-SM tile.
+//
+// CTA roles (192 threads, one CTA per SM, both CTAs of a pair alike):
+//   warp 0      TMA producer for this CTA's halves; completion is counted on the leader's
+//               full barrier (cta_group::2 TMA), whose single expect_tx arrival (leader)
+//               announces the bytes of both CTAs
+//   warp 1      TMEM owner (cta_group::2 alloc in both CTAs); in the leader one lane issues the
+//               256 x NT x 16 MMAs and multicasts its commits to both CTAs
+//   warps 2-5   epilogue over this CTA's 128 channels: TMEM -> registers -> shared staging
+//               [32 tokens][128 channels] -> per-token rows with RoPE (K) -> 16-byte stores
+// Pair tiles run in (layer, group, token block) order, token block fastest, so the pairs
+// running together share each weight tile through L2.
+#include "dv_epilogue.cuh"
+#include "dv_internal.h"
+#include "dv_ptx.cuh"
+
+namespace dv {
+
+constexpr int kPairThreads = 192;
+constexpr int kEpiPairThreads = 128;
+constexpr int kSmemLimit = 232448;  // largest dynamic shared memory of one CTA on sm_103
+constexpr int kStagePitch = 132;    // floats per staged token row: 128 channels + 4 pad
+
+template <int NT>
+struct PairCfg {
+  static constexpr int kHalfN = NT / 2;
+  static constexpr int kABytes = 128 * kBlockK * 2;
+  static constexpr int kBBytes = kHalfN * kBlockK * 2;
+  static constexpr int kStageBytes = kABytes + kBBytes;
+  static constexpr int kStagingBytes = 32 * kStagePitch * 4;
+  static constexpr int kRingBudget = kSmemLimit - kStagingBytes - 1024 - 512;
+  static constexpr int kStagesRaw = kRingBudget / kStageBytes;
+  static constexpr int kStages = kStagesRaw > 8 ? 8 : kStagesRaw;
+  static constexpr int kSmemBytes = kStages * kStageBytes + kStagingBytes + 1024 + 512;
+  static constexpr int kTmemCols = 512;
+  static_assert(NT % 64 == 0 && NT >= 64 && NT <= 256, "N tile");
+  static_assert(kStageBytes % 1024 == 0, "stage tiles must stay 1024-byte aligned");
+  static_assert(2 * NT <= kTmemCols, "two accumulators must fit in TMEM");
+  static_assert(kSmemBytes <= kSmemLimit, "shared memory");
+};
+
+__device__ __forceinline__ bool wait_local_only(uint32_t bar, uint32_t parity, uint64_t timeout_ns) {
+  int never = 0;
+  return mbar_wait(bar, parity, &never, timeout_ns);
+}
+
+// Phase 2 of the epilogue for one staged chunk of 32 tokens: thread (token, sub) writes its
+// part of the token's K (leader) or V (peer) rows for this 128-channel group.
+template <int HD>
+__device__ __forceinline__ void kv_rows_from_staging(const GemmParams& p, const float* staging,
+                                                     int rank, int l, int g, int tok, int tloc,
+                                                     int sub) {
+  const EpiKV& e = p.kv;
+  if (tok >= p.s.M) return;
+  const int b = tok / e.n_vis, i = tok - b * e.n_vis;
+  const float rs = e.rstd[static_cast<size_t>(l) * e.ld_rstd + tok];
+  const int slot = e.slot ? e.slot[tok] : e.slot0 + i;
+  const long long row0 = l * e.s_layer + b * e.s_batch + slot * e.s_seq;
+  const float* src = staging + tloc * kStagePitch;
+  constexpr int kHeadsPerGroup = 128 / HD;
+  if (rank == 0) {
+    // K: 16 rotate-half pairs (j, j + HD/2) of one head.
+    constexpr int kHalf = HD / 2;
+    const int pair0 = sub * 16;
+    const int hl = pair0 / kHalf, j0 = pair0 % kHalf;
+    const int c1 = hl * HD + j0;
+    const int* pp = e.pos + static_cast<size_t>(b) * e.n_pos * e.n_vis + i;
+    const float pt = static_cast<float>(pp[0]);
+    const float ph = e.n_pos == 3 ? static_cast<float>(pp[e.n_vis]) : pt;
+    const float pw = e.n_pos == 3 ? static_cast<float>(pp[2 * e.n_vis]) : pt;
+    const float* bk = e.bk ? e.bk + static_cast<size_t>(l) * e.kv + g * 128 : nullptr;
+    uint32_t plo[8], phi[8];
+#pragma unroll
+    for (int m = 0; m < 16; m += 2) {
+      float y1[2], y2[2];
+#pragma unroll
+      for (int w = 0; w < 2; ++w) {
+        const int j = j0 + m + w;
+        float x1 = src[c1 + m + w] * rs;
+        float x2 = src[c1 + kHalf + m + w] * rs;
+        if (bk) {
+          x1 += bk[c1 + m + w];
+          x2 += bk[c1 + kHalf + m + w];
+        }
+        const float pj = j < e.sec0 ? pt : (j < e.sec01 ? ph : pw);
+        float s, c;
+        rope_sincos(pj, e.inv_freq_hi[j], e.inv_freq_lo[j], e, s, c);
+        y1[w] = x1 * c - x2 * s;
+        y2[w] = x2 * c + x1 * s;
+      }
+      plo[m / 2] = pack_bf16x2(y1[0], y1[1]);
+      phi[m / 2] = pack_bf16x2(y2[0], y2[1]);
+    }
+    uint16_t* krow = e.kc + row0 + static_cast<long long>(g * kHeadsPerGroup + hl) * e.s_head;
+    store_row16(krow + j0, plo);
+    store_row16(krow + kHalf + j0, phi);
+  } else {
+    // V: 32 consecutive channels of one head, no rotation.
+    const int c0 = sub * 32;
+    const int hl = c0 / HD, jv = c0 % HD;
+    const float* bv = e.bv ? e.bv + static_cast<size_t>(l) * e.kv + g * 128 : nullptr;
+    uint32_t pk[16];
+#pragma unroll
+    for (int m = 0; m < 32; m += 2) {
+      float v0 = src[c0 + m] * rs, v1 = src[c0 + m + 1] * rs;
+      if (bv) {
+        v0 += bv[c0 + m];
+        v1 += bv[c0 + m + 1];
+      }
+      pk[m / 2] = pack_bf16x2(v0, v1);
+    }
+    uint16_t* vrow = e.vc + row0 + static_cast<long long>(g * kHeadsPerGroup + hl) * e.s_head;
+    store_row32(vrow + jv, pk);
+  }
+}
+
+template <int HD, int NT>
+__global__ void __launch_bounds__(kPairThreads, 1)
+    dv_kv_pair_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ CUtensorMap tmX,
+                      const __grid_constant__ CUtensorMap tmH, const __grid_constant__ GemmParams p) {
+  using C = PairCfg<NT>;
+  constexpr int S = C::kStages;
+  extern __shared__ uint8_t smem_raw[];
+  const uint32_t raw = smem_addr(smem_raw);
+  const uint32_t ring = (raw + 1023u) & ~1023u;
+  uint8_t* ring_ptr = smem_raw + (ring - raw);
+  float* staging = reinterpret_cast<float*>(ring_ptr + S * C::kStageBytes);
+  uint64_t* bars = reinterpret_cast<uint64_t*>(ring_ptr + S * C::kStageBytes + C::kStagingBytes);
+  const uint32_t bar0 = smem_addr(bars);
+  auto full_bar = [&](int s) { return bar0 + 8u * s; };            // used in the leader
+  auto empty_bar = [&](int s) { return bar0 + 8u * (S + s); };     // both CTAs
+  auto tfull_bar = [&](int a) { return bar0 + 8u * (2 * S + a); };  // both CTAs
+  auto tempty_bar = [&](int a) { return bar0 + 8u * (2 * S + 2 + a); };  // leader
+  const uint32_t drain_bar = bar0 + 8u * (2 * S + 4);
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 2 * S + 5);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const uint32_t rank = cluster_ctarank();
+  const uint64_t tmo = p.timeout_ns;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < S; ++s) {
+      mbar_init(full_bar(s), 1);     // the leader's expect_tx covers the bytes of both CTAs
+      mbar_init(empty_bar(s), 1);
+    }
+    for (int a = 0; a < 2; ++a) {
+      mbar_init(tfull_bar(a), 1);
+      mbar_init(tempty_bar(a), 2 * kEpiPairThreads / 32);  // one lane per epilogue warp
+    }
+    mbar_init(drain_bar, 1);
+    *abort_flag = 0;
+    fence_barrier_init();
+  }
+  if (warp == 0 && lane == 0) {
+    tma_prefetch_desc(&tmW);
+    tma_prefetch_desc(&tmX);
+    if (p.s.k1_slabs > 0) tma_prefetch_desc(&tmH);
+  }
+  if (warp == 1) {
+    tmem_alloc_pair(smem_addr(tmem_slot), C::kTmemCols);
+    tmem_relinquish_pair();
+  }
+  tc_fence_before();
+  cluster_sync();  // barriers of both CTAs initialised, TMEM allocated in both
+  tc_fence_after();
+  const uint32_t tmem_base = *tmem_slot;
+
+  const int tok_tiles = (p.s.M + NT - 1) / NT;
+  const int groups = p.kv.kv / 128;
+  const int num_tiles = tok_tiles * groups * p.s.n_layers;
+  const int k_slabs = p.s.k0_slabs + p.s.k1_slabs;
+  const int pair = static_cast<int>(cluster_id_x());
+  const int num_pairs = static_cast<int>(num_clusters_x());
+
+  if (warp == 0) {
+    if (lane == 0) {
+      // ---------------------------------------------------------------- TMA producer
+      const uint32_t leader_full0 = map_to_rank(full_bar(0), 0);
+      int stage = 0;
+      uint32_t phase = 0;
+      for (int tile = pair; tile < num_tiles && !*abort_flag; tile += num_pairs) {
+        const int nt = tile % tok_tiles;
+        const int rest = tile / tok_tiles;
+        const int g = rest % groups;
+        const int l = rest / groups;
+        const int wrow = l * p.s.n_per_layer + g * 256 + static_cast<int>(rank) * 128;
+        const int trow = nt * NT + static_cast<int>(rank) * C::kHalfN;
+        for (int ks = 0; ks < k_slabs; ++ks) {
+          if (!mbar_wait(empty_bar(stage), phase ^ 1u, abort_flag, tmo)) break;
+          const uint32_t a_dst = ring + stage * C::kStageBytes;
+          const uint32_t b_dst = a_dst + C::kABytes;
+          const uint32_t fb = leader_full0 + 8u * stage;
+          // Only the leader arrives (local, CTA scope) and announces both CTAs' bytes; the
+          // peer's copies may complete on the barrier first (the transaction count is signed).
+          if (rank == 0) mbar_arrive_expect_tx(full_bar(stage), 2 * C::kStageBytes);
+          tma_load_2d_pair(a_dst, &tmW, fb, ks * kBlockK, wrow);
+          if (ks < p.s.k0_slabs) {
+            tma_load_2d_pair(b_dst, &tmX, fb, ks * kBlockK, trow);
+          } else {
+            tma_load_2d_pair(b_dst, &tmH, fb,
+                             l * p.s.a1_cols_per_layer + (ks - p.s.k0_slabs) * kBlockK, trow);
+          }
+          if (++stage == S) {
+            stage = 0;
+            phase ^= 1u;
+          }
+        }
+      }
+    }
+  } else if (warp == 1) {
+    if (lane == 0 && rank == 0) {
+      // ---------------------------------------------------------------- MMA issuer (leader)
+      const uint32_t idesc = idesc_bf16_f32(256, NT);
+      int stage = 0, acc = 0;
+      uint32_t phase = 0, acc_phase = 0;
+      bool issued_any = false;
+      for (int tile = pair; tile < num_tiles && !*abort_flag; tile += num_pairs) {
+        if (!mbar_wait(tempty_bar(acc), acc_phase ^ 1u, abort_flag, tmo)) break;
+        tc_fence_after();
+        const uint32_t d_tmem = tmem_base + static_cast<uint32_t>(acc * NT);
+        bool ok = true;
+        for (int ks = 0; ks < k_slabs; ++ks) {
+          if (!mbar_wait(full_bar(stage), phase, abort_flag, tmo)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t a_s = ring + stage * C::kStageBytes;
+          const uint32_t b_s = a_s + C::kABytes;
+#pragma unroll
+          for (int k = 0; k < kBlockK / 16; ++k) {
+            umma_bf16_pair(d_tmem, sdesc_kmajor_sw128(a_s + 32u * k),
+                           sdesc_kmajor_sw128(b_s + 32u * k), idesc, (ks | k) != 0 ? 1u : 0u);
+          }
+          issued_any = true;
+          umma_commit_pair(empty_bar(stage), 0x3);
+          if (++stage == S) {
+            stage = 0;
+            phase ^= 1u;
+          }
+        }
+        if (!ok) break;
+        umma_commit_pair(tfull_bar(acc), 0x3);
+        if (++acc == 2) {
+          acc = 0;
+          acc_phase ^= 1u;
+        }
+      }
+      if (*abort_flag && issued_any) {  // no teardown while an MMA may still run
+        umma_commit_pair(drain_bar, 0x1);
+        wait_local_only(drain_bar, 0, tmo);
+      }
+    }
+  } else {
+    // ------------------------------------------------------------------ epilogue warps
+    const int q = warp & 3;  // TMEM lane quarter of this warp
+    const int e = threadIdx.x - 64;
+    const int tloc = e >> 2, sub = e & 3;
+    const uint32_t leader_tempty0 = map_to_rank(tempty_bar(0), 0);
+    int acc = 0;
+    uint32_t acc_phase = 0;
+    for (int tile = pair; tile < num_tiles; tile += num_pairs) {
+      const int nt = tile % tok_tiles;
+      const int rest = tile / tok_tiles;
+      const int g = rest % groups;
+      const int l = rest / groups;
+      // All 128 epilogue threads take the same branch: they meet at named barriers below.
+      const bool ready = named_barrier_and(
+          1, kEpiPairThreads, mbar_wait(tfull_bar(acc), acc_phase, abort_flag, tmo));
+      if (!ready) {
+        *abort_flag = 1;
+        break;
+      }
+      tc_fence_after();
+      const uint32_t tbase = tmem_base + (static_cast<uint32_t>(q * 32) << 16) +
+                             static_cast<uint32_t>(acc * NT);
+#pragma unroll 1
+      for (int c = 0; c < NT / 32; ++c) {
+        uint32_t r[32];
+        __syncwarp();
+        tmem_ld32(tbase + c * 32, r);
+        tmem_ld_wait();
+        float* col = staging + q * 32 + lane;
+#pragma unroll
+        for (int u = 0; u < 32; ++u) col[u * kStagePitch] = __uint_as_float(r[u]);
+        named_barrier(1, kEpiPairThreads);
+        kv_rows_from_staging<HD>(p, staging, static_cast<int>(rank), l, g, nt * NT + c * 32 + tloc,
+                                 tloc, sub);
+        named_barrier(1, kEpiPairThreads);
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive_cluster(leader_tempty0 + 8u * acc);
+      if (++acc == 2) {
+        acc = 0;
+        acc_phase ^= 1u;
+      }
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  if (*abort_flag && threadIdx.x == 0) {
+    // Let this CTA's own copies still in flight land before the pair is torn down.
+    const uint64_t t0 = globaltimer_ns();
+    while (globaltimer_ns() - t0 < 200000ull) {
+    }
+    atomicExch(p.status, 6 /* DV_ERR_DEVICE_TIMEOUT */);
+  }
+  cluster_sync();  // neither CTA leaves while its peer may still touch its memory
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc_pair(tmem_base, C::kTmemCols);
+  }
+}
+
+// ------------------------------------------------------------------------------ launch
+
+template <int HD, int NT>
+static cudaError_t launch_pair_t(const CUtensorMap& w, const CUtensorMap& x, const CUtensorMap& h,
+                                 const GemmParams& p, int num_sms, cudaStream_t stream) {
+  using C = PairCfg<NT>;
+  auto kern = dv_kv_pair_kernel<HD, NT>;
+  cudaError_t err =
+      cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, C::kSmemBytes);
+  if (err != cudaSuccess) return err;
+  const long long tiles = static_cast<long long>((p.s.M + NT - 1) / NT) * (p.kv.kv / 128) * p.s.n_layers;
+  if (tiles <= 0) return cudaSuccess;
+  cudaLaunchConfig_t cfg = {};
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = 2;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.blockDim = dim3(kPairThreads, 1, 1);
+  cfg.dynamicSmemBytes = C::kSmemBytes;
+  cfg.stream = stream;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  int max_clusters = 0;
+  cfg.gridDim = dim3(2 * (num_sms / 2), 1, 1);
+  if (cudaOccupancyMaxActiveClusters(&max_clusters, kern, &cfg) != cudaSuccess || max_clusters < 1) {
+    cudaGetLastError();
+    max_clusters = num_sms / 2;
+  }
+  const long long pairs = tiles < max_clusters ? tiles : max_clusters;
+  cfg.gridDim = dim3(static_cast<unsigned>(2 * pairs), 1, 1);
+  err = cudaLaunchKernelEx(&cfg, kern, w, x, h, p);
+  if (err != cudaSuccess) return err;
+  return cudaGetLastError();
+}
+
+int kv_pair_tile_n(long long tokens) {
+  // Fewest padded tokens; per-tile fixed cost counted as 16 tokens; larger tiles win ties.
+  const int cands[4] = {256, 192, 128, 64};
+  int best = 256;
+  long long best_cost = -1;
+  for (int nt : cands) {
+    const long long tiles = (tokens + nt - 1) / nt;
+    const long long cost = tiles * (nt + 16);
+    if (best_cost < 0 || cost < best_cost) {
+      best_cost = cost;
+      best = nt;
+    }
+  }
+  return best;
+}
+
+int kv_pair_smem_bytes(int nt) {
+  switch (nt) {
+    case 64: return PairCfg<64>::kSmemBytes;
+    case 128: return PairCfg<128>::kSmemBytes;
+    case 192: return PairCfg<192>::kSmemBytes;
+    case 256: return PairCfg<256>::kSmemBytes;
+    default: return -1;
+  }
+}
+
+cudaError_t launch_kv_pair(int head_dim, int nt, const CUtensorMap& w, const CUtensorMap& x,
+                           const CUtensorMap& h, const GemmParams& p, int num_sms,
+                           cudaStream_t stream) {
+  if (head_dim == 128) {
+    switch (nt) {
+      case 64: return launch_pair_t<128, 64>(w, x, h, p, num_sms, stream);
+      case 128: return launch_pair_t<128, 128>(w, x, h, p, num_sms, stream);
+      case 192: return launch_pair_t<128, 192>(w, x, h, p, num_sms, stream);
+      case 256: return launch_pair_t<128, 256>(w, x, h, p, num_sms, stream);
+    }
+  } else if (head_dim == 64) {
+    switch (nt) {
+      case 64: return launch_pair_t<64, 64>(w, x, h, p, num_sms, stream);
+      case 128: return launch_pair_t<64, 128>(w, x, h, p, num_sms, stream);
+      case 192: return launch_pair_t<64, 192>(w, x, h, p, num_sms, stream);
+      case 256: return launch_pair_t<64, 256>(w, x, h, p, num_sms, stream);
+    }
+  }
+  return cudaErrorInvalidValue;
+}
+
+}  // namespace dv

@@ -82,3 +82,11 @@ def test_binding_fails_loudly_without_library(dv, monkeypatch):
     monkeypatch.setattr(dv, "LIB_PATH", "/nonexistent/libdv.so")
     with pytest.raises(RuntimeError):
         dv.lib()
+
+
+def test_kv_width_must_be_multiple_of_128(dv):
+    # The K/V kernel pairs 128 K channels with the same 128 V channels per CTA pair.
+    cfg = dv.make_config(512, 4, 3, 64, 16, max_batch=1, max_n_vis=64)   # kv = 192
+    w = dv.DvWeights(*([ctypes.c_void_p(256)] * 5 + [None, None]))
+    h = ctypes.c_void_p()
+    assert dv.lib().dv_memory_plan(ctypes.byref(cfg), ctypes.byref(w), None, ctypes.byref(h)) == 2
