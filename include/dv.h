@@ -131,6 +131,31 @@ int dv_build_visual_memory(dv_plan* plan, const void* x0, int batch, int n_vis, 
                            const int* slot, int slot0, const dv_kv_cache* out, void* stream);
 
 /*
+ * dv_build_visual_memory_noalloc — the same build as dv_build_visual_memory (same arguments,
+ * same output), for callers that must not allocate device memory when they build: engines
+ * that reserve all device memory at start-up and cannot give a plan a workspace sized for
+ * their largest batch, or code that must not risk the device-wide synchronisation that
+ * cudaMalloc / cudaFree can cause. The paper has no counterpart to this entry point; it
+ * only changes where the build keeps its intermediates.
+ *   - It allocates nothing: the intermediates (SiLU(E D_l) of every layer, the RMS statistics
+ *     and the row sums of squares) go to one static device array of 32 MiB that every device
+ *     loading this library holds until the process exits. The plan's own workspace is not
+ *     used, so its max_batch / max_n_vis do not bound this call.
+ *   - Limit: batch * n_vis * (n_layers * r_pad * 2 + n_layers * 4 + 4) bytes (each part
+ *     rounded up to 256 bytes, r_pad = rank rounded up to 64) must fit in 32 MiB; larger
+ *     builds return DV_ERR_UNSUPPORTED_SHAPE and launch nothing.
+ *   - The first call on a device looks up the array's device address with that device current;
+ *     make that first call before any stream capture.
+ *   - All calls on a device share the array and find it as the last call left it (nothing in
+ *     it needs to start at zero). Calls that overlap on the GPU race on it: order them on one
+ *     stream.
+ * Errors: as dv_build_visual_memory, plus DV_ERR_UNSUPPORTED_SHAPE for builds over the limit.
+ */
+int dv_build_visual_memory_noalloc(dv_plan* plan, const void* x0, int batch, int n_vis,
+                                   const int* pos, const int* slot, int slot0,
+                                   const dv_kv_cache* out, void* stream);
+
+/*
  * dv_plan_status — synchronises the device, reads and clears the plan's device status word.
  * Returns DV_OK, DV_ERR_DEVICE_TIMEOUT when a kernel of an earlier build gave up on a wait
  * (its outputs are then incomplete), or DV_ERR_INVALID_ARG for a NULL plan.

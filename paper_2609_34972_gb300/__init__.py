@@ -36,7 +36,7 @@ DV_ROPE_MROPE = 1
 
 EXPORTED = ["dv_memory_plan", "dv_build_visual_memory", "dv_plan_status", "dv_free",
             "dv_error_string", "dv_timing_enable", "dv_timing_read", "dv_kernels_per_build",
-            "dv_debug_wait_timeout", "dv_debug_copy_workspace"]
+            "dv_debug_wait_timeout", "dv_debug_copy_workspace", "dv_build_visual_memory_noalloc"]
 N_STAGES = 4
 STAGE_NAMES = ["row_sumsq", "down_proj_silu", "rms_stats", "kv_proj_rope_store"]
 
@@ -87,9 +87,12 @@ def lib() -> ctypes.CDLL:
         L.dv_kernels_per_build.argtypes = [vp]
         L.dv_debug_wait_timeout.argtypes = [vp, i32, vp]
         L.dv_debug_copy_workspace.argtypes = [vp, i32, vp, vp, vp, ctypes.POINTER(i32), vp]
+        L.dv_build_visual_memory_noalloc.argtypes = [vp, vp, i32, i32, vp, vp, i32,
+                                                     ctypes.POINTER(DvKVCache), vp]
         for name in ("dv_memory_plan", "dv_build_visual_memory", "dv_plan_status",
                      "dv_timing_enable", "dv_timing_read", "dv_kernels_per_build",
-                     "dv_debug_wait_timeout", "dv_debug_copy_workspace"):
+                     "dv_debug_wait_timeout", "dv_debug_copy_workspace",
+                     "dv_build_visual_memory_noalloc"):
             getattr(L, name).restype = i32
         _lib = L
     return _lib
@@ -173,6 +176,20 @@ def build_visual_memory(plan: Plan, x0, pos, k_cache, v_cache, slot=None, slot0:
     _check(lib().dv_build_visual_memory(plan.handle, _ptr(x0), B, N, _ptr(pos), _ptr(slot),
                                         int(slot0), ctypes.byref(kvc), _stream_handle(stream)),
            "dv_build_visual_memory")
+
+
+def build_visual_memory_noalloc(plan: Plan, x0, pos, k_cache, v_cache, slot=None,
+                                slot0: int = 0, stream=None) -> None:
+    """Same build as ``build_visual_memory`` for callers that must not allocate device memory:
+    the intermediates live in the library's static 32 MiB device array, not in the plan's
+    workspace. All such calls on a device share that array, so calls must not overlap on the
+    GPU; builds whose intermediates exceed 32 MiB raise DvError (unsupported shape)."""
+    B, N = int(x0.shape[0]), int(x0.shape[1])
+    kvc = kv_cache_view(k_cache, v_cache)
+    _check(lib().dv_build_visual_memory_noalloc(plan.handle, _ptr(x0), B, N, _ptr(pos), _ptr(slot),
+                                                int(slot0), ctypes.byref(kvc),
+                                                _stream_handle(stream)),
+           "dv_build_visual_memory_noalloc")
 
 
 def plan_status(plan: Plan) -> int:

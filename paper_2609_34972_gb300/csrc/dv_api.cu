@@ -326,6 +326,38 @@ bool dmalloc(T** out, size_t bytes) {
 
 }  // namespace
 
+namespace dv {
+
+bool plan_view(const dv_plan* p, PlanView* v) {
+  if (!p || !v) return false;
+  const dv_config& c = p->cfg;
+  v->d = c.d;
+  v->n_layers = c.n_layers;
+  v->head_dim = c.head_dim;
+  v->rope = c.rope;
+  for (int i = 0; i < 3; ++i) v->mrope_section[i] = c.mrope_section[i];
+  v->rms_eps = c.rms_eps;
+  v->num_sms = p->num_sms;
+  v->r_pad = p->r_pad;
+  v->kv = p->kv;
+  v->k_total = p->k_total;
+  v->bk = p->bk;
+  v->bv = p->bv;
+  v->status = p->status;
+  v->tm_Dst = p->tm_Dst;
+  v->tm_Bn = &p->tm_Bn;
+  v->tm_Wkv = &p->tm_Wkv;
+  v->inv_freq = p->inv_freq;
+  return true;
+}
+
+bool encode_bf16_2d(CUtensorMap* map, const void* ptr, uint64_t cols, uint64_t rows, uint64_t ld,
+                    uint32_t box_rows) {
+  return encode_2d(map, ptr, cols, rows, ld, box_rows);
+}
+
+}  // namespace dv
+
 // ================================================================================== C ABI
 
 extern "C" {

@@ -5,6 +5,8 @@
 #include <cuda.h>
 #include <cuda_runtime.h>
 
+struct dv_plan;
+
 namespace dv {
 
 constexpr int kBlockM = 128;         // UMMA M: one TMEM lane per token row
@@ -93,5 +95,25 @@ cudaError_t launch_kv_pair(int head_dim, int nt, const CUtensorMap& w, const CUt
 // Token tile (64, 128, 192 or 256) of the pair kernel for a build of `tokens` tokens.
 int kv_pair_tile_n(long long tokens);
 int kv_pair_smem_bytes(int nt);
+
+// Read-only view of a plan's repacked weights and shape, for build variants outside dv_api.cu.
+struct PlanView {
+  int d, n_layers, head_dim, rope, mrope_section[3];
+  float rms_eps;
+  int num_sms, r_pad, kv, k_total;
+  const float* bk;
+  const float* bv;
+  int* status;
+  const CUtensorMap* tm_Dst;  // three maps: boxes of 64, 128, 256 rows
+  const CUtensorMap* tm_Bn;
+  const CUtensorMap* tm_Wkv;
+  const double* inv_freq;     // head_dim / 2 values
+};
+bool plan_view(const dv_plan* p, PlanView* out);
+
+// bf16 [rows][cols] (row stride ld elements) tensor map with 128-byte-swizzled boxes of
+// 64 columns x box_rows rows; out-of-range elements read as zero.
+bool encode_bf16_2d(CUtensorMap* map, const void* ptr, uint64_t cols, uint64_t rows, uint64_t ld,
+                    uint32_t box_rows);
 
 }  // namespace dv
