@@ -348,6 +348,7 @@ bool plan_view(const dv_plan* p, PlanView* v) {
   v->tm_Bn = &p->tm_Bn;
   v->tm_Wkv = &p->tm_Wkv;
   v->inv_freq = p->inv_freq;
+  v->Wkv = p->Wkv;
   return true;
 }
 

@@ -108,6 +108,7 @@ struct PlanView {
   const CUtensorMap* tm_Bn;
   const CUtensorMap* tm_Wkv;
   const double* inv_freq;     // head_dim / 2 values
+  const uint16_t* Wkv;        // repacked K/V weights [L*2kv][k_total]
 };
 bool plan_view(const dv_plan* p, PlanView* out);
 

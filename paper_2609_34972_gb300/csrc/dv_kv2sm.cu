@@ -53,8 +53,9 @@ __device__ __forceinline__ bool wait_local_only(uint32_t bar, uint32_t parity, u
   return mbar_wait(bar, parity, &never, timeout_ns);
 }
 
-// Phase 2 of the epilogue for one staged chunk of 32 tokens: thread (token, sub) writes its
-// part of the token's K (leader) or V (peer) rows for this 128-channel group.
+// Phase 2 of the epilogue for one staged chunk of 32 tokens: epilogue warp `sub` handles one
+// quarter of the group's channels and lane `tloc` one token, so the 16-byte shared-memory reads
+// of eight consecutive lanes fall in eight different bank groups (row pitch 132 floats).
 template <int HD>
 __device__ __forceinline__ void kv_rows_from_staging(const GemmParams& p, const float* staging,
                                                      int rank, int l, int g, int tok, int tloc,
@@ -73,6 +74,15 @@ __device__ __forceinline__ void kv_rows_from_staging(const GemmParams& p, const 
     const int pair0 = sub * 16;
     const int hl = pair0 / kHalf, j0 = pair0 % kHalf;
     const int c1 = hl * HD + j0;
+    float x1[16], x2[16];
+    const float4* s1 = reinterpret_cast<const float4*>(src + c1);
+    const float4* s2 = reinterpret_cast<const float4*>(src + c1 + kHalf);
+#pragma unroll
+    for (int v = 0; v < 4; ++v) {
+      const float4 a = s1[v], c = s2[v];
+      x1[4 * v] = a.x; x1[4 * v + 1] = a.y; x1[4 * v + 2] = a.z; x1[4 * v + 3] = a.w;
+      x2[4 * v] = c.x; x2[4 * v + 1] = c.y; x2[4 * v + 2] = c.z; x2[4 * v + 3] = c.w;
+    }
     const int* pp = e.pos + static_cast<size_t>(b) * e.n_pos * e.n_vis + i;
     const float pt = static_cast<float>(pp[0]);
     const float ph = e.n_pos == 3 ? static_cast<float>(pp[e.n_vis]) : pt;
@@ -85,17 +95,17 @@ __device__ __forceinline__ void kv_rows_from_staging(const GemmParams& p, const 
 #pragma unroll
       for (int w = 0; w < 2; ++w) {
         const int j = j0 + m + w;
-        float x1 = src[c1 + m + w] * rs;
-        float x2 = src[c1 + kHalf + m + w] * rs;
+        float a1 = x1[m + w] * rs;
+        float a2 = x2[m + w] * rs;
         if (bk) {
-          x1 += bk[c1 + m + w];
-          x2 += bk[c1 + kHalf + m + w];
+          a1 += bk[c1 + m + w];
+          a2 += bk[c1 + kHalf + m + w];
         }
         const float pj = j < e.sec0 ? pt : (j < e.sec01 ? ph : pw);
         float s, c;
         rope_sincos(pj, e.inv_freq_hi[j], e.inv_freq_lo[j], e, s, c);
-        y1[w] = x1 * c - x2 * s;
-        y2[w] = x2 * c + x1 * s;
+        y1[w] = a1 * c - a2 * s;
+        y2[w] = a2 * c + a1 * s;
       }
       plo[m / 2] = pack_bf16x2(y1[0], y1[1]);
       phi[m / 2] = pack_bf16x2(y2[0], y2[1]);
@@ -108,15 +118,20 @@ __device__ __forceinline__ void kv_rows_from_staging(const GemmParams& p, const 
     const int c0 = sub * 32;
     const int hl = c0 / HD, jv = c0 % HD;
     const float* bv = e.bv ? e.bv + static_cast<size_t>(l) * e.kv + g * 128 : nullptr;
+    const float4* sv = reinterpret_cast<const float4*>(src + c0);
     uint32_t pk[16];
 #pragma unroll
-    for (int m = 0; m < 32; m += 2) {
-      float v0 = src[c0 + m] * rs, v1 = src[c0 + m + 1] * rs;
+    for (int v = 0; v < 8; ++v) {
+      const float4 a = sv[v];
+      float v0 = a.x * rs, v1 = a.y * rs, v2 = a.z * rs, v3 = a.w * rs;
       if (bv) {
-        v0 += bv[c0 + m];
-        v1 += bv[c0 + m + 1];
+        v0 += bv[c0 + 4 * v];
+        v1 += bv[c0 + 4 * v + 1];
+        v2 += bv[c0 + 4 * v + 2];
+        v3 += bv[c0 + 4 * v + 3];
       }
-      pk[m / 2] = pack_bf16x2(v0, v1);
+      pk[2 * v] = pack_bf16x2(v0, v1);
+      pk[2 * v + 1] = pack_bf16x2(v2, v3);
     }
     uint16_t* vrow = e.vc + row0 + static_cast<long long>(g * kHeadsPerGroup + hl) * e.s_head;
     store_row32(vrow + jv, pk);
@@ -264,8 +279,8 @@ __global__ void __launch_bounds__(kPairThreads, 1)
   } else {
     // ------------------------------------------------------------------ epilogue warps
     const int q = warp & 3;  // TMEM lane quarter of this warp
-    const int e = threadIdx.x - 64;
-    const int tloc = e >> 2, sub = e & 3;
+    const int sub = q;       // phase 2: this warp's quarter of the channels ...
+    const int tloc = lane;   // ... for the token of this lane
     const uint32_t leader_tempty0 = map_to_rank(tempty_bar(0), 0);
     int acc = 0;
     uint32_t acc_phase = 0;
