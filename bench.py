@@ -31,7 +31,8 @@ METRIC = "visual tokens/sec of layer-wise visual KV-memory build; % of BF16 tens
 UNIT = "visual tokens/s"
 DEFAULT_WORKLOAD = "llava15_7b"
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
-GEMM_SOURCES = ["paper_2609_34972_gb300/csrc/dv_kv2sm.cu", "paper_2609_34972_gb300/csrc/dv_ptx.cuh",
+GEMM_SOURCES = ["paper_2609_34972_gb300/csrc/dv_kv2sm.cu", "paper_2609_34972_gb300/csrc/dv_pair_tm.cu",
+                "paper_2609_34972_gb300/csrc/dv_ptx.cuh",
                 "paper_2609_34972_gb300/csrc/dv_epilogue.cuh", "paper_2609_34972_gb300/csrc/dv_internal.h"]
 
 

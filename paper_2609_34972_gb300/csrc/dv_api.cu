@@ -39,8 +39,9 @@ struct dv_plan {
   float* xx = nullptr;
   float* rstd = nullptr;
   int* status = nullptr;
-  CUtensorMap tm_Dst[3];  // boxes of 64, 128, 256 rows
-  CUtensorMap tm_Bn, tm_Wkv, tm_H;
+  CUtensorMap tm_Dst[3];       // boxes of 64, 128, 256 rows
+  CUtensorMap tm_Dst_half[3];  // boxes of 32, 64, 128 rows (halves for CTA pairs)
+  CUtensorMap tm_Bn, tm_Bn_half, tm_Wkv;
   double inv_freq[dv::kMaxHalfHead];
   // per-stage timing
   bool timing = false;
@@ -328,6 +329,136 @@ bool dmalloc(T** out, size_t bytes) {
 
 namespace dv {
 
+int check_build_args(const void* x0, int batch, int n_vis, const int* pos, const int* slot,
+                     int slot0, const dv_kv_cache* out) {
+  if (batch < 0 || n_vis < 0 || slot0 < 0) return DV_ERR_INVALID_ARG;
+  if (static_cast<long long>(batch) * n_vis == 0) return DV_OK;
+  if (!x0 || !pos || !out || !out->k || !out->v) return DV_ERR_INVALID_ARG;
+  if (!aligned16(x0) || !aligned16(out->k) || !aligned16(out->v)) return DV_ERR_ALIGNMENT;
+  const long long s[4] = {out->s_layer, out->s_batch, out->s_seq, out->s_head};
+  for (long long x : s) {
+    if (x < 0) return DV_ERR_INVALID_ARG;
+    if (x % 8 != 0) return DV_ERR_ALIGNMENT;
+  }
+  if ((reinterpret_cast<uintptr_t>(pos) & 3u) || (slot && (reinterpret_cast<uintptr_t>(slot) & 3u)))
+    return DV_ERR_ALIGNMENT;
+  return DV_OK;
+}
+
+// Orientation of the GEMMs. The 2-SM kernels with 256-token M blocks balance shared-memory
+// traffic against tensor throughput best, but pad the token count to a multiple of 256; they
+// are used when that padding costs at most 6 % over the 128-token blocks of the 1-SM kernel
+// (rank-r GEMMs) or over the token tile of the weights-as-M K/V kernel.
+static bool prefer_256(long long padded256, long long padded_other) {
+  return padded256 * 100 <= padded_other * 106;
+}
+
+cudaError_t enqueue_build(const PlanView& v, const BuildArgs& a, cudaStream_t st) {
+  const long long T = static_cast<long long>(a.batch) * a.n_vis;
+  const int L = v.n_layers, d = v.d, HD = v.head_dim;
+  const long long n1 = static_cast<long long>(L) * v.r_pad;
+  auto mark = [&](int i) {
+    if (a.marks) cudaEventRecord(a.marks[i], st);
+  };
+  const long long pad128 = (T + 127) / 128 * 128, pad256 = (T + 255) / 256 * 256;
+  const int nt = kv_pair_tile_n(T);
+  const long long pad_nt = (T + nt - 1) / nt * nt;
+  const bool rank_pairs = prefer_256(pad256, pad128);
+  const bool kv_tokens_m = prefer_256(pad256, pad_nt);
+
+  CUtensorMap tm_x0, tm_H, tm_x0_half, tm_H_half;
+  if (!encode_2d(&tm_x0, a.x0, d, static_cast<uint64_t>(T), d, kBlockM) ||
+      !encode_2d(&tm_H, a.H, n1, a.h_rows, n1, kBlockM))
+    return cudaErrorInvalidValue;
+  if (!kv_tokens_m && (!encode_2d(&tm_x0_half, a.x0, d, static_cast<uint64_t>(T), d, nt / 2) ||
+                       !encode_2d(&tm_H_half, a.H, n1, a.h_rows, n1, nt / 2)))
+    return cudaErrorInvalidValue;
+
+  GemmParams gp;
+  std::memset(&gp, 0, sizeof(gp));
+  gp.status = v.status;
+  gp.timeout_ns = kTimeoutNs;
+
+  mark(0);
+  k_row_sumsq<<<static_cast<int>((T + 7) / 8), 256, 0, st>>>(static_cast<const uint16_t*>(a.x0),
+                                                             static_cast<int>(T), d, a.xx);
+  cudaError_t err = cudaGetLastError();
+  mark(1);
+
+  // (1) H = SiLU(x0 [D_1 ... D_L]) — one GEMM over all layers' down-projections.
+  gp.s = {static_cast<int>(T), 1, static_cast<int>(n1), d / 64, 0, 0};
+  gp.silu = {a.H, static_cast<int>(n1)};
+  if (rank_pairs) {
+    const long long pairs = v.num_sms / 2;
+    int bn = 64;
+    for (int cand : {256, 128}) {
+      if (n1 % cand == 0 && (pad256 / 256) * (n1 / cand) >= pairs) {
+        bn = cand;
+        break;
+      }
+    }
+    const CUtensorMap& tmD = v.tm_Dst_half[bn == 64 ? 0 : (bn == 128 ? 1 : 2)];
+    if (err == cudaSuccess) err = launch_pair_tm(EPI_SILU, bn, 0, tm_x0, tm_x0, tmD, gp, v.num_sms, st);
+  } else {
+    const long long m_tiles = pad128 / 128;
+    int bn = 64;
+    for (int cand : {256, 128}) {
+      if (n1 % cand == 0 && m_tiles * (n1 / cand) >= v.num_sms) {
+        bn = cand;
+        break;
+      }
+    }
+    const CUtensorMap& tmD = v.tm_Dst[bn == 64 ? 0 : (bn == 128 ? 1 : 2)];
+    if (err == cudaSuccess) err = launch_gemm(EPI_SILU, bn, 0, tm_x0, tm_x0, tmD, gp, v.num_sms, st);
+  }
+  mark(2);
+
+  // (2) rstd_l from ||x0||^2 + h_l . ([x0 | h_l] [2 U_l^T ; G_l]).
+  gp.s = {static_cast<int>(T), L, v.r_pad, d / 64, v.r_pad / 64, v.r_pad};
+  gp.norm = {a.H, static_cast<int>(n1), v.r_pad, a.xx, a.rstd, a.ld_rstd, 1.0f / d, v.rms_eps};
+  if (err == cudaSuccess) {
+    err = rank_pairs ? launch_pair_tm(EPI_NORM, v.r_pad, 0, tm_x0, tm_H, *v.tm_Bn_half, gp, v.num_sms, st)
+                     : launch_gemm(EPI_NORM, v.r_pad, 0, tm_x0, tm_H, *v.tm_Bn, gp, v.num_sms, st);
+  }
+  mark(3);
+
+  // (3) K/V = rstd_l * ([x0 | h_l] Wkv_l^T) + b, RoPE on K, stored into the cache.
+  gp.s = {static_cast<int>(T), L, 2 * v.kv, d / 64, v.r_pad / 64, v.r_pad};
+  EpiKV& e = gp.kv;
+  e.rstd = a.rstd;
+  e.ld_rstd = a.ld_rstd;
+  e.bk = v.bk;
+  e.bv = v.bv;
+  e.kv = v.kv;
+  e.pos = a.pos;
+  e.slot = a.slot;
+  e.slot0 = a.slot0;
+  e.n_vis = a.n_vis;
+  e.n_pos = v.rope == DV_ROPE_MROPE ? 3 : 1;
+  e.sec0 = v.rope == DV_ROPE_MROPE ? v.mrope_section[0] : HD / 2;
+  e.sec01 = v.rope == DV_ROPE_MROPE ? v.mrope_section[0] + v.mrope_section[1] : HD / 2;
+  e.kc = static_cast<uint16_t*>(const_cast<void*>(a.kc));
+  e.vc = static_cast<uint16_t*>(const_cast<void*>(a.vc));
+  e.s_layer = a.s_layer;
+  e.s_batch = a.s_batch;
+  e.s_seq = a.s_seq;
+  e.s_head = a.s_head;
+  const double two_pi = 6.283185307179586476925286766559;
+  e.two_pi_hi = static_cast<float>(two_pi);
+  e.two_pi_lo = static_cast<float>(two_pi - static_cast<double>(e.two_pi_hi));
+  e.inv_two_pi = static_cast<float>(1.0 / two_pi);
+  for (int j = 0; j < HD / 2; ++j) {
+    e.inv_freq_hi[j] = static_cast<float>(v.inv_freq[j]);
+    e.inv_freq_lo[j] = static_cast<float>(v.inv_freq[j] - static_cast<double>(e.inv_freq_hi[j]));
+  }
+  if (err == cudaSuccess) {
+    err = kv_tokens_m ? launch_pair_tm(EPI_KV, 256, HD, tm_x0, tm_H, *v.tm_Wkv, gp, v.num_sms, st)
+                      : launch_kv_pair(HD, nt, *v.tm_Wkv, tm_x0_half, tm_H_half, gp, v.num_sms, st);
+  }
+  mark(4);
+  return err;
+}
+
 bool plan_view(const dv_plan* p, PlanView* v) {
   if (!p || !v) return false;
   const dv_config& c = p->cfg;
@@ -345,7 +476,9 @@ bool plan_view(const dv_plan* p, PlanView* v) {
   v->bv = p->bv;
   v->status = p->status;
   v->tm_Dst = p->tm_Dst;
+  v->tm_Dst_half = p->tm_Dst_half;
   v->tm_Bn = &p->tm_Bn;
+  v->tm_Bn_half = &p->tm_Bn_half;
   v->tm_Wkv = &p->tm_Wkv;
   v->inv_freq = p->inv_freq;
   v->Wkv = p->Wkv;
@@ -457,9 +590,13 @@ int dv_memory_plan(const dv_config* cfg, const dv_weights* w, void* stream, dv_p
   bool enc = encode_2d(&p->tm_Dst[0], p->Dst, d, 1ull * L * p->r_pad, d, 64) &&
              encode_2d(&p->tm_Dst[1], p->Dst, d, 1ull * L * p->r_pad, d, 128) &&
              encode_2d(&p->tm_Dst[2], p->Dst, d, 1ull * L * p->r_pad, d, 256) &&
+             encode_2d(&p->tm_Dst_half[0], p->Dst, d, 1ull * L * p->r_pad, d, 32) &&
+             encode_2d(&p->tm_Dst_half[1], p->Dst, d, 1ull * L * p->r_pad, d, 64) &&
+             encode_2d(&p->tm_Dst_half[2], p->Dst, d, 1ull * L * p->r_pad, d, 128) &&
+             encode_2d(&p->tm_Bn_half, p->Bn, p->k_total, 1ull * L * p->r_pad, p->k_total,
+                       p->r_pad / 2) &&
              encode_2d(&p->tm_Bn, p->Bn, p->k_total, 1ull * L * p->r_pad, p->k_total, p->r_pad) &&
-             encode_2d(&p->tm_Wkv, p->Wkv, p->k_total, 1ull * L * 2 * p->kv, p->k_total, 128) &&
-             encode_2d(&p->tm_H, p->H, 1ull * L * p->r_pad, T, 1ull * L * p->r_pad, dv::kBlockM);
+             encode_2d(&p->tm_Wkv, p->Wkv, p->k_total, 1ull * L * 2 * p->kv, p->k_total, 128);
   if (!enc) {
     free_plan_memory(p);
     delete p;
@@ -476,107 +613,36 @@ int dv_kernels_per_build(const dv_plan* p) { return p ? kStages : 0; }
 int dv_build_visual_memory(dv_plan* p, const void* x0, int batch, int n_vis, const int* pos,
                            const int* slot, int slot0, const dv_kv_cache* out, void* stream) {
   if (!p) return DV_ERR_INVALID_ARG;
-  if (batch < 0 || n_vis < 0 || slot0 < 0) return DV_ERR_INVALID_ARG;
+  int rc = dv::check_build_args(x0, batch, n_vis, pos, slot, slot0, out);
+  if (rc != DV_OK) return rc;
   const long long T = static_cast<long long>(batch) * n_vis;
   if (T == 0) return DV_OK;
-  if (!x0 || !pos || !out || !out->k || !out->v) return DV_ERR_INVALID_ARG;
   if (batch > p->cfg.max_batch || n_vis > p->cfg.max_n_vis || T > p->max_tokens)
     return DV_ERR_UNSUPPORTED_SHAPE;
-  if (!aligned16(x0) || !aligned16(out->k) || !aligned16(out->v)) return DV_ERR_ALIGNMENT;
-  const long long s[4] = {out->s_layer, out->s_batch, out->s_seq, out->s_head};
-  for (long long v : s) {
-    if (v < 0) return DV_ERR_INVALID_ARG;
-    if (v % 8 != 0) return DV_ERR_ALIGNMENT;
-  }
-  if ((reinterpret_cast<uintptr_t>(pos) & 3u) || (slot && (reinterpret_cast<uintptr_t>(slot) & 3u)))
-    return DV_ERR_ALIGNMENT;
-
-  const dv_config& c = p->cfg;
-  const int L = c.n_layers, d = c.d, HD = c.head_dim;
-  cudaStream_t st = static_cast<cudaStream_t>(stream);
-  CUtensorMap tm_x0;
-  if (!encode_2d(&tm_x0, x0, d, static_cast<uint64_t>(T), d, dv::kBlockM)) return DV_ERR_CUDA;
-
-  cudaEvent_t* ev = nullptr;
-  if (p->timing && p->timed < kMaxTimed) ev = &p->ev[static_cast<size_t>(p->timed++) * kEvPerBuild];
-  auto mark = [&](int i) {
-    if (ev) cudaEventRecord(ev[i], st);
-  };
-
-  GemmParams gp;
-  std::memset(&gp, 0, sizeof(gp));
-  gp.status = p->status;
-  gp.timeout_ns = kTimeoutNs;
-
-  mark(0);
-  k_row_sumsq<<<static_cast<int>((T + 7) / 8), 256, 0, st>>>(static_cast<const uint16_t*>(x0),
-                                                             static_cast<int>(T), d, p->xx);
-  cudaError_t err = cudaGetLastError();
-  mark(1);
-
-  // (1) H = SiLU(x0 [D_1 ... D_L]) — one GEMM over all layers' down-projections.
-  const int n1 = L * p->r_pad;
-  const long long m_tiles = (T + dv::kBlockM - 1) / dv::kBlockM;
-  int bn1 = 64;
-  for (int cand : {256, 128}) {
-    if (n1 % cand == 0 && m_tiles * (n1 / cand) >= p->num_sms) {
-      bn1 = cand;
-      break;
-    }
-  }
-  gp.s = {static_cast<int>(T), 1, n1, d / 64, 0, 0};
-  gp.silu = {p->H, n1};
-  const CUtensorMap& tmD = p->tm_Dst[bn1 == 64 ? 0 : (bn1 == 128 ? 1 : 2)];
-  if (err == cudaSuccess) err = dv::launch_gemm(dv::EPI_SILU, bn1, 0, tm_x0, tm_x0, tmD, gp, p->num_sms, st);
-  mark(2);
-
-  // (2) rstd_l from ||x0||^2 + h_l . ([x0 | h_l] [2 U_l^T ; G_l]).
-  gp.s = {static_cast<int>(T), L, p->r_pad, d / 64, p->r_pad / 64, p->r_pad};
-  gp.norm = {p->H, n1, p->r_pad, p->xx, p->rstd, p->max_tokens, 1.0f / d, c.rms_eps};
-  if (err == cudaSuccess)
-    err = dv::launch_gemm(dv::EPI_NORM, p->r_pad, 0, tm_x0, p->tm_H, p->tm_Bn, gp, p->num_sms, st);
-  mark(3);
-
-  // (3) K/V = rstd_l * (Wkv_l [x0 | h_l]^T) + b, RoPE on K, stored into the cache, on CTA pairs
-  //     with the weights as the M operand and NT-token blocks as the N operand.
-  const int nt = dv::kv_pair_tile_n(T);
-  CUtensorMap tm_x0_half, tm_H_half;
-  if (err == cudaSuccess &&
-      !(encode_2d(&tm_x0_half, x0, d, static_cast<uint64_t>(T), d, nt / 2) &&
-        encode_2d(&tm_H_half, p->H, 1ull * L * p->r_pad, p->max_tokens, 1ull * L * p->r_pad, nt / 2)))
-    err = cudaErrorInvalidValue;
-  gp.s = {static_cast<int>(T), L, 2 * p->kv, d / 64, p->r_pad / 64, p->r_pad};
-  dv::EpiKV& e = gp.kv;
-  e.rstd = p->rstd;
-  e.ld_rstd = p->max_tokens;
-  e.bk = p->bk;
-  e.bv = p->bv;
-  e.kv = p->kv;
-  e.pos = pos;
-  e.slot = slot;
-  e.slot0 = slot0;
-  e.n_vis = n_vis;
-  e.n_pos = c.rope == DV_ROPE_MROPE ? 3 : 1;
-  e.sec0 = c.rope == DV_ROPE_MROPE ? c.mrope_section[0] : HD / 2;
-  e.sec01 = c.rope == DV_ROPE_MROPE ? c.mrope_section[0] + c.mrope_section[1] : HD / 2;
-  e.kc = static_cast<uint16_t*>(out->k);
-  e.vc = static_cast<uint16_t*>(out->v);
-  e.s_layer = out->s_layer;
-  e.s_batch = out->s_batch;
-  e.s_seq = out->s_seq;
-  e.s_head = out->s_head;
-  const double two_pi = 6.283185307179586476925286766559;
-  e.two_pi_hi = static_cast<float>(two_pi);
-  e.two_pi_lo = static_cast<float>(two_pi - static_cast<double>(e.two_pi_hi));
-  e.inv_two_pi = static_cast<float>(1.0 / two_pi);
-  for (int j = 0; j < HD / 2; ++j) {
-    e.inv_freq_hi[j] = static_cast<float>(p->inv_freq[j]);
-    e.inv_freq_lo[j] = static_cast<float>(p->inv_freq[j] - static_cast<double>(e.inv_freq_hi[j]));
-  }
-  if (err == cudaSuccess)
-    err = dv::launch_kv_pair(HD, nt, p->tm_Wkv, tm_x0_half, tm_H_half, gp, p->num_sms, st);
-  mark(4);
-  return err == cudaSuccess ? DV_OK : DV_ERR_CUDA;
+  dv::PlanView v;
+  dv::plan_view(p, &v);
+  dv::BuildArgs a;
+  a.x0 = x0;
+  a.batch = batch;
+  a.n_vis = n_vis;
+  a.pos = pos;
+  a.slot = slot;
+  a.slot0 = slot0;
+  a.kc = out->k;
+  a.vc = out->v;
+  a.s_layer = out->s_layer;
+  a.s_batch = out->s_batch;
+  a.s_seq = out->s_seq;
+  a.s_head = out->s_head;
+  a.H = p->H;
+  a.h_rows = p->max_tokens;
+  a.rstd = p->rstd;
+  a.ld_rstd = p->max_tokens;
+  a.xx = p->xx;
+  a.marks = (p->timing && p->timed < kMaxTimed) ? &p->ev[static_cast<size_t>(p->timed++) * kEvPerBuild]
+                                                : nullptr;
+  return dv::enqueue_build(v, a, static_cast<cudaStream_t>(stream)) == cudaSuccess ? DV_OK
+                                                                                   : DV_ERR_CUDA;
 }
 
 int dv_plan_status(dv_plan* p) {

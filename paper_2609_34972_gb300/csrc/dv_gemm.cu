@@ -50,63 +50,6 @@ __device__ __forceinline__ bool wait_drain(uint32_t bar, uint32_t parity, uint64
 
 // ------------------------------------------------------------------------------ epilogues
 
-// H[t, n*BN + c] = bf16(SiLU(z)), SiLU(z) = z / (1 + e^-z)  (phi of Sec. 3.1 Eq. 4).
-template <int BN>
-__device__ __forceinline__ void epi_silu(const GemmParams& p, uint32_t tbase, int n, int t) {
-  const bool valid = t < p.s.M;
-  uint16_t* out = p.silu.H + static_cast<size_t>(valid ? t : 0) * p.silu.ldh +
-                  static_cast<size_t>(n) * BN;
-#pragma unroll 1
-  for (int c = 0; c < BN / 32; ++c) {
-    uint32_t r[32];
-    __syncwarp();
-    tmem_ld32(tbase + c * 32, r);
-    tmem_ld_wait();
-    uint32_t pk[16];
-#pragma unroll
-    for (int u = 0; u < 16; ++u) {
-      const float z0 = __uint_as_float(r[2 * u]), z1 = __uint_as_float(r[2 * u + 1]);
-      pk[u] = pack_bf16x2(z0 / (1.0f + __expf(-z0)), z1 / (1.0f + __expf(-z1)));
-    }
-    if (valid) store_row32(out + c * 32, pk);
-  }
-}
-
-// ||m||^2 = ||x0||^2 + h . (2 x0 U^T + h G) with G = U U^T, so with acc = [x0 | h] [2U^T; G]
-// the statistic of RMSNorm is rstd = 1 / sqrt((xx + h . acc) / d + eps).
-template <int BN>
-__device__ __forceinline__ void epi_norm(const GemmParams& p, uint32_t tbase, int l, int t) {
-  const bool valid = t < p.s.M;
-  const uint16_t* hrow = p.norm.H + static_cast<size_t>(valid ? t : 0) * p.norm.ldh +
-                         static_cast<size_t>(l) * p.norm.r_pad;
-  float dot = 0.0f;
-#pragma unroll 1
-  for (int c = 0; c < BN / 32; ++c) {
-    uint32_t r[32];
-    __syncwarp();
-    tmem_ld32(tbase + c * 32, r);
-    tmem_ld_wait();
-    if (valid) {
-      const uint4* hv = reinterpret_cast<const uint4*>(hrow + c * 32);
-#pragma unroll
-      for (int q = 0; q < 4; ++q) {
-        const uint4 w = hv[q];
-        const uint32_t ws[4] = {w.x, w.y, w.z, w.w};
-#pragma unroll
-        for (int e = 0; e < 4; ++e) {
-          dot = fmaf(bf16_bits_to_float(ws[e] & 0xFFFFu), __uint_as_float(r[q * 8 + 2 * e]), dot);
-          dot = fmaf(bf16_bits_to_float(ws[e] >> 16), __uint_as_float(r[q * 8 + 2 * e + 1]), dot);
-        }
-      }
-    }
-  }
-  if (valid) {
-    const float ss = fmaxf(p.norm.xx[t] + dot, 0.0f);
-    p.norm.rstd[static_cast<size_t>(l) * p.norm.ld_rstd + t] =
-        rsqrtf(fmaf(ss, p.norm.inv_d, p.norm.eps));
-  }
-}
-
 // ------------------------------------------------------------------------------ the kernel
 
 template <int EPI, int BN, int HD>

@@ -6,6 +6,7 @@
 #include <cuda_runtime.h>
 
 struct dv_plan;
+struct dv_kv_cache;
 
 namespace dv {
 
@@ -16,6 +17,7 @@ constexpr int kMaxHalfHead = 64;     // head_dim <= 128
 enum Epilogue : int {
   EPI_SILU = 0,  // stacked down-projection: H = bf16(SiLU(acc))
   EPI_NORM = 1,  // RMS statistic: rstd = (||x0||^2 + h . acc) / d + eps) ^ -1/2
+  EPI_KV = 2,    // K/V: rstd * acc + bias, RoPE on K, bf16 cache store
 };
 
 // Operand schedule shared by all three GEMMs. The A operand of a tile is the 128-row token
@@ -92,6 +94,13 @@ cudaError_t launch_kv_pair(int head_dim, int nt, const CUtensorMap& w, const CUt
                            const CUtensorMap& h, const GemmParams& p, int num_sms,
                            cudaStream_t stream);
 
+// 2-SM GEMM with 256-token M blocks (tokens as M): EPI_SILU / EPI_NORM with block_n 64/128/256
+// (b: weights with boxes of block_n / 2 rows), EPI_KV with block_n 256 (b: Wkv, 128-row boxes).
+// a0 / a1: x0 and H with 128-row boxes.
+cudaError_t launch_pair_tm(int epi, int block_n, int head_dim, const CUtensorMap& a0,
+                           const CUtensorMap& a1, const CUtensorMap& b, const GemmParams& p,
+                           int num_sms, cudaStream_t stream);
+
 // Token tile (64, 128, 192 or 256) of the pair kernel for a build of `tokens` tokens.
 int kv_pair_tile_n(long long tokens);
 int kv_pair_smem_bytes(int nt);
@@ -104,13 +113,41 @@ struct PlanView {
   const float* bk;
   const float* bv;
   int* status;
-  const CUtensorMap* tm_Dst;  // three maps: boxes of 64, 128, 256 rows
-  const CUtensorMap* tm_Bn;
-  const CUtensorMap* tm_Wkv;
+  const CUtensorMap* tm_Dst;       // three maps: boxes of 64, 128, 256 rows
+  const CUtensorMap* tm_Dst_half;  // three maps: boxes of 32, 64, 128 rows (CTA-pair halves)
+  const CUtensorMap* tm_Bn;        // boxes of r_pad rows
+  const CUtensorMap* tm_Bn_half;   // boxes of r_pad / 2 rows
+  const CUtensorMap* tm_Wkv;       // boxes of 128 rows
   const double* inv_freq;     // head_dim / 2 values
   const uint16_t* Wkv;        // repacked K/V weights [L*2kv][k_total]
 };
 bool plan_view(const dv_plan* p, PlanView* out);
+
+// Everything one build needs besides the plan: caller tensors and where the intermediates go.
+struct BuildArgs {
+  const void* x0;
+  int batch, n_vis;
+  const int* pos;
+  const int* slot;
+  int slot0;
+  const void* kc;
+  const void* vc;
+  long long s_layer, s_batch, s_seq, s_head;
+  uint16_t* H;          // [h_rows][L * r_pad] bf16
+  long long h_rows;     // rows of H that exist (>= tokens)
+  float* rstd;          // [L][ld_rstd]
+  int ld_rstd;
+  float* xx;            // [tokens]
+  cudaEvent_t* marks;   // 5 events around the 4 stages, or null
+};
+
+// Argument checks shared by the build entry points (dv_status value; DV_OK for an empty build).
+int check_build_args(const void* x0, int batch, int n_vis, const int* pos, const int* slot,
+                     int slot0, const ::dv_kv_cache* out);
+
+// Enqueue the four stages of one build on `stream` (arguments already validated).
+// Returns a cudaError_t value.
+cudaError_t enqueue_build(const PlanView& v, const BuildArgs& a, cudaStream_t stream);
 
 // bf16 [rows][cols] (row stride ld elements) tensor map with 128-byte-swizzled boxes of
 // 64 columns x box_rows rows; out-of-range elements read as zero.

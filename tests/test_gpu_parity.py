@@ -123,3 +123,29 @@ def test_full_size_sampled(name):
     assert bool(torch.isfinite(k).all()) and bool(torch.isfinite(v).all())
     del k, v, plan
     torch.cuda.empty_cache()
+
+
+# Token counts at (or just under) multiples of 256 take the 2-SM kernels with 256-token M
+# blocks for all three GEMMs (the others take 128-token 1-SM blocks and the weights-as-M K/V
+# kernel); these cases pin that path, including a ragged 256-block and both head widths.
+
+def test_tokens_as_m_path_ragged_mrope_bias():
+    # T = 2 x 250 = 500 = 256 + 244; r = 80 (r_pad 128); M-RoPE; K/V bias; 2 heads of 128.
+    cfg = gu.small_config("tm_ragged", d=512, n_layers=3, n_kv_heads=2, n_heads=8, head_dim=128,
+                          rank=80, n_vis=250, batch=2, rope="mrope", rope_theta=1e6,
+                          mrope_section=(16, 24, 24), grid=(1, 10, 25), x0_sigma=0.5,
+                          bias_sigma=0.02, seed=31, pos_start=15)
+    _full_check(synth.make_inputs(cfg), "tokens-as-M ragged")
+
+
+def test_tokens_as_m_path_head64():
+    # T = 512, 8 heads of 64 (two heads per 128-channel group), r = 16 (r_pad 64).
+    cfg = synth.config("tiny", n_vis=512, seed=32)
+    _full_check(synth.make_inputs(cfg), "tokens-as-M head 64")
+
+
+def test_tokens_as_m_path_rank64_two_batches():
+    # T = 2 x 256, r = 64: the RMS statistic tile is 64 wide (32 weight rows per CTA).
+    cfg = gu.small_config("tm_r64", d=1024, n_layers=2, n_kv_heads=4, n_heads=8, head_dim=128,
+                          rank=64, n_vis=256, batch=2, x0_sigma=0.5, seed=33, pos_start=35)
+    _full_check(synth.make_inputs(cfg), "tokens-as-M rank 64")

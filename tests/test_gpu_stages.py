@@ -21,6 +21,9 @@ def _cuda():
 
 CASES = {
     "tiny": synth.CONFIGS["tiny"],
+    # 500 tokens: the rank-r GEMMs run on CTA pairs with 256-token blocks (ragged second block)
+    "pairs": gu.small_config("pairs", d=768, n_layers=2, n_kv_heads=2, n_heads=4,
+                             head_dim=128, rank=96, n_vis=500, batch=1, x0_sigma=0.5, seed=22),
     "ragged": gu.small_config("ragged", d=1024, n_layers=3, n_kv_heads=2, n_heads=4,
                               head_dim=128, rank=80, n_vis=300, batch=2, x0_sigma=0.5, seed=21),
 }
