@@ -32,6 +32,8 @@ struct GemmShape {
   int k0_slabs;           // d / 64
   int k1_slabs;           // r_pad / 64, or 0
   int a1_cols_per_layer;  // r_pad
+  int group_m;            // tokens-as-M kernels: token blocks per L2 super-block (0: all)
+  int group_w;            // tokens-as-M kernels: weight tiles per L2 super-block (0: 1)
 };
 
 struct EpiSilu {

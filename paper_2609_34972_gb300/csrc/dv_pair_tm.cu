@@ -12,8 +12,13 @@
 //
 // Roles as in the other kernels: warp 0 lane 0 loads (both CTAs, completion counted on the
 // leader's full barrier whose single expect_tx covers both CTAs), warp 1 owns TMEM and, in the
-// leader, issues the MMAs with multicast commits, warps 2-5 drain the accumulator. Tiles run in
-// (layer, n block, m block) order, m fastest, so pairs that share weight tiles run together.
+// leader, issues the MMAs with multicast commits, warps 2-5 drain the accumulator.
+//
+// Tile order: the tiles form a grid of token blocks (m) x weight tiles (w = layer * n_tiles +
+// n). It is walked in super-blocks of group_m token blocks x group_w weight tiles (token block
+// fastest inside), columns of super-blocks one after the other, so that the operands the
+// running pairs touch fit in L2 together and each is read from DRAM a few times, not once per
+// tile of the other operand.
 #include "dv_epilogue.cuh"
 #include "dv_internal.h"
 #include "dv_ptx.cuh"
@@ -36,6 +41,19 @@ struct TmCfg {
   static_assert(kStageBytes % 1024 == 0, "stage tiles must stay 1024-byte aligned");
   static_assert((kTmemCols & (kTmemCols - 1)) == 0 && kTmemCols <= 512, "TMEM allocation");
 };
+
+// (m, w) of tile t in the super-blocked order described above.
+__device__ __forceinline__ void tm_tile(int t, int m_blocks, int w_tiles, int gm, int gw, int& m,
+                                        int& w) {
+  const int sbw = t / (gw * m_blocks);  // every column before the last one is gw wide
+  const int r = t - sbw * gw * m_blocks;
+  const int gw_eff = min(gw, w_tiles - sbw * gw);
+  const int sbm = r / (gm * gw_eff);
+  const int r2 = r - sbm * gm * gw_eff;
+  const int gm_eff = min(gm, m_blocks - sbm * gm);
+  m = sbm * gm + r2 % gm_eff;
+  w = sbw * gw + r2 / gm_eff;
+}
 
 template <int EPI, int BN, int HD>
 __global__ void __launch_bounds__(kTmThreads, 1)
@@ -90,7 +108,10 @@ __global__ void __launch_bounds__(kTmThreads, 1)
 
   const int m_tiles = (p.s.M + 255) / 256;
   const int n_tiles = p.s.n_per_layer / BN;
-  const int num_tiles = m_tiles * n_tiles * p.s.n_layers;
+  const int w_tiles = n_tiles * p.s.n_layers;
+  const int num_tiles = m_tiles * w_tiles;
+  const int gm = p.s.group_m > 0 ? min(p.s.group_m, m_tiles) : m_tiles;
+  const int gw = p.s.group_w > 0 ? min(p.s.group_w, w_tiles) : 1;
   const int k_slabs = p.s.k0_slabs + p.s.k1_slabs;
   const int pair = static_cast<int>(cluster_id_x());
   const int num_pairs = static_cast<int>(num_clusters_x());
@@ -102,10 +123,10 @@ __global__ void __launch_bounds__(kTmThreads, 1)
       int stage = 0;
       uint32_t phase = 0;
       for (int tile = pair; tile < num_tiles && !*abort_flag; tile += num_pairs) {
-        const int m = tile % m_tiles;
-        const int rest = tile / m_tiles;
-        const int n = rest % n_tiles;
-        const int l = rest / n_tiles;
+        int m, w;
+        tm_tile(tile, m_tiles, w_tiles, gm, gw, m, w);
+        const int n = w % n_tiles;
+        const int l = w / n_tiles;
         const int arow = m * 256 + static_cast<int>(rank) * 128;
         const int brow = l * p.s.n_per_layer + n * BN + static_cast<int>(rank) * (BN / 2);
         for (int ks = 0; ks < k_slabs; ++ks) {
@@ -180,10 +201,10 @@ __global__ void __launch_bounds__(kTmThreads, 1)
     int acc = 0;
     uint32_t acc_phase = 0;
     for (int tile = pair; tile < num_tiles; tile += num_pairs) {
-      const int m = tile % m_tiles;
-      const int rest = tile / m_tiles;
-      const int n = rest % n_tiles;
-      const int l = rest / n_tiles;
+      int m, w;
+      tm_tile(tile, m_tiles, w_tiles, gm, gw, m, w);
+      const int n = w % n_tiles;
+      const int l = w / n_tiles;
       // the warp leaves together (its lanes meet in __syncwarp and the TMEM loads below)
       if (!__all_sync(0xFFFFFFFFu, mbar_wait(tfull_bar(acc), acc_phase, abort_flag, tmo))) {
         *abort_flag = 1;
