@@ -126,6 +126,22 @@ def dist_env():
     return rank, world, local
 
 
+def max_over_ranks(ms: float, dist=None, device=None) -> float:
+    """The slowest rank's time (the job's time): all_reduce MAX over the process group."""
+    if dist is None:
+        return float(ms)
+    import torch
+    t = torch.tensor([float(ms)], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def weak_scaling_value(world: int, tokens_per_rank: int, steps: int, ms_max: float) -> float:
+    """Whole-job visual tokens/s: every rank builds its own batch of the workload (replicas,
+    no collective on the data path), so the job processes world * tokens_per_rank per step."""
+    return world * tokens_per_rank * steps / (ms_max / 1000.0)
+
+
 def time_oracle_sample(inp, budget_s: float, seed: int = 0):
     """Oracle throughput (tokens/s) on a bounded sample of whole tokens (all layers)."""
     import numpy as np
@@ -262,12 +278,9 @@ def run_dv(args):
     st = dv.plan_status(plan)
     if st != dv.DV_OK:
         raise RuntimeError(f"device status after timed region: {dv.error_string(st)}")
-    if dist is not None:
-        t = torch.tensor([ms_total], dtype=torch.float64, device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms_total = float(t.item())
+    ms_total = max_over_ranks(ms_total, dist, dev)
     ms_step = ms_total / args.steps
-    value = world * cfg.tokens * args.steps / (ms_total / 1000.0)
+    value = weak_scaling_value(world, cfg.tokens, args.steps, ms_total)
 
     # ---- end to end through host buffers (pinned), copies inside the timed region
     x0_h = gu.torch_bf16(inp.x0, "cpu").pin_memory()
@@ -286,11 +299,8 @@ def run_dv(args):
     torch.cuda.synchronize()
     barrier()
     ms_e2e = e0.elapsed_time(e1)
-    if dist is not None:
-        t = torch.tensor([ms_e2e], dtype=torch.float64, device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms_e2e = float(t.item())
-    e2e_value = world * cfg.tokens * e2e_steps / (ms_e2e / 1000.0)
+    ms_e2e = max_over_ranks(ms_e2e, dist, dev)
+    e2e_value = weak_scaling_value(world, cfg.tokens, e2e_steps, ms_e2e)
     h2d = x0_h.numel() * 2 + pos_h.numel() * 4
     d2h = (k_h.numel() + v_h.numel()) * 2
 
