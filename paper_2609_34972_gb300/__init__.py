@@ -239,6 +239,54 @@ def debug_workspace(plan: Plan, tokens: int, stream=None):
     return H, rstd, xx, r_pad.value
 
 
+class HostPipeline:
+    """Builds from pinned host buffers with the device-to-host read of one build overlapping the
+    next build (two device buffer sets, a compute stream and a copy stream).
+
+    Every ``submit`` copies that build's E and positions host-to-device, builds (on the compute
+    stream, in submission order: builds share the plan's workspace), and copies the written K/V
+    device-to-host into the caller's pinned buffers. It returns a CUDA event that completes
+    when those host buffers hold the result; the caller must not reuse or read them before.
+    """
+
+    def __init__(self, plan: Plan, x0_shape, pos_shape, cache_shape, depth: int = 2):
+        import torch
+        dev = torch.device("cuda", torch.cuda.current_device())
+        self.plan = plan
+        self.depth = depth
+        self.compute = torch.cuda.Stream(dev)
+        self.copy = torch.cuda.Stream(dev)
+        self.x0 = [torch.empty(x0_shape, dtype=torch.bfloat16, device=dev) for _ in range(depth)]
+        self.pos = [torch.empty(pos_shape, dtype=torch.int32, device=dev) for _ in range(depth)]
+        self.k = [torch.empty(cache_shape, dtype=torch.bfloat16, device=dev) for _ in range(depth)]
+        self.v = [torch.empty(cache_shape, dtype=torch.bfloat16, device=dev) for _ in range(depth)]
+        self.built = [torch.cuda.Event() for _ in range(depth)]
+        self.read = [torch.cuda.Event() for _ in range(depth)]
+        self.n = 0
+
+    def submit(self, x0_host, pos_host, k_host, v_host, slot=None, slot0: int = 0):
+        import torch
+        s = self.n % self.depth
+        self.n += 1
+        with torch.cuda.stream(self.compute):
+            self.compute.wait_event(self.read[s])      # this buffer set's last read is done
+            self.x0[s].copy_(x0_host, non_blocking=True)
+            self.pos[s].copy_(pos_host, non_blocking=True)
+            build_visual_memory(self.plan, self.x0[s], self.pos[s], self.k[s], self.v[s], slot=slot,
+                                slot0=slot0, stream=self.compute)
+            self.built[s].record(self.compute)
+        with torch.cuda.stream(self.copy):
+            self.copy.wait_event(self.built[s])
+            k_host.copy_(self.k[s], non_blocking=True)
+            v_host.copy_(self.v[s], non_blocking=True)
+            self.read[s].record(self.copy)
+        return self.read[s]
+
+    def synchronize(self):
+        self.copy.synchronize()
+        self.compute.synchronize()
+
+
 def build_visual_memory_from_host(plan: Plan, x0_host, pos_host, k_host, v_host, x0_dev, pos_dev,
                                   k_dev, v_dev, stream=None) -> None:
     """End-to-end build from pinned host buffers: copy E and the positions to the device, build,

@@ -4,8 +4,9 @@
 // Plan-time repacking (once per weight set). With r_pad = r rounded up to 64:
 //   Dst  [L*r_pad][d]         stacked down-projections, zero rows past r
 //   Bn   [L*r_pad][d+r_pad]   row n of layer l: [2 U_l[n,:] | G_l[n,:]], G_l = U_l U_l^T
-//   Wkv  [L*2kv][d+r_pad]     per layer, per group of 128 channels: the 128 K rows, then the
-//                             128 V rows of the same channels, each
+//   Wkv  [L*2kv][d+r_pad]     per layer, per group of 128 channels: the 128 K rows (permuted so
+//                             that RoPE partners are 16 rows apart, see wkv_row), then the 128
+//                             V rows of the same channels, each
 //                             [W[c,:] * gamma_l | (W diag(gamma_l) U_l^T)[c,:]]
 // so that, with A_l = [x0 | h_l] (h_l = SiLU(x0 D_l), Sec. 3.1 Eq. 4):
 //   A_l Bn_l^T   = 2 x0 U_l^T + h_l G_l        -> ||M_l||^2 = ||x0||^2 + h_l . (that)
@@ -130,16 +131,26 @@ __global__ void k_pack_norm_u(const uint16_t* __restrict__ U, uint16_t* __restri
 }
 
 // Row rl of layer l in Wkv: group rl / 256 of 128 channels, K (first 128) or V (next 128).
-__device__ __forceinline__ void wkv_row(int rl, int& part, int& c) {
+// V rows are in channel order. K rows are permuted so that rows 32q + i and 32q + 16 + i
+// (i < 16) are the two channels (j, j + HD/2) of rotate-half pair p = 16q + i of the group: a
+// warp that reads 32 consecutive rows (TMEM lanes) or columns then holds 16 complete RoPE pairs.
+__device__ __forceinline__ void wkv_row(int rl, int HD, int& part, int& c) {
   part = (rl >> 7) & 1;
-  c = (rl >> 8) * 128 + (rl & 127);
+  const int i = rl & 127;
+  int within = i;
+  if (part == 0) {
+    const int half = HD / 2;
+    const int p = 16 * (i >> 5) + (i & 15);
+    within = (p / half) * HD + p % half + ((i & 16) ? half : 0);
+  }
+  c = (rl >> 8) * 128 + within;
 }
 
 // Wkv rows: per layer, per 128-channel group, 128 K rows then 128 V rows; columns [0, d) hold
 // W[c][j] * gamma[l][j]; columns [d, k_total) are filled by k_rank_product (zero past r).
 __global__ void k_pack_kv(const uint16_t* __restrict__ Wk, const uint16_t* __restrict__ Wv,
                           const uint16_t* __restrict__ gamma, uint16_t* __restrict__ Wkv, int L,
-                          int kv, int d, int k_total) {
+                          int kv, int HD, int d, int k_total) {
   const long long total = static_cast<long long>(L) * 2 * kv * k_total;
   for (long long e = blockIdx.x * static_cast<long long>(blockDim.x) + threadIdx.x; e < total;
        e += static_cast<long long>(gridDim.x) * blockDim.x) {
@@ -147,7 +158,7 @@ __global__ void k_pack_kv(const uint16_t* __restrict__ Wk, const uint16_t* __res
     const long long row = e / k_total;
     const int rl = static_cast<int>(row % (2 * kv)), l = static_cast<int>(row / (2 * kv));
     int part, c;
-    wkv_row(rl, part, c);
+    wkv_row(rl, HD, part, c);
     float v = 0.0f;
     if (j < d) {
       const uint16_t* W = part ? Wv : Wk;
@@ -169,7 +180,8 @@ __global__ void __launch_bounds__(256) k_rank_product(const uint16_t* __restrict
                                                       const uint16_t* __restrict__ gamma,
                                                       const uint16_t* __restrict__ U,
                                                       uint16_t* __restrict__ out, int rows, int r,
-                                                      int d, int kv, int r_pad, int k_total) {
+                                                      int d, int kv, int HD, int r_pad,
+                                                      int k_total) {
   __shared__ float As[32][65];
   __shared__ float Us[32][65];
   const int l = blockIdx.z;
@@ -185,7 +197,7 @@ __global__ void __launch_bounds__(256) k_rank_product(const uint16_t* __restrict
       if (i < rows && j < d) {
         if (MODE == 0) {
           int part, c;
-          wkv_row(i, part, c);
+          wkv_row(i, HD, part, c);
           const uint16_t* W = part ? Wv : Wk;
           a = bf(W[(static_cast<long long>(l) * kv + c) * d + j]) *
               bf(gamma[static_cast<long long>(l) * d + j]);
@@ -586,13 +598,13 @@ int dv_memory_plan(const dv_config* cfg, const dv_weights* w, void* stream, dv_p
   k_pack_norm_u<<<grid_for(1LL * L * p->r_pad * p->k_total), 256, 0, st>>>(U, p->Bn, L, r, p->r_pad,
                                                                            d, p->k_total);
   k_pack_kv<<<grid_for(1LL * L * 2 * p->kv * p->k_total), 256, 0, st>>>(Wk, Wv, G, p->Wkv, L, p->kv,
-                                                                        d, p->k_total);
+                                                                        HD, d, p->k_total);
   {
     dim3 g1((r + 63) / 64, (r + 63) / 64, L);
-    k_rank_product<1><<<g1, 256, 0, st>>>(Wk, Wv, G, U, p->Bn, r, r, d, p->kv, p->r_pad,
+    k_rank_product<1><<<g1, 256, 0, st>>>(Wk, Wv, G, U, p->Bn, r, r, d, p->kv, HD, p->r_pad,
                                           p->k_total);
     dim3 g0((r + 63) / 64, (2 * p->kv + 63) / 64, L);
-    k_rank_product<0><<<g0, 256, 0, st>>>(Wk, Wv, G, U, p->Wkv, 2 * p->kv, r, d, p->kv,
+    k_rank_product<0><<<g0, 256, 0, st>>>(Wk, Wv, G, U, p->Wkv, 2 * p->kv, r, d, p->kv, HD,
                                           p->r_pad, p->k_total);
   }
   if (cfg->has_kv_bias) {

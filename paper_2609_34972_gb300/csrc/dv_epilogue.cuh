@@ -96,87 +96,113 @@ __device__ __forceinline__ void epi_norm(const GemmParams& p, uint32_t tbase, in
 }
 
 
-// Row-per-thread K/V epilogue for an accumulator whose 256 columns are one 128-channel group
-// of layer l: columns [0, 128) the K channels of the group (128 / HD heads), [128, 256) the
-// same V channels (the Wkv packing). Thread = token t. k = rstd * acc + b_K rotated in
-// rotate-half pairs (j, j + HD/2) of each head; v = rstd * acc + b_V.
+// Per-token context of the K/V store: cache row base, positions, rstd of one token.
+struct KvToken {
+  bool valid;
+  long long row0;  // element offset of (layer, batch, slot) in the cache
+  float rs, pt, ph, pw;
+};
+
+__device__ __forceinline__ KvToken kv_token(const GemmParams& p, int l, int t) {
+  const EpiKV& e = p.kv;
+  KvToken k;
+  k.valid = t < p.s.M;
+  const int tt = k.valid ? t : 0;
+  const int b = tt / e.n_vis, i = tt - b * e.n_vis;
+  k.rs = k.valid ? e.rstd[static_cast<size_t>(l) * e.ld_rstd + tt] : 0.0f;
+  const int slot = e.slot ? e.slot[tt] : e.slot0 + i;
+  k.row0 = l * e.s_layer + b * e.s_batch + slot * e.s_seq;
+  const int* pp = e.pos + static_cast<size_t>(b) * e.n_pos * e.n_vis + i;
+  k.pt = static_cast<float>(pp[0]);
+  k.ph = e.n_pos == 3 ? static_cast<float>(pp[e.n_vis]) : k.pt;
+  k.pw = e.n_pos == 3 ? static_cast<float>(pp[2 * e.n_vis]) : k.pt;
+  return k;
+}
+
+// K block q (0..3) of a 128-channel group for one token: r[m] and r[16 + m] (m < 16) are the
+// accumulators of rotate-half pair p = 16q + m (Wkv K-row permutation). Writes k = rstd * acc
+// + b_K, rotated, as two 32-byte runs of the head row.
+template <int HD>
+__device__ __forceinline__ void kv_store_k16(const GemmParams& p, const KvToken& tk, int l, int g,
+                                             int q, const uint32_t (&r)[32]) {
+  constexpr int kHalf = HD / 2;
+  const EpiKV& e = p.kv;
+  const int hl = (16 * q) / kHalf, j0 = (16 * q) % kHalf;
+  const int c1 = hl * HD + j0;  // channel of the first lower half within the group
+  const float* bk = e.bk ? e.bk + static_cast<size_t>(l) * e.kv + g * 128 : nullptr;
+  uint32_t plo[8], phi[8];
+#pragma unroll
+  for (int m = 0; m < 16; m += 2) {
+    float y1[2], y2[2];
+#pragma unroll
+    for (int w = 0; w < 2; ++w) {
+      const int j = j0 + m + w;
+      float x1 = __uint_as_float(r[m + w]) * tk.rs;
+      float x2 = __uint_as_float(r[16 + m + w]) * tk.rs;
+      if (bk) {
+        x1 += bk[c1 + m + w];
+        x2 += bk[c1 + kHalf + m + w];
+      }
+      const float pj = j < e.sec0 ? tk.pt : (j < e.sec01 ? tk.ph : tk.pw);
+      float s, cs;
+      rope_sincos(pj, e.inv_freq_hi[j], e.inv_freq_lo[j], e, s, cs);
+      y1[w] = x1 * cs - x2 * s;
+      y2[w] = x2 * cs + x1 * s;
+    }
+    plo[m / 2] = pack_bf16x2(y1[0], y1[1]);
+    phi[m / 2] = pack_bf16x2(y2[0], y2[1]);
+  }
+  if (tk.valid) {
+    uint16_t* krow = e.kc + tk.row0 + static_cast<long long>(g * (128 / HD) + hl) * e.s_head;
+    store_row16(krow + j0, plo);
+    store_row16(krow + kHalf + j0, phi);
+  }
+}
+
+// V block q (0..3) of a 128-channel group for one token: r[u] is channel 32q + u.
+template <int HD>
+__device__ __forceinline__ void kv_store_v32(const GemmParams& p, const KvToken& tk, int l, int g,
+                                             int q, const uint32_t (&r)[32]) {
+  const EpiKV& e = p.kv;
+  const int hl = (32 * q) / HD, jv = (32 * q) % HD;
+  const float* bv = e.bv ? e.bv + static_cast<size_t>(l) * e.kv + g * 128 + 32 * q : nullptr;
+  uint32_t pk[16];
+#pragma unroll
+  for (int u = 0; u < 16; ++u) {
+    float v0 = __uint_as_float(r[2 * u]) * tk.rs, v1 = __uint_as_float(r[2 * u + 1]) * tk.rs;
+    if (bv) {
+      v0 += bv[2 * u];
+      v1 += bv[2 * u + 1];
+    }
+    pk[u] = pack_bf16x2(v0, v1);
+  }
+  if (tk.valid) {
+    uint16_t* vrow = e.vc + tk.row0 + static_cast<long long>(g * (128 / HD) + hl) * e.s_head;
+    store_row32(vrow + jv, pk);
+  }
+}
+
+// Row-per-thread K/V epilogue (tokens as M): the thread's token row has 256 accumulator
+// columns, the 128 K rows of group g (permuted, see kv_store_k16) then its 128 V rows.
 template <int HD>
 __device__ __forceinline__ void epi_kv_group(const GemmParams& p, uint32_t tbase, int l, int g,
                                              int t) {
-  constexpr int kHalf = HD / 2;
-  constexpr int kHeads = 128 / HD;
-  const EpiKV& e = p.kv;
-  const bool valid = t < p.s.M;
-  const int tt = valid ? t : 0;
-  const int b = tt / e.n_vis, i = tt - b * e.n_vis;
-  const float rs = valid ? e.rstd[static_cast<size_t>(l) * e.ld_rstd + tt] : 0.0f;
-  const int slot = e.slot ? e.slot[tt] : e.slot0 + i;
-  const long long row0 = l * e.s_layer + b * e.s_batch + slot * e.s_seq;
-  const int* pp = e.pos + static_cast<size_t>(b) * e.n_pos * e.n_vis + i;
-  const float pt = static_cast<float>(pp[0]);
-  const float ph = e.n_pos == 3 ? static_cast<float>(pp[e.n_vis]) : pt;
-  const float pw = e.n_pos == 3 ? static_cast<float>(pp[2 * e.n_vis]) : pt;
-  const float* bk = e.bk ? e.bk + static_cast<size_t>(l) * e.kv + g * 128 : nullptr;
-  const float* bv = e.bv ? e.bv + static_cast<size_t>(l) * e.kv + g * 128 : nullptr;
-
+  const KvToken tk = kv_token(p, l, t);
 #pragma unroll 1
-  for (int c = 0; c < 128 / 64; ++c) {  // 2 blocks of 32 pairs: (head, first or second 32 j)
-    const int hl = (c * 32) / kHalf, jb = (c * 32) % kHalf;
-    const int col = hl * HD + jb;
-    uint32_t lo[32], hi[32];
-    __syncwarp();
-    tmem_ld32(tbase + col, lo);
-    tmem_ld32(tbase + col + kHalf, hi);
-    tmem_ld_wait();
-    uint32_t plo[16], phi[16];
-#pragma unroll
-    for (int u = 0; u < 32; u += 2) {
-      float y1[2], y2[2];
-#pragma unroll
-      for (int w = 0; w < 2; ++w) {
-        const int j = jb + u + w;
-        float x1 = __uint_as_float(lo[u + w]) * rs;
-        float x2 = __uint_as_float(hi[u + w]) * rs;
-        if (bk) {
-          x1 += bk[col + u + w];
-          x2 += bk[col + kHalf + u + w];
-        }
-        const float pj = j < e.sec0 ? pt : (j < e.sec01 ? ph : pw);
-        float s, cs;
-        rope_sincos(pj, e.inv_freq_hi[j], e.inv_freq_lo[j], e, s, cs);
-        y1[w] = x1 * cs - x2 * s;
-        y2[w] = x2 * cs + x1 * s;
-      }
-      plo[u / 2] = pack_bf16x2(y1[0], y1[1]);
-      phi[u / 2] = pack_bf16x2(y2[0], y2[1]);
-    }
-    if (valid) {
-      uint16_t* krow = e.kc + row0 + static_cast<long long>(g * kHeads + hl) * e.s_head;
-      store_row32(krow + jb, plo);
-      store_row32(krow + kHalf + jb, phi);
-    }
-  }
-#pragma unroll 1
-  for (int c = 0; c < 4; ++c) {  // V: 4 blocks of 32 channels
-    const int hl = (c * 32) / HD, jv = (c * 32) % HD;
+  for (int q = 0; q < 4; ++q) {
     uint32_t r[32];
     __syncwarp();
-    tmem_ld32(tbase + 128 + c * 32, r);
+    tmem_ld32(tbase + 32 * q, r);
     tmem_ld_wait();
-    uint32_t pk[16];
-#pragma unroll
-    for (int u = 0; u < 16; ++u) {
-      float v0 = __uint_as_float(r[2 * u]) * rs, v1 = __uint_as_float(r[2 * u + 1]) * rs;
-      if (bv) {
-        v0 += bv[c * 32 + 2 * u];
-        v1 += bv[c * 32 + 2 * u + 1];
-      }
-      pk[u] = pack_bf16x2(v0, v1);
-    }
-    if (valid) {
-      uint16_t* vrow = e.vc + row0 + static_cast<long long>(g * kHeads + hl) * e.s_head;
-      store_row32(vrow + jv, pk);
-    }
+    kv_store_k16<HD>(p, tk, l, g, q, r);
+  }
+#pragma unroll 1
+  for (int q = 0; q < 4; ++q) {
+    uint32_t r[32];
+    __syncwarp();
+    tmem_ld32(tbase + 128 + 32 * q, r);
+    tmem_ld_wait();
+    kv_store_v32<HD>(p, tk, l, g, q, r);
   }
 }
 

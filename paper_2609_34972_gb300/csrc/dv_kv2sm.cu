@@ -15,8 +15,12 @@
 //               announces the bytes of both CTAs
 //   warp 1      TMEM owner (cta_group::2 alloc in both CTAs); in the leader one lane issues the
 //               256 x NT x 16 MMAs and multicasts its commits to both CTAs
-//   warps 2-5   epilogue over this CTA's 128 channels: TMEM -> registers -> shared staging
-//               [32 tokens][128 channels] -> per-token rows with RoPE (K) -> 16-byte stores
+//   warps 2-5   epilogue over this CTA's 128 weight rows: TMEM -> registers -> shared staging
+//               [32 tokens][128 rows]; then warp q reads rows 32q .. 32q + 31 of the token of
+//               each lane (16-byte loads, conflict-free with a 132-float row pitch) and writes
+//               16 complete RoPE pairs of K (the Wkv K rows are permuted so that partners are 16
+//               rows apart) or 32 channels of V, as 32-byte runs. (A register transpose by
+//               xor-shuffles measured slower: shuffles use the same crossbar bandwidth.)
 // Pair tiles run in (layer, group, token block) order, token block fastest, so the pairs
 // running together share each weight tile through L2.
 #include "dv_epilogue.cuh"
@@ -28,7 +32,7 @@ namespace dv {
 constexpr int kPairThreads = 192;
 constexpr int kEpiPairThreads = 128;
 constexpr int kSmemLimit = 232448;  // largest dynamic shared memory of one CTA on sm_103
-constexpr int kStagePitch = 132;    // floats per staged token row: 128 channels + 4 pad
+constexpr int kStagePitch = 132;    // floats per staged token row: 128 weight rows + 4 pad
 
 template <int NT>
 struct PairCfg {
@@ -51,91 +55,6 @@ struct PairCfg {
 __device__ __forceinline__ bool wait_local_only(uint32_t bar, uint32_t parity, uint64_t timeout_ns) {
   int never = 0;
   return mbar_wait(bar, parity, &never, timeout_ns);
-}
-
-// Phase 2 of the epilogue for one staged chunk of 32 tokens: epilogue warp `sub` handles one
-// quarter of the group's channels and lane `tloc` one token, so the 16-byte shared-memory reads
-// of eight consecutive lanes fall in eight different bank groups (row pitch 132 floats).
-template <int HD>
-__device__ __forceinline__ void kv_rows_from_staging(const GemmParams& p, const float* staging,
-                                                     int rank, int l, int g, int tok, int tloc,
-                                                     int sub) {
-  const EpiKV& e = p.kv;
-  if (tok >= p.s.M) return;
-  const int b = tok / e.n_vis, i = tok - b * e.n_vis;
-  const float rs = e.rstd[static_cast<size_t>(l) * e.ld_rstd + tok];
-  const int slot = e.slot ? e.slot[tok] : e.slot0 + i;
-  const long long row0 = l * e.s_layer + b * e.s_batch + slot * e.s_seq;
-  const float* src = staging + tloc * kStagePitch;
-  constexpr int kHeadsPerGroup = 128 / HD;
-  if (rank == 0) {
-    // K: 16 rotate-half pairs (j, j + HD/2) of one head.
-    constexpr int kHalf = HD / 2;
-    const int pair0 = sub * 16;
-    const int hl = pair0 / kHalf, j0 = pair0 % kHalf;
-    const int c1 = hl * HD + j0;
-    float x1[16], x2[16];
-    const float4* s1 = reinterpret_cast<const float4*>(src + c1);
-    const float4* s2 = reinterpret_cast<const float4*>(src + c1 + kHalf);
-#pragma unroll
-    for (int v = 0; v < 4; ++v) {
-      const float4 a = s1[v], c = s2[v];
-      x1[4 * v] = a.x; x1[4 * v + 1] = a.y; x1[4 * v + 2] = a.z; x1[4 * v + 3] = a.w;
-      x2[4 * v] = c.x; x2[4 * v + 1] = c.y; x2[4 * v + 2] = c.z; x2[4 * v + 3] = c.w;
-    }
-    const int* pp = e.pos + static_cast<size_t>(b) * e.n_pos * e.n_vis + i;
-    const float pt = static_cast<float>(pp[0]);
-    const float ph = e.n_pos == 3 ? static_cast<float>(pp[e.n_vis]) : pt;
-    const float pw = e.n_pos == 3 ? static_cast<float>(pp[2 * e.n_vis]) : pt;
-    const float* bk = e.bk ? e.bk + static_cast<size_t>(l) * e.kv + g * 128 : nullptr;
-    uint32_t plo[8], phi[8];
-#pragma unroll
-    for (int m = 0; m < 16; m += 2) {
-      float y1[2], y2[2];
-#pragma unroll
-      for (int w = 0; w < 2; ++w) {
-        const int j = j0 + m + w;
-        float a1 = x1[m + w] * rs;
-        float a2 = x2[m + w] * rs;
-        if (bk) {
-          a1 += bk[c1 + m + w];
-          a2 += bk[c1 + kHalf + m + w];
-        }
-        const float pj = j < e.sec0 ? pt : (j < e.sec01 ? ph : pw);
-        float s, c;
-        rope_sincos(pj, e.inv_freq_hi[j], e.inv_freq_lo[j], e, s, c);
-        y1[w] = a1 * c - a2 * s;
-        y2[w] = a2 * c + a1 * s;
-      }
-      plo[m / 2] = pack_bf16x2(y1[0], y1[1]);
-      phi[m / 2] = pack_bf16x2(y2[0], y2[1]);
-    }
-    uint16_t* krow = e.kc + row0 + static_cast<long long>(g * kHeadsPerGroup + hl) * e.s_head;
-    store_row16(krow + j0, plo);
-    store_row16(krow + kHalf + j0, phi);
-  } else {
-    // V: 32 consecutive channels of one head, no rotation.
-    const int c0 = sub * 32;
-    const int hl = c0 / HD, jv = c0 % HD;
-    const float* bv = e.bv ? e.bv + static_cast<size_t>(l) * e.kv + g * 128 : nullptr;
-    const float4* sv = reinterpret_cast<const float4*>(src + c0);
-    uint32_t pk[16];
-#pragma unroll
-    for (int v = 0; v < 8; ++v) {
-      const float4 a = sv[v];
-      float v0 = a.x * rs, v1 = a.y * rs, v2 = a.z * rs, v3 = a.w * rs;
-      if (bv) {
-        v0 += bv[c0 + 4 * v];
-        v1 += bv[c0 + 4 * v + 1];
-        v2 += bv[c0 + 4 * v + 2];
-        v3 += bv[c0 + 4 * v + 3];
-      }
-      pk[2 * v] = pack_bf16x2(v0, v1);
-      pk[2 * v + 1] = pack_bf16x2(v2, v3);
-    }
-    uint16_t* vrow = e.vc + row0 + static_cast<long long>(g * kHeadsPerGroup + hl) * e.s_head;
-    store_row32(vrow + jv, pk);
-  }
 }
 
 template <int HD, int NT>
@@ -278,9 +197,7 @@ __global__ void __launch_bounds__(kPairThreads, 1)
     }
   } else {
     // ------------------------------------------------------------------ epilogue warps
-    const int q = warp & 3;  // TMEM lane quarter of this warp
-    const int sub = q;       // phase 2: this warp's quarter of the channels ...
-    const int tloc = lane;   // ... for the token of this lane
+    const int q = warp & 3;  // TMEM lane quarter = block of 32 weight rows of this warp
     const uint32_t leader_tempty0 = map_to_rank(tempty_bar(0), 0);
     int acc = 0;
     uint32_t acc_phase = 0;
@@ -303,14 +220,27 @@ __global__ void __launch_bounds__(kPairThreads, 1)
       for (int c = 0; c < NT / 32; ++c) {
         uint32_t r[32];
         __syncwarp();
-        tmem_ld32(tbase + c * 32, r);
+        tmem_ld32(tbase + c * 32, r);  // lane i: weight row 32q + i, 32 tokens
         tmem_ld_wait();
         float* col = staging + q * 32 + lane;
 #pragma unroll
         for (int u = 0; u < 32; ++u) col[u * kStagePitch] = __uint_as_float(r[u]);
         named_barrier(1, kEpiPairThreads);
-        kv_rows_from_staging<HD>(p, staging, static_cast<int>(rank), l, g, nt * NT + c * 32 + tloc,
-                                 tloc, sub);
+        const float4* src = reinterpret_cast<const float4*>(staging + lane * kStagePitch + q * 32);
+#pragma unroll
+        for (int v = 0; v < 8; ++v) {  // lane: token 32c + lane, weight rows 32q .. 32q + 31
+          const float4 w = src[v];
+          r[4 * v] = __float_as_uint(w.x);
+          r[4 * v + 1] = __float_as_uint(w.y);
+          r[4 * v + 2] = __float_as_uint(w.z);
+          r[4 * v + 3] = __float_as_uint(w.w);
+        }
+        const KvToken tk = kv_token(p, l, nt * NT + c * 32 + lane);
+        if (rank == 0) {
+          kv_store_k16<HD>(p, tk, l, g, q, r);
+        } else {
+          kv_store_v32<HD>(p, tk, l, g, q, r);
+        }
         named_barrier(1, kEpiPairThreads);
       }
       tc_fence_before();

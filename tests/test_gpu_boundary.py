@@ -109,3 +109,25 @@ def test_gpu_matches_cublas_bf16_sanity(env):
         got = v[l, 0].reshape(cfg.n_vis, -1).float()
         assert torch.allclose(got, ref, rtol=2e-2, atol=2e-2 * ref.abs().mean().item())
     dv.free(plan)
+
+
+def test_host_pipeline_matches_device_build(env):
+    # The overlapped host path returns, for every submitted build, exactly the device build's K/V.
+    import torch
+    dv, inp, plan = env
+    cfg = inp.cfg
+    k_ref, v_ref, _ = gu.run_build(inp, plan=plan)
+    x0_h = gu.torch_bf16(inp.x0, "cpu").pin_memory()
+    pos_h = torch.from_numpy(np.ascontiguousarray(inp.pos)).pin_memory()
+    x0_b = gu.torch_bf16(synth.normal_bf16(77, 0, inp.x0.shape, 0.0, 1.0), "cpu").pin_memory()
+    shape = tuple(k_ref.shape)
+    pipe = dv.HostPipeline(plan, tuple(x0_h.shape), tuple(pos_h.shape), shape)
+    outs = [(torch.empty(shape, dtype=torch.bfloat16).pin_memory(),
+             torch.empty(shape, dtype=torch.bfloat16).pin_memory()) for _ in range(4)]
+    for i, (kh, vh) in enumerate(outs):
+        pipe.submit(x0_h if i % 2 == 0 else x0_b, pos_h, kh, vh)
+    pipe.synchronize()
+    for i in (0, 2):
+        assert torch.equal(outs[i][0], k_ref.cpu()) and torch.equal(outs[i][1], v_ref.cpu())
+    assert not torch.equal(outs[1][0], k_ref.cpu())
+    assert torch.equal(outs[1][0], outs[3][0]) and torch.equal(outs[1][1], outs[3][1])
