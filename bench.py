@@ -227,12 +227,23 @@ def run_dv(args):
         from dataclasses import replace
         cfg = replace(cfg, n_layers=args.layers, name=f"{args.config}_L{args.layers}")
     peaks, peak_src = load_peaks()
+    modes = None
+    layers_built = cfg.n_layers
+    if args.skip_layers:
+        first, last = (int(x) for x in args.skip_layers.split(","))
+        modes = [dv.DV_LAYER_DROP if (l < first or l >= cfg.n_layers - last) else dv.DV_LAYER_ADAPTER
+                 for l in range(cfg.n_layers)]
+        layers_built = sum(m != dv.DV_LAYER_DROP for m in modes)
+    from dataclasses import replace as _replace
+    # the algorithmic work counts the layers that get visual memory
+    work = _replace(cfg, n_layers=layers_built,
+                    name=cfg.name + (f"_skip{args.skip_layers.replace(',', '_')}" if modes else ""))
 
     # ---- inputs (host, seeded) -> device; plan once outside the timing
     inp = synth.make_inputs(cfg)
     from tests import gpu_util as gu
     weights = gu.device_weights(inp, dev)
-    plan = dv.memory_plan(gu.dv_config(cfg), weights)
+    plan = dv.memory_plan(gu.dv_config(cfg), weights, layer_modes=modes)
     del weights
     x0 = gu.torch_bf16(inp.x0, dev)
     pos = torch.from_numpy(np.ascontiguousarray(inp.pos)).to(dev)
@@ -315,11 +326,11 @@ def run_dv(args):
 
     # ---- roofline of the dominant kernel (K/V projection + RoPE + store) and of the step
     kv_ms = stage_ms[3] / max(n_timed, 1)
-    kv_flops = 4.0 * cfg.d * cfg.kv * cfg.tokens * cfg.n_layers
+    kv_flops = 4.0 * work.d * work.kv * work.tokens * work.n_layers
     peak_tf = peaks["bf16_tflops"]
     achieved_tf = kv_flops / (kv_ms * 1e-3) / 1e12
-    t_roof_ms = max(cfg.flops() / (peak_tf * 1e12), cfg.min_bytes() / (peaks["hbm_gbs"] * 1e9)) * 1e3
-    traffic = profiled_traffic(cfg.name)
+    t_roof_ms = max(work.flops() / (peak_tf * 1e12), work.min_bytes() / (peaks["hbm_gbs"] * 1e9)) * 1e3
+    traffic = profiled_traffic(work.name)
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
@@ -330,10 +341,11 @@ def run_dv(args):
             "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
-            "config": {"workload": cfg.name, "description": cfg.description,
+            "config": {"workload": work.name, "description": cfg.description,
+                       "layers_with_visual_memory": work.n_layers,
                        "tokens_per_step_per_gpu": cfg.tokens, "layers": cfg.n_layers,
-                       "l2": f"inputs larger than L2: the {cfg.n_layers}-layer weight set "
-                             f"({(cfg.min_bytes() - cfg.tokens * cfg.n_layers * 4 * cfg.kv) / 1e9:.2f} GB "
+                       "l2": f"inputs larger than L2: the {work.n_layers}-layer weight set "
+                             f"({(work.min_bytes() - work.tokens * work.n_layers * 4 * work.kv) / 1e9:.2f} GB "
                              f"incl. x0) is streamed from HBM every step",
                        "parallelism": "replicas (weak scaling, no collective)" if world > 1 else "1 GPU"},
             "clocks": clk,
@@ -349,9 +361,9 @@ def run_dv(args):
                          "peak_source": f"bf16_tflops (burst) of {peak_src}",
                          "flops_per_launch": kv_flops, "ms_per_launch": kv_ms},
             "roofline_step": {"t_roof_ms": t_roof_ms, "frac": t_roof_ms / ms_step,
-                              "frac_sustained": max(cfg.flops() / (peaks["bf16_tflops_sustained"] * 1e12),
-                                                    cfg.min_bytes() / (peaks["hbm_gbs"] * 1e9)) * 1e3 / ms_step,
-                              "plain_flops": cfg.flops(), "min_bytes": cfg.min_bytes()},
+                              "frac_sustained": max(work.flops() / (peaks["bf16_tflops_sustained"] * 1e12),
+                                                    work.min_bytes() / (peaks["hbm_gbs"] * 1e9)) * 1e3 / ms_step,
+                              "plain_flops": work.flops(), "min_bytes": work.min_bytes()},
             "stage_ms_per_step": dict(zip(dv.STAGE_NAMES, [s / max(n_timed, 1) for s in stage_ms])),
             "cpu_baseline": cpu,
         }
@@ -369,6 +381,9 @@ def main():
     ap.add_argument("--config", default=DEFAULT_WORKLOAD)
     ap.add_argument("--layers", type=int, default=0,
                     help="override the layer count (smaller profiling cases of the same shape)")
+    ap.add_argument("--skip-layers", default="",
+                    help="F,K: no visual memory at the first F and last K layers (App. J adapter "
+                         "skipping, DV_LAYER_DROP)")
     ap.add_argument("--impl", choices=["dv", "reference"], default="dv")
     ap.add_argument("--e2e-steps", type=int, default=100)
     ap.add_argument("--no-cpu-baseline", action="store_true")

@@ -39,6 +39,12 @@ typedef enum {
 } dv_status;
 
 enum { DV_ACT_SILU = 0 };                  /* phi of Sec. 3.1 Eq. 4 */
+/* Per-layer treatment of the visual memory (App. J, layer-wise adapter skipping). */
+enum {
+  DV_LAYER_ADAPTER = 0,   /* M_l = E + SiLU(E D_l) U_l: the embedding adapter (Sec. 3.1 Eq. 5) */
+  DV_LAYER_IDENTITY = 1,  /* adapter skipped, M_l = E: visual K/V still built from E */
+  DV_LAYER_DROP = 2       /* adapter and visual memory skipped: no K/V entries for this layer */
+};
 enum { DV_ROPE_1D = 0, DV_ROPE_MROPE = 1 };
 
 /* Model shape and build limits. Supported (else DV_ERR_UNSUPPORTED_SHAPE):
@@ -71,7 +77,12 @@ typedef struct dv_config {
  *   U      [L][d][r]    up-projection U_l, nn.Linear layout [out][in]
  *   gamma  [L][d]       gain of the frozen input RMSNorm LN_l (Sec. 3.2 Eq. 7)
  *   Wk, Wv [L][kv][d]   frozen key / value projections W_K,l, W_V,l (kv = n_kv_heads*head_dim)
- *   bk, bv [L][kv]      biases, or NULL when has_kv_bias == 0 */
+ *   bk, bv [L][kv]      biases, or NULL when has_kv_bias == 0
+ *   layer_mode          HOST array of L DV_LAYER_* values, or NULL for DV_LAYER_ADAPTER at every
+ *                       layer (App. J skips the adapters of early and late layers). Layers in
+ *                       DV_LAYER_DROP get no K/V entries: builds leave their cache rows untouched,
+ *                       and the plan keeps neither repacked weights nor workspace for them.
+ *                       At least one layer must not be DV_LAYER_DROP. */
 typedef struct dv_weights {
   const void* D;
   const void* U;
@@ -80,6 +91,7 @@ typedef struct dv_weights {
   const void* Wv;
   const void* bk;
   const void* bv;
+  const unsigned char* layer_mode;
 } dv_weights;
 
 /* Destination KV cache (bf16, caller-owned). Element (layer l, batch b, slot s, head h, j) of
@@ -196,11 +208,12 @@ int dv_debug_wait_timeout(dv_plan* plan, int timeout_us, void* stream);
 /*
  * dv_debug_copy_workspace — copies the intermediate results of the last build on this plan
  * into caller-owned device buffers (stream-ordered), for stage-wise testing:
- *   H     bf16 [tokens][n_layers * r_pad]  SiLU(E D_l) of every layer, r_pad = rank rounded
- *         up to 64 (columns past rank are zero)
- *   rstd  fp32 [n_layers][tokens]           1 / sqrt(mean(M_l^2) + eps)
+ *   H     bf16 [tokens][n_planned * r_pad]  SiLU(E D_l) of every planned layer, r_pad = rank
+ *         rounded up to 64 (columns past rank are zero)
+ *   rstd  fp32 [n_planned][tokens]           1 / sqrt(mean(M_l^2) + eps)
  *   xx    fp32 [tokens]                     sum of squares of each row of E
- * Any of the three may be NULL. tokens must not exceed the plan's limit; *r_pad_out (if not
+ * n_planned is the number of layers whose mode is not DV_LAYER_DROP (n_layers when the plan
+ * was made without layer modes); planned layers appear in layer order. Any of the three may be NULL. tokens must not exceed the plan's limit; *r_pad_out (if not
  * NULL) receives r_pad.
  */
 int dv_debug_copy_workspace(dv_plan* plan, int tokens, void* H, void* rstd, void* xx,

@@ -33,6 +33,9 @@ DV_ERR_UNSUPPORTED_DEVICE = 7
 DV_ACT_SILU = 0
 DV_ROPE_1D = 0
 DV_ROPE_MROPE = 1
+DV_LAYER_ADAPTER = 0
+DV_LAYER_IDENTITY = 1
+DV_LAYER_DROP = 2
 
 EXPORTED = ["dv_memory_plan", "dv_build_visual_memory", "dv_plan_status", "dv_free",
             "dv_error_string", "dv_timing_enable", "dv_timing_read", "dv_kernels_per_build",
@@ -51,7 +54,8 @@ class DvConfig(ctypes.Structure):
 
 
 class DvWeights(ctypes.Structure):
-    _fields_ = [(n, ctypes.c_void_p) for n in ("D", "U", "gamma", "Wk", "Wv", "bk", "bv")]
+    _fields_ = [(n, ctypes.c_void_p) for n in ("D", "U", "gamma", "Wk", "Wv", "bk", "bv",
+                                               "layer_mode")]
 
 
 class DvKVCache(ctypes.Structure):
@@ -136,9 +140,11 @@ def make_config(d, n_layers, n_kv_heads, head_dim, rank, rope="1d", rope_theta=1
 class Plan:
     """Owns a ``dv_plan*``: repacked weights, workspace and TMA descriptors on one device."""
 
-    def __init__(self, handle: ctypes.c_void_p, cfg: DvConfig):
+    def __init__(self, handle: ctypes.c_void_p, cfg: DvConfig, layers=None):
         self.handle = handle
         self.cfg = cfg
+        # cache layers the plan builds (all but the DV_LAYER_DROP ones), in order
+        self.layers = list(range(cfg.n_layers)) if layers is None else list(layers)
 
     @property
     def alive(self) -> bool:
@@ -151,13 +157,22 @@ class Plan:
             pass
 
 
-def memory_plan(cfg: DvConfig, weights: dict, stream=None) -> Plan:
-    """Plan a build for ``cfg`` from device weights (dict of torch tensors, see module doc)."""
-    w = DvWeights(*[_ptr(weights.get(n)) for n in ("D", "U", "gamma", "Wk", "Wv", "bk", "bv")])
+def memory_plan(cfg: DvConfig, weights: dict, stream=None, layer_modes=None) -> Plan:
+    """Plan a build for ``cfg`` from device weights (dict of torch tensors, see module doc).
+    ``layer_modes``: optional sequence of DV_LAYER_* per layer (App. J adapter skipping)."""
+    modes = None
+    if layer_modes is not None:
+        if len(layer_modes) != cfg.n_layers:
+            raise ValueError("layer_modes needs one entry per layer")
+        modes = (ctypes.c_ubyte * cfg.n_layers)(*[int(m) for m in layer_modes])
+    w = DvWeights(*[_ptr(weights.get(n)) for n in ("D", "U", "gamma", "Wk", "Wv", "bk", "bv")],
+                  ctypes.cast(modes, ctypes.c_void_p) if modes is not None else None)
     h = ctypes.c_void_p()
     _check(lib().dv_memory_plan(ctypes.byref(cfg), ctypes.byref(w), _stream_handle(stream),
                                 ctypes.byref(h)), "dv_memory_plan")
-    return Plan(h, cfg)
+    kept = None if layer_modes is None else [l for l, m in enumerate(layer_modes)
+                                             if int(m) != DV_LAYER_DROP]
+    return Plan(h, cfg, kept)
 
 
 def kv_cache_view(k, v) -> DvKVCache:
@@ -225,12 +240,13 @@ def debug_wait_timeout(plan: Plan, timeout_us: int, stream=None) -> None:
 
 
 def debug_workspace(plan: Plan, tokens: int, stream=None):
-    """(H [tokens, L*r_pad] bf16, rstd [L, tokens] fp32, xx [tokens] fp32) of the last build."""
+    """(H [tokens, L*r_pad] bf16, rstd [L, tokens] fp32, xx [tokens] fp32) of the last build;
+    L counts the planned layers (``plan.layers``), which excludes dropped ones."""
     import torch
     r_pad = ctypes.c_int()
     _check(lib().dv_debug_copy_workspace(plan.handle, 0, None, None, None, ctypes.byref(r_pad),
                                          None), "dv_debug_copy_workspace")
-    L = plan.cfg.n_layers
+    L = len(plan.layers)
     H = torch.empty((tokens, L * r_pad.value), dtype=torch.bfloat16, device="cuda")
     rstd = torch.empty((L, tokens), dtype=torch.float32, device="cuda")
     xx = torch.empty((tokens,), dtype=torch.float32, device="cuda")

@@ -44,6 +44,9 @@ struct dv_plan {
   CUtensorMap tm_Dst_half[3];  // boxes of 32, 64, 128 rows (halves for CTA pairs)
   CUtensorMap tm_Bn, tm_Bn_half, tm_Wkv;
   double inv_freq[dv::kMaxHalfHead];
+  unsigned char mode[dv::kMaxLayers];  // DV_LAYER_* per layer
+  int n_active = 0;                    // layers not dropped
+  int16_t active[dv::kMaxLayers];      // their indices
   // per-stage timing
   bool timing = false;
   std::vector<cudaEvent_t> ev;  // kMaxTimed * kStages1
@@ -407,6 +410,7 @@ cudaError_t enqueue_build(const PlanView& v, const BuildArgs& a, cudaStream_t st
   std::memset(&gp, 0, sizeof(gp));
   gp.status = v.status;
   gp.timeout_ns = kTimeoutNs;
+  for (int i = 0; i < L; ++i) gp.layer_map[i] = v.active[i];
 
   mark(0);
   k_row_sumsq<<<static_cast<int>((T + 7) / 8), 256, 0, st>>>(static_cast<const uint16_t*>(a.x0),
@@ -495,7 +499,7 @@ bool plan_view(const dv_plan* p, PlanView* v) {
   if (!p || !v) return false;
   const dv_config& c = p->cfg;
   v->d = c.d;
-  v->n_layers = c.n_layers;
+  v->n_layers = p->n_active;
   v->head_dim = c.head_dim;
   v->rope = c.rope;
   for (int i = 0; i < 3; ++i) v->mrope_section[i] = c.mrope_section[i];
@@ -514,6 +518,7 @@ bool plan_view(const dv_plan* p, PlanView* v) {
   v->tm_Wkv = &p->tm_Wkv;
   v->inv_freq = p->inv_freq;
   v->Wkv = p->Wkv;
+  v->active = p->active;
   return true;
 }
 
@@ -554,6 +559,14 @@ int dv_memory_plan(const dv_config* cfg, const dv_weights* w, void* stream, dv_p
     if (!aligned2(q)) return DV_ERR_ALIGNMENT;
   if (cfg->has_kv_bias && (!aligned2(w->bk) || !aligned2(w->bv))) return DV_ERR_ALIGNMENT;
 
+  int n_active = 0;
+  for (int l = 0; l < cfg->n_layers; ++l) {
+    const unsigned char m = w->layer_mode ? w->layer_mode[l] : DV_LAYER_ADAPTER;
+    if (m != DV_LAYER_ADAPTER && m != DV_LAYER_IDENTITY && m != DV_LAYER_DROP) return DV_ERR_INVALID_ARG;
+    if (m != DV_LAYER_DROP) ++n_active;
+  }
+  if (n_active == 0) return DV_ERR_INVALID_ARG;
+
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess) return DV_ERR_CUDA;
   cudaDeviceProp prop;
@@ -566,7 +579,14 @@ int dv_memory_plan(const dv_config* cfg, const dv_weights* w, void* stream, dv_p
   p->cfg = *cfg;
   p->device = dev;
   p->num_sms = prop.multiProcessorCount;
-  const int L = cfg->n_layers, d = cfg->d, r = cfg->rank, HD = cfg->head_dim;
+  const int d = cfg->d, r = cfg->rank, HD = cfg->head_dim;
+  for (int l = 0; l < cfg->n_layers; ++l) {
+    p->mode[l] = w->layer_mode ? w->layer_mode[l] : DV_LAYER_ADAPTER;
+    if (p->mode[l] != DV_LAYER_DROP) p->active[p->n_active++] = static_cast<int16_t>(l);
+  }
+  // The plan holds the layers that are not dropped, compacted: planned layer i is cache layer
+  // active[i]; dropped layers take no weight or workspace memory.
+  const int L = p->n_active;
   p->r_pad = (r + 63) / 64 * 64;
   p->kv = cfg->n_kv_heads * HD;
   p->k_total = d + p->r_pad;
@@ -574,6 +594,10 @@ int dv_memory_plan(const dv_config* cfg, const dv_weights* w, void* stream, dv_p
   const long long T = p->max_tokens;
   cudaStream_t st = static_cast<cudaStream_t>(stream);
 
+  bool any_identity = false;
+  for (int i = 0; i < L; ++i) any_identity |= p->mode[p->active[i]] == DV_LAYER_IDENTITY;
+  const size_t per_du = sizeof(uint16_t) * static_cast<size_t>(r) * d;  // one layer of D or U
+  uint16_t* zero_du = nullptr;
   bool ok = dmalloc(&p->Dst, sizeof(uint16_t) * L * p->r_pad * d) &&
             dmalloc(&p->Bn, sizeof(uint16_t) * L * p->r_pad * p->k_total) &&
             dmalloc(&p->Wkv, sizeof(uint16_t) * static_cast<size_t>(L) * 2 * p->kv * p->k_total) &&
@@ -582,11 +606,14 @@ int dv_memory_plan(const dv_config* cfg, const dv_weights* w, void* stream, dv_p
             dmalloc(&p->status, sizeof(int));
   if (ok && cfg->has_kv_bias)
     ok = dmalloc(&p->bk, sizeof(float) * L * p->kv) && dmalloc(&p->bv, sizeof(float) * L * p->kv);
+  if (ok && any_identity) ok = dmalloc(&zero_du, per_du);
   if (!ok) {
+    if (zero_du) cudaFree(zero_du);
     free_plan_memory(p);
     delete p;
     return DV_ERR_OOM;
   }
+  if (zero_du) cudaMemsetAsync(zero_du, 0, per_du, st);
 
   const uint16_t* D = static_cast<const uint16_t*>(w->D);
   const uint16_t* U = static_cast<const uint16_t*>(w->U);
@@ -594,25 +621,43 @@ int dv_memory_plan(const dv_config* cfg, const dv_weights* w, void* stream, dv_p
   const uint16_t* Wk = static_cast<const uint16_t*>(w->Wk);
   const uint16_t* Wv = static_cast<const uint16_t*>(w->Wv);
   cudaMemsetAsync(p->status, 0, sizeof(int), st);
-  k_pack_down<<<grid_for(1LL * L * p->r_pad * d), 256, 0, st>>>(D, p->Dst, L, r, p->r_pad, d);
-  k_pack_norm_u<<<grid_for(1LL * L * p->r_pad * p->k_total), 256, 0, st>>>(U, p->Bn, L, r, p->r_pad,
-                                                                           d, p->k_total);
-  k_pack_kv<<<grid_for(1LL * L * 2 * p->kv * p->k_total), 256, 0, st>>>(Wk, Wv, G, p->Wkv, L, p->kv,
-                                                                        HD, d, p->k_total);
-  {
-    dim3 g1((r + 63) / 64, (r + 63) / 64, L);
-    k_rank_product<1><<<g1, 256, 0, st>>>(Wk, Wv, G, U, p->Bn, r, r, d, p->kv, HD, p->r_pad,
+  const size_t w_per = static_cast<size_t>(p->kv) * d;  // one layer of W_K or W_V
+  for (int i = 0; i < L; ++i) {
+    const int l = p->active[i];
+    // A layer whose adapter is skipped (DV_LAYER_IDENTITY) is packed from zero D_l and U_l,
+    // which makes every adapter term of the fold vanish: M_l = E exactly (Sec. 3.1, U = 0 is
+    // the identity).
+    const bool ident = p->mode[l] == DV_LAYER_IDENTITY;
+    const uint16_t* Dl = ident ? zero_du : D + static_cast<size_t>(l) * r * d;
+    const uint16_t* Ul = ident ? zero_du : U + static_cast<size_t>(l) * r * d;
+    const uint16_t* Gl = G + static_cast<size_t>(l) * d;
+    const uint16_t* Wkl = Wk + static_cast<size_t>(l) * w_per;
+    const uint16_t* Wvl = Wv + static_cast<size_t>(l) * w_per;
+    uint16_t* Dst_i = p->Dst + static_cast<size_t>(i) * p->r_pad * d;
+    uint16_t* Bn_i = p->Bn + static_cast<size_t>(i) * p->r_pad * p->k_total;
+    uint16_t* Wkv_i = p->Wkv + static_cast<size_t>(i) * 2 * p->kv * p->k_total;
+    k_pack_down<<<grid_for(1LL * p->r_pad * d), 256, 0, st>>>(Dl, Dst_i, 1, r, p->r_pad, d);
+    k_pack_norm_u<<<grid_for(1LL * p->r_pad * p->k_total), 256, 0, st>>>(Ul, Bn_i, 1, r, p->r_pad,
+                                                                         d, p->k_total);
+    k_pack_kv<<<grid_for(1LL * 2 * p->kv * p->k_total), 256, 0, st>>>(Wkl, Wvl, Gl, Wkv_i, 1, p->kv,
+                                                                      HD, d, p->k_total);
+    dim3 g1((r + 63) / 64, (r + 63) / 64, 1);
+    k_rank_product<1><<<g1, 256, 0, st>>>(Wkl, Wvl, Gl, Ul, Bn_i, r, r, d, p->kv, HD, p->r_pad,
                                           p->k_total);
-    dim3 g0((r + 63) / 64, (2 * p->kv + 63) / 64, L);
-    k_rank_product<0><<<g0, 256, 0, st>>>(Wk, Wv, G, U, p->Wkv, 2 * p->kv, r, d, p->kv, HD,
+    dim3 g0((r + 63) / 64, (2 * p->kv + 63) / 64, 1);
+    k_rank_product<0><<<g0, 256, 0, st>>>(Wkl, Wvl, Gl, Ul, Wkv_i, 2 * p->kv, r, d, p->kv, HD,
                                           p->r_pad, p->k_total);
-  }
-  if (cfg->has_kv_bias) {
-    k_bias_to_f32<<<grid_for(1LL * L * p->kv), 256, 0, st>>>(static_cast<const uint16_t*>(w->bk), p->bk, 1LL * L * p->kv);
-    k_bias_to_f32<<<grid_for(1LL * L * p->kv), 256, 0, st>>>(static_cast<const uint16_t*>(w->bv), p->bv, 1LL * L * p->kv);
+    if (cfg->has_kv_bias) {
+      const size_t b0 = static_cast<size_t>(l) * p->kv;
+      k_bias_to_f32<<<grid_for(p->kv), 256, 0, st>>>(static_cast<const uint16_t*>(w->bk) + b0,
+                                                     p->bk + static_cast<size_t>(i) * p->kv, p->kv);
+      k_bias_to_f32<<<grid_for(p->kv), 256, 0, st>>>(static_cast<const uint16_t*>(w->bv) + b0,
+                                                     p->bv + static_cast<size_t>(i) * p->kv, p->kv);
+    }
   }
   cudaError_t err = cudaGetLastError();
   if (err == cudaSuccess) err = cudaStreamSynchronize(st);
+  if (zero_du) cudaFree(zero_du);
   if (err != cudaSuccess) {
     free_plan_memory(p);
     delete p;
@@ -733,7 +778,7 @@ int dv_debug_copy_workspace(dv_plan* p, int tokens, void* H, void* rstd, void* x
   if (!p || tokens < 0 || tokens > p->max_tokens) return DV_ERR_INVALID_ARG;
   if (r_pad_out) *r_pad_out = p->r_pad;
   cudaStream_t st = static_cast<cudaStream_t>(stream);
-  const int L = p->cfg.n_layers;
+  const int L = p->n_active;  // the workspace holds the planned (not dropped) layers
   const size_t hrow = static_cast<size_t>(L) * p->r_pad;
   cudaError_t err = cudaSuccess;
   if (H && tokens > 0)

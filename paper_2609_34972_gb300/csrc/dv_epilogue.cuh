@@ -111,7 +111,7 @@ __device__ __forceinline__ KvToken kv_token(const GemmParams& p, int l, int t) {
   const int b = tt / e.n_vis, i = tt - b * e.n_vis;
   k.rs = k.valid ? e.rstd[static_cast<size_t>(l) * e.ld_rstd + tt] : 0.0f;
   const int slot = e.slot ? e.slot[tt] : e.slot0 + i;
-  k.row0 = l * e.s_layer + b * e.s_batch + slot * e.s_seq;
+  k.row0 = static_cast<long long>(p.layer_map[l]) * e.s_layer + b * e.s_batch + slot * e.s_seq;
   const int* pp = e.pos + static_cast<size_t>(b) * e.n_pos * e.n_vis + i;
   k.pt = static_cast<float>(pp[0]);
   k.ph = e.n_pos == 3 ? static_cast<float>(pp[e.n_vis]) : k.pt;

@@ -13,6 +13,7 @@ namespace dv {
 constexpr int kBlockM = 128;         // UMMA M: one TMEM lane per token row
 constexpr int kBlockK = 64;          // bf16 elements per 128-byte swizzled row of a K slab
 constexpr int kMaxHalfHead = 64;     // head_dim <= 128
+constexpr int kMaxLayers = 256;
 
 enum Epilogue : int {
   EPI_SILU = 0,  // stacked down-projection: H = bf16(SiLU(acc))
@@ -74,6 +75,9 @@ struct EpiKV {
 
 struct GemmParams {
   GemmShape s;
+  // The plan holds the layers that are not dropped, in order; logical layer i of a launch (its
+  // weights, H columns, rstd rows and biases) writes cache layer layer_map[i].
+  int16_t layer_map[kMaxLayers];
   EpiSilu silu;
   EpiNorm norm;
   EpiKV kv;
@@ -109,7 +113,7 @@ int kv_pair_smem_bytes(int nt);
 
 // Read-only view of a plan's repacked weights and shape, for build variants outside dv_api.cu.
 struct PlanView {
-  int d, n_layers, head_dim, rope, mrope_section[3];
+  int d, n_layers, head_dim, rope, mrope_section[3];  // n_layers: layers the plan holds
   float rms_eps;
   int num_sms, r_pad, kv, k_total;
   const float* bk;
@@ -122,6 +126,7 @@ struct PlanView {
   const CUtensorMap* tm_Wkv;       // boxes of 128 rows
   const double* inv_freq;     // head_dim / 2 values
   const uint16_t* Wkv;        // repacked K/V weights [L*2kv][k_total]
+  const int16_t* active;      // cache layer of each planned layer
 };
 bool plan_view(const dv_plan* p, PlanView* out);
 

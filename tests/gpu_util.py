@@ -42,14 +42,15 @@ def dv_config(cfg, max_batch=None, max_n_vis=None):
                           has_kv_bias=cfg.bias_sigma > 0)
 
 
-def run_build(inp, plan=None, seq_len=None, batch_cache=None, slot=None, slot0=0, fill=0.0):
+def run_build(inp, plan=None, seq_len=None, batch_cache=None, slot=None, slot0=0, fill=0.0,
+              layer_modes=None, noalloc=False):
     """Plan (unless given) and build into a fresh [L, B_c, S, H, D_h] cache; returns (k, v, plan)."""
     import torch
     import paper_2609_34972_gb300 as dv
     cfg = inp.cfg
     dev = torch.device("cuda")
     if plan is None:
-        plan = dv.memory_plan(dv_config(cfg), device_weights(inp, dev))
+        plan = dv.memory_plan(dv_config(cfg), device_weights(inp, dev), layer_modes=layer_modes)
     S = seq_len or cfg.n_vis
     Bc = batch_cache or cfg.batch
     shape = (cfg.n_layers, Bc, S, cfg.n_kv_heads, cfg.head_dim)
@@ -58,7 +59,8 @@ def run_build(inp, plan=None, seq_len=None, batch_cache=None, slot=None, slot0=0
     x0 = torch_bf16(inp.x0, dev)
     pos = torch.from_numpy(np.ascontiguousarray(inp.pos)).to(dev)
     sl = None if slot is None else torch.from_numpy(np.ascontiguousarray(slot, np.int32)).to(dev)
-    dv.build_visual_memory(plan, x0, pos, k, v, slot=sl, slot0=slot0)
+    build = dv.build_visual_memory_noalloc if noalloc else dv.build_visual_memory
+    build(plan, x0, pos, k, v, slot=sl, slot0=slot0)
     torch.cuda.synchronize()
     assert dv.plan_status(plan) == dv.DV_OK
     return k, v, plan

@@ -56,7 +56,7 @@ def test_null_arguments_rejected(dv):
 def test_bad_config_rejected_before_device(dv, field, value, code):
     cfg = dv.make_config(512, 4, 8, 64, 16, max_batch=1, max_n_vis=64)
     setattr(cfg, field, value)
-    w = dv.DvWeights(*([ctypes.c_void_p(256)] * 5 + [None, None]))
+    w = dv.DvWeights(*([ctypes.c_void_p(256)] * 5 + [None, None, None]))
     h = ctypes.c_void_p()
     assert dv.lib().dv_memory_plan(ctypes.byref(cfg), ctypes.byref(w), None, ctypes.byref(h)) == code
     assert not h.value
@@ -65,14 +65,14 @@ def test_bad_config_rejected_before_device(dv, field, value, code):
 def test_mrope_sections_must_cover_half_head(dv):
     cfg = dv.make_config(512, 4, 8, 128, 16, rope="mrope", mrope_section=(16, 24, 20),
                          max_batch=1, max_n_vis=64)
-    w = dv.DvWeights(*([ctypes.c_void_p(256)] * 5 + [None, None]))
+    w = dv.DvWeights(*([ctypes.c_void_p(256)] * 5 + [None, None, None]))
     h = ctypes.c_void_p()
     assert dv.lib().dv_memory_plan(ctypes.byref(cfg), ctypes.byref(w), None, ctypes.byref(h)) == 2
 
 
 def test_missing_weights_rejected(dv):
     cfg = dv.make_config(512, 4, 8, 64, 16, max_batch=1, max_n_vis=64, has_kv_bias=True)
-    w = dv.DvWeights(*([ctypes.c_void_p(256)] * 5 + [None, None]))   # bias asked for, not given
+    w = dv.DvWeights(*([ctypes.c_void_p(256)] * 5 + [None, None, None]))   # bias asked for, not given
     h = ctypes.c_void_p()
     assert dv.lib().dv_memory_plan(ctypes.byref(cfg), ctypes.byref(w), None, ctypes.byref(h)) == 1
 
@@ -87,6 +87,16 @@ def test_binding_fails_loudly_without_library(dv, monkeypatch):
 def test_kv_width_must_be_multiple_of_128(dv):
     # The K/V kernel pairs 128 K channels with the same 128 V channels per CTA pair.
     cfg = dv.make_config(512, 4, 3, 64, 16, max_batch=1, max_n_vis=64)   # kv = 192
-    w = dv.DvWeights(*([ctypes.c_void_p(256)] * 5 + [None, None]))
+    w = dv.DvWeights(*([ctypes.c_void_p(256)] * 5 + [None, None, None]))
     h = ctypes.c_void_p()
     assert dv.lib().dv_memory_plan(ctypes.byref(cfg), ctypes.byref(w), None, ctypes.byref(h)) == 2
+
+
+@pytest.mark.parametrize("modes", [[0, 3, 0, 0], [2, 2, 2, 2]])
+def test_bad_layer_modes_rejected(dv, modes):
+    # an unknown mode, or every layer dropped, is an argument error found before the device
+    cfg = dv.make_config(512, 4, 8, 64, 16, max_batch=1, max_n_vis=64)
+    arr = (ctypes.c_ubyte * 4)(*modes)
+    w = dv.DvWeights(*([ctypes.c_void_p(256)] * 5 + [None, None, ctypes.cast(arr, ctypes.c_void_p)]))
+    h = ctypes.c_void_p()
+    assert dv.lib().dv_memory_plan(ctypes.byref(cfg), ctypes.byref(w), None, ctypes.byref(h)) == 1

@@ -149,3 +149,44 @@ def test_tokens_as_m_path_rank64_two_batches():
     cfg = gu.small_config("tm_r64", d=1024, n_layers=2, n_kv_heads=4, n_heads=8, head_dim=128,
                           rank=64, n_vis=256, batch=2, x0_sigma=0.5, seed=33, pos_start=35)
     _full_check(synth.make_inputs(cfg), "tokens-as-M rank 64")
+
+
+# Layer-wise adapter skipping (App. J): DV_LAYER_DROP layers get no K/V (their cache rows keep
+# the fill value); DV_LAYER_IDENTITY layers build K/V from M_l = E, which the oracle computes with
+# that layer's adapter weights set to zero (U_l = 0 gives the identity, Sec. 3.1).
+
+def _check_layer_modes(inp, modes, label, **kw):
+    import torch
+    cfg = inp.cfg
+    k, v, plan = gu.run_build(inp, fill=-5.0, layer_modes=modes, **kw)
+    ref_inp = synth.Inputs(cfg=cfg, x0=inp.x0, D=inp.D.copy(), U=inp.U.copy(), gamma=inp.gamma,
+                           Wk=inp.Wk, Wv=inp.Wv, bk=inp.bk, bv=inp.bv, pos=inp.pos)
+    for l, m in enumerate(modes):
+        if m == 1:
+            ref_inp.D[l] = 0
+            ref_inp.U[l] = 0
+    kept = [l for l, m in enumerate(modes) if m != 2]
+    toks = np.arange(cfg.tokens)
+    ref = oracle.build_tokens(ref_inp, toks, layers=kept)
+    gk = gu.gather(k, cfg, toks)[:, kept]
+    gv = gu.gather(v, cfg, toks)[:, kept]
+    gu.assert_parity(gk, gv, ref["k"], ref["v"], cfg.head_dim, label)
+    for l, m in enumerate(modes):
+        if m == 2:
+            assert bool((k[l] == -5.0).all()) and bool((v[l] == -5.0).all()), f"layer {l} written"
+
+
+def test_layer_modes_weights_as_m_path():
+    inp = synth.make_inputs(synth.config("tiny", n_vis=64))
+    _check_layer_modes(inp, [2, 1, 0, 2], "layer modes (weights-as-M K/V)")
+
+
+def test_layer_modes_tokens_as_m_path():
+    cfg = gu.small_config("modes_tm", d=512, n_layers=4, n_kv_heads=2, n_heads=4, head_dim=128,
+                          rank=64, n_vis=512, batch=1, x0_sigma=0.5, seed=41, pos_start=35)
+    _check_layer_modes(synth.make_inputs(cfg), [1, 0, 2, 0], "layer modes (tokens-as-M)")
+
+
+def test_layer_modes_noalloc_entry():
+    inp = synth.make_inputs(synth.config("tiny", n_vis=64, seed=42))
+    _check_layer_modes(inp, [0, 2, 2, 1], "layer modes (no-alloc entry)", noalloc=True)

@@ -55,3 +55,31 @@ def test_stage_outputs(name):
     rs = rstd.double().cpu().numpy().T
     np.testing.assert_allclose(rs, rs_ref, rtol=5e-3)
     dv.free(plan)
+
+
+def test_stage_workspace_holds_only_planned_layers():
+    # With DV_LAYER_DROP layers the plan is compacted: H and rstd hold the kept layers in order,
+    # and an IDENTITY layer's statistic is that of E itself.
+    import torch
+    import paper_2609_34972_gb300 as dv
+    cfg = CASES["ragged"]
+    inp = synth.make_inputs(cfg)
+    modes = [dv.DV_LAYER_DROP, dv.DV_LAYER_ADAPTER, dv.DV_LAYER_IDENTITY]
+    k, v, plan = gu.run_build(inp, layer_modes=modes)
+    assert plan.layers == [1, 2]
+    H, rstd, xx, r_pad = dv.debug_workspace(plan, cfg.tokens)
+    torch.cuda.synchronize()
+    assert tuple(H.shape) == (cfg.tokens, 2 * r_pad) and tuple(rstd.shape) == (2, cfg.tokens)
+    ref = oracle.build_tokens(inp, np.arange(cfg.tokens), want=("h", "m"), layers=[1])
+    Hn = H.double().cpu().numpy().reshape(cfg.tokens, 2, r_pad)
+    h = ref["h"][:, 0]
+    scale = np.sqrt(np.mean(h * h))
+    err = np.abs(Hn[:, 0, :cfg.rank] - h) / np.maximum(np.abs(h), scale)
+    assert err.max() <= 1e-2, f"H max scaled err {err.max():.3e}"
+    assert np.all(Hn[:, 1] == 0.0)                      # D = 0 for the identity layer
+    m = ref["m"][:, 0]
+    x = synth.bf16_to_f32(inp.x0).astype(np.float64).reshape(cfg.tokens, cfg.d)
+    rs = rstd.double().cpu().numpy()
+    np.testing.assert_allclose(rs[0], 1.0 / np.sqrt(np.mean(m * m, axis=1) + cfg.rms_eps), rtol=5e-3)
+    np.testing.assert_allclose(rs[1], 1.0 / np.sqrt(np.mean(x * x, axis=1) + cfg.rms_eps), rtol=5e-3)
+    dv.free(plan)
