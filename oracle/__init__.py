@@ -1,9 +1,10 @@
 """ORACLE — TEST INFRASTRUCTURE ONLY.
 
-ctypes access to ``oracle.c``, the plain fp64 CPU statement of the embedding-adapter
-visual-memory build (Sec. 3.1 Eqs. 4-5, Sec. 3.2 Eq. 7, RMSNorm per App. K, RoPE at
-the original visual positions). Only ``tests/``, ``__graft_entry__.smoke()`` and the
-CPU-baseline leg of ``bench.py`` may import this module. It imports nothing from the
+ctypes access to ``oracle.c``, the plain fp64 CPU statement of the visual-memory build
+with the embedding adapter (Sec. 3.1 Eqs. 4-5) or the recurrent adapter (Sec. 3.1 Eq. 6),
+then Sec. 3.2 Eq. 7 with RMSNorm per App. K and RoPE at the original visual positions.
+Only ``tests/``, ``__graft_entry__.smoke()`` and the CPU-baseline leg of ``bench.py`` may
+import this module. It imports nothing from the
 CUDA path, and the CUDA path imports nothing from it.
 """
 from __future__ import annotations
@@ -25,7 +26,7 @@ class _Cfg(ctypes.Structure):
     _fields_ = [("d", ctypes.c_int), ("n_layers", ctypes.c_int), ("n_kv_heads", ctypes.c_int),
                 ("head_dim", ctypes.c_int), ("rank", ctypes.c_int), ("rope", ctypes.c_int),
                 ("rope_theta", ctypes.c_double), ("mrope_section", ctypes.c_int * 3),
-                ("rms_eps", ctypes.c_double)]
+                ("rms_eps", ctypes.c_double), ("recurrent", ctypes.c_int)]
 
 
 def build(force: bool = False) -> str:
@@ -122,14 +123,15 @@ def build_tokens(inp, tokens=None, want=("k", "v"), layers=None):
     (default: all, in order).
 
     ``inp`` carries ``cfg`` (d, n_layers, n_kv_heads, head_dim, rank, rope, rope_theta,
-    mrope_section, rms_eps, n_vis) and the bf16-bit arrays x0, D, U, gamma, Wk, Wv, bk, bv
-    and int32 pos [B][P][N_v]. Returns a dict of fp64 arrays: k, v [n][Ls][kv], m, n [n][Ls][d],
+    mrope_section, rms_eps, n_vis, adapter) and the bf16-bit arrays x0, D, U, gamma, Wk, Wv,
+    bk, bv and int32 pos [B][P][N_v]. Returns a dict of fp64 arrays: k, v [n][Ls][kv], m, n [n][Ls][d],
     h [n][Ls][r] (Ls = number of evaluated layers), for the names in ``want``.
     """
     cfg = inp.cfg
     c = _Cfg(cfg.d, cfg.n_layers, cfg.n_kv_heads, cfg.head_dim, cfg.rank,
              1 if cfg.rope == "mrope" else 0, float(cfg.rope_theta),
-             (ctypes.c_int * 3)(*cfg.mrope_section), float(cfg.rms_eps))
+             (ctypes.c_int * 3)(*cfg.mrope_section), float(cfg.rms_eps),
+             1 if getattr(cfg, "adapter", "embedding") == "recurrent" else 0)
     B = inp.x0.shape[0]
     if tokens is None:
         tokens = np.arange(B * cfg.n_vis, dtype=np.int64)

@@ -22,6 +22,11 @@
  *                                      Sec. 1 / App. H keep the visual positions, so the
  *                                      backbone's rotary embedding is applied to visual keys
  *                                      at their original positions; V is not rotated.
+ * Recurrent variant (Sec. 3.1 Eq. 6): M_0 = E and M_l = A_l(M_{l-1}) for l = 1..L, where
+ * A_l(X) = X + phi(X D_l) U_l is the same adapter as above; each layer's norm, projections
+ * and rotation then act on that layer's M_l exactly as listed. The chain runs through the
+ * layers in order for each token on its own (the adapter acts row by row).
+ *
  * RoPE reading: rotate-half pairs (j, j + D_h/2) of each head, inverse frequency
  * theta^(-2j/D_h); the angle of pair j is p * theta^(-2j/D_h), where p is the 1-D
  * position, or for M-RoPE the (t, h, w) position selected by the contiguous section
@@ -47,6 +52,7 @@ typedef struct {
   double rope_theta;
   int mrope_section[3];
   double rms_eps;
+  int recurrent;       /* 0: embedding adapter (Sec. 3.1 Eq. 5), 1: recurrent (Eq. 6) */
 } oracle_cfg;
 
 static double bf16_to_f64(uint16_t b) {
@@ -115,6 +121,76 @@ void oracle_rope_head(int head_dim, double theta, int mrope, const int* section,
   }
 }
 
+/* Norm, projections, rotation and output of one token's memory m at layer l (the steps of
+ * Sec. 3.2 Eq. 7 and the RoPE reading above), written at output index o. */
+static void memory_outputs(const oracle_cfg* c, int l, const double* m, const double* h,
+                           const uint16_t* gamma, const uint16_t* Wk, const uint16_t* Wv,
+                           const uint16_t* bk, const uint16_t* bv, const double* p3, int64_t o,
+                           double* g, double* n, double* kk, double* vv, double* k_out,
+                           double* v_out, double* m_out, double* h_out, double* n_out) {
+  const int d = c->d, r = c->rank, Dh = c->head_dim, kv = c->n_kv_heads * Dh;
+  for (int j = 0; j < d; ++j) g[j] = bf16_to_f64(gamma[(int64_t)l * d + j]);
+  oracle_rmsnorm_row(d, m, g, c->rms_eps, n);
+  oracle_project_row(d, kv, Wk + (int64_t)l * kv * d, bk ? bk + (int64_t)l * kv : NULL, n, kk);
+  oracle_project_row(d, kv, Wv + (int64_t)l * kv * d, bv ? bv + (int64_t)l * kv : NULL, n, vv);
+  for (int hh = 0; hh < c->n_kv_heads; ++hh)
+    oracle_rope_head(Dh, c->rope_theta, c->rope, c->mrope_section, p3, kk + hh * Dh);
+  if (k_out) memcpy(k_out + o * kv, kk, sizeof(double) * kv);
+  if (v_out) memcpy(v_out + o * kv, vv, sizeof(double) * kv);
+  if (m_out) memcpy(m_out + o * d, m, sizeof(double) * d);
+  if (n_out) memcpy(n_out + o * d, n, sizeof(double) * d);
+  if (h_out) memcpy(h_out + o * r, h, sizeof(double) * r);
+}
+
+/* Recurrent variant (Sec. 3.1 Eq. 6) of oracle_build_tokens: for each token, M_0 = E and
+ * M_l = A_l(M_{l-1}) through the layers in order; the memory of every requested layer goes
+ * through memory_outputs. Same arguments and output layout as oracle_build_tokens. */
+static int build_tokens_recurrent(const oracle_cfg* c, const uint16_t* x0, int n_vis,
+                                  const int32_t* pos, const uint16_t* D, const uint16_t* U,
+                                  const uint16_t* gamma, const uint16_t* Wk, const uint16_t* Wv,
+                                  const uint16_t* bk, const uint16_t* bv, const int64_t* tokens,
+                                  int64_t n_tokens, const int32_t* layers, int Ls,
+                                  double* k_out, double* v_out, double* m_out, double* h_out,
+                                  double* n_out) {
+  const int d = c->d, L = c->n_layers, r = c->rank, kv = c->n_kv_heads * c->head_dim;
+  const int P = c->rope ? 3 : 1;
+  int last = 0;  /* deepest layer any output needs */
+  for (int s = 0; s < Ls; ++s) {
+    const int l = layers ? layers[s] : s;
+    if (l > last) last = l;
+  }
+#pragma omp parallel
+  {
+    double* prev = malloc(sizeof(double) * d);
+    double* m = malloc(sizeof(double) * d);
+    double* n = malloc(sizeof(double) * d);
+    double* g = malloc(sizeof(double) * d);
+    double* z = malloc(sizeof(double) * r);
+    double* h = malloc(sizeof(double) * r);
+    double* kk = malloc(sizeof(double) * kv);
+    double* vv = malloc(sizeof(double) * kv);
+#pragma omp for schedule(dynamic, 1)
+    for (int64_t q = 0; q < n_tokens; ++q) {
+      const int64_t t = tokens[q];
+      const int64_t b = t / n_vis, i = t % n_vis;
+      double p3[3];
+      for (int a = 0; a < P; ++a) p3[a] = (double)pos[(b * P + a) * n_vis + i];
+      for (int j = 0; j < d; ++j) prev[j] = bf16_to_f64(x0[t * d + j]);  /* M_0 = E */
+      for (int l = 0; l <= last && l < L; ++l) {
+        /* M_l = A_l(M_{l-1}) (layer l + 1 of Eq. 6 in the paper's 1-based numbering) */
+        oracle_adapter_row(d, r, prev, D + (int64_t)l * r * d, U + (int64_t)l * d * r, z, h, m);
+        for (int s = 0; s < Ls; ++s)
+          if ((layers ? layers[s] : s) == l)
+            memory_outputs(c, l, m, h, gamma, Wk, Wv, bk, bv, p3, q * Ls + s, g, n, kk, vv,
+                           k_out, v_out, m_out, h_out, n_out);
+        memcpy(prev, m, sizeof(double) * d);
+      }
+    }
+    free(prev); free(m); free(n); free(g); free(z); free(h); free(kk); free(vv);
+  }
+  return 0;
+}
+
 /*
  * The whole build for a list of tokens.
  *   x0    bf16 [B][n_vis][d];   pos int32 [B][P][n_vis], P = 1 (1-D) or 3 (M-RoPE)
@@ -144,6 +220,9 @@ int oracle_build_tokens(const oracle_cfg* c, const uint16_t* x0, int n_vis, cons
   if (Ls <= 0) return -1;
   for (int s = 0; layers && s < Ls; ++s)
     if (layers[s] < 0 || layers[s] >= L) return -1;
+  if (c->recurrent) return build_tokens_recurrent(c, x0, n_vis, pos, D, U, gamma, Wk, Wv, bk, bv,
+                                                 tokens, n_tokens, layers, Ls, k_out, v_out,
+                                                 m_out, h_out, n_out);
 #pragma omp parallel
   {
     double* x = malloc(sizeof(double) * d);
@@ -161,23 +240,12 @@ int oracle_build_tokens(const oracle_cfg* c, const uint16_t* x0, int n_vis, cons
         const int64_t t = tokens[q];
         const int64_t b = t / n_vis, i = t % n_vis;
         for (int j = 0; j < d; ++j) x[j] = bf16_to_f64(x0[t * d + j]);
+        /* M_l = A_l(E) (Eq. 5) */
         oracle_adapter_row(d, r, x, D + (int64_t)l * r * d, U + (int64_t)l * d * r, z, h, m);
-        for (int j = 0; j < d; ++j) g[j] = bf16_to_f64(gamma[(int64_t)l * d + j]);
-        oracle_rmsnorm_row(d, m, g, c->rms_eps, n);
-        oracle_project_row(d, kv, Wk + (int64_t)l * kv * d, bk ? bk + (int64_t)l * kv : NULL,
-                           n, kk);
-        oracle_project_row(d, kv, Wv + (int64_t)l * kv * d, bv ? bv + (int64_t)l * kv : NULL,
-                           n, vv);
         double p3[3];
         for (int a = 0; a < P; ++a) p3[a] = (double)pos[(b * P + a) * n_vis + i];
-        for (int hh = 0; hh < c->n_kv_heads; ++hh)
-          oracle_rope_head(Dh, c->rope_theta, c->rope, c->mrope_section, p3, kk + hh * Dh);
-        const int64_t o = q * Ls + ls;
-        if (k_out) memcpy(k_out + o * kv, kk, sizeof(double) * kv);
-        if (v_out) memcpy(v_out + o * kv, vv, sizeof(double) * kv);
-        if (m_out) memcpy(m_out + o * d, m, sizeof(double) * d);
-        if (n_out) memcpy(n_out + o * d, n, sizeof(double) * d);
-        if (h_out) memcpy(h_out + o * r, h, sizeof(double) * r);
+        memory_outputs(c, l, m, h, gamma, Wk, Wv, bk, bv, p3, q * Ls + ls, g, n, kk, vv, k_out,
+                       v_out, m_out, h_out, n_out);
       }
     }
     free(x); free(m); free(n); free(g); free(z); free(h); free(kk); free(vv);

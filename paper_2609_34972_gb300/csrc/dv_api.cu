@@ -104,31 +104,41 @@ __device__ __forceinline__ uint16_t to_bf16(float f) {
   return static_cast<uint16_t>(dv::pack_bf16x2(f, 0.0f) & 0xFFFFu);
 }
 
-// Dst[l*r_pad + k][j] = D[l][k][j] for k < r, else 0.
+// Planned layer i of the repacked weights comes from source layer src[i]. A layer whose
+// adapter is skipped (DV_LAYER_IDENTITY, zero_du[i] != 0) is packed as if D_l = U_l = 0, which
+// makes every adapter term of the fold vanish: M_l = E exactly (Sec. 3.1, U = 0 is the
+// identity). Passed by value (768 bytes of kernel parameters).
+struct PackLayers {
+  int16_t src[dv::kMaxLayers];
+  unsigned char zero_du[dv::kMaxLayers];
+};
+
+// Dst[i*r_pad + k][j] = D[src[i]][k][j] for k < r, else 0.
 __global__ void k_pack_down(const uint16_t* __restrict__ D, uint16_t* __restrict__ Dst, int L,
-                            int r, int r_pad, int d) {
+                            int r, int r_pad, int d, PackLayers pl) {
   const long long total = static_cast<long long>(L) * r_pad * d;
   for (long long e = blockIdx.x * static_cast<long long>(blockDim.x) + threadIdx.x; e < total;
        e += static_cast<long long>(gridDim.x) * blockDim.x) {
     const int j = static_cast<int>(e % d);
     const long long row = e / d;
-    const int k = static_cast<int>(row % r_pad), l = static_cast<int>(row / r_pad);
-    Dst[e] = k < r ? D[(static_cast<long long>(l) * r + k) * d + j] : 0;
+    const int k = static_cast<int>(row % r_pad), i = static_cast<int>(row / r_pad);
+    Dst[e] = (k < r && !pl.zero_du[i]) ? D[(static_cast<long long>(pl.src[i]) * r + k) * d + j] : 0;
   }
 }
 
-// Bn[l*r_pad + n][j] = 2 U[l][j][n] (j < d, n < r), zero for padded rows. The G block is
+// Bn[i*r_pad + n][j] = 2 U[src[i]][j][n] (j < d, n < r), zero for padded rows. The G block is
 // written by k_rank_product.
 __global__ void k_pack_norm_u(const uint16_t* __restrict__ U, uint16_t* __restrict__ Bn, int L,
-                              int r, int r_pad, int d, int k_total) {
+                              int r, int r_pad, int d, int k_total, PackLayers pl) {
   const long long total = static_cast<long long>(L) * r_pad * k_total;
   for (long long e = blockIdx.x * static_cast<long long>(blockDim.x) + threadIdx.x; e < total;
        e += static_cast<long long>(gridDim.x) * blockDim.x) {
     const int j = static_cast<int>(e % k_total);
     const long long row = e / k_total;
-    const int n = static_cast<int>(row % r_pad), l = static_cast<int>(row / r_pad);
+    const int n = static_cast<int>(row % r_pad), i = static_cast<int>(row / r_pad);
     float v = 0.0f;
-    if (j < d && n < r) v = 2.0f * bf(U[(static_cast<long long>(l) * d + j) * r + n]);
+    if (j < d && n < r && !pl.zero_du[i])
+      v = 2.0f * bf(U[(static_cast<long long>(pl.src[i]) * d + j) * r + n]);
     Bn[e] = to_bf16(v);  // the G columns (j >= d) are zero here and filled afterwards
   }
 }
@@ -149,17 +159,19 @@ __device__ __forceinline__ void wkv_row(int rl, int HD, int& part, int& c) {
   c = (rl >> 8) * 128 + within;
 }
 
-// Wkv rows: per layer, per 128-channel group, 128 K rows then 128 V rows; columns [0, d) hold
-// W[c][j] * gamma[l][j]; columns [d, k_total) are filled by k_rank_product (zero past r).
+// Wkv rows: per planned layer, per 128-channel group, 128 K rows then 128 V rows; columns
+// [0, d) hold W[c][j] * gamma[l][j] of source layer l = src[i]; columns [d, k_total) are filled
+// by k_rank_product (zero past r).
 __global__ void k_pack_kv(const uint16_t* __restrict__ Wk, const uint16_t* __restrict__ Wv,
                           const uint16_t* __restrict__ gamma, uint16_t* __restrict__ Wkv, int L,
-                          int kv, int HD, int d, int k_total) {
+                          int kv, int HD, int d, int k_total, PackLayers pl) {
   const long long total = static_cast<long long>(L) * 2 * kv * k_total;
   for (long long e = blockIdx.x * static_cast<long long>(blockDim.x) + threadIdx.x; e < total;
        e += static_cast<long long>(gridDim.x) * blockDim.x) {
     const int j = static_cast<int>(e % k_total);
     const long long row = e / k_total;
-    const int rl = static_cast<int>(row % (2 * kv)), l = static_cast<int>(row / (2 * kv));
+    const int rl = static_cast<int>(row % (2 * kv));
+    const int l = pl.src[row / (2 * kv)];
     int part, c;
     wkv_row(rl, HD, part, c);
     float v = 0.0f;
@@ -171,10 +183,11 @@ __global__ void k_pack_kv(const uint16_t* __restrict__ Wk, const uint16_t* __res
   }
 }
 
-// out[l][i][n] = sum_j A(l, i, j) * U[l][j][n] for n < r, accumulated in fp32 over j < d:
+// out[p][i][n] = sum_j A(l, i, j) * U[l][j][n] for n < r, accumulated in fp32 over j < d, for
+// planned layer p = blockIdx.z of source layer l = src[p] (U taken as zero where zero_du[p]):
 //   MODE 0 (fold):  A(l, i, j) = W_part[l][c][j] * gamma[l][j], i indexes the 2*kv Wkv rows
-//                   of layer l; the result goes to Wkv row (l, i), column d + n
-//   MODE 1 (gram):  A(l, i, j) = U[l][j][i], i < r; the result goes to Bn row l*r_pad + i,
+//                   of the layer; the result goes to Wkv row (p, i), column d + n
+//   MODE 1 (gram):  A(l, i, j) = U[l][j][i], i < r; the result goes to Bn row p*r_pad + i,
 //                   column d + n
 // 64 x 64 output tile per block, 256 threads with 4 x 4 outputs each, j in steps of 32.
 template <int MODE>
@@ -184,10 +197,11 @@ __global__ void __launch_bounds__(256) k_rank_product(const uint16_t* __restrict
                                                       const uint16_t* __restrict__ U,
                                                       uint16_t* __restrict__ out, int rows, int r,
                                                       int d, int kv, int HD, int r_pad,
-                                                      int k_total) {
+                                                      int k_total, PackLayers pl) {
   __shared__ float As[32][65];
   __shared__ float Us[32][65];
-  const int l = blockIdx.z;
+  const int p = blockIdx.z, l = pl.src[p];
+  const bool zero_u = pl.zero_du[p] != 0;
   const int i0 = blockIdx.y * 64, n0 = blockIdx.x * 64;
   const int tx = threadIdx.x & 15, ty = threadIdx.x >> 4;
   float acc[4][4] = {};
@@ -205,13 +219,13 @@ __global__ void __launch_bounds__(256) k_rank_product(const uint16_t* __restrict
           a = bf(W[(static_cast<long long>(l) * kv + c) * d + j]) *
               bf(gamma[static_cast<long long>(l) * d + j]);
         } else {
-          a = bf(Ul[static_cast<long long>(j) * r + i]);
+          a = zero_u ? 0.0f : bf(Ul[static_cast<long long>(j) * r + i]);
         }
       }
       As[jj][ii] = a;
       const int nn = e % 64, jk = e / 64;
       const int n = n0 + nn, j2 = j0 + jk;
-      Us[jk][nn] = (n < r && j2 < d) ? bf(Ul[static_cast<long long>(j2) * r + n]) : 0.0f;
+      Us[jk][nn] = (n < r && j2 < d && !zero_u) ? bf(Ul[static_cast<long long>(j2) * r + n]) : 0.0f;
     }
     __syncthreads();
 #pragma unroll 8
@@ -233,8 +247,8 @@ __global__ void __launch_bounds__(256) k_rank_product(const uint16_t* __restrict
   for (int q = 0; q < 4; ++q) {
     const int i = i0 + ty * 4 + q;
     if (i >= rows) continue;
-    const long long orow = MODE == 0 ? static_cast<long long>(l) * 2 * kv + i
-                                     : static_cast<long long>(l) * r_pad + i;
+    const long long orow = MODE == 0 ? static_cast<long long>(p) * 2 * kv + i
+                                     : static_cast<long long>(p) * r_pad + i;
 #pragma unroll
     for (int w = 0; w < 4; ++w) {
       const int n = n0 + tx * 4 + w;
@@ -243,10 +257,13 @@ __global__ void __launch_bounds__(256) k_rank_product(const uint16_t* __restrict
   }
 }
 
-__global__ void k_bias_to_f32(const uint16_t* __restrict__ b, float* __restrict__ out, long long n) {
+// out[i][c] = b[src[i]][c] in fp32.
+__global__ void k_bias_to_f32(const uint16_t* __restrict__ b, float* __restrict__ out, int L,
+                              int kv, PackLayers pl) {
+  const long long n = static_cast<long long>(L) * kv;
   for (long long e = blockIdx.x * static_cast<long long>(blockDim.x) + threadIdx.x; e < n;
        e += static_cast<long long>(gridDim.x) * blockDim.x)
-    out[e] = bf(b[e]);
+    out[e] = bf(b[static_cast<long long>(pl.src[e / kv]) * kv + e % kv]);
 }
 
 // xx[t] = sum_j x0[t][j]^2 (fp32), one warp per token row, 16-byte loads.
@@ -594,10 +611,6 @@ int dv_memory_plan(const dv_config* cfg, const dv_weights* w, void* stream, dv_p
   const long long T = p->max_tokens;
   cudaStream_t st = static_cast<cudaStream_t>(stream);
 
-  bool any_identity = false;
-  for (int i = 0; i < L; ++i) any_identity |= p->mode[p->active[i]] == DV_LAYER_IDENTITY;
-  const size_t per_du = sizeof(uint16_t) * static_cast<size_t>(r) * d;  // one layer of D or U
-  uint16_t* zero_du = nullptr;
   bool ok = dmalloc(&p->Dst, sizeof(uint16_t) * L * p->r_pad * d) &&
             dmalloc(&p->Bn, sizeof(uint16_t) * L * p->r_pad * p->k_total) &&
             dmalloc(&p->Wkv, sizeof(uint16_t) * static_cast<size_t>(L) * 2 * p->kv * p->k_total) &&
@@ -606,58 +619,45 @@ int dv_memory_plan(const dv_config* cfg, const dv_weights* w, void* stream, dv_p
             dmalloc(&p->status, sizeof(int));
   if (ok && cfg->has_kv_bias)
     ok = dmalloc(&p->bk, sizeof(float) * L * p->kv) && dmalloc(&p->bv, sizeof(float) * L * p->kv);
-  if (ok && any_identity) ok = dmalloc(&zero_du, per_du);
   if (!ok) {
-    if (zero_du) cudaFree(zero_du);
     free_plan_memory(p);
     delete p;
     return DV_ERR_OOM;
   }
-  if (zero_du) cudaMemsetAsync(zero_du, 0, per_du, st);
 
+  PackLayers pl;
+  std::memset(&pl, 0, sizeof(pl));
+  for (int i = 0; i < L; ++i) {
+    pl.src[i] = p->active[i];
+    pl.zero_du[i] = p->mode[p->active[i]] == DV_LAYER_IDENTITY;
+  }
   const uint16_t* D = static_cast<const uint16_t*>(w->D);
   const uint16_t* U = static_cast<const uint16_t*>(w->U);
   const uint16_t* G = static_cast<const uint16_t*>(w->gamma);
   const uint16_t* Wk = static_cast<const uint16_t*>(w->Wk);
   const uint16_t* Wv = static_cast<const uint16_t*>(w->Wv);
   cudaMemsetAsync(p->status, 0, sizeof(int), st);
-  const size_t w_per = static_cast<size_t>(p->kv) * d;  // one layer of W_K or W_V
-  for (int i = 0; i < L; ++i) {
-    const int l = p->active[i];
-    // A layer whose adapter is skipped (DV_LAYER_IDENTITY) is packed from zero D_l and U_l,
-    // which makes every adapter term of the fold vanish: M_l = E exactly (Sec. 3.1, U = 0 is
-    // the identity).
-    const bool ident = p->mode[l] == DV_LAYER_IDENTITY;
-    const uint16_t* Dl = ident ? zero_du : D + static_cast<size_t>(l) * r * d;
-    const uint16_t* Ul = ident ? zero_du : U + static_cast<size_t>(l) * r * d;
-    const uint16_t* Gl = G + static_cast<size_t>(l) * d;
-    const uint16_t* Wkl = Wk + static_cast<size_t>(l) * w_per;
-    const uint16_t* Wvl = Wv + static_cast<size_t>(l) * w_per;
-    uint16_t* Dst_i = p->Dst + static_cast<size_t>(i) * p->r_pad * d;
-    uint16_t* Bn_i = p->Bn + static_cast<size_t>(i) * p->r_pad * p->k_total;
-    uint16_t* Wkv_i = p->Wkv + static_cast<size_t>(i) * 2 * p->kv * p->k_total;
-    k_pack_down<<<grid_for(1LL * p->r_pad * d), 256, 0, st>>>(Dl, Dst_i, 1, r, p->r_pad, d);
-    k_pack_norm_u<<<grid_for(1LL * p->r_pad * p->k_total), 256, 0, st>>>(Ul, Bn_i, 1, r, p->r_pad,
-                                                                         d, p->k_total);
-    k_pack_kv<<<grid_for(1LL * 2 * p->kv * p->k_total), 256, 0, st>>>(Wkl, Wvl, Gl, Wkv_i, 1, p->kv,
-                                                                      HD, d, p->k_total);
-    dim3 g1((r + 63) / 64, (r + 63) / 64, 1);
-    k_rank_product<1><<<g1, 256, 0, st>>>(Wkl, Wvl, Gl, Ul, Bn_i, r, r, d, p->kv, HD, p->r_pad,
-                                          p->k_total);
-    dim3 g0((r + 63) / 64, (2 * p->kv + 63) / 64, 1);
-    k_rank_product<0><<<g0, 256, 0, st>>>(Wkl, Wvl, Gl, Ul, Wkv_i, 2 * p->kv, r, d, p->kv, HD,
-                                          p->r_pad, p->k_total);
-    if (cfg->has_kv_bias) {
-      const size_t b0 = static_cast<size_t>(l) * p->kv;
-      k_bias_to_f32<<<grid_for(p->kv), 256, 0, st>>>(static_cast<const uint16_t*>(w->bk) + b0,
-                                                     p->bk + static_cast<size_t>(i) * p->kv, p->kv);
-      k_bias_to_f32<<<grid_for(p->kv), 256, 0, st>>>(static_cast<const uint16_t*>(w->bv) + b0,
-                                                     p->bv + static_cast<size_t>(i) * p->kv, p->kv);
-    }
+  k_pack_down<<<grid_for(1LL * L * p->r_pad * d), 256, 0, st>>>(D, p->Dst, L, r, p->r_pad, d, pl);
+  k_pack_norm_u<<<grid_for(1LL * L * p->r_pad * p->k_total), 256, 0, st>>>(U, p->Bn, L, r, p->r_pad,
+                                                                           d, p->k_total, pl);
+  k_pack_kv<<<grid_for(1LL * L * 2 * p->kv * p->k_total), 256, 0, st>>>(Wk, Wv, G, p->Wkv, L, p->kv,
+                                                                        HD, d, p->k_total, pl);
+  {
+    dim3 g1((r + 63) / 64, (r + 63) / 64, L);
+    k_rank_product<1><<<g1, 256, 0, st>>>(Wk, Wv, G, U, p->Bn, r, r, d, p->kv, HD, p->r_pad,
+                                          p->k_total, pl);
+    dim3 g0((r + 63) / 64, (2 * p->kv + 63) / 64, L);
+    k_rank_product<0><<<g0, 256, 0, st>>>(Wk, Wv, G, U, p->Wkv, 2 * p->kv, r, d, p->kv, HD,
+                                          p->r_pad, p->k_total, pl);
+  }
+  if (cfg->has_kv_bias) {
+    k_bias_to_f32<<<grid_for(1LL * L * p->kv), 256, 0, st>>>(static_cast<const uint16_t*>(w->bk),
+                                                             p->bk, L, p->kv, pl);
+    k_bias_to_f32<<<grid_for(1LL * L * p->kv), 256, 0, st>>>(static_cast<const uint16_t*>(w->bv),
+                                                             p->bv, L, p->kv, pl);
   }
   cudaError_t err = cudaGetLastError();
   if (err == cudaSuccess) err = cudaStreamSynchronize(st);
-  if (zero_du) cudaFree(zero_du);
   if (err != cudaSuccess) {
     free_plan_memory(p);
     delete p;

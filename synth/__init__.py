@@ -127,6 +127,7 @@ class Config:
     pos_start: int = 0
     grid: tuple = ()            # (frames, rows, cols) of the visual grid, M-RoPE only
     ar1_rho: float = 0.0        # > 0: frame-correlated x0 (video), per token-in-frame element
+    adapter: str = "embedding"  # "embedding" (Sec. 3.1 Eq. 5) or "recurrent" (Sec. 3.1 Eq. 6)
     description: str = ""
 
     @property

@@ -32,6 +32,13 @@ MUTANTS = {
                       "{ oracle_rope_head(Dh, c->rope_theta, c->rope, c->mrope_section, p3, kk + hh * Dh); "
                       "oracle_rope_head(Dh, c->rope_theta, c->rope, c->mrope_section, p3, vv + hh * Dh); }"),
     "position_of_wrong_batch": ("pos[(b * P + a) * n_vis + i]", "pos[a * n_vis + i]"),
+    "recurrent_chain_not_carried": ("memcpy(prev, m, sizeof(double) * d);", ";"),
+    "recurrent_starts_from_zero": ("prev[j] = bf16_to_f64(x0[t * d + j]);  /* M_0 = E */",
+                                   "prev[j] = 0.0;"),
+    "recurrent_down_of_next_layer": ("oracle_adapter_row(d, r, prev, D + (int64_t)l * r * d,",
+                                     "oracle_adapter_row(d, r, prev, D + (int64_t)((l + 1) % L) * r * d,"),
+    "recurrent_outputs_previous_state": ("memory_outputs(c, l, m, h, gamma, Wk, Wv, bk, bv, p3, q * Ls + s,",
+                                         "memory_outputs(c, l, prev, h, gamma, Wk, Wv, bk, bv, p3, q * Ls + s,"),
 }
 
 

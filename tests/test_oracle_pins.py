@@ -5,6 +5,7 @@ a transposed operand, a wrong index), using closed forms, invariants, hand-deriv
 examples and special cases that reduce to a library routine. None of them re-types the
 oracle's formula and compares the oracle with itself.
 """
+import dataclasses
 import math
 
 import numpy as np
@@ -327,3 +328,94 @@ def test_layer_subset_matches_full_run():
     part = oracle.build_tokens(inp, np.array([4, 1]), layers=[3, 0])
     assert np.array_equal(part["k"][0, 0], full["k"][4, 3]) and np.array_equal(part["k"][1, 1], full["k"][1, 0])
     assert np.array_equal(part["v"][0, 1], full["v"][4, 0])
+
+
+# ---------------------------------------------------------------- recurrent adapter (Sec. 3.1 Eq. 6)
+
+def _silu_by_hand(u):
+    return u / (1.0 + math.exp(-u))
+
+
+def test_recurrent_two_layer_hand_example():
+    # E = [a, b, 0, 0]. Layer 1: D_1 reads channel 0, U_1 writes u * h_1 to channel 2, so
+    # M_1 = [a, b, u SiLU(a), 0]. Layer 2: D_2 reads channel 2 (zero in E, so only the chained
+    # state M_1 feeds it), U_2 writes w * h_2 to channel 3:
+    # M_2 = [a, b, u SiLU(a), w SiLU(u SiLU(a))].
+    a, b, u, w = 1.0, 2.0, 0.5, 2.0
+    cfg = _tiny_cfg(n_layers=2, rank=1, adapter="recurrent")
+    D = [[[1, 0, 0, 0]], [[0, 0, 1, 0]]]                           # [L][r][d]
+    U = [[[0], [0], [u], [0]], [[0], [0], [0], [w]]]               # [L][d][r]
+    eye = np.eye(4)
+    inp = _inputs(cfg, [[[a, b, 0, 0]]], D, U, [[1] * 4] * 2, [eye] * 2, [eye] * 2, [[[0]]])
+    out = oracle.build_tokens(inp, want=("m", "h"))
+    h1 = _silu_by_hand(a)
+    h2 = _silu_by_hand(u * h1)
+    np.testing.assert_allclose(out["h"][0, :, 0], [h1, h2], rtol=1e-15)
+    np.testing.assert_allclose(out["m"][0, 0], [a, b, u * h1, 0.0], rtol=1e-15, atol=0)
+    np.testing.assert_allclose(out["m"][0, 1], [a, b, u * h1, w * h2], rtol=1e-15, atol=0)
+
+
+def test_recurrent_single_layer_equals_embedding():
+    # With L = 1, M_1 = A_1(M_0) = A_1(E) for both variants (Eqs. 5 and 6).
+    cfg, inp = _random_inputs(n_vis=8, n_layers=1)
+    emb = oracle.build_tokens(inp, want=("k", "v", "m"))
+    inp_r = dataclasses.replace(inp, cfg=synth.config("tiny", n_vis=8, n_layers=1,
+                                                      adapter="recurrent"))
+    rec = oracle.build_tokens(inp_r, want=("k", "v", "m"))
+    for n in ("k", "v", "m"):
+        assert np.array_equal(emb[n], rec[n])
+
+
+def test_recurrent_zero_up_keeps_embeddings():
+    # U_l = 0 makes every A_l the identity, so M_l = E at every depth of the chain.
+    cfg = synth.config("tiny", zero_up=True, n_vis=16, adapter="recurrent")
+    inp = synth.make_inputs(cfg)
+    out = oracle.build_tokens(inp, want=("m",))
+    x = synth.bf16_to_f32(inp.x0).astype(np.float64).reshape(cfg.tokens, 1, cfg.d)
+    assert np.array_equal(out["m"], np.broadcast_to(x, out["m"].shape))
+
+
+def test_recurrent_frozen_after_first_layer_matches_embedding_of_first_adapter():
+    # U_l = 0 for l >= 2 freezes the chain at M_1 = A_1(E). The embedding variant with A_1
+    # copied into every layer also gives M_l = A_1(E), so K/V agree at every layer.
+    cfg = synth.config("tiny", n_vis=8, adapter="recurrent", w_sigma=0.1)
+    inp = synth.make_inputs(cfg)
+    inp.U[1:] = 0
+    rec = oracle.build_tokens(inp, want=("k", "v"))
+    emb_cfg = synth.config("tiny", n_vis=8, w_sigma=0.1)
+    D1 = np.broadcast_to(inp.D[0], inp.D.shape).copy()
+    U1 = np.broadcast_to(inp.U[0], inp.U.shape).copy()
+    emb = oracle.build_tokens(dataclasses.replace(inp, cfg=emb_cfg, D=D1, U=U1))
+    np.testing.assert_allclose(rec["k"], emb["k"], rtol=1e-12, atol=1e-14)
+    np.testing.assert_allclose(rec["v"], emb["v"], rtol=1e-12, atol=1e-14)
+
+
+def test_recurrent_updates_lie_in_each_layers_up_span():
+    # M_l - M_{l-1} = phi(M_{l-1} D_l) U_l: every token's step at layer l lies in the row space
+    # of U_l (r directions), and the accumulated change M_l - E spans at most l * r directions.
+    cfg = synth.config("tiny", n_vis=64, rank=4, adapter="recurrent", w_sigma=0.2, x0_sigma=1.0)
+    inp = synth.make_inputs(cfg)
+    out = oracle.build_tokens(inp, want=("m",))
+    x = synth.bf16_to_f32(inp.x0).astype(np.float64).reshape(cfg.tokens, cfg.d)
+    prev = x
+    for l in range(cfg.n_layers):
+        Ul = synth.bf16_to_f32(inp.U[l]).astype(np.float64)          # [d][r]
+        q, _ = np.linalg.qr(Ul)                                        # basis of its columns
+        step = out["m"][:, l] - prev
+        resid = step - (step @ q) @ q.T
+        assert np.abs(resid).max() <= 1e-12 * max(np.abs(step).max(), 1e-300)
+        assert np.abs(step).max() > 1e-6
+        s = np.linalg.svd(out["m"][:, l] - x, compute_uv=False)
+        if (l + 1) * cfg.rank < len(s):
+            assert s[(l + 1) * cfg.rank] < 1e-9 * s[0]
+        prev = out["m"][:, l]
+
+
+def test_recurrent_layer_subset_matches_full_run():
+    # Selected layers still see the whole chain before them.
+    cfg = synth.config("tiny", n_vis=6, adapter="recurrent")
+    inp = synth.make_inputs(cfg)
+    full = oracle.build_tokens(inp)
+    part = oracle.build_tokens(inp, np.array([4, 1]), layers=[3, 1])
+    assert np.array_equal(part["k"][0, 0], full["k"][4, 3]) and np.array_equal(part["k"][1, 1], full["k"][1, 1])
+    assert np.array_equal(part["v"][0, 1], full["v"][4, 1])
