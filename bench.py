@@ -161,6 +161,19 @@ def time_oracle_sample(inp, budget_s: float, seed: int = 0):
                       f"{cfg.name} workload, fp64, {dt:.1f} s"}
 
 
+def workload_config(args):
+    """The synthetic workload of --config, with --layers and --adapter applied."""
+    from dataclasses import replace
+    import synth
+    cfg = synth.CONFIGS[args.config]
+    if args.layers:
+        cfg = replace(cfg, n_layers=args.layers, name=f"{cfg.name}_L{args.layers}")
+    if args.adapter == "recurrent":
+        cfg = replace(cfg, adapter="recurrent", name=f"{cfg.name}_recurrent",
+                      description=cfg.description + "; recurrent adapter (Sec. 3.1 Eq. 6)")
+    return cfg
+
+
 def run_reference(args):
     """The oracle as the reference arm: every step is a bounded sample of (token, layer) pairs."""
     import numpy as np
@@ -169,12 +182,14 @@ def run_reference(args):
     rank, world, _ = dist_env()
     if rank != 0:
         return
-    cfg = synth.CONFIGS[args.config]
+    cfg = workload_config(args)
     inp = synth.make_inputs(cfg)
     rng = np.random.default_rng(0)
+    # The recurrent chain of a layer needs every layer before it: evaluate whole tokens.
+    whole = cfg.adapter == "recurrent"
     t0 = time.perf_counter()
-    oracle.build_tokens(inp, np.array([0], dtype=np.int64), layers=[0])
-    t_pair = max(time.perf_counter() - t0, 1e-4)
+    oracle.build_tokens(inp, np.array([0], dtype=np.int64), layers=None if whole else [0])
+    t_pair = max(time.perf_counter() - t0, 1e-4) / (cfg.n_layers if whole else 1)
     n_steps = args.warmup + args.steps
     cores = oracle.num_threads()
     # one random layer per step, evaluated for per_step random tokens (parallel over tokens)
@@ -182,13 +197,15 @@ def run_reference(args):
     total_t, total_pairs = 0.0, 0
     for step in range(n_steps):
         toks = np.sort(rng.choice(cfg.tokens, size=per_step, replace=False)).astype(np.int64)
-        lay = [int(rng.integers(0, cfg.n_layers))]
+        if whole:
+            toks = toks[:max(1, per_step // cfg.n_layers)]
+        lay = None if whole else [int(rng.integers(0, cfg.n_layers))]
         t0 = time.perf_counter()
         oracle.build_tokens(inp, toks, layers=lay)
         dt = time.perf_counter() - t0
         if step >= args.warmup:
             total_t += dt
-            total_pairs += per_step
+            total_pairs += len(toks) * (cfg.n_layers if whole else 1)
     value = (total_pairs / cfg.n_layers) / total_t
     out = {
         "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world,
@@ -196,11 +213,14 @@ def run_reference(args):
         "ms_per_step": 1000.0 * total_t / args.steps, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
         "config": {"workload": cfg.name, "description": cfg.description,
-                   "sample_per_step": f"{per_step} tokens x 1 random layer"},
+                   "sample_per_step": (f"{max(1, per_step // cfg.n_layers)} tokens x all layers"
+                                       if whole else f"{per_step} tokens x 1 random layer")},
         "cpu_baseline": {"value": value, "unit": UNIT, "cores": oracle.num_threads(), "kind": "oracle",
-                         "sample": f"{per_step} random tokens at one random layer per step of the "
-                                   f"{cfg.name} workload; tokens/s = (token, layer) pairs/s / "
-                                   f"{cfg.n_layers} layers"},
+                         "sample": (f"{max(1, per_step // cfg.n_layers)} random whole tokens per "
+                                    f"step of the {cfg.name} workload" if whole else
+                                    f"{per_step} random tokens at one random layer per step of the "
+                                    f"{cfg.name} workload; tokens/s = (token, layer) pairs/s / "
+                                    f"{cfg.n_layers} layers")},
         "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }
     print(json.dumps(out), flush=True)
@@ -222,10 +242,7 @@ def run_dv(args):
         dist = tdist
     torch.cuda.set_device(local)
     dev = torch.device("cuda", local)
-    cfg = synth.CONFIGS[args.config]
-    if args.layers:
-        from dataclasses import replace
-        cfg = replace(cfg, n_layers=args.layers, name=f"{args.config}_L{args.layers}")
+    cfg = workload_config(args)
     peaks, peak_src = load_peaks()
     modes = None
     layers_built = cfg.n_layers
@@ -357,14 +374,14 @@ def run_dv(args):
             "gpu_launches": args.steps * dv.kernels_per_build(plan),
             "roofline": {"bound": "tensor", "achieved": achieved_tf, "peak": peak_tf,
                          "unit": "TFLOP/s", "frac": achieved_tf / peak_tf, "traffic": traffic,
-                         "kernel": "dv_kv_pair_kernel (K/V projection + RoPE + cache store, 2-SM UMMA)",
+                         "kernel": dv.kv_kernel(plan, cfg.tokens) + ": K/V projection + RoPE + cache store",
                          "peak_source": f"bf16_tflops (burst) of {peak_src}",
                          "flops_per_launch": kv_flops, "ms_per_launch": kv_ms},
             "roofline_step": {"t_roof_ms": t_roof_ms, "frac": t_roof_ms / ms_step,
                               "frac_sustained": max(work.flops() / (peaks["bf16_tflops_sustained"] * 1e12),
                                                     work.min_bytes() / (peaks["hbm_gbs"] * 1e9)) * 1e3 / ms_step,
                               "plain_flops": work.flops(), "min_bytes": work.min_bytes()},
-            "stage_ms_per_step": dict(zip(dv.STAGE_NAMES, [s / max(n_timed, 1) for s in stage_ms])),
+            "stage_ms_per_step": dict(zip(dv.stage_names(plan), [s / max(n_timed, 1) for s in stage_ms])),
             "cpu_baseline": cpu,
         }
         print(json.dumps(out), flush=True)
@@ -384,6 +401,9 @@ def main():
     ap.add_argument("--skip-layers", default="",
                     help="F,K: no visual memory at the first F and last K layers (App. J adapter "
                          "skipping, DV_LAYER_DROP)")
+    ap.add_argument("--adapter", choices=["embedding", "recurrent"], default="embedding",
+                    help="embedding adapter (Sec. 3.1 Eq. 5, the default workload) or the "
+                         "recurrent adapter (Eq. 6)")
     ap.add_argument("--impl", choices=["dv", "reference"], default="dv")
     ap.add_argument("--e2e-steps", type=int, default=100)
     ap.add_argument("--no-cpu-baseline", action="store_true")

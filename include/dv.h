@@ -5,6 +5,8 @@
  * The library builds, for every visual token and every layer l, the key/value cache entries
  * that text tokens read:
  *     M_l = E + SiLU(E D_l) U_l                 (Sec. 3.1, Eqs. 4-5: embedding adapter)
+ *  or M_0 = E, M_l = M_{l-1} + SiLU(M_{l-1} D_l) U_l
+ *                                               (Sec. 3.1, Eq. 6: recurrent adapter)
  *     K_l = RoPE(W_K,l RMSNorm_l(M_l) [+ b_K,l]),  V_l = W_V,l RMSNorm_l(M_l) [+ b_V,l]
  *                                               (Sec. 3.2, Eq. 7; RMSNorm per App. K; RoPE
  *                                                at the original visual positions)
@@ -46,6 +48,11 @@ enum {
   DV_LAYER_DROP = 2       /* adapter and visual memory skipped: no K/V entries for this layer */
 };
 enum { DV_ROPE_1D = 0, DV_ROPE_MROPE = 1 };
+/* How M_l is formed from the visual embeddings E (Sec. 3.1). */
+enum {
+  DV_ADAPTER_EMBEDDING = 0,  /* M_l = A_l(E) for every layer (Eq. 5) */
+  DV_ADAPTER_RECURRENT = 1   /* M_0 = E, M_l = A_l(M_{l-1}) through the planned layers (Eq. 6) */
+};
 
 /* Model shape and build limits. Supported (else DV_ERR_UNSUPPORTED_SHAPE):
  *   d % 64 == 0, 64 <= d <= 16384;  1 <= rank <= 256;  head_dim in {64, 128};
@@ -54,6 +61,7 @@ enum { DV_ROPE_1D = 0, DV_ROPE_MROPE = 1 };
  *   act == DV_ACT_SILU;  rope_theta > 0;  rms_eps >= 0;
  *   DV_ROPE_MROPE: mrope_section[i] >= 0 and their sum == head_dim / 2 (contiguous sections
  *   of the frequency index: t first, then h, then w);
+ *   adapter in {DV_ADAPTER_EMBEDDING, DV_ADAPTER_RECURRENT};
  *   max_batch * max_n_vis >= 1 and <= 2^24 (the tokens one build may carry). */
 typedef struct dv_config {
   int d;                 /* hidden size of the language model */
@@ -69,6 +77,7 @@ typedef struct dv_config {
   int max_batch;         /* largest batch a build may pass */
   int max_n_vis;         /* largest number of visual tokens per batch element */
   int has_kv_bias;       /* 1: weights carry b_K, b_V; 0: no bias */
+  int adapter;           /* DV_ADAPTER_EMBEDDING or DV_ADAPTER_RECURRENT */
 } dv_config;
 
 /* Weights of all L layers, bf16, device pointers. Read only during dv_memory_plan: the plan
@@ -82,7 +91,9 @@ typedef struct dv_config {
  *                       layer (App. J skips the adapters of early and late layers). Layers in
  *                       DV_LAYER_DROP get no K/V entries: builds leave their cache rows untouched,
  *                       and the plan keeps neither repacked weights nor workspace for them.
- *                       At least one layer must not be DV_LAYER_DROP. */
+ *                       At least one layer must not be DV_LAYER_DROP. With the recurrent
+ *                       adapter a skipped layer passes its input state on unchanged
+ *                       (M_l = M_{l-1}), whether it is DV_LAYER_IDENTITY or DV_LAYER_DROP. */
 typedef struct dv_weights {
   const void* D;
   const void* U;
@@ -111,10 +122,11 @@ typedef struct dv_plan dv_plan;
 
 /*
  * dv_memory_plan — validate the configuration, allocate the plan and its workspace on the
- * current device, and repack the weights for the build kernels (all L down-projections
- * stacked into one matrix, since every layer reads only E: Sec. 3.1 "conditionally
- * independent across layers given E"; RMSNorm gain and the rank-r update folded into
- * the K/V weights).
+ * current device, and repack the weights for the build kernels. Embedding adapter: all L
+ * down-projections stacked into one matrix, since every layer reads only E (Sec. 3.1: the
+ * memories are conditionally independent across layers given E), and the RMSNorm gain and
+ * the rank-r update folded into the K/V weights. Recurrent adapter: per-layer down- and
+ * up-projections, and the RMSNorm gain folded into the K/V weights.
  *   cfg     shape and limits (copied)
  *   w       device weights (read on `stream` before this call returns; not retained)
  *   stream  cudaStream_t as void*; the repack kernels run on it and this call waits for them
@@ -126,7 +138,9 @@ int dv_memory_plan(const dv_config* cfg, const dv_weights* w, void* stream, dv_p
 
 /*
  * dv_build_visual_memory — the hot path. For batch*n_vis visual tokens writes K^v_l and V^v_l
- * of every layer (Sec. 3.1 Eqs. 4-5, Sec. 3.2 Eq. 7) into the cache.
+ * of every layer (Sec. 3.1 Eqs. 4-6, Sec. 3.2 Eq. 7) into the cache. With the recurrent
+ * adapter the state M_l is carried in fp32 from layer to layer; each layer's K/V read its
+ * bf16 rounding.
  *   x0     bf16 [batch][n_vis][d]: the visual embeddings E (Sec. 2 Eq. 1); 16-byte aligned
  *   pos    int32 [batch][P][n_vis], P = 1 (DV_ROPE_1D) or 3 (DV_ROPE_MROPE: t, h, w): the
  *          original positions of the visual tokens (Sec. 1 and App. H keep them unchanged)
@@ -154,8 +168,10 @@ int dv_build_visual_memory(dv_plan* plan, const void* x0, int batch, int n_vis, 
  *     loading this library holds until the process exits. The plan's own workspace is not
  *     used, so its max_batch / max_n_vis do not bound this call.
  *   - Limit: batch * n_vis * (n_layers * r_pad * 2 + n_layers * 4 + 4) bytes (each part
- *     rounded up to 256 bytes, r_pad = rank rounded up to 64) must fit in 32 MiB; larger
- *     builds return DV_ERR_UNSUPPORTED_SHAPE and launch nothing.
+ *     rounded up to 256 bytes, r_pad = rank rounded up to 64, n_layers counting the planned
+ *     layers) must fit in 32 MiB; the recurrent adapter adds batch * n_vis * (4 d +
+ *     n_layers * (2 d + 4 d / 64)) bytes (fp32 state, bf16 M_l of every layer, partial sums
+ *     of squares). Larger builds return DV_ERR_UNSUPPORTED_SHAPE and launch nothing.
  *   - The first call on a device looks up the array's device address with that device current;
  *     make that first call before any stream capture.
  *   - All calls on a device share the array and find it as the last call left it (nothing in
@@ -188,13 +204,22 @@ const char* dv_error_string(int status);
  *   dv_timing_read(plan, ms, n_stages, n_builds) synchronises on the recorded events and
  *   writes the summed milliseconds of each stage into ms[0..n_stages-1] (stage order:
  *   0 row sums of squares of E, 1 stacked down-projection + SiLU, 2 RMS statistics,
- *   3 K/V projection + RoPE + cache store) and the number of builds into *n_builds.
+ *   3 K/V projection + RoPE + cache store; recurrent adapter: 0 empty, 1 the adapter chain
+ *   through all layers, 2 RMS statistics from the chain's partial sums, 3 as above) and the
+ *   number of builds into *n_builds.
  */
 int dv_timing_enable(dv_plan* plan, int on);
 int dv_timing_read(dv_plan* plan, double* ms, int n_stages, int* n_builds);
 
 /* Number of kernels one build launches (for launch accounting). */
 int dv_kernels_per_build(const dv_plan* plan);
+
+/* Which kernel computes K/V (Sec. 3.2 Eq. 7) in a build of `tokens` tokens, for reporting:
+ * DV_KV_ENGINE_WEIGHTS_AS_M (weight rows as the MMA's M, tokens as N: dv_kv_pair_kernel) or
+ * DV_KV_ENGINE_TOKENS_AS_M (256-token blocks as M: dv_pair_tm_kernel); 0 for a NULL plan or
+ * tokens <= 0. */
+enum { DV_KV_ENGINE_WEIGHTS_AS_M = 1, DV_KV_ENGINE_TOKENS_AS_M = 2 };
+int dv_kv_engine(const dv_plan* plan, long long tokens);
 
 /*
  * dv_debug_wait_timeout — failure-detection self-test. Launches one kernel whose single
@@ -208,16 +233,27 @@ int dv_debug_wait_timeout(dv_plan* plan, int timeout_us, void* stream);
 /*
  * dv_debug_copy_workspace — copies the intermediate results of the last build on this plan
  * into caller-owned device buffers (stream-ordered), for stage-wise testing:
- *   H     bf16 [tokens][n_planned * r_pad]  SiLU(E D_l) of every planned layer, r_pad = rank
- *         rounded up to 64 (columns past rank are zero)
+ *   H     bf16 [tokens][n_planned * r_pad]  SiLU(E D_l) (recurrent: SiLU(M_{l-1} D_l)) of
+ *         every planned layer, r_pad = rank rounded up to 64 (columns past rank are zero)
  *   rstd  fp32 [n_planned][tokens]           1 / sqrt(mean(M_l^2) + eps)
- *   xx    fp32 [tokens]                     sum of squares of each row of E
+ *   xx    fp32 [tokens]                     sum of squares of each row of E (embedding
+ *         adapter only; not written by recurrent builds)
  * n_planned is the number of layers whose mode is not DV_LAYER_DROP (n_layers when the plan
- * was made without layer modes); planned layers appear in layer order. Any of the three may be NULL. tokens must not exceed the plan's limit; *r_pad_out (if not
- * NULL) receives r_pad.
+ * was made without layer modes); planned layers appear in layer order. Any of the three may
+ * be NULL. tokens must not exceed the last build's token count; *r_pad_out (if not NULL)
+ * receives r_pad.
  */
 int dv_debug_copy_workspace(dv_plan* plan, int tokens, void* H, void* rstd, void* xx,
                             int* r_pad_out, void* stream);
+
+/*
+ * dv_debug_copy_memory — recurrent adapter only: copies bf16 M_l of every planned layer of the
+ * last build, [n_planned][tokens][d], into a caller-owned device buffer (stream-ordered), for
+ * stage-wise testing of the chain M_l = M_{l-1} + SiLU(M_{l-1} D_l) U_l (Sec. 3.1 Eq. 6).
+ * tokens must not exceed the last build's token count. DV_ERR_INVALID_ARG for a plan with the
+ * embedding adapter (it never forms M_l).
+ */
+int dv_debug_copy_memory(dv_plan* plan, int tokens, void* mem, void* stream);
 
 #ifdef __cplusplus
 }

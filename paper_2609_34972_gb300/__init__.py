@@ -36,12 +36,17 @@ DV_ROPE_MROPE = 1
 DV_LAYER_ADAPTER = 0
 DV_LAYER_IDENTITY = 1
 DV_LAYER_DROP = 2
+DV_ADAPTER_EMBEDDING = 0
+DV_ADAPTER_RECURRENT = 1
 
 EXPORTED = ["dv_memory_plan", "dv_build_visual_memory", "dv_plan_status", "dv_free",
             "dv_error_string", "dv_timing_enable", "dv_timing_read", "dv_kernels_per_build",
-            "dv_debug_wait_timeout", "dv_debug_copy_workspace", "dv_build_visual_memory_noalloc"]
+            "dv_debug_wait_timeout", "dv_debug_copy_workspace", "dv_build_visual_memory_noalloc",
+            "dv_debug_copy_memory", "dv_kv_engine"]
 N_STAGES = 4
 STAGE_NAMES = ["row_sumsq", "down_proj_silu", "rms_stats", "kv_proj_rope_store"]
+# Stage names of a recurrent-adapter build (stage 0 is empty there).
+STAGE_NAMES_RECURRENT = ["none", "adapter_chain", "rms_stats", "kv_proj_rope_store"]
 
 
 class DvConfig(ctypes.Structure):
@@ -50,7 +55,7 @@ class DvConfig(ctypes.Structure):
                 ("rope", ctypes.c_int), ("rope_theta", ctypes.c_float),
                 ("mrope_section", ctypes.c_int * 3), ("rms_eps", ctypes.c_float),
                 ("max_batch", ctypes.c_int), ("max_n_vis", ctypes.c_int),
-                ("has_kv_bias", ctypes.c_int)]
+                ("has_kv_bias", ctypes.c_int), ("adapter", ctypes.c_int)]
 
 
 class DvWeights(ctypes.Structure):
@@ -93,10 +98,12 @@ def lib() -> ctypes.CDLL:
         L.dv_debug_copy_workspace.argtypes = [vp, i32, vp, vp, vp, ctypes.POINTER(i32), vp]
         L.dv_build_visual_memory_noalloc.argtypes = [vp, vp, i32, i32, vp, vp, i32,
                                                      ctypes.POINTER(DvKVCache), vp]
+        L.dv_debug_copy_memory.argtypes = [vp, i32, vp, vp]
+        L.dv_kv_engine.argtypes = [vp, ctypes.c_longlong]
         for name in ("dv_memory_plan", "dv_build_visual_memory", "dv_plan_status",
                      "dv_timing_enable", "dv_timing_read", "dv_kernels_per_build",
                      "dv_debug_wait_timeout", "dv_debug_copy_workspace",
-                     "dv_build_visual_memory_noalloc"):
+                     "dv_build_visual_memory_noalloc", "dv_debug_copy_memory", "dv_kv_engine"):
             getattr(L, name).restype = i32
         _lib = L
     return _lib
@@ -130,11 +137,16 @@ def _ptr(t):
 
 def make_config(d, n_layers, n_kv_heads, head_dim, rank, rope="1d", rope_theta=10000.0,
                 mrope_section=(0, 0, 0), rms_eps=1e-6, max_batch=1, max_n_vis=1,
-                has_kv_bias=False) -> DvConfig:
+                has_kv_bias=False, adapter="embedding") -> DvConfig:
+    """``adapter``: "embedding" (M_l = A_l(E), Sec. 3.1 Eq. 5) or "recurrent"
+    (M_l = A_l(M_{l-1}), Sec. 3.1 Eq. 6)."""
+    if adapter not in ("embedding", "recurrent"):
+        raise ValueError(f"unknown adapter {adapter!r}")
     return DvConfig(int(d), int(n_layers), int(n_kv_heads), int(head_dim), int(rank),
                     DV_ACT_SILU, DV_ROPE_MROPE if rope == "mrope" else DV_ROPE_1D,
                     float(rope_theta), (ctypes.c_int * 3)(*mrope_section), float(rms_eps),
-                    int(max_batch), int(max_n_vis), int(bool(has_kv_bias)))
+                    int(max_batch), int(max_n_vis), int(bool(has_kv_bias)),
+                    DV_ADAPTER_RECURRENT if adapter == "recurrent" else DV_ADAPTER_EMBEDDING)
 
 
 class Plan:
@@ -253,6 +265,29 @@ def debug_workspace(plan: Plan, tokens: int, stream=None):
     _check(lib().dv_debug_copy_workspace(plan.handle, int(tokens), _ptr(H), _ptr(rstd), _ptr(xx),
                                          None, _stream_handle(stream)), "dv_debug_copy_workspace")
     return H, rstd, xx, r_pad.value
+
+
+def debug_memory(plan: Plan, tokens: int, stream=None):
+    """bf16 M_l of every planned layer of the last (recurrent) build: [L_planned, tokens, d]."""
+    import torch
+    mem = torch.empty((len(plan.layers), tokens, plan.cfg.d), dtype=torch.bfloat16, device="cuda")
+    _check(lib().dv_debug_copy_memory(plan.handle, int(tokens), _ptr(mem), _stream_handle(stream)),
+           "dv_debug_copy_memory")
+    return mem
+
+
+KV_KERNELS = {1: "dv_kv_pair_kernel (weights as M, 2-SM UMMA)",
+              2: "dv_pair_tm_kernel<EPI_KV> (256-token blocks as M, 2-SM UMMA)"}
+
+
+def kv_kernel(plan: Plan, tokens: int) -> str:
+    """Name of the kernel that computes K/V in a build of ``tokens`` tokens."""
+    return KV_KERNELS.get(int(lib().dv_kv_engine(plan.handle, int(tokens))), "none")
+
+
+def stage_names(plan: Plan):
+    """Names of the four timed stages of a build with this plan."""
+    return STAGE_NAMES_RECURRENT if plan.cfg.adapter == DV_ADAPTER_RECURRENT else STAGE_NAMES
 
 
 class HostPipeline:

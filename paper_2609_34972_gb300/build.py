@@ -1,6 +1,6 @@
 """Builds ``libdv.so`` (the C-ABI library of ``include/dv.h``) in-tree for sm_103a.
 
-Two translation units are compiled in parallel with nvcc and linked into one shared library
+The translation units are compiled in parallel with nvcc and linked into one shared library
 next to this file. No torch extension machinery is involved: the library has a plain C ABI.
 """
 from __future__ import annotations
@@ -13,7 +13,7 @@ HERE = os.path.dirname(os.path.abspath(__file__))
 ROOT = os.path.dirname(HERE)
 CSRC = os.path.join(HERE, "csrc")
 LIB_PATH = os.path.join(HERE, "libdv.so")
-SOURCES = ["dv_api.cu", "dv_gemm.cu", "dv_kv2sm.cu", "dv_pair_tm.cu", "dv_noalloc.cu"]
+SOURCES = ["dv_api.cu", "dv_gemm.cu", "dv_kv2sm.cu", "dv_pair_tm.cu", "dv_recurrent.cu", "dv_noalloc.cu"]
 HEADERS = ["dv_internal.h", "dv_ptx.cuh", "dv_epilogue.cuh"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 NVCC_FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-Xptxas", "-v"]

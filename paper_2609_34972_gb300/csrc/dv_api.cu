@@ -34,15 +34,17 @@ struct dv_plan {
   uint16_t* Dst = nullptr;
   uint16_t* Bn = nullptr;
   uint16_t* Wkv = nullptr;
+  uint16_t* Uup = nullptr;     // recurrent adapter: U_l as [L*d][r_pad]
   float* bk = nullptr;
   float* bv = nullptr;
-  uint16_t* H = nullptr;
-  float* xx = nullptr;
-  float* rstd = nullptr;
+  void* ws = nullptr;          // workspace of a build of max_tokens tokens (carve_workspace)
+  long long last_tokens = 0;   // tokens of the last build (layout of the workspace)
   int* status = nullptr;
   CUtensorMap tm_Dst[3];       // boxes of 64, 128, 256 rows
   CUtensorMap tm_Dst_half[3];  // boxes of 32, 64, 128 rows (halves for CTA pairs)
   CUtensorMap tm_Bn, tm_Bn_half, tm_Wkv;
+  CUtensorMap tm_Dst_rp, tm_Uup;  // recurrent adapter
+  int resid_bn = 0;
   double inv_freq[dv::kMaxHalfHead];
   unsigned char mode[dv::kMaxLayers];  // DV_LAYER_* per layer
   int n_active = 0;                    // layers not dropped
@@ -266,6 +268,35 @@ __global__ void k_bias_to_f32(const uint16_t* __restrict__ b, float* __restrict_
     out[e] = bf(b[static_cast<long long>(pl.src[e / kv]) * kv + e % kv]);
 }
 
+// Uup[i*d + j][n] = U[src[i]][j][n] for n < r, else 0: the up-projection of the recurrent
+// adapter as a K-major B operand (rows = output channels j, K = bottleneck n).
+__global__ void k_pack_up(const uint16_t* __restrict__ U, uint16_t* __restrict__ Uup, int L, int r,
+                          int r_pad, int d, PackLayers pl) {
+  const long long total = static_cast<long long>(L) * d * r_pad;
+  for (long long e = blockIdx.x * static_cast<long long>(blockDim.x) + threadIdx.x; e < total;
+       e += static_cast<long long>(gridDim.x) * blockDim.x) {
+    const int n = static_cast<int>(e % r_pad);
+    const long long row = e / r_pad;
+    const int j = static_cast<int>(row % d), i = static_cast<int>(row / d);
+    Uup[e] = (n < r && !pl.zero_du[i]) ? U[(static_cast<long long>(pl.src[i]) * d + j) * r + n] : 0;
+  }
+}
+
+// rstd[i][t] = 1 / sqrt(sum_n part[i][n][t] / d + eps), the partial sums of squares of the
+// recurrent state M_i summed in column-tile order (n < n_parts; layer stride ld_part).
+__global__ void k_rstd_parts(const float* __restrict__ part, int L, long long T, int n_parts,
+                             long long ld_part, float inv_d, float eps, float* __restrict__ rstd) {
+  const long long total = static_cast<long long>(L) * T;
+  for (long long e = blockIdx.x * static_cast<long long>(blockDim.x) + threadIdx.x; e < total;
+       e += static_cast<long long>(gridDim.x) * blockDim.x) {
+    const long long i = e / T, t = e % T;
+    const float* pp = part + i * ld_part + t;
+    float ss = 0.0f;
+    for (int n = 0; n < n_parts; ++n) ss += pp[static_cast<long long>(n) * T];
+    rstd[e] = rsqrtf(fmaf(ss, inv_d, eps));
+  }
+}
+
 // xx[t] = sum_j x0[t][j]^2 (fp32), one warp per token row, 16-byte loads.
 __global__ void k_row_sumsq(const uint16_t* __restrict__ x0, int T, int d, float* __restrict__ xx) {
   const int warp = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
@@ -322,6 +353,8 @@ int check_config(const dv_config* c) {
       !std::isfinite(c->rms_eps))
     return DV_ERR_INVALID_ARG;
   if (c->has_kv_bias != 0 && c->has_kv_bias != 1) return DV_ERR_INVALID_ARG;
+  if (c->adapter != DV_ADAPTER_EMBEDDING && c->adapter != DV_ADAPTER_RECURRENT)
+    return DV_ERR_INVALID_ARG;
   if (c->d % 64 != 0 || c->d > 16384) return DV_ERR_UNSUPPORTED_SHAPE;
   if (c->rank > 256) return DV_ERR_UNSUPPORTED_SHAPE;
   if (c->head_dim != 64 && c->head_dim != 128) return DV_ERR_UNSUPPORTED_SHAPE;
@@ -338,7 +371,7 @@ int check_config(const dv_config* c) {
 }
 
 void free_plan_memory(dv_plan* p) {
-  void* ptrs[] = {p->Dst, p->Bn, p->Wkv, p->bk, p->bv, p->H, p->xx, p->rstd, p->status};
+  void* ptrs[] = {p->Dst, p->Bn, p->Wkv, p->Uup, p->bk, p->bv, p->ws, p->status};
   for (void* q : ptrs)
     if (q) cudaFree(q);
   for (cudaEvent_t e : p->ev) cudaEventDestroy(e);
@@ -402,25 +435,143 @@ static void tm_groups(GemmShape& s, int block_n, long long tokens) {
   s.group_w = static_cast<int>(gw < 1 ? 1 : (gw > w_tiles ? w_tiles : gw));
 }
 
-cudaError_t enqueue_build(const PlanView& v, const BuildArgs& a, cudaStream_t st) {
+// Epilogue constants of the K/V stage: biases, positions, cache, RoPE frequencies.
+static void fill_epi_kv(const PlanView& v, const BuildArgs& a, long long T, EpiKV& e) {
+  const int HD = v.head_dim;
+  e.rstd = a.rstd;
+  e.ld_rstd = static_cast<int>(T);
+  e.bk = v.bk;
+  e.bv = v.bv;
+  e.kv = v.kv;
+  e.pos = a.pos;
+  e.slot = a.slot;
+  e.slot0 = a.slot0;
+  e.n_vis = a.n_vis;
+  e.n_pos = v.rope == DV_ROPE_MROPE ? 3 : 1;
+  e.sec0 = v.rope == DV_ROPE_MROPE ? v.mrope_section[0] : HD / 2;
+  e.sec01 = v.rope == DV_ROPE_MROPE ? v.mrope_section[0] + v.mrope_section[1] : HD / 2;
+  e.kc = static_cast<uint16_t*>(const_cast<void*>(a.kc));
+  e.vc = static_cast<uint16_t*>(const_cast<void*>(a.vc));
+  e.s_layer = a.s_layer;
+  e.s_batch = a.s_batch;
+  e.s_seq = a.s_seq;
+  e.s_head = a.s_head;
+  const double two_pi = 6.283185307179586476925286766559;
+  e.two_pi_hi = static_cast<float>(two_pi);
+  e.two_pi_lo = static_cast<float>(two_pi - static_cast<double>(e.two_pi_hi));
+  e.inv_two_pi = static_cast<float>(1.0 / two_pi);
+  for (int j = 0; j < HD / 2; ++j) {
+    e.inv_freq_hi[j] = static_cast<float>(v.inv_freq[j]);
+    e.inv_freq_lo[j] = static_cast<float>(v.inv_freq[j] - static_cast<double>(e.inv_freq_hi[j]));
+  }
+}
+
+// K/V stage over all planned layers: K/V = rstd_l * (A_l [| h_l] Wkv_l^T) + b, RoPE on K,
+// stored into the cache. gp.s holds the operand schedule; the engine is chosen by token count
+// (tokens-as-M pairs when 256-token blocks pad little, else weights-as-M pairs). a_full /
+// h_full: token operands with 128-row boxes; a_half / h_half: with nt / 2-row boxes.
+static cudaError_t launch_kv_stage(const PlanView& v, GemmParams& gp, long long T,
+                                   const void* a_ptr, uint64_t a_rows, const CUtensorMap& a_full,
+                                   const void* h_ptr, uint64_t h_cols, const CUtensorMap& h_full,
+                                   cudaStream_t st) {
+  const int nt = kv_pair_tile_n(T);
+  const long long pad256 = (T + 255) / 256 * 256, pad_nt = (T + nt - 1) / nt * nt;
+  if (prefer_256(pad256, pad_nt)) {
+    tm_groups(gp.s, 256, T);
+    return launch_pair_tm(EPI_KV, 256, v.head_dim, a_full, h_full, *v.tm_Wkv, gp, v.num_sms, st);
+  }
+  CUtensorMap a_half, h_half;
+  if (!encode_2d(&a_half, a_ptr, v.d, a_rows, v.d, nt / 2)) return cudaErrorInvalidValue;
+  if (h_ptr && !encode_2d(&h_half, h_ptr, h_cols, static_cast<uint64_t>(T), h_cols, nt / 2))
+    return cudaErrorInvalidValue;
+  return launch_kv_pair(v.head_dim, nt, *v.tm_Wkv, a_half, h_ptr ? h_half : a_half, gp, v.num_sms,
+                        st);
+}
+
+// Recurrent adapter (Sec. 3.1 Eq. 6): the chain M_i = M_{i-1} + SiLU(M_{i-1} D_i) U_i runs
+// layer by layer (a split-K down-projection, then the up-projection whose epilogue adds the
+// fp32 state and writes bf16 M_i and partial sums of squares); the RMS statistics of all
+// layers follow in one kernel, and one K/V launch covers every layer, reading M_i as A.
+static cudaError_t enqueue_recurrent(const PlanView& v, const BuildArgs& a, cudaStream_t st) {
   const long long T = static_cast<long long>(a.batch) * a.n_vis;
-  const int L = v.n_layers, d = v.d, HD = v.head_dim;
+  const int L = v.n_layers, d = v.d;
+  const long long n1 = static_cast<long long>(L) * v.r_pad;
+  auto mark = [&](int i) {
+    if (a.marks) cudaEventRecord(a.marks[i], st);
+  };
+  CUtensorMap tm_x0, tm_mem, tm_H;
+  if (!encode_2d(&tm_x0, a.x0, d, static_cast<uint64_t>(T), d, kBlockM) ||
+      !encode_2d(&tm_mem, a.mem, d, static_cast<uint64_t>(L) * T, d, kBlockM) ||
+      !encode_2d(&tm_H, a.H, n1, static_cast<uint64_t>(T), n1, kBlockM))
+    return cudaErrorInvalidValue;
+
+  mark(0);
+  mark(1);
+  const long long m_tiles = (T + kBlockM - 1) / kBlockM;
+  const int splits = down_splits(m_tiles, d / kBlockK, v.num_sms);
+  DownParams dp;
+  dp.M = static_cast<int>(T);
+  dp.k_slabs = d / kBlockK;
+  dp.H = a.H;
+  dp.ldh = static_cast<int>(n1);
+  dp.status = v.status;
+  dp.timeout_ns = kTimeoutNs;
+
+  GemmParams gp;
+  std::memset(&gp, 0, sizeof(gp));
+  gp.status = v.status;
+  gp.timeout_ns = kTimeoutNs;
+  // up-projection step: A = h_i (H columns from i * r_pad), B = U_i ([d][r_pad] rows i * d)
+  gp.s = {static_cast<int>(T), 1, d, 0, v.r_pad / 64, v.r_pad, 0, 0, 0, 0};
+  const long long part_ld = static_cast<long long>(d / 64) * T;
+  cudaError_t err = cudaSuccess;
+  for (int i = 0; i < L && err == cudaSuccess; ++i) {
+    dp.a_row0 = i == 0 ? 0 : static_cast<int>((i - 1) * T);
+    dp.b_row0 = i * v.r_pad;
+    dp.h_col0 = i * v.r_pad;
+    err = launch_down_split(v.r_pad, splits, i == 0 ? tm_x0 : tm_mem, *v.tm_Dst_rp, dp, st);
+    if (err != cudaSuccess) break;
+    gp.s.layer0 = i;
+    gp.resid = {static_cast<const uint16_t*>(a.x0), a.state,
+                a.mem + static_cast<size_t>(i) * T * d, a.part + static_cast<size_t>(i) * part_ld,
+                d, i == 0 ? 1 : 0};
+    err = launch_gemm(EPI_RESID, v.resid_bn, 0, tm_H, tm_H, *v.tm_Uup, gp, v.num_sms, st);
+  }
+  mark(2);
+  if (err == cudaSuccess) {
+    k_rstd_parts<<<grid_for(static_cast<long long>(L) * T), 256, 0, st>>>(
+        a.part, L, T, d / v.resid_bn, part_ld, 1.0f / d, v.rms_eps, a.rstd);
+    err = cudaGetLastError();
+  }
+  mark(3);
+
+  std::memset(&gp, 0, sizeof(gp));
+  gp.status = v.status;
+  gp.timeout_ns = kTimeoutNs;
+  for (int i = 0; i < L; ++i) gp.layer_map[i] = v.active[i];
+  gp.s = {static_cast<int>(T), L, 2 * v.kv, d / 64, 0, 0, 0, 0, 0, static_cast<int>(T)};
+  fill_epi_kv(v, a, T, gp.kv);
+  if (err == cudaSuccess)
+    err = launch_kv_stage(v, gp, T, a.mem, static_cast<uint64_t>(L) * T, tm_mem, nullptr, 0,
+                          tm_mem, st);
+  mark(4);
+  return err;
+}
+
+cudaError_t enqueue_build(const PlanView& v, const BuildArgs& a, cudaStream_t st) {
+  if (v.adapter == DV_ADAPTER_RECURRENT) return enqueue_recurrent(v, a, st);
+  const long long T = static_cast<long long>(a.batch) * a.n_vis;
+  const int L = v.n_layers, d = v.d;
   const long long n1 = static_cast<long long>(L) * v.r_pad;
   auto mark = [&](int i) {
     if (a.marks) cudaEventRecord(a.marks[i], st);
   };
   const long long pad128 = (T + 127) / 128 * 128, pad256 = (T + 255) / 256 * 256;
-  const int nt = kv_pair_tile_n(T);
-  const long long pad_nt = (T + nt - 1) / nt * nt;
   const bool rank_pairs = prefer_256(pad256, pad128);
-  const bool kv_tokens_m = prefer_256(pad256, pad_nt);
 
-  CUtensorMap tm_x0, tm_H, tm_x0_half, tm_H_half;
+  CUtensorMap tm_x0, tm_H;
   if (!encode_2d(&tm_x0, a.x0, d, static_cast<uint64_t>(T), d, kBlockM) ||
-      !encode_2d(&tm_H, a.H, n1, a.h_rows, n1, kBlockM))
-    return cudaErrorInvalidValue;
-  if (!kv_tokens_m && (!encode_2d(&tm_x0_half, a.x0, d, static_cast<uint64_t>(T), d, nt / 2) ||
-                       !encode_2d(&tm_H_half, a.H, n1, a.h_rows, n1, nt / 2)))
+      !encode_2d(&tm_H, a.H, n1, static_cast<uint64_t>(T), n1, kBlockM))
     return cudaErrorInvalidValue;
 
   GemmParams gp;
@@ -436,7 +587,7 @@ cudaError_t enqueue_build(const PlanView& v, const BuildArgs& a, cudaStream_t st
   mark(1);
 
   // (1) H = SiLU(x0 [D_1 ... D_L]) — one GEMM over all layers' down-projections.
-  gp.s = {static_cast<int>(T), 1, static_cast<int>(n1), d / 64, 0, 0, 0, 0};
+  gp.s = {static_cast<int>(T), 1, static_cast<int>(n1), d / 64, 0, 0, 0, 0, 0, 0};
   gp.silu = {a.H, static_cast<int>(n1)};
   if (rank_pairs) {
     const long long pairs = v.num_sms / 2;
@@ -465,9 +616,10 @@ cudaError_t enqueue_build(const PlanView& v, const BuildArgs& a, cudaStream_t st
   mark(2);
 
   // (2) rstd_l from ||x0||^2 + h_l . ([x0 | h_l] [2 U_l^T ; G_l]).
-  gp.s = {static_cast<int>(T), L, v.r_pad, d / 64, v.r_pad / 64, v.r_pad, 0, 0};
+  gp.s = {static_cast<int>(T), L, v.r_pad, d / 64, v.r_pad / 64, v.r_pad, 0, 0, 0, 0};
   if (rank_pairs) tm_groups(gp.s, v.r_pad, T);
-  gp.norm = {a.H, static_cast<int>(n1), v.r_pad, a.xx, a.rstd, a.ld_rstd, 1.0f / d, v.rms_eps};
+  gp.norm = {a.H, static_cast<int>(n1), v.r_pad, a.xx, a.rstd, static_cast<int>(T), 1.0f / d,
+             v.rms_eps};
   if (err == cudaSuccess) {
     err = rank_pairs ? launch_pair_tm(EPI_NORM, v.r_pad, 0, tm_x0, tm_H, *v.tm_Bn_half, gp, v.num_sms, st)
                      : launch_gemm(EPI_NORM, v.r_pad, 0, tm_x0, tm_H, *v.tm_Bn, gp, v.num_sms, st);
@@ -475,41 +627,42 @@ cudaError_t enqueue_build(const PlanView& v, const BuildArgs& a, cudaStream_t st
   mark(3);
 
   // (3) K/V = rstd_l * ([x0 | h_l] Wkv_l^T) + b, RoPE on K, stored into the cache.
-  gp.s = {static_cast<int>(T), L, 2 * v.kv, d / 64, v.r_pad / 64, v.r_pad, 0, 0};
-  if (kv_tokens_m) tm_groups(gp.s, 256, T);
-  EpiKV& e = gp.kv;
-  e.rstd = a.rstd;
-  e.ld_rstd = a.ld_rstd;
-  e.bk = v.bk;
-  e.bv = v.bv;
-  e.kv = v.kv;
-  e.pos = a.pos;
-  e.slot = a.slot;
-  e.slot0 = a.slot0;
-  e.n_vis = a.n_vis;
-  e.n_pos = v.rope == DV_ROPE_MROPE ? 3 : 1;
-  e.sec0 = v.rope == DV_ROPE_MROPE ? v.mrope_section[0] : HD / 2;
-  e.sec01 = v.rope == DV_ROPE_MROPE ? v.mrope_section[0] + v.mrope_section[1] : HD / 2;
-  e.kc = static_cast<uint16_t*>(const_cast<void*>(a.kc));
-  e.vc = static_cast<uint16_t*>(const_cast<void*>(a.vc));
-  e.s_layer = a.s_layer;
-  e.s_batch = a.s_batch;
-  e.s_seq = a.s_seq;
-  e.s_head = a.s_head;
-  const double two_pi = 6.283185307179586476925286766559;
-  e.two_pi_hi = static_cast<float>(two_pi);
-  e.two_pi_lo = static_cast<float>(two_pi - static_cast<double>(e.two_pi_hi));
-  e.inv_two_pi = static_cast<float>(1.0 / two_pi);
-  for (int j = 0; j < HD / 2; ++j) {
-    e.inv_freq_hi[j] = static_cast<float>(v.inv_freq[j]);
-    e.inv_freq_lo[j] = static_cast<float>(v.inv_freq[j] - static_cast<double>(e.inv_freq_hi[j]));
-  }
-  if (err == cudaSuccess) {
-    err = kv_tokens_m ? launch_pair_tm(EPI_KV, 256, HD, tm_x0, tm_H, *v.tm_Wkv, gp, v.num_sms, st)
-                      : launch_kv_pair(HD, nt, *v.tm_Wkv, tm_x0_half, tm_H_half, gp, v.num_sms, st);
-  }
+  gp.s = {static_cast<int>(T), L, 2 * v.kv, d / 64, v.r_pad / 64, v.r_pad, 0, 0, 0, 0};
+  fill_epi_kv(v, a, T, gp.kv);
+  if (err == cudaSuccess)
+    err = launch_kv_stage(v, gp, T, a.x0, static_cast<uint64_t>(T), tm_x0, a.H,
+                          static_cast<uint64_t>(n1), tm_H, st);
   mark(4);
   return err;
+}
+
+size_t carve_workspace(const PlanView& v, long long T, void* base, BuildArgs* a) {
+  size_t off = 0;
+  auto take = [&](size_t bytes) {
+    const size_t o = off;
+    off += (bytes + 255) / 256 * 256;
+    return o;
+  };
+  const size_t L = static_cast<size_t>(v.n_layers), t = static_cast<size_t>(T);
+  const size_t d = static_cast<size_t>(v.d);
+  const size_t oH = take(t * L * v.r_pad * 2), oR = take(L * t * 4), oX = take(t * 4);
+  size_t oS = 0, oM = 0, oP = 0;
+  const bool rec = v.adapter == DV_ADAPTER_RECURRENT;
+  if (rec) {
+    oS = take(t * d * 4);
+    oM = take(L * t * d * 2);
+    oP = take(L * (d / 64) * t * 4);
+  }
+  if (base && a) {
+    unsigned char* b = static_cast<unsigned char*>(base);
+    a->H = reinterpret_cast<uint16_t*>(b + oH);
+    a->rstd = reinterpret_cast<float*>(b + oR);
+    a->xx = reinterpret_cast<float*>(b + oX);
+    a->state = rec ? reinterpret_cast<float*>(b + oS) : nullptr;
+    a->mem = rec ? reinterpret_cast<uint16_t*>(b + oM) : nullptr;
+    a->part = rec ? reinterpret_cast<float*>(b + oP) : nullptr;
+  }
+  return off;
 }
 
 bool plan_view(const dv_plan* p, PlanView* v) {
@@ -517,6 +670,7 @@ bool plan_view(const dv_plan* p, PlanView* v) {
   const dv_config& c = p->cfg;
   v->d = c.d;
   v->n_layers = p->n_active;
+  v->adapter = c.adapter;
   v->head_dim = c.head_dim;
   v->rope = c.rope;
   for (int i = 0; i < 3; ++i) v->mrope_section[i] = c.mrope_section[i];
@@ -533,6 +687,9 @@ bool plan_view(const dv_plan* p, PlanView* v) {
   v->tm_Bn = &p->tm_Bn;
   v->tm_Bn_half = &p->tm_Bn_half;
   v->tm_Wkv = &p->tm_Wkv;
+  v->tm_Dst_rp = &p->tm_Dst_rp;
+  v->tm_Uup = &p->tm_Uup;
+  v->resid_bn = p->resid_bn;
   v->inv_freq = p->inv_freq;
   v->Wkv = p->Wkv;
   v->active = p->active;
@@ -604,19 +761,30 @@ int dv_memory_plan(const dv_config* cfg, const dv_weights* w, void* stream, dv_p
   // The plan holds the layers that are not dropped, compacted: planned layer i is cache layer
   // active[i]; dropped layers take no weight or workspace memory.
   const int L = p->n_active;
+  const bool rec = cfg->adapter == DV_ADAPTER_RECURRENT;
   p->r_pad = (r + 63) / 64 * 64;
   p->kv = cfg->n_kv_heads * HD;
-  p->k_total = d + p->r_pad;
+  // Embedding adapter: K/V weights carry the folded rank-r columns. Recurrent: the K/V GEMM
+  // reads M_l itself, so only the d columns of W diag(gamma).
+  p->k_total = rec ? d : d + p->r_pad;
+  p->resid_bn = d % 256 == 0 ? 256 : (d % 128 == 0 ? 128 : 64);
   p->max_tokens = cfg->max_batch * cfg->max_n_vis;
   const long long T = p->max_tokens;
   cudaStream_t st = static_cast<cudaStream_t>(stream);
+  // The recurrent K/V GEMM addresses the stacked M_l as L * T rows (32-bit TMA coordinates).
+  if (rec && static_cast<long long>(L) * T + dv::kBlockM >= (1LL << 31)) {
+    delete p;
+    return DV_ERR_UNSUPPORTED_SHAPE;
+  }
+  dv::PlanView pv;
+  dv::plan_view(p, &pv);
+  const size_t ws_bytes = dv::carve_workspace(pv, T, nullptr, nullptr);
 
   bool ok = dmalloc(&p->Dst, sizeof(uint16_t) * L * p->r_pad * d) &&
-            dmalloc(&p->Bn, sizeof(uint16_t) * L * p->r_pad * p->k_total) &&
+            (rec ? dmalloc(&p->Uup, sizeof(uint16_t) * static_cast<size_t>(L) * d * p->r_pad)
+                 : dmalloc(&p->Bn, sizeof(uint16_t) * L * p->r_pad * p->k_total)) &&
             dmalloc(&p->Wkv, sizeof(uint16_t) * static_cast<size_t>(L) * 2 * p->kv * p->k_total) &&
-            dmalloc(&p->H, sizeof(uint16_t) * T * L * p->r_pad) &&
-            dmalloc(&p->xx, sizeof(float) * T) && dmalloc(&p->rstd, sizeof(float) * T * L) &&
-            dmalloc(&p->status, sizeof(int));
+            dmalloc(&p->ws, ws_bytes) && dmalloc(&p->status, sizeof(int));
   if (ok && cfg->has_kv_bias)
     ok = dmalloc(&p->bk, sizeof(float) * L * p->kv) && dmalloc(&p->bv, sizeof(float) * L * p->kv);
   if (!ok) {
@@ -638,11 +806,13 @@ int dv_memory_plan(const dv_config* cfg, const dv_weights* w, void* stream, dv_p
   const uint16_t* Wv = static_cast<const uint16_t*>(w->Wv);
   cudaMemsetAsync(p->status, 0, sizeof(int), st);
   k_pack_down<<<grid_for(1LL * L * p->r_pad * d), 256, 0, st>>>(D, p->Dst, L, r, p->r_pad, d, pl);
-  k_pack_norm_u<<<grid_for(1LL * L * p->r_pad * p->k_total), 256, 0, st>>>(U, p->Bn, L, r, p->r_pad,
-                                                                           d, p->k_total, pl);
   k_pack_kv<<<grid_for(1LL * L * 2 * p->kv * p->k_total), 256, 0, st>>>(Wk, Wv, G, p->Wkv, L, p->kv,
                                                                         HD, d, p->k_total, pl);
-  {
+  if (rec) {
+    k_pack_up<<<grid_for(1LL * L * d * p->r_pad), 256, 0, st>>>(U, p->Uup, L, r, p->r_pad, d, pl);
+  } else {
+    k_pack_norm_u<<<grid_for(1LL * L * p->r_pad * p->k_total), 256, 0, st>>>(U, p->Bn, L, r, p->r_pad,
+                                                                             d, p->k_total, pl);
     dim3 g1((r + 63) / 64, (r + 63) / 64, L);
     k_rank_product<1><<<g1, 256, 0, st>>>(Wk, Wv, G, U, p->Bn, r, r, d, p->kv, HD, p->r_pad,
                                           p->k_total, pl);
@@ -670,10 +840,15 @@ int dv_memory_plan(const dv_config* cfg, const dv_weights* w, void* stream, dv_p
              encode_2d(&p->tm_Dst_half[0], p->Dst, d, 1ull * L * p->r_pad, d, 32) &&
              encode_2d(&p->tm_Dst_half[1], p->Dst, d, 1ull * L * p->r_pad, d, 64) &&
              encode_2d(&p->tm_Dst_half[2], p->Dst, d, 1ull * L * p->r_pad, d, 128) &&
-             encode_2d(&p->tm_Bn_half, p->Bn, p->k_total, 1ull * L * p->r_pad, p->k_total,
-                       p->r_pad / 2) &&
-             encode_2d(&p->tm_Bn, p->Bn, p->k_total, 1ull * L * p->r_pad, p->k_total, p->r_pad) &&
              encode_2d(&p->tm_Wkv, p->Wkv, p->k_total, 1ull * L * 2 * p->kv, p->k_total, 128);
+  if (enc && rec) {
+    enc = encode_2d(&p->tm_Dst_rp, p->Dst, d, 1ull * L * p->r_pad, d, p->r_pad) &&
+          encode_2d(&p->tm_Uup, p->Uup, p->r_pad, 1ull * L * d, p->r_pad, p->resid_bn);
+  } else if (enc) {
+    enc = encode_2d(&p->tm_Bn_half, p->Bn, p->k_total, 1ull * L * p->r_pad, p->k_total,
+                    p->r_pad / 2) &&
+          encode_2d(&p->tm_Bn, p->Bn, p->k_total, 1ull * L * p->r_pad, p->k_total, p->r_pad);
+  }
   if (!enc) {
     free_plan_memory(p);
     delete p;
@@ -685,7 +860,19 @@ int dv_memory_plan(const dv_config* cfg, const dv_weights* w, void* stream, dv_p
   return DV_OK;
 }
 
-int dv_kernels_per_build(const dv_plan* p) { return p ? kStages : 0; }
+int dv_kv_engine(const dv_plan* p, long long tokens) {
+  if (!p || tokens <= 0) return 0;
+  const int nt = dv::kv_pair_tile_n(tokens);
+  const long long pad256 = (tokens + 255) / 256 * 256, pad_nt = (tokens + nt - 1) / nt * nt;
+  return dv::prefer_256(pad256, pad_nt) ? DV_KV_ENGINE_TOKENS_AS_M : DV_KV_ENGINE_WEIGHTS_AS_M;
+}
+
+// Embedding adapter: row sums, stacked down-projection, RMS statistics, K/V. Recurrent: two
+// launches per planned layer, the RMS statistics and K/V.
+int dv_kernels_per_build(const dv_plan* p) {
+  if (!p) return 0;
+  return p->cfg.adapter == DV_ADAPTER_RECURRENT ? 2 * p->n_active + 2 : kStages;
+}
 
 int dv_build_visual_memory(dv_plan* p, const void* x0, int batch, int n_vis, const int* pos,
                            const int* slot, int slot0, const dv_kv_cache* out, void* stream) {
@@ -711,11 +898,8 @@ int dv_build_visual_memory(dv_plan* p, const void* x0, int batch, int n_vis, con
   a.s_batch = out->s_batch;
   a.s_seq = out->s_seq;
   a.s_head = out->s_head;
-  a.H = p->H;
-  a.h_rows = p->max_tokens;
-  a.rstd = p->rstd;
-  a.ld_rstd = p->max_tokens;
-  a.xx = p->xx;
+  dv::carve_workspace(v, T, p->ws, &a);
+  p->last_tokens = T;
   a.marks = (p->timing && p->timed < kMaxTimed) ? &p->ev[static_cast<size_t>(p->timed++) * kEvPerBuild]
                                                 : nullptr;
   return dv::enqueue_build(v, a, static_cast<cudaStream_t>(stream)) == cudaSuccess ? DV_OK
@@ -775,20 +959,41 @@ int dv_debug_wait_timeout(dv_plan* p, int timeout_us, void* stream) {
 
 int dv_debug_copy_workspace(dv_plan* p, int tokens, void* H, void* rstd, void* xx,
                             int* r_pad_out, void* stream) {
-  if (!p || tokens < 0 || tokens > p->max_tokens) return DV_ERR_INVALID_ARG;
+  if (!p || tokens < 0 || tokens > p->last_tokens) return DV_ERR_INVALID_ARG;
   if (r_pad_out) *r_pad_out = p->r_pad;
+  if (tokens == 0) return DV_OK;
   cudaStream_t st = static_cast<cudaStream_t>(stream);
+  dv::PlanView v;
+  dv::plan_view(p, &v);
+  dv::BuildArgs a;
+  dv::carve_workspace(v, p->last_tokens, p->ws, &a);  // the layout of the last build
   const int L = p->n_active;  // the workspace holds the planned (not dropped) layers
   const size_t hrow = static_cast<size_t>(L) * p->r_pad;
+  const size_t T = static_cast<size_t>(p->last_tokens);
   cudaError_t err = cudaSuccess;
-  if (H && tokens > 0)
-    err = cudaMemcpyAsync(H, p->H, sizeof(uint16_t) * hrow * tokens, cudaMemcpyDeviceToDevice, st);
-  if (rstd && tokens > 0 && err == cudaSuccess)
-    err = cudaMemcpy2DAsync(rstd, sizeof(float) * tokens, p->rstd, sizeof(float) * p->max_tokens,
+  if (H) err = cudaMemcpyAsync(H, a.H, sizeof(uint16_t) * hrow * tokens, cudaMemcpyDeviceToDevice, st);
+  if (rstd && err == cudaSuccess)
+    err = cudaMemcpy2DAsync(rstd, sizeof(float) * tokens, a.rstd, sizeof(float) * T,
                             sizeof(float) * tokens, L, cudaMemcpyDeviceToDevice, st);
-  if (xx && tokens > 0 && err == cudaSuccess)
-    err = cudaMemcpyAsync(xx, p->xx, sizeof(float) * tokens, cudaMemcpyDeviceToDevice, st);
+  if (xx && err == cudaSuccess)
+    err = cudaMemcpyAsync(xx, a.xx, sizeof(float) * tokens, cudaMemcpyDeviceToDevice, st);
   return err == cudaSuccess ? DV_OK : DV_ERR_CUDA;
+}
+
+int dv_debug_copy_memory(dv_plan* p, int tokens, void* mem, void* stream) {
+  if (!p || !mem || tokens < 0 || tokens > p->last_tokens) return DV_ERR_INVALID_ARG;
+  if (p->cfg.adapter != DV_ADAPTER_RECURRENT) return DV_ERR_INVALID_ARG;
+  if (tokens == 0) return DV_OK;
+  dv::PlanView v;
+  dv::plan_view(p, &v);
+  dv::BuildArgs a;
+  dv::carve_workspace(v, p->last_tokens, p->ws, &a);
+  const size_t row = sizeof(uint16_t) * p->cfg.d;
+  const size_t T = static_cast<size_t>(p->last_tokens);
+  return cudaMemcpy2DAsync(mem, row * tokens, a.mem, row * T, row * tokens, p->n_active,
+                           cudaMemcpyDeviceToDevice, static_cast<cudaStream_t>(stream)) == cudaSuccess
+             ? DV_OK
+             : DV_ERR_CUDA;
 }
 
 }  // extern "C"

@@ -95,6 +95,62 @@ __device__ __forceinline__ void epi_norm(const GemmParams& p, uint32_t tbase, in
   }
 }
 
+// One step of the recurrent adapter (Sec. 3.1 Eq. 6) for token row t and columns
+// [n*BN, (n+1)*BN): M = prev + h U^T with prev = x0 (first planned layer) or the fp32 state.
+// Writes the new fp32 state, bf16(M) for the K/V GEMM, and the sum of M^2 over the tile.
+template <int BN>
+__device__ __forceinline__ void epi_resid(const GemmParams& p, uint32_t tbase, int n, int t) {
+  const EpiResid& e = p.resid;
+  const bool valid = t < p.s.M;
+  const size_t row = static_cast<size_t>(valid ? t : 0) * e.d + static_cast<size_t>(n) * BN;
+  float ss = 0.0f;
+#pragma unroll 1
+  for (int c = 0; c < BN / 32; ++c) {
+    uint32_t r[32];
+    __syncwarp();
+    tmem_ld32(tbase + c * 32, r);
+    tmem_ld_wait();
+    if (valid) {
+      float mv[32];
+      if (e.first) {
+        const uint4* xv = reinterpret_cast<const uint4*>(e.x0 + row + c * 32);
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+          const uint4 w = xv[q];
+          const uint32_t ws[4] = {w.x, w.y, w.z, w.w};
+#pragma unroll
+          for (int u = 0; u < 4; ++u) {
+            mv[q * 8 + 2 * u] = bf16_bits_to_float(ws[u] & 0xFFFFu);
+            mv[q * 8 + 2 * u + 1] = bf16_bits_to_float(ws[u] >> 16);
+          }
+        }
+      } else {
+        const float4* sv = reinterpret_cast<const float4*>(e.state + row + c * 32);
+#pragma unroll
+        for (int q = 0; q < 8; ++q) {
+          const float4 w = sv[q];
+          mv[4 * q] = w.x;
+          mv[4 * q + 1] = w.y;
+          mv[4 * q + 2] = w.z;
+          mv[4 * q + 3] = w.w;
+        }
+      }
+      uint32_t pk[16];
+#pragma unroll
+      for (int u = 0; u < 32; ++u) {
+        mv[u] += __uint_as_float(r[u]);
+        ss = fmaf(mv[u], mv[u], ss);
+      }
+#pragma unroll
+      for (int u = 0; u < 16; ++u) pk[u] = pack_bf16x2(mv[2 * u], mv[2 * u + 1]);
+      float4* so = reinterpret_cast<float4*>(e.state + row + c * 32);
+#pragma unroll
+      for (int q = 0; q < 8; ++q) so[q] = make_float4(mv[4 * q], mv[4 * q + 1], mv[4 * q + 2], mv[4 * q + 3]);
+      store_row32(e.mem + row + c * 32, pk);
+    }
+  }
+  if (valid) e.part[static_cast<size_t>(n) * p.s.M + t] = ss;
+}
 
 // Per-token context of the K/V store: cache row base, positions, rstd of one token.
 struct KvToken {

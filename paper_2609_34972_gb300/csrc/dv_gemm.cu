@@ -1,11 +1,13 @@
-// Persistent, warp-specialised 1-SM tcgen05 GEMM for the two rank-r contractions of the
+// Persistent, warp-specialised 1-SM tcgen05 GEMM for the rank-r contractions of the
 // visual-memory build, each with its own fused epilogue (the K/V contraction runs on CTA pairs,
-// dv_kv2sm.cu):
+// dv_kv2sm.cu / dv_pair_tm.cu):
 //   EPI_SILU  H   = SiLU(x0 [D_1 ... D_L])          all L down-projections as one GEMM, since
 //                                                    every layer reads only E (Sec. 3.1 Eq. 5)
 //   EPI_NORM  rstd_l = (||M_l||^2 / d + eps)^-1/2    the RMS statistic of M_l = x0 + h_l U_l
 //                                                    (Sec. 3.1 Eq. 4), from [x0 | h_l] times
 //                                                    [2 U_l^T ; U_l U_l^T]
+//   EPI_RESID M_l = M_{l-1} + h_l U_l                one step of the recurrent adapter
+//                                                    (Sec. 3.1 Eq. 6), fp32 state in HBM
 //
 // CTA layout (192 threads, one CTA per SM):
 //   warp 0      TMA producer: one lane streams 64-wide K slabs of A (128 token rows) and B
@@ -116,15 +118,16 @@ __global__ void __launch_bounds__(kNumThreads, 1)
         const int m = tile % m_tiles;
         const int rest = tile / m_tiles;
         const int n = rest % n_tiles;
-        const int l = rest / n_tiles;
+        const int l = p.s.layer0 + rest / n_tiles;
         const int brow = l * p.s.n_per_layer + n * BN;
+        const int arow = l * p.s.a0_rows_per_layer + m * kBlockM;
         for (int ks = 0; ks < k_slabs; ++ks) {
           if (!mbar_wait(empty_bar(stage), phase ^ 1u, abort_flag, tmo)) break;
           const uint32_t a_dst = ring + stage * C::kStageBytes;
           const uint32_t b_dst = a_dst + C::kABytes;
           mbar_arrive_expect_tx(full_bar(stage), C::kStageBytes);
           if (ks < p.s.k0_slabs) {
-            tma_load_2d(a_dst, &tmA0, full_bar(stage), ks * kBlockK, m * kBlockM);
+            tma_load_2d(a_dst, &tmA0, full_bar(stage), ks * kBlockK, arow);
           } else {
             tma_load_2d(a_dst, &tmA1, full_bar(stage),
                         l * p.s.a1_cols_per_layer + (ks - p.s.k0_slabs) * kBlockK, m * kBlockM);
@@ -197,7 +200,7 @@ __global__ void __launch_bounds__(kNumThreads, 1)
       const int m = tile % m_tiles;
       const int rest = tile / m_tiles;
       const int n = rest % n_tiles;
-      const int l = rest / n_tiles;
+      const int l = p.s.layer0 + rest / n_tiles;
       if (!mbar_wait(tfull_bar(acc), acc_phase, abort_flag, tmo)) break;
       tc_fence_after();
       const uint32_t tbase =
@@ -205,8 +208,10 @@ __global__ void __launch_bounds__(kNumThreads, 1)
       const int t = m * kBlockM + row;
       if constexpr (EPI == EPI_SILU) {
         epi_silu<BN>(p, tbase, n, t);
-      } else {
+      } else if constexpr (EPI == EPI_NORM) {
         epi_norm<BN>(p, tbase, l, t);
+      } else {
+        epi_resid<BN>(p, tbase, n, t);
       }
       tc_fence_before();
       mbar_arrive(tempty_bar(acc));
@@ -264,6 +269,10 @@ cudaError_t launch_gemm(int epi, int block_n, int head_dim, const CUtensorMap& a
     if (block_n == 64) return launch_t<EPI_NORM, 64, 0>(a0, a1, b, p, num_sms, stream);
     if (block_n == 128) return launch_t<EPI_NORM, 128, 0>(a0, a1, b, p, num_sms, stream);
     if (block_n == 256) return launch_t<EPI_NORM, 256, 0>(a0, a1, b, p, num_sms, stream);
+  } else if (epi == EPI_RESID) {
+    if (block_n == 64) return launch_t<EPI_RESID, 64, 0>(a0, a1, b, p, num_sms, stream);
+    if (block_n == 128) return launch_t<EPI_RESID, 128, 0>(a0, a1, b, p, num_sms, stream);
+    if (block_n == 256) return launch_t<EPI_RESID, 256, 0>(a0, a1, b, p, num_sms, stream);
   }
   return cudaErrorInvalidValue;
 }

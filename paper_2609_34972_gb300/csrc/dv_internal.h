@@ -1,5 +1,5 @@
-// Internal interface between the C-ABI / plan code (dv_api.cu) and the tcgen05 GEMM kernels
-// (dv_gemm.cu). Not part of the public ABI.
+// Internal interface between the C-ABI / plan code (dv_api.cu) and the tcgen05 kernels
+// (dv_gemm.cu, dv_kv2sm.cu, dv_pair_tm.cu, dv_recurrent.cu). Not part of the public ABI.
 #pragma once
 #include <cstdint>
 #include <cuda.h>
@@ -19,13 +19,15 @@ enum Epilogue : int {
   EPI_SILU = 0,  // stacked down-projection: H = bf16(SiLU(acc))
   EPI_NORM = 1,  // RMS statistic: rstd = (||x0||^2 + h . acc) / d + eps) ^ -1/2
   EPI_KV = 2,    // K/V: rstd * acc + bias, RoPE on K, bf16 cache store
+  EPI_RESID = 3, // recurrent step: M_l = M_{l-1} + acc (fp32 state), bf16 M_l, sums of squares
 };
 
-// Operand schedule shared by all three GEMMs. The A operand of a tile is the 128-row token
-// block of [x0 | H_l]: k0_slabs 64-wide slabs of x0 (tensor map A0), then k1_slabs slabs of H
-// starting at column layer * a1_cols_per_layer (tensor map A1). B is one stacked weight
+// Operand schedule shared by all GEMMs. The A operand of a tile is the 128-row token block of
+// [A0 | H_l]: k0_slabs 64-wide slabs of A0 starting at row layer * a0_rows_per_layer (x0 for
+// every layer, or the stacked per-layer M_l of the recurrent adapter), then k1_slabs slabs of
+// H starting at column layer * a1_cols_per_layer (tensor map A1). B is one stacked weight
 // matrix whose rows for layer l start at l * n_per_layer; its columns follow the same slab
-// order as A.
+// order as A. "layer" counts from layer0 (1-SM kernel only; 0 elsewhere).
 struct GemmShape {
   int M;                  // tokens in this build
   int n_layers;           // groups (layers)
@@ -35,6 +37,8 @@ struct GemmShape {
   int a1_cols_per_layer;  // r_pad
   int group_m;            // tokens-as-M kernels: token blocks per L2 super-block (0: all)
   int group_w;            // tokens-as-M kernels: weight tiles per L2 super-block (0: 1)
+  int layer0;             // first planned layer of the launch
+  int a0_rows_per_layer;  // 0: one A0 for every layer; else A0 rows of layer l start at l * it
 };
 
 struct EpiSilu {
@@ -73,6 +77,19 @@ struct EpiKV {
   float inv_freq_lo[kMaxHalfHead];
 };
 
+// Recurrent step of one layer (Sec. 3.1 Eq. 6): for token row t and the tile's columns,
+// M = prev + acc with prev = x0 (first planned layer) or the fp32 state; the state is
+// overwritten with M, bf16(M) goes to the layer's slice of the stacked memories, and the
+// tile's sum of M^2 over its columns to part[n][t].
+struct EpiResid {
+  const uint16_t* x0;  // bf16 [M][d]
+  float* state;        // fp32 [M][d]
+  uint16_t* mem;       // bf16 [M][d]: this layer's M_l
+  float* part;         // fp32 [d / BLOCK_N][M]: this layer's partial sums of squares
+  int d;
+  int first;           // 1: prev = x0
+};
+
 struct GemmParams {
   GemmShape s;
   // The plan holds the layers that are not dropped, in order; logical layer i of a launch (its
@@ -81,12 +98,13 @@ struct GemmParams {
   EpiSilu silu;
   EpiNorm norm;
   EpiKV kv;
+  EpiResid resid;
   int* status;              // device status word
   unsigned long long timeout_ns;
 };
 
-// Launches one persistent warp-specialised 1-SM tcgen05 GEMM (EPI_SILU or EPI_NORM,
-// block_n 64/128/256). Returns a cudaError_t value.
+// Launches one persistent warp-specialised 1-SM tcgen05 GEMM (EPI_SILU, EPI_NORM or
+// EPI_RESID, block_n 64/128/256). Returns a cudaError_t value.
 cudaError_t launch_gemm(int epi, int block_n, int head_dim, const CUtensorMap& a0,
                         const CUtensorMap& a1, const CUtensorMap& b, const GemmParams& p,
                         int num_sms, cudaStream_t stream);
@@ -107,6 +125,27 @@ cudaError_t launch_pair_tm(int epi, int block_n, int head_dim, const CUtensorMap
                            const CUtensorMap& a1, const CUtensorMap& b, const GemmParams& p,
                            int num_sms, cudaStream_t stream);
 
+// Recurrent down-projection of one layer: H[:, h_col0 + n] = bf16(SiLU(A B^T)) with A the
+// layer's input state (bf16 [M][k_slabs * 64], rows from a_row0) and B the layer's r_pad rows
+// of the stacked down-projection (from b_row0). The K dimension is split over the CTAs of a
+// thread-block cluster (size `splits`, 1/2/4/8) and the fp32 partials are summed in a fixed
+// order through distributed shared memory.
+struct DownParams {
+  int M;
+  int a_row0;
+  int b_row0;
+  int k_slabs;
+  uint16_t* H;
+  int ldh;
+  int h_col0;
+  int* status;
+  unsigned long long timeout_ns;
+};
+cudaError_t launch_down_split(int r_pad, int splits, const CUtensorMap& a, const CUtensorMap& b,
+                              const DownParams& p, cudaStream_t stream);
+// K splits (1, 2, 4 or 8) for m_tiles token blocks of 128 rows and k_slabs slabs.
+int down_splits(long long m_tiles, int k_slabs, int num_sms);
+
 // Token tile (64, 128, 192 or 256) of the pair kernel for a build of `tokens` tokens.
 int kv_pair_tile_n(long long tokens);
 int kv_pair_smem_bytes(int nt);
@@ -114,6 +153,7 @@ int kv_pair_smem_bytes(int nt);
 // Read-only view of a plan's repacked weights and shape, for build variants outside dv_api.cu.
 struct PlanView {
   int d, n_layers, head_dim, rope, mrope_section[3];  // n_layers: layers the plan holds
+  int adapter;                                         // DV_ADAPTER_*
   float rms_eps;
   int num_sms, r_pad, kv, k_total;
   const float* bk;
@@ -124,6 +164,9 @@ struct PlanView {
   const CUtensorMap* tm_Bn;        // boxes of r_pad rows
   const CUtensorMap* tm_Bn_half;   // boxes of r_pad / 2 rows
   const CUtensorMap* tm_Wkv;       // boxes of 128 rows
+  const CUtensorMap* tm_Dst_rp;    // recurrent: boxes of r_pad rows (one layer's D)
+  const CUtensorMap* tm_Uup;       // recurrent: [L*d][r_pad], boxes of resid_bn rows
+  int resid_bn;                    // recurrent: column tile of the up-projection step
   const double* inv_freq;     // head_dim / 2 values
   const uint16_t* Wkv;        // repacked K/V weights [L*2kv][k_total]
   const int16_t* active;      // cache layer of each planned layer
@@ -140,13 +183,18 @@ struct BuildArgs {
   const void* kc;
   const void* vc;
   long long s_layer, s_batch, s_seq, s_head;
-  uint16_t* H;          // [h_rows][L * r_pad] bf16
-  long long h_rows;     // rows of H that exist (>= tokens)
-  float* rstd;          // [L][ld_rstd]
-  int ld_rstd;
+  uint16_t* H;          // [tokens][L * r_pad] bf16
+  float* rstd;          // [L][tokens]
   float* xx;            // [tokens]
+  float* state;         // recurrent: fp32 [tokens][d]
+  uint16_t* mem;        // recurrent: bf16 [L][tokens][d]
+  float* part;          // recurrent: fp32 [L][d / 64][tokens]
   cudaEvent_t* marks;   // 5 events around the 4 stages, or null
 };
+
+// Bytes of the intermediates of a build of `tokens` tokens (each part 256-byte aligned). With
+// a non-null base, also points the intermediates of `a` into [base, base + bytes).
+size_t carve_workspace(const PlanView& v, long long tokens, void* base, BuildArgs* a);
 
 // Argument checks shared by the build entry points (dv_status value; DV_OK for an empty build).
 int check_build_args(const void* x0, int batch, int n_vis, const int* pos, const int* slot,

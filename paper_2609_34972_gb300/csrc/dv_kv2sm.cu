@@ -129,6 +129,7 @@ __global__ void __launch_bounds__(kPairThreads, 1)
         const int l = rest / groups;
         const int wrow = l * p.s.n_per_layer + g * 256 + static_cast<int>(rank) * 128;
         const int trow = nt * NT + static_cast<int>(rank) * C::kHalfN;
+        const int xrow = l * p.s.a0_rows_per_layer + trow;
         for (int ks = 0; ks < k_slabs; ++ks) {
           if (!mbar_wait(empty_bar(stage), phase ^ 1u, abort_flag, tmo)) break;
           const uint32_t a_dst = ring + stage * C::kStageBytes;
@@ -139,7 +140,7 @@ __global__ void __launch_bounds__(kPairThreads, 1)
           if (rank == 0) mbar_arrive_expect_tx(full_bar(stage), 2 * C::kStageBytes);
           tma_load_2d_pair(a_dst, &tmW, fb, ks * kBlockK, wrow);
           if (ks < p.s.k0_slabs) {
-            tma_load_2d_pair(b_dst, &tmX, fb, ks * kBlockK, trow);
+            tma_load_2d_pair(b_dst, &tmX, fb, ks * kBlockK, xrow);
           } else {
             tma_load_2d_pair(b_dst, &tmH, fb,
                              l * p.s.a1_cols_per_layer + (ks - p.s.k0_slabs) * kBlockK, trow);

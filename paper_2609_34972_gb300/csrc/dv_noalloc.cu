@@ -7,6 +7,7 @@
 // batch is not acceptable, and code that must not risk the implicit device synchronisation
 // of cudaMalloc / cudaFree in its latency-critical path. For them this file keeps the build's
 // intermediate buffers (SiLU(E D_l) for every layer, the RMS statistics and the row sums of
+// squares; for the recurrent adapter also the fp32 state, M_l of every layer and partial sums of
 // squares) in one file-scope static device array of kScratchBytes instead of the plan's
 // workspace. The plan's repacked weights are still used; nothing here allocates.
 //
@@ -56,8 +57,6 @@ int scratch_address(void** out) {
   return DV_OK;
 }
 
-size_t round256(size_t n) { return (n + 255) / 256 * 256; }
-
 }  // namespace
 
 extern "C" int dv_build_visual_memory_noalloc(dv_plan* plan, const void* x0, int batch,
@@ -70,13 +69,11 @@ extern "C" int dv_build_visual_memory_noalloc(dv_plan* plan, const void* x0, int
   const long long T = static_cast<long long>(batch) * n_vis;
   if (T == 0) return DV_OK;
 
-  // Scratch layout: H [T][L*r_pad] bf16 | rstd [L][T] fp32 | xx [T] fp32, 256-byte aligned.
-  const int L = v.n_layers;
-  const long long n1 = static_cast<long long>(L) * v.r_pad;
-  const size_t h_bytes = round256(static_cast<size_t>(T) * n1 * 2);
-  const size_t r_bytes = round256(static_cast<size_t>(T) * L * 4);
-  const size_t x_bytes = round256(static_cast<size_t>(T) * 4);
-  if (h_bytes + r_bytes + x_bytes > kScratchBytes || T > (1LL << 24)) return DV_ERR_UNSUPPORTED_SHAPE;
+  // Scratch layout: the build's intermediates as carve_workspace lays them out for T tokens.
+  const size_t bytes = dv::carve_workspace(v, T, nullptr, nullptr);
+  if (bytes > kScratchBytes || T > (1LL << 24)) return DV_ERR_UNSUPPORTED_SHAPE;
+  if (v.adapter == DV_ADAPTER_RECURRENT && static_cast<long long>(v.n_layers) * T + 128 >= (1LL << 31))
+    return DV_ERR_UNSUPPORTED_SHAPE;
 
   void* base = nullptr;
   rc = scratch_address(&base);
@@ -95,11 +92,7 @@ extern "C" int dv_build_visual_memory_noalloc(dv_plan* plan, const void* x0, int
   a.s_batch = out->s_batch;
   a.s_seq = out->s_seq;
   a.s_head = out->s_head;
-  a.H = static_cast<uint16_t*>(base);
-  a.h_rows = T;
-  a.rstd = reinterpret_cast<float*>(static_cast<unsigned char*>(base) + h_bytes);
-  a.ld_rstd = static_cast<int>(T);
-  a.xx = reinterpret_cast<float*>(static_cast<unsigned char*>(base) + h_bytes + r_bytes);
+  dv::carve_workspace(v, T, base, &a);
   a.marks = nullptr;
   return dv::enqueue_build(v, a, static_cast<cudaStream_t>(stream)) == cudaSuccess ? DV_OK
                                                                                    : DV_ERR_CUDA;

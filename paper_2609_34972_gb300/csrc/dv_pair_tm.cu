@@ -128,6 +128,7 @@ __global__ void __launch_bounds__(kTmThreads, 1)
         const int n = w % n_tiles;
         const int l = w / n_tiles;
         const int arow = m * 256 + static_cast<int>(rank) * 128;
+        const int a0row = l * p.s.a0_rows_per_layer + arow;
         const int brow = l * p.s.n_per_layer + n * BN + static_cast<int>(rank) * (BN / 2);
         for (int ks = 0; ks < k_slabs; ++ks) {
           if (!mbar_wait(empty_bar(stage), phase ^ 1u, abort_flag, tmo)) break;
@@ -136,7 +137,7 @@ __global__ void __launch_bounds__(kTmThreads, 1)
           const uint32_t fb = leader_full0 + 8u * stage;
           if (rank == 0) mbar_arrive_expect_tx(full_bar(stage), 2 * C::kStageBytes);
           if (ks < p.s.k0_slabs) {
-            tma_load_2d_pair(a_dst, &tmA0, fb, ks * kBlockK, arow);
+            tma_load_2d_pair(a_dst, &tmA0, fb, ks * kBlockK, a0row);
           } else {
             tma_load_2d_pair(a_dst, &tmA1, fb,
                              l * p.s.a1_cols_per_layer + (ks - p.s.k0_slabs) * kBlockK, arow);

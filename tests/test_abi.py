@@ -45,13 +45,17 @@ def test_null_arguments_rejected(dv):
     assert lib.dv_memory_plan(None, None, None, ctypes.byref(h)) == dv.DV_ERR_INVALID_ARG
     assert lib.dv_build_visual_memory(None, None, 1, 1, None, None, 0, None, None) == dv.DV_ERR_INVALID_ARG
     assert lib.dv_plan_status(None) == dv.DV_ERR_INVALID_ARG
+    assert lib.dv_debug_copy_memory(None, 0, None, None) == dv.DV_ERR_INVALID_ARG
     lib.dv_free(None)  # no-op
+    with pytest.raises(ValueError):
+        dv.make_config(512, 4, 8, 64, 16, adapter="stacked")
 
 
 @pytest.mark.parametrize("field,value,code", [
     ("d", 100, 2), ("d", 0, 1), ("rank", 0, 1), ("rank", 300, 2), ("head_dim", 96, 2),
     ("n_layers", -1, 1), ("act", 3, 1), ("rope", 5, 1), ("max_batch", 0, 1),
     ("rope_theta", -1.0, 1), ("rms_eps", -1e-6, 1), ("n_kv_heads", 129, 2),
+    ("adapter", 2, 1), ("adapter", -1, 1),
 ])
 def test_bad_config_rejected_before_device(dv, field, value, code):
     cfg = dv.make_config(512, 4, 8, 64, 16, max_batch=1, max_n_vis=64)
