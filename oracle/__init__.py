@@ -26,7 +26,10 @@ class _Cfg(ctypes.Structure):
     _fields_ = [("d", ctypes.c_int), ("n_layers", ctypes.c_int), ("n_kv_heads", ctypes.c_int),
                 ("head_dim", ctypes.c_int), ("rank", ctypes.c_int), ("rope", ctypes.c_int),
                 ("rope_theta", ctypes.c_double), ("mrope_section", ctypes.c_int * 3),
-                ("rms_eps", ctypes.c_double), ("recurrent", ctypes.c_int)]
+                ("rms_eps", ctypes.c_double), ("recurrent", ctypes.c_int),
+                ("k_norm", ctypes.c_int), ("k_norm_eps", ctypes.c_double)]
+
+_ROPE_MODES = {"1d": 0, "mrope": 1, "mrope_interleaved": 2}
 
 
 def build(force: bool = False) -> str:
@@ -55,8 +58,9 @@ def _load():
         lib.oracle_rmsnorm_row.argtypes = [i32, vp, vp, dbl, vp]
         lib.oracle_project_row.argtypes = [i32, i32, vp, vp, vp, vp]
         lib.oracle_rope_head.argtypes = [i32, dbl, i32, vp, vp, vp]
+        lib.oracle_head_rmsnorm.argtypes = [i32, vp, dbl, vp]
         lib.oracle_build_tokens.argtypes = [ctypes.POINTER(_Cfg), vp, i32, vp, vp, vp, vp, vp,
-                                            vp, vp, vp, vp, i64, vp, i32, vp, vp, vp, vp, vp]
+                                            vp, vp, vp, vp, vp, i64, vp, i32, vp, vp, vp, vp, vp]
         lib.oracle_build_tokens.restype = i32
         lib.oracle_num_threads.restype = i32
         _lib = lib
@@ -108,13 +112,23 @@ def project_row(W, b, n):
     return out
 
 
-def rope_head(x, pos3, theta: float, mrope: bool = False, section=(0, 0, 0)):
+def rope_head(x, pos3, theta: float, mrope=False, section=(0, 0, 0)):
+    """RoPE of one head. ``mrope``: False / "1d", True / "mrope" (contiguous sections) or
+    "mrope_interleaved"."""
     x = _f64(x).copy()
     p3 = np.zeros(3)
     p3[:len(np.atleast_1d(pos3))] = np.atleast_1d(pos3)
     sec = (ctypes.c_int * 3)(*section)
-    _load().oracle_rope_head(x.shape[0], float(theta), int(bool(mrope)), ctypes.addressof(sec),
-                             _p(p3), _p(x))
+    mode = _ROPE_MODES[mrope] if isinstance(mrope, str) else int(bool(mrope))
+    _load().oracle_rope_head(x.shape[0], float(theta), mode, ctypes.addressof(sec), _p(p3), _p(x))
+    return x
+
+
+def head_rmsnorm(x, gain, eps: float):
+    """Per-head K normalisation of one head x[D_h] with bf16-bit gain [D_h]."""
+    x = _f64(x).copy()
+    g = _u16(gain)
+    _load().oracle_head_rmsnorm(x.shape[0], _p(g), float(eps), _p(x))
     return x
 
 
@@ -123,15 +137,16 @@ def build_tokens(inp, tokens=None, want=("k", "v"), layers=None):
     (default: all, in order).
 
     ``inp`` carries ``cfg`` (d, n_layers, n_kv_heads, head_dim, rank, rope, rope_theta,
-    mrope_section, rms_eps, n_vis, adapter) and the bf16-bit arrays x0, D, U, gamma, Wk, Wv,
-    bk, bv and int32 pos [B][P][N_v]. Returns a dict of fp64 arrays: k, v [n][Ls][kv], m, n [n][Ls][d],
+    mrope_section, rms_eps, n_vis, adapter, k_norm, k_norm_eps) and the bf16-bit arrays x0, D,
+    U, gamma, Wk, Wv, bk, bv, kgamma and int32 pos [B][P][N_v]. Returns a dict of fp64 arrays: k, v [n][Ls][kv], m, n [n][Ls][d],
     h [n][Ls][r] (Ls = number of evaluated layers), for the names in ``want``.
     """
     cfg = inp.cfg
     c = _Cfg(cfg.d, cfg.n_layers, cfg.n_kv_heads, cfg.head_dim, cfg.rank,
-             1 if cfg.rope == "mrope" else 0, float(cfg.rope_theta),
+             _ROPE_MODES[cfg.rope], float(cfg.rope_theta),
              (ctypes.c_int * 3)(*cfg.mrope_section), float(cfg.rms_eps),
-             1 if getattr(cfg, "adapter", "embedding") == "recurrent" else 0)
+             1 if getattr(cfg, "adapter", "embedding") == "recurrent" else 0,
+             1 if getattr(cfg, "k_norm", False) else 0, float(getattr(cfg, "k_norm_eps", 1e-6)))
     B = inp.x0.shape[0]
     if tokens is None:
         tokens = np.arange(B * cfg.n_vis, dtype=np.int64)
@@ -145,10 +160,11 @@ def build_tokens(inp, tokens=None, want=("k", "v"), layers=None):
     for name in want:
         out[name] = np.empty(shapes[name])
     arrs = [_u16(inp.x0), np.ascontiguousarray(inp.pos, dtype=np.int32), _u16(inp.D), _u16(inp.U),
-            _u16(inp.gamma), _u16(inp.Wk), _u16(inp.Wv), _u16(inp.bk), _u16(inp.bv)]
+            _u16(inp.gamma), _u16(inp.Wk), _u16(inp.Wv), _u16(inp.bk), _u16(inp.bv),
+            _u16(getattr(inp, "kgamma", None))]
     rc = _load().oracle_build_tokens(
         ctypes.byref(c), _p(arrs[0]), cfg.n_vis, _p(arrs[1]), _p(arrs[2]), _p(arrs[3]),
-        _p(arrs[4]), _p(arrs[5]), _p(arrs[6]), _p(arrs[7]), _p(arrs[8]), _p(tokens), nt,
+        _p(arrs[4]), _p(arrs[5]), _p(arrs[6]), _p(arrs[7]), _p(arrs[8]), _p(arrs[9]), _p(tokens), nt,
         _p(lay), 0 if lay is None else int(lay.shape[0]), _p(out.get("k")), _p(out.get("v")), _p(out.get("m")), _p(out.get("h")), _p(out.get("n")))
     if rc != 0:
         raise ValueError("oracle_build_tokens rejected its arguments")

@@ -29,8 +29,14 @@
  *
  * RoPE reading: rotate-half pairs (j, j + D_h/2) of each head, inverse frequency
  * theta^(-2j/D_h); the angle of pair j is p * theta^(-2j/D_h), where p is the 1-D
- * position, or for M-RoPE the (t, h, w) position selected by the contiguous section
- * that j falls in (sections s0, s1, s2 with s0 + s1 + s2 = D_h / 2).
+ * position, or for M-RoPE the (t, h, w) position of the axis that frequency j belongs to:
+ * contiguous sections (j < s0 -> t, then s1 of h, then s2 of w), or the interleaved layout
+ * of Qwen3-VL backbones (j = 1 mod 3 with j < 3 s1 -> h, j = 2 mod 3 with j < 3 s2 -> w,
+ * every other j -> t).
+ *
+ * Per-head K normalisation (Qwen3-VL backbones normalise each key head before RoPE, the
+ * "query normalization" the paper's default backbone applies): when enabled, each head of
+ * k (after the bias) becomes g * k_h / sqrt(mean(k_h^2) + eps_k), g the layer's gain [D_h].
  *
  * Every input is a bf16 bit pattern widened exactly to double; every step runs in double.
  * Tokens are independent of each other (every step above acts on one row), so the only
@@ -53,6 +59,8 @@ typedef struct {
   int mrope_section[3];
   double rms_eps;
   int recurrent;       /* 0: embedding adapter (Sec. 3.1 Eq. 5), 1: recurrent (Eq. 6) */
+  int k_norm;          /* 1: per-head RMSNorm of K before RoPE */
+  double k_norm_eps;
 } oracle_cfg;
 
 static double bf16_to_f64(uint16_t b) {
@@ -101,18 +109,38 @@ void oracle_project_row(int d, int kv, const uint16_t* W, const uint16_t* b, con
   }
 }
 
+/* Axis (0 = t, 1 = h, 2 = w) of frequency j under M-RoPE layout `mrope`
+ * (1: contiguous sections, 2: interleaved). */
+static int mrope_axis(int mrope, const int* section, int j) {
+  if (mrope == 1) {
+    if (j >= section[0] + section[1]) return 2;
+    if (j >= section[0]) return 1;
+    return 0;
+  }
+  if (j % 3 == 1 && j < 3 * section[1]) return 1;
+  if (j % 3 == 2 && j < 3 * section[2]) return 2;
+  return 0;
+}
+
+/* Per-head RMSNorm of a key head x[head_dim] with gain g (bf16 [head_dim]):
+ * x_j <- g_j * x_j / sqrt(mean(x^2) + eps). */
+void oracle_head_rmsnorm(int head_dim, const uint16_t* g, double eps, double* x) {
+  double ss = 0.0;
+  for (int j = 0; j < head_dim; ++j) ss += x[j] * x[j];
+  const double inv = 1.0 / sqrt(ss / (double)head_dim + eps);
+  for (int j = 0; j < head_dim; ++j) x[j] = bf16_to_f64(g[j]) * x[j] * inv;
+}
+
 /* Rotary position embedding of one head (rotate-half pairs (j, j + D/2)).
- * pos3 holds the position of each axis: pos3[0] for 1-D RoPE; (t, h, w) for M-RoPE,
- * where pair j takes the axis whose contiguous section contains j. */
+ * pos3 holds the position of each axis: pos3[0] for 1-D RoPE (mrope = 0); (t, h, w) for
+ * M-RoPE (mrope = 1 contiguous sections, 2 interleaved), where pair j takes its axis's
+ * position. */
 void oracle_rope_head(int head_dim, double theta, int mrope, const int* section,
                       const double* pos3, double* x) {
   int half = head_dim / 2;
   for (int j = 0; j < half; ++j) {
     double p = pos3[0];
-    if (mrope) {
-      if (j >= section[0] + section[1]) p = pos3[2];
-      else if (j >= section[0]) p = pos3[1];
-    }
+    if (mrope) p = pos3[mrope_axis(mrope, section, j)];
     double a = p * pow(theta, -2.0 * (double)j / (double)head_dim);
     double c = cos(a), s = sin(a);
     double x1 = x[j], x2 = x[j + half];
@@ -125,7 +153,8 @@ void oracle_rope_head(int head_dim, double theta, int mrope, const int* section,
  * Sec. 3.2 Eq. 7 and the RoPE reading above), written at output index o. */
 static void memory_outputs(const oracle_cfg* c, int l, const double* m, const double* h,
                            const uint16_t* gamma, const uint16_t* Wk, const uint16_t* Wv,
-                           const uint16_t* bk, const uint16_t* bv, const double* p3, int64_t o,
+                           const uint16_t* bk, const uint16_t* bv, const uint16_t* kgamma,
+                           const double* p3, int64_t o,
                            double* g, double* n, double* kk, double* vv, double* k_out,
                            double* v_out, double* m_out, double* h_out, double* n_out) {
   const int d = c->d, r = c->rank, Dh = c->head_dim, kv = c->n_kv_heads * Dh;
@@ -133,6 +162,9 @@ static void memory_outputs(const oracle_cfg* c, int l, const double* m, const do
   oracle_rmsnorm_row(d, m, g, c->rms_eps, n);
   oracle_project_row(d, kv, Wk + (int64_t)l * kv * d, bk ? bk + (int64_t)l * kv : NULL, n, kk);
   oracle_project_row(d, kv, Wv + (int64_t)l * kv * d, bv ? bv + (int64_t)l * kv : NULL, n, vv);
+  if (c->k_norm)
+    for (int hh = 0; hh < c->n_kv_heads; ++hh)
+      oracle_head_rmsnorm(Dh, kgamma + (int64_t)l * Dh, c->k_norm_eps, kk + hh * Dh);
   for (int hh = 0; hh < c->n_kv_heads; ++hh)
     oracle_rope_head(Dh, c->rope_theta, c->rope, c->mrope_section, p3, kk + hh * Dh);
   if (k_out) memcpy(k_out + o * kv, kk, sizeof(double) * kv);
@@ -148,7 +180,8 @@ static void memory_outputs(const oracle_cfg* c, int l, const double* m, const do
 static int build_tokens_recurrent(const oracle_cfg* c, const uint16_t* x0, int n_vis,
                                   const int32_t* pos, const uint16_t* D, const uint16_t* U,
                                   const uint16_t* gamma, const uint16_t* Wk, const uint16_t* Wv,
-                                  const uint16_t* bk, const uint16_t* bv, const int64_t* tokens,
+                                  const uint16_t* bk, const uint16_t* bv, const uint16_t* kgamma,
+                                  const int64_t* tokens,
                                   int64_t n_tokens, const int32_t* layers, int Ls,
                                   double* k_out, double* v_out, double* m_out, double* h_out,
                                   double* n_out) {
@@ -181,7 +214,7 @@ static int build_tokens_recurrent(const oracle_cfg* c, const uint16_t* x0, int n
         oracle_adapter_row(d, r, prev, D + (int64_t)l * r * d, U + (int64_t)l * d * r, z, h, m);
         for (int s = 0; s < Ls; ++s)
           if ((layers ? layers[s] : s) == l)
-            memory_outputs(c, l, m, h, gamma, Wk, Wv, bk, bv, p3, q * Ls + s, g, n, kk, vv,
+            memory_outputs(c, l, m, h, gamma, Wk, Wv, bk, bv, kgamma, p3, q * Ls + s, g, n, kk, vv,
                            k_out, v_out, m_out, h_out, n_out);
         memcpy(prev, m, sizeof(double) * d);
       }
@@ -194,7 +227,8 @@ static int build_tokens_recurrent(const oracle_cfg* c, const uint16_t* x0, int n
 /*
  * The whole build for a list of tokens.
  *   x0    bf16 [B][n_vis][d];   pos int32 [B][P][n_vis], P = 1 (1-D) or 3 (M-RoPE)
- *   D [L][r][d], U [L][d][r], gamma [L][d], Wk/Wv [L][kv][d], bk/bv [L][kv] or NULL
+ *   D [L][r][d], U [L][d][r], gamma [L][d], Wk/Wv [L][kv][d], bk/bv [L][kv] or NULL,
+ *   kgamma [L][D_h] per-head K-norm gain (read when cfg->k_norm)
  *   tokens: flat token ids t = b * n_vis + i;  n_tokens of them
  *   layers: the layers to evaluate (n_sel_layers of them), or NULL for all L in order
  * Outputs (each may be NULL), indexed by the position q of the token in `tokens` and the
@@ -205,7 +239,8 @@ static int build_tokens_recurrent(const oracle_cfg* c, const uint16_t* x0, int n
 int oracle_build_tokens(const oracle_cfg* c, const uint16_t* x0, int n_vis, const int32_t* pos,
                         const uint16_t* D, const uint16_t* U, const uint16_t* gamma,
                         const uint16_t* Wk, const uint16_t* Wv, const uint16_t* bk,
-                        const uint16_t* bv, const int64_t* tokens, int64_t n_tokens,
+                        const uint16_t* bv, const uint16_t* kgamma, const int64_t* tokens,
+                        int64_t n_tokens,
                         const int32_t* layers, int n_sel_layers,
                         double* k_out, double* v_out, double* m_out, double* h_out,
                         double* n_out) {
@@ -214,6 +249,7 @@ int oracle_build_tokens(const oracle_cfg* c, const uint16_t* x0, int n_vis, cons
   const int kv = c->n_kv_heads * Dh;
   const int P = c->rope ? 3 : 1;
   if (d <= 0 || L <= 0 || r <= 0 || Dh <= 0 || (Dh & 1) || n_vis <= 0) return -1;
+  if (c->rope < 0 || c->rope > 2 || (c->k_norm && !kgamma)) return -1;
   if (c->rope && c->mrope_section[0] + c->mrope_section[1] + c->mrope_section[2] != Dh / 2)
     return -1;
   const int Ls = layers ? n_sel_layers : L;
@@ -221,8 +257,8 @@ int oracle_build_tokens(const oracle_cfg* c, const uint16_t* x0, int n_vis, cons
   for (int s = 0; layers && s < Ls; ++s)
     if (layers[s] < 0 || layers[s] >= L) return -1;
   if (c->recurrent) return build_tokens_recurrent(c, x0, n_vis, pos, D, U, gamma, Wk, Wv, bk, bv,
-                                                 tokens, n_tokens, layers, Ls, k_out, v_out,
-                                                 m_out, h_out, n_out);
+                                                 kgamma, tokens, n_tokens, layers, Ls, k_out,
+                                                 v_out, m_out, h_out, n_out);
 #pragma omp parallel
   {
     double* x = malloc(sizeof(double) * d);
@@ -244,8 +280,8 @@ int oracle_build_tokens(const oracle_cfg* c, const uint16_t* x0, int n_vis, cons
         oracle_adapter_row(d, r, x, D + (int64_t)l * r * d, U + (int64_t)l * d * r, z, h, m);
         double p3[3];
         for (int a = 0; a < P; ++a) p3[a] = (double)pos[(b * P + a) * n_vis + i];
-        memory_outputs(c, l, m, h, gamma, Wk, Wv, bk, bv, p3, q * Ls + ls, g, n, kk, vv, k_out,
-                       v_out, m_out, h_out, n_out);
+        memory_outputs(c, l, m, h, gamma, Wk, Wv, bk, bv, kgamma, p3, q * Ls + ls, g, n, kk, vv,
+                       k_out, v_out, m_out, h_out, n_out);
       }
     }
     free(x); free(m); free(n); free(g); free(z); free(h); free(kk); free(vv);

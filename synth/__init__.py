@@ -25,6 +25,7 @@ _lib = None
 
 # Counter streams, one per tensor, so that changing one shape never shifts another tensor.
 STREAM_X0, STREAM_D, STREAM_U, STREAM_GAMMA, STREAM_WK, STREAM_WV, STREAM_BK, STREAM_BV = range(8)
+STREAM_KGAMMA = 8
 
 
 def build(force: bool = False) -> str:
@@ -114,7 +115,7 @@ class Config:
     rank: int
     n_vis: int
     batch: int
-    rope: str             # "1d" or "mrope"
+    rope: str             # "1d", "mrope" (contiguous sections) or "mrope_interleaved"
     rope_theta: float
     mrope_section: tuple = (0, 0, 0)
     rms_eps: float = 1e-6
@@ -128,6 +129,9 @@ class Config:
     grid: tuple = ()            # (frames, rows, cols) of the visual grid, M-RoPE only
     ar1_rho: float = 0.0        # > 0: frame-correlated x0 (video), per token-in-frame element
     adapter: str = "embedding"  # "embedding" (Sec. 3.1 Eq. 5) or "recurrent" (Sec. 3.1 Eq. 6)
+    k_norm: bool = False        # per-head RMSNorm of K before RoPE (Qwen3-VL backbones)
+    k_norm_eps: float = 1e-6
+    k_norm_sigma: float = 0.1   # per-head K-norm gain = 1 + N(0, k_norm_sigma)
     description: str = ""
 
     @property
@@ -140,7 +144,7 @@ class Config:
 
     @property
     def n_pos(self) -> int:
-        return 3 if self.rope == "mrope" else 1
+        return 1 if self.rope == "1d" else 3
 
     def flops(self) -> float:
         """Plain-definition FLOPs of one build: 4*d*r + 4*d*kv per token and layer."""
@@ -177,6 +181,14 @@ CONFIGS = {
         rms_eps=1e-6, x0_sigma=0.5, seed=3, pos_start=15, grid=(1, 36, 36),
         description="Qwen2.5-VL-7B-shaped image: d=3584, L=28, GQA 28/4x128, r=128, N_v=1296 "
                     "(36x36), batch 4, M-RoPE [16,24,24] over a 1x36x36 grid"),
+    "qwen3vl_4b_image": Config(
+        name="qwen3vl_4b_image", d=2560, n_layers=36, n_heads=32, n_kv_heads=8, head_dim=128,
+        rank=128, n_vis=1024, batch=4, rope="mrope_interleaved", rope_theta=5e6,
+        mrope_section=(24, 20, 20), rms_eps=1e-6, x0_sigma=0.5, seed=5, pos_start=15,
+        grid=(1, 32, 32), k_norm=True,
+        description="Qwen3-VL-4B-shaped image (the paper's default backbone): d=2560, L=36, "
+                    "GQA 32/8x128, r=128, N_v=1024 (32x32), batch 4, interleaved M-RoPE "
+                    "[24,20,20], per-head K RMSNorm"),
     "qwen25vl_7b_video": Config(
         name="qwen25vl_7b_video", d=3584, n_layers=28, n_heads=28, n_kv_heads=4, head_dim=128,
         rank=256, n_vis=16384, batch=1, rope="mrope", rope_theta=1e6, mrope_section=(16, 24, 24),
@@ -185,7 +197,8 @@ CONFIGS = {
                     "(32 frames x 16x32), batch 1, M-RoPE over a 32x16x32 grid, frame-correlated x0"),
 }
 
-CONFIG_ORDER = ["tiny", "llava15_7b", "llava_next_7b", "qwen25vl_7b_image", "qwen25vl_7b_video"]
+CONFIG_ORDER = ["tiny", "llava15_7b", "llava_next_7b", "qwen25vl_7b_image", "qwen25vl_7b_video",
+                "qwen3vl_4b_image"]
 
 
 def config(name: str, **overrides) -> Config:
@@ -225,6 +238,7 @@ class Inputs:
     bk: np.ndarray | None = None  # [L][kv]
     bv: np.ndarray | None = None
     pos: np.ndarray = field(default=None)  # int32 [B][P][N_v]
+    kgamma: np.ndarray | None = None  # [L][head_dim] per-head K-norm gain (k_norm configs)
 
 
 def make_x0(cfg: Config) -> np.ndarray:
@@ -258,6 +272,9 @@ def make_inputs(cfg: Config, with_x0: bool = True) -> Inputs:
     if cfg.bias_sigma > 0:
         bk = normal_bf16(s, STREAM_BK, (L, kv), 0.0, cfg.bias_sigma)
         bv = normal_bf16(s, STREAM_BV, (L, kv), 0.0, cfg.bias_sigma)
+    kgamma = None
+    if cfg.k_norm:
+        kgamma = normal_bf16(s, STREAM_KGAMMA, (L, cfg.head_dim), 1.0, cfg.k_norm_sigma)
     x0 = make_x0(cfg) if with_x0 else None
     return Inputs(cfg=cfg, x0=x0, D=D, U=U, gamma=gamma, Wk=Wk, Wv=Wv, bk=bk, bv=bv,
-                  pos=positions(cfg))
+                  pos=positions(cfg), kgamma=kgamma)

@@ -27,7 +27,24 @@ MUTANTS = {
     "rope_wrong_direction": ("x[j] = x1 * c - x2 * s;", "x[j] = x1 * c + x2 * s;"),
     "rope_interleaved_pairs": ("double x1 = x[j], x2 = x[j + half];", "double x1 = x[2 * j], x2 = x[2 * j + 1];"),
     "rope_frequency_exponent": ("pow(theta, -2.0 * (double)j / (double)head_dim)", "pow(theta, -(double)j / (double)head_dim)"),
-    "mrope_axes_swapped": ("if (j >= section[0] + section[1]) p = pos3[2];", "if (j >= section[0] + section[1]) p = pos3[1];"),
+    "mrope_axes_swapped": ("if (j >= section[0] + section[1]) return 2;", "if (j >= section[0] + section[1]) return 1;"),
+    "mrope_interleave_offset": ("if (j % 3 == 1 && j < 3 * section[1]) return 1;",
+                                "if (j % 3 == 0 && j < 3 * section[1]) return 1;"),
+    "k_norm_over_whole_vector": ("oracle_head_rmsnorm(Dh, kgamma + (int64_t)l * Dh, c->k_norm_eps, kk + hh * Dh);",
+                                 "{ if (hh == 0) { double ss = 0.0; for (int j = 0; j < kv; ++j) ss += kk[j] * kk[j]; "
+                                 "const double inv = 1.0 / sqrt(ss / kv + c->k_norm_eps); for (int j = 0; j < kv; ++j) "
+                                 "kk[j] *= bf16_to_f64(kgamma[(int64_t)l * Dh + j % Dh]) * inv; } }"),
+    "k_norm_after_rope": ("  if (c->k_norm)\n    for (int hh = 0; hh < c->n_kv_heads; ++hh)\n"
+                          "      oracle_head_rmsnorm(Dh, kgamma + (int64_t)l * Dh, c->k_norm_eps, kk + hh * Dh);\n"
+                          "  for (int hh = 0; hh < c->n_kv_heads; ++hh)\n"
+                          "    oracle_rope_head(Dh, c->rope_theta, c->rope, c->mrope_section, p3, kk + hh * Dh);",
+                          "  for (int hh = 0; hh < c->n_kv_heads; ++hh)\n"
+                          "    oracle_rope_head(Dh, c->rope_theta, c->rope, c->mrope_section, p3, kk + hh * Dh);\n"
+                          "  if (c->k_norm)\n    for (int hh = 0; hh < c->n_kv_heads; ++hh)\n"
+                          "      oracle_head_rmsnorm(Dh, kgamma + (int64_t)l * Dh, c->k_norm_eps, kk + hh * Dh);"),
+    "k_norm_without_gain": ("x[j] = bf16_to_f64(g[j]) * x[j] * inv;", "x[j] = x[j] * inv;"),
+    "k_norm_mean_as_sum": ("const double inv = 1.0 / sqrt(ss / (double)head_dim + eps);",
+                           "const double inv = 1.0 / sqrt(ss + eps);"),
     "value_rotated": ("oracle_rope_head(Dh, c->rope_theta, c->rope, c->mrope_section, p3, kk + hh * Dh);",
                       "{ oracle_rope_head(Dh, c->rope_theta, c->rope, c->mrope_section, p3, kk + hh * Dh); "
                       "oracle_rope_head(Dh, c->rope_theta, c->rope, c->mrope_section, p3, vv + hh * Dh); }"),
@@ -37,8 +54,8 @@ MUTANTS = {
                                    "prev[j] = 0.0;"),
     "recurrent_down_of_next_layer": ("oracle_adapter_row(d, r, prev, D + (int64_t)l * r * d,",
                                      "oracle_adapter_row(d, r, prev, D + (int64_t)((l + 1) % L) * r * d,"),
-    "recurrent_outputs_previous_state": ("memory_outputs(c, l, m, h, gamma, Wk, Wv, bk, bv, p3, q * Ls + s,",
-                                         "memory_outputs(c, l, prev, h, gamma, Wk, Wv, bk, bv, p3, q * Ls + s,"),
+    "recurrent_outputs_previous_state": ("memory_outputs(c, l, m, h, gamma, Wk, Wv, bk, bv, kgamma, p3, q * Ls + s,",
+                                         "memory_outputs(c, l, prev, h, gamma, Wk, Wv, bk, bv, kgamma, p3, q * Ls + s,"),
 }
 
 

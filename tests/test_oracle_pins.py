@@ -419,3 +419,70 @@ def test_recurrent_layer_subset_matches_full_run():
     part = oracle.build_tokens(inp, np.array([4, 1]), layers=[3, 1])
     assert np.array_equal(part["k"][0, 0], full["k"][4, 3]) and np.array_equal(part["k"][1, 1], full["k"][1, 1])
     assert np.array_equal(part["v"][0, 1], full["v"][4, 1])
+
+
+# ---------------------------------------------------------------- Qwen3-VL backbone variant
+# Per-head RMSNorm of K before RoPE and the interleaved M-RoPE frequency layout.
+
+def test_k_norm_hand_example_norm_before_rope():
+    # x0 = [1, 0, 0, 0], eps = 0: RMSNorm gives n = [2, 0, 0, 0]. W_K = 2 I: k = [4, 0, 0, 0]
+    # (head rms 2), normalised to [2, 0, 0, 0], times the gain g = [2, 1, 1, 1]: [4, 0, 0, 0].
+    # Then RoPE at p = 1 turns pair (0, 2) by 1 rad: K = [4 cos 1, 0, 4 sin 1, 0]. (Rotating
+    # first and normalising after would give [4 cos 1, 0, 2 sin 1, 0].) V = 2 n is not normed.
+    cfg = _tiny_cfg(k_norm=True, k_norm_eps=0.0)
+    inp = _inputs(cfg, x0=[[[1, 0, 0, 0]]], D=np.zeros((1, 2, 4)), U=np.zeros((1, 4, 2)),
+                  gamma=[[1, 1, 1, 1]], Wk=[2 * np.eye(4)], Wv=[2 * np.eye(4)], pos=[[[1]]])
+    inp.kgamma = bf(np.array([[2.0, 1.0, 1.0, 1.0]]))
+    out = oracle.build_tokens(inp)
+    np.testing.assert_allclose(out["k"][0, 0], [4 * math.cos(1.0), 0, 4 * math.sin(1.0), 0],
+                               rtol=1e-14, atol=1e-15)
+    np.testing.assert_allclose(out["v"][0, 0], [4.0, 0, 0, 0], rtol=0, atol=0)
+
+
+def test_k_norm_closed_form_rms_and_head_independence():
+    # Gain 1 and position 0: every key head has rms 1 (eps 0). Scaling the W_K rows of head 0
+    # by 4 leaves every head unchanged (each head is normed on its own).
+    cfg = synth.config("tiny", n_vis=8, pos_start=0, k_norm=True, k_norm_eps=0.0, k_norm_sigma=0.0)
+    inp = synth.make_inputs(cfg)
+    inp.pos[:] = 0
+    a = oracle.build_tokens(inp)
+    kh = a["k"].reshape(cfg.tokens, cfg.n_layers, cfg.n_kv_heads, cfg.head_dim)
+    np.testing.assert_allclose(np.sqrt(np.mean(kh * kh, axis=-1)), 1.0, rtol=1e-12)
+    Wk = synth.bf16_to_f32(inp.Wk).astype(np.float64)
+    Wk[:, :cfg.head_dim] *= 4.0                                 # head 0 of every layer, exact in bf16
+    inp.Wk = bf(Wk)
+    b = oracle.build_tokens(inp)
+    np.testing.assert_allclose(b["k"], a["k"], rtol=1e-12, atol=1e-14)
+    np.testing.assert_array_equal(b["v"], a["v"])
+
+
+def test_k_norm_leaves_values_alone():
+    cfg = synth.config("tiny", n_vis=8, k_norm=True)
+    inp = synth.make_inputs(cfg)
+    plain = oracle.build_tokens(dataclasses.replace(inp, cfg=synth.config("tiny", n_vis=8)))
+    normed = oracle.build_tokens(inp)
+    np.testing.assert_array_equal(plain["v"], normed["v"])
+    assert not np.allclose(plain["k"], normed["k"])
+
+
+def test_interleaved_mrope_equal_axes_is_1d():
+    x = np.random.default_rng(5).normal(size=128)
+    for p in (0, 15, 51):
+        np.testing.assert_allclose(oracle.rope_head(x, (p, p, p), 5e6, "mrope_interleaved",
+                                                    (24, 20, 20)),
+                                   oracle.rope_head(x, p, 5e6), rtol=0, atol=0)
+
+
+def test_interleaved_mrope_mapping():
+    # D = 16 (8 pairs), sections (t, h, w) = (4, 2, 2): h takes j = 1, 4 (j = 1 mod 3, j < 6),
+    # w takes j = 2, 5 (j = 2 mod 3, j < 6), t takes j = 0, 3, 6, 7.
+    sec, theta = (4, 2, 2), 10000.0
+    owner = [0, 1, 2, 0, 1, 2, 0, 0]
+    for axis in range(3):
+        pos = [0, 0, 0]
+        pos[axis] = 5
+        for j in range(8):
+            y = oracle.rope_head(_basis(16, j), pos, theta, "mrope_interleaved", sec)
+            a = 5 * theta ** (-2.0 * j / 16) if owner[j] == axis else 0.0
+            assert y[j] == pytest.approx(math.cos(a), abs=1e-15)
+            assert y[j + 8] == pytest.approx(math.sin(a), abs=1e-15)
