@@ -10,7 +10,8 @@
  *     K_l = RoPE(W_K,l RMSNorm_l(M_l) [+ b_K,l]),  V_l = W_V,l RMSNorm_l(M_l) [+ b_V,l]
  *                                               (Sec. 3.2, Eq. 7; RMSNorm per App. K; RoPE
  *                                                at the original visual positions)
- * and stores them as bf16 into a caller-owned KV cache. Visual tokens get no query,
+ * (with k_norm, each head of K is RMS-normalised with a learned gain before RoPE), and stores
+ * them as bf16 into a caller-owned KV cache. Visual tokens get no query,
  * attention output or feed-forward update (Sec. 3.2), so K/V entries are the only output.
  *
  * Conventions for every entry point:
@@ -47,7 +48,11 @@ enum {
   DV_LAYER_IDENTITY = 1,  /* adapter skipped, M_l = E: visual K/V still built from E */
   DV_LAYER_DROP = 2       /* adapter and visual memory skipped: no K/V entries for this layer */
 };
-enum { DV_ROPE_1D = 0, DV_ROPE_MROPE = 1 };
+/* Rotary embedding of visual keys: 1-D positions, or M-RoPE (t, h, w) with the frequency
+ * pairs split into contiguous sections (t first, then h, then w) or interleaved as in
+ * Qwen3-VL backbones (pair j follows h when j = 1 mod 3 and j < 3 s_h, w when j = 2 mod 3
+ * and j < 3 s_w, t otherwise). */
+enum { DV_ROPE_1D = 0, DV_ROPE_MROPE = 1, DV_ROPE_MROPE_INTERLEAVED = 2 };
 /* How M_l is formed from the visual embeddings E (Sec. 3.1). */
 enum {
   DV_ADAPTER_EMBEDDING = 0,  /* M_l = A_l(E) for every layer (Eq. 5) */
@@ -59,8 +64,9 @@ enum {
  *   1 <= n_kv_heads, n_kv_heads * head_dim <= 8192 and a multiple of 128;
  *   1 <= n_layers <= 256;
  *   act == DV_ACT_SILU;  rope_theta > 0;  rms_eps >= 0;
- *   DV_ROPE_MROPE: mrope_section[i] >= 0 and their sum == head_dim / 2 (contiguous sections
- *   of the frequency index: t first, then h, then w);
+ *   DV_ROPE_MROPE / DV_ROPE_MROPE_INTERLEAVED: mrope_section[i] >= 0 and their sum ==
+ *   head_dim / 2 (interleaved: the layout must give each axis exactly its section's count);
+ *   k_norm in {0, 1}; k_norm_eps >= 0;
  *   adapter in {DV_ADAPTER_EMBEDDING, DV_ADAPTER_RECURRENT};
  *   max_batch * max_n_vis >= 1 and <= 2^24 (the tokens one build may carry). */
 typedef struct dv_config {
@@ -72,12 +78,16 @@ typedef struct dv_config {
   int act;               /* DV_ACT_SILU */
   int rope;              /* DV_ROPE_1D or DV_ROPE_MROPE */
   float rope_theta;      /* RoPE base */
-  int mrope_section[3];  /* frequency pairs per axis (t, h, w); DV_ROPE_MROPE only */
+  int mrope_section[3];  /* frequency pairs per axis (t, h, w); M-RoPE modes only */
   float rms_eps;         /* epsilon inside the RMSNorm square root */
   int max_batch;         /* largest batch a build may pass */
   int max_n_vis;         /* largest number of visual tokens per batch element */
   int has_kv_bias;       /* 1: weights carry b_K, b_V; 0: no bias */
   int adapter;           /* DV_ADAPTER_EMBEDDING or DV_ADAPTER_RECURRENT */
+  int k_norm;            /* 1: each key head is RMS-normalised before RoPE, with the gain
+                            dv_weights.k_norm_gamma (the per-head K norm of Qwen3-VL backbones,
+                            applied after the bias) */
+  float k_norm_eps;      /* epsilon inside that norm's square root */
 } dv_config;
 
 /* Weights of all L layers, bf16, device pointers. Read only during dv_memory_plan: the plan
@@ -87,6 +97,7 @@ typedef struct dv_config {
  *   gamma  [L][d]       gain of the frozen input RMSNorm LN_l (Sec. 3.2 Eq. 7)
  *   Wk, Wv [L][kv][d]   frozen key / value projections W_K,l, W_V,l (kv = n_kv_heads*head_dim)
  *   bk, bv [L][kv]      biases, or NULL when has_kv_bias == 0
+ *   k_norm_gamma [L][head_dim]  gain of the per-head K norm when k_norm == 1, else NULL
  *   layer_mode          HOST array of L DV_LAYER_* values, or NULL for DV_LAYER_ADAPTER at every
  *                       layer (App. J skips the adapters of early and late layers). Layers in
  *                       DV_LAYER_DROP get no K/V entries: builds leave their cache rows untouched,
@@ -103,6 +114,7 @@ typedef struct dv_weights {
   const void* bk;
   const void* bv;
   const unsigned char* layer_mode;
+  const void* k_norm_gamma;
 } dv_weights;
 
 /* Destination KV cache (bf16, caller-owned). Element (layer l, batch b, slot s, head h, j) of
@@ -142,7 +154,7 @@ int dv_memory_plan(const dv_config* cfg, const dv_weights* w, void* stream, dv_p
  * adapter the state M_l is carried in fp32 from layer to layer; each layer's K/V read its
  * bf16 rounding.
  *   x0     bf16 [batch][n_vis][d]: the visual embeddings E (Sec. 2 Eq. 1); 16-byte aligned
- *   pos    int32 [batch][P][n_vis], P = 1 (DV_ROPE_1D) or 3 (DV_ROPE_MROPE: t, h, w): the
+ *   pos    int32 [batch][P][n_vis], P = 1 (DV_ROPE_1D) or 3 (M-RoPE modes: t, h, w): the
  *          original positions of the visual tokens (Sec. 1 and App. H keep them unchanged)
  *   slot   int32 [batch][n_vis] cache slot of each token, or NULL for slot0 + i
  *   slot0  first slot when slot == NULL

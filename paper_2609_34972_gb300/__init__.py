@@ -11,7 +11,8 @@ is missing, every call raises.
 Tensor layouts (bf16 unless stated, all on the current CUDA device):
     x0      [B, N_v, d]          visual embeddings E (Sec. 2 Eq. 1)
     pos     int32 [B, P, N_v]    P = 1 (1-D RoPE) or 3 (M-RoPE t, h, w)
-    weights D [L, r, d], U [L, d, r], gamma [L, d], Wk, Wv [L, kv, d], bk, bv [L, kv] (optional)
+    weights D [L, r, d], U [L, d, r], gamma [L, d], Wk, Wv [L, kv, d], bk, bv [L, kv] (optional),
+            kgamma [L, D_h] (per-head K-norm gain, with k_norm)
     k/v cache [L, B_c, S, H_kv, D_h] or any strided view with D_h contiguous
 """
 from __future__ import annotations
@@ -33,6 +34,8 @@ DV_ERR_UNSUPPORTED_DEVICE = 7
 DV_ACT_SILU = 0
 DV_ROPE_1D = 0
 DV_ROPE_MROPE = 1
+DV_ROPE_MROPE_INTERLEAVED = 2
+_ROPE = {"1d": DV_ROPE_1D, "mrope": DV_ROPE_MROPE, "mrope_interleaved": DV_ROPE_MROPE_INTERLEAVED}
 DV_LAYER_ADAPTER = 0
 DV_LAYER_IDENTITY = 1
 DV_LAYER_DROP = 2
@@ -55,12 +58,13 @@ class DvConfig(ctypes.Structure):
                 ("rope", ctypes.c_int), ("rope_theta", ctypes.c_float),
                 ("mrope_section", ctypes.c_int * 3), ("rms_eps", ctypes.c_float),
                 ("max_batch", ctypes.c_int), ("max_n_vis", ctypes.c_int),
-                ("has_kv_bias", ctypes.c_int), ("adapter", ctypes.c_int)]
+                ("has_kv_bias", ctypes.c_int), ("adapter", ctypes.c_int),
+                ("k_norm", ctypes.c_int), ("k_norm_eps", ctypes.c_float)]
 
 
 class DvWeights(ctypes.Structure):
     _fields_ = [(n, ctypes.c_void_p) for n in ("D", "U", "gamma", "Wk", "Wv", "bk", "bv",
-                                               "layer_mode")]
+                                               "layer_mode", "k_norm_gamma")]
 
 
 class DvKVCache(ctypes.Structure):
@@ -137,16 +141,21 @@ def _ptr(t):
 
 def make_config(d, n_layers, n_kv_heads, head_dim, rank, rope="1d", rope_theta=10000.0,
                 mrope_section=(0, 0, 0), rms_eps=1e-6, max_batch=1, max_n_vis=1,
-                has_kv_bias=False, adapter="embedding") -> DvConfig:
+                has_kv_bias=False, adapter="embedding", k_norm=False,
+                k_norm_eps=1e-6) -> DvConfig:
     """``adapter``: "embedding" (M_l = A_l(E), Sec. 3.1 Eq. 5) or "recurrent"
-    (M_l = A_l(M_{l-1}), Sec. 3.1 Eq. 6)."""
+    (M_l = A_l(M_{l-1}), Sec. 3.1 Eq. 6). ``rope``: "1d", "mrope" (contiguous sections) or
+    "mrope_interleaved". ``k_norm``: per-head RMSNorm of K before RoPE (weights["kgamma"])."""
     if adapter not in ("embedding", "recurrent"):
         raise ValueError(f"unknown adapter {adapter!r}")
+    if rope not in _ROPE:
+        raise ValueError(f"unknown rope {rope!r}")
     return DvConfig(int(d), int(n_layers), int(n_kv_heads), int(head_dim), int(rank),
-                    DV_ACT_SILU, DV_ROPE_MROPE if rope == "mrope" else DV_ROPE_1D,
+                    DV_ACT_SILU, _ROPE[rope],
                     float(rope_theta), (ctypes.c_int * 3)(*mrope_section), float(rms_eps),
                     int(max_batch), int(max_n_vis), int(bool(has_kv_bias)),
-                    DV_ADAPTER_RECURRENT if adapter == "recurrent" else DV_ADAPTER_EMBEDDING)
+                    DV_ADAPTER_RECURRENT if adapter == "recurrent" else DV_ADAPTER_EMBEDDING,
+                    int(bool(k_norm)), float(k_norm_eps))
 
 
 class Plan:
@@ -178,7 +187,8 @@ def memory_plan(cfg: DvConfig, weights: dict, stream=None, layer_modes=None) -> 
             raise ValueError("layer_modes needs one entry per layer")
         modes = (ctypes.c_ubyte * cfg.n_layers)(*[int(m) for m in layer_modes])
     w = DvWeights(*[_ptr(weights.get(n)) for n in ("D", "U", "gamma", "Wk", "Wv", "bk", "bv")],
-                  ctypes.cast(modes, ctypes.c_void_p) if modes is not None else None)
+                  ctypes.cast(modes, ctypes.c_void_p) if modes is not None else None,
+                  _ptr(weights.get("kgamma")))
     h = ctypes.c_void_p()
     _check(lib().dv_memory_plan(ctypes.byref(cfg), ctypes.byref(w), _stream_handle(stream),
                                 ctypes.byref(h)), "dv_memory_plan")

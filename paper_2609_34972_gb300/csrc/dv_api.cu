@@ -37,6 +37,7 @@ struct dv_plan {
   uint16_t* Uup = nullptr;     // recurrent adapter: U_l as [L*d][r_pad]
   float* bk = nullptr;
   float* bv = nullptr;
+  float* kg = nullptr;         // per-head K-norm gain fp32 [L][head_dim] (k_norm)
   void* ws = nullptr;          // workspace of a build of max_tokens tokens (carve_workspace)
   long long last_tokens = 0;   // tokens of the last build (layout of the workspace)
   int* status = nullptr;
@@ -259,7 +260,7 @@ __global__ void __launch_bounds__(256) k_rank_product(const uint16_t* __restrict
   }
 }
 
-// out[i][c] = b[src[i]][c] in fp32.
+// out[i][c] = b[src[i]][c] in fp32 (K/V biases, K-norm gains: c < kv).
 __global__ void k_bias_to_f32(const uint16_t* __restrict__ b, float* __restrict__ out, int L,
                               int kv, PackLayers pl) {
   const long long n = static_cast<long long>(L) * kv;
@@ -342,10 +343,28 @@ int grid_for(long long n) {
 bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 bool aligned2(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 1u) == 0; }
 
+}  // namespace
+
+// Position axis (0 t, 1 h, 2 w) of rotary frequency pair j: contiguous M-RoPE sections, or
+// the interleaved layout (j = 1 mod 3 below 3 s_h -> h, j = 2 mod 3 below 3 s_w -> w, else t).
+int dv::rope_axis(int rope, const int* sec, int j) {
+  if (rope == DV_ROPE_MROPE) return j < sec[0] ? 0 : (j < sec[0] + sec[1] ? 1 : 2);
+  if (rope == DV_ROPE_MROPE_INTERLEAVED) {
+    if (j % 3 == 1 && j < 3 * sec[1]) return 1;
+    if (j % 3 == 2 && j < 3 * sec[2]) return 2;
+  }
+  return 0;
+}
+
+namespace {
+
 int check_config(const dv_config* c) {
   if (!c) return DV_ERR_INVALID_ARG;
   if (c->act != DV_ACT_SILU) return DV_ERR_INVALID_ARG;
-  if (c->rope != DV_ROPE_1D && c->rope != DV_ROPE_MROPE) return DV_ERR_INVALID_ARG;
+  if (c->rope != DV_ROPE_1D && c->rope != DV_ROPE_MROPE && c->rope != DV_ROPE_MROPE_INTERLEAVED)
+    return DV_ERR_INVALID_ARG;
+  if (c->k_norm != 0 && c->k_norm != 1) return DV_ERR_INVALID_ARG;
+  if (!(c->k_norm_eps >= 0.0f) || !std::isfinite(c->k_norm_eps)) return DV_ERR_INVALID_ARG;
   if (c->d <= 0 || c->n_layers <= 0 || c->n_kv_heads <= 0 || c->head_dim <= 0 || c->rank <= 0 ||
       c->max_batch <= 0 || c->max_n_vis <= 0)
     return DV_ERR_INVALID_ARG;
@@ -362,16 +381,19 @@ int check_config(const dv_config* c) {
   if ((c->n_kv_heads * c->head_dim) % 128 != 0) return DV_ERR_UNSUPPORTED_SHAPE;
   if (c->n_layers > 256) return DV_ERR_UNSUPPORTED_SHAPE;
   if (static_cast<long long>(c->max_batch) * c->max_n_vis > (1LL << 24)) return DV_ERR_UNSUPPORTED_SHAPE;
-  if (c->rope == DV_ROPE_MROPE) {
+  if (c->rope == DV_ROPE_MROPE || c->rope == DV_ROPE_MROPE_INTERLEAVED) {
     const int* s = c->mrope_section;
     if (s[0] < 0 || s[1] < 0 || s[2] < 0) return DV_ERR_INVALID_ARG;
     if (s[0] + s[1] + s[2] != c->head_dim / 2) return DV_ERR_UNSUPPORTED_SHAPE;
+    int count[3] = {0, 0, 0};
+    for (int j = 0; j < c->head_dim / 2; ++j) ++count[dv::rope_axis(c->rope, s, j)];
+    if (count[0] != s[0] || count[1] != s[1] || count[2] != s[2]) return DV_ERR_UNSUPPORTED_SHAPE;
   }
   return DV_OK;
 }
 
 void free_plan_memory(dv_plan* p) {
-  void* ptrs[] = {p->Dst, p->Bn, p->Wkv, p->Uup, p->bk, p->bv, p->ws, p->status};
+  void* ptrs[] = {p->Dst, p->Bn, p->Wkv, p->Uup, p->bk, p->bv, p->kg, p->ws, p->status};
   for (void* q : ptrs)
     if (q) cudaFree(q);
   for (cudaEvent_t e : p->ev) cudaEventDestroy(e);
@@ -447,9 +469,10 @@ static void fill_epi_kv(const PlanView& v, const BuildArgs& a, long long T, EpiK
   e.slot = a.slot;
   e.slot0 = a.slot0;
   e.n_vis = a.n_vis;
-  e.n_pos = v.rope == DV_ROPE_MROPE ? 3 : 1;
-  e.sec0 = v.rope == DV_ROPE_MROPE ? v.mrope_section[0] : HD / 2;
-  e.sec01 = v.rope == DV_ROPE_MROPE ? v.mrope_section[0] + v.mrope_section[1] : HD / 2;
+  e.n_pos = v.rope == DV_ROPE_1D ? 1 : 3;
+  for (int j = 0; j < HD / 2; ++j) e.axis[j] = static_cast<uint8_t>(rope_axis(v.rope, v.mrope_section, j));
+  e.kg = v.kg;
+  e.k_eps = v.k_eps;
   e.kc = static_cast<uint16_t*>(const_cast<void*>(a.kc));
   e.vc = static_cast<uint16_t*>(const_cast<void*>(a.vc));
   e.s_layer = a.s_layer;
@@ -671,6 +694,8 @@ bool plan_view(const dv_plan* p, PlanView* v) {
   v->d = c.d;
   v->n_layers = p->n_active;
   v->adapter = c.adapter;
+  v->kg = p->kg;
+  v->k_eps = c.k_norm_eps;
   v->head_dim = c.head_dim;
   v->rope = c.rope;
   for (int i = 0; i < 3; ++i) v->mrope_section[i] = c.mrope_section[i];
@@ -732,6 +757,8 @@ int dv_memory_plan(const dv_config* cfg, const dv_weights* w, void* stream, dv_p
   for (const void* q : wp)
     if (!aligned2(q)) return DV_ERR_ALIGNMENT;
   if (cfg->has_kv_bias && (!aligned2(w->bk) || !aligned2(w->bv))) return DV_ERR_ALIGNMENT;
+  if (cfg->k_norm && !w->k_norm_gamma) return DV_ERR_INVALID_ARG;
+  if (cfg->k_norm && !aligned2(w->k_norm_gamma)) return DV_ERR_ALIGNMENT;
 
   int n_active = 0;
   for (int l = 0; l < cfg->n_layers; ++l) {
@@ -787,6 +814,7 @@ int dv_memory_plan(const dv_config* cfg, const dv_weights* w, void* stream, dv_p
             dmalloc(&p->ws, ws_bytes) && dmalloc(&p->status, sizeof(int));
   if (ok && cfg->has_kv_bias)
     ok = dmalloc(&p->bk, sizeof(float) * L * p->kv) && dmalloc(&p->bv, sizeof(float) * L * p->kv);
+  if (ok && cfg->k_norm) ok = dmalloc(&p->kg, sizeof(float) * L * HD);
   if (!ok) {
     free_plan_memory(p);
     delete p;
@@ -826,6 +854,9 @@ int dv_memory_plan(const dv_config* cfg, const dv_weights* w, void* stream, dv_p
     k_bias_to_f32<<<grid_for(1LL * L * p->kv), 256, 0, st>>>(static_cast<const uint16_t*>(w->bv),
                                                              p->bv, L, p->kv, pl);
   }
+  if (cfg->k_norm)
+    k_bias_to_f32<<<grid_for(1LL * L * HD), 256, 0, st>>>(
+        static_cast<const uint16_t*>(w->k_norm_gamma), p->kg, L, HD, pl);
   cudaError_t err = cudaGetLastError();
   if (err == cudaSuccess) err = cudaStreamSynchronize(st);
   if (err != cudaSuccess) {

@@ -175,17 +175,51 @@ __device__ __forceinline__ KvToken kv_token(const GemmParams& p, int l, int t) {
   return k;
 }
 
-// K block q (0..3) of a 128-channel group for one token: r[m] and r[16 + m] (m < 16) are the
-// accumulators of rotate-half pair p = 16q + m (Wkv K-row permutation). Writes k = rstd * acc
-// + b_K, rotated, as two 32-byte runs of the head row.
+// K values of block q (0..3) of a 128-channel group for one token: r[m] and r[16 + m]
+// (m < 16) are the accumulators of rotate-half pair p = 16q + m (Wkv K-row permutation); the
+// key channels are x1 = rstd * r[m] + b_K (channel j of head hl) and x2 = rstd * r[16 + m] + b_K
+// (channel j + HD/2), j = (16q + m) mod HD/2.
 template <int HD>
-__device__ __forceinline__ void kv_store_k16(const GemmParams& p, const KvToken& tk, int l, int g,
-                                             int q, const uint32_t (&r)[32]) {
+__device__ __forceinline__ void k_pair_values(const GemmParams& p, const KvToken& tk, int l,
+                                              int g, int q, const uint32_t (&r)[32], int m,
+                                              float& x1, float& x2) {
   constexpr int kHalf = HD / 2;
   const EpiKV& e = p.kv;
   const int hl = (16 * q) / kHalf, j0 = (16 * q) % kHalf;
-  const int c1 = hl * HD + j0;  // channel of the first lower half within the group
-  const float* bk = e.bk ? e.bk + static_cast<size_t>(l) * e.kv + g * 128 : nullptr;
+  x1 = __uint_as_float(r[m]) * tk.rs;
+  x2 = __uint_as_float(r[16 + m]) * tk.rs;
+  if (e.bk) {
+    const float* bk = e.bk + static_cast<size_t>(l) * e.kv + g * 128 + hl * HD + j0;
+    x1 += bk[m];
+    x2 += bk[kHalf + m];
+  }
+}
+
+// Sum of squares of the 32 key channels of block q (the head's share for its K norm).
+template <int HD>
+__device__ __forceinline__ float kv_k16_sumsq(const GemmParams& p, const KvToken& tk, int l, int g,
+                                              int q, const uint32_t (&r)[32]) {
+  float ss = 0.0f;
+#pragma unroll
+  for (int m = 0; m < 16; ++m) {
+    float x1, x2;
+    k_pair_values<HD>(p, tk, l, g, q, r, m, x1, x2);
+    ss = fmaf(x1, x1, ss);
+    ss = fmaf(x2, x2, ss);
+  }
+  return ss;
+}
+
+// K block q (0..3) of a 128-channel group for one token: k = rstd * acc + b_K (k_pair_values),
+// with the per-head K norm when enabled (kinv = 1 / sqrt(mean(k_h^2) + eps) of this head, times
+// the gain of each channel), rotated, and written as two 32-byte runs of the head row.
+template <int HD>
+__device__ __forceinline__ void kv_store_k16(const GemmParams& p, const KvToken& tk, int l, int g,
+                                             int q, const uint32_t (&r)[32], float kinv) {
+  constexpr int kHalf = HD / 2;
+  const EpiKV& e = p.kv;
+  const int hl = (16 * q) / kHalf, j0 = (16 * q) % kHalf;
+  const float* kg = e.kg ? e.kg + static_cast<size_t>(l) * HD : nullptr;
   uint32_t plo[8], phi[8];
 #pragma unroll
   for (int m = 0; m < 16; m += 2) {
@@ -193,13 +227,14 @@ __device__ __forceinline__ void kv_store_k16(const GemmParams& p, const KvToken&
 #pragma unroll
     for (int w = 0; w < 2; ++w) {
       const int j = j0 + m + w;
-      float x1 = __uint_as_float(r[m + w]) * tk.rs;
-      float x2 = __uint_as_float(r[16 + m + w]) * tk.rs;
-      if (bk) {
-        x1 += bk[c1 + m + w];
-        x2 += bk[c1 + kHalf + m + w];
+      float x1, x2;
+      k_pair_values<HD>(p, tk, l, g, q, r, m + w, x1, x2);
+      if (kg) {
+        x1 *= kinv * kg[j];
+        x2 *= kinv * kg[kHalf + j];
       }
-      const float pj = j < e.sec0 ? tk.pt : (j < e.sec01 ? tk.ph : tk.pw);
+      const int ax = e.axis[j];
+      const float pj = ax == 0 ? tk.pt : (ax == 1 ? tk.ph : tk.pw);
       float s, cs;
       rope_sincos(pj, e.inv_freq_hi[j], e.inv_freq_lo[j], e, s, cs);
       y1[w] = x1 * cs - x2 * s;
@@ -244,13 +279,31 @@ template <int HD>
 __device__ __forceinline__ void epi_kv_group(const GemmParams& p, uint32_t tbase, int l, int g,
                                              int t) {
   const KvToken tk = kv_token(p, l, t);
+  // Per-head K norm: a first pass over the K blocks sums each head's squares (one head per
+  // group for HD = 128, blocks {0, 1} and {2, 3} for HD = 64).
+  float kinv0 = 1.0f, kinv1 = 1.0f;  // heads of blocks {0, 1} and {2, 3} (the same for HD = 128)
+  if (p.kv.kg) {
+    float ss0 = 0.0f, ss1 = 0.0f;
+#pragma unroll 1
+    for (int q = 0; q < 4; ++q) {
+      uint32_t r[32];
+      __syncwarp();
+      tmem_ld32(tbase + 32 * q, r);
+      tmem_ld_wait();
+      const float part = kv_k16_sumsq<HD>(p, tk, l, g, q, r);
+      if (HD == 128 || q < 2) ss0 += part;
+      else ss1 += part;
+    }
+    kinv0 = rsqrtf(fmaf(ss0, 1.0f / HD, p.kv.k_eps));
+    kinv1 = HD == 128 ? kinv0 : rsqrtf(fmaf(ss1, 1.0f / HD, p.kv.k_eps));
+  }
 #pragma unroll 1
   for (int q = 0; q < 4; ++q) {
     uint32_t r[32];
     __syncwarp();
     tmem_ld32(tbase + 32 * q, r);
     tmem_ld_wait();
-    kv_store_k16<HD>(p, tk, l, g, q, r);
+    kv_store_k16<HD>(p, tk, l, g, q, r, (HD == 128 || q < 2) ? kinv0 : kinv1);
   }
 #pragma unroll 1
   for (int q = 0; q < 4; ++q) {

@@ -68,7 +68,9 @@ struct EpiKV {
   int slot0;
   int n_vis;
   int n_pos;          // 1 or 3
-  int sec0, sec01;    // M-RoPE: pairs [0,sec0) -> t, [sec0,sec01) -> h, rest -> w
+  const float* kg;    // per-head K-norm gain fp32 [L][head_dim], or null (no K norm)
+  float k_eps;
+  uint8_t axis[kMaxHalfHead];  // position axis (0 t, 1 h, 2 w) of each frequency pair
   uint16_t* kc;
   uint16_t* vc;
   long long s_layer, s_batch, s_seq, s_head;
@@ -150,11 +152,17 @@ int down_splits(long long m_tiles, int k_slabs, int num_sms);
 int kv_pair_tile_n(long long tokens);
 int kv_pair_smem_bytes(int nt);
 
+// Position axis (0 t, 1 h, 2 w) of rotary frequency pair j for rope mode `rope` (DV_ROPE_*)
+// and M-RoPE sections `sec` (t, h, w).
+int rope_axis(int rope, const int* sec, int j);
+
 // Read-only view of a plan's repacked weights and shape, for build variants outside dv_api.cu.
 struct PlanView {
   int d, n_layers, head_dim, rope, mrope_section[3];  // n_layers: layers the plan holds
   int adapter;                                         // DV_ADAPTER_*
   float rms_eps;
+  const float* kg;                 // per-head K-norm gain [L][head_dim], or null
+  float k_eps;
   int num_sms, r_pad, kv, k_total;
   const float* bk;
   const float* bv;

@@ -238,7 +238,19 @@ __global__ void __launch_bounds__(kPairThreads, 1)
         }
         const KvToken tk = kv_token(p, l, nt * NT + c * 32 + lane);
         if (rank == 0) {
-          kv_store_k16<HD>(p, tk, l, g, q, r);
+          float kinv = 1.0f;
+          if (p.kv.kg) {
+            // Per-head K norm: a head spans warps (4 blocks of 32 channels for HD = 128,
+            // 2 for HD = 64). Each warp leaves its block's sum of squares in the unused pad
+            // columns of the token's staging row; the head's blocks are summed in block order.
+            float* pad = staging + lane * kStagePitch + 128;
+            pad[q] = kv_k16_sumsq<HD>(p, tk, l, g, q, r);
+            named_barrier(1, kEpiPairThreads);
+            const float ss = HD == 128 ? ((pad[0] + pad[1]) + pad[2]) + pad[3]
+                                       : (q < 2 ? pad[0] + pad[1] : pad[2] + pad[3]);
+            kinv = rsqrtf(fmaf(ss, 1.0f / HD, p.kv.k_eps));
+          }
+          kv_store_k16<HD>(p, tk, l, g, q, r, kinv);
         } else {
           kv_store_v32<HD>(p, tk, l, g, q, r);
         }

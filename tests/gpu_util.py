@@ -30,6 +30,8 @@ def device_weights(inp, device="cuda"):
     if inp.bk is not None:
         w["bk"] = torch_bf16(inp.bk, device)
         w["bv"] = torch_bf16(inp.bv, device)
+    if getattr(inp, "kgamma", None) is not None:
+        w["kgamma"] = torch_bf16(inp.kgamma, device)
     return w
 
 
@@ -39,7 +41,8 @@ def dv_config(cfg, max_batch=None, max_n_vis=None):
                           rope=cfg.rope, rope_theta=cfg.rope_theta,
                           mrope_section=cfg.mrope_section, rms_eps=cfg.rms_eps,
                           max_batch=max_batch or cfg.batch, max_n_vis=max_n_vis or cfg.n_vis,
-                          has_kv_bias=cfg.bias_sigma > 0, adapter=cfg.adapter)
+                          has_kv_bias=cfg.bias_sigma > 0, adapter=cfg.adapter,
+                          k_norm=cfg.k_norm, k_norm_eps=cfg.k_norm_eps)
 
 
 def run_build(inp, plan=None, seq_len=None, batch_cache=None, slot=None, slot0=0, fill=0.0,

@@ -55,7 +55,8 @@ def test_null_arguments_rejected(dv):
     ("d", 100, 2), ("d", 0, 1), ("rank", 0, 1), ("rank", 300, 2), ("head_dim", 96, 2),
     ("n_layers", -1, 1), ("act", 3, 1), ("rope", 5, 1), ("max_batch", 0, 1),
     ("rope_theta", -1.0, 1), ("rms_eps", -1e-6, 1), ("n_kv_heads", 129, 2),
-    ("adapter", 2, 1), ("adapter", -1, 1),
+    ("adapter", 2, 1), ("adapter", -1, 1), ("rope", 3, 1), ("k_norm", 2, 1),
+    ("k_norm_eps", -1.0, 1),
 ])
 def test_bad_config_rejected_before_device(dv, field, value, code):
     cfg = dv.make_config(512, 4, 8, 64, 16, max_batch=1, max_n_vis=64)
@@ -72,6 +73,27 @@ def test_mrope_sections_must_cover_half_head(dv):
     w = dv.DvWeights(*([ctypes.c_void_p(256)] * 5 + [None, None, None]))
     h = ctypes.c_void_p()
     assert dv.lib().dv_memory_plan(ctypes.byref(cfg), ctypes.byref(w), None, ctypes.byref(h)) == 2
+
+
+@pytest.mark.parametrize("sections", [(16, 24, 24), (20, 22, 22), (10, 27, 27)])
+def test_interleaved_mrope_sections_must_match_the_layout(dv, sections):
+    # The interleaved layout over 64 pairs gives h the pairs j = 1 mod 3 below 3 s_h and w the
+    # pairs j = 2 mod 3 below 3 s_w. These sections sum to 64 but the layout cannot give each
+    # axis its count (e.g. (16, 24, 24) would need pair 71), so the plan is refused before
+    # any device work. (24, 20, 20), the Qwen3-VL layout, is accepted on the GPU.
+    cfg = dv.make_config(512, 4, 8, 128, 16, rope="mrope_interleaved", mrope_section=sections,
+                         max_batch=1, max_n_vis=64)
+    w = dv.DvWeights(*([ctypes.c_void_p(256)] * 5 + [None, None, None, None]))
+    h = ctypes.c_void_p()
+    rc = dv.lib().dv_memory_plan(ctypes.byref(cfg), ctypes.byref(w), None, ctypes.byref(h))
+    assert rc == dv.DV_ERR_UNSUPPORTED_SHAPE and not h.value
+
+
+def test_k_norm_needs_its_gain(dv):
+    cfg = dv.make_config(512, 4, 8, 64, 16, max_batch=1, max_n_vis=64, k_norm=True)
+    w = dv.DvWeights(*([ctypes.c_void_p(256)] * 5 + [None, None, None, None]))
+    h = ctypes.c_void_p()
+    assert dv.lib().dv_memory_plan(ctypes.byref(cfg), ctypes.byref(w), None, ctypes.byref(h)) == 1
 
 
 def test_missing_weights_rejected(dv):
