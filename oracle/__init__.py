@@ -63,6 +63,9 @@ def _load():
                                             vp, vp, vp, vp, vp, i64, vp, i32, vp, vp, vp, vp, vp]
         lib.oracle_build_tokens.restype = i32
         lib.oracle_num_threads.restype = i32
+        lib.oracle_text_attention.argtypes = [i32, i32, i32, i32, i32, i32, vp, vp, vp, vp, vp,
+                                              dbl, vp]
+        lib.oracle_text_attention.restype = i32
         _lib = lib
     return _lib
 
@@ -168,4 +171,21 @@ def build_tokens(inp, tokens=None, want=("k", "v"), layers=None):
         _p(lay), 0 if lay is None else int(lay.shape[0]), _p(out.get("k")), _p(out.get("v")), _p(out.get("m")), _p(out.get("h")), _p(out.get("n")))
     if rc != 0:
         raise ValueError("oracle_build_tokens rejected its arguments")
+    return out
+
+
+def text_attention(q, k, v, n_keys, q_slot, scale: float):
+    """Causal text-query attention over cache slots (Sec. 3.2): q [B][Hq][Nt][D], k, v
+    [B][S][Hkv][D] (fp64-convertible), n_keys int [B], q_slot int [B][Nt]. Returns fp64
+    [B][Hq][Nt][D]."""
+    q, k, v = _f64(q), _f64(k), _f64(v)
+    B, Hq, Nt, D = q.shape
+    S, Hkv = k.shape[1], k.shape[2]
+    nk = np.ascontiguousarray(n_keys, dtype=np.int32)
+    qs = np.ascontiguousarray(q_slot, dtype=np.int32)
+    out = np.empty_like(q)
+    rc = _load().oracle_text_attention(B, Hq, Hkv, Nt, S, D, _p(q), _p(k), _p(v), _p(nk), _p(qs),
+                                       float(scale), _p(out))
+    if rc != 0:
+        raise ValueError("oracle_text_attention rejected its arguments")
     return out

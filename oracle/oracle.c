@@ -1,10 +1,12 @@
 /*
  * ORACLE — TEST INFRASTRUCTURE ONLY.
  *
- * A plain, slow, fp64 CPU statement of the embedding-adapter visual-memory build of
- * "Just MLPs: Efficient Visual State Reconstruction for Multimodal Language Models"
- * (delta-Vision). Only the tests, the smoke check and the benchmark's CPU-baseline leg
- * may load it. It shares no code, header, table or helper with the CUDA path.
+ * A plain, slow, fp64 CPU statement of the visual-memory build of "Just MLPs: Efficient
+ * Visual State Reconstruction for Multimodal Language Models" (delta-Vision), with the
+ * embedding or the recurrent adapter, and of its consumer, the text queries' causal attention
+ * over the visual and text keys/values (oracle_text_attention, at the end). Only the tests,
+ * the smoke check and the benchmark's CPU-baseline and reference legs may load it. It shares
+ * no code, header, table or helper with the CUDA path.
  *
  * What it computes, for every visual token row x = E_i (a row of the initial visual
  * embeddings, Sec. 2 Eq. 1) and every layer l, in this order:
@@ -298,4 +300,55 @@ int oracle_num_threads(void) {
     nt = omp_get_num_threads();
   }
   return nt;
+}
+
+/*
+ * Consumer of the visual memory (Sec. 3.2): text queries attend jointly to the visual
+ * keys/values and the text context, with the original causal structure, O = Attn(Q, [K^v; K^t],
+ * [V^v; V^t]). The sequence is a list of cache slots in order; query t of batch element b sits
+ * at slot q_slot[b][t] and sees slot s when s <= q_slot[b][t] and s < n_keys[b]. Grouped
+ * queries: query head hq reads key head hq / (n_q_heads / n_kv_heads).
+ *   q    [B][Hq][Nt][D];  k, v [B][S][Hkv][D] (slots);  out [B][Hq][Nt][D]   (all fp64)
+ *   o = sum_s softmax_s(scale * q . k_s) v_s over the visible slots; 0 when none is visible.
+ * Returns 0, or -1 on a bad argument.
+ */
+int oracle_text_attention(int B, int Hq, int Hkv, int Nt, int S, int D, const double* q,
+                          const double* k, const double* v, const int32_t* n_keys,
+                          const int32_t* q_slot, double scale, double* out) {
+  if (B <= 0 || Hq <= 0 || Hkv <= 0 || Hq % Hkv || Nt <= 0 || S <= 0 || D <= 0) return -1;
+  const int G = Hq / Hkv;
+#pragma omp parallel for collapse(3) schedule(dynamic, 1)
+  for (int b = 0; b < B; ++b) {
+    for (int hq = 0; hq < Hq; ++hq) {
+      for (int t = 0; t < Nt; ++t) {
+        const int h = hq / G;
+        const double* qr = q + (((int64_t)b * Hq + hq) * Nt + t) * D;
+        double* o = out + (((int64_t)b * Hq + hq) * Nt + t) * D;
+        int last = q_slot[(int64_t)b * Nt + t];
+        if (last >= n_keys[b]) last = n_keys[b] - 1;
+        if (last >= S) last = S - 1;
+        for (int j = 0; j < D; ++j) o[j] = 0.0;
+        if (last < 0) continue;
+        double mx = -INFINITY;
+        for (int s = 0; s <= last; ++s) {
+          const double* kr = k + (((int64_t)b * S + s) * Hkv + h) * D;
+          double dot = 0.0;
+          for (int j = 0; j < D; ++j) dot += qr[j] * kr[j];
+          if (scale * dot > mx) mx = scale * dot;
+        }
+        double den = 0.0;
+        for (int s = 0; s <= last; ++s) {
+          const double* kr = k + (((int64_t)b * S + s) * Hkv + h) * D;
+          const double* vr = v + (((int64_t)b * S + s) * Hkv + h) * D;
+          double dot = 0.0;
+          for (int j = 0; j < D; ++j) dot += qr[j] * kr[j];
+          const double w = exp(scale * dot - mx);
+          den += w;
+          for (int j = 0; j < D; ++j) o[j] += w * vr[j];
+        }
+        for (int j = 0; j < D; ++j) o[j] /= den;
+      }
+    }
+  }
+  return 0;
 }

@@ -43,6 +43,11 @@ MUTANTS = {
                           "  if (c->k_norm)\n    for (int hh = 0; hh < c->n_kv_heads; ++hh)\n"
                           "      oracle_head_rmsnorm(Dh, kgamma + (int64_t)l * Dh, c->k_norm_eps, kk + hh * Dh);"),
     "k_norm_without_gain": ("x[j] = bf16_to_f64(g[j]) * x[j] * inv;", "x[j] = x[j] * inv;"),
+    "attention_scale_dropped": ("const double w = exp(scale * dot - mx);", "const double w = exp(dot - mx);"),
+    "attention_causal_off_by_one": ("for (int s = 0; s <= last; ++s) {\n          const double* kr = k + (((int64_t)b * S + s) * Hkv + h) * D;\n          const double* vr",
+                                    "for (int s = 0; s < last; ++s) {\n          const double* kr = k + (((int64_t)b * S + s) * Hkv + h) * D;\n          const double* vr"),
+    "attention_group_mapping": ("const int h = hq / G;", "const int h = hq % Hkv;"),
+    "attention_not_normalised": ("for (int j = 0; j < D; ++j) o[j] /= den;", "(void)den;"),
     "k_norm_mean_as_sum": ("const double inv = 1.0 / sqrt(ss / (double)head_dim + eps);",
                            "const double inv = 1.0 / sqrt(ss + eps);"),
     "value_rotated": ("oracle_rope_head(Dh, c->rope_theta, c->rope, c->mrope_section, p3, kk + hh * Dh);",

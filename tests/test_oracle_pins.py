@@ -486,3 +486,75 @@ def test_interleaved_mrope_mapping():
             a = 5 * theta ** (-2.0 * j / 16) if owner[j] == axis else 0.0
             assert y[j] == pytest.approx(math.cos(a), abs=1e-15)
             assert y[j + 8] == pytest.approx(math.sin(a), abs=1e-15)
+
+
+# ---------------------------------------------------------------- consumer: text-query attention
+# Sec. 3.2: text queries attend causally to [K^v; K^t], [V^v; V^t] (slots in sequence order).
+
+def test_attention_single_visible_key_returns_its_value():
+    rng = np.random.default_rng(10)
+    q = rng.normal(size=(1, 2, 3, 8))
+    k = rng.normal(size=(1, 5, 1, 8))
+    v = rng.normal(size=(1, 5, 1, 8))
+    out = oracle.text_attention(q, k, v, [5], [[0, 0, 0]], 0.3)
+    np.testing.assert_array_equal(out, np.broadcast_to(v[0, 0, 0], out.shape))
+
+
+def test_attention_two_keys_hand_example_and_no_visible_key():
+    # q = e_0, keys 2 e_0 and 0, scale 1/2: scores 1 and 0, weights e/(e+1), 1/(e+1).
+    q = np.zeros((1, 1, 2, 4)); q[0, 0, :, 0] = 1.0
+    k = np.zeros((1, 3, 1, 4)); k[0, 0, 0, 0] = 2.0
+    v = np.zeros((1, 3, 1, 4)); v[0, 0, 0] = [1, 0, 0, 0]; v[0, 1, 0] = [0, 3, 0, 0]
+    out = oracle.text_attention(q, k, v, [3], [[1, -1]], 0.5)
+    e = math.e
+    np.testing.assert_allclose(out[0, 0, 0], [e / (e + 1), 3 / (e + 1), 0, 0], rtol=1e-15)
+    np.testing.assert_array_equal(out[0, 0, 1], 0.0)      # slot -1: nothing visible
+
+
+def test_attention_is_causal_and_respects_key_count():
+    # Changing what lies after a query's slot (or past n_keys) leaves its output unchanged.
+    rng = np.random.default_rng(11)
+    q = rng.normal(size=(2, 2, 4, 16))
+    k = rng.normal(size=(2, 12, 2, 16))
+    v = rng.normal(size=(2, 12, 2, 16))
+    n_keys, q_slot = [12, 9], [[3, 5, 8, 11], [2, 4, 8, 10]]
+    a = oracle.text_attention(q, k, v, n_keys, q_slot, 0.25)
+    k2, v2 = k.copy(), v.copy()
+    k2[0, 9:] += 5.0
+    v2[0, 9:] -= 3.0
+    k2[1, 9:] *= -2.0                                       # past n_keys of batch 1
+    b = oracle.text_attention(q, k2, v2, n_keys, q_slot, 0.25)
+    np.testing.assert_array_equal(a[0, :, :3], b[0, :, :3])
+    np.testing.assert_array_equal(a[1], b[1])
+    assert not np.allclose(a[0, :, 3], b[0, :, 3])
+
+
+def test_attention_grouped_heads_share_their_kv_head():
+    # Hq = 4 over Hkv = 2: heads 0, 1 read kv head 0 and heads 2, 3 kv head 1.
+    rng = np.random.default_rng(12)
+    q = np.broadcast_to(rng.normal(size=(1, 1, 2, 8)), (1, 4, 2, 8)).copy()
+    k = rng.normal(size=(1, 6, 2, 8))
+    v = rng.normal(size=(1, 6, 2, 8))
+    out = oracle.text_attention(q, k, v, [6], [[4, 5]], 0.35)
+    np.testing.assert_array_equal(out[0, 0], out[0, 1])
+    np.testing.assert_array_equal(out[0, 2], out[0, 3])
+    assert not np.allclose(out[0, 0], out[0, 2])
+
+
+def test_attention_matches_library_routine():
+    torch = pytest.importorskip("torch")
+    rng = np.random.default_rng(13)
+    B, Hq, Hkv, Nt, S, D = 2, 4, 2, 5, 20, 16
+    q = rng.normal(size=(B, Hq, Nt, D))
+    k = rng.normal(size=(B, S, Hkv, D))
+    v = rng.normal(size=(B, S, Hkv, D))
+    n_keys, q_slot = [20, 15], [[14, 15, 16, 18, 19], [3, 7, 9, 12, 14]]
+    got = oracle.text_attention(q, k, v, n_keys, q_slot, 0.25)
+    kk = torch.from_numpy(k).permute(0, 2, 1, 3).repeat_interleave(Hq // Hkv, dim=1)
+    vv = torch.from_numpy(v).permute(0, 2, 1, 3).repeat_interleave(Hq // Hkv, dim=1)
+    s = torch.arange(S)
+    mask = torch.stack([(s[None, :] <= torch.tensor(q_slot[b])[:, None]) & (s[None, :] < n_keys[b])
+                        for b in range(B)])[:, None]
+    ref = torch.nn.functional.scaled_dot_product_attention(torch.from_numpy(q), kk, vv,
+                                                           attn_mask=mask, scale=0.25)
+    np.testing.assert_allclose(got, ref.numpy(), rtol=1e-12, atol=1e-13)
