@@ -390,6 +390,94 @@ def run_dv(args):
         dist.destroy_process_group()
 
 
+def run_consumer(args):
+    """The consumer of the visual memory (Sec. 3.2): one step = the causal attention of the
+    prefill's text queries over every layer's cache (system-prompt text slots, the visual slots
+    written by the build, the text slots), through dv_text_attention, one launch per layer."""
+    import numpy as np
+    import torch
+    import synth
+    from paper_2609_34972_gb300.build import build_library
+    build_library()
+    import paper_2609_34972_gb300 as dv
+    from tests import gpu_util as gu
+    rank, world, local = dist_env()
+    if rank != 0:
+        return
+    torch.cuda.set_device(local)
+    cfg = workload_config(args)
+    n_sys, n_text, hq = args.consumer_sys, args.consumer_text, cfg.n_heads
+    B, Nv, H, D, L = cfg.batch, cfg.n_vis, cfg.n_kv_heads, cfg.head_dim, cfg.n_layers
+    S = n_sys + Nv + n_text
+    inp = synth.make_inputs(cfg)
+    k, v, plan = gu.run_build(inp, seq_len=S, slot0=n_sys)
+    gen = torch.Generator(device="cuda").manual_seed(7)
+    for l in range(L):
+        k[l, :, :n_sys].normal_(generator=gen)
+        v[l, :, :n_sys].normal_(generator=gen)
+        k[l, :, n_sys + Nv:].normal_(generator=gen)
+        v[l, :, n_sys + Nv:].normal_(generator=gen)
+    q = torch.randn((L, B, hq, n_text, D), generator=gen, device="cuda").to(torch.bfloat16)
+    out = torch.empty((B, hq, n_text, D), dtype=torch.bfloat16, device="cuda")
+    nk = torch.full((B,), S, dtype=torch.int32, device="cuda")
+    qs = (n_sys + Nv + torch.arange(n_text, dtype=torch.int32, device="cuda")).repeat(B, 1)
+    scale = 1.0 / D ** 0.5
+
+    def step():
+        for l in range(L):
+            dv.text_attention(q[l], k, v, l, nk, qs, scale, out=out)
+
+    for _ in range(args.warmup):
+        step()
+    torch.cuda.synchronize()
+    # A decoder calls the attention layer by layer; a serving engine replays that sequence as a
+    # CUDA graph, so the step is captured once and replayed (no per-call host cost in the timing).
+    graph = torch.cuda.CUDAGraph()
+    side = torch.cuda.Stream()
+    side.wait_stream(torch.cuda.current_stream())
+    with torch.cuda.stream(side):
+        step()
+    torch.cuda.current_stream().wait_stream(side)
+    with torch.cuda.graph(graph):
+        step()
+    graph.replay()
+    torch.cuda.synchronize()
+    clk = ClockSampler(os.environ.get("CUDA_VISIBLE_DEVICES", "").split(",")[0] or None)
+    clk.start()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record()
+    for _ in range(args.steps):
+        graph.replay()
+    e1.record()
+    torch.cuda.synchronize()
+    clocks = clk.stop()
+    assert dv.text_attention_status() == dv.DV_OK
+    ms = e0.elapsed_time(e1) / args.steps
+    # each query row sees all S slots (the text slots up to its own): keys read once per layer
+    kv_bytes = L * B * H * S * D * 2 * 2
+    qo_bytes = L * B * hq * n_text * D * 2 * 2
+    flops = sum(4.0 * B * hq * D * (n_sys + Nv + t + 1) for t in range(n_text)) * L
+    peaks, _ = load_peaks()
+    gbs = (kv_bytes + qo_bytes) / (ms * 1e-3) / 1e9
+    print(json.dumps({
+        "metric": "text-query attention over the visual memory: text tokens/s (all layers)",
+        "value": B * n_text / (ms * 1e-3), "unit": "text tokens/s", "n_gpus": 1,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
+        "dtype": "bf16", "data": "synthetic",
+        "config": {"workload": cfg.name + "_consumer", "layers": L, "batch": B,
+                   "slots": {"system": n_sys, "visual": Nv, "text": n_text},
+                   "q_heads": hq, "kv_heads": H, "head_dim": D,
+                   "l2": f"{(kv_bytes + qo_bytes) / 1e6:.0f} MB read per step (> L2)",
+                   "timing": "the step (one dv_text_attention per layer) captured in a CUDA graph "
+                             "and replayed"},
+        "roofline": {"bound": "hbm", "achieved": gbs, "peak": peaks["hbm_gbs"], "unit": "GB/s",
+                     "frac": gbs / peaks["hbm_gbs"], "traffic": None,
+                     "kernel": "dv_attn_kernel", "bytes_per_step": kv_bytes + qo_bytes,
+                     "tflops": flops / (ms * 1e-3) / 1e12},
+        "clocks": clocks, "gpu_launches": args.steps * L,
+    }), flush=True)
+
+
 def main():
     ap = argparse.ArgumentParser(description=__doc__, formatter_class=argparse.RawDescriptionHelpFormatter)
     ap.add_argument("--gpus", type=int, default=1)
@@ -405,6 +493,11 @@ def main():
                     help="embedding adapter (Sec. 3.1 Eq. 5, the default workload) or the "
                          "recurrent adapter (Eq. 6)")
     ap.add_argument("--impl", choices=["dv", "reference"], default="dv")
+    ap.add_argument("--consumer", action="store_true",
+                    help="measure the consumer instead: causal text-query attention over every "
+                         "layer's cache (dv_text_attention)")
+    ap.add_argument("--consumer-sys", type=int, default=35, help="system-prompt slots before the visual slots")
+    ap.add_argument("--consumer-text", type=int, default=64, help="text query tokens after them")
     ap.add_argument("--e2e-steps", type=int, default=100)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-budget-s", type=float, default=15.0)
@@ -415,6 +508,8 @@ def main():
         ap.error("--steps must be <= 4096 (per-stage timing records at most 4096 builds)")
     if args.impl == "reference":
         run_reference(args)
+    elif args.consumer:
+        run_consumer(args)
     else:
         run_dv(args)
 

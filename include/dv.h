@@ -202,6 +202,34 @@ int dv_build_visual_memory_noalloc(dv_plan* plan, const void* x0, int batch, int
  */
 int dv_plan_status(dv_plan* plan);
 
+/*
+ * dv_text_attention — the consumer of the visual memory (Sec. 3.2): the text queries of one
+ * layer attend jointly to the visual keys/values the build wrote and the text context, with
+ * the original causal structure: O = Attn(Q^t, [K^v; K^t], [V^v; V^t]). Reads the cache in
+ * place; needs no plan and allocates nothing.
+ *   q         bf16 [batch][n_q_heads][n_text][head_dim]: the text queries, already rotated
+ *   cache     the KV cache (the strides of dv_kv_cache); `layer` selects the layer
+ *   max_keys  slots per batch element the cache holds (slots >= max_keys are never read)
+ *   n_keys    int32 [batch]: slots 0 .. n_keys[b] - 1 hold keys (visual and text, in sequence
+ *             order); later slots are ignored
+ *   q_slot    int32 [batch][n_text]: the slot of each query's own token; query t sees slot s
+ *             when s <= q_slot[b][t] and s < n_keys[b] (it sees nothing when q_slot < 0)
+ *   scale     softmax scale (> 0), e.g. 1 / sqrt(head_dim)
+ *   out       bf16 [batch][n_q_heads][n_text][head_dim]; a query that sees no key gets zeros
+ * Query head hq reads key head hq / (n_q_heads / n_kv_heads). head_dim in {64, 128}. q and out
+ * 16-byte aligned; cache strides as for dv_build_visual_memory. batch * n_text == 0 is a no-op.
+ * Errors: DV_ERR_INVALID_ARG, DV_ERR_UNSUPPORTED_SHAPE, DV_ERR_ALIGNMENT,
+ * DV_ERR_UNSUPPORTED_DEVICE, DV_ERR_CUDA. Stream-ordered and asynchronous.
+ */
+int dv_text_attention(const void* q, int batch, int n_q_heads, int n_kv_heads, int n_text,
+                      int head_dim, const dv_kv_cache* cache, int layer, int max_keys,
+                      const int* n_keys, const int* q_slot, float scale, void* out, void* stream);
+
+/* dv_text_attention_status — synchronises the device, reads and clears the status word of the
+ * attention launches on the current device: DV_OK, or DV_ERR_DEVICE_TIMEOUT when a launch gave
+ * up on a wait (its output is then incomplete). */
+int dv_text_attention_status(void);
+
 /* dv_free — release the plan and everything it owns (synchronises the device first).
  * dv_free(NULL) is a no-op. */
 void dv_free(dv_plan* plan);

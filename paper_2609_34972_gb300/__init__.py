@@ -45,7 +45,7 @@ DV_ADAPTER_RECURRENT = 1
 EXPORTED = ["dv_memory_plan", "dv_build_visual_memory", "dv_plan_status", "dv_free",
             "dv_error_string", "dv_timing_enable", "dv_timing_read", "dv_kernels_per_build",
             "dv_debug_wait_timeout", "dv_debug_copy_workspace", "dv_build_visual_memory_noalloc",
-            "dv_debug_copy_memory", "dv_kv_engine"]
+            "dv_debug_copy_memory", "dv_kv_engine", "dv_text_attention", "dv_text_attention_status"]
 N_STAGES = 4
 STAGE_NAMES = ["row_sumsq", "down_proj_silu", "rms_stats", "kv_proj_rope_store"]
 # Stage names of a recurrent-adapter build (stage 0 is empty there).
@@ -104,10 +104,14 @@ def lib() -> ctypes.CDLL:
                                                      ctypes.POINTER(DvKVCache), vp]
         L.dv_debug_copy_memory.argtypes = [vp, i32, vp, vp]
         L.dv_kv_engine.argtypes = [vp, ctypes.c_longlong]
+        L.dv_text_attention.argtypes = [vp, i32, i32, i32, i32, i32, ctypes.POINTER(DvKVCache),
+                                        i32, i32, vp, vp, ctypes.c_float, vp, vp]
+        L.dv_text_attention_status.argtypes = []
         for name in ("dv_memory_plan", "dv_build_visual_memory", "dv_plan_status",
                      "dv_timing_enable", "dv_timing_read", "dv_kernels_per_build",
                      "dv_debug_wait_timeout", "dv_debug_copy_workspace",
-                     "dv_build_visual_memory_noalloc", "dv_debug_copy_memory", "dv_kv_engine"):
+                     "dv_build_visual_memory_noalloc", "dv_debug_copy_memory", "dv_kv_engine",
+                     "dv_text_attention", "dv_text_attention_status"):
             getattr(L, name).restype = i32
         _lib = L
     return _lib
@@ -284,6 +288,28 @@ def debug_memory(plan: Plan, tokens: int, stream=None):
     _check(lib().dv_debug_copy_memory(plan.handle, int(tokens), _ptr(mem), _stream_handle(stream)),
            "dv_debug_copy_memory")
     return mem
+
+
+def text_attention(q, k_cache, v_cache, layer: int, n_keys, q_slot, scale: float, out=None,
+                   stream=None):
+    """Causal attention of text queries over one layer of the cache (Sec. 3.2).
+
+    q: bf16 [B, Hq, Nt, D_h] (rotated); k_cache / v_cache: the [L, B_c, S, H_kv, D_h] cache views
+    the build writes; n_keys int32 [B]; q_slot int32 [B, Nt]. Returns bf16 [B, Hq, Nt, D_h]."""
+    import torch
+    B, Hq, Nt, D = (int(x) for x in q.shape)
+    kvc = kv_cache_view(k_cache, v_cache)
+    if out is None:
+        out = torch.empty((B, Hq, Nt, D), dtype=torch.bfloat16, device=q.device)
+    _check(lib().dv_text_attention(_ptr(q), B, Hq, int(k_cache.shape[3]), Nt, D, ctypes.byref(kvc),
+                                   int(layer), int(k_cache.shape[2]), _ptr(n_keys), _ptr(q_slot),
+                                   float(scale), _ptr(out), _stream_handle(stream)),
+           "dv_text_attention")
+    return out
+
+
+def text_attention_status() -> int:
+    return int(lib().dv_text_attention_status())
 
 
 KV_KERNELS = {1: "dv_kv_pair_kernel (weights as M, 2-SM UMMA)",

@@ -1,0 +1,637 @@
+// Consumer of the visual memory (Sec. 3.2): the text queries of one layer attend causally to
+// the keys/values of a KV cache that holds the visual K/V written by the build (and whatever
+// text K/V the caller stored), O = softmax(scale * Q K^T, causal) V, as a tcgen05 flash-
+// attention kernel. It reads the cache in place, through 4-D tensor maps over its strides
+// (head_dim, kv head, slot, batch), so it checks the build's cache layout end to end.
+//
+// One cluster of S CTAs (S = 1, 2, 4 or 8) handles 128 query rows of one (batch, kv head):
+// the rows of the kv head's query group (query head-major, then text token). The cluster's
+// key range (up to the last slot any of its rows may see) is split into S runs of 128-key
+// blocks. For each block a CTA:
+//   1. loads the K and V tiles by TMA (rows = slots, 128 B per 64 channels, 128-byte swizzle);
+//   2. one thread issues S = Q K^T (M = 128 rows, N = 128 keys, K = head_dim) into TMEM;
+//   3. the four warps transpose V into a K-major [head_dim][keys] tile (ldmatrix.trans /
+//      stmatrix), so both MMAs read K-major operands;
+//   4. each thread owns one query row: it reads its scores from TMEM twice (the block maximum,
+//      then exp2 of the masked, scaled scores), keeps the running maximum m and sum l, and
+//      writes the row's probabilities as bf16 into the A tile of the second MMA;
+//   5. one thread issues P V (N = head_dim) into TMEM; each thread rescales its fp32 output row
+//      (registers) by exp2(m_old - m_new) and adds the block.
+// The partial (O, m, l) of each CTA then go to shared memory, and after a cluster barrier CTA s
+// combines rows [s * 128 / S, (s + 1) * 128 / S) over the S partials through distributed
+// shared memory, in the fixed order 0..S-1, and stores bf16 rows. Every wait is bounded; a CTA
+// that gives up still passes both cluster barriers and flags the status word.
+#include <cmath>
+#include <mutex>
+
+#include "../../include/dv.h"
+#include "dv_internal.h"
+#include "dv_ptx.cuh"
+
+namespace dv {
+namespace {
+
+constexpr int kAttnThreads = 128;
+constexpr int kKeyBlock = 128;
+
+struct AttnParams {
+  int Hq, Hkv, Nt, G;
+  int rows_per_group;  // G * Nt query rows per kv head
+  int q_blocks;        // 128-row blocks of one group
+  int max_keys;
+  const int* n_keys;   // [B]
+  const int* q_slot;   // [B][Nt]
+  float scale_log2;    // softmax scale * log2(e): scores are kept in base 2
+  uint16_t* out;       // bf16 [B][Hq][Nt][head_dim]
+  unsigned long long timeout_ns;
+};
+
+// Device status word of the attention launches on this device (DV_ERR_DEVICE_TIMEOUT when a
+// wait gave up); read and cleared by dv_text_attention_status.
+__device__ int g_attn_status;
+
+template <int HD>
+struct AttnCfg {
+  static constexpr int kSlabs = HD / 64;
+  static constexpr int kTile = 128 * 128;        // 128 rows x 64 bf16 (one 128-byte-swizzled slab)
+  static constexpr int kKV = kSlabs * kTile;     // one K or V tile of 128 keys
+  static constexpr int kOffQ = 0;
+  static constexpr int kOffStage = kOffQ + kKV;  // two stages of [K | V]
+  static constexpr int kStage = 2 * kKV;
+  static constexpr int kOffVt = kOffStage + 2 * kStage;   // 2 key slabs of [HD rows][64 keys]
+  static constexpr int kVtSlab = HD * 128;
+  // P (2 key slabs of [128 rows][64 keys]) takes the K slot of the current stage when that is
+  // large enough (HD = 128): K is dead once the score MMA has completed.
+  static constexpr bool kPInK = kKV >= 2 * kTile;
+  static constexpr int kOffP = kOffVt + 2 * kVtSlab;
+  static constexpr int kEnd = kOffP + (kPInK ? 0 : 2 * kTile);
+  static constexpr int kPitch = HD + 4;                   // floats per partial output row
+  static constexpr int kPartBytes = 128 * kPitch * 4;
+  static constexpr int kMisc = 2048;                      // barriers, m, l, key end
+  static constexpr int kSmemBytes = kEnd + kMisc + 1024;
+  static_assert(kPartBytes <= 2 * kStage, "partial outputs reuse the stages");
+  static_assert(kVtSlab % 1024 == 0 && kKV % 1024 == 0, "tiles stay 1024-byte aligned");
+  static_assert(kSmemBytes <= 232448, "shared memory of one CTA");
+};
+
+// 4-D tiled load (c0 innermost); completion counted as transaction bytes on `bar`.
+__device__ __forceinline__ void tma_load_4d(uint32_t dst, const CUtensorMap* map, uint32_t bar,
+                                            int c0, int c1, int c2, int c3) {
+  asm volatile(
+      "cp.async.bulk.tensor.4d.shared::cluster.global.mbarrier::complete_tx::bytes"
+      " [%0], [%1, {%3, %4, %5, %6}], [%2];" ::"r"(dst),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(bar), "r"(c0), "r"(c1), "r"(c2), "r"(c3)
+      : "memory");
+}
+
+// Four 8x8 b16 matrices from shared memory, transposed (lanes 8i..8i+7 give the row
+// addresses of matrix i; register i receives this lane's fragment of its transpose).
+__device__ __forceinline__ void ldmatrix_x4_trans(uint32_t addr, uint32_t (&r)[4]) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0, %1, %2, %3}, [%4];"
+               : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
+               : "r"(addr)
+               : "memory");
+}
+
+// Four 8x8 b16 matrices to shared memory (same fragment and address convention).
+__device__ __forceinline__ void stmatrix_x4(uint32_t addr, const uint32_t (&r)[4]) {
+  asm volatile("stmatrix.sync.aligned.m8n8.x4.shared.b16 [%0], {%1, %2, %3, %4};" ::"r"(addr),
+               "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3])
+               : "memory");
+}
+
+// Orders this thread's generic-proxy shared-memory writes before later async-proxy reads
+// (tcgen05.mma operands) of the same memory.
+__device__ __forceinline__ void fence_proxy_async_smem() {
+  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+
+__device__ __forceinline__ uint32_t cluster_size() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%cluster_nctarank;" : "=r"(r));
+  return r;
+}
+
+__device__ __forceinline__ float ld_cluster_f32(uint32_t caddr) {
+  float v;
+  asm volatile("ld.shared::cluster.f32 %0, [%1];" : "=f"(v) : "r"(caddr) : "memory");
+  return v;
+}
+
+__device__ __forceinline__ float4 ld_cluster_f4(uint32_t caddr) {
+  float4 v;
+  asm volatile("ld.shared::cluster.v4.f32 {%0, %1, %2, %3}, [%4];"
+               : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w)
+               : "r"(caddr)
+               : "memory");
+  return v;
+}
+
+__device__ __forceinline__ bool wait_bounded(uint32_t bar, uint32_t parity, uint64_t timeout_ns) {
+  int never = 0;
+  return mbar_wait(bar, parity, &never, timeout_ns);
+}
+
+template <int HD>
+__global__ void __launch_bounds__(kAttnThreads, 1)
+    dv_attn_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
+                   const __grid_constant__ CUtensorMap tmV, const __grid_constant__ AttnParams p) {
+  using C = AttnCfg<HD>;
+  extern __shared__ uint8_t smem_raw[];
+  const uint32_t raw = smem_addr(smem_raw);
+  const uint32_t base = (raw + 1023u) & ~1023u;
+  uint8_t* base_ptr = smem_raw + (base - raw);
+  uint64_t* bars = reinterpret_cast<uint64_t*>(base_ptr + C::kEnd);
+  const uint32_t bar0 = smem_addr(bars);
+  // barriers: Q, K of stage 0/1, V of stage 0/1, scores ready, block output ready, drain
+  const uint32_t bar_q = bar0, bar_s = bar0 + 40, bar_o = bar0 + 48, bar_drain = bar0 + 56;
+  auto bar_k = [&](int st) { return bar0 + 8u + 8u * st; };
+  auto bar_v = [&](int st) { return bar0 + 24u + 8u * st; };
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 8);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+  int* key_end = reinterpret_cast<int*>(tmem_slot + 2);
+  float* part_m = reinterpret_cast<float*>(base_ptr + C::kEnd + 256);
+  float* part_l = part_m + 128;
+  float* part_o = reinterpret_cast<float*>(base_ptr + C::kOffStage);
+
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const uint64_t tmo = p.timeout_ns;
+  const int split = static_cast<int>(cluster_ctarank());
+  const int S = static_cast<int>(cluster_size());
+  const int unit = static_cast<int>(cluster_id_x());
+  const int qb = unit % p.q_blocks;
+  const int h = (unit / p.q_blocks) % p.Hkv;
+  const int b = unit / (p.q_blocks * p.Hkv);
+
+  // This thread's query row and the last slot it may see.
+  const int i = qb * 128 + tid;
+  const int nk = min(p.n_keys[b], p.max_keys);
+  int last = -1;
+  if (i < p.rows_per_group) last = min(p.q_slot[b * p.Nt + i % p.Nt], nk - 1);
+
+  if (tid == 0) {
+    mbar_init(bar_q, 1);
+    for (int st = 0; st < 2; ++st) {
+      mbar_init(bar_k(st), 1);
+      mbar_init(bar_v(st), 1);
+    }
+    mbar_init(bar_s, 1);
+    mbar_init(bar_o, 1);
+    mbar_init(bar_drain, 1);
+    *abort_flag = 0;
+    *key_end = 0;
+    fence_barrier_init();
+  }
+  if (warp == 0) {
+    tmem_alloc(smem_addr(tmem_slot), 256);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  atomicMax(key_end, last + 1);
+  __syncthreads();
+  const uint32_t tmem = *tmem_slot;
+  const uint32_t t_s = tmem, t_o = tmem + 128;
+  const uint32_t lane_base = static_cast<uint32_t>(warp * 32) << 16;
+  const int n_blocks = (*key_end + kKeyBlock - 1) / kKeyBlock;
+  const int kb0 = split * n_blocks / S, kb1 = (split + 1) * n_blocks / S;
+
+  const uint32_t sQ = base + C::kOffQ, sVt = base + C::kOffVt;
+  const int q_row0 = (b * p.Hq + h * p.G) * p.Nt + qb * 128;
+  auto sK = [&](int st) { return base + C::kOffStage + st * C::kStage; };
+  auto sV = [&](int st) { return base + C::kOffStage + st * C::kStage + C::kKV; };
+  auto load_kv = [&](int j) {  // block kb0 + j into stage j & 1
+    const int st = j & 1, kb = kb0 + j;
+    mbar_arrive_expect_tx(bar_k(st), C::kKV);
+    for (int ds = 0; ds < C::kSlabs; ++ds)
+      tma_load_4d(sK(st) + ds * C::kTile, &tmK, bar_k(st), ds * 64, h, kb * kKeyBlock, b);
+    mbar_arrive_expect_tx(bar_v(st), C::kKV);
+    for (int ds = 0; ds < C::kSlabs; ++ds)
+      tma_load_4d(sV(st) + ds * C::kTile, &tmV, bar_v(st), ds * 64, h, kb * kKeyBlock, b);
+  };
+
+  float o[HD];
+#pragma unroll
+  for (int d = 0; d < HD; ++d) o[d] = 0.0f;
+  float m_run = -INFINITY, l_run = 0.0f;
+
+  const int n_mine = kb1 - kb0;
+  if (tid == 0 && n_mine > 0) {
+    mbar_arrive_expect_tx(bar_q, C::kKV);
+    for (int ds = 0; ds < C::kSlabs; ++ds)
+      tma_load_2d(sQ + ds * C::kTile, &tmQ, bar_q, ds * 64, q_row0);
+    load_kv(0);
+  }
+  int last_issued = n_mine > 0 ? 0 : -1;  // thread 0: last block whose K/V loads it issued
+
+  bool ok = true;
+  for (int j = 0; j < n_mine && ok; ++j) {
+    const int st = j & 1, kb = kb0 + j;
+    const uint32_t sph = static_cast<uint32_t>(j >> 1) & 1u;  // phase of this stage's barriers
+    const uint32_t ph = static_cast<uint32_t>(j) & 1u;        // phase of bar_s / bar_o
+    const uint32_t sP = C::kPInK ? sK(st) : base + C::kOffP;
+    if (warp == 0) {
+      if (lane == 0) {
+        if (j + 1 < n_mine) {  // the other stage was freed by the previous block
+          load_kv(j + 1);
+          last_issued = j + 1;
+        }
+        // S = Q K^T
+        if (mbar_wait(bar_q, 0, abort_flag, tmo) && mbar_wait(bar_k(st), sph, abort_flag, tmo)) {
+          tc_fence_after();
+          const uint32_t idesc = idesc_bf16_f32(128, kKeyBlock);
+          for (int ds = 0; ds < C::kSlabs; ++ds)
+#pragma unroll
+            for (int k = 0; k < 4; ++k)
+              umma_bf16(t_s, sdesc_kmajor_sw128(sQ + ds * C::kTile + 32u * k),
+                        sdesc_kmajor_sw128(sK(st) + ds * C::kTile + 32u * k), idesc,
+                        (ds | k) != 0 ? 1u : 0u);
+          umma_commit(bar_s);
+        }
+      }
+      __syncwarp();
+    }
+
+    // V -> Vt: 8x8 blocks (8 keys x 8 channels); lane 8i + j8 addresses row j8 of block i.
+    ok = mbar_wait(bar_v(st), sph, abort_flag, tmo);
+    if (__all_sync(0xFFFFFFFFu, ok)) {
+      constexpr int kBlocks = (kKeyBlock / 8) * (HD / 8);
+      const int mi = lane >> 3, j8 = lane & 7;
+      const uint32_t v_base = sV(st);
+#pragma unroll 1
+      for (int quad = warp; quad < kBlocks / 4; quad += 4) {
+        const int blk = quad * 4 + mi;
+        const int key0 = (blk % (kKeyBlock / 8)) * 8, d0 = (blk / (kKeyBlock / 8)) * 8;
+        // stored row j8: key key0 + j8, channels d0 .. d0 + 7 (slab d0 / 64, 128-byte swizzle)
+        const int key = key0 + j8;
+        const uint32_t src = v_base + (d0 / 64) * C::kTile + key * 128 +
+                             ((((d0 % 64) / 8) ^ (key & 7)) << 4);
+        // transposed row j8: channel d0 + j8, keys key0 .. key0 + 7 (slab key0 / 64)
+        const int d = d0 + j8;
+        const uint32_t dst = sVt + (key0 / 64) * C::kVtSlab + d * 128 +
+                             ((((key0 % 64) / 8) ^ (d & 7)) << 4);
+        uint32_t r[4];
+        ldmatrix_x4_trans(src, r);
+        stmatrix_x4(dst, r);
+      }
+    }
+    fence_proxy_async_smem();
+
+    // Scores -> probabilities (this thread: query row tid).
+    ok = ok && mbar_wait(bar_s, ph, abort_flag, tmo);
+    float alpha = 1.0f;
+    if (__all_sync(0xFFFFFFFFu, ok)) {
+      tc_fence_after();
+      const int key_base = kb * kKeyBlock;
+      float mb = -INFINITY;
+#pragma unroll 1
+      for (int c = 0; c < kKeyBlock / 32; ++c) {
+        uint32_t r[32];
+        __syncwarp();
+        tmem_ld32(t_s + lane_base + c * 32, r);
+        tmem_ld_wait();
+#pragma unroll
+        for (int u = 0; u < 32; ++u)
+          if (key_base + c * 32 + u <= last) mb = fmaxf(mb, __uint_as_float(r[u]) * p.scale_log2);
+      }
+      const float m_new = fmaxf(m_run, mb);
+      alpha = m_new == -INFINITY ? 1.0f : exp2f(m_run - m_new);
+      float lb = 0.0f;
+#pragma unroll 1
+      for (int c = 0; c < kKeyBlock / 32; ++c) {
+        uint32_t r[32];
+        __syncwarp();
+        tmem_ld32(t_s + lane_base + c * 32, r);
+        tmem_ld_wait();
+        uint32_t pk[16];
+#pragma unroll
+        for (int u = 0; u < 32; u += 2) {
+          const int key = key_base + c * 32 + u;
+          const float p0 = key <= last ? exp2f(__uint_as_float(r[u]) * p.scale_log2 - m_new) : 0.0f;
+          const float p1 =
+              key + 1 <= last ? exp2f(__uint_as_float(r[u + 1]) * p.scale_log2 - m_new) : 0.0f;
+          lb += p0 + p1;
+          pk[u / 2] = pack_bf16x2(p0, p1);
+        }
+        // keys 32c .. 32c + 31 = 4 chunks of 8 keys in key slab c / 2
+        uint8_t* p_row = base_ptr + (sP - base) + (c / 2) * C::kTile + tid * 128;
+#pragma unroll
+        for (int q4 = 0; q4 < 4; ++q4) {
+          const int chunk = (c % 2) * 4 + q4;
+          *reinterpret_cast<uint4*>(p_row + ((chunk ^ (tid & 7)) << 4)) =
+              make_uint4(pk[4 * q4], pk[4 * q4 + 1], pk[4 * q4 + 2], pk[4 * q4 + 3]);
+        }
+      }
+      l_run = alpha * l_run + lb;
+      m_run = m_new;
+    }
+    fence_proxy_async_smem();
+    tc_fence_before();
+    ok = __syncthreads_and(ok) != 0;
+
+    // O_block = P V
+    if (ok && tid == 0) {
+      tc_fence_after();
+      const uint32_t idesc = idesc_bf16_f32(128, HD);
+      for (int ks = 0; ks < 2; ++ks)
+#pragma unroll
+        for (int k = 0; k < 4; ++k)
+          umma_bf16(t_o, sdesc_kmajor_sw128(sP + ks * C::kTile + 32u * k),
+                    sdesc_kmajor_sw128(sVt + ks * C::kVtSlab + 32u * k), idesc,
+                    (ks | k) != 0 ? 1u : 0u);
+      umma_commit(bar_o);
+    }
+    ok = ok && mbar_wait(bar_o, ph, abort_flag, tmo);
+    if (__all_sync(0xFFFFFFFFu, ok)) {
+      tc_fence_after();
+#pragma unroll
+      for (int c = 0; c < HD / 32; ++c) {
+        uint32_t r[32];
+        __syncwarp();
+        tmem_ld32(t_o + lane_base + c * 32, r);
+        tmem_ld_wait();
+#pragma unroll
+        for (int u = 0; u < 32; ++u) o[c * 32 + u] = fmaf(o[c * 32 + u], alpha, __uint_as_float(r[u]));
+      }
+    }
+    tc_fence_before();
+    ok = __syncthreads_and(ok) != 0;
+  }
+
+  if (!ok && tid == 0) {
+    // Let the copies in flight (the last block issued on each stage) land and every issued MMA
+    // finish before the memory is reused; each wait targets its stage's latest phase.
+    for (int jj = last_issued; jj >= 0 && jj >= last_issued - 1; --jj) {
+      const uint32_t sp = static_cast<uint32_t>(jj >> 1) & 1u;
+      wait_bounded(bar_k(jj & 1), sp, tmo);
+      wait_bounded(bar_v(jj & 1), sp, tmo);
+    }
+    if (last_issued >= 0) wait_bounded(bar_q, 0, tmo);
+    umma_commit(bar_drain);
+    wait_bounded(bar_drain, 0, tmo);
+  }
+  __syncthreads();
+
+  // Partial (O, m, l) of this CTA's key run -> shared memory, then the cluster combines.
+  {
+    float4* dst = reinterpret_cast<float4*>(part_o + tid * C::kPitch);
+#pragma unroll
+    for (int c = 0; c < HD / 4; ++c)
+      dst[c] = make_float4(o[4 * c], o[4 * c + 1], o[4 * c + 2], o[4 * c + 3]);
+    part_m[tid] = m_run;
+    part_l[tid] = l_run;
+  }
+  __syncwarp();
+  cluster_sync();
+  {
+    // CTA `split` combines rows [split * rows, (split + 1) * rows); tpr threads share a row.
+    // All remote loads of a step are issued before their values are used, so they overlap.
+    constexpr int kV4 = HD / 4;
+    const int rows = 128 / S, tpr = kAttnThreads / rows, per = kV4 / tpr;
+    const int rr = split * rows + tid / tpr, c4_0 = (tid % tpr) * per;
+    const int ii = qb * 128 + rr;
+    if (ii < p.rows_per_group) {
+      float ms[8], ls[8], w[8];
+#pragma unroll
+      for (int s = 0; s < 8; ++s) {
+        if (s < S) {
+          ms[s] = ld_cluster_f32(map_to_rank(smem_addr(part_m + rr), static_cast<uint32_t>(s)));
+          ls[s] = ld_cluster_f32(map_to_rank(smem_addr(part_l + rr), static_cast<uint32_t>(s)));
+        }
+      }
+      float M = -INFINITY;
+#pragma unroll
+      for (int s = 0; s < 8; ++s)
+        if (s < S) M = fmaxf(M, ms[s]);
+      float L = 0.0f;
+#pragma unroll
+      for (int s = 0; s < 8; ++s) {
+        w[s] = (s < S && ms[s] != -INFINITY) ? exp2f(ms[s] - M) : 0.0f;
+        if (s < S) L = fmaf(w[s], ls[s], L);
+      }
+      const float inv = L > 0.0f ? 1.0f / L : 0.0f;
+      const int hq = h * p.G + ii / p.Nt, t = ii % p.Nt;
+      uint16_t* orow = p.out + ((static_cast<size_t>(b) * p.Hq + hq) * p.Nt + t) * HD;
+#pragma unroll 1
+      for (int c = 0; c < per; ++c) {
+        const int c4 = c4_0 + c;
+        const uint32_t laddr = smem_addr(part_o + rr * C::kPitch + c4 * 4);
+        float4 v[8];
+#pragma unroll
+        for (int s = 0; s < 8; ++s)
+          if (s < S) v[s] = ld_cluster_f4(map_to_rank(laddr, static_cast<uint32_t>(s)));
+        float4 acc = make_float4(0.0f, 0.0f, 0.0f, 0.0f);
+#pragma unroll
+        for (int s = 0; s < 8; ++s) {
+          if (s < S) {
+            acc.x = fmaf(w[s], v[s].x, acc.x);
+            acc.y = fmaf(w[s], v[s].y, acc.y);
+            acc.z = fmaf(w[s], v[s].z, acc.z);
+            acc.w = fmaf(w[s], v[s].w, acc.w);
+          }
+        }
+        uint2 out;
+        out.x = pack_bf16x2(acc.x * inv, acc.y * inv);
+        out.y = pack_bf16x2(acc.z * inv, acc.w * inv);
+        *reinterpret_cast<uint2*>(orow + c4 * 4) = out;
+      }
+    }
+  }
+  __syncwarp();
+  cluster_sync();
+
+  if (warp == 0) {
+    tc_fence_after();
+    tmem_dealloc(tmem, 256);
+  }
+  if (tid == 0 && *abort_flag) atomicExch(&g_attn_status, DV_ERR_DEVICE_TIMEOUT);
+}
+
+typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,
+                                  const cuuint64_t*, const cuuint64_t*, const cuuint32_t*,
+                                  const cuuint32_t*, CUtensorMapInterleave, CUtensorMapSwizzle,
+                                  CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiledFn encode_fn() {
+  static EncodeTiledFn fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* q = nullptr;
+    cudaDriverEntryPointQueryResult r;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &q, 12000, cudaEnableDefault,
+                                         &r) == cudaSuccess &&
+        r == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<EncodeTiledFn>(q);
+  });
+  return fn;
+}
+
+// Cache layer as a 4-D bf16 tensor (head_dim, kv head, slot, batch), boxes of 64 channels x
+// 1 head x 128 slots x 1 batch element with 128-byte swizzle; slots past max_keys read zero.
+bool encode_cache_4d(CUtensorMap* map, const void* ptr, int HD, int Hkv, int keys, int B,
+                     long long s_head, long long s_seq, long long s_batch) {
+  EncodeTiledFn fn = encode_fn();
+  if (!fn) return false;
+  // strides of dimensions of extent 1 are never used; any valid multiple of 16 bytes will do
+  const long long sh = Hkv > 1 ? s_head : 8, sb = B > 1 ? s_batch : 8;
+  cuuint64_t dims[4] = {static_cast<cuuint64_t>(HD), static_cast<cuuint64_t>(Hkv),
+                        static_cast<cuuint64_t>(keys), static_cast<cuuint64_t>(B)};
+  cuuint64_t strides[3] = {static_cast<cuuint64_t>(sh * 2), static_cast<cuuint64_t>(s_seq * 2),
+                           static_cast<cuuint64_t>(sb * 2)};
+  cuuint32_t box[4] = {64, 1, static_cast<cuuint32_t>(kKeyBlock), 1};
+  cuuint32_t estr[4] = {1, 1, 1, 1};
+  return fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void*>(ptr), dims, strides, box,
+            estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+            CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+int device_ok() {
+  static int state[64] = {};  // 0 unknown, 1 sm_103, 2 other
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return DV_ERR_CUDA;
+  if (state[dev] == 0) {
+    cudaDeviceProp prop;
+    if (cudaGetDeviceProperties(&prop, dev) != cudaSuccess) return DV_ERR_CUDA;
+    state[dev] = (prop.major == 10 && prop.minor == 3) ? 1 : 2;
+  }
+  return state[dev] == 1 ? DV_OK : DV_ERR_UNSUPPORTED_DEVICE;
+}
+
+int num_sms_of_device() {
+  static int sms[64] = {};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 148;
+  if (sms[dev] == 0) {
+    int n = 0;
+    if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return 148;
+    sms[dev] = n;
+  }
+  return sms[dev];
+}
+
+template <int HD>
+cudaError_t launch_attn(int splits, int units, const CUtensorMap& q, const CUtensorMap& k,
+                        const CUtensorMap& v, const AttnParams& p, cudaStream_t stream) {
+  using C = AttnCfg<HD>;
+  auto kern = dv_attn_kernel<HD>;
+  static bool attr_set[64] = {};  // the shared-memory opt-in, once per device
+  int dev = 0;
+  cudaError_t err = cudaGetDevice(&dev);
+  if (err != cudaSuccess) return err;
+  if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
+  if (!attr_set[dev]) {
+    err = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, C::kSmemBytes);
+    if (err != cudaSuccess) return err;
+    attr_set[dev] = true;
+  }
+  cudaLaunchConfig_t cfg = {};
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = static_cast<unsigned>(splits);
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.gridDim = dim3(static_cast<unsigned>(units * splits), 1, 1);
+  cfg.blockDim = dim3(kAttnThreads, 1, 1);
+  cfg.dynamicSmemBytes = C::kSmemBytes;
+  cfg.stream = stream;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  err = cudaLaunchKernelEx(&cfg, kern, q, k, v, p);
+  if (err != cudaSuccess) return err;
+  return cudaGetLastError();
+}
+
+bool al16(const void* x) { return (reinterpret_cast<uintptr_t>(x) & 15u) == 0; }
+
+}  // namespace
+}  // namespace dv
+
+extern "C" int dv_text_attention(const void* q, int batch, int n_q_heads, int n_kv_heads,
+                                 int n_text, int head_dim, const dv_kv_cache* cache, int layer,
+                                 int max_keys, const int* n_keys, const int* q_slot, float scale,
+                                 void* out, void* stream) {
+  using namespace dv;
+  if (batch < 0 || n_text < 0) return DV_ERR_INVALID_ARG;
+  if (batch == 0 || n_text == 0) return DV_OK;
+  if (!q || !cache || !cache->k || !cache->v || !n_keys || !q_slot || !out) return DV_ERR_INVALID_ARG;
+  if (n_q_heads <= 0 || n_kv_heads <= 0 || n_q_heads % n_kv_heads != 0 || layer < 0 ||
+      max_keys <= 0 || !(scale > 0.0f) || !std::isfinite(scale))
+    return DV_ERR_INVALID_ARG;
+  if (head_dim != 64 && head_dim != 128) return DV_ERR_UNSUPPORTED_SHAPE;
+  const long long rows = static_cast<long long>(batch) * n_q_heads * n_text;
+  if (rows > (1LL << 30) || max_keys > (1 << 24) || n_kv_heads > 4096 || batch > 65535)
+    return DV_ERR_UNSUPPORTED_SHAPE;
+  if (!al16(q) || !al16(out) || !al16(cache->k) || !al16(cache->v)) return DV_ERR_ALIGNMENT;
+  if ((reinterpret_cast<uintptr_t>(n_keys) & 3u) || (reinterpret_cast<uintptr_t>(q_slot) & 3u))
+    return DV_ERR_ALIGNMENT;
+  const long long st[4] = {cache->s_layer, cache->s_batch, cache->s_seq, cache->s_head};
+  for (long long x : st) {
+    if (x < 0) return DV_ERR_INVALID_ARG;
+    if (x % 8 != 0) return DV_ERR_ALIGNMENT;
+  }
+  if (cache->s_seq == 0) return DV_ERR_INVALID_ARG;
+  int rc = device_ok();
+  if (rc != DV_OK) return rc;
+  if (!encode_fn()) return DV_ERR_CUDA;
+
+  const long long off = static_cast<long long>(layer) * cache->s_layer;
+  const uint16_t* kl = static_cast<const uint16_t*>(cache->k) + off;
+  const uint16_t* vl = static_cast<const uint16_t*>(cache->v) + off;
+  CUtensorMap tq, tk, tv;
+  {
+    EncodeTiledFn fn = encode_fn();
+    cuuint64_t dims[2] = {static_cast<cuuint64_t>(head_dim), static_cast<cuuint64_t>(rows)};
+    cuuint64_t strides[1] = {static_cast<cuuint64_t>(head_dim) * 2};
+    cuuint32_t box[2] = {64, 128};
+    cuuint32_t estr[2] = {1, 1};
+    if (fn(&tq, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(q), dims, strides, box,
+           estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+           CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+      return DV_ERR_UNSUPPORTED_SHAPE;
+  }
+  if (!encode_cache_4d(&tk, kl, head_dim, n_kv_heads, max_keys, batch, cache->s_head,
+                       cache->s_seq, cache->s_batch) ||
+      !encode_cache_4d(&tv, vl, head_dim, n_kv_heads, max_keys, batch, cache->s_head,
+                       cache->s_seq, cache->s_batch))
+    return DV_ERR_UNSUPPORTED_SHAPE;
+
+  AttnParams p;
+  p.Hq = n_q_heads;
+  p.Hkv = n_kv_heads;
+  p.Nt = n_text;
+  p.G = n_q_heads / n_kv_heads;
+  p.rows_per_group = p.G * n_text;
+  p.q_blocks = (p.rows_per_group + 127) / 128;
+  p.max_keys = max_keys;
+  p.n_keys = n_keys;
+  p.q_slot = q_slot;
+  p.scale_log2 = static_cast<float>(static_cast<double>(scale) * 1.4426950408889634);
+  p.out = static_cast<uint16_t*>(out);
+  p.timeout_ns = 2000000000ull;
+
+  const long long units = static_cast<long long>(batch) * n_kv_heads * p.q_blocks;
+  if (units > (1LL << 30)) return DV_ERR_UNSUPPORTED_SHAPE;
+  const int blocks_max = (max_keys + kKeyBlock - 1) / kKeyBlock;
+  const int sms = num_sms_of_device();
+  int splits = 1;
+  for (int s : {2, 4, 8})
+    if (s <= blocks_max && units * s <= sms) splits = s;
+  cudaError_t err = head_dim == 128
+                        ? launch_attn<128>(splits, static_cast<int>(units), tq, tk, tv, p,
+                                           static_cast<cudaStream_t>(stream))
+                        : launch_attn<64>(splits, static_cast<int>(units), tq, tk, tv, p,
+                                          static_cast<cudaStream_t>(stream));
+  return err == cudaSuccess ? DV_OK : DV_ERR_CUDA;
+}
+
+extern "C" int dv_text_attention_status(void) {
+  int st = 0;
+  if (cudaDeviceSynchronize() != cudaSuccess) return DV_ERR_CUDA;
+  if (cudaMemcpyFromSymbol(&st, dv::g_attn_status, sizeof(int)) != cudaSuccess) return DV_ERR_CUDA;
+  if (st != 0) {
+    const int zero = 0;
+    if (cudaMemcpyToSymbol(dv::g_attn_status, &zero, sizeof(int)) != cudaSuccess) return DV_ERR_CUDA;
+  }
+  return st;
+}

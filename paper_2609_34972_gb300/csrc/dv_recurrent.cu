@@ -198,13 +198,20 @@ __global__ void __launch_bounds__(kDownThreads, 1)
       const int t = m * kBlockM + rr;
       if (t >= p.M) continue;
       const uint32_t laddr = smem_addr(red + rr * C::kPitch + c4 * 4);
+      // all S loads first (independent, so their latencies overlap), then the sum in order
+      float4 part[8];
+#pragma unroll
+      for (int s = 0; s < 8; ++s)
+        if (s < S) part[s] = ld_cluster_f4(map_to_rank(laddr, static_cast<uint32_t>(s)));
       float4 z = make_float4(0.0f, 0.0f, 0.0f, 0.0f);
-      for (int s = 0; s < S; ++s) {
-        const float4 v = ld_cluster_f4(map_to_rank(laddr, static_cast<uint32_t>(s)));
-        z.x += v.x;
-        z.y += v.y;
-        z.z += v.z;
-        z.w += v.w;
+#pragma unroll
+      for (int s = 0; s < 8; ++s) {
+        if (s < S) {
+          z.x += part[s].x;
+          z.y += part[s].y;
+          z.z += part[s].z;
+          z.w += part[s].w;
+        }
       }
       uint2 out;
       out.x = pack_bf16x2(silu(z.x), silu(z.y));

@@ -93,7 +93,7 @@ def parity(g, o, head_dim):
     return float(err.max()), float(cos.min())
 
 
-def assert_parity(gk, gv, ok, ov, head_dim, label=""):
+def assert_parity(gk, gv, ok, ov, head_dim, label="", rel_tol=REL_TOL, cos_tol=COS_TOL):
     ek, ck = parity(gk, ok, head_dim)
     ev, cv = parity(gv, ov, head_dim)
     msg = f"{label}: K max err {ek:.3e} min cos {ck:.7f}; V max err {ev:.3e} min cos {cv:.7f}"
@@ -103,8 +103,8 @@ def assert_parity(gk, gv, ok, ov, head_dim, label=""):
             f.write(json.dumps({"case": label, "k_max_err": ek, "k_min_cos": ck, "v_max_err": ev,
                                 "v_min_cos": cv, "n_tokens": int(ok.shape[0])}) + "\n")
     assert np.all(np.isfinite(gk)) and np.all(np.isfinite(gv)), msg
-    assert ek <= REL_TOL and ev <= REL_TOL, msg
-    assert ck >= COS_TOL and cv >= COS_TOL, msg
+    assert ek <= rel_tol and ev <= rel_tol, msg
+    assert ck >= cos_tol and cv >= cos_tol, msg
     return ek, ev, ck, cv
 
 

@@ -126,3 +126,21 @@ def test_bad_layer_modes_rejected(dv, modes):
     w = dv.DvWeights(*([ctypes.c_void_p(256)] * 5 + [None, None, ctypes.cast(arr, ctypes.c_void_p)]))
     h = ctypes.c_void_p()
     assert dv.lib().dv_memory_plan(ctypes.byref(cfg), ctypes.byref(w), None, ctypes.byref(h)) == 1
+
+
+def test_text_attention_validates_before_device(dv):
+    lib = dv.lib()
+    kvc = dv.DvKVCache(256, 512, 8 * 64 * 100, 8 * 64 * 100, 8 * 64, 64)
+    p = ctypes.c_void_p(1024)
+    args = lambda **kw: [kw.get("q", p), kw.get("batch", 1), kw.get("hq", 8), kw.get("hkv", 8),
+                         kw.get("nt", 4), kw.get("hd", 64), ctypes.byref(kw.get("cache", kvc)),
+                         kw.get("layer", 0), kw.get("max_keys", 100), p, p,
+                         ctypes.c_float(kw.get("scale", 0.125)), kw.get("out", p), None]
+    assert lib.dv_text_attention(*args(batch=0)) == dv.DV_OK          # empty: nothing to do
+    assert lib.dv_text_attention(*args(q=None)) == dv.DV_ERR_INVALID_ARG
+    assert lib.dv_text_attention(*args(hq=6, hkv=4)) == dv.DV_ERR_INVALID_ARG
+    assert lib.dv_text_attention(*args(scale=0.0)) == dv.DV_ERR_INVALID_ARG
+    assert lib.dv_text_attention(*args(hd=96)) == dv.DV_ERR_UNSUPPORTED_SHAPE
+    assert lib.dv_text_attention(*args(q=ctypes.c_void_p(1026))) == dv.DV_ERR_ALIGNMENT
+    bad = dv.DvKVCache(256, 512, 8 * 64 * 100, 8 * 64 * 100, 8 * 64 + 4, 64)
+    assert lib.dv_text_attention(*args(cache=bad)) == dv.DV_ERR_ALIGNMENT
