@@ -38,6 +38,7 @@ struct dv_plan {
   float* bk = nullptr;
   float* bv = nullptr;
   float* kg = nullptr;         // per-head K-norm gain fp32 [L][head_dim] (k_norm)
+  float* Gf = nullptr;         // embedding adapter: G_l = U_l^T U_l, fp32 [L][r_pad][r_pad]
   void* ws = nullptr;          // workspace of a build of max_tokens tokens (carve_workspace)
   long long last_tokens = 0;   // tokens of the last build (layout of the workspace)
   int* status = nullptr;
@@ -116,16 +117,17 @@ struct PackLayers {
   unsigned char zero_du[dv::kMaxLayers];
 };
 
-// Dst[i*r_pad + k][j] = D[src[i]][k][j] for k < r, else 0.
+// Dst[i*r_pad + k][j] = D[src[i]][k][j] for k < r, else 0 (row stride ld).
 __global__ void k_pack_down(const uint16_t* __restrict__ D, uint16_t* __restrict__ Dst, int L,
-                            int r, int r_pad, int d, PackLayers pl) {
+                            int r, int r_pad, int d, int ld, PackLayers pl) {
   const long long total = static_cast<long long>(L) * r_pad * d;
   for (long long e = blockIdx.x * static_cast<long long>(blockDim.x) + threadIdx.x; e < total;
        e += static_cast<long long>(gridDim.x) * blockDim.x) {
     const int j = static_cast<int>(e % d);
     const long long row = e / d;
     const int k = static_cast<int>(row % r_pad), i = static_cast<int>(row / r_pad);
-    Dst[e] = (k < r && !pl.zero_du[i]) ? D[(static_cast<long long>(pl.src[i]) * r + k) * d + j] : 0;
+    Dst[row * ld + j] =
+        (k < r && !pl.zero_du[i]) ? D[(static_cast<long long>(pl.src[i]) * r + k) * d + j] : 0;
   }
 }
 
@@ -143,6 +145,22 @@ __global__ void k_pack_norm_u(const uint16_t* __restrict__ U, uint16_t* __restri
     if (j < d && n < r && !pl.zero_du[i])
       v = 2.0f * bf(U[(static_cast<long long>(pl.src[i]) * d + j) * r + n]);
     Bn[e] = to_bf16(v);  // the G columns (j >= d) are zero here and filled afterwards
+  }
+}
+
+// Dst[row0 + i*r_pad + n][j] = 2 U[src[i]][j][n] (n < r), else 0: the x0 (2 U_l)^T part of the
+// statistic of M_l, stacked after the down-projections so that one GEMM over x0 forms both.
+__global__ void k_pack_2u(const uint16_t* __restrict__ U, uint16_t* __restrict__ Dst, int L, int r,
+                          int r_pad, int d, int ld, PackLayers pl) {
+  const long long total = static_cast<long long>(L) * r_pad * d;
+  for (long long e = blockIdx.x * static_cast<long long>(blockDim.x) + threadIdx.x; e < total;
+       e += static_cast<long long>(gridDim.x) * blockDim.x) {
+    const int j = static_cast<int>(e % d);
+    const long long row = e / d;
+    const int n = static_cast<int>(row % r_pad), i = static_cast<int>(row / r_pad);
+    float v = 0.0f;
+    if (n < r && !pl.zero_du[i]) v = 2.0f * bf(U[(static_cast<long long>(pl.src[i]) * d + j) * r + n]);
+    Dst[row * ld + j] = to_bf16(v);
   }
 }
 
@@ -187,7 +205,8 @@ __global__ void k_pack_kv(const uint16_t* __restrict__ Wk, const uint16_t* __res
 }
 
 // out[p][i][n] = sum_j A(l, i, j) * U[l][j][n] for n < r, accumulated in fp32 over j < d, for
-// planned layer p = blockIdx.z of source layer l = src[p] (U taken as zero where zero_du[p]):
+// planned layer p = blockIdx.z of source layer l = src[p] (U taken as zero where zero_du[p]);
+// in MODE 1 the fp32 result also goes to gout[p][i][n] when gout is given:
 //   MODE 0 (fold):  A(l, i, j) = W_part[l][c][j] * gamma[l][j], i indexes the 2*kv Wkv rows
 //                   of the layer; the result goes to Wkv row (p, i), column d + n
 //   MODE 1 (gram):  A(l, i, j) = U[l][j][i], i < r; the result goes to Bn row p*r_pad + i,
@@ -200,7 +219,8 @@ __global__ void __launch_bounds__(256) k_rank_product(const uint16_t* __restrict
                                                       const uint16_t* __restrict__ U,
                                                       uint16_t* __restrict__ out, int rows, int r,
                                                       int d, int kv, int HD, int r_pad,
-                                                      int k_total, PackLayers pl) {
+                                                      int k_total, PackLayers pl,
+                                                      float* __restrict__ gout) {
   __shared__ float As[32][65];
   __shared__ float Us[32][65];
   const int p = blockIdx.z, l = pl.src[p];
@@ -255,7 +275,9 @@ __global__ void __launch_bounds__(256) k_rank_product(const uint16_t* __restrict
 #pragma unroll
     for (int w = 0; w < 4; ++w) {
       const int n = n0 + tx * 4 + w;
-      if (n < r) out[orow * k_total + d + n] = to_bf16(acc[q][w]);
+      if (n >= r) continue;
+      if (out) out[orow * k_total + d + n] = to_bf16(acc[q][w]);
+      if (MODE == 1 && gout) gout[(static_cast<long long>(p) * r_pad + i) * r_pad + n] = acc[q][w];
     }
   }
 }
@@ -298,6 +320,112 @@ __global__ void k_rstd_parts(const float* __restrict__ part, int L, long long T,
   }
 }
 
+// Statistic of M_l = x0 + h_l U_l for small token counts: ||M_l||^2 = ||x0||^2 +
+// h_l . (c_l + G_l h_l), with c_l = x0 (2 U_l)^T (fp32, from the stacked GEMM) and
+// G_l = U_l^T U_l (fp32, from the plan), so rstd_l = ((xx + h . (c + G h)) / d + eps)^-1/2.
+// One block of 64 threads per (layer, 64 tokens): thread (tg, k) keeps u_n = c_n + (G h)_n for
+// the 4 tokens 4 tg .. 4 tg + 3 and n in quarter k ([16 k, 16 k + 16)) in registers. G is
+// symmetric, so row m scales h_m into all sums; G_l sits in shared memory with each row's
+// quarters interleaved (float4 n4 of quarter k at word 16 n4 + 4 k) so that the four quarters
+// read together fall in distinct banks, and h as [m][token], read as float4 over 4 tokens. The
+// four partial dots of a token are summed with two shuffles (fixed order).
+template <int RP>
+__global__ void __launch_bounds__(64) k_rstd_hc(const uint16_t* __restrict__ H, int ldh,
+                                                const float* __restrict__ C, int ldc,
+                                                const float* __restrict__ xx,
+                                                const float* __restrict__ Gf, int T, float inv_d,
+                                                float eps, float* __restrict__ rstd) {
+  static_assert(RP == 64, "one quarter = 16 sums = 4 float4");
+  __shared__ __align__(16) float g[RP * RP];
+  __shared__ __align__(16) float hs[RP][64];
+  const int l = blockIdx.y, tid = threadIdx.x;
+  const int tg = tid >> 2, k = tid & 3;
+  const float* gl = Gf + static_cast<long long>(l) * RP * RP;
+  {  // all 16 loads of this thread first, then the stores (interleaved quarters)
+    float4 gv[RP * RP / 4 / 64];
+    const float4* gl4 = reinterpret_cast<const float4*>(gl);
+#pragma unroll
+    for (int i = 0; i < RP * RP / 4 / 64; ++i) gv[i] = gl4[tid + 64 * i];
+#pragma unroll
+    for (int i = 0; i < RP * RP / 4 / 64; ++i) {
+      const int e = 4 * (tid + 64 * i);  // e = m*64 + n, n a multiple of 4
+      const int m = e >> 6, n = e & 63, kk = n >> 4, n4 = (n >> 2) & 3;
+      *reinterpret_cast<float4*>(g + m * RP + n4 * 16 + kk * 4) = gv[i];
+    }
+  }
+  {  // token tid, all RP channels: 8 independent 16-byte loads, then the widening stores
+    const int t = min(static_cast<int>(blockIdx.x) * 64 + tid, T - 1);
+    const uint4* hrow = reinterpret_cast<const uint4*>(H + static_cast<long long>(t) * ldh + l * RP);
+    uint4 hw[RP / 8];
+#pragma unroll
+    for (int c8 = 0; c8 < RP / 8; ++c8) hw[c8] = hrow[c8];
+#pragma unroll
+    for (int c8 = 0; c8 < RP / 8; ++c8) {
+      const uint32_t ws[4] = {hw[c8].x, hw[c8].y, hw[c8].z, hw[c8].w};
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        hs[c8 * 8 + 2 * q][tid] = __uint_as_float(ws[q] << 16);
+        hs[c8 * 8 + 2 * q + 1][tid] = __uint_as_float(ws[q] & 0xFFFF0000u);
+      }
+    }
+  }
+  __syncthreads();
+  float u[4][16];
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const int t = min(blockIdx.x * 64 + tg * 4 + i, T - 1);
+    const float4* cr = reinterpret_cast<const float4*>(C + static_cast<long long>(t) * ldc + l * RP + k * 16);
+#pragma unroll
+    for (int n4 = 0; n4 < 4; ++n4) {
+      const float4 c4 = cr[n4];
+      u[i][4 * n4] = c4.x;
+      u[i][4 * n4 + 1] = c4.y;
+      u[i][4 * n4 + 2] = c4.z;
+      u[i][4 * n4 + 3] = c4.w;
+    }
+  }
+#pragma unroll 2
+  for (int m = 0; m < RP; ++m) {
+    const float4 hm = *reinterpret_cast<const float4*>(&hs[m][tg * 4]);
+    const float hv[4] = {hm.x, hm.y, hm.z, hm.w};
+#pragma unroll
+    for (int n4 = 0; n4 < 4; ++n4) {
+      const float4 gv = *reinterpret_cast<const float4*>(g + m * RP + n4 * 16 + k * 4);
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        u[i][4 * n4] = fmaf(gv.x, hv[i], u[i][4 * n4]);
+        u[i][4 * n4 + 1] = fmaf(gv.y, hv[i], u[i][4 * n4 + 1]);
+        u[i][4 * n4 + 2] = fmaf(gv.z, hv[i], u[i][4 * n4 + 2]);
+        u[i][4 * n4 + 3] = fmaf(gv.w, hv[i], u[i][4 * n4 + 3]);
+      }
+    }
+  }
+  float dot[4] = {0.0f, 0.0f, 0.0f, 0.0f};
+#pragma unroll
+  for (int n = 0; n < 16; ++n) {
+    const float4 hn = *reinterpret_cast<const float4*>(&hs[k * 16 + n][tg * 4]);
+    dot[0] = fmaf(hn.x, u[0][n], dot[0]);
+    dot[1] = fmaf(hn.y, u[1][n], dot[1]);
+    dot[2] = fmaf(hn.z, u[2][n], dot[2]);
+    dot[3] = fmaf(hn.w, u[3][n], dot[3]);
+  }
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    dot[i] += __shfl_xor_sync(0xFFFFFFFFu, dot[i], 1);
+    dot[i] += __shfl_xor_sync(0xFFFFFFFFu, dot[i], 2);
+  }
+  if (k == 0) {
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      const int t = blockIdx.x * 64 + tg * 4 + i;
+      if (t < T) {
+        const float ss = fmaxf(xx[t] + dot[i], 0.0f);
+        rstd[static_cast<long long>(l) * T + t] = rsqrtf(fmaf(ss, inv_d, eps));
+      }
+    }
+  }
+}
+
 // xx[t] = sum_j x0[t][j]^2 (fp32), one warp per token row, 16-byte loads.
 __global__ void k_row_sumsq(const uint16_t* __restrict__ x0, int T, int d, float* __restrict__ xx) {
   const int warp = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
@@ -305,6 +433,7 @@ __global__ void k_row_sumsq(const uint16_t* __restrict__ x0, int T, int d, float
   if (warp >= T) return;
   const uint4* row = reinterpret_cast<const uint4*>(x0 + static_cast<long long>(warp) * d);
   float s = 0.0f;
+#pragma unroll 8
   for (int c = lane; c < d / 8; c += 32) {
     const uint4 v = row[c];
     const uint32_t w[4] = {v.x, v.y, v.z, v.w};
@@ -393,7 +522,7 @@ int check_config(const dv_config* c) {
 }
 
 void free_plan_memory(dv_plan* p) {
-  void* ptrs[] = {p->Dst, p->Bn, p->Wkv, p->Uup, p->bk, p->bv, p->kg, p->ws, p->status};
+  void* ptrs[] = {p->Dst, p->Bn, p->Wkv, p->Uup, p->bk, p->bv, p->kg, p->Gf, p->ws, p->status};
   for (void* q : ptrs)
     if (q) cudaFree(q);
   for (cudaEvent_t e : p->ev) cudaEventDestroy(e);
@@ -611,7 +740,33 @@ cudaError_t enqueue_build(const PlanView& v, const BuildArgs& a, cudaStream_t st
 
   // (1) H = SiLU(x0 [D_1 ... D_L]) — one GEMM over all layers' down-projections.
   gp.s = {static_cast<int>(T), 1, static_cast<int>(n1), d / 64, 0, 0, 0, 0, 0, 0};
-  gp.silu = {a.H, static_cast<int>(n1)};
+  gp.silu = {a.H, static_cast<int>(n1), static_cast<int>(n1), nullptr, 0};
+  if (!rank_pairs && a.c) {
+    // Small or awkward token counts: x0 [D_1 .. D_L | 2U_1 .. 2U_L]^T as one GEMM (the
+    // down-projections get SiLU, the second half is c_l = x0 (2 U_l)^T in fp32), then the
+    // statistic of M_l from h_l, c_l and G_l in a small kernel: one tensor-core pass over x0
+    // instead of two GEMMs of long K over few token blocks.
+    // On CTA pairs (256-token blocks, each SM staging half of the weight rows): the K loop is
+    // long and the tiles few, so the bytes each SM must stage per slab, not the MMA work, set the
+    // time; the 256-token padding only adds MMA work.
+    const long long n2 = 2 * n1;
+    // a tile is either all down-projection columns or all c columns: bn divides n1
+    const int bn = n1 % 256 == 0 ? 256 : (n1 % 128 == 0 ? 128 : 64);
+    gp.s = {static_cast<int>(T), 1, static_cast<int>(n2), d / 64, 0, 0, 0, 0, 0, 0};
+    gp.silu = {a.H, static_cast<int>(n1), static_cast<int>(n1), a.c, static_cast<int>(n1)};
+    tm_groups(gp.s, bn, T);
+    const CUtensorMap& tmD = v.tm_Dst_half[bn == 64 ? 0 : (bn == 128 ? 1 : 2)];
+    if (err == cudaSuccess) err = launch_pair_tm(EPI_SILU, bn, 0, tm_x0, tm_x0, tmD, gp, v.num_sms, st);
+    mark(2);
+    if (err == cudaSuccess) {
+      dim3 grid(static_cast<unsigned>((T + 63) / 64), static_cast<unsigned>(L));
+      k_rstd_hc<64><<<grid, 64, 0, st>>>(a.H, static_cast<int>(n1), a.c, static_cast<int>(n1),
+                                         a.xx, v.Gf, static_cast<int>(T), 1.0f / d, v.rms_eps,
+                                         a.rstd);
+      err = cudaGetLastError();
+    }
+    mark(3);
+  } else {
   if (rank_pairs) {
     const long long pairs = v.num_sms / 2;
     int bn = 64;
@@ -648,6 +803,7 @@ cudaError_t enqueue_build(const PlanView& v, const BuildArgs& a, cudaStream_t st
                      : launch_gemm(EPI_NORM, v.r_pad, 0, tm_x0, tm_H, *v.tm_Bn, gp, v.num_sms, st);
   }
   mark(3);
+  }
 
   // (3) K/V = rstd_l * ([x0 | h_l] Wkv_l^T) + b, RoPE on K, stored into the cache.
   gp.s = {static_cast<int>(T), L, 2 * v.kv, d / 64, v.r_pad / 64, v.r_pad, 0, 0, 0, 0};
@@ -669,8 +825,10 @@ size_t carve_workspace(const PlanView& v, long long T, void* base, BuildArgs* a)
   const size_t L = static_cast<size_t>(v.n_layers), t = static_cast<size_t>(T);
   const size_t d = static_cast<size_t>(v.d);
   const size_t oH = take(t * L * v.r_pad * 2), oR = take(L * t * 4), oX = take(t * 4);
-  size_t oS = 0, oM = 0, oP = 0;
+  size_t oS = 0, oM = 0, oP = 0, oC = 0;
   const bool rec = v.adapter == DV_ADAPTER_RECURRENT;
+  const bool small_path = !rec && v.r_pad == 64;  // x0 (2 U_l)^T in fp32 (see enqueue_build)
+  if (small_path) oC = take(t * L * v.r_pad * 4);
   if (rec) {
     oS = take(t * d * 4);
     oM = take(L * t * d * 2);
@@ -684,6 +842,7 @@ size_t carve_workspace(const PlanView& v, long long T, void* base, BuildArgs* a)
     a->state = rec ? reinterpret_cast<float*>(b + oS) : nullptr;
     a->mem = rec ? reinterpret_cast<uint16_t*>(b + oM) : nullptr;
     a->part = rec ? reinterpret_cast<float*>(b + oP) : nullptr;
+    a->c = small_path ? reinterpret_cast<float*>(b + oC) : nullptr;
   }
   return off;
 }
@@ -708,6 +867,7 @@ bool plan_view(const dv_plan* p, PlanView* v) {
   v->bv = p->bv;
   v->status = p->status;
   v->tm_Dst = p->tm_Dst;
+  v->Gf = p->Gf;
   v->tm_Dst_half = p->tm_Dst_half;
   v->tm_Bn = &p->tm_Bn;
   v->tm_Bn_half = &p->tm_Bn_half;
@@ -775,6 +935,18 @@ int dv_memory_plan(const dv_config* cfg, const dv_weights* w, void* stream, dv_p
   if (prop.major != 10 || prop.minor != 3) return DV_ERR_UNSUPPORTED_DEVICE;
   if (!encode_fn()) return DV_ERR_CUDA;
 
+  // The build's small kernels ask for the same shared-memory carveout as its GEMMs (all of it),
+  // so that consecutive launches need no L1 / shared-memory reconfiguration between them.
+  {
+    const void* small[] = {reinterpret_cast<const void*>(k_row_sumsq),
+                           reinterpret_cast<const void*>(k_rstd_parts),
+                           reinterpret_cast<const void*>(k_rstd_hc<64>)};
+    for (const void* f : small)
+      if (cudaFuncSetAttribute(f, cudaFuncAttributePreferredSharedMemoryCarveout,
+                               cudaSharedmemCarveoutMaxShared) != cudaSuccess)
+        cudaGetLastError();
+  }
+
   dv_plan* p = new (std::nothrow) dv_plan();
   if (!p) return DV_ERR_OOM;
   p->cfg = *cfg;
@@ -807,7 +979,13 @@ int dv_memory_plan(const dv_config* cfg, const dv_weights* w, void* stream, dv_p
   dv::plan_view(p, &pv);
   const size_t ws_bytes = dv::carve_workspace(pv, T, nullptr, nullptr);
 
-  bool ok = dmalloc(&p->Dst, sizeof(uint16_t) * L * p->r_pad * d) &&
+  // Embedding adapter: Dst stacks 2 U^T under D (rows [L r_pad, 2 L r_pad)) for the small-token
+  // path, which forms the statistic of M_l from x0 (2 U_l)^T and the fp32 G_l.
+  const int dst_rows = (rec ? 1 : 2) * L * p->r_pad;
+  // Rows padded by 64 elements: a stride that is not a power of two spreads the rows of a
+  // 128-row TMA box over the L2 (the K/V weights' d + r_pad stride does the same).
+  const int dst_ld = d + 64;
+  bool ok = dmalloc(&p->Dst, sizeof(uint16_t) * dst_rows * dst_ld) &&
             (rec ? dmalloc(&p->Uup, sizeof(uint16_t) * static_cast<size_t>(L) * d * p->r_pad)
                  : dmalloc(&p->Bn, sizeof(uint16_t) * L * p->r_pad * p->k_total)) &&
             dmalloc(&p->Wkv, sizeof(uint16_t) * static_cast<size_t>(L) * 2 * p->kv * p->k_total) &&
@@ -815,6 +993,7 @@ int dv_memory_plan(const dv_config* cfg, const dv_weights* w, void* stream, dv_p
   if (ok && cfg->has_kv_bias)
     ok = dmalloc(&p->bk, sizeof(float) * L * p->kv) && dmalloc(&p->bv, sizeof(float) * L * p->kv);
   if (ok && cfg->k_norm) ok = dmalloc(&p->kg, sizeof(float) * L * HD);
+  if (ok && !rec) ok = dmalloc(&p->Gf, sizeof(float) * L * p->r_pad * p->r_pad);
   if (!ok) {
     free_plan_memory(p);
     delete p;
@@ -833,20 +1012,24 @@ int dv_memory_plan(const dv_config* cfg, const dv_weights* w, void* stream, dv_p
   const uint16_t* Wk = static_cast<const uint16_t*>(w->Wk);
   const uint16_t* Wv = static_cast<const uint16_t*>(w->Wv);
   cudaMemsetAsync(p->status, 0, sizeof(int), st);
-  k_pack_down<<<grid_for(1LL * L * p->r_pad * d), 256, 0, st>>>(D, p->Dst, L, r, p->r_pad, d, pl);
+  k_pack_down<<<grid_for(1LL * L * p->r_pad * d), 256, 0, st>>>(D, p->Dst, L, r, p->r_pad, d,
+                                                                dst_ld, pl);
   k_pack_kv<<<grid_for(1LL * L * 2 * p->kv * p->k_total), 256, 0, st>>>(Wk, Wv, G, p->Wkv, L, p->kv,
                                                                         HD, d, p->k_total, pl);
   if (rec) {
     k_pack_up<<<grid_for(1LL * L * d * p->r_pad), 256, 0, st>>>(U, p->Uup, L, r, p->r_pad, d, pl);
   } else {
+    k_pack_2u<<<grid_for(1LL * L * p->r_pad * d), 256, 0, st>>>(
+        U, p->Dst + static_cast<size_t>(L) * p->r_pad * dst_ld, L, r, p->r_pad, d, dst_ld, pl);
+    cudaMemsetAsync(p->Gf, 0, sizeof(float) * L * p->r_pad * p->r_pad, st);
     k_pack_norm_u<<<grid_for(1LL * L * p->r_pad * p->k_total), 256, 0, st>>>(U, p->Bn, L, r, p->r_pad,
                                                                              d, p->k_total, pl);
     dim3 g1((r + 63) / 64, (r + 63) / 64, L);
     k_rank_product<1><<<g1, 256, 0, st>>>(Wk, Wv, G, U, p->Bn, r, r, d, p->kv, HD, p->r_pad,
-                                          p->k_total, pl);
+                                          p->k_total, pl, p->Gf);
     dim3 g0((r + 63) / 64, (2 * p->kv + 63) / 64, L);
     k_rank_product<0><<<g0, 256, 0, st>>>(Wk, Wv, G, U, p->Wkv, 2 * p->kv, r, d, p->kv, HD,
-                                          p->r_pad, p->k_total, pl);
+                                          p->r_pad, p->k_total, pl, nullptr);
   }
   if (cfg->has_kv_bias) {
     k_bias_to_f32<<<grid_for(1LL * L * p->kv), 256, 0, st>>>(static_cast<const uint16_t*>(w->bk),
@@ -865,15 +1048,15 @@ int dv_memory_plan(const dv_config* cfg, const dv_weights* w, void* stream, dv_p
     return DV_ERR_CUDA;
   }
 
-  bool enc = encode_2d(&p->tm_Dst[0], p->Dst, d, 1ull * L * p->r_pad, d, 64) &&
-             encode_2d(&p->tm_Dst[1], p->Dst, d, 1ull * L * p->r_pad, d, 128) &&
-             encode_2d(&p->tm_Dst[2], p->Dst, d, 1ull * L * p->r_pad, d, 256) &&
-             encode_2d(&p->tm_Dst_half[0], p->Dst, d, 1ull * L * p->r_pad, d, 32) &&
-             encode_2d(&p->tm_Dst_half[1], p->Dst, d, 1ull * L * p->r_pad, d, 64) &&
-             encode_2d(&p->tm_Dst_half[2], p->Dst, d, 1ull * L * p->r_pad, d, 128) &&
+  bool enc = encode_2d(&p->tm_Dst[0], p->Dst, d, dst_rows, dst_ld, 64) &&
+             encode_2d(&p->tm_Dst[1], p->Dst, d, dst_rows, dst_ld, 128) &&
+             encode_2d(&p->tm_Dst[2], p->Dst, d, dst_rows, dst_ld, 256) &&
+             encode_2d(&p->tm_Dst_half[0], p->Dst, d, dst_rows, dst_ld, 32) &&
+             encode_2d(&p->tm_Dst_half[1], p->Dst, d, dst_rows, dst_ld, 64) &&
+             encode_2d(&p->tm_Dst_half[2], p->Dst, d, dst_rows, dst_ld, 128) &&
              encode_2d(&p->tm_Wkv, p->Wkv, p->k_total, 1ull * L * 2 * p->kv, p->k_total, 128);
   if (enc && rec) {
-    enc = encode_2d(&p->tm_Dst_rp, p->Dst, d, 1ull * L * p->r_pad, d, p->r_pad) &&
+    enc = encode_2d(&p->tm_Dst_rp, p->Dst, d, 1ull * L * p->r_pad, dst_ld, p->r_pad) &&
           encode_2d(&p->tm_Uup, p->Uup, p->r_pad, 1ull * L * d, p->r_pad, p->resid_bn);
   } else if (enc) {
     enc = encode_2d(&p->tm_Bn_half, p->Bn, p->k_total, 1ull * L * p->r_pad, p->k_total,

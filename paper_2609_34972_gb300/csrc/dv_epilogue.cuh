@@ -38,12 +38,33 @@ __device__ __forceinline__ void rope_sincos(float pos, float fhi, float flo, con
   __sincosf(r, &s, &c);
 }
 
-// H[t, n*BN + c] = bf16(SiLU(z)), SiLU(z) = z / (1 + e^-z)  (phi of Sec. 3.1 Eq. 4).
+// H[t, n*BN + c] = bf16(SiLU(z)), SiLU(z) = z / (1 + e^-z)  (phi of Sec. 3.1 Eq. 4); tiles past
+// the down-projection columns store the raw fp32 product into C instead (the launch picks BN
+// dividing n_h, so no tile straddles the two).
 template <int BN>
 __device__ __forceinline__ void epi_silu(const GemmParams& p, uint32_t tbase, int n, int t) {
   const bool valid = t < p.s.M;
+  const int col0 = n * BN;
+  if (col0 >= p.silu.n_h) {
+    float* crow = p.silu.C + static_cast<size_t>(valid ? t : 0) * p.silu.ldc + (col0 - p.silu.n_h);
+#pragma unroll 1
+    for (int c = 0; c < BN / 32; ++c) {
+      uint32_t r[32];
+      __syncwarp();
+      tmem_ld32(tbase + c * 32, r);
+      tmem_ld_wait();
+      if (valid) {
+        float4* dst = reinterpret_cast<float4*>(crow + c * 32);
+#pragma unroll
+        for (int q = 0; q < 8; ++q)
+          dst[q] = make_float4(__uint_as_float(r[4 * q]), __uint_as_float(r[4 * q + 1]),
+                               __uint_as_float(r[4 * q + 2]), __uint_as_float(r[4 * q + 3]));
+      }
+    }
+    return;
+  }
   uint16_t* out = p.silu.H + static_cast<size_t>(valid ? t : 0) * p.silu.ldh +
-                  static_cast<size_t>(n) * BN;
+                  static_cast<size_t>(col0);
 #pragma unroll 1
   for (int c = 0; c < BN / 32; ++c) {
     uint32_t r[32];

@@ -41,9 +41,14 @@ struct GemmShape {
   int a0_rows_per_layer;  // 0: one A0 for every layer; else A0 rows of layer l start at l * it
 };
 
+// Columns [0, n_h) of the product are down-projections: H = bf16(SiLU(acc)). Columns from n_h
+// on (x0 (2 U_l)^T when the statistic of M_l is formed outside a GEMM) go to C as fp32.
 struct EpiSilu {
-  uint16_t* H;   // bf16 [M_ld][ldh]
+  uint16_t* H;   // bf16 [M][ldh]
   int ldh;
+  int n_h;       // columns that are down-projections
+  float* C;      // fp32 [M][ldc] or null
+  int ldc;
 };
 
 struct EpiNorm {
@@ -167,7 +172,9 @@ struct PlanView {
   const float* bk;
   const float* bv;
   int* status;
-  const CUtensorMap* tm_Dst;       // three maps: boxes of 64, 128, 256 rows
+  const CUtensorMap* tm_Dst;       // three maps: boxes of 64, 128, 256 rows; embedding adapter:
+                                   // rows [0, L r_pad) D, rows [L r_pad, 2 L r_pad) 2 U^T
+  const float* Gf;                 // embedding adapter: G_l = U_l^T U_l, fp32 [L][r_pad][r_pad]
   const CUtensorMap* tm_Dst_half;  // three maps: boxes of 32, 64, 128 rows (CTA-pair halves)
   const CUtensorMap* tm_Bn;        // boxes of r_pad rows
   const CUtensorMap* tm_Bn_half;   // boxes of r_pad / 2 rows
@@ -194,6 +201,7 @@ struct BuildArgs {
   uint16_t* H;          // [tokens][L * r_pad] bf16
   float* rstd;          // [L][tokens]
   float* xx;            // [tokens]
+  float* c;             // embedding adapter, small token counts: fp32 [tokens][L * r_pad]
   float* state;         // recurrent: fp32 [tokens][d]
   uint16_t* mem;        // recurrent: bf16 [L][tokens][d]
   float* part;          // recurrent: fp32 [L][d / 64][tokens]
