@@ -13,7 +13,7 @@ HERE = os.path.dirname(os.path.abspath(__file__))
 ROOT = os.path.dirname(HERE)
 CSRC = os.path.join(HERE, "csrc")
 LIB_PATH = os.path.join(HERE, "libdv.so")
-SOURCES = ["dv_api.cu", "dv_gemm.cu", "dv_kv2sm.cu", "dv_pair_tm.cu", "dv_recurrent.cu", "dv_attention.cu",
+SOURCES = ["dv_api.cu", "dv_gemm.cu", "dv_kv2sm.cu", "dv_pair_tm.cu", "dv_recurrent.cu", "dv_chain.cu", "dv_attention.cu",
            "dv_noalloc.cu"]
 HEADERS = ["dv_internal.h", "dv_ptx.cuh", "dv_epilogue.cuh"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]

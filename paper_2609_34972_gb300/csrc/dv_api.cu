@@ -100,6 +100,21 @@ bool encode_2d(CUtensorMap* map, const void* ptr, uint64_t cols, uint64_t rows, 
             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+// bf16 3-D tensor [L][rows][cols] (rows x cols per layer, packed), boxes of 64 columns x
+// box_rows rows x 1 layer with 128-byte swizzle: a store past `rows` is clipped per layer.
+bool encode_3d(CUtensorMap* map, const void* ptr, uint64_t cols, uint64_t rows, uint64_t layers,
+               uint32_t box_rows) {
+  EncodeTiledFn fn = encode_fn();
+  if (!fn) return false;
+  cuuint64_t dims[3] = {cols, rows, layers};
+  cuuint64_t strides[2] = {cols * 2, cols * rows * 2};
+  cuuint32_t box[3] = {static_cast<cuuint32_t>(dv::kBlockK), box_rows, 1};
+  cuuint32_t estr[3] = {1, 1, 1};
+  return fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(ptr), dims, strides, box,
+            estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+            CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
 // ------------------------------------------------------------------------------ small kernels
 
 __device__ __forceinline__ float bf(uint16_t b) { return __uint_as_float(static_cast<uint32_t>(b) << 16); }
@@ -640,6 +655,24 @@ static cudaError_t launch_kv_stage(const PlanView& v, GemmParams& gp, long long 
                         st);
 }
 
+// K/V stage of a recurrent build: every layer in one launch, A = the stacked M_l.
+template <typename Mark>
+static cudaError_t launch_recurrent_kv(const PlanView& v, const BuildArgs& a, long long T,
+                                       const CUtensorMap& tm_mem, cudaStream_t st, Mark& mark) {
+  const int L = v.n_layers, d = v.d;
+  GemmParams gp;
+  std::memset(&gp, 0, sizeof(gp));
+  gp.status = v.status;
+  gp.timeout_ns = kTimeoutNs;
+  for (int i = 0; i < L; ++i) gp.layer_map[i] = v.active[i];
+  gp.s = {static_cast<int>(T), L, 2 * v.kv, d / 64, 0, 0, 0, 0, 0, static_cast<int>(T)};
+  fill_epi_kv(v, a, T, gp.kv);
+  const cudaError_t err = launch_kv_stage(v, gp, T, a.mem, static_cast<uint64_t>(L) * T, tm_mem,
+                                          nullptr, 0, tm_mem, st);
+  mark(4);
+  return err;
+}
+
 // Recurrent adapter (Sec. 3.1 Eq. 6): the chain M_i = M_{i-1} + SiLU(M_{i-1} D_i) U_i runs
 // layer by layer (a split-K down-projection, then the up-projection whose epilogue adds the
 // fp32 state and writes bf16 M_i and partial sums of squares); the RMS statistics of all
@@ -659,6 +692,28 @@ static cudaError_t enqueue_recurrent(const PlanView& v, const BuildArgs& a, cuda
 
   mark(0);
   mark(1);
+  const long long part_ld = static_cast<long long>(d / 64) * T;
+  cudaError_t err = cudaSuccess;
+  // On chip: one cluster per 128-token block runs the whole chain with the state in TMEM.
+  int spc = 0, S = 0;
+  if (chain_shape(d, v.r_pad, &spc, &S)) {
+    CUtensorMap tm_u, tm_m3;
+    if (!encode_2d(&tm_u, v.Uup, v.r_pad, static_cast<uint64_t>(L) * d, v.r_pad, 64 * spc) ||
+        !encode_3d(&tm_m3, a.mem, d, static_cast<uint64_t>(T), L, kBlockM))
+      return cudaErrorInvalidValue;
+    err = launch_chain(v.r_pad, spc, S, T, L, d, tm_x0, *v.tm_Dst_rp, tm_u, tm_m3, a.part, part_ld,
+                       a.H, v.status, kTimeoutNs, st);
+    if (err == cudaSuccess) {
+      mark(2);
+      k_rstd_parts<<<grid_for(static_cast<long long>(L) * T), 256, 0, st>>>(
+          a.part, L, T, S, part_ld, 1.0f / d, v.rms_eps, a.rstd);
+      err = cudaGetLastError();
+      mark(3);
+      return err == cudaSuccess ? launch_recurrent_kv(v, a, T, tm_mem, st, mark) : err;
+    }
+    if (err != cudaErrorNotSupported) return err;
+    err = cudaSuccess;  // no cluster of that size fits: the per-layer launches below
+  }
   const long long m_tiles = (T + kBlockM - 1) / kBlockM;
   const int splits = down_splits(m_tiles, d / kBlockK, v.num_sms);
   DownParams dp;
@@ -675,8 +730,6 @@ static cudaError_t enqueue_recurrent(const PlanView& v, const BuildArgs& a, cuda
   gp.timeout_ns = kTimeoutNs;
   // up-projection step: A = h_i (H columns from i * r_pad), B = U_i ([d][r_pad] rows i * d)
   gp.s = {static_cast<int>(T), 1, d, 0, v.r_pad / 64, v.r_pad, 0, 0, 0, 0};
-  const long long part_ld = static_cast<long long>(d / 64) * T;
-  cudaError_t err = cudaSuccess;
   for (int i = 0; i < L && err == cudaSuccess; ++i) {
     dp.a_row0 = i == 0 ? 0 : static_cast<int>((i - 1) * T);
     dp.b_row0 = i * v.r_pad;
@@ -696,18 +749,7 @@ static cudaError_t enqueue_recurrent(const PlanView& v, const BuildArgs& a, cuda
     err = cudaGetLastError();
   }
   mark(3);
-
-  std::memset(&gp, 0, sizeof(gp));
-  gp.status = v.status;
-  gp.timeout_ns = kTimeoutNs;
-  for (int i = 0; i < L; ++i) gp.layer_map[i] = v.active[i];
-  gp.s = {static_cast<int>(T), L, 2 * v.kv, d / 64, 0, 0, 0, 0, 0, static_cast<int>(T)};
-  fill_epi_kv(v, a, T, gp.kv);
-  if (err == cudaSuccess)
-    err = launch_kv_stage(v, gp, T, a.mem, static_cast<uint64_t>(L) * T, tm_mem, nullptr, 0,
-                          tm_mem, st);
-  mark(4);
-  return err;
+  return err == cudaSuccess ? launch_recurrent_kv(v, a, T, tm_mem, st, mark) : err;
 }
 
 cudaError_t enqueue_build(const PlanView& v, const BuildArgs& a, cudaStream_t st) {
@@ -874,6 +916,7 @@ bool plan_view(const dv_plan* p, PlanView* v) {
   v->tm_Wkv = &p->tm_Wkv;
   v->tm_Dst_rp = &p->tm_Dst_rp;
   v->tm_Uup = &p->tm_Uup;
+  v->Uup = p->Uup;
   v->resid_bn = p->resid_bn;
   v->inv_freq = p->inv_freq;
   v->Wkv = p->Wkv;

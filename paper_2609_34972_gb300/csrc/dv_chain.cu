@@ -1,0 +1,494 @@
+// The recurrent adapter's chain (Sec. 3.1 Eq. 6) kept on chip: M_0 = E and
+//   M_l = M_{l-1} + SiLU(M_{l-1} D_l) U_l,   l = 1 .. L,
+// for one 128-token block per thread-block cluster, through all layers in one launch.
+//
+// The cluster's S CTAs split the hidden dimension: CTA s owns columns [s CW, (s + 1) CW).
+//   - Its slice of the fp32 state M (128 rows x CW) lives in TMEM for the whole chain; the
+//     up-projection MMA accumulates h_l U_l^T straight into it.
+//   - Its bf16 copy of that slice sits in shared memory (128-byte-swizzled K-major slabs): the A
+//     operand of its part of the down-projection and the source of the TMA store of M_l.
+// Per layer:
+//   1. down-projection partial: z_s = bf16(M_{l-1})[:, slice] D_l[:, slice]^T (TMEM, fp32);
+//   2. the partial goes to shared memory (over the bf16 slice, whose readers are done) and,
+//      after a cluster barrier, CTA s sums rows [s 128 / S, (s + 1) 128 / S) over the S partials
+//      through distributed shared memory in the fixed order 0 .. S-1, applies SiLU and writes
+//      bf16 h straight into the h tile (A operand of the up-projection) of every CTA;
+//   3. after a second cluster barrier: state += h U_l[slice, :]^T (TMEM);
+//   4. the state slice is read back, its bf16 rounding written over the bf16 slice (next layer's
+//      A operand, then stored to the stacked M_l by TMA) and its rows' sums of squares written to
+//      `part` (the K/V stage's RMS statistic adds the S partials).
+// D_{l+1} and U_{l+1} load (TMA) while the rest of layer l runs. Only bf16 M_l and the partial
+// sums of squares leave the chip; the state never does. Every wait is bounded; a CTA that gives
+// up keeps passing the cluster barriers (so its peers finish), stops issuing work, drains what
+// it issued and flags the plan's status word.
+#include "../../include/dv.h"
+#include "dv_internal.h"
+#include "dv_ptx.cuh"
+
+namespace dv {
+namespace {
+
+constexpr int kChainThreads = 128;
+
+template <int RP, int SPC>
+struct ChainCfg {
+  static constexpr int CW = 64 * SPC;             // hidden columns per CTA
+  static constexpr int kSlab = 128 * 128;         // [128 rows][64 bf16], 128-byte swizzle
+  static constexpr int kA = SPC * kSlab;          // bf16 state slice
+  static constexpr int kH = (RP / 64) * kSlab;    // bf16 h
+  static constexpr int kDslab = RP * 128;         // D_l: RP rows x 64 columns
+  static constexpr int kD = SPC * kDslab;
+  static constexpr int kUslab = CW * 128;         // U_l: CW rows x 64 rank columns
+  static constexpr int kU = (RP / 64) * kUslab;
+  static constexpr int kOffA = 0;
+  static constexpr int kOffH = kOffA + kA;
+  static constexpr int kOffD = kOffH + kH;
+  static constexpr int kOffU = kOffD + kD;
+  static constexpr int kEnd = kOffU + kU;
+  static constexpr int kZ = 128 * RP * 4;         // fp32 partial z over the bf16 slice
+  static constexpr int kSmemBytes = kEnd + 1024 + 256;
+  static constexpr int kTmemCols = CW + RP <= 256 ? 256 : 512;
+  static_assert(kZ <= kA, "the partial z reuses the bf16 state slice");
+  static_assert(kSmemBytes <= 232448, "shared memory of one CTA");
+  static_assert(kDslab % 1024 == 0 && kUslab % 1024 == 0, "tiles stay 1024-byte aligned");
+};
+
+struct ChainParams {
+  int M;              // tokens
+  int L;              // planned layers
+  int d;
+  float* part;        // fp32 [L][part_ld / M][M]: partial sums of squares of M_l
+  long long part_ld;  // layer stride of part
+  uint16_t* H;        // bf16 [M][ldh]: h_l at columns l r_pad (kept for stage-wise checks)
+  int ldh;
+  int* status;
+  unsigned long long timeout_ns;
+};
+
+__device__ __forceinline__ uint32_t n_cluster_ctas() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%cluster_nctarank;" : "=r"(r));
+  return r;
+}
+
+__device__ __forceinline__ float4 ld_cluster_f4(uint32_t caddr) {
+  float4 v;
+  asm volatile("ld.shared::cluster.v4.f32 {%0, %1, %2, %3}, [%4];"
+               : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w)
+               : "r"(caddr)
+               : "memory");
+  return v;
+}
+
+__device__ __forceinline__ void st_cluster_u2(uint32_t caddr, uint2 v) {
+  asm volatile("st.shared::cluster.v2.b32 [%0], {%1, %2};" ::"r"(caddr), "r"(v.x), "r"(v.y)
+               : "memory");
+}
+
+// Registers -> TMEM: lane i of the warp writes TMEM lane (taddr.lane + i), 32 columns.
+__device__ __forceinline__ void tmem_st32(uint32_t taddr, const uint32_t (&r)[32]) {
+  asm volatile(
+      "tcgen05.st.sync.aligned.32x32b.x32.b32 [%0],"
+      " {%1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, %16,"
+      " %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31, %32};" ::"r"(
+          taddr),
+      "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7]),
+      "r"(r[8]), "r"(r[9]), "r"(r[10]), "r"(r[11]), "r"(r[12]), "r"(r[13]), "r"(r[14]),
+      "r"(r[15]), "r"(r[16]), "r"(r[17]), "r"(r[18]), "r"(r[19]), "r"(r[20]), "r"(r[21]),
+      "r"(r[22]), "r"(r[23]), "r"(r[24]), "r"(r[25]), "r"(r[26]), "r"(r[27]), "r"(r[28]),
+      "r"(r[29]), "r"(r[30]), "r"(r[31])
+      : "memory");
+}
+
+__device__ __forceinline__ void tmem_st_wait() {
+  asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
+}
+
+// 3-D tiled store from shared memory (bulk-group completion).
+__device__ __forceinline__ void tma_store_3d(const CUtensorMap* map, uint32_t src, int c0, int c1,
+                                             int c2) {
+  asm volatile(
+      "cp.async.bulk.tensor.3d.global.shared::cta.bulk_group [%0, {%2, %3, %4}], [%1];" ::"l"(
+          reinterpret_cast<uint64_t>(map)),
+      "r"(src), "r"(c0), "r"(c1), "r"(c2)
+      : "memory");
+}
+
+__device__ __forceinline__ void bulk_commit() { asm volatile("cp.async.bulk.commit_group;" ::: "memory"); }
+__device__ __forceinline__ void bulk_wait_read0() {
+  asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory");
+}
+__device__ __forceinline__ void bulk_wait0() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
+
+__device__ __forceinline__ void fence_proxy_async_cta() {
+  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+__device__ __forceinline__ void fence_proxy_async_cluster() {
+  asm volatile("fence.proxy.async.shared::cluster;" ::: "memory");
+}
+
+__device__ __forceinline__ bool wait_bounded(uint32_t bar, uint32_t parity, uint64_t timeout_ns) {
+  int never = 0;
+  return mbar_wait(bar, parity, &never, timeout_ns);
+}
+
+__device__ __forceinline__ float silu(float z) { return z / (1.0f + __expf(-z)); }
+
+// Byte offset of 16-byte chunk `c` (8 bf16, c < 8) of row `row` in a 128-byte-swizzled slab.
+__device__ __forceinline__ uint32_t sw128(int row, int c) {
+  return static_cast<uint32_t>(row * 128 + ((c ^ (row & 7)) << 4));
+}
+
+template <int RP, int SPC>
+__global__ void __launch_bounds__(kChainThreads, 1)
+    dv_chain_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_constant__ CUtensorMap tmD,
+                    const __grid_constant__ CUtensorMap tmU, const __grid_constant__ CUtensorMap tmM,
+                    const __grid_constant__ ChainParams p) {
+  using C = ChainCfg<RP, SPC>;
+  constexpr int CW = C::CW;
+  extern __shared__ uint8_t smem_raw[];
+  const uint32_t raw = smem_addr(smem_raw);
+  const uint32_t base = (raw + 1023u) & ~1023u;
+  uint8_t* base_ptr = smem_raw + (base - raw);
+  uint64_t* bars = reinterpret_cast<uint64_t*>(base_ptr + C::kEnd);
+  const uint32_t bar0 = smem_addr(bars);
+  const uint32_t bar_x = bar0, bar_d = bar0 + 8, bar_u = bar0 + 16, bar_z = bar0 + 24,
+                 bar_up = bar0 + 32, bar_drain = bar0 + 40;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 6);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+
+  const int tid = threadIdx.x, warp = tid >> 5;
+  const uint64_t tmo = p.timeout_ns;
+  const int s = static_cast<int>(cluster_ctarank());
+  const int S = static_cast<int>(n_cluster_ctas());
+  const int m = static_cast<int>(cluster_id_x());
+  const int col0 = s * CW, row0 = m * 128;
+  const int t = row0 + tid;  // this thread's token row
+  const uint32_t sA = base + C::kOffA, sH = base + C::kOffH, sD = base + C::kOffD,
+                 sU = base + C::kOffU;
+  float* zpart = reinterpret_cast<float*>(base_ptr + C::kOffA);
+
+  if (tid == 0) {
+    mbar_init(bar_x, 1);
+    mbar_init(bar_d, 1);
+    mbar_init(bar_u, 1);
+    mbar_init(bar_z, 1);
+    mbar_init(bar_up, 1);
+    mbar_init(bar_drain, 1);
+    *abort_flag = 0;
+    fence_barrier_init();
+  }
+  if (warp == 0) {
+    tmem_alloc(smem_addr(tmem_slot), C::kTmemCols);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+  const uint32_t t_state = tmem, t_z = tmem + CW;
+  const uint32_t lane_base = static_cast<uint32_t>(warp * 32) << 16;
+
+  // thread 0's bookkeeping of async work, for the drain after an abort
+  int d_loads = 0, d_waits = 0, u_loads = 0, u_waits = 0;
+  bool mma_open = false;
+  auto load_d = [&](int l) {
+    mbar_arrive_expect_tx(bar_d, C::kD);
+    for (int j = 0; j < SPC; ++j)
+      tma_load_2d(sD + j * C::kDslab, &tmD, bar_d, col0 + 64 * j, l * RP);
+    ++d_loads;
+  };
+  auto load_u = [&](int l) {
+    mbar_arrive_expect_tx(bar_u, C::kU);
+    for (int j = 0; j < RP / 64; ++j)
+      tma_load_2d(sU + j * C::kUslab, &tmU, bar_u, 64 * j, l * p.d + col0);
+    ++u_loads;
+  };
+
+  if (tid == 0) {
+    tma_prefetch_desc(&tmX);
+    tma_prefetch_desc(&tmD);
+    tma_prefetch_desc(&tmU);
+    tma_prefetch_desc(&tmM);
+    mbar_arrive_expect_tx(bar_x, C::kA);
+    for (int j = 0; j < SPC; ++j) tma_load_2d(sA + j * C::kSlab, &tmX, bar_x, col0 + 64 * j, row0);
+    load_d(0);
+    load_u(0);
+  }
+
+  // M_0 = E: the state slice in TMEM is the fp32 widening of the bf16 slice just loaded.
+  bool ok = mbar_wait(bar_x, 0, abort_flag, tmo);
+  if (__all_sync(0xFFFFFFFFu, ok)) {
+#pragma unroll 1
+    for (int c = 0; c < CW / 32; ++c) {
+      const uint8_t* slab = base_ptr + C::kOffA + (c / 2) * C::kSlab;
+      uint32_t r[32];
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        const uint4 w = *reinterpret_cast<const uint4*>(slab + sw128(tid, (c % 2) * 4 + q));
+        const uint32_t ws[4] = {w.x, w.y, w.z, w.w};
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          r[q * 8 + 2 * e] = ws[e] << 16;
+          r[q * 8 + 2 * e + 1] = ws[e] & 0xFFFF0000u;
+        }
+      }
+      tmem_st32(t_state + lane_base + c * 32, r);
+    }
+    tmem_st_wait();
+  }
+  tc_fence_before();
+  ok = __syncthreads_and(ok) != 0;
+
+  for (int l = 0; l < p.L; ++l) {
+    const uint32_t ph = static_cast<uint32_t>(l) & 1u;
+
+    // (1) down-projection partial z = bf16(M_{l-1})[:, slice] D_l[:, slice]^T; store M_{l-1}
+    if (tid == 0 && ok && !*abort_flag) {
+      tc_fence_after();
+      fence_proxy_async_cta();  // the bf16 slice was written by the threads
+      if (mbar_wait(bar_d, ph, abort_flag, tmo)) {
+        ++d_waits;
+        const uint32_t idesc = idesc_bf16_f32(128, RP);
+        for (int j = 0; j < SPC; ++j)
+#pragma unroll
+          for (int k = 0; k < 4; ++k)
+            umma_bf16(t_z, sdesc_kmajor_sw128(sA + j * C::kSlab + 32u * k),
+                      sdesc_kmajor_sw128(sD + j * C::kDslab + 32u * k), idesc,
+                      (j | k) != 0 ? 1u : 0u);
+        umma_commit(bar_z);
+        mma_open = true;
+      }
+      if (l >= 1) {
+        for (int j = 0; j < SPC; ++j)
+          tma_store_3d(&tmM, sA + j * C::kSlab, col0 + 64 * j, row0, l - 1);
+        bulk_commit();
+      }
+    }
+
+    // (2) z partial -> shared memory, over the bf16 slice (down MMA and store have read it)
+    bool zok = ok && mbar_wait(bar_z, ph, abort_flag, tmo);
+    if (tid == 0) {
+      bulk_wait_read0();
+      if (zok) mma_open = false;
+    }
+    zok = __syncthreads_and(zok) != 0;
+    if (zok) {
+      tc_fence_after();
+      float* zrow = zpart + tid * RP;
+#pragma unroll 1
+      for (int c = 0; c < RP / 32; ++c) {
+        uint32_t r[32];
+        __syncwarp();
+        tmem_ld32(t_z + lane_base + c * 32, r);
+        tmem_ld_wait();
+#pragma unroll
+        for (int q = 0; q < 8; ++q) {
+          const int c4 = c * 8 + q;
+          reinterpret_cast<float4*>(zrow)[c4 ^ (tid & 7)] =
+              make_float4(__uint_as_float(r[4 * q]), __uint_as_float(r[4 * q + 1]),
+                          __uint_as_float(r[4 * q + 2]), __uint_as_float(r[4 * q + 3]));
+        }
+      }
+      if (tid == 0 && l + 1 < p.L) load_d(l + 1);  // the D buffer is free
+    }
+    ok = zok;
+    tc_fence_before();
+    __syncwarp();
+    cluster_sync();
+
+    // (3) rows [s 128 / S, (s + 1) 128 / S): sum the S partials in order, SiLU, bf16 h into the
+    // h tile of every CTA (8-byte pieces, swizzled as the MMA reads them). One item is 4 values
+    // (one float4) of one row: its S remote loads are all in flight before the sum.
+    {
+      const int r_lo = s * 128 / S, r_hi = (s + 1) * 128 / S;
+      const int items = (r_hi - r_lo) * (RP / 4);
+#pragma unroll 1
+      for (int it = tid; it < items; it += kChainThreads) {
+        const int row = r_lo + it / (RP / 4), c4 = it % (RP / 4);
+        const uint32_t zl = smem_addr(zpart + row * RP) + ((c4 ^ (row & 7)) << 4);
+        float4 v[16];
+#pragma unroll
+        for (int b = 0; b < 16; ++b)
+          if (b < S) v[b] = ld_cluster_f4(map_to_rank(zl, static_cast<uint32_t>(b)));
+        float4 z = make_float4(0.0f, 0.0f, 0.0f, 0.0f);
+#pragma unroll
+        for (int b = 0; b < 16; ++b) {
+          if (b < S) {
+            z.x += v[b].x;
+            z.y += v[b].y;
+            z.z += v[b].z;
+            z.w += v[b].w;
+          }
+        }
+        uint2 hv;
+        hv.x = pack_bf16x2(silu(z.x), silu(z.y));
+        hv.y = pack_bf16x2(silu(z.z), silu(z.w));
+        // columns 4 c4 .. 4 c4 + 3: slab c4 / 16, 16-byte chunk (c4 % 16) / 2, half c4 % 2
+        const uint32_t hl = sH + (c4 / 16) * C::kSlab + sw128(row, (c4 % 16) / 2) + (c4 % 2) * 8;
+        for (int b = 0; b < S; ++b) st_cluster_u2(map_to_rank(hl, static_cast<uint32_t>(b)), hv);
+        if (row0 + row < p.M)
+          *reinterpret_cast<uint2*>(p.H + static_cast<long long>(row0 + row) * p.ldh + l * RP +
+                                    c4 * 4) = hv;
+      }
+    }
+    fence_proxy_async_cluster();
+    __syncwarp();
+    cluster_sync();
+
+    // (4) state += h U_l[slice, :]^T
+    if (tid == 0 && ok && !*abort_flag) {
+      fence_proxy_async_cta();
+      tc_fence_after();
+      if (mbar_wait(bar_u, ph, abort_flag, tmo)) {
+        ++u_waits;
+        const uint32_t idesc = idesc_bf16_f32(128, CW);
+        for (int j = 0; j < RP / 64; ++j)
+#pragma unroll
+          for (int k = 0; k < 4; ++k)
+            umma_bf16(t_state, sdesc_kmajor_sw128(sH + j * C::kSlab + 32u * k),
+                      sdesc_kmajor_sw128(sU + j * C::kUslab + 32u * k), idesc, 1u);
+        umma_commit(bar_up);
+        mma_open = true;
+      }
+    }
+    bool uok = ok && mbar_wait(bar_up, ph, abort_flag, tmo);
+    if (tid == 0 && uok) {
+      mma_open = false;
+      if (l + 1 < p.L) load_u(l + 1);  // the U buffer is free
+    }
+    // (5) state -> bf16 slice (next A operand, stored next layer) and sums of squares
+    if (__all_sync(0xFFFFFFFFu, uok)) {
+      tc_fence_after();
+      float ss = 0.0f;
+#pragma unroll 1
+      for (int c2 = 0; c2 < CW / 64; ++c2) {  // one 64-column slab: two TMEM loads in flight
+        uint32_t r[2][32];
+        __syncwarp();
+        tmem_ld32(t_state + lane_base + c2 * 64, r[0]);
+        tmem_ld32(t_state + lane_base + c2 * 64 + 32, r[1]);
+        tmem_ld_wait();
+        uint8_t* slab = base_ptr + C::kOffA + c2 * C::kSlab;
+#pragma unroll
+        for (int h2 = 0; h2 < 2; ++h2) {
+          uint32_t pk[16];
+#pragma unroll
+          for (int u = 0; u < 16; ++u) {
+            const float a = __uint_as_float(r[h2][2 * u]), b = __uint_as_float(r[h2][2 * u + 1]);
+            ss = fmaf(a, a, ss);
+            ss = fmaf(b, b, ss);
+            pk[u] = pack_bf16x2(a, b);
+          }
+#pragma unroll
+          for (int q = 0; q < 4; ++q)
+            *reinterpret_cast<uint4*>(slab + sw128(tid, h2 * 4 + q)) =
+                make_uint4(pk[4 * q], pk[4 * q + 1], pk[4 * q + 2], pk[4 * q + 3]);
+        }
+      }
+      if (t < p.M) p.part[l * p.part_ld + static_cast<long long>(s) * p.M + t] = ss;
+    }
+    fence_proxy_async_cta();
+    tc_fence_before();
+    ok = __syncthreads_and(uok) != 0;
+  }
+
+  if (tid == 0) {
+    if (ok && !*abort_flag && p.L > 0) {
+      for (int j = 0; j < SPC; ++j)
+        tma_store_3d(&tmM, sA + j * C::kSlab, col0 + 64 * j, row0, p.L - 1);
+      bulk_commit();
+    }
+    bulk_wait0();
+    if (!ok || *abort_flag) {  // let issued loads land and issued MMAs finish
+      if (d_loads > d_waits) wait_bounded(bar_d, static_cast<uint32_t>(d_loads - 1) & 1u, tmo);
+      if (u_loads > u_waits) wait_bounded(bar_u, static_cast<uint32_t>(u_loads - 1) & 1u, tmo);
+      if (mma_open) {
+        umma_commit(bar_drain);
+        wait_bounded(bar_drain, 0, tmo);
+      }
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  __syncwarp();
+  cluster_sync();
+  if (warp == 0) {
+    tc_fence_after();
+    tmem_dealloc(tmem, C::kTmemCols);
+  }
+  if (tid == 0 && (!ok || *abort_flag)) atomicExch(p.status, DV_ERR_DEVICE_TIMEOUT);
+}
+
+template <int RP, int SPC>
+cudaError_t launch_t(int S, long long blocks, const CUtensorMap& x, const CUtensorMap& dmap,
+                     const CUtensorMap& umap, const CUtensorMap& mmap, const ChainParams& p,
+                     cudaStream_t stream) {
+  using C = ChainCfg<RP, SPC>;
+  auto kern = dv_chain_kernel<RP, SPC>;
+  cudaError_t err =
+      cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, C::kSmemBytes);
+  if (err == cudaSuccess && S > 8)
+    err = cudaFuncSetAttribute(kern, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+  if (err != cudaSuccess) return err;
+  cudaLaunchConfig_t cfg = {};
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = static_cast<unsigned>(S);
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.gridDim = dim3(static_cast<unsigned>(blocks * S), 1, 1);
+  cfg.blockDim = dim3(kChainThreads, 1, 1);
+  cfg.dynamicSmemBytes = C::kSmemBytes;
+  cfg.stream = stream;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  int clusters = 0;
+  if (cudaOccupancyMaxActiveClusters(&clusters, kern, &cfg) != cudaSuccess || clusters < 1) {
+    cudaGetLastError();
+    return cudaErrorNotSupported;  // the caller falls back to the per-layer launches
+  }
+  err = cudaLaunchKernelEx(&cfg, kern, x, dmap, umap, mmap, p);
+  if (err != cudaSuccess) return err;
+  return cudaGetLastError();
+}
+
+}  // namespace
+
+bool chain_shape(int d, int r_pad, int* spc_out, int* s_out) {
+  if (r_pad != 64 && r_pad != 128) return false;
+  const int k_slabs = d / 64;
+  const int min_spc = r_pad == 128 ? 4 : 2;  // the fp32 partial z must fit over the bf16 slice
+  for (int spc = min_spc; spc <= 4; ++spc) {
+    if (k_slabs % spc) continue;
+    const int S = k_slabs / spc;
+    if (S < 1 || S > 16) continue;
+    *spc_out = spc;
+    *s_out = S;
+    return true;
+  }
+  return false;
+}
+
+cudaError_t launch_chain(int r_pad, int spc, int S, long long tokens, int n_layers, int d,
+                         const CUtensorMap& x, const CUtensorMap& dmap, const CUtensorMap& umap,
+                         const CUtensorMap& mmap, float* part, long long part_ld, uint16_t* H,
+                         int* status, unsigned long long timeout_ns, cudaStream_t stream) {
+  ChainParams p;
+  p.H = H;
+  p.ldh = n_layers * r_pad;
+  p.M = static_cast<int>(tokens);
+  p.L = n_layers;
+  p.d = d;
+  p.part = part;
+  p.part_ld = part_ld;
+  p.status = status;
+  p.timeout_ns = timeout_ns;
+  const long long blocks = (tokens + 127) / 128;
+  if (r_pad == 64 && spc == 2) return launch_t<64, 2>(S, blocks, x, dmap, umap, mmap, p, stream);
+  if (r_pad == 64 && spc == 3) return launch_t<64, 3>(S, blocks, x, dmap, umap, mmap, p, stream);
+  if (r_pad == 64 && spc == 4) return launch_t<64, 4>(S, blocks, x, dmap, umap, mmap, p, stream);
+  if (r_pad == 128 && spc == 4) return launch_t<128, 4>(S, blocks, x, dmap, umap, mmap, p, stream);
+  return cudaErrorInvalidValue;
+}
+
+}  // namespace dv

@@ -153,6 +153,18 @@ cudaError_t launch_down_split(int r_pad, int splits, const CUtensorMap& a, const
 // K splits (1, 2, 4 or 8) for m_tiles token blocks of 128 rows and k_slabs slabs.
 int down_splits(long long m_tiles, int k_slabs, int num_sms);
 
+// The recurrent chain on chip (dv_chain.cu): one cluster of S CTAs per 128-token block runs all
+// layers with the fp32 state in TMEM. chain_shape gives the slabs per CTA (spc) and S for a
+// hidden size and r_pad, or false when the chain does not fit (then the per-layer launches
+// run). launch_chain returns cudaErrorNotSupported when no cluster of that size can be resident.
+// x: x0 (128-row boxes); dmap: stacked D (r_pad-row boxes); umap: U as [L d][r_pad] (64 spc-row
+// boxes); mmap: the stacked M_l as a 3-D (d, tokens, L) map with (64, 128, 1) boxes.
+bool chain_shape(int d, int r_pad, int* spc_out, int* s_out);
+cudaError_t launch_chain(int r_pad, int spc, int S, long long tokens, int n_layers, int d,
+                         const CUtensorMap& x, const CUtensorMap& dmap, const CUtensorMap& umap,
+                         const CUtensorMap& mmap, float* part, long long part_ld, uint16_t* H,
+                         int* status, unsigned long long timeout_ns, cudaStream_t stream);
+
 // Token tile (64, 128, 192 or 256) of the pair kernel for a build of `tokens` tokens.
 int kv_pair_tile_n(long long tokens);
 int kv_pair_smem_bytes(int nt);
@@ -181,6 +193,7 @@ struct PlanView {
   const CUtensorMap* tm_Wkv;       // boxes of 128 rows
   const CUtensorMap* tm_Dst_rp;    // recurrent: boxes of r_pad rows (one layer's D)
   const CUtensorMap* tm_Uup;       // recurrent: [L*d][r_pad], boxes of resid_bn rows
+  const uint16_t* Uup;             // recurrent: U_l as [L*d][r_pad]
   int resid_bn;                    // recurrent: column tile of the up-projection step
   const double* inv_freq;     // head_dim / 2 values
   const uint16_t* Wkv;        // repacked K/V weights [L*2kv][k_total]
