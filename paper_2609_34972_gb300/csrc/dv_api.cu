@@ -43,8 +43,10 @@ struct dv_plan {
   long long last_tokens = 0;   // tokens of the last build (layout of the workspace)
   int* status = nullptr;
   CUtensorMap tm_Dst[3];       // boxes of 64, 128, 256 rows
-  CUtensorMap tm_Dst_half[3];  // boxes of 32, 64, 128 rows (halves for CTA pairs)
-  CUtensorMap tm_Bn, tm_Bn_half, tm_Wkv;
+  CUtensorMap tm_Dst_half[3];  // slab maps, boxes of 32, 64, 128 rows (halves for CTA pairs)
+  CUtensorMap tm_Bn;           // boxes of r_pad rows
+  CUtensorMap tm_Bn_half;      // slab map, boxes of r_pad / 2 rows
+  CUtensorMap tm_Wkv;          // slab map, boxes of 128 rows
   CUtensorMap tm_Dst_rp, tm_Uup;  // recurrent adapter
   int resid_bn = 0;
   double inv_freq[dv::kMaxHalfHead];
@@ -96,6 +98,24 @@ bool encode_2d(CUtensorMap* map, const void* ptr, uint64_t cols, uint64_t rows, 
   cuuint32_t box[2] = {static_cast<cuuint32_t>(dv::kBlockK), box_rows};
   cuuint32_t estr[2] = {1, 1};
   return fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(ptr), dims, strides, box,
+            estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+            CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+// bf16 [rows][cols] (row stride ld elements) viewed as {64 columns, rows, cols / 64 slabs} for
+// the 2-SM kernels: one box = box_rows rows x kSlabsPerStep consecutive K slabs, each slab a
+// 128-byte-swizzled [box_rows][64] tile. cols must be a multiple of 64; slabs past the end of
+// the matrix read as zero.
+bool encode_slabs(CUtensorMap* map, const void* ptr, uint64_t cols, uint64_t rows, uint64_t ld,
+                  uint32_t box_rows) {
+  EncodeTiledFn fn = encode_fn();
+  if (!fn || cols % dv::kBlockK != 0) return false;
+  cuuint64_t dims[3] = {static_cast<cuuint64_t>(dv::kBlockK), rows, cols / dv::kBlockK};
+  cuuint64_t strides[2] = {ld * 2, static_cast<cuuint64_t>(dv::kBlockK) * 2};
+  cuuint32_t box[3] = {static_cast<cuuint32_t>(dv::kBlockK), box_rows,
+                       static_cast<cuuint32_t>(dv::kSlabsPerStep)};
+  cuuint32_t estr[3] = {1, 1, 1};
+  return fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(ptr), dims, strides, box,
             estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
@@ -635,8 +655,9 @@ static void fill_epi_kv(const PlanView& v, const BuildArgs& a, long long T, EpiK
 
 // K/V stage over all planned layers: K/V = rstd_l * (A_l [| h_l] Wkv_l^T) + b, RoPE on K,
 // stored into the cache. gp.s holds the operand schedule; the engine is chosen by token count
-// (tokens-as-M pairs when 256-token blocks pad little, else weights-as-M pairs). a_full /
-// h_full: token operands with 128-row boxes; a_half / h_half: with nt / 2-row boxes.
+// (tokens-as-M pairs when 256-token blocks pad little, else weights-as-M pairs). The token
+// operands are slab maps: a_full / h_full with 128-row boxes, a_half / h_half (made here) with
+// nt / 2-row boxes.
 static cudaError_t launch_kv_stage(const PlanView& v, GemmParams& gp, long long T,
                                    const void* a_ptr, uint64_t a_rows, const CUtensorMap& a_full,
                                    const void* h_ptr, uint64_t h_cols, const CUtensorMap& h_full,
@@ -648,17 +669,18 @@ static cudaError_t launch_kv_stage(const PlanView& v, GemmParams& gp, long long 
     return launch_pair_tm(EPI_KV, 256, v.head_dim, a_full, h_full, *v.tm_Wkv, gp, v.num_sms, st);
   }
   CUtensorMap a_half, h_half;
-  if (!encode_2d(&a_half, a_ptr, v.d, a_rows, v.d, nt / 2)) return cudaErrorInvalidValue;
-  if (h_ptr && !encode_2d(&h_half, h_ptr, h_cols, static_cast<uint64_t>(T), h_cols, nt / 2))
+  if (!encode_slabs(&a_half, a_ptr, v.d, a_rows, v.d, nt / 2)) return cudaErrorInvalidValue;
+  if (h_ptr && !encode_slabs(&h_half, h_ptr, h_cols, static_cast<uint64_t>(T), h_cols, nt / 2))
     return cudaErrorInvalidValue;
   return launch_kv_pair(v.head_dim, nt, *v.tm_Wkv, a_half, h_ptr ? h_half : a_half, gp, v.num_sms,
                         st);
 }
 
-// K/V stage of a recurrent build: every layer in one launch, A = the stacked M_l.
+// K/V stage of a recurrent build: every layer in one launch, A = the stacked M_l (tm_mem_s: its
+// slab map with 128-row boxes).
 template <typename Mark>
 static cudaError_t launch_recurrent_kv(const PlanView& v, const BuildArgs& a, long long T,
-                                       const CUtensorMap& tm_mem, cudaStream_t st, Mark& mark) {
+                                       const CUtensorMap& tm_mem_s, cudaStream_t st, Mark& mark) {
   const int L = v.n_layers, d = v.d;
   GemmParams gp;
   std::memset(&gp, 0, sizeof(gp));
@@ -667,8 +689,8 @@ static cudaError_t launch_recurrent_kv(const PlanView& v, const BuildArgs& a, lo
   for (int i = 0; i < L; ++i) gp.layer_map[i] = v.active[i];
   gp.s = {static_cast<int>(T), L, 2 * v.kv, d / 64, 0, 0, 0, 0, 0, static_cast<int>(T)};
   fill_epi_kv(v, a, T, gp.kv);
-  const cudaError_t err = launch_kv_stage(v, gp, T, a.mem, static_cast<uint64_t>(L) * T, tm_mem,
-                                          nullptr, 0, tm_mem, st);
+  const cudaError_t err = launch_kv_stage(v, gp, T, a.mem, static_cast<uint64_t>(L) * T, tm_mem_s,
+                                          nullptr, 0, tm_mem_s, st);
   mark(4);
   return err;
 }
@@ -684,10 +706,11 @@ static cudaError_t enqueue_recurrent(const PlanView& v, const BuildArgs& a, cuda
   auto mark = [&](int i) {
     if (a.marks) cudaEventRecord(a.marks[i], st);
   };
-  CUtensorMap tm_x0, tm_mem, tm_H;
+  CUtensorMap tm_x0, tm_mem, tm_H, tm_mem_s;
   if (!encode_2d(&tm_x0, a.x0, d, static_cast<uint64_t>(T), d, kBlockM) ||
       !encode_2d(&tm_mem, a.mem, d, static_cast<uint64_t>(L) * T, d, kBlockM) ||
-      !encode_2d(&tm_H, a.H, n1, static_cast<uint64_t>(T), n1, kBlockM))
+      !encode_2d(&tm_H, a.H, n1, static_cast<uint64_t>(T), n1, kBlockM) ||
+      !encode_slabs(&tm_mem_s, a.mem, d, static_cast<uint64_t>(L) * T, d, kBlockM))
     return cudaErrorInvalidValue;
 
   mark(0);
@@ -709,7 +732,7 @@ static cudaError_t enqueue_recurrent(const PlanView& v, const BuildArgs& a, cuda
           a.part, L, T, S, part_ld, 1.0f / d, v.rms_eps, a.rstd);
       err = cudaGetLastError();
       mark(3);
-      return err == cudaSuccess ? launch_recurrent_kv(v, a, T, tm_mem, st, mark) : err;
+      return err == cudaSuccess ? launch_recurrent_kv(v, a, T, tm_mem_s, st, mark) : err;
     }
     if (err != cudaErrorNotSupported) return err;
     err = cudaSuccess;  // no cluster of that size fits: the per-layer launches below
@@ -749,7 +772,7 @@ static cudaError_t enqueue_recurrent(const PlanView& v, const BuildArgs& a, cuda
     err = cudaGetLastError();
   }
   mark(3);
-  return err == cudaSuccess ? launch_recurrent_kv(v, a, T, tm_mem, st, mark) : err;
+  return err == cudaSuccess ? launch_recurrent_kv(v, a, T, tm_mem_s, st, mark) : err;
 }
 
 cudaError_t enqueue_build(const PlanView& v, const BuildArgs& a, cudaStream_t st) {
@@ -763,9 +786,12 @@ cudaError_t enqueue_build(const PlanView& v, const BuildArgs& a, cudaStream_t st
   const long long pad128 = (T + 127) / 128 * 128, pad256 = (T + 255) / 256 * 256;
   const bool rank_pairs = prefer_256(pad256, pad128);
 
-  CUtensorMap tm_x0, tm_H;
+  // 2-D maps for the 1-SM kernel, slab maps (two K slabs per box) for the CTA-pair kernels
+  CUtensorMap tm_x0, tm_H, tm_x0_s, tm_H_s;
   if (!encode_2d(&tm_x0, a.x0, d, static_cast<uint64_t>(T), d, kBlockM) ||
-      !encode_2d(&tm_H, a.H, n1, static_cast<uint64_t>(T), n1, kBlockM))
+      !encode_2d(&tm_H, a.H, n1, static_cast<uint64_t>(T), n1, kBlockM) ||
+      !encode_slabs(&tm_x0_s, a.x0, d, static_cast<uint64_t>(T), d, kBlockM) ||
+      !encode_slabs(&tm_H_s, a.H, n1, static_cast<uint64_t>(T), n1, kBlockM))
     return cudaErrorInvalidValue;
 
   GemmParams gp;
@@ -798,7 +824,7 @@ cudaError_t enqueue_build(const PlanView& v, const BuildArgs& a, cudaStream_t st
     gp.silu = {a.H, static_cast<int>(n1), static_cast<int>(n1), a.c, static_cast<int>(n1)};
     tm_groups(gp.s, bn, T);
     const CUtensorMap& tmD = v.tm_Dst_half[bn == 64 ? 0 : (bn == 128 ? 1 : 2)];
-    if (err == cudaSuccess) err = launch_pair_tm(EPI_SILU, bn, 0, tm_x0, tm_x0, tmD, gp, v.num_sms, st);
+    if (err == cudaSuccess) err = launch_pair_tm(EPI_SILU, bn, 0, tm_x0_s, tm_x0_s, tmD, gp, v.num_sms, st);
     mark(2);
     if (err == cudaSuccess) {
       dim3 grid(static_cast<unsigned>((T + 63) / 64), static_cast<unsigned>(L));
@@ -820,7 +846,7 @@ cudaError_t enqueue_build(const PlanView& v, const BuildArgs& a, cudaStream_t st
     }
     const CUtensorMap& tmD = v.tm_Dst_half[bn == 64 ? 0 : (bn == 128 ? 1 : 2)];
     tm_groups(gp.s, bn, T);
-    if (err == cudaSuccess) err = launch_pair_tm(EPI_SILU, bn, 0, tm_x0, tm_x0, tmD, gp, v.num_sms, st);
+    if (err == cudaSuccess) err = launch_pair_tm(EPI_SILU, bn, 0, tm_x0_s, tm_x0_s, tmD, gp, v.num_sms, st);
   } else {
     const long long m_tiles = pad128 / 128;
     int bn = 64;
@@ -841,7 +867,7 @@ cudaError_t enqueue_build(const PlanView& v, const BuildArgs& a, cudaStream_t st
   gp.norm = {a.H, static_cast<int>(n1), v.r_pad, a.xx, a.rstd, static_cast<int>(T), 1.0f / d,
              v.rms_eps};
   if (err == cudaSuccess) {
-    err = rank_pairs ? launch_pair_tm(EPI_NORM, v.r_pad, 0, tm_x0, tm_H, *v.tm_Bn_half, gp, v.num_sms, st)
+    err = rank_pairs ? launch_pair_tm(EPI_NORM, v.r_pad, 0, tm_x0_s, tm_H_s, *v.tm_Bn_half, gp, v.num_sms, st)
                      : launch_gemm(EPI_NORM, v.r_pad, 0, tm_x0, tm_H, *v.tm_Bn, gp, v.num_sms, st);
   }
   mark(3);
@@ -851,8 +877,8 @@ cudaError_t enqueue_build(const PlanView& v, const BuildArgs& a, cudaStream_t st
   gp.s = {static_cast<int>(T), L, 2 * v.kv, d / 64, v.r_pad / 64, v.r_pad, 0, 0, 0, 0};
   fill_epi_kv(v, a, T, gp.kv);
   if (err == cudaSuccess)
-    err = launch_kv_stage(v, gp, T, a.x0, static_cast<uint64_t>(T), tm_x0, a.H,
-                          static_cast<uint64_t>(n1), tm_H, st);
+    err = launch_kv_stage(v, gp, T, a.x0, static_cast<uint64_t>(T), tm_x0_s, a.H,
+                          static_cast<uint64_t>(n1), tm_H_s, st);
   mark(4);
   return err;
 }
@@ -1094,16 +1120,16 @@ int dv_memory_plan(const dv_config* cfg, const dv_weights* w, void* stream, dv_p
   bool enc = encode_2d(&p->tm_Dst[0], p->Dst, d, dst_rows, dst_ld, 64) &&
              encode_2d(&p->tm_Dst[1], p->Dst, d, dst_rows, dst_ld, 128) &&
              encode_2d(&p->tm_Dst[2], p->Dst, d, dst_rows, dst_ld, 256) &&
-             encode_2d(&p->tm_Dst_half[0], p->Dst, d, dst_rows, dst_ld, 32) &&
-             encode_2d(&p->tm_Dst_half[1], p->Dst, d, dst_rows, dst_ld, 64) &&
-             encode_2d(&p->tm_Dst_half[2], p->Dst, d, dst_rows, dst_ld, 128) &&
-             encode_2d(&p->tm_Wkv, p->Wkv, p->k_total, 1ull * L * 2 * p->kv, p->k_total, 128);
+             encode_slabs(&p->tm_Dst_half[0], p->Dst, d, dst_rows, dst_ld, 32) &&
+             encode_slabs(&p->tm_Dst_half[1], p->Dst, d, dst_rows, dst_ld, 64) &&
+             encode_slabs(&p->tm_Dst_half[2], p->Dst, d, dst_rows, dst_ld, 128) &&
+             encode_slabs(&p->tm_Wkv, p->Wkv, p->k_total, 1ull * L * 2 * p->kv, p->k_total, 128);
   if (enc && rec) {
     enc = encode_2d(&p->tm_Dst_rp, p->Dst, d, 1ull * L * p->r_pad, dst_ld, p->r_pad) &&
           encode_2d(&p->tm_Uup, p->Uup, p->r_pad, 1ull * L * d, p->r_pad, p->resid_bn);
   } else if (enc) {
-    enc = encode_2d(&p->tm_Bn_half, p->Bn, p->k_total, 1ull * L * p->r_pad, p->k_total,
-                    p->r_pad / 2) &&
+    enc = encode_slabs(&p->tm_Bn_half, p->Bn, p->k_total, 1ull * L * p->r_pad, p->k_total,
+                       p->r_pad / 2) &&
           encode_2d(&p->tm_Bn, p->Bn, p->k_total, 1ull * L * p->r_pad, p->k_total, p->r_pad);
   }
   if (!enc) {

@@ -132,8 +132,6 @@ __device__ __forceinline__ bool wait_bounded(uint32_t bar, uint32_t parity, uint
   return mbar_wait(bar, parity, &never, timeout_ns);
 }
 
-__device__ __forceinline__ float silu(float z) { return z / (1.0f + __expf(-z)); }
-
 // Byte offset of 16-byte chunk `c` (8 bf16, c < 8) of row `row` in a 128-byte-swizzled slab.
 __device__ __forceinline__ uint32_t sw128(int row, int c) {
   return static_cast<uint32_t>(row * 128 + ((c ^ (row & 7)) << 4));

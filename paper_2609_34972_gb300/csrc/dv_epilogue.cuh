@@ -23,6 +23,51 @@ __device__ __forceinline__ void store_row16(uint16_t* dst, const uint32_t (&pk)[
   d[1] = make_uint4(pk[4], pk[5], pk[6], pk[7]);
 }
 
+// A warp's 32 x 32 block of an output in global memory: lane i holds row i. Stored through the
+// warp's shared staging (kWarpStageFloats floats) so that each store instruction writes whole
+// row segments (8 lanes x 16 bytes per fp32 row, 4 lanes per bf16 row) instead of 32 scattered
+// 16-byte pieces: one L2 request per 128-byte line, not one per lane.
+constexpr int kWarpStagePitch = 36;                      // floats per staged row (32 + 4 pad)
+constexpr int kWarpStageFloats = 32 * kWarpStagePitch;   // 4608 bytes per warp
+
+// fp32: rows [row0, row0 + rows) of dst (row stride ld floats) get lane-row's 32 values.
+__device__ __forceinline__ void warp_store_f32(float* stage, const uint32_t (&r)[32], float* dst,
+                                               long long ld, int rows) {
+  const int lane = threadIdx.x & 31;
+  float4* srow = reinterpret_cast<float4*>(stage + lane * kWarpStagePitch);
+#pragma unroll
+  for (int q = 0; q < 8; ++q)
+    srow[q] = make_float4(__uint_as_float(r[4 * q]), __uint_as_float(r[4 * q + 1]),
+                          __uint_as_float(r[4 * q + 2]), __uint_as_float(r[4 * q + 3]));
+  __syncwarp();
+#pragma unroll
+  for (int k = 0; k < 8; ++k) {
+    const int row = 4 * k + (lane >> 3), c4 = lane & 7;
+    const float4 v = reinterpret_cast<const float4*>(stage + row * kWarpStagePitch)[c4];
+    if (row < rows) reinterpret_cast<float4*>(dst + row * ld)[c4] = v;
+  }
+  __syncwarp();
+}
+
+// bf16: rows [0, rows) of dst (row stride ld elements) get lane-row's 32 packed values.
+__device__ __forceinline__ void warp_store_bf16(float* stage, const uint32_t (&pk)[16],
+                                                uint16_t* dst, long long ld, int rows) {
+  const int lane = threadIdx.x & 31;
+  uint32_t* st = reinterpret_cast<uint32_t*>(stage);
+  constexpr int kPitch = 20;  // words per staged row (16 + 4 pad)
+  uint4* srow = reinterpret_cast<uint4*>(st + lane * kPitch);
+#pragma unroll
+  for (int q = 0; q < 4; ++q) srow[q] = make_uint4(pk[4 * q], pk[4 * q + 1], pk[4 * q + 2], pk[4 * q + 3]);
+  __syncwarp();
+#pragma unroll
+  for (int k = 0; k < 4; ++k) {
+    const int row = 8 * k + (lane >> 2), c4 = lane & 3;
+    const uint4 v = reinterpret_cast<const uint4*>(st + row * kPitch)[c4];
+    if (row < rows) reinterpret_cast<uint4*>(dst + row * ld)[c4] = v;
+  }
+  __syncwarp();
+}
+
 // sin and cos of the rotary angle pos * theta^(-2j/D_h). The product is kept as an
 // unevaluated sum of two floats (fma residual, inverse frequency split in two floats), then
 // reduced to [-pi, pi] by Cody-Waite subtraction of k * 2pi (2pi split in two floats) before
@@ -38,33 +83,30 @@ __device__ __forceinline__ void rope_sincos(float pos, float fhi, float flo, con
   __sincosf(r, &s, &c);
 }
 
-// H[t, n*BN + c] = bf16(SiLU(z)), SiLU(z) = z / (1 + e^-z)  (phi of Sec. 3.1 Eq. 4); tiles past
+// H[t, n*BN + c] = bf16(SiLU(z)) (phi of Sec. 3.1 Eq. 4); tiles past
 // the down-projection columns store the raw fp32 product into C instead (the launch picks BN
-// dividing n_h, so no tile straddles the two).
+// dividing n_h, so no tile straddles the two). t: this lane's token row; the warp's rows are
+// t - lane .. t - lane + 31, written through the warp's staging `wstage`.
 template <int BN>
-__device__ __forceinline__ void epi_silu(const GemmParams& p, uint32_t tbase, int n, int t) {
-  const bool valid = t < p.s.M;
+__device__ __forceinline__ void epi_silu(const GemmParams& p, uint32_t tbase, int n, int t,
+                                         float* wstage) {
+  const int row0 = t - (threadIdx.x & 31);
+  const int rows = p.s.M - row0;  // valid rows of this warp's block (may be <= 0)
   const int col0 = n * BN;
   if (col0 >= p.silu.n_h) {
-    float* crow = p.silu.C + static_cast<size_t>(valid ? t : 0) * p.silu.ldc + (col0 - p.silu.n_h);
+    float* c0 = p.silu.C + static_cast<size_t>(rows > 0 ? row0 : 0) * p.silu.ldc + (col0 - p.silu.n_h);
 #pragma unroll 1
     for (int c = 0; c < BN / 32; ++c) {
       uint32_t r[32];
       __syncwarp();
       tmem_ld32(tbase + c * 32, r);
       tmem_ld_wait();
-      if (valid) {
-        float4* dst = reinterpret_cast<float4*>(crow + c * 32);
-#pragma unroll
-        for (int q = 0; q < 8; ++q)
-          dst[q] = make_float4(__uint_as_float(r[4 * q]), __uint_as_float(r[4 * q + 1]),
-                               __uint_as_float(r[4 * q + 2]), __uint_as_float(r[4 * q + 3]));
-      }
+      warp_store_f32(wstage, r, c0 + c * 32, p.silu.ldc, rows);
     }
     return;
   }
-  uint16_t* out = p.silu.H + static_cast<size_t>(valid ? t : 0) * p.silu.ldh +
-                  static_cast<size_t>(col0);
+  uint16_t* h0 = p.silu.H + static_cast<size_t>(rows > 0 ? row0 : 0) * p.silu.ldh +
+                 static_cast<size_t>(col0);
 #pragma unroll 1
   for (int c = 0; c < BN / 32; ++c) {
     uint32_t r[32];
@@ -75,9 +117,9 @@ __device__ __forceinline__ void epi_silu(const GemmParams& p, uint32_t tbase, in
 #pragma unroll
     for (int u = 0; u < 16; ++u) {
       const float z0 = __uint_as_float(r[2 * u]), z1 = __uint_as_float(r[2 * u + 1]);
-      pk[u] = pack_bf16x2(z0 / (1.0f + __expf(-z0)), z1 / (1.0f + __expf(-z1)));
+      pk[u] = pack_bf16x2(silu(z0), silu(z1));
     }
-    if (valid) store_row32(out + c * 32, pk);
+    warp_store_bf16(wstage, pk, h0 + c * 32, p.silu.ldh, rows);
   }
 }
 

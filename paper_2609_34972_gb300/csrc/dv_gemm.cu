@@ -38,7 +38,8 @@ struct TileCfg {
   static constexpr int kStagesRaw = kRingBytes / kStageBytes;
   static constexpr int kStages = kStagesRaw > 8 ? 8 : kStagesRaw;
   static constexpr int kTmemCols = 2 * BN;
-  static constexpr int kSmemBytes = kStages * kStageBytes + 1024 + 256;
+  static constexpr int kEpiStageBytes = 4 * kWarpStageFloats * 4;  // one block per epilogue warp
+  static constexpr int kSmemBytes = kStages * kStageBytes + kEpiStageBytes + 1024 + 256;
   static_assert(kStageBytes % 1024 == 0, "stage tiles must stay 1024-byte aligned");
   static_assert(kTmemCols >= 32 && kTmemCols <= 512 && (kTmemCols & (kTmemCols - 1)) == 0,
                 "TMEM allocation must be a power of two in [32, 512]");
@@ -64,7 +65,8 @@ __global__ void __launch_bounds__(kNumThreads, 1)
   const uint32_t raw = smem_addr(smem_raw);
   const uint32_t ring = (raw + 1023u) & ~1023u;
   uint8_t* ring_ptr = smem_raw + (ring - raw);
-  uint64_t* bars = reinterpret_cast<uint64_t*>(ring_ptr + S * C::kStageBytes);
+  float* epi_stage = reinterpret_cast<float*>(ring_ptr + S * C::kStageBytes);
+  uint64_t* bars = reinterpret_cast<uint64_t*>(ring_ptr + S * C::kStageBytes + C::kEpiStageBytes);
   const uint32_t bar0 = smem_addr(bars);
   auto full_bar = [&](int s) { return bar0 + 8u * s; };
   auto empty_bar = [&](int s) { return bar0 + 8u * (S + s); };
@@ -201,13 +203,14 @@ __global__ void __launch_bounds__(kNumThreads, 1)
       const int rest = tile / m_tiles;
       const int n = rest % n_tiles;
       const int l = p.s.layer0 + rest / n_tiles;
-      if (!mbar_wait(tfull_bar(acc), acc_phase, abort_flag, tmo)) break;
+      // the warp leaves together (its lanes meet in __syncwarp and the TMEM loads below)
+      if (!__all_sync(0xFFFFFFFFu, mbar_wait(tfull_bar(acc), acc_phase, abort_flag, tmo))) break;
       tc_fence_after();
       const uint32_t tbase =
           tmem_base + (static_cast<uint32_t>(q * 32) << 16) + static_cast<uint32_t>(acc * BN);
       const int t = m * kBlockM + row;
       if constexpr (EPI == EPI_SILU) {
-        epi_silu<BN>(p, tbase, n, t);
+        epi_silu<BN>(p, tbase, n, t, epi_stage + q * kWarpStageFloats);
       } else if constexpr (EPI == EPI_NORM) {
         epi_norm<BN>(p, tbase, l, t);
       } else {

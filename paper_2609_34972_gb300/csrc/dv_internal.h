@@ -41,6 +41,37 @@ struct GemmShape {
   int a0_rows_per_layer;  // 0: one A0 for every layer; else A0 rows of layer l start at l * it
 };
 
+// The 2-SM kernels move two K slabs per pipeline step: one 3-D TMA box per operand and step
+// (a TMA instruction has a fixed cost that 16 KB boxes do not amortise). A step stays inside
+// one segment of the K schedule (A0, then A1); the last step of a segment with an odd slab
+// count uses its first slab only (the box's second slab is zero fill or unused data).
+constexpr int kSlabsPerStep = 2;
+
+struct KStep {
+  int seg;   // 0: A0 slabs (x0 or M_l), 1: A1 slabs (h_l)
+  int slab;  // first slab of the step within its segment
+  int n;     // slabs of the step that the MMA uses: 1 or 2
+};
+
+__host__ __device__ inline int k_steps(int k0_slabs, int k1_slabs) {
+  return (k0_slabs + 1) / 2 + (k1_slabs + 1) / 2;
+}
+
+__host__ __device__ inline KStep k_step(int j, int k0_slabs, int k1_slabs) {
+  const int s0 = (k0_slabs + 1) / 2;
+  KStep r;
+  if (j < s0) {
+    r.seg = 0;
+    r.slab = 2 * j;
+    r.n = k0_slabs - 2 * j < 2 ? k0_slabs - 2 * j : 2;
+  } else {
+    r.seg = 1;
+    r.slab = 2 * (j - s0);
+    r.n = k1_slabs - r.slab < 2 ? k1_slabs - r.slab : 2;
+  }
+  return r;
+}
+
 // Columns [0, n_h) of the product are down-projections: H = bf16(SiLU(acc)). Columns from n_h
 // on (x0 (2 U_l)^T when the statistic of M_l is formed outside a GEMM) go to C as fp32.
 struct EpiSilu {
@@ -119,15 +150,16 @@ cudaError_t launch_gemm(int epi, int block_n, int head_dim, const CUtensorMap& a
 // Shared-memory bytes one CTA of that GEMM asks for (for validation and reporting).
 int gemm_smem_bytes(int block_n);
 
-// K/V projection + RoPE + cache store on CTA pairs (2-SM UMMA). w: Wkv with 128-row boxes;
-// x / h: x0 and H with boxes of nt/2 token rows. nt from kv_pair_tile_n.
+// K/V projection + RoPE + cache store on CTA pairs (2-SM UMMA). All maps are slab maps (two K
+// slabs per box): w: Wkv with 128-row boxes; x / h: x0 and H with boxes of nt/2 token rows. nt
+// from kv_pair_tile_n.
 cudaError_t launch_kv_pair(int head_dim, int nt, const CUtensorMap& w, const CUtensorMap& x,
                            const CUtensorMap& h, const GemmParams& p, int num_sms,
                            cudaStream_t stream);
 
 // 2-SM GEMM with 256-token M blocks (tokens as M): EPI_SILU / EPI_NORM with block_n 64/128/256
 // (b: weights with boxes of block_n / 2 rows), EPI_KV with block_n 256 (b: Wkv, 128-row boxes).
-// a0 / a1: x0 and H with 128-row boxes.
+// a0 / a1: x0 and H with 128-row boxes. All maps are slab maps (two K slabs per box).
 cudaError_t launch_pair_tm(int epi, int block_n, int head_dim, const CUtensorMap& a0,
                            const CUtensorMap& a1, const CUtensorMap& b, const GemmParams& p,
                            int num_sms, cudaStream_t stream);
@@ -187,10 +219,10 @@ struct PlanView {
   const CUtensorMap* tm_Dst;       // three maps: boxes of 64, 128, 256 rows; embedding adapter:
                                    // rows [0, L r_pad) D, rows [L r_pad, 2 L r_pad) 2 U^T
   const float* Gf;                 // embedding adapter: G_l = U_l^T U_l, fp32 [L][r_pad][r_pad]
-  const CUtensorMap* tm_Dst_half;  // three maps: boxes of 32, 64, 128 rows (CTA-pair halves)
+  const CUtensorMap* tm_Dst_half;  // three slab maps: boxes of 32, 64, 128 rows (pair halves)
   const CUtensorMap* tm_Bn;        // boxes of r_pad rows
-  const CUtensorMap* tm_Bn_half;   // boxes of r_pad / 2 rows
-  const CUtensorMap* tm_Wkv;       // boxes of 128 rows
+  const CUtensorMap* tm_Bn_half;   // slab map, boxes of r_pad / 2 rows
+  const CUtensorMap* tm_Wkv;       // slab map, boxes of 128 rows
   const CUtensorMap* tm_Dst_rp;    // recurrent: boxes of r_pad rows (one layer's D)
   const CUtensorMap* tm_Uup;       // recurrent: [L*d][r_pad], boxes of resid_bn rows
   const uint16_t* Uup;             // recurrent: U_l as [L*d][r_pad]

@@ -10,9 +10,11 @@
 // NT/2 token rows), which halves the shared-memory traffic per MMA against a 1-SM tile.
 //
 // CTA roles (192 threads, one CTA per SM, both CTAs of a pair alike):
-//   warp 0      TMA producer for this CTA's halves; completion is counted on the leader's
-//               full barrier (cta_group::2 TMA), whose single expect_tx arrival (leader)
-//               announces the bytes of both CTAs
+//   warp 0      TMA producer for this CTA's halves, two K slabs per pipeline step (one 3-D
+//               box per operand: a TMA instruction has a fixed cost, and two-slab boxes let one
+//               SM's copies keep pace with the MMA); completion is counted on the leader's full
+//               barrier (cta_group::2 TMA), whose single expect_tx arrival (leader) announces
+//               the bytes of both CTAs
 //   warp 1      TMEM owner (cta_group::2 alloc in both CTAs); in the leader one lane issues the
 //               256 x NT x 16 MMAs and multicasts its commits to both CTAs
 //   warps 2-5   epilogue over this CTA's 128 weight rows: TMEM -> registers -> shared staging
@@ -37,8 +39,10 @@ constexpr int kStagePitch = 132;    // floats per staged token row: 128 weight r
 template <int NT>
 struct PairCfg {
   static constexpr int kHalfN = NT / 2;
-  static constexpr int kABytes = 128 * kBlockK * 2;
-  static constexpr int kBBytes = kHalfN * kBlockK * 2;
+  static constexpr int kASlab = 128 * kBlockK * 2;     // one K slab of this CTA's weight rows
+  static constexpr int kBSlab = kHalfN * kBlockK * 2;  // one K slab of its token rows
+  static constexpr int kABytes = kSlabsPerStep * kASlab;
+  static constexpr int kBBytes = kSlabsPerStep * kBSlab;
   static constexpr int kStageBytes = kABytes + kBBytes;
   static constexpr int kStagingBytes = 32 * kStagePitch * 4;
   static constexpr int kRingBudget = kSmemLimit - kStagingBytes - 1024 - 512;
@@ -47,7 +51,8 @@ struct PairCfg {
   static constexpr int kSmemBytes = kStages * kStageBytes + kStagingBytes + 1024 + 512;
   static constexpr int kTmemCols = 512;
   static_assert(NT % 64 == 0 && NT >= 64 && NT <= 256, "N tile");
-  static_assert(kStageBytes % 1024 == 0, "stage tiles must stay 1024-byte aligned");
+  static_assert(kASlab % 1024 == 0 && kBSlab % 1024 == 0, "slab tiles must stay 1024-byte aligned");
+  static_assert(kStages >= 2, "pipeline depth");
   static_assert(2 * NT <= kTmemCols, "two accumulators must fit in TMEM");
   static_assert(kSmemBytes <= kSmemLimit, "shared memory");
 };
@@ -112,7 +117,8 @@ __global__ void __launch_bounds__(kPairThreads, 1)
   const int tok_tiles = (p.s.M + NT - 1) / NT;
   const int groups = p.kv.kv / 128;
   const int num_tiles = tok_tiles * groups * p.s.n_layers;
-  const int k_slabs = p.s.k0_slabs + p.s.k1_slabs;
+  const int k0 = p.s.k0_slabs, k1 = p.s.k1_slabs;
+  const int n_steps = k_steps(k0, k1);
   const int pair = static_cast<int>(cluster_id_x());
   const int num_pairs = static_cast<int>(num_clusters_x());
 
@@ -130,20 +136,22 @@ __global__ void __launch_bounds__(kPairThreads, 1)
         const int wrow = l * p.s.n_per_layer + g * 256 + static_cast<int>(rank) * 128;
         const int trow = nt * NT + static_cast<int>(rank) * C::kHalfN;
         const int xrow = l * p.s.a0_rows_per_layer + trow;
-        for (int ks = 0; ks < k_slabs; ++ks) {
+        for (int j = 0; j < n_steps; ++j) {
+          const KStep ks = k_step(j, k0, k1);
           if (!mbar_wait(empty_bar(stage), phase ^ 1u, abort_flag, tmo)) break;
           const uint32_t a_dst = ring + stage * C::kStageBytes;
           const uint32_t b_dst = a_dst + C::kABytes;
           const uint32_t fb = leader_full0 + 8u * stage;
-          // Only the leader arrives (local, CTA scope) and announces both CTAs' bytes; the
-          // peer's copies may complete on the barrier first (the transaction count is signed).
+          // Only the leader arrives (local, CTA scope) and announces both CTAs' bytes (whole
+          // boxes, zero fill included); the peer's copies may complete on the barrier first
+          // (the transaction count is signed).
           if (rank == 0) mbar_arrive_expect_tx(full_bar(stage), 2 * C::kStageBytes);
-          tma_load_2d_pair(a_dst, &tmW, fb, ks * kBlockK, wrow);
-          if (ks < p.s.k0_slabs) {
-            tma_load_2d_pair(b_dst, &tmX, fb, ks * kBlockK, xrow);
+          tma_load_3d_pair(a_dst, &tmW, fb, wrow, ks.seg == 0 ? ks.slab : k0 + ks.slab);
+          if (ks.seg == 0) {
+            tma_load_3d_pair(b_dst, &tmX, fb, xrow, ks.slab);
           } else {
-            tma_load_2d_pair(b_dst, &tmH, fb,
-                             l * p.s.a1_cols_per_layer + (ks - p.s.k0_slabs) * kBlockK, trow);
+            tma_load_3d_pair(b_dst, &tmH, fb, trow,
+                             l * (p.s.a1_cols_per_layer / kBlockK) + ks.slab);
           }
           if (++stage == S) {
             stage = 0;
@@ -164,7 +172,8 @@ __global__ void __launch_bounds__(kPairThreads, 1)
         tc_fence_after();
         const uint32_t d_tmem = tmem_base + static_cast<uint32_t>(acc * NT);
         bool ok = true;
-        for (int ks = 0; ks < k_slabs; ++ks) {
+        for (int j = 0; j < n_steps; ++j) {
+          const int n_used = k_step(j, k0, k1).n;
           if (!mbar_wait(full_bar(stage), phase, abort_flag, tmo)) {
             ok = false;
             break;
@@ -173,9 +182,15 @@ __global__ void __launch_bounds__(kPairThreads, 1)
           const uint32_t a_s = ring + stage * C::kStageBytes;
           const uint32_t b_s = a_s + C::kABytes;
 #pragma unroll
-          for (int k = 0; k < kBlockK / 16; ++k) {
-            umma_bf16_pair(d_tmem, sdesc_kmajor_sw128(a_s + 32u * k),
-                           sdesc_kmajor_sw128(b_s + 32u * k), idesc, (ks | k) != 0 ? 1u : 0u);
+          for (int sl = 0; sl < kSlabsPerStep; ++sl) {
+            if (sl < n_used) {
+#pragma unroll
+              for (int k = 0; k < kBlockK / 16; ++k) {
+                umma_bf16_pair(d_tmem, sdesc_kmajor_sw128(a_s + sl * C::kASlab + 32u * k),
+                               sdesc_kmajor_sw128(b_s + sl * C::kBSlab + 32u * k), idesc,
+                               (j | sl | k) != 0 ? 1u : 0u);
+              }
+            }
           }
           issued_any = true;
           umma_commit_pair(empty_bar(stage), 0x3);

@@ -10,9 +10,10 @@
 // tensor throughput. Each epilogue thread owns one token row of its CTA's accumulator, so RoPE
 // pairs and head rows are in registers and go straight to 16-byte stores.
 //
-// Roles as in the other kernels: warp 0 lane 0 loads (both CTAs, completion counted on the
-// leader's full barrier whose single expect_tx covers both CTAs), warp 1 owns TMEM and, in the
-// leader, issues the MMAs with multicast commits, warps 2-5 drain the accumulator.
+// Roles as in the other kernels: warp 0 lane 0 loads (both CTAs, two K slabs per pipeline
+// step as one 3-D box per operand, completion counted on the leader's full barrier whose single
+// expect_tx covers both CTAs), warp 1 owns TMEM and, in the leader, issues the MMAs with
+// multicast commits, warps 2-5 drain the accumulator.
 //
 // Tile order: the tiles form a grid of token blocks (m) x weight tiles (w = layer * n_tiles +
 // n). It is walked in super-blocks of group_m token blocks x group_w weight tiles (token block
@@ -30,15 +31,19 @@ constexpr int kTmSmemLimit = 232448;
 
 template <int BN>
 struct TmCfg {
-  static constexpr int kABytes = 128 * kBlockK * 2;        // 128 token rows
-  static constexpr int kBBytes = (BN / 2) * kBlockK * 2;   // BN / 2 weight rows
+  static constexpr int kASlab = 128 * kBlockK * 2;         // one K slab of 128 token rows
+  static constexpr int kBSlab = (BN / 2) * kBlockK * 2;    // one K slab of BN / 2 weight rows
+  static constexpr int kABytes = kSlabsPerStep * kASlab;
+  static constexpr int kBBytes = kSlabsPerStep * kBSlab;
   static constexpr int kStageBytes = kABytes + kBBytes;
-  static constexpr int kStagesRaw = (kTmSmemLimit - 1024 - 512) / kStageBytes;
+  static constexpr int kEpiStageBytes = 4 * kWarpStageFloats * 4;  // one block per epilogue warp
+  static constexpr int kStagesRaw = (kTmSmemLimit - kEpiStageBytes - 1024 - 512) / kStageBytes;
   static constexpr int kStages = kStagesRaw > 8 ? 8 : kStagesRaw;
-  static constexpr int kSmemBytes = kStages * kStageBytes + 1024 + 512;
+  static constexpr int kSmemBytes = kStages * kStageBytes + kEpiStageBytes + 1024 + 512;
   static constexpr int kTmemCols = 2 * BN < 32 ? 32 : 2 * BN;
   static_assert(BN == 64 || BN == 128 || BN == 256, "N tile");
-  static_assert(kStageBytes % 1024 == 0, "stage tiles must stay 1024-byte aligned");
+  static_assert(kASlab % 1024 == 0 && kBSlab % 1024 == 0, "slab tiles must stay 1024-byte aligned");
+  static_assert(kStages >= 2, "pipeline depth");
   static_assert((kTmemCols & (kTmemCols - 1)) == 0 && kTmemCols <= 512, "TMEM allocation");
 };
 
@@ -65,7 +70,8 @@ __global__ void __launch_bounds__(kTmThreads, 1)
   const uint32_t raw = smem_addr(smem_raw);
   const uint32_t ring = (raw + 1023u) & ~1023u;
   uint8_t* ring_ptr = smem_raw + (ring - raw);
-  uint64_t* bars = reinterpret_cast<uint64_t*>(ring_ptr + S * C::kStageBytes);
+  float* epi_stage = reinterpret_cast<float*>(ring_ptr + S * C::kStageBytes);
+  uint64_t* bars = reinterpret_cast<uint64_t*>(ring_ptr + S * C::kStageBytes + C::kEpiStageBytes);
   const uint32_t bar0 = smem_addr(bars);
   auto full_bar = [&](int s) { return bar0 + 8u * s; };                   // leader
   auto empty_bar = [&](int s) { return bar0 + 8u * (S + s); };            // both
@@ -112,7 +118,8 @@ __global__ void __launch_bounds__(kTmThreads, 1)
   const int num_tiles = m_tiles * w_tiles;
   const int gm = p.s.group_m > 0 ? min(p.s.group_m, m_tiles) : m_tiles;
   const int gw = p.s.group_w > 0 ? min(p.s.group_w, w_tiles) : 1;
-  const int k_slabs = p.s.k0_slabs + p.s.k1_slabs;
+  const int k0 = p.s.k0_slabs, k1 = p.s.k1_slabs;
+  const int n_steps = k_steps(k0, k1);
   const int pair = static_cast<int>(cluster_id_x());
   const int num_pairs = static_cast<int>(num_clusters_x());
 
@@ -130,19 +137,20 @@ __global__ void __launch_bounds__(kTmThreads, 1)
         const int arow = m * 256 + static_cast<int>(rank) * 128;
         const int a0row = l * p.s.a0_rows_per_layer + arow;
         const int brow = l * p.s.n_per_layer + n * BN + static_cast<int>(rank) * (BN / 2);
-        for (int ks = 0; ks < k_slabs; ++ks) {
+        for (int j = 0; j < n_steps; ++j) {
+          const KStep ks = k_step(j, k0, k1);
           if (!mbar_wait(empty_bar(stage), phase ^ 1u, abort_flag, tmo)) break;
           const uint32_t a_dst = ring + stage * C::kStageBytes;
           const uint32_t b_dst = a_dst + C::kABytes;
           const uint32_t fb = leader_full0 + 8u * stage;
           if (rank == 0) mbar_arrive_expect_tx(full_bar(stage), 2 * C::kStageBytes);
-          if (ks < p.s.k0_slabs) {
-            tma_load_2d_pair(a_dst, &tmA0, fb, ks * kBlockK, a0row);
+          if (ks.seg == 0) {
+            tma_load_3d_pair(a_dst, &tmA0, fb, a0row, ks.slab);
           } else {
-            tma_load_2d_pair(a_dst, &tmA1, fb,
-                             l * p.s.a1_cols_per_layer + (ks - p.s.k0_slabs) * kBlockK, arow);
+            tma_load_3d_pair(a_dst, &tmA1, fb, arow,
+                             l * (p.s.a1_cols_per_layer / kBlockK) + ks.slab);
           }
-          tma_load_2d_pair(b_dst, &tmB, fb, ks * kBlockK, brow);
+          tma_load_3d_pair(b_dst, &tmB, fb, brow, ks.seg == 0 ? ks.slab : k0 + ks.slab);
           if (++stage == S) {
             stage = 0;
             phase ^= 1u;
@@ -162,7 +170,8 @@ __global__ void __launch_bounds__(kTmThreads, 1)
         tc_fence_after();
         const uint32_t d_tmem = tmem_base + static_cast<uint32_t>(acc * BN);
         bool ok = true;
-        for (int ks = 0; ks < k_slabs; ++ks) {
+        for (int j = 0; j < n_steps; ++j) {
+          const int n_used = k_step(j, k0, k1).n;
           if (!mbar_wait(full_bar(stage), phase, abort_flag, tmo)) {
             ok = false;
             break;
@@ -171,9 +180,15 @@ __global__ void __launch_bounds__(kTmThreads, 1)
           const uint32_t a_s = ring + stage * C::kStageBytes;
           const uint32_t b_s = a_s + C::kABytes;
 #pragma unroll
-          for (int k = 0; k < kBlockK / 16; ++k) {
-            umma_bf16_pair(d_tmem, sdesc_kmajor_sw128(a_s + 32u * k),
-                           sdesc_kmajor_sw128(b_s + 32u * k), idesc, (ks | k) != 0 ? 1u : 0u);
+          for (int sl = 0; sl < kSlabsPerStep; ++sl) {
+            if (sl < n_used) {
+#pragma unroll
+              for (int k = 0; k < kBlockK / 16; ++k) {
+                umma_bf16_pair(d_tmem, sdesc_kmajor_sw128(a_s + sl * C::kASlab + 32u * k),
+                               sdesc_kmajor_sw128(b_s + sl * C::kBSlab + 32u * k), idesc,
+                               (j | sl | k) != 0 ? 1u : 0u);
+              }
+            }
           }
           issued_any = true;
           umma_commit_pair(empty_bar(stage), 0x3);
@@ -216,7 +231,7 @@ __global__ void __launch_bounds__(kTmThreads, 1)
           tmem_base + (static_cast<uint32_t>(q * 32) << 16) + static_cast<uint32_t>(acc * BN);
       const int t = m * 256 + static_cast<int>(rank) * 128 + q * 32 + lane;
       if constexpr (EPI == EPI_SILU) {
-        epi_silu<BN>(p, tbase, n, t);
+        epi_silu<BN>(p, tbase, n, t, epi_stage + q * kWarpStageFloats);
       } else if constexpr (EPI == EPI_NORM) {
         epi_norm<BN>(p, tbase, l, t);
       } else {

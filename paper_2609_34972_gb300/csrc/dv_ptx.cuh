@@ -252,6 +252,18 @@ __device__ __forceinline__ void tma_load_2d_pair(uint32_t dst, const CUtensorMap
       : "memory");
 }
 
+// 3-D form of tma_load_2d_pair, for tensor maps that view a [rows][cols] matrix as
+// {64 columns, rows, cols / 64 slabs}: one box brings several consecutive K slabs of a row
+// block, each slab a 128-byte-swizzled [rows][64] tile, the slabs one after another.
+__device__ __forceinline__ void tma_load_3d_pair(uint32_t dst, const CUtensorMap* map,
+                                                 uint32_t cbar, int row, int slab) {
+  asm volatile(
+      "cp.async.bulk.tensor.3d.cta_group::2.shared::cluster.global.mbarrier::complete_tx::bytes"
+      " [%0], [%1, {%3, %4, %5}], [%2];" ::"r"(dst),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(cbar), "r"(0), "r"(row), "r"(slab)
+      : "memory");
+}
+
 // Both CTAs' warps call these together (one warp in each CTA of the pair).
 __device__ __forceinline__ void tmem_alloc_pair(uint32_t slot, uint32_t ncols) {
   asm volatile("tcgen05.alloc.cta_group::2.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(slot),
@@ -311,6 +323,16 @@ __device__ __forceinline__ bool named_barrier_and(uint32_t id, uint32_t nthreads
 // ------------------------------------------------------------------------------ misc
 
 __device__ __forceinline__ float bf16_bits_to_float(uint32_t b) { return __uint_as_float(b << 16); }
+
+// SiLU(z) = z / (1 + e^-z), the adapter's activation (phi of Sec. 3.1 Eq. 4). The quotient uses
+// the fast division (2 ulp; its result is rounded to bf16 next). The IEEE division's slow path
+// was taken for every zero numerator (the zero-filled rows of a ragged token block) and made
+// those rows several times slower than the others. e^-z is capped at e^80 to keep the divisor in
+// the fast division's range; below z = -80 the result (|SiLU| < 1e-33) changes only in those
+// negligible digits.
+__device__ __forceinline__ float silu(float z) {
+  return __fdividef(z, 1.0f + __expf(fminf(-z, 80.0f)));
+}
 
 // Round-to-nearest-even float -> bf16 for two values, packed low/high.
 __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {

@@ -62,8 +62,6 @@ __device__ __forceinline__ bool wait_bounded(uint32_t bar, uint32_t parity, uint
   return mbar_wait(bar, parity, &never, timeout_ns);
 }
 
-__device__ __forceinline__ float silu(float z) { return z / (1.0f + __expf(-z)); }
-
 template <int RP>
 __global__ void __launch_bounds__(kDownThreads, 1)
     dv_down_split_kernel(const __grid_constant__ CUtensorMap tmA,
