@@ -68,6 +68,26 @@ __device__ __forceinline__ void warp_store_bf16(float* stage, const uint32_t (&p
   __syncwarp();
 }
 
+// In-register transpose of a warp's 32 x 32 block: on entry lane i holds row i (r[j] = M[i][j]),
+// on exit lane i holds column i (r[j] = M[j][i]). Five butterfly rounds: in the round of bit b,
+// registers j and j + b (j without bit b) of lanes i and i ^ b swap the two off-diagonal
+// b x b sub-blocks, one shuffle per register pair.
+__device__ __forceinline__ void warp_transpose32(uint32_t (&r)[32]) {
+  const int lane = threadIdx.x & 31;
+#pragma unroll
+  for (int b = 16; b >= 1; b >>= 1) {
+    const bool upper = (lane & b) != 0;
+#pragma unroll
+    for (int j = 0; j < 32; ++j) {
+      if (j & b) continue;
+      const uint32_t send = upper ? r[j] : r[j + b];
+      const uint32_t recv = __shfl_xor_sync(0xFFFFFFFFu, send, b);
+      if (upper) r[j] = recv;
+      else r[j + b] = recv;
+    }
+  }
+}
+
 // sin and cos of the rotary angle pos * theta^(-2j/D_h). The product is kept as an
 // unevaluated sum of two floats (fma residual, inverse frequency split in two floats), then
 // reduced to [-pi, pi] by Cody-Waite subtraction of k * 2pi (2pi split in two floats) before

@@ -17,12 +17,13 @@
 //               the bytes of both CTAs
 //   warp 1      TMEM owner (cta_group::2 alloc in both CTAs); in the leader one lane issues the
 //               256 x NT x 16 MMAs and multicasts its commits to both CTAs
-//   warps 2-5   epilogue over this CTA's 128 weight rows: TMEM -> registers -> shared staging
-//               [32 tokens][128 rows]; then warp q reads rows 32q .. 32q + 31 of the token of
-//               each lane (16-byte loads, conflict-free with a 132-float row pitch) and writes
-//               16 complete RoPE pairs of K (the Wkv K rows are permuted so that partners are 16
-//               rows apart) or 32 channels of V, as 32-byte runs. (A register transpose by
-//               xor-shuffles measured slower: shuffles use the same crossbar bandwidth.)
+//   warps 2-5   epilogue over this CTA's 128 weight rows: TMEM -> registers (lane = weight
+//               row, 32 tokens), an in-register 32 x 32 transpose by xor-shuffles (lane = token,
+//               the warp's 32 weight rows), then 16 complete RoPE pairs of K (the Wkv K rows are
+//               permuted so that partners are 16 rows apart) or 32 channels of V per lane, as
+//               32-byte runs. The transpose needs no shared memory, which leaves room for a
+//               fourth two-slab pipeline step (the weights stream from HBM and need the depth);
+//               only the per-head K norm exchanges one float per warp and token.
 // Pair tiles run in (layer, group, token block) order, token block fastest, so the pairs
 // running together share each weight tile through L2.
 #include "dv_epilogue.cuh"
@@ -34,7 +35,6 @@ namespace dv {
 constexpr int kPairThreads = 192;
 constexpr int kEpiPairThreads = 128;
 constexpr int kSmemLimit = 232448;  // largest dynamic shared memory of one CTA on sm_103
-constexpr int kStagePitch = 132;    // floats per staged token row: 128 weight rows + 4 pad
 
 template <int NT>
 struct PairCfg {
@@ -44,7 +44,7 @@ struct PairCfg {
   static constexpr int kABytes = kSlabsPerStep * kASlab;
   static constexpr int kBBytes = kSlabsPerStep * kBSlab;
   static constexpr int kStageBytes = kABytes + kBBytes;
-  static constexpr int kStagingBytes = 32 * kStagePitch * 4;
+  static constexpr int kStagingBytes = 2 * 32 * 4 * 4;  // K-norm partial sums [2][token][warp]
   static constexpr int kRingBudget = kSmemLimit - kStagingBytes - 1024 - 512;
   static constexpr int kStagesRaw = kRingBudget / kStageBytes;
   static constexpr int kStages = kStagesRaw > 8 ? 8 : kStagesRaw;
@@ -238,27 +238,16 @@ __global__ void __launch_bounds__(kPairThreads, 1)
         __syncwarp();
         tmem_ld32(tbase + c * 32, r);  // lane i: weight row 32q + i, 32 tokens
         tmem_ld_wait();
-        float* col = staging + q * 32 + lane;
-#pragma unroll
-        for (int u = 0; u < 32; ++u) col[u * kStagePitch] = __uint_as_float(r[u]);
-        named_barrier(1, kEpiPairThreads);
-        const float4* src = reinterpret_cast<const float4*>(staging + lane * kStagePitch + q * 32);
-#pragma unroll
-        for (int v = 0; v < 8; ++v) {  // lane: token 32c + lane, weight rows 32q .. 32q + 31
-          const float4 w = src[v];
-          r[4 * v] = __float_as_uint(w.x);
-          r[4 * v + 1] = __float_as_uint(w.y);
-          r[4 * v + 2] = __float_as_uint(w.z);
-          r[4 * v + 3] = __float_as_uint(w.w);
-        }
+        warp_transpose32(r);           // lane i: token 32c + i, weight rows 32q .. 32q + 31
         const KvToken tk = kv_token(p, l, nt * NT + c * 32 + lane);
         if (rank == 0) {
           float kinv = 1.0f;
           if (p.kv.kg) {
             // Per-head K norm: a head spans warps (4 blocks of 32 channels for HD = 128,
-            // 2 for HD = 64). Each warp leaves its block's sum of squares in the unused pad
-            // columns of the token's staging row; the head's blocks are summed in block order.
-            float* pad = staging + lane * kStagePitch + 128;
+            // 2 for HD = 64). Each warp leaves its block's sum of squares for the token of each
+            // lane; the head's blocks are summed in block order. Two buffers by chunk parity:
+            // a warp rewrites one only after every warp has passed the next chunk's barrier.
+            float* pad = staging + ((c & 1) * 32 + lane) * 4;
             pad[q] = kv_k16_sumsq<HD>(p, tk, l, g, q, r);
             named_barrier(1, kEpiPairThreads);
             const float ss = HD == 128 ? ((pad[0] + pad[1]) + pad[2]) + pad[3]
@@ -269,7 +258,6 @@ __global__ void __launch_bounds__(kPairThreads, 1)
         } else {
           kv_store_v32<HD>(p, tk, l, g, q, r);
         }
-        named_barrier(1, kEpiPairThreads);
       }
       tc_fence_before();
       __syncwarp();
