@@ -344,9 +344,16 @@ def run_dv(args):
     # ---- roofline of the dominant kernel (K/V projection + RoPE + store) and of the step
     kv_ms = stage_ms[3] / max(n_timed, 1)
     kv_flops = 4.0 * work.d * work.kv * work.tokens * work.n_layers
-    peak_tf = peaks["bf16_tflops"]
+    # The K/V kernel is timed inside a run of back-to-back builds. Once that run lasts long
+    # enough for the power cap to set the clock (about half a second), its peak is the
+    # sustained cuBLAS rate (a seconds-long loop under the same cap); a short run is compared
+    # with the burst rate.
+    sustained = ms_total >= 500.0
+    peak_tf = peaks["bf16_tflops_sustained"] if sustained else peaks["bf16_tflops"]
+    peak_name = "bf16_tflops_sustained" if sustained else "bf16_tflops (burst)"
     achieved_tf = kv_flops / (kv_ms * 1e-3) / 1e12
-    t_roof_ms = max(work.flops() / (peak_tf * 1e12), work.min_bytes() / (peaks["hbm_gbs"] * 1e9)) * 1e3
+    t_roof_ms = max(work.flops() / (peaks["bf16_tflops"] * 1e12),
+                    work.min_bytes() / (peaks["hbm_gbs"] * 1e9)) * 1e3
     traffic = profiled_traffic(work.name)
 
     cpu = None
@@ -375,7 +382,10 @@ def run_dv(args):
             "roofline": {"bound": "tensor", "achieved": achieved_tf, "peak": peak_tf,
                          "unit": "TFLOP/s", "frac": achieved_tf / peak_tf, "traffic": traffic,
                          "kernel": dv.kv_kernel(plan, cfg.tokens) + ": K/V projection + RoPE + cache store",
-                         "peak_source": f"bf16_tflops (burst) of {peak_src}",
+                         "peak_source": f"{peak_name} of {peak_src}; timed region {ms_total:.0f} ms of "
+                                        f"back-to-back builds",
+                         "frac_burst": achieved_tf / peaks["bf16_tflops"],
+                         "frac_sustained": achieved_tf / peaks["bf16_tflops_sustained"],
                          "flops_per_launch": kv_flops, "ms_per_launch": kv_ms},
             "roofline_step": {"t_roof_ms": t_roof_ms, "frac": t_roof_ms / ms_step,
                               "frac_sustained": max(work.flops() / (peaks["bf16_tflops_sustained"] * 1e12),

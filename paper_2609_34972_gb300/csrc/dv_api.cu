@@ -3,7 +3,9 @@
 //
 // Plan-time repacking (once per weight set). With r_pad = r rounded up to 64:
 //   Dst  [L*r_pad][d]         stacked down-projections, zero rows past r
-//   Bn   [L*r_pad][d+r_pad]   row n of layer l: [2 U_l[n,:] | G_l[n,:]], G_l = U_l U_l^T
+//   Bn   [G*256][d+lpt*r_pad]  the statistic's B operand, lpt layers per 256-row group (norm_group):
+//                             row j*rn + n of group g (layer l = g*lpt + j): [2 U_l[n,:] | 0 ..
+//                             G_l[n,:] at columns d + j*r_pad .. | 0], G_l = U_l U_l^T
 //   Wkv  [L*2kv][d+r_pad]     per layer, per group of 128 channels: the 128 K rows (permuted so
 //                             that RoPE partners are 16 rows apart, see wkv_row), then the 128
 //                             V rows of the same channels, each
@@ -31,6 +33,7 @@ struct dv_plan {
   int device = 0;
   int num_sms = 0;
   int r_pad = 0, kv = 0, k_total = 0, max_tokens = 0;
+  int bn_lpt = 0, bn_rn = 0, bn_groups = 0, bn_k = 0;  // Bn layout (norm_group)
   uint16_t* Dst = nullptr;
   uint16_t* Bn = nullptr;
   uint16_t* Wkv = nullptr;
@@ -44,8 +47,8 @@ struct dv_plan {
   int* status = nullptr;
   CUtensorMap tm_Dst[3];       // boxes of 64, 128, 256 rows
   CUtensorMap tm_Dst_half[3];  // slab maps, boxes of 32, 64, 128 rows (halves for CTA pairs)
-  CUtensorMap tm_Bn;           // boxes of r_pad rows
-  CUtensorMap tm_Bn_half;      // slab map, boxes of r_pad / 2 rows
+  CUtensorMap tm_Bn;           // boxes of 256 rows (one layer group)
+  CUtensorMap tm_Bn_half;      // slab map, boxes of 128 rows (CTA-pair halves)
   CUtensorMap tm_Wkv;          // slab map, boxes of 128 rows
   CUtensorMap tm_Dst_rp, tm_Uup;  // recurrent adapter
   int resid_bn = 0;
@@ -166,20 +169,22 @@ __global__ void k_pack_down(const uint16_t* __restrict__ D, uint16_t* __restrict
   }
 }
 
-// Bn[i*r_pad + n][j] = 2 U[src[i]][j][n] (j < d, n < r), zero for padded rows. The G block is
-// written by k_rank_product.
+// Bn row j*rn + n of group g (planned layer i = g*lpt + j): columns [0, d) hold 2 U[src[i]][:][n]
+// for n < r and i < L; everything else is zero here. The G blocks are written by
+// k_rank_product.
 __global__ void k_pack_norm_u(const uint16_t* __restrict__ U, uint16_t* __restrict__ Bn, int L,
-                              int r, int r_pad, int d, int k_total, PackLayers pl) {
-  const long long total = static_cast<long long>(L) * r_pad * k_total;
+                              int r, int d, int lpt, int rn, int groups, int bn_k, PackLayers pl) {
+  const long long total = static_cast<long long>(groups) * 256 * bn_k;
   for (long long e = blockIdx.x * static_cast<long long>(blockDim.x) + threadIdx.x; e < total;
        e += static_cast<long long>(gridDim.x) * blockDim.x) {
-    const int j = static_cast<int>(e % k_total);
-    const long long row = e / k_total;
-    const int n = static_cast<int>(row % r_pad), i = static_cast<int>(row / r_pad);
+    const int j = static_cast<int>(e % bn_k);
+    const long long row = e / bn_k;
+    const int jr = static_cast<int>(row % 256), g = static_cast<int>(row / 256);
+    const int n = jr % rn, i = g * lpt + jr / rn;
     float v = 0.0f;
-    if (j < d && n < r && !pl.zero_du[i])
+    if (j < d && n < r && i < L && !pl.zero_du[i])
       v = 2.0f * bf(U[(static_cast<long long>(pl.src[i]) * d + j) * r + n]);
-    Bn[e] = to_bf16(v);  // the G columns (j >= d) are zero here and filled afterwards
+    Bn[e] = to_bf16(v);
   }
 }
 
@@ -244,8 +249,8 @@ __global__ void k_pack_kv(const uint16_t* __restrict__ Wk, const uint16_t* __res
 // in MODE 1 the fp32 result also goes to gout[p][i][n] when gout is given:
 //   MODE 0 (fold):  A(l, i, j) = W_part[l][c][j] * gamma[l][j], i indexes the 2*kv Wkv rows
 //                   of the layer; the result goes to Wkv row (p, i), column d + n
-//   MODE 1 (gram):  A(l, i, j) = U[l][j][i], i < r; the result goes to Bn row p*r_pad + i,
-//                   column d + n
+//   MODE 1 (gram):  A(l, i, j) = U[l][j][i], i < r; the result goes to Bn row
+//                   (p / lpt) * 256 + (p % lpt) * rn + i, column d + (p % lpt) * r_pad + n
 // 64 x 64 output tile per block, 256 threads with 4 x 4 outputs each, j in steps of 32.
 template <int MODE>
 __global__ void __launch_bounds__(256) k_rank_product(const uint16_t* __restrict__ Wk,
@@ -255,7 +260,7 @@ __global__ void __launch_bounds__(256) k_rank_product(const uint16_t* __restrict
                                                       uint16_t* __restrict__ out, int rows, int r,
                                                       int d, int kv, int HD, int r_pad,
                                                       int k_total, PackLayers pl,
-                                                      float* __restrict__ gout) {
+                                                      float* __restrict__ gout, int lpt, int rn) {
   __shared__ float As[32][65];
   __shared__ float Us[32][65];
   const int p = blockIdx.z, l = pl.src[p];
@@ -306,12 +311,13 @@ __global__ void __launch_bounds__(256) k_rank_product(const uint16_t* __restrict
     const int i = i0 + ty * 4 + q;
     if (i >= rows) continue;
     const long long orow = MODE == 0 ? static_cast<long long>(p) * 2 * kv + i
-                                     : static_cast<long long>(p) * r_pad + i;
+                                     : static_cast<long long>(p / lpt) * 256 + (p % lpt) * rn + i;
+    const int ocol = MODE == 0 ? d : d + (p % lpt) * r_pad;
 #pragma unroll
     for (int w = 0; w < 4; ++w) {
       const int n = n0 + tx * 4 + w;
       if (n >= r) continue;
-      if (out) out[orow * k_total + d + n] = to_bf16(acc[q][w]);
+      if (out) out[orow * k_total + ocol + n] = to_bf16(acc[q][w]);
       if (MODE == 1 && gout) gout[(static_cast<long long>(p) * r_pad + i) * r_pad + n] = acc[q][w];
     }
   }
@@ -861,14 +867,17 @@ cudaError_t enqueue_build(const PlanView& v, const BuildArgs& a, cudaStream_t st
   }
   mark(2);
 
-  // (2) rstd_l from ||x0||^2 + h_l . ([x0 | h_l] [2 U_l^T ; G_l]).
-  gp.s = {static_cast<int>(T), L, v.r_pad, d / 64, v.r_pad / 64, v.r_pad, 0, 0, 0, 0};
-  if (rank_pairs) tm_groups(gp.s, v.r_pad, T);
-  gp.norm = {a.H, static_cast<int>(n1), v.r_pad, a.xx, a.rstd, static_cast<int>(T), 1.0f / d,
-             v.rms_eps};
+  // (2) rstd_l from ||x0||^2 + h_l . ([x0 | h_l] [2 U_l^T ; G_l]): 256-column tiles of lpt
+  // layers each, A = [x0 | h of the group's layers] (contiguous H columns), B = the group's
+  // Bn rows (block-diagonal G).
+  const int lpt = v.bn_lpt;
+  gp.s = {static_cast<int>(T), v.bn_groups, 256, d / 64, lpt * v.r_pad / 64, lpt * v.r_pad, 0, 0, 0, 0};
+  if (rank_pairs) tm_groups(gp.s, 256, T);
+  gp.norm = {a.H, static_cast<int>(n1), v.r_pad, lpt, v.bn_rn, L, a.xx, a.rstd,
+             static_cast<int>(T), 1.0f / d, v.rms_eps};
   if (err == cudaSuccess) {
-    err = rank_pairs ? launch_pair_tm(EPI_NORM, v.r_pad, 0, tm_x0_s, tm_H_s, *v.tm_Bn_half, gp, v.num_sms, st)
-                     : launch_gemm(EPI_NORM, v.r_pad, 0, tm_x0, tm_H, *v.tm_Bn, gp, v.num_sms, st);
+    err = rank_pairs ? launch_pair_tm(EPI_NORM, 256, 0, tm_x0_s, tm_H_s, *v.tm_Bn_half, gp, v.num_sms, st)
+                     : launch_gemm(EPI_NORM, 256, 0, tm_x0, tm_H, *v.tm_Bn, gp, v.num_sms, st);
   }
   mark(3);
   }
@@ -938,6 +947,9 @@ bool plan_view(const dv_plan* p, PlanView* v) {
   v->Gf = p->Gf;
   v->tm_Dst_half = p->tm_Dst_half;
   v->tm_Bn = &p->tm_Bn;
+  v->bn_lpt = p->bn_lpt;
+  v->bn_rn = p->bn_rn;
+  v->bn_groups = p->bn_groups;
   v->tm_Bn_half = &p->tm_Bn_half;
   v->tm_Wkv = &p->tm_Wkv;
   v->tm_Dst_rp = &p->tm_Dst_rp;
@@ -1035,6 +1047,9 @@ int dv_memory_plan(const dv_config* cfg, const dv_weights* w, void* stream, dv_p
   // Embedding adapter: K/V weights carry the folded rank-r columns. Recurrent: the K/V GEMM
   // reads M_l itself, so only the d columns of W diag(gamma).
   p->k_total = rec ? d : d + p->r_pad;
+  dv::norm_group(p->r_pad, &p->bn_lpt, &p->bn_rn);
+  p->bn_groups = (L + p->bn_lpt - 1) / p->bn_lpt;
+  p->bn_k = d + p->bn_lpt * p->r_pad;
   p->resid_bn = d % 256 == 0 ? 256 : (d % 128 == 0 ? 128 : 64);
   p->max_tokens = cfg->max_batch * cfg->max_n_vis;
   const long long T = p->max_tokens;
@@ -1056,7 +1071,7 @@ int dv_memory_plan(const dv_config* cfg, const dv_weights* w, void* stream, dv_p
   const int dst_ld = d + 64;
   bool ok = dmalloc(&p->Dst, sizeof(uint16_t) * dst_rows * dst_ld) &&
             (rec ? dmalloc(&p->Uup, sizeof(uint16_t) * static_cast<size_t>(L) * d * p->r_pad)
-                 : dmalloc(&p->Bn, sizeof(uint16_t) * L * p->r_pad * p->k_total)) &&
+                 : dmalloc(&p->Bn, sizeof(uint16_t) * p->bn_groups * 256 * p->bn_k)) &&
             dmalloc(&p->Wkv, sizeof(uint16_t) * static_cast<size_t>(L) * 2 * p->kv * p->k_total) &&
             dmalloc(&p->ws, ws_bytes) && dmalloc(&p->status, sizeof(int));
   if (ok && cfg->has_kv_bias)
@@ -1091,14 +1106,14 @@ int dv_memory_plan(const dv_config* cfg, const dv_weights* w, void* stream, dv_p
     k_pack_2u<<<grid_for(1LL * L * p->r_pad * d), 256, 0, st>>>(
         U, p->Dst + static_cast<size_t>(L) * p->r_pad * dst_ld, L, r, p->r_pad, d, dst_ld, pl);
     cudaMemsetAsync(p->Gf, 0, sizeof(float) * L * p->r_pad * p->r_pad, st);
-    k_pack_norm_u<<<grid_for(1LL * L * p->r_pad * p->k_total), 256, 0, st>>>(U, p->Bn, L, r, p->r_pad,
-                                                                             d, p->k_total, pl);
+    k_pack_norm_u<<<grid_for(1LL * p->bn_groups * 256 * p->bn_k), 256, 0, st>>>(
+        U, p->Bn, L, r, d, p->bn_lpt, p->bn_rn, p->bn_groups, p->bn_k, pl);
     dim3 g1((r + 63) / 64, (r + 63) / 64, L);
     k_rank_product<1><<<g1, 256, 0, st>>>(Wk, Wv, G, U, p->Bn, r, r, d, p->kv, HD, p->r_pad,
-                                          p->k_total, pl, p->Gf);
+                                          p->bn_k, pl, p->Gf, p->bn_lpt, p->bn_rn);
     dim3 g0((r + 63) / 64, (2 * p->kv + 63) / 64, L);
     k_rank_product<0><<<g0, 256, 0, st>>>(Wk, Wv, G, U, p->Wkv, 2 * p->kv, r, d, p->kv, HD,
-                                          p->r_pad, p->k_total, pl, nullptr);
+                                          p->r_pad, p->k_total, pl, nullptr, 1, 0);
   }
   if (cfg->has_kv_bias) {
     k_bias_to_f32<<<grid_for(1LL * L * p->kv), 256, 0, st>>>(static_cast<const uint16_t*>(w->bk),
@@ -1128,9 +1143,8 @@ int dv_memory_plan(const dv_config* cfg, const dv_weights* w, void* stream, dv_p
     enc = encode_2d(&p->tm_Dst_rp, p->Dst, d, 1ull * L * p->r_pad, dst_ld, p->r_pad) &&
           encode_2d(&p->tm_Uup, p->Uup, p->r_pad, 1ull * L * d, p->r_pad, p->resid_bn);
   } else if (enc) {
-    enc = encode_slabs(&p->tm_Bn_half, p->Bn, p->k_total, 1ull * L * p->r_pad, p->k_total,
-                       p->r_pad / 2) &&
-          encode_2d(&p->tm_Bn, p->Bn, p->k_total, 1ull * L * p->r_pad, p->k_total, p->r_pad);
+    enc = encode_slabs(&p->tm_Bn_half, p->Bn, p->bn_k, 256ull * p->bn_groups, p->bn_k, 128) &&
+          encode_2d(&p->tm_Bn, p->Bn, p->bn_k, 256ull * p->bn_groups, p->bn_k, 256);
   }
   if (!enc) {
     free_plan_memory(p);

@@ -144,37 +144,43 @@ __device__ __forceinline__ void epi_silu(const GemmParams& p, uint32_t tbase, in
 }
 
 // ||m||^2 = ||x0||^2 + h . (2 x0 U^T + h G) with G = U U^T, so with acc = [x0 | h] [2U^T; G]
-// the statistic of RMSNorm is rstd = 1 / sqrt((xx + h . acc) / d + eps).
+// the statistic of RMSNorm is rstd = 1 / sqrt((xx + h . acc) / d + eps). A tile of group l
+// holds the lpt layers l * lpt + j in columns [j rn, j rn + r_pad) (the B operand's G blocks
+// are block-diagonal against [h_{l lpt} | h_{l lpt + 1} | ...]); columns past r_pad within a
+// layer's rn are zero rows and skipped.
 template <int BN>
 __device__ __forceinline__ void epi_norm(const GemmParams& p, uint32_t tbase, int l, int t) {
+  const EpiNorm& e = p.norm;
   const bool valid = t < p.s.M;
-  const uint16_t* hrow = p.norm.H + static_cast<size_t>(valid ? t : 0) * p.norm.ldh +
-                         static_cast<size_t>(l) * p.norm.r_pad;
+  const uint16_t* hrow = e.H + static_cast<size_t>(valid ? t : 0) * e.ldh;
   float dot = 0.0f;
 #pragma unroll 1
   for (int c = 0; c < BN / 32; ++c) {
+    const int j = (c * 32) / e.rn, n0 = (c * 32) % e.rn;
+    const int layer = l * e.lpt + j;
+    if (layer >= e.n_layers || n0 >= e.r_pad) continue;  // uniform over the warp
     uint32_t r[32];
     __syncwarp();
     tmem_ld32(tbase + c * 32, r);
     tmem_ld_wait();
     if (valid) {
-      const uint4* hv = reinterpret_cast<const uint4*>(hrow + c * 32);
+      const uint4* hv = reinterpret_cast<const uint4*>(hrow + static_cast<size_t>(layer) * e.r_pad + n0);
 #pragma unroll
       for (int q = 0; q < 4; ++q) {
         const uint4 w = hv[q];
         const uint32_t ws[4] = {w.x, w.y, w.z, w.w};
 #pragma unroll
-        for (int e = 0; e < 4; ++e) {
-          dot = fmaf(bf16_bits_to_float(ws[e] & 0xFFFFu), __uint_as_float(r[q * 8 + 2 * e]), dot);
-          dot = fmaf(bf16_bits_to_float(ws[e] >> 16), __uint_as_float(r[q * 8 + 2 * e + 1]), dot);
+        for (int u = 0; u < 4; ++u) {
+          dot = fmaf(bf16_bits_to_float(ws[u] & 0xFFFFu), __uint_as_float(r[q * 8 + 2 * u]), dot);
+          dot = fmaf(bf16_bits_to_float(ws[u] >> 16), __uint_as_float(r[q * 8 + 2 * u + 1]), dot);
         }
       }
+      if (n0 + 32 == e.r_pad) {  // the layer's last columns: its statistic is complete
+        const float ss = fmaxf(e.xx[t] + dot, 0.0f);
+        e.rstd[static_cast<size_t>(layer) * e.ld_rstd + t] = rsqrtf(fmaf(ss, e.inv_d, e.eps));
+        dot = 0.0f;
+      }
     }
-  }
-  if (valid) {
-    const float ss = fmaxf(p.norm.xx[t] + dot, 0.0f);
-    p.norm.rstd[static_cast<size_t>(l) * p.norm.ld_rstd + t] =
-        rsqrtf(fmaf(ss, p.norm.inv_d, p.norm.eps));
   }
 }
 

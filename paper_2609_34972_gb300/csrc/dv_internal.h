@@ -82,10 +82,20 @@ struct EpiSilu {
   int ldc;
 };
 
+// Layers of the statistic GEMM per 256-column tile: its B operand (Bn) groups `lpt` layers, a
+// layer's rows `rn` apart: r_pad <= 64: 4 layers of 64 rows; <= 128: 2 of 128; else 1 of 256
+// (r_pad = 192 leaves 64 zero rows).
+__host__ __device__ inline void norm_group(int r_pad, int* lpt, int* rn) {
+  *lpt = r_pad <= 64 ? 4 : (r_pad <= 128 ? 2 : 1);
+  *rn = 256 / *lpt;
+}
+
 struct EpiNorm {
   const uint16_t* H;  // bf16 [M_ld][ldh], h_l at columns l * r_pad
   int ldh;
   int r_pad;
+  int lpt, rn;        // layers per 256-column tile and their row stride (norm_group)
+  int n_layers;       // planned layers (the last group may hold fewer)
   const float* xx;    // [M] row sums of squares of x0
   float* rstd;        // [L][ld_rstd]
   int ld_rstd;
@@ -220,8 +230,9 @@ struct PlanView {
                                    // rows [0, L r_pad) D, rows [L r_pad, 2 L r_pad) 2 U^T
   const float* Gf;                 // embedding adapter: G_l = U_l^T U_l, fp32 [L][r_pad][r_pad]
   const CUtensorMap* tm_Dst_half;  // three slab maps: boxes of 32, 64, 128 rows (pair halves)
-  const CUtensorMap* tm_Bn;        // boxes of r_pad rows
-  const CUtensorMap* tm_Bn_half;   // slab map, boxes of r_pad / 2 rows
+  const CUtensorMap* tm_Bn;        // boxes of 256 rows (one layer group, norm_group)
+  const CUtensorMap* tm_Bn_half;   // slab map, boxes of 128 rows
+  int bn_lpt, bn_rn, bn_groups;    // statistic GEMM: layers per group, their row stride, groups
   const CUtensorMap* tm_Wkv;       // slab map, boxes of 128 rows
   const CUtensorMap* tm_Dst_rp;    // recurrent: boxes of r_pad rows (one layer's D)
   const CUtensorMap* tm_Uup;       // recurrent: [L*d][r_pad], boxes of resid_bn rows

@@ -151,6 +151,27 @@ def test_tokens_as_m_path_rank64_two_batches():
     _full_check(synth.make_inputs(cfg), "tokens-as-M rank 64")
 
 
+# The statistic GEMM groups layers into 256-column tiles (4 layers for r_pad = 64, 2 for 128, 1
+# for 192 and 256, a 192-wide rank leaving 64 zero rows). These cases pin ranks padded to 192 on
+# both rank-r engines and layer counts that leave the last group partly empty.
+
+@pytest.mark.parametrize("n_vis,batch,engine", [(256, 2, "2-SM tokens as M"), (150, 2, "1-SM")])
+def test_rank_padded_to_192(n_vis, batch, engine):
+    cfg = gu.small_config(f"r150_{n_vis}", d=768, n_layers=3, n_kv_heads=2, n_heads=4, head_dim=128,
+                          rank=150, n_vis=n_vis, batch=batch, x0_sigma=0.5, seed=41, pos_start=35)
+    _full_check(synth.make_inputs(cfg), f"rank 150 (r_pad 192), {engine}")
+
+
+@pytest.mark.parametrize("rank,n_layers,n_vis,engine", [(16, 5, 512, "2-SM, groups of 4"),
+                                                        (96, 3, 512, "2-SM, groups of 2"),
+                                                        (96, 3, 300, "1-SM, groups of 2")])
+def test_statistic_layer_groups_partly_empty(rank, n_layers, n_vis, engine):
+    cfg = gu.small_config(f"grp_{rank}_{n_layers}_{n_vis}", d=512, n_layers=n_layers, n_kv_heads=2,
+                          n_heads=4, head_dim=128, rank=rank, n_vis=n_vis, batch=1, x0_sigma=0.5,
+                          seed=42 + n_layers, pos_start=35)
+    _full_check(synth.make_inputs(cfg), f"rank {rank}, {n_layers} layers, {engine}")
+
+
 # Layer-wise adapter skipping (App. J): DV_LAYER_DROP layers get no K/V (their cache rows keep
 # the fill value); DV_LAYER_IDENTITY layers build K/V from M_l = E, which the oracle computes with
 # that layer's adapter weights set to zero (U_l = 0 gives the identity, Sec. 3.1).
