@@ -20,6 +20,7 @@
 #include <cstdlib>
 #include <cstring>
 #include <mutex>
+#include <utility>
 #include <vector>
 
 #include "../../include/dv.h"
@@ -136,6 +137,22 @@ bool encode_3d(CUtensorMap* map, const void* ptr, uint64_t cols, uint64_t rows, 
   return fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(ptr), dims, strides, box,
             estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+// Launch of a build kernel with programmatic stream serialization (dv::pdl_attribute); the
+// kernel calls dv::pdl_wait() before touching global memory.
+template <typename... KArgs, typename... Args>
+cudaError_t launch_pdl(void (*kern)(KArgs...), dim3 grid, dim3 block, cudaStream_t st,
+                       Args&&... args) {
+  cudaLaunchConfig_t cfg = {};
+  cudaLaunchAttribute attr[1] = {dv::pdl_attribute()};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = 0;
+  cfg.stream = st;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kern, std::forward<Args>(args)...);
 }
 
 // ------------------------------------------------------------------------------ small kernels
@@ -350,6 +367,8 @@ __global__ void k_pack_up(const uint16_t* __restrict__ U, uint16_t* __restrict__
 // recurrent state M_i summed in column-tile order (n < n_parts; layer stride ld_part).
 __global__ void k_rstd_parts(const float* __restrict__ part, int L, long long T, int n_parts,
                              long long ld_part, float inv_d, float eps, float* __restrict__ rstd) {
+  dv::pdl_wait();
+  dv::pdl_trigger();
   const long long total = static_cast<long long>(L) * T;
   for (long long e = blockIdx.x * static_cast<long long>(blockDim.x) + threadIdx.x; e < total;
        e += static_cast<long long>(gridDim.x) * blockDim.x) {
@@ -377,6 +396,8 @@ __global__ void __launch_bounds__(64) k_rstd_hc(const uint16_t* __restrict__ H, 
                                                 const float* __restrict__ Gf, int T, float inv_d,
                                                 float eps, float* __restrict__ rstd) {
   static_assert(RP == 64, "one quarter = 16 sums = 4 float4");
+  dv::pdl_wait();
+  dv::pdl_trigger();
   __shared__ __align__(16) float g[RP * RP];
   __shared__ __align__(16) float hs[RP][64];
   const int l = blockIdx.y, tid = threadIdx.x;
@@ -469,6 +490,8 @@ __global__ void __launch_bounds__(64) k_rstd_hc(const uint16_t* __restrict__ H, 
 
 // xx[t] = sum_j x0[t][j]^2 (fp32), one warp per token row, 16-byte loads.
 __global__ void k_row_sumsq(const uint16_t* __restrict__ x0, int T, int d, float* __restrict__ xx) {
+  dv::pdl_wait();
+  dv::pdl_trigger();
   const int warp = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
   const int lane = threadIdx.x & 31;
   if (warp >= T) return;
@@ -734,9 +757,8 @@ static cudaError_t enqueue_recurrent(const PlanView& v, const BuildArgs& a, cuda
                        a.H, v.status, kTimeoutNs, st);
     if (err == cudaSuccess) {
       mark(2);
-      k_rstd_parts<<<grid_for(static_cast<long long>(L) * T), 256, 0, st>>>(
-          a.part, L, T, S, part_ld, 1.0f / d, v.rms_eps, a.rstd);
-      err = cudaGetLastError();
+      err = launch_pdl(k_rstd_parts, dim3(grid_for(static_cast<long long>(L) * T)), dim3(256), st,
+                       a.part, L, T, S, part_ld, 1.0f / d, v.rms_eps, a.rstd);
       mark(3);
       return err == cudaSuccess ? launch_recurrent_kv(v, a, T, tm_mem_s, st, mark) : err;
     }
@@ -773,9 +795,8 @@ static cudaError_t enqueue_recurrent(const PlanView& v, const BuildArgs& a, cuda
   }
   mark(2);
   if (err == cudaSuccess) {
-    k_rstd_parts<<<grid_for(static_cast<long long>(L) * T), 256, 0, st>>>(
-        a.part, L, T, d / v.resid_bn, part_ld, 1.0f / d, v.rms_eps, a.rstd);
-    err = cudaGetLastError();
+    err = launch_pdl(k_rstd_parts, dim3(grid_for(static_cast<long long>(L) * T)), dim3(256), st,
+                     a.part, L, T, d / v.resid_bn, part_ld, 1.0f / d, v.rms_eps, a.rstd);
   }
   mark(3);
   return err == cudaSuccess ? launch_recurrent_kv(v, a, T, tm_mem_s, st, mark) : err;
@@ -807,9 +828,8 @@ cudaError_t enqueue_build(const PlanView& v, const BuildArgs& a, cudaStream_t st
   for (int i = 0; i < L; ++i) gp.layer_map[i] = v.active[i];
 
   mark(0);
-  k_row_sumsq<<<static_cast<int>((T + 7) / 8), 256, 0, st>>>(static_cast<const uint16_t*>(a.x0),
-                                                             static_cast<int>(T), d, a.xx);
-  cudaError_t err = cudaGetLastError();
+  cudaError_t err = launch_pdl(k_row_sumsq, dim3(static_cast<unsigned>((T + 7) / 8)), dim3(256), st,
+                               static_cast<const uint16_t*>(a.x0), static_cast<int>(T), d, a.xx);
   mark(1);
 
   // (1) H = SiLU(x0 [D_1 ... D_L]) — one GEMM over all layers' down-projections.
@@ -834,10 +854,10 @@ cudaError_t enqueue_build(const PlanView& v, const BuildArgs& a, cudaStream_t st
     mark(2);
     if (err == cudaSuccess) {
       dim3 grid(static_cast<unsigned>((T + 63) / 64), static_cast<unsigned>(L));
-      k_rstd_hc<64><<<grid, 64, 0, st>>>(a.H, static_cast<int>(n1), a.c, static_cast<int>(n1),
-                                         a.xx, v.Gf, static_cast<int>(T), 1.0f / d, v.rms_eps,
-                                         a.rstd);
-      err = cudaGetLastError();
+      err = launch_pdl(k_rstd_hc<64>, grid, dim3(64), st, static_cast<const uint16_t*>(a.H),
+                       static_cast<int>(n1), static_cast<const float*>(a.c), static_cast<int>(n1),
+                       static_cast<const float*>(a.xx), v.Gf, static_cast<int>(T), 1.0f / d,
+                       v.rms_eps, a.rstd);
     }
     mark(3);
   } else {

@@ -184,6 +184,8 @@ __global__ void __launch_bounds__(kChainThreads, 1)
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
+  pdl_wait();
+  pdl_trigger();
   const uint32_t t_state = tmem, t_z = tmem + CW;
   const uint32_t lane_base = static_cast<uint32_t>(warp * 32) << 16;
 
@@ -429,7 +431,7 @@ cudaError_t launch_t(int S, long long blocks, const CUtensorMap& x, const CUtens
     err = cudaFuncSetAttribute(kern, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
   if (err != cudaSuccess) return err;
   cudaLaunchConfig_t cfg = {};
-  cudaLaunchAttribute attr[1];
+  cudaLaunchAttribute attr[2];
   attr[0].id = cudaLaunchAttributeClusterDimension;
   attr[0].val.clusterDim.x = static_cast<unsigned>(S);
   attr[0].val.clusterDim.y = 1;
@@ -445,6 +447,8 @@ cudaError_t launch_t(int S, long long blocks, const CUtensorMap& x, const CUtens
     cudaGetLastError();
     return cudaErrorNotSupported;  // the caller falls back to the per-layer launches
   }
+  attr[1] = pdl_attribute();
+  cfg.numAttrs = 2;
   err = cudaLaunchKernelEx(&cfg, kern, x, dmap, umap, mmap, p);
   if (err != cudaSuccess) return err;
   return cudaGetLastError();

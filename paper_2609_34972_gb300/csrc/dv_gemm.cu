@@ -105,6 +105,8 @@ __global__ void __launch_bounds__(kNumThreads, 1)
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
+  pdl_wait();
+  pdl_trigger();
 
   const int m_tiles = (p.s.M + kBlockM - 1) / kBlockM;
   const int n_tiles = p.s.n_per_layer / BN;
@@ -248,7 +250,16 @@ static cudaError_t launch_t(const CUtensorMap& a0, const CUtensorMap& a1, const 
   const long long tiles = m_tiles * (p.s.n_per_layer / BN) * p.s.n_layers;
   if (tiles <= 0) return cudaSuccess;
   const int grid = static_cast<int>(tiles < num_sms ? tiles : num_sms);
-  kern<<<grid, kNumThreads, C::kSmemBytes, stream>>>(a0, a1, b, p);
+  cudaLaunchConfig_t cfg = {};
+  cudaLaunchAttribute attr[1] = {pdl_attribute()};
+  cfg.gridDim = dim3(static_cast<unsigned>(grid), 1, 1);
+  cfg.blockDim = dim3(kNumThreads, 1, 1);
+  cfg.dynamicSmemBytes = C::kSmemBytes;
+  cfg.stream = stream;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  err = cudaLaunchKernelEx(&cfg, kern, a0, a1, b, p);
+  if (err != cudaSuccess) return err;
   return cudaGetLastError();
 }
 

@@ -82,6 +82,15 @@ struct EpiSilu {
   int ldc;
 };
 
+// Launch attribute of the build's kernels: programmatic stream serialization (see pdl_wait in
+// dv_ptx.cuh; every kernel launched with it calls pdl_wait before touching global memory).
+inline cudaLaunchAttribute pdl_attribute() {
+  cudaLaunchAttribute a;
+  a.id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  a.val.programmaticStreamSerializationAllowed = 1;
+  return a;
+}
+
 // Layers of the statistic GEMM per 256-column tile: its B operand (Bn) groups `lpt` layers, a
 // layer's rows `rn` apart: r_pad <= 64: 4 layers of 64 rows; <= 128: 2 of 128; else 1 of 256
 // (r_pad = 192 leaves 64 zero rows).

@@ -113,6 +113,8 @@ __global__ void __launch_bounds__(kPairThreads, 1)
   cluster_sync();  // barriers of both CTAs initialised, TMEM allocated in both
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
+  pdl_wait();
+  pdl_trigger();
 
   const int tok_tiles = (p.s.M + NT - 1) / NT;
   const int groups = p.kv.kv / 128;
@@ -298,7 +300,7 @@ static cudaError_t launch_pair_t(const CUtensorMap& w, const CUtensorMap& x, con
   const long long tiles = static_cast<long long>((p.s.M + NT - 1) / NT) * (p.kv.kv / 128) * p.s.n_layers;
   if (tiles <= 0) return cudaSuccess;
   cudaLaunchConfig_t cfg = {};
-  cudaLaunchAttribute attr[1];
+  cudaLaunchAttribute attr[2];
   attr[0].id = cudaLaunchAttributeClusterDimension;
   attr[0].val.clusterDim.x = 2;
   attr[0].val.clusterDim.y = 1;
@@ -316,6 +318,8 @@ static cudaError_t launch_pair_t(const CUtensorMap& w, const CUtensorMap& x, con
   }
   const long long pairs = tiles < max_clusters ? tiles : max_clusters;
   cfg.gridDim = dim3(static_cast<unsigned>(2 * pairs), 1, 1);
+  attr[1] = pdl_attribute();
+  cfg.numAttrs = 2;
   err = cudaLaunchKernelEx(&cfg, kern, w, x, h, p);
   if (err != cudaSuccess) return err;
   return cudaGetLastError();

@@ -111,6 +111,8 @@ __global__ void __launch_bounds__(kTmThreads, 1)
   cluster_sync();
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
+  pdl_wait();
+  pdl_trigger();
 
   const int m_tiles = (p.s.M + 255) / 256;
   const int n_tiles = p.s.n_per_layer / BN;
@@ -275,7 +277,7 @@ static cudaError_t launch_tm_t(const CUtensorMap& a0, const CUtensorMap& a1, con
       static_cast<long long>((p.s.M + 255) / 256) * (p.s.n_per_layer / BN) * p.s.n_layers;
   if (tiles <= 0) return cudaSuccess;
   cudaLaunchConfig_t cfg = {};
-  cudaLaunchAttribute attr[1];
+  cudaLaunchAttribute attr[2];
   attr[0].id = cudaLaunchAttributeClusterDimension;
   attr[0].val.clusterDim.x = 2;
   attr[0].val.clusterDim.y = 1;
@@ -293,6 +295,8 @@ static cudaError_t launch_tm_t(const CUtensorMap& a0, const CUtensorMap& a1, con
   }
   const long long pairs = tiles < max_clusters ? tiles : max_clusters;
   cfg.gridDim = dim3(static_cast<unsigned>(2 * pairs), 1, 1);
+  attr[1] = pdl_attribute();
+  cfg.numAttrs = 2;
   err = cudaLaunchKernelEx(&cfg, kern, a0, a1, b, p);
   if (err != cudaSuccess) return err;
   return cudaGetLastError();
