@@ -96,28 +96,6 @@ __device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* map
       : "memory");
 }
 
-// Same, with an L2 cache-policy hint (createpolicy value).
-__device__ __forceinline__ void tma_load_2d_hint(uint32_t dst, const CUtensorMap* map,
-                                                 uint32_t bar, int c0, int c1, uint64_t policy) {
-  asm volatile(
-      "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes.L2::cache_hint"
-      " [%0], [%1, {%3, %4}], [%2], %5;" ::"r"(dst),
-      "l"(reinterpret_cast<uint64_t>(map)), "r"(bar), "r"(c0), "r"(c1), "l"(policy)
-      : "memory");
-}
-
-__device__ __forceinline__ uint64_t policy_evict_first() {
-  uint64_t p;
-  asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(p));
-  return p;
-}
-
-__device__ __forceinline__ uint64_t policy_evict_last() {
-  uint64_t p;
-  asm volatile("createpolicy.fractional.L2::evict_last.b64 %0, 1.0;" : "=l"(p));
-  return p;
-}
-
 // ------------------------------------------------------------------------------ tcgen05
 
 // Warp-wide: allocate `ncols` TMEM columns (power of two >= 32); base address -> smem slot.
@@ -246,27 +224,11 @@ __device__ __forceinline__ void mbar_arrive_cluster(uint32_t cbar) {
                : "memory");
 }
 
-__device__ __forceinline__ void mbar_arrive_expect_tx_cluster(uint32_t cbar, uint32_t bytes) {
-  asm volatile("mbarrier.arrive.expect_tx.release.cluster.shared::cluster.b64 _, [%0], %1;" ::"r"(
-                   cbar),
-               "r"(bytes)
-               : "memory");
-}
-
-// TMA tile load into this CTA's shared memory whose completion is counted on an mbarrier
-// that may live in the peer CTA of the pair (`cbar` is a shared::cluster address).
-__device__ __forceinline__ void tma_load_2d_pair(uint32_t dst, const CUtensorMap* map,
-                                                 uint32_t cbar, int c0, int c1) {
-  asm volatile(
-      "cp.async.bulk.tensor.2d.cta_group::2.shared::cluster.global.mbarrier::complete_tx::bytes"
-      " [%0], [%1, {%3, %4}], [%2];" ::"r"(dst),
-      "l"(reinterpret_cast<uint64_t>(map)), "r"(cbar), "r"(c0), "r"(c1)
-      : "memory");
-}
-
-// 3-D form of tma_load_2d_pair, for tensor maps that view a [rows][cols] matrix as
-// {64 columns, rows, cols / 64 slabs}: one box brings several consecutive K slabs of a row
-// block, each slab a 128-byte-swizzled [rows][64] tile, the slabs one after another.
+// TMA load into this CTA's shared memory whose completion is counted on an mbarrier that may
+// live in the peer CTA of the pair (`cbar` is a shared::cluster address), for tensor maps that
+// view a [rows][cols] matrix as {64 columns, rows, cols / 64 slabs}: one box brings several
+// consecutive K slabs of a row block, each slab a 128-byte-swizzled [rows][64] tile, the slabs
+// one after another.
 __device__ __forceinline__ void tma_load_3d_pair(uint32_t dst, const CUtensorMap* map,
                                                  uint32_t cbar, int row, int slab) {
   asm volatile(
