@@ -44,11 +44,11 @@ struct PairCfg {
   static constexpr int kABytes = kSlabsPerStep * kASlab;
   static constexpr int kBBytes = kSlabsPerStep * kBSlab;
   static constexpr int kStageBytes = kABytes + kBBytes;
-  static constexpr int kStagingBytes = 2 * 32 * 4 * 4;  // K-norm partial sums [2][token][warp]
-  static constexpr int kRingBudget = kSmemLimit - kStagingBytes - 1024 - 512;
+  static constexpr int kKnormBytes = 2 * 32 * 4 * 4;  // K-norm partial sums [2][token][warp]
+  static constexpr int kRingBudget = kSmemLimit - kKnormBytes - 1024 - 512;
   static constexpr int kStagesRaw = kRingBudget / kStageBytes;
   static constexpr int kStages = kStagesRaw > 8 ? 8 : kStagesRaw;
-  static constexpr int kSmemBytes = kStages * kStageBytes + kStagingBytes + 1024 + 512;
+  static constexpr int kSmemBytes = kStages * kStageBytes + kKnormBytes + 1024 + 512;
   static constexpr int kTmemCols = 512;
   static_assert(NT % 64 == 0 && NT >= 64 && NT <= 256, "N tile");
   static_assert(kASlab % 1024 == 0 && kBSlab % 1024 == 0, "slab tiles must stay 1024-byte aligned");
@@ -72,8 +72,8 @@ __global__ void __launch_bounds__(kPairThreads, 1)
   const uint32_t raw = smem_addr(smem_raw);
   const uint32_t ring = (raw + 1023u) & ~1023u;
   uint8_t* ring_ptr = smem_raw + (ring - raw);
-  float* staging = reinterpret_cast<float*>(ring_ptr + S * C::kStageBytes);
-  uint64_t* bars = reinterpret_cast<uint64_t*>(ring_ptr + S * C::kStageBytes + C::kStagingBytes);
+  float* knorm_pad = reinterpret_cast<float*>(ring_ptr + S * C::kStageBytes);  // K-norm partials
+  uint64_t* bars = reinterpret_cast<uint64_t*>(ring_ptr + S * C::kStageBytes + C::kKnormBytes);
   const uint32_t bar0 = smem_addr(bars);
   auto full_bar = [&](int s) { return bar0 + 8u * s; };            // used in the leader
   auto empty_bar = [&](int s) { return bar0 + 8u * (S + s); };     // both CTAs
@@ -249,7 +249,7 @@ __global__ void __launch_bounds__(kPairThreads, 1)
             // 2 for HD = 64). Each warp leaves its block's sum of squares for the token of each
             // lane; the head's blocks are summed in block order. Two buffers by chunk parity:
             // a warp rewrites one only after every warp has passed the next chunk's barrier.
-            float* pad = staging + ((c & 1) * 32 + lane) * 4;
+            float* pad = knorm_pad + ((c & 1) * 32 + lane) * 4;
             pad[q] = kv_k16_sumsq<HD>(p, tk, l, g, q, r);
             named_barrier(1, kEpiPairThreads);
             const float ss = HD == 128 ? ((pad[0] + pad[1]) + pad[2]) + pad[3]
