@@ -10,8 +10,8 @@
 // blocks. For each block a CTA:
 //   1. loads the K and V tiles by TMA (rows = slots, 128 B per 64 channels, 128-byte swizzle);
 //   2. one thread issues S = Q K^T (M = 128 rows, N = 128 keys, K = head_dim) into TMEM;
-//   3. the four warps transpose V into a K-major [head_dim][keys] tile (ldmatrix.trans /
-//      stmatrix), so both MMAs read K-major operands;
+//   3. the P V MMA reads V as it lies ([keys][channels] rows, an MN-major B operand), so V needs
+//      no transpose;
 //   4. each thread owns one query row: it reads its scores from TMEM twice (the block maximum,
 //      then exp2 of the masked, scaled scores), keeps the running maximum m and sum l, and
 //      writes the row's probabilities as bf16 into the A tile of the second MMA;
@@ -58,19 +58,17 @@ struct AttnCfg {
   static constexpr int kOffQ = 0;
   static constexpr int kOffStage = kOffQ + kKV;  // two stages of [K | V]
   static constexpr int kStage = 2 * kKV;
-  static constexpr int kOffVt = kOffStage + 2 * kStage;   // 2 key slabs of [HD rows][64 keys]
-  static constexpr int kVtSlab = HD * 128;
   // P (2 key slabs of [128 rows][64 keys]) takes the K slot of the current stage when that is
   // large enough (HD = 128): K is dead once the score MMA has completed.
   static constexpr bool kPInK = kKV >= 2 * kTile;
-  static constexpr int kOffP = kOffVt + 2 * kVtSlab;
+  static constexpr int kOffP = kOffStage + 2 * kStage;
   static constexpr int kEnd = kOffP + (kPInK ? 0 : 2 * kTile);
   static constexpr int kPitch = HD + 4;                   // floats per partial output row
   static constexpr int kPartBytes = 128 * kPitch * 4;
   static constexpr int kMisc = 2048;                      // barriers, m, l, key end
   static constexpr int kSmemBytes = kEnd + kMisc + 1024;
   static_assert(kPartBytes <= 2 * kStage, "partial outputs reuse the stages");
-  static_assert(kVtSlab % 1024 == 0 && kKV % 1024 == 0, "tiles stay 1024-byte aligned");
+  static_assert(kKV % 1024 == 0, "tiles stay 1024-byte aligned");
   static_assert(kSmemBytes <= 232448, "shared memory of one CTA");
 };
 
@@ -84,20 +82,18 @@ __device__ __forceinline__ void tma_load_4d(uint32_t dst, const CUtensorMap* map
       : "memory");
 }
 
-// Four 8x8 b16 matrices from shared memory, transposed (lanes 8i..8i+7 give the row
-// addresses of matrix i; register i receives this lane's fragment of its transpose).
-__device__ __forceinline__ void ldmatrix_x4_trans(uint32_t addr, uint32_t (&r)[4]) {
-  asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0, %1, %2, %3}, [%4];"
-               : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
-               : "r"(addr)
-               : "memory");
-}
-
-// Four 8x8 b16 matrices to shared memory (same fragment and address convention).
-__device__ __forceinline__ void stmatrix_x4(uint32_t addr, const uint32_t (&r)[4]) {
-  asm volatile("stmatrix.sync.aligned.m8n8.x4.shared.b16 [%0], {%1, %2, %3, %4};" ::"r"(addr),
-               "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3])
-               : "memory");
+// Shared-memory descriptor of an MN-major operand written by TMA with 128-byte swizzling, as V
+// lies in shared memory for the P V MMA: each 128-byte row holds 64 consecutive N elements
+// (channels) of one K index (key); 8-row (8-key) swizzle atoms are 1024 B apart along K (stride
+// byte offset) and the next 64 N elements sit `n_stride` bytes further (leading byte offset).
+__device__ __forceinline__ uint64_t sdesc_mnmajor_sw128(uint32_t saddr, uint32_t n_stride) {
+  uint64_t desc = 0;
+  desc |= static_cast<uint64_t>((saddr & 0x3FFFFu) >> 4);
+  desc |= static_cast<uint64_t>((n_stride >> 4) & 0x3FFFu) << 16;
+  desc |= static_cast<uint64_t>(1024 >> 4) << 32;
+  desc |= static_cast<uint64_t>(1) << 46;
+  desc |= static_cast<uint64_t>(2) << 61;
+  return desc;
 }
 
 // Orders this thread's generic-proxy shared-memory writes before later async-proxy reads
@@ -197,7 +193,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
   const int n_blocks = (*key_end + kKeyBlock - 1) / kKeyBlock;
   const int kb0 = split * n_blocks / S, kb1 = (split + 1) * n_blocks / S;
 
-  const uint32_t sQ = base + C::kOffQ, sVt = base + C::kOffVt;
+  const uint32_t sQ = base + C::kOffQ;
   const int q_row0 = (b * p.Hq + h * p.G) * p.Nt + qb * 128;
   auto sK = [&](int st) { return base + C::kOffStage + st * C::kStage; };
   auto sV = [&](int st) { return base + C::kOffStage + st * C::kStage + C::kKV; };
@@ -253,30 +249,8 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
       __syncwarp();
     }
 
-    // V -> Vt: 8x8 blocks (8 keys x 8 channels); lane 8i + j8 addresses row j8 of block i.
+    // V is read by the P V MMA as it lies ([keys][channels], an MN-major operand).
     ok = mbar_wait(bar_v(st), sph, abort_flag, tmo);
-    if (__all_sync(0xFFFFFFFFu, ok)) {
-      constexpr int kBlocks = (kKeyBlock / 8) * (HD / 8);
-      const int mi = lane >> 3, j8 = lane & 7;
-      const uint32_t v_base = sV(st);
-#pragma unroll 1
-      for (int quad = warp; quad < kBlocks / 4; quad += 4) {
-        const int blk = quad * 4 + mi;
-        const int key0 = (blk % (kKeyBlock / 8)) * 8, d0 = (blk / (kKeyBlock / 8)) * 8;
-        // stored row j8: key key0 + j8, channels d0 .. d0 + 7 (slab d0 / 64, 128-byte swizzle)
-        const int key = key0 + j8;
-        const uint32_t src = v_base + (d0 / 64) * C::kTile + key * 128 +
-                             ((((d0 % 64) / 8) ^ (key & 7)) << 4);
-        // transposed row j8: channel d0 + j8, keys key0 .. key0 + 7 (slab key0 / 64)
-        const int d = d0 + j8;
-        const uint32_t dst = sVt + (key0 / 64) * C::kVtSlab + d * 128 +
-                             ((((key0 % 64) / 8) ^ (d & 7)) << 4);
-        uint32_t r[4];
-        ldmatrix_x4_trans(src, r);
-        stmatrix_x4(dst, r);
-      }
-    }
-    fence_proxy_async_smem();
 
     // Scores -> probabilities (this thread: query row tid).
     ok = ok && mbar_wait(bar_s, ph, abort_flag, tmo);
@@ -333,12 +307,12 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
     // O_block = P V
     if (ok && tid == 0) {
       tc_fence_after();
-      const uint32_t idesc = idesc_bf16_f32(128, HD);
+      const uint32_t idesc = idesc_bf16_f32(128, HD) | (1u << 16);  // B (V) MN-major
       for (int ks = 0; ks < 2; ++ks)
 #pragma unroll
         for (int k = 0; k < 4; ++k)
           umma_bf16(t_o, sdesc_kmajor_sw128(sP + ks * C::kTile + 32u * k),
-                    sdesc_kmajor_sw128(sVt + ks * C::kVtSlab + 32u * k), idesc,
+                    sdesc_mnmajor_sw128(sV(st) + (ks * 64 + k * 16) * 128, C::kTile), idesc,
                     (ks | k) != 0 ? 1u : 0u);
       umma_commit(bar_o);
     }
