@@ -50,24 +50,26 @@ struct AttnParams {
 // wait gave up); read and cleared by dv_text_attention_status.
 __device__ int g_attn_status;
 
-template <int HD>
+// NST = 2: two stages of [K | V] (the next block loads during this one), one CTA per SM.
+// NST = 1: one stage, small enough for two CTAs per SM; used when that allows more key splits.
+template <int HD, int NST>
 struct AttnCfg {
   static constexpr int kSlabs = HD / 64;
   static constexpr int kTile = 128 * 128;        // 128 rows x 64 bf16 (one 128-byte-swizzled slab)
   static constexpr int kKV = kSlabs * kTile;     // one K or V tile of 128 keys
   static constexpr int kOffQ = 0;
-  static constexpr int kOffStage = kOffQ + kKV;  // two stages of [K | V]
+  static constexpr int kOffStage = kOffQ + kKV;  // NST stages of [K | V]
   static constexpr int kStage = 2 * kKV;
   // P (2 key slabs of [128 rows][64 keys]) takes the K slot of the current stage when that is
   // large enough (HD = 128): K is dead once the score MMA has completed.
   static constexpr bool kPInK = kKV >= 2 * kTile;
-  static constexpr int kOffP = kOffStage + 2 * kStage;
+  static constexpr int kOffP = kOffStage + NST * kStage;
   static constexpr int kEnd = kOffP + (kPInK ? 0 : 2 * kTile);
   static constexpr int kPitch = HD + 4;                   // floats per partial output row
   static constexpr int kPartBytes = 128 * kPitch * 4;
   static constexpr int kMisc = 2048;                      // barriers, m, l, key end
   static constexpr int kSmemBytes = kEnd + kMisc + 1024;
-  static_assert(kPartBytes <= 2 * kStage, "partial outputs reuse the stages");
+  static_assert(kPartBytes <= kKV + NST * kStage, "partial outputs reuse Q and the stages");
   static_assert(kKV % 1024 == 0, "tiles stay 1024-byte aligned");
   static_assert(kSmemBytes <= 232448, "shared memory of one CTA");
 };
@@ -128,11 +130,11 @@ __device__ __forceinline__ bool wait_bounded(uint32_t bar, uint32_t parity, uint
   return mbar_wait(bar, parity, &never, timeout_ns);
 }
 
-template <int HD>
+template <int HD, int NST>
 __global__ void __launch_bounds__(kAttnThreads, 1)
     dv_attn_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
                    const __grid_constant__ CUtensorMap tmV, const __grid_constant__ AttnParams p) {
-  using C = AttnCfg<HD>;
+  using C = AttnCfg<HD, NST>;
   extern __shared__ uint8_t smem_raw[];
   const uint32_t raw = smem_addr(smem_raw);
   const uint32_t base = (raw + 1023u) & ~1023u;
@@ -148,7 +150,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
   int* key_end = reinterpret_cast<int*>(tmem_slot + 2);
   float* part_m = reinterpret_cast<float*>(base_ptr + C::kEnd + 256);
   float* part_l = part_m + 128;
-  float* part_o = reinterpret_cast<float*>(base_ptr + C::kOffStage);
+  float* part_o = reinterpret_cast<float*>(base_ptr + C::kOffQ);  // after the last MMA
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const uint64_t tmo = p.timeout_ns;
@@ -197,8 +199,8 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
   const int q_row0 = (b * p.Hq + h * p.G) * p.Nt + qb * 128;
   auto sK = [&](int st) { return base + C::kOffStage + st * C::kStage; };
   auto sV = [&](int st) { return base + C::kOffStage + st * C::kStage + C::kKV; };
-  auto load_kv = [&](int j) {  // block kb0 + j into stage j & 1
-    const int st = j & 1, kb = kb0 + j;
+  auto load_kv = [&](int j) {  // block kb0 + j into stage j % NST
+    const int st = j % NST, kb = kb0 + j;
     mbar_arrive_expect_tx(bar_k(st), C::kKV);
     for (int ds = 0; ds < C::kSlabs; ++ds)
       tma_load_4d(sK(st) + ds * C::kTile, &tmK, bar_k(st), ds * 64, h, kb * kKeyBlock, b);
@@ -223,15 +225,18 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
 
   bool ok = true;
   for (int j = 0; j < n_mine && ok; ++j) {
-    const int st = j & 1, kb = kb0 + j;
-    const uint32_t sph = static_cast<uint32_t>(j >> 1) & 1u;  // phase of this stage's barriers
+    const int st = j % NST, kb = kb0 + j;
+    const uint32_t sph = static_cast<uint32_t>(j / NST) & 1u;  // phase of this stage's barriers
     const uint32_t ph = static_cast<uint32_t>(j) & 1u;        // phase of bar_s / bar_o
     const uint32_t sP = C::kPInK ? sK(st) : base + C::kOffP;
     if (warp == 0) {
       if (lane == 0) {
-        if (j + 1 < n_mine) {  // the other stage was freed by the previous block
+        if (NST == 2 && j + 1 < n_mine) {  // the other stage was freed by the previous block
           load_kv(j + 1);
           last_issued = j + 1;
+        } else if (NST == 1 && j > 0) {  // the one stage was freed when block j - 1 ended
+          load_kv(j);
+          last_issued = j;
         }
         // S = Q K^T
         if (mbar_wait(bar_q, 0, abort_flag, tmo) && mbar_wait(bar_k(st), sph, abort_flag, tmo)) {
@@ -336,10 +341,10 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
   if (!ok && tid == 0) {
     // Let the copies in flight (the last block issued on each stage) land and every issued MMA
     // finish before the memory is reused; each wait targets its stage's latest phase.
-    for (int jj = last_issued; jj >= 0 && jj >= last_issued - 1; --jj) {
-      const uint32_t sp = static_cast<uint32_t>(jj >> 1) & 1u;
-      wait_bounded(bar_k(jj & 1), sp, tmo);
-      wait_bounded(bar_v(jj & 1), sp, tmo);
+    for (int jj = last_issued; jj >= 0 && jj > last_issued - NST; --jj) {
+      const uint32_t sp = static_cast<uint32_t>(jj / NST) & 1u;
+      wait_bounded(bar_k(jj % NST), sp, tmo);
+      wait_bounded(bar_v(jj % NST), sp, tmo);
     }
     if (last_issued >= 0) wait_bounded(bar_q, 0, tmo);
     umma_commit(bar_drain);
@@ -484,11 +489,11 @@ int num_sms_of_device() {
   return sms[dev];
 }
 
-template <int HD>
+template <int HD, int NST>
 cudaError_t launch_attn(int splits, int units, const CUtensorMap& q, const CUtensorMap& k,
                         const CUtensorMap& v, const AttnParams& p, cudaStream_t stream) {
-  using C = AttnCfg<HD>;
-  auto kern = dv_attn_kernel<HD>;
+  using C = AttnCfg<HD, NST>;
+  auto kern = dv_attn_kernel<HD, NST>;
   static bool attr_set[64] = {};  // the shared-memory opt-in, once per device
   int dev = 0;
   cudaError_t err = cudaGetDevice(&dev);
@@ -587,15 +592,26 @@ extern "C" int dv_text_attention(const void* q, int batch, int n_q_heads, int n_
   const long long units = static_cast<long long>(batch) * n_kv_heads * p.q_blocks;
   if (units > (1LL << 30)) return DV_ERR_UNSUPPORTED_SHAPE;
   const int blocks_max = (max_keys + kKeyBlock - 1) / kKeyBlock;
+  // Key splits (cluster size): as many as the key blocks allow while the CTAs fit in one wave,
+  // with two stages and one CTA per SM, or with one stage and two CTAs per SM when that
+  // allows more splits (each CTA then has few blocks, so losing the prefetch costs little).
   const int sms = num_sms_of_device();
-  int splits = 1;
-  for (int s : {2, 4, 8})
-    if (s <= blocks_max && units * s <= sms) splits = s;
-  cudaError_t err = head_dim == 128
-                        ? launch_attn<128>(splits, static_cast<int>(units), tq, tk, tv, p,
-                                           static_cast<cudaStream_t>(stream))
-                        : launch_attn<64>(splits, static_cast<int>(units), tq, tk, tv, p,
-                                          static_cast<cudaStream_t>(stream));
+  int split2 = 1, split1 = 1;
+  for (int s : {2, 4, 8}) {
+    if (s <= blocks_max && units * s <= sms) split2 = s;
+    if (s <= blocks_max && units * s <= 2LL * sms) split1 = s;
+  }
+  const bool one_stage = split1 > split2;
+  const int splits = one_stage ? split1 : split2;
+  const cudaStream_t cs = static_cast<cudaStream_t>(stream);
+  const int u = static_cast<int>(units);
+  cudaError_t err;
+  if (head_dim == 128)
+    err = one_stage ? launch_attn<128, 1>(splits, u, tq, tk, tv, p, cs)
+                    : launch_attn<128, 2>(splits, u, tq, tk, tv, p, cs);
+  else
+    err = one_stage ? launch_attn<64, 1>(splits, u, tq, tk, tv, p, cs)
+                    : launch_attn<64, 2>(splits, u, tq, tk, tv, p, cs);
   return err == cudaSuccess ? DV_OK : DV_ERR_CUDA;
 }
 
