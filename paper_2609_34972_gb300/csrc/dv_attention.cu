@@ -130,6 +130,62 @@ __device__ __forceinline__ bool wait_bounded(uint32_t bar, uint32_t parity, uint
   return mbar_wait(bar, parity, &never, timeout_ns);
 }
 
+// Combine of the S key runs of a cluster: CTA `split` takes rows [split * rows, (split + 1) *
+// rows), S threads per row, each HD / (4 S) float4 of it. Every remote load (the S partial
+// maxima and sums, then all S partial output pieces of the thread) is issued before any value
+// is used, so the distributed-shared-memory latency is paid twice, not once per piece; the S
+// partials are summed in the fixed order 0 .. S-1.
+template <int HD, int S>
+__device__ __forceinline__ void combine_rows(const float* part_o, const float* part_m,
+                                             const float* part_l, int pitch, int split, int qb,
+                                             int h, int b, const AttnParams& p) {
+  constexpr int kRows = 128 / S, kTpr = kAttnThreads / kRows, kPer = HD / 4 / kTpr;
+  const int tid = threadIdx.x;
+  const int rr = split * kRows + tid / kTpr, c4_0 = (tid % kTpr) * kPer;
+  const int ii = qb * 128 + rr;
+  if (ii >= p.rows_per_group) return;
+  float ms[S], ls[S], w[S];
+#pragma unroll
+  for (int s = 0; s < S; ++s) {
+    ms[s] = ld_cluster_f32(map_to_rank(smem_addr(part_m + rr), static_cast<uint32_t>(s)));
+    ls[s] = ld_cluster_f32(map_to_rank(smem_addr(part_l + rr), static_cast<uint32_t>(s)));
+  }
+  const uint32_t row_addr = smem_addr(part_o + rr * pitch + c4_0 * 4);
+  float4 v[kPer * S];
+#pragma unroll
+  for (int c = 0; c < kPer; ++c)
+#pragma unroll
+    for (int s = 0; s < S; ++s)
+      v[c * S + s] = ld_cluster_f4(map_to_rank(row_addr + 16u * c, static_cast<uint32_t>(s)));
+  float M = -INFINITY;
+#pragma unroll
+  for (int s = 0; s < S; ++s) M = fmaxf(M, ms[s]);
+  float L = 0.0f;
+#pragma unroll
+  for (int s = 0; s < S; ++s) {
+    w[s] = ms[s] != -INFINITY ? exp2f(ms[s] - M) : 0.0f;
+    L = fmaf(w[s], ls[s], L);
+  }
+  const float inv = L > 0.0f ? 1.0f / L : 0.0f;
+  const int hq = h * p.G + ii / p.Nt, t = ii % p.Nt;
+  uint16_t* orow = p.out + ((static_cast<size_t>(b) * p.Hq + hq) * p.Nt + t) * HD;
+#pragma unroll
+  for (int c = 0; c < kPer; ++c) {
+    float4 acc = make_float4(0.0f, 0.0f, 0.0f, 0.0f);
+#pragma unroll
+    for (int s = 0; s < S; ++s) {
+      acc.x = fmaf(w[s], v[c * S + s].x, acc.x);
+      acc.y = fmaf(w[s], v[c * S + s].y, acc.y);
+      acc.z = fmaf(w[s], v[c * S + s].z, acc.z);
+      acc.w = fmaf(w[s], v[c * S + s].w, acc.w);
+    }
+    uint2 out;
+    out.x = pack_bf16x2(acc.x * inv, acc.y * inv);
+    out.y = pack_bf16x2(acc.z * inv, acc.w * inv);
+    *reinterpret_cast<uint2*>(orow + (c4_0 + c) * 4) = out;
+  }
+}
+
 template <int HD, int NST>
 __global__ void __launch_bounds__(kAttnThreads, 1)
     dv_attn_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
@@ -363,59 +419,11 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
   }
   __syncwarp();
   cluster_sync();
-  {
-    // CTA `split` combines rows [split * rows, (split + 1) * rows); tpr threads share a row.
-    // All remote loads of a step are issued before their values are used, so they overlap.
-    constexpr int kV4 = HD / 4;
-    const int rows = 128 / S, tpr = kAttnThreads / rows, per = kV4 / tpr;
-    const int rr = split * rows + tid / tpr, c4_0 = (tid % tpr) * per;
-    const int ii = qb * 128 + rr;
-    if (ii < p.rows_per_group) {
-      float ms[8], ls[8], w[8];
-#pragma unroll
-      for (int s = 0; s < 8; ++s) {
-        if (s < S) {
-          ms[s] = ld_cluster_f32(map_to_rank(smem_addr(part_m + rr), static_cast<uint32_t>(s)));
-          ls[s] = ld_cluster_f32(map_to_rank(smem_addr(part_l + rr), static_cast<uint32_t>(s)));
-        }
-      }
-      float M = -INFINITY;
-#pragma unroll
-      for (int s = 0; s < 8; ++s)
-        if (s < S) M = fmaxf(M, ms[s]);
-      float L = 0.0f;
-#pragma unroll
-      for (int s = 0; s < 8; ++s) {
-        w[s] = (s < S && ms[s] != -INFINITY) ? exp2f(ms[s] - M) : 0.0f;
-        if (s < S) L = fmaf(w[s], ls[s], L);
-      }
-      const float inv = L > 0.0f ? 1.0f / L : 0.0f;
-      const int hq = h * p.G + ii / p.Nt, t = ii % p.Nt;
-      uint16_t* orow = p.out + ((static_cast<size_t>(b) * p.Hq + hq) * p.Nt + t) * HD;
-#pragma unroll 1
-      for (int c = 0; c < per; ++c) {
-        const int c4 = c4_0 + c;
-        const uint32_t laddr = smem_addr(part_o + rr * C::kPitch + c4 * 4);
-        float4 v[8];
-#pragma unroll
-        for (int s = 0; s < 8; ++s)
-          if (s < S) v[s] = ld_cluster_f4(map_to_rank(laddr, static_cast<uint32_t>(s)));
-        float4 acc = make_float4(0.0f, 0.0f, 0.0f, 0.0f);
-#pragma unroll
-        for (int s = 0; s < 8; ++s) {
-          if (s < S) {
-            acc.x = fmaf(w[s], v[s].x, acc.x);
-            acc.y = fmaf(w[s], v[s].y, acc.y);
-            acc.z = fmaf(w[s], v[s].z, acc.z);
-            acc.w = fmaf(w[s], v[s].w, acc.w);
-          }
-        }
-        uint2 out;
-        out.x = pack_bf16x2(acc.x * inv, acc.y * inv);
-        out.y = pack_bf16x2(acc.z * inv, acc.w * inv);
-        *reinterpret_cast<uint2*>(orow + c4 * 4) = out;
-      }
-    }
+  switch (S) {  // the cluster size: 1, 2, 4 or 8
+    case 1: combine_rows<HD, 1>(part_o, part_m, part_l, C::kPitch, split, qb, h, b, p); break;
+    case 2: combine_rows<HD, 2>(part_o, part_m, part_l, C::kPitch, split, qb, h, b, p); break;
+    case 4: combine_rows<HD, 4>(part_o, part_m, part_l, C::kPitch, split, qb, h, b, p); break;
+    default: combine_rows<HD, 8>(part_o, part_m, part_l, C::kPitch, split, qb, h, b, p); break;
   }
   __syncwarp();
   cluster_sync();
