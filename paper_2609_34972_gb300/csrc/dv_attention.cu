@@ -17,10 +17,11 @@
 //      writes the row's probabilities as bf16 into the A tile of the second MMA;
 //   5. one thread issues P V (N = head_dim) into TMEM; each thread rescales its fp32 output row
 //      (registers) by exp2(m_old - m_new) and adds the block.
-// The partial (O, m, l) of each CTA then go to shared memory, and after a cluster barrier CTA s
-// combines rows [s * 128 / S, (s + 1) * 128 / S) over the S partials through distributed
+// Each thread then stores its partial (O, m, l) row straight into the shared memory of the CTA
+// that combines that row (distributed-shared-memory stores, no reply awaited); after one cluster
+// barrier CTA s combines rows [s * 128 / S, (s + 1) * 128 / S) over the S partials from its own
 // shared memory, in the fixed order 0..S-1, and stores bf16 rows. Every wait is bounded; a CTA
-// that gives up still passes both cluster barriers and flags the status word.
+// that gives up still passes the cluster barriers and flags the status word.
 #include <cmath>
 #include <mutex>
 
@@ -65,11 +66,15 @@ struct AttnCfg {
   static constexpr bool kPInK = kKV >= 2 * kTile;
   static constexpr int kOffP = kOffStage + NST * kStage;
   static constexpr int kEnd = kOffP + (kPInK ? 0 : 2 * kTile);
-  static constexpr int kPitch = HD + 4;                   // floats per partial output row
-  static constexpr int kPartBytes = 128 * kPitch * 4;
   static constexpr int kMisc = 2048;                      // barriers, m, l, key end
-  static constexpr int kSmemBytes = kEnd + kMisc + 1024;
-  static_assert(kPartBytes <= kKV + NST * kStage, "partial outputs reuse Q and the stages");
+  // Partial outputs received from the cluster: 128 rows of HD fp32 (16-byte chunks swizzled by
+  // the row, no padding). With two stages they get a region of their own, so peers may write
+  // them while this CTA still computes; the one-stage variant reuses Q and its stage.
+  static constexpr int kRecvBytes = 128 * HD * 4;
+  static constexpr bool kRecvOwn = NST == 2;
+  static constexpr int kOffRecv = kRecvOwn ? kEnd + kMisc : kOffQ;
+  static constexpr int kSmemBytes = kEnd + kMisc + (kRecvOwn ? kRecvBytes : 0) + 1024;
+  static_assert(kRecvOwn || kRecvBytes <= kKV + NST * kStage, "partials reuse Q and the stage");
   static_assert(kKV % 1024 == 0, "tiles stay 1024-byte aligned");
   static_assert(kSmemBytes <= 232448, "shared memory of one CTA");
 };
@@ -110,53 +115,79 @@ __device__ __forceinline__ uint32_t cluster_size() {
   return r;
 }
 
-__device__ __forceinline__ float ld_cluster_f32(uint32_t caddr) {
-  float v;
-  asm volatile("ld.shared::cluster.f32 %0, [%1];" : "=f"(v) : "r"(caddr) : "memory");
-  return v;
-}
-
-__device__ __forceinline__ float4 ld_cluster_f4(uint32_t caddr) {
-  float4 v;
-  asm volatile("ld.shared::cluster.v4.f32 {%0, %1, %2, %3}, [%4];"
-               : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w)
-               : "r"(caddr)
-               : "memory");
-  return v;
-}
-
 __device__ __forceinline__ bool wait_bounded(uint32_t bar, uint32_t parity, uint64_t timeout_ns) {
   int never = 0;
   return mbar_wait(bar, parity, &never, timeout_ns);
 }
 
-// Combine of the S key runs of a cluster: CTA `split` takes rows [split * rows, (split + 1) *
-// rows), S threads per row, each HD / (4 S) float4 of it. Every remote load (the S partial
-// maxima and sums, then all S partial output pieces of the thread) is issued before any value
-// is used, so the distributed-shared-memory latency is paid twice, not once per piece; the S
-// partials are summed in the fixed order 0 .. S-1.
+// Partial rows travel between the CTAs of a cluster as fp32 rows of HD / 4 16-byte chunks,
+// chunk c of row R stored at chunk position c ^ rev3(R mod 8) (rev3 reverses 3 bits). Eight
+// consecutive rows writing one chunk, and the combine's reads (S threads of a row on
+// consecutive chunks, 8 / S rows per quarter warp), then touch 8 distinct bank groups.
+__device__ __forceinline__ uint32_t chunk_swizzle(int R) {
+  return static_cast<uint32_t>(((R & 1) << 2) | (R & 2) | ((R >> 2) & 1));
+}
+
+__device__ __forceinline__ void st_cluster_f4(uint32_t caddr, float a, float b, float c, float d) {
+  asm volatile("st.shared::cluster.v4.f32 [%0], {%1, %2, %3, %4};" ::"r"(caddr), "f"(a), "f"(b),
+               "f"(c), "f"(d)
+               : "memory");
+}
+
+__device__ __forceinline__ void st_cluster_f32(uint32_t caddr, float v) {
+  asm volatile("st.shared::cluster.f32 [%0], %1;" ::"r"(caddr), "f"(v) : "memory");
+}
+
+// Thread `tid` holds query row tid of this CTA's key run: (o, m, l). Row tid is combined by CTA
+// d = tid / (128 / S); it goes into d's receive rows at R = split * 128 / S + tid mod (128 / S),
+// by distributed-shared-memory stores (local stores when d is this CTA). The stores need no
+// reply; the cluster barrier that follows makes them visible.
+template <int HD>
+__device__ __forceinline__ void push_partial(const float* o, float m_run, float l_run,
+                                             uint32_t recv, uint32_t recv_m, uint32_t recv_l,
+                                             int split, int S) {
+  const int tid = threadIdx.x, rows = 128 / S;
+  const int d = tid / rows, R = split * rows + tid % rows;
+  const uint32_t sw = chunk_swizzle(R);
+  const uint32_t row = recv + static_cast<uint32_t>(R) * (HD * 4);
+  if (d == split) {
+#pragma unroll
+    for (int c = 0; c < HD / 4; ++c) {
+      float4* dst = reinterpret_cast<float4*>(__cvta_shared_to_generic(row + ((c ^ sw) << 4)));
+      *dst = make_float4(o[4 * c], o[4 * c + 1], o[4 * c + 2], o[4 * c + 3]);
+    }
+    *reinterpret_cast<float*>(__cvta_shared_to_generic(recv_m + 4u * R)) = m_run;
+    *reinterpret_cast<float*>(__cvta_shared_to_generic(recv_l + 4u * R)) = l_run;
+  } else {
+    const uint32_t rank = static_cast<uint32_t>(d);
+    const uint32_t crow = map_to_rank(row, rank);
+#pragma unroll
+    for (int c = 0; c < HD / 4; ++c)
+      st_cluster_f4(crow + ((c ^ sw) << 4), o[4 * c], o[4 * c + 1], o[4 * c + 2], o[4 * c + 3]);
+    st_cluster_f32(map_to_rank(recv_m + 4u * R, rank), m_run);
+    st_cluster_f32(map_to_rank(recv_l + 4u * R, rank), l_run);
+  }
+}
+
+// Combine of the S key runs of a cluster from this CTA's receive rows: CTA `split` owns query
+// rows [split * 128 / S, (split + 1) * 128 / S); S threads per row, thread j taking chunks j,
+// j + S, j + 2 S, ...; the S partials are summed in the fixed order 0 .. S-1.
 template <int HD, int S>
-__device__ __forceinline__ void combine_rows(const float* part_o, const float* part_m,
-                                             const float* part_l, int pitch, int split, int qb,
-                                             int h, int b, const AttnParams& p) {
+__device__ __forceinline__ void combine_rows(uint32_t recv, const float* recv_m,
+                                             const float* recv_l, int split, int qb, int h, int b,
+                                             const AttnParams& p) {
   constexpr int kRows = 128 / S, kTpr = kAttnThreads / kRows, kPer = HD / 4 / kTpr;
   const int tid = threadIdx.x;
-  const int rr = split * kRows + tid / kTpr, c4_0 = (tid % kTpr) * kPer;
-  const int ii = qb * 128 + rr;
+  const int rr = tid / kTpr, j = tid % kTpr;
+  const int ii = qb * 128 + split * kRows + rr;
   if (ii >= p.rows_per_group) return;
+  const uint32_t sw = chunk_swizzle(rr);  // rows R = s * kRows + rr share rr mod 8
   float ms[S], ls[S], w[S];
 #pragma unroll
   for (int s = 0; s < S; ++s) {
-    ms[s] = ld_cluster_f32(map_to_rank(smem_addr(part_m + rr), static_cast<uint32_t>(s)));
-    ls[s] = ld_cluster_f32(map_to_rank(smem_addr(part_l + rr), static_cast<uint32_t>(s)));
+    ms[s] = recv_m[s * kRows + rr];
+    ls[s] = recv_l[s * kRows + rr];
   }
-  const uint32_t row_addr = smem_addr(part_o + rr * pitch + c4_0 * 4);
-  float4 v[kPer * S];
-#pragma unroll
-  for (int c = 0; c < kPer; ++c)
-#pragma unroll
-    for (int s = 0; s < S; ++s)
-      v[c * S + s] = ld_cluster_f4(map_to_rank(row_addr + 16u * c, static_cast<uint32_t>(s)));
   float M = -INFINITY;
 #pragma unroll
   for (int s = 0; s < S; ++s) M = fmaxf(M, ms[s]);
@@ -170,19 +201,23 @@ __device__ __forceinline__ void combine_rows(const float* part_o, const float* p
   const int hq = h * p.G + ii / p.Nt, t = ii % p.Nt;
   uint16_t* orow = p.out + ((static_cast<size_t>(b) * p.Hq + hq) * p.Nt + t) * HD;
 #pragma unroll
-  for (int c = 0; c < kPer; ++c) {
+  for (int i = 0; i < kPer; ++i) {
+    const int c = i * kTpr + j;
     float4 acc = make_float4(0.0f, 0.0f, 0.0f, 0.0f);
 #pragma unroll
     for (int s = 0; s < S; ++s) {
-      acc.x = fmaf(w[s], v[c * S + s].x, acc.x);
-      acc.y = fmaf(w[s], v[c * S + s].y, acc.y);
-      acc.z = fmaf(w[s], v[c * S + s].z, acc.z);
-      acc.w = fmaf(w[s], v[c * S + s].w, acc.w);
+      const uint32_t a = recv + static_cast<uint32_t>(s * kRows + rr) * (HD * 4) +
+                         ((static_cast<uint32_t>(c) ^ sw) << 4);
+      const float4 v = *reinterpret_cast<const float4*>(__cvta_shared_to_generic(a));
+      acc.x = fmaf(w[s], v.x, acc.x);
+      acc.y = fmaf(w[s], v.y, acc.y);
+      acc.z = fmaf(w[s], v.z, acc.z);
+      acc.w = fmaf(w[s], v.w, acc.w);
     }
     uint2 out;
     out.x = pack_bf16x2(acc.x * inv, acc.y * inv);
     out.y = pack_bf16x2(acc.z * inv, acc.w * inv);
-    *reinterpret_cast<uint2*>(orow + (c4_0 + c) * 4) = out;
+    *reinterpret_cast<uint2*>(orow + c * 4) = out;
   }
 }
 
@@ -204,15 +239,18 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 8);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
   int* key_end = reinterpret_cast<int*>(tmem_slot + 2);
-  float* part_m = reinterpret_cast<float*>(base_ptr + C::kEnd + 256);
-  float* part_l = part_m + 128;
-  float* part_o = reinterpret_cast<float*>(base_ptr + C::kOffQ);  // after the last MMA
+  float* recv_m = reinterpret_cast<float*>(base_ptr + C::kEnd + 256);
+  float* recv_l = recv_m + 128;
+  const uint32_t recv = base + C::kOffRecv;
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const uint64_t tmo = p.timeout_ns;
   const int split = static_cast<int>(cluster_ctarank());
   const int S = static_cast<int>(cluster_size());
   const int unit = static_cast<int>(cluster_id_x());
+  // Peers write into this CTA's receive rows as soon as their own key runs end; this arrival
+  // (waited for before those writes) tells them that this CTA has started.
+  if (C::kRecvOwn) asm volatile("barrier.cluster.arrive.relaxed.aligned;" ::: "memory");
   const int qb = unit % p.q_blocks;
   const int h = (unit / p.q_blocks) % p.Hkv;
   const int b = unit / (p.q_blocks * p.Hkv);
@@ -408,25 +446,22 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
   }
   __syncthreads();
 
-  // Partial (O, m, l) of this CTA's key run -> shared memory, then the cluster combines.
-  {
-    float4* dst = reinterpret_cast<float4*>(part_o + tid * C::kPitch);
-#pragma unroll
-    for (int c = 0; c < HD / 4; ++c)
-      dst[c] = make_float4(o[4 * c], o[4 * c + 1], o[4 * c + 2], o[4 * c + 3]);
-    part_m[tid] = m_run;
-    part_l[tid] = l_run;
-  }
+  // Partial (O, m, l) of this CTA's key run -> the receive rows of the CTA that combines each
+  // row; after one cluster barrier every CTA combines from its own shared memory. The one-stage
+  // variant receives into Q and its stage, free only once every key run of the cluster ended.
+  if (C::kRecvOwn)
+    asm volatile("barrier.cluster.wait.aligned;" ::: "memory");
+  else
+    cluster_sync();
+  push_partial<HD>(o, m_run, l_run, recv, smem_addr(recv_m), smem_addr(recv_l), split, S);
   __syncwarp();
   cluster_sync();
   switch (S) {  // the cluster size: 1, 2, 4 or 8
-    case 1: combine_rows<HD, 1>(part_o, part_m, part_l, C::kPitch, split, qb, h, b, p); break;
-    case 2: combine_rows<HD, 2>(part_o, part_m, part_l, C::kPitch, split, qb, h, b, p); break;
-    case 4: combine_rows<HD, 4>(part_o, part_m, part_l, C::kPitch, split, qb, h, b, p); break;
-    default: combine_rows<HD, 8>(part_o, part_m, part_l, C::kPitch, split, qb, h, b, p); break;
+    case 1: combine_rows<HD, 1>(recv, recv_m, recv_l, split, qb, h, b, p); break;
+    case 2: combine_rows<HD, 2>(recv, recv_m, recv_l, split, qb, h, b, p); break;
+    case 4: combine_rows<HD, 4>(recv, recv_m, recv_l, split, qb, h, b, p); break;
+    default: combine_rows<HD, 8>(recv, recv_m, recv_l, split, qb, h, b, p); break;
   }
-  __syncwarp();
-  cluster_sync();
 
   if (warp == 0) {
     tc_fence_after();
