@@ -127,17 +127,18 @@ def test_attention_llava15_full_layer():
     _run_case(cfg, n_sys=35, n_text=64, n_q_heads=32, layer=5, label="llava15 layer")
 
 
-@pytest.mark.parametrize("hd,hq,hkv,nt", [(128, 32, 32, 64), (128, 28, 4, 50), (64, 8, 2, 33)])
-def test_attention_kernel_on_exact_inputs(hd, hq, hkv, nt):
+def _exact_case(hd, B, hq, hkv, nt, n_keys, S, seed, label):
     # Every slot holds synthetic bf16 K/V (no build): the oracle reads the same values.
     import torch
     import paper_2609_34972_gb300 as dv
-    B, L, S_used, S = 2, 2, 700, 768
-    kb = synth.normal_bf16(90 + hd, 30, (L, B, S, hkv, hd), 0.0, 1.0)
-    vb = synth.normal_bf16(90 + hd, 31, (L, B, S, hkv, hd), 0.0, 1.0)
-    qb = synth.normal_bf16(90 + hd, 32, (B, hq, nt, hd), 0.0, 1.0)
-    q_slot = np.stack([S_used - nt + np.arange(nt), 300 + 7 * np.arange(nt)]).astype(np.int32)
-    n_keys = np.array([S_used, 650], dtype=np.int32)
+    L = 2
+    kb = synth.normal_bf16(seed, 30, (L, B, S, hkv, hd), 0.0, 1.0)
+    vb = synth.normal_bf16(seed, 31, (L, B, S, hkv, hd), 0.0, 1.0)
+    qb = synth.normal_bf16(seed, 32, (B, hq, nt, hd), 0.0, 1.0)
+    n_keys = np.asarray(n_keys, dtype=np.int32)
+    # even batch rows: the last nt slots; odd rows: strided slots (some past n_keys)
+    q_slot = np.stack([n_keys[b] - nt + np.arange(nt) if b % 2 == 0 else 300 + 7 * np.arange(nt)
+                       for b in range(B)]).astype(np.int32)
     scale = 1.0 / np.sqrt(hd)
     k = gu.torch_bf16(kb, "cuda")
     v = gu.torch_bf16(vb, "cuda")
@@ -149,4 +150,27 @@ def test_attention_kernel_on_exact_inputs(hd, hq, hkv, nt):
     want = oracle.text_attention(f(qb), f(kb[1]), f(vb[1]), n_keys, q_slot, scale)
     g = out.double().cpu().numpy().reshape(-1, 1, hd)
     o = want.reshape(-1, 1, hd)
-    gu.assert_parity(g, g, o, o, hd, f"attention kernel hd{hd} hq{hq}/{hkv}")
+    gu.assert_parity(g, g, o, o, hd, label)
+
+
+@pytest.mark.parametrize("hd,hq,hkv,nt", [(128, 32, 32, 64), (128, 28, 4, 50), (64, 8, 2, 33)])
+def test_attention_kernel_on_exact_inputs(hd, hq, hkv, nt):
+    _exact_case(hd, 2, hq, hkv, nt, [700, 650], 768, 90 + hd, f"attention kernel hd{hd} hq{hq}/{hkv}")
+
+
+# Launch shapes that reach every kernel variant and cluster size the launcher picks (clusters =
+# batch x kv heads x 128-row query blocks, cluster size S = the largest of 2, 4, 8 within the key
+# blocks and one CTA per SM (two stages) or two per SM (one stage) on 152 SMs):
+#   two stages, S = 8: 2 clusters, 9 key blocks; one stage, S = 8: 24 clusters;
+#   one stage, S = 2: 80 clusters, 3 key blocks; one stage, S = 4 at head_dim 64: 64 clusters.
+@pytest.mark.parametrize("hd,B,hq,hkv,nt,n_keys,S", [
+    (128, 1, 8, 2, 30, [1100], 1152),
+    (64, 1, 8, 2, 30, [1100], 1152),
+    (128, 2, 12, 12, 20, [1000, 977], 1024),
+    (64, 2, 12, 12, 20, [1000, 977], 1024),
+    (128, 4, 20, 20, 16, [300, 290, 300, 257], 320),
+    (64, 2, 32, 32, 64, [700, 650], 768),
+])
+def test_attention_every_cluster_shape(hd, B, hq, hkv, nt, n_keys, S):
+    _exact_case(hd, B, hq, hkv, nt, n_keys, S, 500 + hd + B + hq,
+                f"attention hd{hd} B{B} hq{hq}/{hkv} nt{nt}")
