@@ -12,11 +12,12 @@
 //   2. one thread issues S = Q K^T (M = 128 rows, N = 128 keys, K = head_dim) into TMEM;
 //   3. the P V MMA reads V as it lies ([keys][channels] rows, an MN-major B operand), so V needs
 //      no transpose;
-//   4. each thread owns one query row: it reads its scores from TMEM twice (the block maximum,
-//      then exp2 of the masked, scaled scores), keeps the running maximum m and sum l, and
-//      writes the row's probabilities as bf16 into the A tile of the second MMA;
-//   5. one thread issues P V (N = head_dim) into TMEM; each thread rescales its fp32 output row
-//      (registers) by exp2(m_old - m_new) and adds the block.
+//   4. each thread owns one query row: it reads the row's 128 scores from TMEM at once, keeps
+//      the running maximum m and sum l, and writes the row's probabilities exp2(scaled score -
+//      m) as bf16 into the A tile of the second MMA;
+//   5. one thread issues O += P V (N = head_dim): O stays in TMEM over the CTA's key run. m is
+//      only moved (and O rescaled in TMEM) when the block maximum exceeds it by more than 2^8,
+//      a bound on the probabilities; O / l is the same for any common reference maximum.
 // Each thread then stores its partial (O, m, l) row straight into the shared memory of the CTA
 // that combines that row (distributed-shared-memory stores, no reply awaited); after one cluster
 // barrier CTA s combines rows [s * 128 / S, (s + 1) * 128 / S) over the S partials from its own
@@ -117,6 +118,51 @@ __device__ __forceinline__ uint32_t cluster_size() {
   uint32_t r;
   asm volatile("mov.u32 %0, %%cluster_nctarank;" : "=r"(r));
   return r;
+}
+
+// Largest growth (base 2) of a row's maximum absorbed without rescaling O: probabilities
+// relative to a stale maximum stay <= 2^8, far inside bf16 and fp32 range.
+constexpr float kRescaleLog2 = 8.0f;
+
+__device__ __forceinline__ float ex2_approx(float x) {  // 2^x (PTX ex2.approx, -inf -> +0)
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+
+__device__ __forceinline__ uint32_t (&chunk32(uint32_t* r, int c))[32] {
+  return *reinterpret_cast<uint32_t(*)[32]>(r + 32 * c);
+}
+
+// Uses of registers loaded by tcgen05.ld stay after tcgen05.wait::ld: the empty statement
+// (ordered after the wait like every volatile asm) redefines them.
+__device__ __forceinline__ void reg_fence32(uint32_t (&r)[32]) {
+  asm volatile(""
+               : "+r"(r[0]), "+r"(r[1]), "+r"(r[2]), "+r"(r[3]), "+r"(r[4]), "+r"(r[5]),
+                 "+r"(r[6]), "+r"(r[7]), "+r"(r[8]), "+r"(r[9]), "+r"(r[10]), "+r"(r[11]),
+                 "+r"(r[12]), "+r"(r[13]), "+r"(r[14]), "+r"(r[15]), "+r"(r[16]), "+r"(r[17]),
+                 "+r"(r[18]), "+r"(r[19]), "+r"(r[20]), "+r"(r[21]), "+r"(r[22]), "+r"(r[23]),
+                 "+r"(r[24]), "+r"(r[25]), "+r"(r[26]), "+r"(r[27]), "+r"(r[28]), "+r"(r[29]),
+                 "+r"(r[30]), "+r"(r[31]));
+}
+
+// Warp-wide registers -> TMEM, the inverse of tmem_ld32 (lane i writes TMEM lane taddr.lane + i).
+__device__ __forceinline__ void tmem_st32(uint32_t taddr, const uint32_t (&r)[32]) {
+  asm volatile(
+      "tcgen05.st.sync.aligned.32x32b.x32.b32 [%0],"
+      " {%1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, %16,"
+      " %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31, %32};" ::"r"(
+          taddr),
+      "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7]),
+      "r"(r[8]), "r"(r[9]), "r"(r[10]), "r"(r[11]), "r"(r[12]), "r"(r[13]), "r"(r[14]),
+      "r"(r[15]), "r"(r[16]), "r"(r[17]), "r"(r[18]), "r"(r[19]), "r"(r[20]), "r"(r[21]),
+      "r"(r[22]), "r"(r[23]), "r"(r[24]), "r"(r[25]), "r"(r[26]), "r"(r[27]), "r"(r[28]),
+      "r"(r[29]), "r"(r[30]), "r"(r[31])
+      : "memory");
+}
+
+__device__ __forceinline__ void tmem_st_wait() {
+  asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
 }
 
 __device__ __forceinline__ bool wait_bounded(uint32_t bar, uint32_t parity, uint64_t timeout_ns) {
@@ -373,9 +419,6 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
       tma_load_4d(sV(st) + ds * C::kTile, &tmV, bar_v(st), ds * 64, h, kb * kKeyBlock, b);
   };
 
-  float o[HD];
-#pragma unroll
-  for (int d = 0; d < HD; ++d) o[d] = 0.0f;
   float m_run = -INFINITY, l_run = 0.0f;
 
   const int n_mine = kb1 - kb0;
@@ -423,38 +466,63 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
 
     // Scores -> probabilities (this thread: query row tid).
     ok = ok && mbar_wait(bar_s, ph, abort_flag, tmo);
-    float alpha = 1.0f;
     if (__all_sync(0xFFFFFFFFu, ok)) {
       tc_fence_after();
-      const int key_base = kb * kKeyBlock;
-      float mb = -INFINITY;
-#pragma unroll 1
-      for (int c = 0; c < kKeyBlock / 32; ++c) {
-        uint32_t r[32];
-        __syncwarp();
-        tmem_ld32(t_s + lane_base + c * 32, r);
-        tmem_ld_wait();
+      // the row's 128 scores in one TMEM round trip; keys past the row's last slot are masked
+      uint32_t r[kKeyBlock];
 #pragma unroll
-        for (int u = 0; u < 32; ++u)
-          if (key_base + c * 32 + u <= last) mb = fmaxf(mb, __uint_as_float(r[u]) * p.scale_log2);
-      }
+      for (int c = 0; c < kKeyBlock / 32; ++c) tmem_ld32(t_s + lane_base + c * 32, chunk32(r, c));
+      tmem_ld_wait();
+#pragma unroll
+      for (int c = 0; c < kKeyBlock / 32; ++c) reg_fence32(chunk32(r, c));
+      const int n_valid = last - kb * kKeyBlock + 1;
+      float x[kKeyBlock];
+#pragma unroll
+      for (int u = 0; u < kKeyBlock; ++u)
+        x[u] = u < n_valid ? __uint_as_float(r[u]) * p.scale_log2 : -INFINITY;
+      float mx[8];
+#pragma unroll
+      for (int u = 0; u < 8; ++u) mx[u] = x[u];
+#pragma unroll
+      for (int u = 8; u < kKeyBlock; ++u) mx[u % 8] = fmaxf(mx[u % 8], x[u]);
+      const float mb = fmaxf(fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3])),
+                             fmaxf(fmaxf(mx[4], mx[5]), fmaxf(mx[6], mx[7])));
       const float m_new = fmaxf(m_run, mb);
-      alpha = m_new == -INFINITY ? 1.0f : exp2f(m_run - m_new);
-      float lb = 0.0f;
+      // The row keeps its reference maximum while the new scores exceed it by at most
+      // kRescaleLog2 (probabilities stay <= 2^kRescaleLog2); O and l only need the same
+      // reference, so O in TMEM is rescaled only when the maximum grows by more than that.
+      // A row that has seen no key yet (m_run = -inf) has O = 0 and l = 0: it takes the new
+      // maximum with nothing to rescale.
+      float alpha = 1.0f, m_use = m_run;
+      if (m_run == -INFINITY) {
+        m_use = m_new;
+      } else if (m_new > m_run + kRescaleLog2) {
+        alpha = ex2_approx(m_run - m_new);
+        m_use = m_new;
+      }
+      if (__any_sync(0xFFFFFFFFu, alpha != 1.0f)) {  // rows of this warp whose reference moved
 #pragma unroll 1
+        for (int c = 0; c < HD / 32; ++c) {
+          uint32_t q[32];
+          tmem_ld32(t_o + lane_base + c * 32, q);
+          tmem_ld_wait();
+          reg_fence32(q);
+#pragma unroll
+          for (int u = 0; u < 32; ++u) q[u] = __float_as_uint(__uint_as_float(q[u]) * alpha);
+          tmem_st32(t_o + lane_base + c * 32, q);
+        }
+        tmem_st_wait();
+      }
+      const float m_sub = m_use == -INFINITY ? 0.0f : m_use;
+      float lb[4] = {0.0f, 0.0f, 0.0f, 0.0f};
+#pragma unroll
       for (int c = 0; c < kKeyBlock / 32; ++c) {
-        uint32_t r[32];
-        __syncwarp();
-        tmem_ld32(t_s + lane_base + c * 32, r);
-        tmem_ld_wait();
         uint32_t pk[16];
 #pragma unroll
         for (int u = 0; u < 32; u += 2) {
-          const int key = key_base + c * 32 + u;
-          const float p0 = key <= last ? exp2f(__uint_as_float(r[u]) * p.scale_log2 - m_new) : 0.0f;
-          const float p1 =
-              key + 1 <= last ? exp2f(__uint_as_float(r[u + 1]) * p.scale_log2 - m_new) : 0.0f;
-          lb += p0 + p1;
+          const float p0 = ex2_approx(x[c * 32 + u] - m_sub);
+          const float p1 = ex2_approx(x[c * 32 + u + 1] - m_sub);
+          lb[(u / 2) % 4] += p0 + p1;
           pk[u / 2] = pack_bf16x2(p0, p1);
         }
         // keys 32c .. 32c + 31 = 4 chunks of 8 keys in key slab c / 2
@@ -466,14 +534,14 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
               make_uint4(pk[4 * q4], pk[4 * q4 + 1], pk[4 * q4 + 2], pk[4 * q4 + 3]);
         }
       }
-      l_run = alpha * l_run + lb;
-      m_run = m_new;
+      l_run = alpha * l_run + ((lb[0] + lb[1]) + (lb[2] + lb[3]));
+      m_run = m_use;
     }
     fence_proxy_async_smem();
     tc_fence_before();
     ok = __syncthreads_and(ok) != 0;
 
-    // O_block = P V
+    // O (+)= P V in TMEM; the CTA's first block initialises O
     if (ok && tid == 0) {
       tc_fence_after();
       const uint32_t idesc = idesc_bf16_f32(128, HD) | (1u << 16);  // B (V) MN-major
@@ -482,24 +550,29 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
         for (int k = 0; k < 4; ++k)
           umma_bf16(t_o, sdesc_kmajor_sw128(sP + ks * C::kTile + 32u * k),
                     sdesc_mnmajor_sw128(sV(st) + (ks * 64 + k * 16) * 128, C::kTile), idesc,
-                    (ks | k) != 0 ? 1u : 0u);
+                    (j | ks | k) != 0 ? 1u : 0u);
       umma_commit(bar_o);
     }
     ok = ok && mbar_wait(bar_o, ph, abort_flag, tmo);
-    if (__all_sync(0xFFFFFFFFu, ok)) {
-      tc_fence_after();
-#pragma unroll
-      for (int c = 0; c < HD / 32; ++c) {
-        uint32_t r[32];
-        __syncwarp();
-        tmem_ld32(t_o + lane_base + c * 32, r);
-        tmem_ld_wait();
-#pragma unroll
-        for (int u = 0; u < 32; ++u) o[c * 32 + u] = fmaf(o[c * 32 + u], alpha, __uint_as_float(r[u]));
-      }
-    }
     tc_fence_before();
     ok = __syncthreads_and(ok) != 0;
+  }
+
+  // This CTA's partial output rows (O relative to m_run, unnormalised) out of TMEM.
+  float o[HD];
+  if (ok && n_mine > 0) {
+    tc_fence_after();
+    uint32_t ob[HD];
+#pragma unroll
+    for (int c = 0; c < HD / 32; ++c) tmem_ld32(t_o + lane_base + c * 32, chunk32(ob, c));
+    tmem_ld_wait();
+#pragma unroll
+    for (int c = 0; c < HD / 32; ++c) reg_fence32(chunk32(ob, c));
+#pragma unroll
+    for (int d = 0; d < HD; ++d) o[d] = __uint_as_float(ob[d]);
+  } else {
+#pragma unroll
+    for (int d = 0; d < HD; ++d) o[d] = 0.0f;
   }
 
   if (!ok && tid == 0) {

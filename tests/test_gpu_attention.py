@@ -127,12 +127,16 @@ def test_attention_llava15_full_layer():
     _run_case(cfg, n_sys=35, n_text=64, n_q_heads=32, layer=5, label="llava15 layer")
 
 
-def _exact_case(hd, B, hq, hkv, nt, n_keys, S, seed, label):
+def _exact_case(hd, B, hq, hkv, nt, n_keys, S, seed, label, k_gain=None):
     # Every slot holds synthetic bf16 K/V (no build): the oracle reads the same values.
+    # k_gain (per slot) scales the keys before their bf16 rounding.
     import torch
     import paper_2609_34972_gb300 as dv
     L = 2
     kb = synth.normal_bf16(seed, 30, (L, B, S, hkv, hd), 0.0, 1.0)
+    if k_gain is not None:
+        kb = synth.f64_to_bf16(synth.bf16_to_f32(kb).astype(np.float64) *
+                               np.asarray(k_gain, dtype=np.float64)[None, None, :, None, None])
     vb = synth.normal_bf16(seed, 31, (L, B, S, hkv, hd), 0.0, 1.0)
     qb = synth.normal_bf16(seed, 32, (B, hq, nt, hd), 0.0, 1.0)
     n_keys = np.asarray(n_keys, dtype=np.int32)
@@ -174,3 +178,20 @@ def test_attention_kernel_on_exact_inputs(hd, hq, hkv, nt):
 def test_attention_every_cluster_shape(hd, B, hq, hkv, nt, n_keys, S):
     _exact_case(hd, B, hq, hkv, nt, n_keys, S, 500 + hd + B + hq,
                 f"attention hd{hd} B{B} hq{hq}/{hkv} nt{nt}")
+
+
+@pytest.mark.parametrize("hd,B,hq,hkv,nt,n_keys,S,gain", [
+    # two stages, 8-CTA clusters, 2 key blocks per CTA; keys growing with the slot
+    (128, 1, 8, 2, 30, [2000], 2048, "rise"),
+    # one stage, 8-CTA clusters, 4 key blocks per CTA; growing, then a falling gain
+    (128, 2, 12, 12, 20, [4000, 3900], 4096, "rise"),
+    (64, 2, 12, 12, 20, [4000, 3900], 4096, "fall"),
+])
+def test_attention_running_maximum_grows_across_blocks(hd, B, hq, hkv, nt, n_keys, S, gain):
+    # Key magnitudes that change along the slots make each row's running maximum jump by more
+    # than 2^8 between key blocks (so O in TMEM is rescaled) or stay put (no rescale), with
+    # softmax weights far from uniform.
+    slots = np.arange(S, dtype=np.float64)
+    g = 1.0 + slots / 96.0 if gain == "rise" else 1.0 + (S - slots) / 96.0
+    _exact_case(hd, B, hq, hkv, nt, n_keys, S, 700 + hd + B, f"attention max growth hd{hd} {gain}",
+                k_gain=g)
