@@ -10,19 +10,22 @@
 // blocks. For each block a CTA:
 //   1. loads the K and V tiles by TMA (rows = slots, 128 B per 64 channels, 128-byte swizzle);
 //   2. one thread issues S = Q K^T (M = 128 rows, N = 128 keys, K = head_dim) into TMEM;
-//   3. the P V MMA reads V as it lies ([keys][channels] rows, an MN-major B operand), so V needs
-//      no transpose;
-//   4. each thread owns one query row: it reads the row's 128 scores from TMEM at once, keeps
+//   3. each thread owns one query row: it reads the row's 128 scores from TMEM at once, keeps
 //      the running maximum m and sum l, and writes the row's probabilities exp2(scaled score -
-//      m) as bf16 into the A tile of the second MMA;
-//   5. one thread issues O += P V (N = head_dim): O stays in TMEM over the CTA's key run. m is
-//      only moved (and O rescaled in TMEM) when the block maximum exceeds it by more than 2^8,
-//      a bound on the probabilities; O / l is the same for any common reference maximum.
-// Each thread then stores its partial (O, m, l) row straight into the shared memory of the CTA
-// that combines that row (distributed-shared-memory stores, no reply awaited); after one cluster
-// barrier CTA s combines rows [s * 128 / S, (s + 1) * 128 / S) over the S partials from its own
-// shared memory, in the fixed order 0..S-1, and stores bf16 rows. Every wait is bounded; a CTA
-// that gives up still passes the cluster barriers and flags the status word.
+//      m) as bf16 pairs back into TMEM over the first 64 score columns;
+//   4. one thread issues O += P V (N = head_dim) with P (the A operand) read from TMEM and V
+//      read as it lies ([keys][channels] rows, an MN-major B operand, no transpose). O stays in
+//      TMEM over the CTA's key run; m is only moved (and O rescaled in TMEM) when the block
+//      maximum exceeds it by more than 2^8, a bound on the probabilities, since O / l is the
+//      same for any common reference maximum.
+// With two stages the next block's K and V load during this block; with one stage the next K
+// loads once the score MMA has read K, the next V once the P V MMA has read V.
+// The partial (O, m, l) rows then go to the CTA that combines them: with two stages staged in
+// shared memory and moved by bulk copies that complete on the receiver's barrier, with one
+// stage by distributed-shared-memory stores and a cluster barrier. CTA s combines rows
+// [s * 128 / S, (s + 1) * 128 / S) over the S partials from its own shared memory, in the fixed
+// order 0..S-1, and stores bf16 rows. Every wait is bounded; a CTA that gives up still passes
+// the cluster barriers and flags the status word.
 #include <cmath>
 #include <mutex>
 
@@ -62,11 +65,7 @@ struct AttnCfg {
   static constexpr int kOffQ = 0;
   static constexpr int kOffStage = kOffQ + kKV;  // NST stages of [K | V]
   static constexpr int kStage = 2 * kKV;
-  // P (2 key slabs of [128 rows][64 keys]) takes the K slot of the current stage when that is
-  // large enough (HD = 128): K is dead once the score MMA has completed.
-  static constexpr bool kPInK = kKV >= 2 * kTile;
-  static constexpr int kOffP = kOffStage + NST * kStage;
-  static constexpr int kEnd = kOffP + (kPInK ? 0 : 2 * kTile);
+  static constexpr int kEnd = kOffStage + NST * kStage;  // P lives in TMEM, not here
   static constexpr int kMisc = 2048;                      // barriers, m, l, key end
   // Partial outputs received from the cluster: 128 rows of HD fp32 (16-byte chunks swizzled by
   // the row, no padding). With two stages they get a region of their own, so peers may write
@@ -118,6 +117,18 @@ __device__ __forceinline__ uint32_t cluster_size() {
   uint32_t r;
   asm volatile("mov.u32 %0, %%cluster_nctarank;" : "=r"(r));
   return r;
+}
+
+// D (+)= A B with A (M x 16, K-major, bf16) in TMEM at `a_tmem` (lane = row, column c = the
+// bf16 pair k = 2c, 2c + 1) and B from shared memory.
+__device__ __forceinline__ void umma_bf16_tmem_a(uint32_t d_tmem, uint32_t a_tmem, uint64_t b_desc,
+                                                 uint32_t idesc, uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n\t}" ::"r"(d_tmem),
+      "r"(a_tmem), "l"(b_desc), "r"(idesc), "r"(accumulate)
+      : "memory");
 }
 
 // Largest growth (base 2) of a row's maximum absorbed without rescaling O: probabilities
@@ -409,14 +420,22 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
   const int q_row0 = (b * p.Hq + h * p.G) * p.Nt + qb * 128;
   auto sK = [&](int st) { return base + C::kOffStage + st * C::kStage; };
   auto sV = [&](int st) { return base + C::kOffStage + st * C::kStage + C::kKV; };
-  auto load_kv = [&](int j) {  // block kb0 + j into stage j % NST
+  // K or V of block kb0 + j into stage j % NST (thread 0); last_k / last_v: the latest blocks
+  // whose K and V loads were issued, waited for before the memory is reused after an abort.
+  int last_k = -1, last_v = -1;
+  auto load_k = [&](int j) {
     const int st = j % NST, kb = kb0 + j;
     mbar_arrive_expect_tx(bar_k(st), C::kKV);
     for (int ds = 0; ds < C::kSlabs; ++ds)
       tma_load_4d(sK(st) + ds * C::kTile, &tmK, bar_k(st), ds * 64, h, kb * kKeyBlock, b);
+    last_k = j;
+  };
+  auto load_v = [&](int j) {
+    const int st = j % NST, kb = kb0 + j;
     mbar_arrive_expect_tx(bar_v(st), C::kKV);
     for (int ds = 0; ds < C::kSlabs; ++ds)
       tma_load_4d(sV(st) + ds * C::kTile, &tmV, bar_v(st), ds * 64, h, kb * kKeyBlock, b);
+    last_v = j;
   };
 
   float m_run = -INFINITY, l_run = 0.0f;
@@ -426,24 +445,23 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
     mbar_arrive_expect_tx(bar_q, C::kKV);
     for (int ds = 0; ds < C::kSlabs; ++ds)
       tma_load_2d(sQ + ds * C::kTile, &tmQ, bar_q, ds * 64, q_row0);
-    load_kv(0);
+    load_k(0);
+    load_v(0);
   }
-  int last_issued = n_mine > 0 ? 0 : -1;  // thread 0: last block whose K/V loads it issued
 
   bool ok = true;
   for (int j = 0; j < n_mine && ok; ++j) {
     const int st = j % NST, kb = kb0 + j;
     const uint32_t sph = static_cast<uint32_t>(j / NST) & 1u;  // phase of this stage's barriers
     const uint32_t ph = static_cast<uint32_t>(j) & 1u;        // phase of bar_s / bar_o
-    const uint32_t sP = C::kPInK ? sK(st) : base + C::kOffP;
     if (warp == 0) {
       if (lane == 0) {
-        if (NST == 2 && j + 1 < n_mine) {  // the other stage was freed by the previous block
-          load_kv(j + 1);
-          last_issued = j + 1;
-        } else if (NST == 1 && j > 0) {  // the one stage was freed when block j - 1 ended
-          load_kv(j);
-          last_issued = j;
+        // Two stages: the other stage was freed by the previous block. One stage: K of this
+        // block was issued once the previous score MMA had read K, V once the previous P V
+        // MMA had read V.
+        if (NST == 2 && j + 1 < n_mine) {
+          load_k(j + 1);
+          load_v(j + 1);
         }
         // S = Q K^T
         if (mbar_wait(bar_q, 0, abort_flag, tmo) && mbar_wait(bar_k(st), sph, abort_flag, tmo)) {
@@ -461,11 +479,9 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
       __syncwarp();
     }
 
-    // V is read by the P V MMA as it lies ([keys][channels], an MN-major operand).
-    ok = mbar_wait(bar_v(st), sph, abort_flag, tmo);
-
     // Scores -> probabilities (this thread: query row tid).
-    ok = ok && mbar_wait(bar_s, ph, abort_flag, tmo);
+    ok = mbar_wait(bar_s, ph, abort_flag, tmo);
+    if (NST == 1 && tid == 0 && ok && j + 1 < n_mine) load_k(j + 1);  // K slot read
     if (__all_sync(0xFFFFFFFFu, ok)) {
       tc_fence_after();
       // the row's 128 scores in one TMEM round trip; keys past the row's last slot are masked
@@ -514,46 +530,41 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
         tmem_st_wait();
       }
       const float m_sub = m_use == -INFINITY ? 0.0f : m_use;
+      // P as bf16 pairs (keys 2c, 2c + 1 in column c) over the first 64 score columns: the A
+      // operand of the P V MMA, read from TMEM (the scores are all in registers by now).
       float lb[4] = {0.0f, 0.0f, 0.0f, 0.0f};
 #pragma unroll
-      for (int c = 0; c < kKeyBlock / 32; ++c) {
-        uint32_t pk[16];
+      for (int c = 0; c < kKeyBlock / 64; ++c) {
+        uint32_t pk[32];
 #pragma unroll
-        for (int u = 0; u < 32; u += 2) {
-          const float p0 = ex2_approx(x[c * 32 + u] - m_sub);
-          const float p1 = ex2_approx(x[c * 32 + u + 1] - m_sub);
+        for (int u = 0; u < 64; u += 2) {
+          const float p0 = ex2_approx(x[c * 64 + u] - m_sub);
+          const float p1 = ex2_approx(x[c * 64 + u + 1] - m_sub);
           lb[(u / 2) % 4] += p0 + p1;
           pk[u / 2] = pack_bf16x2(p0, p1);
         }
-        // keys 32c .. 32c + 31 = 4 chunks of 8 keys in key slab c / 2
-        uint8_t* p_row = base_ptr + (sP - base) + (c / 2) * C::kTile + tid * 128;
-#pragma unroll
-        for (int q4 = 0; q4 < 4; ++q4) {
-          const int chunk = (c % 2) * 4 + q4;
-          *reinterpret_cast<uint4*>(p_row + ((chunk ^ (tid & 7)) << 4)) =
-              make_uint4(pk[4 * q4], pk[4 * q4 + 1], pk[4 * q4 + 2], pk[4 * q4 + 3]);
-        }
+        tmem_st32(t_s + lane_base + c * 32, pk);
       }
+      tmem_st_wait();
       l_run = alpha * l_run + ((lb[0] + lb[1]) + (lb[2] + lb[3]));
       m_run = m_use;
     }
-    fence_proxy_async_smem();
     tc_fence_before();
     ok = __syncthreads_and(ok) != 0;
 
-    // O (+)= P V in TMEM; the CTA's first block initialises O
-    if (ok && tid == 0) {
+    // O (+)= P V in TMEM; the CTA's first block initialises O. V is read as it lies ([keys]
+    // [channels], an MN-major B operand); P (A, K-major) from TMEM, 16 keys = 8 columns.
+    if (ok && tid == 0 && mbar_wait(bar_v(st), sph, abort_flag, tmo)) {
       tc_fence_after();
-      const uint32_t idesc = idesc_bf16_f32(128, HD) | (1u << 16);  // B (V) MN-major
-      for (int ks = 0; ks < 2; ++ks)
+      const uint32_t idesc = idesc_bf16_f32(128, HD) | (1u << 16);
 #pragma unroll
-        for (int k = 0; k < 4; ++k)
-          umma_bf16(t_o, sdesc_kmajor_sw128(sP + ks * C::kTile + 32u * k),
-                    sdesc_mnmajor_sw128(sV(st) + (ks * 64 + k * 16) * 128, C::kTile), idesc,
-                    (j | ks | k) != 0 ? 1u : 0u);
+      for (int kk = 0; kk < kKeyBlock / 16; ++kk)
+        umma_bf16_tmem_a(t_o, t_s + kk * 8, sdesc_mnmajor_sw128(sV(st) + kk * 16 * 128, C::kTile),
+                         idesc, (j | kk) != 0 ? 1u : 0u);
       umma_commit(bar_o);
     }
     ok = ok && mbar_wait(bar_o, ph, abort_flag, tmo);
+    if (NST == 1 && tid == 0 && ok && j + 1 < n_mine) load_v(j + 1);  // V slot read
     tc_fence_before();
     ok = __syncthreads_and(ok) != 0;
   }
@@ -578,12 +589,11 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
   if (!ok && tid == 0) {
     // Let the copies in flight (the last block issued on each stage) land and every issued MMA
     // finish before the memory is reused; each wait targets its stage's latest phase.
-    for (int jj = last_issued; jj >= 0 && jj > last_issued - NST; --jj) {
-      const uint32_t sp = static_cast<uint32_t>(jj / NST) & 1u;
-      wait_bounded(bar_k(jj % NST), sp, tmo);
-      wait_bounded(bar_v(jj % NST), sp, tmo);
-    }
-    if (last_issued >= 0) wait_bounded(bar_q, 0, tmo);
+    for (int jj = last_k; jj >= 0 && jj > last_k - NST; --jj)
+      wait_bounded(bar_k(jj % NST), static_cast<uint32_t>(jj / NST) & 1u, tmo);
+    for (int jj = last_v; jj >= 0 && jj > last_v - NST; --jj)
+      wait_bounded(bar_v(jj % NST), static_cast<uint32_t>(jj / NST) & 1u, tmo);
+    if (last_k >= 0) wait_bounded(bar_q, 0, tmo);
     umma_commit(bar_drain);
     wait_bounded(bar_drain, 0, tmo);
   }
