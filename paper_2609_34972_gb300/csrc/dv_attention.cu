@@ -269,17 +269,33 @@ __device__ __forceinline__ void stage_partial(const float* o, float m_run, float
   fence_proxy_async_smem();  // the staged rows are read by the bulk copies (async proxy)
 }
 
+// Query rows of its 128 / S that CTA d combines and stores: those of the tile's `tile_rows`
+// valid rows (rows past the query group are never stored, so they are neither sent nor
+// combined). Sender and receiver use this same count.
+__device__ __forceinline__ int rows_combined(int tile_rows, int d, int S) {
+  const int rows = 128 / S;
+  return max(0, min(rows, tile_rows - d * rows));
+}
+
+// Bytes CTA `d` receives from each peer: its valid rows, then all m and l of its rows.
+template <int HD>
+__device__ __forceinline__ uint32_t bytes_from_peer(int tile_rows, int d, int S) {
+  const int n = rows_combined(tile_rows, d, S);
+  return n > 0 ? static_cast<uint32_t>(n * HD * 4 + 8 * (128 / S)) : 0u;
+}
+
 template <int HD>
 __device__ __forceinline__ void send_partial(uint32_t recv, uint32_t recv_ml, uint32_t send,
                                              uint32_t send_ml, uint32_t bar_recv, int split,
-                                             int S) {
+                                             int S, int tile_rows) {
   const int rows = 128 / S;
   for (int dd = 0; dd < S; ++dd) {
-    if (dd == split) continue;
+    const int n = rows_combined(tile_rows, dd, S);
+    if (dd == split || n == 0) continue;
     const uint32_t rank = static_cast<uint32_t>(dd), cbar = map_to_rank(bar_recv, rank);
     bulk_copy_to_peer(map_to_rank(recv + static_cast<uint32_t>(split * rows) * (HD * 4), rank),
                       send + static_cast<uint32_t>(dd * rows) * (HD * 4),
-                      static_cast<uint32_t>(rows * HD * 4), cbar);
+                      static_cast<uint32_t>(n * HD * 4), cbar);
     bulk_copy_to_peer(map_to_rank(recv_ml + 4u * (2 * split * rows), rank),
                       send_ml + 4u * (2 * dd * rows), static_cast<uint32_t>(8 * rows), cbar);
   }
@@ -366,6 +382,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
   const int qb = unit % p.q_blocks;
   const int h = (unit / p.q_blocks) % p.Hkv;
   const int b = unit / (p.q_blocks * p.Hkv);
+  const int tile_rows = min(128, p.rows_per_group - qb * 128);  // valid query rows of the tile
 
   if (tid == 0) {
     tma_prefetch_desc(&tmQ);
@@ -381,8 +398,8 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
     mbar_init(bar_drain, 1);
     if (C::kRecvOwn) {
       mbar_init(bar_recv, 1);
-      const uint32_t rows = 128u / static_cast<uint32_t>(S);
-      mbar_arrive_expect_tx(bar_recv, static_cast<uint32_t>(S - 1) * (rows * HD * 4 + 8 * rows));
+      mbar_arrive_expect_tx(bar_recv, static_cast<uint32_t>(S - 1) *
+                                          bytes_from_peer<HD>(tile_rows, split, S));
     }
     *abort_flag = 0;
     *key_end = 0;
@@ -491,18 +508,24 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
       tmem_ld_wait();
 #pragma unroll
       for (int c = 0; c < kKeyBlock / 32; ++c) reg_fence32(chunk32(r, c));
+      // raw scores; the scale (> 0) is applied after the maximum and inside the exponent
       const int n_valid = last - kb * kKeyBlock + 1;
       float x[kKeyBlock];
+      if (n_valid >= kKeyBlock) {
 #pragma unroll
-      for (int u = 0; u < kKeyBlock; ++u)
-        x[u] = u < n_valid ? __uint_as_float(r[u]) * p.scale_log2 : -INFINITY;
+        for (int u = 0; u < kKeyBlock; ++u) x[u] = __uint_as_float(r[u]);
+      } else {
+#pragma unroll
+        for (int u = 0; u < kKeyBlock; ++u) x[u] = u < n_valid ? __uint_as_float(r[u]) : -INFINITY;
+      }
       float mx[8];
 #pragma unroll
       for (int u = 0; u < 8; ++u) mx[u] = x[u];
 #pragma unroll
       for (int u = 8; u < kKeyBlock; ++u) mx[u % 8] = fmaxf(mx[u % 8], x[u]);
       const float mb = fmaxf(fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3])),
-                             fmaxf(fmaxf(mx[4], mx[5]), fmaxf(mx[6], mx[7])));
+                             fmaxf(fmaxf(mx[4], mx[5]), fmaxf(mx[6], mx[7]))) *
+                       p.scale_log2;
       const float m_new = fmaxf(m_run, mb);
       // The row keeps its reference maximum while the new scores exceed it by at most
       // kRescaleLog2 (probabilities stay <= 2^kRescaleLog2); O and l only need the same
@@ -538,8 +561,8 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
         uint32_t pk[32];
 #pragma unroll
         for (int u = 0; u < 64; u += 2) {
-          const float p0 = ex2_approx(x[c * 64 + u] - m_sub);
-          const float p1 = ex2_approx(x[c * 64 + u + 1] - m_sub);
+          const float p0 = ex2_approx(fmaf(x[c * 64 + u], p.scale_log2, -m_sub));
+          const float p1 = ex2_approx(fmaf(x[c * 64 + u + 1], p.scale_log2, -m_sub));
           lb[(u / 2) % 4] += p0 + p1;
           pk[u / 2] = pack_bf16x2(p0, p1);
         }
@@ -608,7 +631,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
     asm volatile("barrier.cluster.wait.aligned;" ::: "memory");  // peers' barriers initialised
     if (tid == 0)
       send_partial<HD>(recv, smem_addr(recv_ml), base + C::kOffQ, base + C::kOffSendML, bar_recv,
-                       split, S);
+                       split, S, tile_rows);
     // Not cut short by the abort flag: the copies into this CTA must land before it may exit.
     if (!wait_bounded(bar_recv, 0, tmo)) *abort_flag = 1;
     // Everything sent to this CTA has landed; once all CTAs say so (the wait before exit), no
