@@ -20,12 +20,12 @@
 //      same for any common reference maximum.
 // With two stages the next block's K and V load during this block; with one stage the next K
 // loads once the score MMA has read K, the next V once the P V MMA has read V.
-// The partial (O, m, l) rows then go to the CTA that combines them: with two stages staged in
-// shared memory and moved by bulk copies that complete on the receiver's barrier, with one
-// stage by distributed-shared-memory stores and a cluster barrier. CTA s combines rows
-// [s * 128 / S, (s + 1) * 128 / S) over the S partials from its own shared memory, in the fixed
-// order 0..S-1, and stores bf16 rows. Every wait is bounded; a CTA that gives up still passes
-// the cluster barriers and flags the status word.
+// The partial (O, m, l) rows then go to the CTA that combines them, staged in shared memory and
+// moved by bulk copies that complete on the receiver's barrier. CTA s combines rows
+// [s * 128 / S, (s + 1) * 128 / S) over the S partials, in the fixed order 0..S-1, and stores
+// bf16 rows: with two stages from a receive region of its own, with one stage (S <= 4, two CTAs
+// per SM) from its own registers and the peers' rows received over Q and K. Every wait is
+// bounded; a CTA that gives up still passes the cluster barriers and flags the status word.
 #include <cmath>
 #include <mutex>
 
@@ -79,6 +79,10 @@ struct AttnCfg {
   // their maxima and sums right after them.
   static constexpr int kOffSendML = kOffQ + kRecvBytes;
   static_assert(kOffSendML + 1024 <= kKV + NST * kStage, "staged partials fit Q and the stages");
+  // One stage (S <= 4): up to 96 rows received over Q and K, 96 staged after them; their m and
+  // l lists at kEnd + 256 and kEnd + 1280 (768 bytes each at most).
+  static_assert(NST == 2 || 2 * 96 * HD * 4 <= kKV + kStage, "one-stage exchange fits Q, K, V");
+  static constexpr int kOffSendML1 = kEnd + 1280;
   static_assert(kKV % 1024 == 0, "tiles stay 1024-byte aligned");
   static_assert(kSmemBytes <= 232448, "shared memory of one CTA");
 };
@@ -189,51 +193,9 @@ __device__ __forceinline__ uint32_t chunk_swizzle(int R) {
   return static_cast<uint32_t>(((R & 1) << 2) | (R & 2) | ((R >> 2) & 1));
 }
 
-__device__ __forceinline__ void st_cluster_f4(uint32_t caddr, float a, float b, float c, float d) {
-  asm volatile("st.shared::cluster.v4.f32 [%0], {%1, %2, %3, %4};" ::"r"(caddr), "f"(a), "f"(b),
-               "f"(c), "f"(d)
-               : "memory");
-}
-
-__device__ __forceinline__ void st_cluster_f32(uint32_t caddr, float v) {
-  asm volatile("st.shared::cluster.f32 [%0], %1;" ::"r"(caddr), "f"(v) : "memory");
-}
-
 // Thread `tid` holds query row tid of this CTA's key run: (o, m, l). Row tid is combined by CTA
-// d = tid / (128 / S); it goes into d's receive rows at R = split * 128 / S + tid mod (128 / S),
-// its maximum and sum into d's receive list at [split][0][R mod rows] and [split][1][...]
-// ([source][m | l][row], rows = 128 / S). Rows are a multiple of 8, so R and tid share the
-// chunk swizzle.
-//
-// One-stage variant: distributed-shared-memory stores (local stores when d is this CTA), which
-// need no reply; the cluster barrier that follows makes them visible.
-template <int HD>
-__device__ __forceinline__ void push_partial(const float* o, float m_run, float l_run,
-                                             uint32_t recv, uint32_t recv_ml, int split, int S) {
-  const int tid = threadIdx.x, rows = 128 / S;
-  const int d = tid / rows, R = split * rows + tid % rows;
-  const uint32_t sw = chunk_swizzle(R);
-  const uint32_t recv_m = recv_ml + 4u * (2 * split * rows + tid % rows), recv_l = recv_m + 4u * rows;
-  const uint32_t row = recv + static_cast<uint32_t>(R) * (HD * 4);
-  if (d == split) {
-#pragma unroll
-    for (int c = 0; c < HD / 4; ++c) {
-      float4* dst = reinterpret_cast<float4*>(__cvta_shared_to_generic(row + ((c ^ sw) << 4)));
-      *dst = make_float4(o[4 * c], o[4 * c + 1], o[4 * c + 2], o[4 * c + 3]);
-    }
-    *reinterpret_cast<float*>(__cvta_shared_to_generic(recv_m)) = m_run;
-    *reinterpret_cast<float*>(__cvta_shared_to_generic(recv_l)) = l_run;
-  } else {
-    const uint32_t rank = static_cast<uint32_t>(d);
-    const uint32_t crow = map_to_rank(row, rank);
-#pragma unroll
-    for (int c = 0; c < HD / 4; ++c)
-      st_cluster_f4(crow + ((c ^ sw) << 4), o[4 * c], o[4 * c + 1], o[4 * c + 2], o[4 * c + 3]);
-    st_cluster_f32(map_to_rank(recv_m, rank), m_run);
-    st_cluster_f32(map_to_rank(recv_l, rank), l_run);
-  }
-}
-
+// d = tid / rows (rows = 128 / S, a multiple of 8, so a row's chunk swizzle is that of tid mod
+// rows); its maximum and sum travel as lists [source][m | l][row].
 __device__ __forceinline__ void bulk_copy_to_peer(uint32_t dst_cluster, uint32_t src, uint32_t bytes,
                                                   uint32_t bar_cluster) {
   asm volatile(
@@ -242,8 +204,9 @@ __device__ __forceinline__ void bulk_copy_to_peer(uint32_t dst_cluster, uint32_t
       : "memory");
 }
 
-// Two-stage variant: the same placement, but rows for a peer are staged in this CTA's shared
-// memory (`send`, `send_ml`, laid out as the peer will hold them) and one thread moves each
+// Two-stage variant: receive rows R = source * rows + row in a region of their own. Rows for a
+// peer are staged in this CTA's shared memory (`send`, `send_ml`, laid out as the peer will hold
+// them), this CTA's own rows go straight into its receive rows, and one thread moves each
 // peer's share with two bulk copies, which complete on the peer's receive barrier. Bulk copies
 // move the 16 KB shares about twice as fast as per-thread remote stores. Precondition: every
 // CTA of the cluster has initialised its receive barrier (the caller's cluster wait).
@@ -298,6 +261,122 @@ __device__ __forceinline__ void send_partial(uint32_t recv, uint32_t recv_ml, ui
                       static_cast<uint32_t>(n * HD * 4), cbar);
     bulk_copy_to_peer(map_to_rank(recv_ml + 4u * (2 * split * rows), rank),
                       send_ml + 4u * (2 * dd * rows), static_cast<uint32_t>(8 * rows), cbar);
+  }
+}
+
+// One-stage variant (S = 2 or 4, the shared memory of two CTAs per SM): a CTA's own rows stay in
+// the registers of the threads that hold them, so it receives only its S - 1 peers' rows, in
+// slots of `rows` rows (peer s in slot s, or s - 1 past this CTA's rank), over Q and the K slot
+// (free once every key run of the cluster has ended). Rows for peer d are staged after them,
+// in slots numbered the same way (d, or d - 1 past this CTA's rank).
+__device__ __forceinline__ int peer_slot(int s, int self) { return s < self ? s : s - 1; }
+
+template <int HD>
+__device__ __forceinline__ void stage_peer_rows(const float* o, float m_run, float l_run,
+                                                uint32_t send, uint32_t send_ml, int split, int S) {
+  const int tid = threadIdx.x, rows = 128 / S;
+  const int d = tid / rows, rr = tid % rows;
+  if (d == split) return;
+  const int di = peer_slot(d, split);
+  const uint32_t sw = chunk_swizzle(rr);
+  const uint32_t row = send + static_cast<uint32_t>(di * rows + rr) * (HD * 4);
+#pragma unroll
+  for (int c = 0; c < HD / 4; ++c) {
+    float4* dst = reinterpret_cast<float4*>(__cvta_shared_to_generic(row + ((c ^ sw) << 4)));
+    *dst = make_float4(o[4 * c], o[4 * c + 1], o[4 * c + 2], o[4 * c + 3]);
+  }
+  const uint32_t ml = send_ml + 4u * (2 * di * rows + rr);
+  *reinterpret_cast<float*>(__cvta_shared_to_generic(ml)) = m_run;
+  *reinterpret_cast<float*>(__cvta_shared_to_generic(ml + 4u * rows)) = l_run;
+  fence_proxy_async_smem();  // the staged rows are read by the bulk copies (async proxy)
+}
+
+template <int HD>
+__device__ __forceinline__ void send_peer_rows(uint32_t recv, uint32_t recv_ml, uint32_t send,
+                                               uint32_t send_ml, uint32_t bar_recv, int split,
+                                               int S, int tile_rows) {
+  const int rows = 128 / S;
+  for (int dd = 0; dd < S; ++dd) {
+    const int n = rows_combined(tile_rows, dd, S);
+    if (dd == split || n == 0) continue;
+    const int di = peer_slot(dd, split), slot = peer_slot(split, dd);
+    const uint32_t rank = static_cast<uint32_t>(dd), cbar = map_to_rank(bar_recv, rank);
+    bulk_copy_to_peer(map_to_rank(recv + static_cast<uint32_t>(slot * rows) * (HD * 4), rank),
+                      send + static_cast<uint32_t>(di * rows) * (HD * 4),
+                      static_cast<uint32_t>(n * HD * 4), cbar);
+    bulk_copy_to_peer(map_to_rank(recv_ml + 4u * (2 * slot * rows), rank),
+                      send_ml + 4u * (2 * di * rows), static_cast<uint32_t>(8 * rows), cbar);
+  }
+}
+
+// The threads holding this CTA's own rows combine them: own partial from registers, the peers'
+// from the receive slots, summed in the fixed order of the sources 0 .. S-1.
+template <int HD, int S>
+__device__ __forceinline__ void combine_own_rows(const float* o, float m_run, float l_run,
+                                                 uint32_t recv, const float* recv_ml, int split,
+                                                 int qb, int h, int b, const AttnParams& p) {
+  constexpr int kRows = 128 / S;
+  const int tid = threadIdx.x;
+  if (tid / kRows != split) return;
+  const int rr = tid % kRows, ii = qb * 128 + tid;
+  if (ii >= p.rows_per_group) return;
+  const uint32_t sw = chunk_swizzle(rr);
+  float ms[S], ls[S], w[S];
+  uint32_t prow[S];
+#pragma unroll
+  for (int s = 0; s < S; ++s) {
+    if (s == split) {
+      ms[s] = m_run;
+      ls[s] = l_run;
+      prow[s] = 0;
+    } else {
+      const int slot = peer_slot(s, split);
+      ms[s] = recv_ml[(2 * slot) * kRows + rr];
+      ls[s] = recv_ml[(2 * slot + 1) * kRows + rr];
+      prow[s] = recv + static_cast<uint32_t>(slot * kRows + rr) * (HD * 4);
+    }
+  }
+  float M = -INFINITY;
+#pragma unroll
+  for (int s = 0; s < S; ++s) M = fmaxf(M, ms[s]);
+  float L = 0.0f;
+#pragma unroll
+  for (int s = 0; s < S; ++s) {
+    w[s] = ms[s] != -INFINITY ? exp2f(ms[s] - M) : 0.0f;
+    L = fmaf(w[s], ls[s], L);
+  }
+  const float inv = L > 0.0f ? 1.0f / L : 0.0f;
+  const int hq = h * p.G + ii / p.Nt, t = ii % p.Nt;
+  uint16_t* orow = p.out + ((static_cast<size_t>(b) * p.Hq + hq) * p.Nt + t) * HD;
+#pragma unroll
+  for (int c2 = 0; c2 < HD / 8; ++c2) {
+    float acc[8];
+#pragma unroll
+    for (int e = 0; e < 8; ++e) acc[e] = 0.0f;
+#pragma unroll
+    for (int s = 0; s < S; ++s) {
+#pragma unroll
+      for (int h2 = 0; h2 < 2; ++h2) {
+        const int c = 2 * c2 + h2;
+        float4 v;
+        if (s == split) {
+          v = make_float4(o[4 * c], o[4 * c + 1], o[4 * c + 2], o[4 * c + 3]);
+        } else {
+          v = *reinterpret_cast<const float4*>(
+              __cvta_shared_to_generic(prow[s] + ((static_cast<uint32_t>(c) ^ sw) << 4)));
+        }
+        acc[4 * h2] = fmaf(w[s], v.x, acc[4 * h2]);
+        acc[4 * h2 + 1] = fmaf(w[s], v.y, acc[4 * h2 + 1]);
+        acc[4 * h2 + 2] = fmaf(w[s], v.z, acc[4 * h2 + 2]);
+        acc[4 * h2 + 3] = fmaf(w[s], v.w, acc[4 * h2 + 3]);
+      }
+    }
+    uint4 out;
+    out.x = pack_bf16x2(acc[0] * inv, acc[1] * inv);
+    out.y = pack_bf16x2(acc[2] * inv, acc[3] * inv);
+    out.z = pack_bf16x2(acc[4] * inv, acc[5] * inv);
+    out.w = pack_bf16x2(acc[6] * inv, acc[7] * inv);
+    *reinterpret_cast<uint4*>(orow + c2 * 8) = out;
   }
 }
 
@@ -365,7 +444,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
   const uint32_t bar0 = smem_addr(bars);
   // barriers: Q, K of stage 0/1, V of stage 0/1, scores ready, block output ready, drain
   const uint32_t bar_q = bar0, bar_s = bar0 + 40, bar_o = bar0 + 48, bar_drain = bar0 + 56;
-  const uint32_t bar_recv = bar0 + 80;  // partial rows received from the peers (two stages)
+  const uint32_t bar_recv = bar0 + 80;  // partial rows received from the peers
   auto bar_k = [&](int st) { return bar0 + 8u + 8u * st; };
   auto bar_v = [&](int st) { return bar0 + 24u + 8u * st; };
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 8);
@@ -396,11 +475,9 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
     mbar_init(bar_s, 1);
     mbar_init(bar_o, 1);
     mbar_init(bar_drain, 1);
-    if (C::kRecvOwn) {
-      mbar_init(bar_recv, 1);
-      mbar_arrive_expect_tx(bar_recv, static_cast<uint32_t>(S - 1) *
-                                          bytes_from_peer<HD>(tile_rows, split, S));
-    }
+    mbar_init(bar_recv, 1);
+    mbar_arrive_expect_tx(bar_recv,
+                          static_cast<uint32_t>(S - 1) * bytes_from_peer<HD>(tile_rows, split, S));
     *abort_flag = 0;
     *key_end = 0;
     fence_barrier_init();
@@ -622,8 +699,10 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
   }
   __syncthreads();
 
-  // Partial (O, m, l) of this CTA's key run -> the receive rows of the CTA that combines each
-  // row, then every CTA combines from its own shared memory.
+  // Partial (O, m, l) of this CTA's key run -> the CTA that combines each row, by bulk copies
+  // that complete on the receiver's barrier; the waits for them are not cut short by the abort
+  // flag, since the copies into a CTA must land before it may exit. Once every CTA has seen
+  // its copies land (the cluster barrier before exit), no copy touches any CTA's memory.
   if (C::kRecvOwn) {
     stage_partial<HD>(o, m_run, l_run, recv, smem_addr(recv_ml), base + C::kOffQ,
                       base + C::kOffSendML, split, S);
@@ -632,26 +711,34 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
     if (tid == 0)
       send_partial<HD>(recv, smem_addr(recv_ml), base + C::kOffQ, base + C::kOffSendML, bar_recv,
                        split, S, tile_rows);
-    // Not cut short by the abort flag: the copies into this CTA must land before it may exit.
     if (!wait_bounded(bar_recv, 0, tmo)) *abort_flag = 1;
-    // Everything sent to this CTA has landed; once all CTAs say so (the wait before exit), no
-    // copy reads or writes any CTA's shared memory.
     __syncwarp();
     asm volatile("barrier.cluster.arrive.aligned;" ::: "memory");
-  } else {  // the receive rows reuse Q and the stage, free once every key run has ended
-    cluster_sync();
-    push_partial<HD>(o, m_run, l_run, recv, smem_addr(recv_ml), split, S);
+    switch (S) {  // the cluster size: 1, 2, 4 or 8
+      case 1: combine_rows<HD, 1>(recv, recv_ml, split, qb, h, b, p); break;
+      case 2: combine_rows<HD, 2>(recv, recv_ml, split, qb, h, b, p); break;
+      case 4: combine_rows<HD, 4>(recv, recv_ml, split, qb, h, b, p); break;
+      default: combine_rows<HD, 8>(recv, recv_ml, split, qb, h, b, p); break;
+    }
+  } else {  // one stage: S = 2 or 4
+    const int rows = 128 / S;
+    const uint32_t send = base + static_cast<uint32_t>((128 - rows) * HD * 4);
+    const uint32_t send_ml = base + C::kOffSendML1;
+    stage_peer_rows<HD>(o, m_run, l_run, send, send_ml, split, S);
+    __syncthreads();
+    cluster_sync();  // every key run of the cluster has ended: Q and K may receive
+    if (tid == 0)
+      send_peer_rows<HD>(recv, smem_addr(recv_ml), send, send_ml, bar_recv, split, S, tile_rows);
+    if (!wait_bounded(bar_recv, 0, tmo)) *abort_flag = 1;
     __syncwarp();
-    cluster_sync();
-  }
-  switch (S) {  // the cluster size: 1, 2, 4 or 8
-    case 1: combine_rows<HD, 1>(recv, recv_ml, split, qb, h, b, p); break;
-    case 2: combine_rows<HD, 2>(recv, recv_ml, split, qb, h, b, p); break;
-    case 4: combine_rows<HD, 4>(recv, recv_ml, split, qb, h, b, p); break;
-    default: combine_rows<HD, 8>(recv, recv_ml, split, qb, h, b, p); break;
+    asm volatile("barrier.cluster.arrive.aligned;" ::: "memory");
+    if (S == 2)
+      combine_own_rows<HD, 2>(o, m_run, l_run, recv, recv_ml, split, qb, h, b, p);
+    else
+      combine_own_rows<HD, 4>(o, m_run, l_run, recv, recv_ml, split, qb, h, b, p);
   }
   __syncwarp();
-  if (C::kRecvOwn) asm volatile("barrier.cluster.wait.aligned;" ::: "memory");
+  asm volatile("barrier.cluster.wait.aligned;" ::: "memory");
 
   if (warp == 0) {
     tc_fence_after();
@@ -833,7 +920,7 @@ extern "C" int dv_text_attention(const void* q, int batch, int n_q_heads, int n_
   int split2 = 1, split1 = 1;
   for (int s : {2, 4, 8}) {
     if (s <= blocks_max && units * s <= sms) split2 = s;
-    if (s <= blocks_max && units * s <= 2LL * sms) split1 = s;
+    if (s <= 4 && s <= blocks_max && units * s <= 2LL * sms) split1 = s;  // one stage: S <= 4
   }
   const bool one_stage = split1 > split2;
   const int splits = one_stage ? split1 : split2;

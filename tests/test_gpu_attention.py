@@ -163,17 +163,21 @@ def test_attention_kernel_on_exact_inputs(hd, hq, hkv, nt):
 
 
 # Launch shapes that reach every kernel variant and cluster size the launcher picks (clusters =
-# batch x kv heads x 128-row query blocks, cluster size S = the largest of 2, 4, 8 within the key
-# blocks and one CTA per SM (two stages) or two per SM (one stage) on 152 SMs):
-#   two stages, S = 8: 2 clusters, 9 key blocks; one stage, S = 8: 24 clusters;
-#   one stage, S = 2: 80 clusters, 3 key blocks; one stage, S = 4 at head_dim 64: 64 clusters.
+# batch x kv heads x 128-row query blocks; cluster size S = the largest of 2, 4, 8 within the key
+# blocks with one CTA per SM (two stages), or of 2, 4 with two CTAs per SM (one stage) when
+# that is larger, on 152 SMs):
+#   two stages, S = 8: 2 clusters, 9 key blocks; two stages, S = 4: 24 clusters;
+#   one stage, S = 2: 80 clusters, 3 key blocks; one stage, S = 4: 64 clusters (64 of 128 query
+#   rows valid) and 48 clusters (tiles of 128, 128 and 94 query rows).
 @pytest.mark.parametrize("hd,B,hq,hkv,nt,n_keys,S", [
     (128, 1, 8, 2, 30, [1100], 1152),
     (64, 1, 8, 2, 30, [1100], 1152),
     (128, 2, 12, 12, 20, [1000, 977], 1024),
     (64, 2, 12, 12, 20, [1000, 977], 1024),
     (128, 4, 20, 20, 16, [300, 290, 300, 257], 320),
+    (64, 4, 20, 20, 16, [300, 290, 300, 257], 320),
     (64, 2, 32, 32, 64, [700, 650], 768),
+    (128, 4, 28, 4, 50, [700, 650, 700, 690], 768),
 ])
 def test_attention_every_cluster_shape(hd, B, hq, hkv, nt, n_keys, S):
     _exact_case(hd, B, hq, hkv, nt, n_keys, S, 500 + hd + B + hq,
@@ -183,8 +187,8 @@ def test_attention_every_cluster_shape(hd, B, hq, hkv, nt, n_keys, S):
 @pytest.mark.parametrize("hd,B,hq,hkv,nt,n_keys,S,gain", [
     # two stages, 8-CTA clusters, 2 key blocks per CTA; keys growing with the slot
     (128, 1, 8, 2, 30, [2000], 2048, "rise"),
-    # one stage, 8-CTA clusters, 4 key blocks per CTA; growing, then a falling gain
-    (128, 2, 12, 12, 20, [4000, 3900], 4096, "rise"),
+    # one stage, 4-CTA clusters, 4 key blocks per CTA; two stages, 4-CTA clusters, 8 blocks
+    (128, 4, 28, 4, 50, [2000, 1900, 2000, 1950], 2048, "rise"),
     (64, 2, 12, 12, 20, [4000, 3900], 4096, "fall"),
 ])
 def test_attention_running_maximum_grows_across_blocks(hd, B, hq, hkv, nt, n_keys, S, gain):
