@@ -23,8 +23,8 @@
 // The partial (O, m, l) rows then go to the CTA that combines them, staged in shared memory and
 // moved by bulk copies that complete on the receiver's barrier. CTA s combines rows
 // [s * 128 / S, (s + 1) * 128 / S) over the S partials, in the fixed order 0..S-1, and stores
-// bf16 rows: with two stages from a receive region of its own, with one stage (S <= 4, two CTAs
-// per SM) from its own registers and the peers' rows received over Q and K. Every wait is
+// bf16 rows: with two stages from a receive region of its own, with one stage (S = 2, two CTAs
+// per SM) from its own registers and the peer's rows received over Q and K. Every wait is
 // bounded; a CTA that gives up still passes the cluster barriers and flags the status word.
 #include <cmath>
 #include <mutex>
@@ -56,7 +56,8 @@ struct AttnParams {
 __device__ int g_attn_status;
 
 // NST = 2: two stages of [K | V] (the next block loads during this one), one CTA per SM.
-// NST = 1: one stage, small enough for two CTAs per SM; used when that allows more key splits.
+// NST = 1: one stage, small enough for two CTAs per SM; used in clusters of 2 where two stages
+// could not split the keys at all.
 template <int HD, int NST>
 struct AttnCfg {
   static constexpr int kSlabs = HD / 64;
@@ -79,9 +80,9 @@ struct AttnCfg {
   // their maxima and sums right after them.
   static constexpr int kOffSendML = kOffQ + kRecvBytes;
   static_assert(kOffSendML + 1024 <= kKV + NST * kStage, "staged partials fit Q and the stages");
-  // One stage (S <= 4): up to 96 rows received over Q and K, 96 staged after them; their m and
-  // l lists at kEnd + 256 and kEnd + 1280 (768 bytes each at most).
-  static_assert(NST == 2 || 2 * 96 * HD * 4 <= kKV + kStage, "one-stage exchange fits Q, K, V");
+  // One stage (S = 2): 64 rows received over Q and K, 64 staged after them; their m and l lists
+  // at kEnd + 256 and kEnd + 1280 (512 bytes each).
+  static_assert(NST == 2 || 2 * 64 * HD * 4 <= kKV + kStage, "one-stage exchange fits Q, K, V");
   static constexpr int kOffSendML1 = kEnd + 1280;
   static_assert(kKV % 1024 == 0, "tiles stay 1024-byte aligned");
   static_assert(kSmemBytes <= 232448, "shared memory of one CTA");
@@ -264,7 +265,7 @@ __device__ __forceinline__ void send_partial(uint32_t recv, uint32_t recv_ml, ui
   }
 }
 
-// One-stage variant (S = 2 or 4, the shared memory of two CTAs per SM): a CTA's own rows stay in
+// One-stage variant (S = 2, the shared memory of two CTAs per SM): a CTA's own rows stay in
 // the registers of the threads that hold them, so it receives only its S - 1 peers' rows, in
 // slots of `rows` rows (peer s in slot s, or s - 1 past this CTA's rank), over Q and the K slot
 // (free once every key run of the cluster has ended). Rows for peer d are staged after them,
@@ -720,7 +721,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
       case 4: combine_rows<HD, 4>(recv, recv_ml, split, qb, h, b, p); break;
       default: combine_rows<HD, 8>(recv, recv_ml, split, qb, h, b, p); break;
     }
-  } else {  // one stage: S = 2 or 4
+  } else {  // one stage: S = 2
     const int rows = 128 / S;
     const uint32_t send = base + static_cast<uint32_t>((128 - rows) * HD * 4);
     const uint32_t send_ml = base + C::kOffSendML1;
@@ -732,10 +733,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
     if (!wait_bounded(bar_recv, 0, tmo)) *abort_flag = 1;
     __syncwarp();
     asm volatile("barrier.cluster.arrive.aligned;" ::: "memory");
-    if (S == 2)
-      combine_own_rows<HD, 2>(o, m_run, l_run, recv, recv_ml, split, qb, h, b, p);
-    else
-      combine_own_rows<HD, 4>(o, m_run, l_run, recv, recv_ml, split, qb, h, b, p);
+    combine_own_rows<HD, 2>(o, m_run, l_run, recv, recv_ml, split, qb, h, b, p);
   }
   __syncwarp();
   asm volatile("barrier.cluster.wait.aligned;" ::: "memory");
@@ -920,9 +918,13 @@ extern "C" int dv_text_attention(const void* q, int batch, int n_q_heads, int n_
   int split2 = 1, split1 = 1;
   for (int s : {2, 4, 8}) {
     if (s <= blocks_max && units * s <= sms) split2 = s;
-    if (s <= 4 && s <= blocks_max && units * s <= 2LL * sms) split1 = s;  // one stage: S <= 4
+    if (s == 2 && s <= blocks_max && units * s <= 2LL * sms) split1 = s;
   }
-  const bool one_stage = split1 > split2;
+  // One stage (two CTAs per SM, clusters of 2) only where two stages cannot split the keys at
+  // all: measured on GB300 it then beats unsplit key runs (16.0 vs 18.0 us per layer at 128
+  // clusters of 6 key blocks), while clusters of 4 lose to two stages in clusters of 2 (18.3 vs
+  // 17.1 us at 64 clusters of 11 blocks).
+  const bool one_stage = split2 == 1 && split1 == 2;
   const int splits = one_stage ? split1 : split2;
   const cudaStream_t cs = static_cast<cudaStream_t>(stream);
   const int u = static_cast<int>(units);

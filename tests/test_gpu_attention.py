@@ -164,11 +164,12 @@ def test_attention_kernel_on_exact_inputs(hd, hq, hkv, nt):
 
 # Launch shapes that reach every kernel variant and cluster size the launcher picks (clusters =
 # batch x kv heads x 128-row query blocks; cluster size S = the largest of 2, 4, 8 within the key
-# blocks with one CTA per SM (two stages), or of 2, 4 with two CTAs per SM (one stage) when
-# that is larger, on 152 SMs):
-#   two stages, S = 8: 2 clusters, 9 key blocks; two stages, S = 4: 24 clusters;
-#   one stage, S = 2: 80 clusters, 3 key blocks; one stage, S = 4: 64 clusters (64 of 128 query
-#   rows valid) and 48 clusters (tiles of 128, 128 and 94 query rows).
+# blocks with one CTA per SM (two stages); where that is 1, one stage with two CTAs per SM in
+# clusters of 2 if those fit, on 152 SMs):
+#   two stages, S = 8: 2 clusters, 9 key blocks; two stages, S = 4: 24 clusters; two stages,
+#   S = 2: 64 clusters (64 of 128 query rows valid) and 48 clusters (tiles of 128, 128 and 94
+#   query rows); one stage, S = 2: 80 clusters of 16 query rows and 120 clusters (tiles of 128
+#   and 72 rows), 3 key blocks.
 @pytest.mark.parametrize("hd,B,hq,hkv,nt,n_keys,S", [
     (128, 1, 8, 2, 30, [1100], 1152),
     (64, 1, 8, 2, 30, [1100], 1152),
@@ -178,6 +179,7 @@ def test_attention_kernel_on_exact_inputs(hd, hq, hkv, nt):
     (64, 4, 20, 20, 16, [300, 290, 300, 257], 320),
     (64, 2, 32, 32, 64, [700, 650], 768),
     (128, 4, 28, 4, 50, [700, 650, 700, 690], 768),
+    (128, 3, 40, 20, 100, [300, 290, 277], 320),
 ])
 def test_attention_every_cluster_shape(hd, B, hq, hkv, nt, n_keys, S):
     _exact_case(hd, B, hq, hkv, nt, n_keys, S, 500 + hd + B + hq,
@@ -187,8 +189,8 @@ def test_attention_every_cluster_shape(hd, B, hq, hkv, nt, n_keys, S):
 @pytest.mark.parametrize("hd,B,hq,hkv,nt,n_keys,S,gain", [
     # two stages, 8-CTA clusters, 2 key blocks per CTA; keys growing with the slot
     (128, 1, 8, 2, 30, [2000], 2048, "rise"),
-    # one stage, 4-CTA clusters, 4 key blocks per CTA; two stages, 4-CTA clusters, 8 blocks
-    (128, 4, 28, 4, 50, [2000, 1900, 2000, 1950], 2048, "rise"),
+    # one stage, 2-CTA clusters, 8 key blocks per CTA; two stages, 4-CTA clusters, 8 blocks
+    (128, 4, 20, 20, 16, [2000, 1900, 2000, 1950], 2048, "rise"),
     (64, 2, 12, 12, 20, [4000, 3900], 4096, "fall"),
 ])
 def test_attention_running_maximum_grows_across_blocks(hd, B, hq, hkv, nt, n_keys, S, gain):
