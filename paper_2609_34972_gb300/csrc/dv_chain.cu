@@ -9,18 +9,24 @@
 //     operand of its part of the down-projection and the source of the TMA store of M_l.
 // Per layer:
 //   1. down-projection partial: z_s = bf16(M_{l-1})[:, slice] D_l[:, slice]^T (TMEM, fp32);
-//   2. the partial goes to shared memory (over the bf16 slice, whose readers are done) and,
-//      after a cluster barrier, CTA s sums rows [s 128 / S, (s + 1) 128 / S) over the S partials
-//      through distributed shared memory in the fixed order 0 .. S-1, applies SiLU and writes
-//      bf16 h straight into the h tile (A operand of the up-projection) of every CTA;
-//   3. after a second cluster barrier: state += h U_l[slice, :]^T (TMEM);
+//   2. the partial goes to shared memory (over the bf16 slice, whose readers are done). CTA s
+//      owns rows [s 128 / S, (s + 1) 128 / S): every CTA sends each peer the peer's rows of its
+//      partial by bulk copies into the peer's D buffer (read by then), completing on the peer's
+//      barrier. CTA s sums its rows over the S partials in the fixed order 0 .. S-1, applies
+//      SiLU, writes bf16 h into its h tile (A operand of the up-projection) and sends its rows of
+//      h to every peer's h tile the same way;
+//   3. once all h rows have landed: state += h U_l[slice, :]^T (TMEM);
 //   4. the state slice is read back, its bf16 rounding written over the bf16 slice (next layer's
 //      A operand, then stored to the stacked M_l by TMA) and its rows' sums of squares written to
 //      `part` (the K/V stage's RMS statistic adds the S partials).
-// D_{l+1} and U_{l+1} load (TMA) while the rest of layer l runs. Only bf16 M_l and the partial
-// sums of squares leave the chip; the state never does. Every wait is bounded; a CTA that gives
-// up keeps passing the cluster barriers (so its peers finish), stops issuing work, drains what
-// it issued and flags the plan's status word.
+// One cluster barrier per layer (arrival once the down MMA has read D_l, wait before sending z)
+// keeps a CTA from sending into a peer's D buffer too early; every other ordering follows from
+// the data: a CTA sends z_{l+1} only after it has all of h_l, so every receiver has finished
+// with z_l, and so on. D_{l+1} loads once the z rows are summed, U_{l+1} after the up MMA.
+// Only bf16 M_l and the partial sums of squares leave the chip; the state never does. Every
+// wait is bounded; a CTA that gives up keeps passing the cluster barriers and keeps sending (so
+// its peers' waits end and no copy lands after a CTA has exited), stops issuing MMAs and loads,
+// drains what it issued and flags the plan's status word.
 #include "../../include/dv.h"
 #include "dv_internal.h"
 #include "dv_ptx.cuh"
@@ -40,11 +46,15 @@ struct ChainCfg {
   static constexpr int kD = SPC * kDslab;
   static constexpr int kUslab = CW * 128;         // U_l: CW rows x 64 rank columns
   static constexpr int kU = (RP / 64) * kUslab;
+  // The peers' z rows land in the D buffer and past it: (S - 1) ceil(128 / S) rows, at most
+  // 130 (S = 14), of RP fp32.
+  static constexpr int kRecvMax = 130 * RP * 4;
+  static constexpr int kDRegion = kD > kRecvMax ? kD : kRecvMax;
   static constexpr int kOffA = 0;
   static constexpr int kOffH = kOffA + kA;
-  static constexpr int kOffD = kOffH + kH;
-  static constexpr int kOffU = kOffD + kD;
-  static constexpr int kEnd = kOffU + kU;
+  static constexpr int kOffU = kOffH + kH;
+  static constexpr int kOffD = kOffU + kU;
+  static constexpr int kEnd = kOffD + kDRegion;
   static constexpr int kZ = 128 * RP * 4;         // fp32 partial z over the bf16 slice
   static constexpr int kSmemBytes = kEnd + 1024 + 256;
   static constexpr int kTmemCols = CW + RP <= 256 ? 256 : 512;
@@ -71,19 +81,18 @@ __device__ __forceinline__ uint32_t n_cluster_ctas() {
   return r;
 }
 
-__device__ __forceinline__ float4 ld_cluster_f4(uint32_t caddr) {
-  float4 v;
-  asm volatile("ld.shared::cluster.v4.f32 {%0, %1, %2, %3}, [%4];"
-               : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w)
-               : "r"(caddr)
-               : "memory");
-  return v;
+// Bulk copy of `bytes` from this CTA's shared memory to a shared::cluster address (a peer's),
+// completing as transaction bytes on the peer's barrier `cbar`.
+__device__ __forceinline__ void bulk_copy_to_peer(uint32_t dst_cluster, uint32_t src, uint32_t bytes,
+                                                  uint32_t cbar) {
+  asm volatile(
+      "cp.async.bulk.shared::cluster.shared::cta.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];"
+      ::"r"(dst_cluster), "r"(src), "r"(bytes), "r"(cbar)
+      : "memory");
 }
 
-__device__ __forceinline__ void st_cluster_u2(uint32_t caddr, uint2 v) {
-  asm volatile("st.shared::cluster.v2.b32 [%0], {%1, %2};" ::"r"(caddr), "r"(v.x), "r"(v.y)
-               : "memory");
-}
+__device__ __forceinline__ int chain_row_lo(int s, int S) { return s * 128 / S; }
+__device__ __forceinline__ int peer_slot(int src, int self) { return src < self ? src : src - 1; }
 
 // Registers -> TMEM: lane i of the warp writes TMEM lane (taddr.lane + i), 32 columns.
 __device__ __forceinline__ void tmem_st32(uint32_t taddr, const uint32_t (&r)[32]) {
@@ -123,9 +132,6 @@ __device__ __forceinline__ void bulk_wait0() { asm volatile("cp.async.bulk.wait_
 __device__ __forceinline__ void fence_proxy_async_cta() {
   asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
 }
-__device__ __forceinline__ void fence_proxy_async_cluster() {
-  asm volatile("fence.proxy.async.shared::cluster;" ::: "memory");
-}
 
 __device__ __forceinline__ bool wait_bounded(uint32_t bar, uint32_t parity, uint64_t timeout_ns) {
   int never = 0;
@@ -151,8 +157,8 @@ __global__ void __launch_bounds__(kChainThreads, 1)
   uint64_t* bars = reinterpret_cast<uint64_t*>(base_ptr + C::kEnd);
   const uint32_t bar0 = smem_addr(bars);
   const uint32_t bar_x = bar0, bar_d = bar0 + 8, bar_u = bar0 + 16, bar_z = bar0 + 24,
-                 bar_up = bar0 + 32, bar_drain = bar0 + 40;
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 6);
+                 bar_up = bar0 + 32, bar_drain = bar0 + 40, bar_rz = bar0 + 48, bar_rh = bar0 + 56;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 8);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
 
   const int tid = threadIdx.x, warp = tid >> 5;
@@ -162,6 +168,7 @@ __global__ void __launch_bounds__(kChainThreads, 1)
   const int m = static_cast<int>(cluster_id_x());
   const int col0 = s * CW, row0 = m * 128;
   const int t = row0 + tid;  // this thread's token row
+  const int r_lo = chain_row_lo(s, S), n_rows = chain_row_lo(s + 1, S) - r_lo;  // rows summed here
   const uint32_t sA = base + C::kOffA, sH = base + C::kOffH, sD = base + C::kOffD,
                  sU = base + C::kOffU;
   float* zpart = reinterpret_cast<float*>(base_ptr + C::kOffA);
@@ -173,6 +180,8 @@ __global__ void __launch_bounds__(kChainThreads, 1)
     mbar_init(bar_z, 1);
     mbar_init(bar_up, 1);
     mbar_init(bar_drain, 1);
+    mbar_init(bar_rz, 1);  // the peers' z rows of this CTA, once per layer
+    mbar_init(bar_rh, 1);  // the peers' h rows, once per layer
     *abort_flag = 0;
     fence_barrier_init();
   }
@@ -242,6 +251,10 @@ __global__ void __launch_bounds__(kChainThreads, 1)
 
   for (int l = 0; l < p.L; ++l) {
     const uint32_t ph = static_cast<uint32_t>(l) & 1u;
+    if (tid == 0) {  // this layer's transfers into this CTA: the peers' z rows, then h rows
+      mbar_arrive_expect_tx(bar_rz, static_cast<uint32_t>((S - 1) * n_rows * RP * 4));
+      mbar_arrive_expect_tx(bar_rh, static_cast<uint32_t>((128 - n_rows) * RP * 2));
+    }
 
     // (1) down-projection partial z = bf16(M_{l-1})[:, slice] D_l[:, slice]^T; store M_{l-1}
     if (tid == 0 && ok && !*abort_flag) {
@@ -272,6 +285,9 @@ __global__ void __launch_bounds__(kChainThreads, 1)
       bulk_wait_read0();
       if (zok) mma_open = false;
     }
+    // The down MMA has read D_l (or this CTA issues no more MMAs): the D buffer may receive.
+    __syncwarp();
+    asm volatile("barrier.cluster.arrive.aligned;" ::: "memory");
     zok = __syncthreads_and(zok) != 0;
     if (zok) {
       tc_fence_after();
@@ -290,66 +306,91 @@ __global__ void __launch_bounds__(kChainThreads, 1)
                           __uint_as_float(r[4 * q + 2]), __uint_as_float(r[4 * q + 3]));
         }
       }
-      if (tid == 0 && l + 1 < p.L) load_d(l + 1);  // the D buffer is free
     }
     ok = zok;
+    fence_proxy_async_cta();  // the partial is read by the bulk copies
     tc_fence_before();
+    __syncthreads();
     __syncwarp();
-    cluster_sync();
+    asm volatile("barrier.cluster.wait.aligned;" ::: "memory");  // every D buffer is free
+    // Each peer's rows of this partial into its D buffer, slot peer_slot(s, peer). A CTA that
+    // gave up sends too, so that every receiver's wait ends.
+    if (tid == 0) {
+      for (int dd = 0; dd < S; ++dd) {
+        if (dd == s) continue;
+        const int lo = chain_row_lo(dd, S), n = chain_row_lo(dd + 1, S) - lo;
+        const uint32_t rank = static_cast<uint32_t>(dd);
+        bulk_copy_to_peer(
+            map_to_rank(sD + static_cast<uint32_t>(peer_slot(s, dd) * n * RP * 4), rank),
+            sA + static_cast<uint32_t>(lo * RP * 4), static_cast<uint32_t>(n * RP * 4),
+            map_to_rank(bar_rz, rank));
+      }
+    }
 
-    // (3) rows [s 128 / S, (s + 1) 128 / S): sum the S partials in order, SiLU, bf16 h into the
-    // h tile of every CTA (8-byte pieces, swizzled as the MMA reads them). One item is 4 values
-    // (one float4) of one row: its S remote loads are all in flight before the sum.
+    // (3) rows [r_lo, r_lo + n_rows): sum the S partials in order (this CTA's own from its
+    // partial, the peers' from the D buffer), SiLU, bf16 h into this CTA's h tile (8-byte
+    // pieces, swizzled as the MMA reads them) and into H. Not cut short by the abort flag: the
+    // copies into this CTA must land before it may exit.
+    if (!wait_bounded(bar_rz, ph, tmo)) *abort_flag = 1;
     {
-      const int r_lo = s * 128 / S, r_hi = (s + 1) * 128 / S;
-      const int items = (r_hi - r_lo) * (RP / 4);
+      const int items = n_rows * (RP / 4);
 #pragma unroll 1
       for (int it = tid; it < items; it += kChainThreads) {
-        const int row = r_lo + it / (RP / 4), c4 = it % (RP / 4);
-        const uint32_t zl = smem_addr(zpart + row * RP) + ((c4 ^ (row & 7)) << 4);
-        float4 v[16];
-#pragma unroll
-        for (int b = 0; b < 16; ++b)
-          if (b < S) v[b] = ld_cluster_f4(map_to_rank(zl, static_cast<uint32_t>(b)));
+        const int rr = it / (RP / 4), row = r_lo + rr, c4 = it % (RP / 4);
+        const uint32_t chunk = static_cast<uint32_t>((c4 ^ (row & 7)) << 4);
         float4 z = make_float4(0.0f, 0.0f, 0.0f, 0.0f);
-#pragma unroll
-        for (int b = 0; b < 16; ++b) {
-          if (b < S) {
-            z.x += v[b].x;
-            z.y += v[b].y;
-            z.z += v[b].z;
-            z.w += v[b].w;
-          }
+        for (int b = 0; b < S; ++b) {
+          const uint32_t src =
+              b == s ? sA + static_cast<uint32_t>(row * RP * 4) + chunk
+                     : sD + static_cast<uint32_t>((peer_slot(b, s) * n_rows + rr) * RP * 4) + chunk;
+          const float4 v = *reinterpret_cast<const float4*>(__cvta_shared_to_generic(src));
+          z.x += v.x;
+          z.y += v.y;
+          z.z += v.z;
+          z.w += v.w;
         }
         uint2 hv;
         hv.x = pack_bf16x2(silu(z.x), silu(z.y));
         hv.y = pack_bf16x2(silu(z.z), silu(z.w));
         // columns 4 c4 .. 4 c4 + 3: slab c4 / 16, 16-byte chunk (c4 % 16) / 2, half c4 % 2
-        const uint32_t hl = sH + (c4 / 16) * C::kSlab + sw128(row, (c4 % 16) / 2) + (c4 % 2) * 8;
-        for (int b = 0; b < S; ++b) st_cluster_u2(map_to_rank(hl, static_cast<uint32_t>(b)), hv);
+        *reinterpret_cast<uint2*>(base_ptr + C::kOffH + (c4 / 16) * C::kSlab +
+                                  sw128(row, (c4 % 16) / 2) + (c4 % 2) * 8) = hv;
         if (row0 + row < p.M)
           *reinterpret_cast<uint2*>(p.H + static_cast<long long>(row0 + row) * p.ldh + l * RP +
                                     c4 * 4) = hv;
       }
     }
-    fence_proxy_async_cluster();
-    __syncwarp();
-    cluster_sync();
+    fence_proxy_async_cta();  // this CTA's h rows: read by the bulk copies and the up MMA
+    __syncthreads();
+    if (tid == 0) {
+      // this CTA's rows of h into every peer's h tile (the same bytes of each 64-column slab)
+      for (int dd = 0; dd < S; ++dd) {
+        if (dd == s) continue;
+        const uint32_t rank = static_cast<uint32_t>(dd), cbar = map_to_rank(bar_rh, rank);
+        for (int j = 0; j < RP / 64; ++j) {
+          const uint32_t off = sH + static_cast<uint32_t>(j * C::kSlab + r_lo * 128);
+          bulk_copy_to_peer(map_to_rank(off, rank), off, static_cast<uint32_t>(n_rows * 128), cbar);
+        }
+      }
+      if (ok && !*abort_flag && l + 1 < p.L) load_d(l + 1);  // the z rows are summed
+    }
 
-    // (4) state += h U_l[slice, :]^T
-    if (tid == 0 && ok && !*abort_flag) {
-      fence_proxy_async_cta();
-      tc_fence_after();
-      if (mbar_wait(bar_u, ph, abort_flag, tmo)) {
-        ++u_waits;
-        const uint32_t idesc = idesc_bf16_f32(128, CW);
-        for (int j = 0; j < RP / 64; ++j)
+    // (4) state += h U_l[slice, :]^T, once every peer's h rows have landed
+    if (tid == 0) {
+      if (!wait_bounded(bar_rh, ph, tmo)) *abort_flag = 1;
+      if (ok && !*abort_flag) {
+        tc_fence_after();
+        if (mbar_wait(bar_u, ph, abort_flag, tmo)) {
+          ++u_waits;
+          const uint32_t idesc = idesc_bf16_f32(128, CW);
+          for (int j = 0; j < RP / 64; ++j)
 #pragma unroll
-          for (int k = 0; k < 4; ++k)
-            umma_bf16(t_state, sdesc_kmajor_sw128(sH + j * C::kSlab + 32u * k),
-                      sdesc_kmajor_sw128(sU + j * C::kUslab + 32u * k), idesc, 1u);
-        umma_commit(bar_up);
-        mma_open = true;
+            for (int k = 0; k < 4; ++k)
+              umma_bf16(t_state, sdesc_kmajor_sw128(sH + j * C::kSlab + 32u * k),
+                        sdesc_kmajor_sw128(sU + j * C::kUslab + 32u * k), idesc, 1u);
+          umma_commit(bar_up);
+          mma_open = true;
+        }
       }
     }
     bool uok = ok && mbar_wait(bar_up, ph, abort_flag, tmo);
