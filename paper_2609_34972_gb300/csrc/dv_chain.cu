@@ -9,7 +9,8 @@
 //     operand of its part of the down-projection and the source of the TMA store of M_l.
 // Per layer:
 //   1. down-projection partial: z_s = bf16(M_{l-1})[:, slice] D_l[:, slice]^T (TMEM, fp32);
-//   2. the partial goes to shared memory (over the bf16 slice, whose readers are done). CTA s
+//   2. the partial goes to shared memory (a region of its own where shared memory allows, else
+//      over the bf16 slice once its readers are done). CTA s
 //      owns rows [s 128 / S, (s + 1) 128 / S): every CTA sends each peer the peer's rows of its
 //      partial by bulk copies into the peer's D buffer (read by then), completing on the peer's
 //      barrier. CTA s sums its rows over the S partials in the fixed order 0 .. S-1, applies
@@ -54,11 +55,16 @@ struct ChainCfg {
   static constexpr int kOffH = kOffA + kA;
   static constexpr int kOffU = kOffH + kH;
   static constexpr int kOffD = kOffU + kU;
-  static constexpr int kEnd = kOffD + kDRegion;
-  static constexpr int kZ = 128 * RP * 4;         // fp32 partial z over the bf16 slice
+  // The fp32 partial z gets a region of its own where shared memory allows, so the store of
+  // M_{l-1} (reading the bf16 slice) runs alongside the rest of the layer; otherwise it reuses
+  // the bf16 slice once the store has read it.
+  static constexpr int kZ = 128 * RP * 4;
+  static constexpr bool kZOwn = kOffD + kDRegion + kZ + 1024 + 256 <= 232448;
+  static constexpr int kOffZ = kZOwn ? kOffD + kDRegion : kOffA;
+  static constexpr int kEnd = kOffD + kDRegion + (kZOwn ? kZ : 0);
   static constexpr int kSmemBytes = kEnd + 1024 + 256;
   static constexpr int kTmemCols = CW + RP <= 256 ? 256 : 512;
-  static_assert(kZ <= kA, "the partial z reuses the bf16 state slice");
+  static_assert(kZOwn || kZ <= kA, "the partial z reuses the bf16 state slice");
   static_assert(kSmemBytes <= 232448, "shared memory of one CTA");
   static_assert(kDslab % 1024 == 0 && kUslab % 1024 == 0, "tiles stay 1024-byte aligned");
 };
@@ -171,7 +177,8 @@ __global__ void __launch_bounds__(kChainThreads, 1)
   const int r_lo = chain_row_lo(s, S), n_rows = chain_row_lo(s + 1, S) - r_lo;  // rows summed here
   const uint32_t sA = base + C::kOffA, sH = base + C::kOffH, sD = base + C::kOffD,
                  sU = base + C::kOffU;
-  float* zpart = reinterpret_cast<float*>(base_ptr + C::kOffA);
+  float* zpart = reinterpret_cast<float*>(base_ptr + C::kOffZ);
+  const uint32_t sZ = base + C::kOffZ;
 
   if (tid == 0) {
     mbar_init(bar_x, 1);
@@ -279,15 +286,18 @@ __global__ void __launch_bounds__(kChainThreads, 1)
       }
     }
 
-    // (2) z partial -> shared memory, over the bf16 slice (down MMA and store have read it)
+    // (2) z partial -> shared memory (over the bf16 slice: once the down MMA and the store of
+    // M_{l-1} have read it)
     bool zok = ok && mbar_wait(bar_z, ph, abort_flag, tmo);
     if (tid == 0) {
-      bulk_wait_read0();
+      if (!C::kZOwn) bulk_wait_read0();
       if (zok) mma_open = false;
     }
     // The down MMA has read D_l (or this CTA issues no more MMAs): the D buffer may receive.
+    // Relaxed: the arrival publishes no data, and a release would first wait for this thread's
+    // earlier global stores (h rows, sums of squares) to complete, about 2 us.
     __syncwarp();
-    asm volatile("barrier.cluster.arrive.aligned;" ::: "memory");
+    asm volatile("barrier.cluster.arrive.relaxed.aligned;" ::: "memory");
     zok = __syncthreads_and(zok) != 0;
     if (zok) {
       tc_fence_after();
@@ -322,7 +332,7 @@ __global__ void __launch_bounds__(kChainThreads, 1)
         const uint32_t rank = static_cast<uint32_t>(dd);
         bulk_copy_to_peer(
             map_to_rank(sD + static_cast<uint32_t>(peer_slot(s, dd) * n * RP * 4), rank),
-            sA + static_cast<uint32_t>(lo * RP * 4), static_cast<uint32_t>(n * RP * 4),
+            sZ + static_cast<uint32_t>(lo * RP * 4), static_cast<uint32_t>(n * RP * 4),
             map_to_rank(bar_rz, rank));
       }
     }
@@ -341,7 +351,7 @@ __global__ void __launch_bounds__(kChainThreads, 1)
         float4 z = make_float4(0.0f, 0.0f, 0.0f, 0.0f);
         for (int b = 0; b < S; ++b) {
           const uint32_t src =
-              b == s ? sA + static_cast<uint32_t>(row * RP * 4) + chunk
+              b == s ? sZ + static_cast<uint32_t>(row * RP * 4) + chunk
                      : sD + static_cast<uint32_t>((peer_slot(b, s) * n_rows + rr) * RP * 4) + chunk;
           const float4 v = *reinterpret_cast<const float4*>(__cvta_shared_to_generic(src));
           z.x += v.x;
@@ -375,9 +385,12 @@ __global__ void __launch_bounds__(kChainThreads, 1)
       if (ok && !*abort_flag && l + 1 < p.L) load_d(l + 1);  // the z rows are summed
     }
 
-    // (4) state += h U_l[slice, :]^T, once every peer's h rows have landed
+    // (4) state += h U_l[slice, :]^T, once every peer's h rows have landed. The readback after
+    // it overwrites the bf16 slice: the store of M_{l-1} must have read it (every thread's
+    // readback waits for this MMA).
     if (tid == 0) {
       if (!wait_bounded(bar_rh, ph, tmo)) *abort_flag = 1;
+      if (C::kZOwn) bulk_wait_read0();
       if (ok && !*abort_flag) {
         tc_fence_after();
         if (mbar_wait(bar_u, ph, abort_flag, tmo)) {
