@@ -323,11 +323,12 @@ __global__ void __launch_bounds__(kChainThreads, 1)
     __syncthreads();
     __syncwarp();
     asm volatile("barrier.cluster.wait.aligned;" ::: "memory");  // every D buffer is free
-    // Each peer's rows of this partial into its D buffer, slot peer_slot(s, peer). A CTA that
-    // gave up sends too, so that every receiver's wait ends.
-    if (tid == 0) {
-      for (int dd = 0; dd < S; ++dd) {
-        if (dd == s) continue;
+    // Each peer's rows of this partial into its D buffer, slot peer_slot(s, peer): lane dd of
+    // warp 0 sends to peer dd, so the copies issue in parallel. A CTA that gave up sends too, so
+    // that every receiver's wait ends.
+    if (warp == 0) {
+      const int dd = tid;
+      if (dd < S && dd != s) {
         const int lo = chain_row_lo(dd, S), n = chain_row_lo(dd + 1, S) - lo;
         const uint32_t rank = static_cast<uint32_t>(dd);
         bulk_copy_to_peer(
@@ -372,17 +373,18 @@ __global__ void __launch_bounds__(kChainThreads, 1)
     }
     fence_proxy_async_cta();  // this CTA's h rows: read by the bulk copies and the up MMA
     __syncthreads();
-    if (tid == 0) {
-      // this CTA's rows of h into every peer's h tile (the same bytes of each 64-column slab)
-      for (int dd = 0; dd < S; ++dd) {
-        if (dd == s) continue;
+    if (warp == 0) {
+      // this CTA's rows of h into every peer's h tile (the same bytes of each 64-column slab),
+      // lane dd to peer dd
+      const int dd = tid;
+      if (dd < S && dd != s) {
         const uint32_t rank = static_cast<uint32_t>(dd), cbar = map_to_rank(bar_rh, rank);
         for (int j = 0; j < RP / 64; ++j) {
           const uint32_t off = sH + static_cast<uint32_t>(j * C::kSlab + r_lo * 128);
           bulk_copy_to_peer(map_to_rank(off, rank), off, static_cast<uint32_t>(n_rows * 128), cbar);
         }
       }
-      if (ok && !*abort_flag && l + 1 < p.L) load_d(l + 1);  // the z rows are summed
+      if (tid == 0 && ok && !*abort_flag && l + 1 < p.L) load_d(l + 1);  // the z rows are summed
     }
 
     // (4) state += h U_l[slice, :]^T, once every peer's h rows have landed. The readback after
