@@ -67,6 +67,11 @@ struct AttnCfg {
   static constexpr int kOffStage = kOffQ + kKV;  // NST stages of [K | V]
   static constexpr int kStage = 2 * kKV;
   static constexpr int kEnd = kOffStage + NST * kStage;  // P lives in TMEM, not here
+  // TMEM: two score buffers (block j + 1's score MMA runs while block j finishes) and O at one
+  // CTA per SM; one score buffer and O at two.
+  static constexpr int kSBuf = NST == 2 ? 2 : 1;
+  static constexpr int kTmemCols = NST == 2 ? 512 : 256;
+  static constexpr int kTmemO = 128 * kSBuf;
   static constexpr int kMisc = 2048;                      // barriers, m, l, key end
   // Partial outputs received from the cluster: 128 rows of HD fp32 (16-byte chunks swizzled by
   // the row, no padding). With two stages they get a region of their own, so peers may write
@@ -454,7 +459,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
   float* recv_ml = reinterpret_cast<float*>(base_ptr + C::kEnd + 256);  // [S][m | l][128 / S]
   const uint32_t recv = base + C::kOffRecv;
 
-  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int tid = threadIdx.x, warp = tid >> 5;
   const uint64_t tmo = p.timeout_ns;
   const int split = static_cast<int>(cluster_ctarank());
   const int S = static_cast<int>(cluster_size());
@@ -484,7 +489,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
     fence_barrier_init();
   }
   if (warp == 0) {
-    tmem_alloc(smem_addr(tmem_slot), 256);
+    tmem_alloc(smem_addr(tmem_slot), C::kTmemCols);
     tmem_relinquish();
   }
   tc_fence_before();
@@ -506,7 +511,8 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
   atomicMax(key_end, last + 1);
   __syncthreads();
   const uint32_t tmem = *tmem_slot;
-  const uint32_t t_s = tmem, t_o = tmem + 128;
+  const uint32_t t_o = tmem + C::kTmemO;
+  auto t_s = [&](int j) { return tmem + static_cast<uint32_t>((j % C::kSBuf) * 128); };
   const uint32_t lane_base = static_cast<uint32_t>(warp * 32) << 16;
   const int n_blocks = (*key_end + kKeyBlock - 1) / kKeyBlock;
   const int kb0 = split * n_blocks / S, kb1 = (split + 1) * n_blocks / S;
@@ -532,6 +538,21 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
       tma_load_4d(sV(st) + ds * C::kTile, &tmV, bar_v(st), ds * 64, h, kb * kKeyBlock, b);
     last_v = j;
   };
+  auto issue_s = [&](int j) {  // thread 0: S_j = Q K_j^T into score buffer j % kSBuf
+    const int st = j % NST;
+    if (mbar_wait(bar_q, 0, abort_flag, tmo) &&
+        mbar_wait(bar_k(st), static_cast<uint32_t>(j / NST) & 1u, abort_flag, tmo)) {
+      tc_fence_after();
+      const uint32_t idesc = idesc_bf16_f32(128, kKeyBlock);
+      for (int ds = 0; ds < C::kSlabs; ++ds)
+#pragma unroll
+        for (int k = 0; k < 4; ++k)
+          umma_bf16(t_s(j), sdesc_kmajor_sw128(sQ + ds * C::kTile + 32u * k),
+                    sdesc_kmajor_sw128(sK(st) + ds * C::kTile + 32u * k), idesc,
+                    (ds | k) != 0 ? 1u : 0u);
+      umma_commit(bar_s);
+    }
+  };
 
   float m_run = -INFINITY, l_run = 0.0f;
 
@@ -542,6 +563,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
       tma_load_2d(sQ + ds * C::kTile, &tmQ, bar_q, ds * 64, q_row0);
     load_k(0);
     load_v(0);
+    issue_s(0);
   }
 
   bool ok = true;
@@ -549,29 +571,12 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
     const int st = j % NST, kb = kb0 + j;
     const uint32_t sph = static_cast<uint32_t>(j / NST) & 1u;  // phase of this stage's barriers
     const uint32_t ph = static_cast<uint32_t>(j) & 1u;        // phase of bar_s / bar_o
-    if (warp == 0) {
-      if (lane == 0) {
-        // Two stages: the other stage was freed by the previous block. One stage: K of this
-        // block was issued once the previous score MMA had read K, V once the previous P V
-        // MMA had read V.
-        if (NST == 2 && j + 1 < n_mine) {
-          load_k(j + 1);
-          load_v(j + 1);
-        }
-        // S = Q K^T
-        if (mbar_wait(bar_q, 0, abort_flag, tmo) && mbar_wait(bar_k(st), sph, abort_flag, tmo)) {
-          tc_fence_after();
-          const uint32_t idesc = idesc_bf16_f32(128, kKeyBlock);
-          for (int ds = 0; ds < C::kSlabs; ++ds)
-#pragma unroll
-            for (int k = 0; k < 4; ++k)
-              umma_bf16(t_s, sdesc_kmajor_sw128(sQ + ds * C::kTile + 32u * k),
-                        sdesc_kmajor_sw128(sK(st) + ds * C::kTile + 32u * k), idesc,
-                        (ds | k) != 0 ? 1u : 0u);
-          umma_commit(bar_s);
-        }
-      }
-      __syncwarp();
+    // Two stages: the other stage was freed by the previous block. One stage: K of this block
+    // was issued once the previous score MMA had read K, V once the previous P V MMA had read V.
+    // S_j itself was issued with the previous block (or before the loop).
+    if (NST == 2 && tid == 0 && j + 1 < n_mine) {
+      load_k(j + 1);
+      load_v(j + 1);
     }
 
     // Scores -> probabilities (this thread: query row tid).
@@ -582,7 +587,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
       // the row's 128 scores in one TMEM round trip; keys past the row's last slot are masked
       uint32_t r[kKeyBlock];
 #pragma unroll
-      for (int c = 0; c < kKeyBlock / 32; ++c) tmem_ld32(t_s + lane_base + c * 32, chunk32(r, c));
+      for (int c = 0; c < kKeyBlock / 32; ++c) tmem_ld32(t_s(j) + lane_base + c * 32, chunk32(r, c));
       tmem_ld_wait();
 #pragma unroll
       for (int c = 0; c < kKeyBlock / 32; ++c) reg_fence32(chunk32(r, c));
@@ -644,7 +649,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
           lb[(u / 2) % 4] += p0 + p1;
           pk[u / 2] = pack_bf16x2(p0, p1);
         }
-        tmem_st32(t_s + lane_base + c * 32, pk);
+        tmem_st32(t_s(j) + lane_base + c * 32, pk);
       }
       tmem_st_wait();
       l_run = alpha * l_run + ((lb[0] + lb[1]) + (lb[2] + lb[3]));
@@ -660,12 +665,19 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
       const uint32_t idesc = idesc_bf16_f32(128, HD) | (1u << 16);
 #pragma unroll
       for (int kk = 0; kk < kKeyBlock / 16; ++kk)
-        umma_bf16_tmem_a(t_o, t_s + kk * 8, sdesc_mnmajor_sw128(sV(st) + kk * 16 * 128, C::kTile),
-                         idesc, (j | kk) != 0 ? 1u : 0u);
+        umma_bf16_tmem_a(t_o, t_s(j) + kk * 8,
+                         sdesc_mnmajor_sw128(sV(st) + kk * 16 * 128, C::kTile), idesc,
+                         (j | kk) != 0 ? 1u : 0u);
       umma_commit(bar_o);
+      // Two score buffers: S_{j+1} runs behind P V (its buffer's P_{j-1} was read by the previous
+      // P V, which has completed).
+      if (C::kSBuf == 2 && j + 1 < n_mine) issue_s(j + 1);
     }
     ok = ok && mbar_wait(bar_o, ph, abort_flag, tmo);
-    if (NST == 1 && tid == 0 && ok && j + 1 < n_mine) load_v(j + 1);  // V slot read
+    if (NST == 1 && tid == 0 && ok && j + 1 < n_mine) {
+      load_v(j + 1);  // V slot read
+      issue_s(j + 1);  // P_j (in the one score buffer) read
+    }
     tc_fence_before();
     ok = __syncthreads_and(ok) != 0;
   }
@@ -740,7 +752,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
 
   if (warp == 0) {
     tc_fence_after();
-    tmem_dealloc(tmem, 256);
+    tmem_dealloc(tmem, C::kTmemCols);
   }
   if (tid == 0 && *abort_flag) atomicExch(&g_attn_status, DV_ERR_DEVICE_TIMEOUT);
 }
