@@ -55,16 +55,17 @@ struct ChainCfg {
   static constexpr int kOffH = kOffA + kA;
   static constexpr int kOffU = kOffH + kH;
   static constexpr int kOffD = kOffU + kU;
-  // The fp32 partial z gets a region of its own where shared memory allows, so the store of
-  // M_{l-1} (reading the bf16 slice) runs alongside the rest of the layer; otherwise it reuses
-  // the bf16 slice once the store has read it.
+  // The fp32 partial z gets a region of its own where shared memory allows. Otherwise it takes
+  // the U buffer: U_l then loads once the peers have acknowledged z (every copy out of the
+  // partial has landed), still well before the up MMA. Either way the store of M_{l-1},
+  // reading the bf16 slice, runs alongside the rest of the layer.
   static constexpr int kZ = 128 * RP * 4;
   static constexpr bool kZOwn = kOffD + kDRegion + kZ + 1024 + 256 <= 232448;
-  static constexpr int kOffZ = kZOwn ? kOffD + kDRegion : kOffA;
+  static constexpr int kOffZ = kZOwn ? kOffD + kDRegion : kOffU;
   static constexpr int kEnd = kOffD + kDRegion + (kZOwn ? kZ : 0);
   static constexpr int kSmemBytes = kEnd + 1024 + 256;
   static constexpr int kTmemCols = CW + RP <= 256 ? 256 : 512;
-  static_assert(kZOwn || kZ <= kA, "the partial z reuses the bf16 state slice");
+  static_assert(kZOwn || kZ <= kU, "the partial z takes the U buffer");
   static_assert(kSmemBytes <= 232448, "shared memory of one CTA");
   static_assert(kDslab % 1024 == 0 && kUslab % 1024 == 0, "tiles stay 1024-byte aligned");
 };
@@ -98,6 +99,13 @@ __device__ __forceinline__ void bulk_copy_to_peer(uint32_t dst_cluster, uint32_t
 }
 
 __device__ __forceinline__ int chain_row_lo(int s, int S) { return s * 128 / S; }
+
+// Arrive on an mbarrier given by a shared::cluster address (a peer's), with no release: the
+// arrival publishes no data, and a release would first wait for this thread's global stores.
+__device__ __forceinline__ void mbar_arrive_cluster_relaxed(uint32_t cbar) {
+  asm volatile("mbarrier.arrive.relaxed.cluster.shared::cluster.b64 _, [%0];" ::"r"(cbar)
+               : "memory");
+}
 __device__ __forceinline__ int peer_slot(int src, int self) { return src < self ? src : src - 1; }
 
 // Registers -> TMEM: lane i of the warp writes TMEM lane (taddr.lane + i), 32 columns.
@@ -163,8 +171,9 @@ __global__ void __launch_bounds__(kChainThreads, 1)
   uint64_t* bars = reinterpret_cast<uint64_t*>(base_ptr + C::kEnd);
   const uint32_t bar0 = smem_addr(bars);
   const uint32_t bar_x = bar0, bar_d = bar0 + 8, bar_u = bar0 + 16, bar_z = bar0 + 24,
-                 bar_up = bar0 + 32, bar_drain = bar0 + 40, bar_rz = bar0 + 48, bar_rh = bar0 + 56;
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 8);
+                 bar_up = bar0 + 32, bar_drain = bar0 + 40, bar_rz = bar0 + 48, bar_rh = bar0 + 56,
+                 bar_zs = bar0 + 64;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 10);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
 
   const int tid = threadIdx.x, warp = tid >> 5;
@@ -189,6 +198,8 @@ __global__ void __launch_bounds__(kChainThreads, 1)
     mbar_init(bar_drain, 1);
     mbar_init(bar_rz, 1);  // the peers' z rows of this CTA, once per layer
     mbar_init(bar_rh, 1);  // the peers' h rows, once per layer
+    // partial z in the U buffer: every peer acknowledges that this CTA's z rows have landed
+    if (!C::kZOwn && S > 1) mbar_init(bar_zs, S - 1);
     *abort_flag = 0;
     fence_barrier_init();
   }
@@ -229,7 +240,7 @@ __global__ void __launch_bounds__(kChainThreads, 1)
     mbar_arrive_expect_tx(bar_x, C::kA);
     for (int j = 0; j < SPC; ++j) tma_load_2d(sA + j * C::kSlab, &tmX, bar_x, col0 + 64 * j, row0);
     load_d(0);
-    load_u(0);
+    if (C::kZOwn) load_u(0);  // else once the layer's z rows have left the U buffer
   }
 
   // M_0 = E: the state slice in TMEM is the fp32 widening of the bf16 slice just loaded.
@@ -290,7 +301,6 @@ __global__ void __launch_bounds__(kChainThreads, 1)
     // M_{l-1} have read it)
     bool zok = ok && mbar_wait(bar_z, ph, abort_flag, tmo);
     if (tid == 0) {
-      if (!C::kZOwn) bulk_wait_read0();
       if (zok) mma_open = false;
     }
     // The down MMA has read D_l (or this CTA issues no more MMAs): the D buffer may receive.
@@ -343,6 +353,10 @@ __global__ void __launch_bounds__(kChainThreads, 1)
     // pieces, swizzled as the MMA reads them) and into H. Not cut short by the abort flag: the
     // copies into this CTA must land before it may exit.
     if (!wait_bounded(bar_rz, ph, tmo)) *abort_flag = 1;
+    // Partial z in the U buffer: tell each peer that its z rows have landed here (thread i
+    // < S - 1, one peer each; relaxed, as nothing is published).
+    if (!C::kZOwn && tid < S - 1)
+      mbar_arrive_cluster_relaxed(map_to_rank(bar_zs, static_cast<uint32_t>(tid < s ? tid : tid + 1)));
     {
       const int items = n_rows * (RP / 4);
 #pragma unroll 1
@@ -386,13 +400,17 @@ __global__ void __launch_bounds__(kChainThreads, 1)
       }
       if (tid == 0 && ok && !*abort_flag && l + 1 < p.L) load_d(l + 1);  // the z rows are summed
     }
+    if (!C::kZOwn && tid == 0) {  // every copy out of the partial has landed: U_l may load
+      if (S > 1 && !wait_bounded(bar_zs, ph, tmo)) *abort_flag = 1;
+      if (ok && !*abort_flag) load_u(l);
+    }
 
     // (4) state += h U_l[slice, :]^T, once every peer's h rows have landed. The readback after
     // it overwrites the bf16 slice: the store of M_{l-1} must have read it (every thread's
     // readback waits for this MMA).
     if (tid == 0) {
       if (!wait_bounded(bar_rh, ph, tmo)) *abort_flag = 1;
-      if (C::kZOwn) bulk_wait_read0();
+      bulk_wait_read0();
       if (ok && !*abort_flag) {
         tc_fence_after();
         if (mbar_wait(bar_u, ph, abort_flag, tmo)) {
@@ -411,7 +429,7 @@ __global__ void __launch_bounds__(kChainThreads, 1)
     bool uok = ok && mbar_wait(bar_up, ph, abort_flag, tmo);
     if (tid == 0 && uok) {
       mma_open = false;
-      if (l + 1 < p.L) load_u(l + 1);  // the U buffer is free
+      if (C::kZOwn && l + 1 < p.L) load_u(l + 1);  // the U buffer is free
     }
     // (5) state -> bf16 slice (next A operand, stored next layer) and sums of squares
     if (__all_sync(0xFFFFFFFFu, uok)) {
