@@ -103,6 +103,15 @@ __device__ __forceinline__ void tma_load_4d(uint32_t dst, const CUtensorMap* map
       : "memory");
 }
 
+// 4-D tiled prefetch of one box into L2 (no shared memory, no completion).
+__device__ __forceinline__ void tma_prefetch_l2_4d(const CUtensorMap* map, int c0, int c1, int c2,
+                                                   int c3) {
+  asm volatile("cp.async.bulk.prefetch.tensor.4d.L2.global.tile [%0, {%1, %2, %3, %4}];" ::"l"(
+                   reinterpret_cast<uint64_t>(map)),
+               "r"(c0), "r"(c1), "r"(c2), "r"(c3)
+               : "memory");
+}
+
 // Shared-memory descriptor of an MN-major operand written by TMA with 128-byte swizzling, as V
 // lies in shared memory for the P V MMA: each 128-byte row holds 64 consecutive N elements
 // (channels) of one K index (key); 8-row (8-key) swizzle atoms are 1024 B apart along K (stride
@@ -503,12 +512,31 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
   pdl_wait();
   pdl_trigger();
 
-  // This thread's query row and the last slot it may see.
+  // Q does not depend on the key range: it loads while the range is found. So does the first
+  // K/V block this CTA would take if the keys filled the cache (max_keys), prefetched into L2;
+  // a wrong guess costs only L2 bandwidth.
+  const int q_row0 = (b * p.Hq + h * p.G) * p.Nt + qb * 128;
+  if (tid == 0) {
+    mbar_arrive_expect_tx(bar_q, C::kKV);
+    for (int ds = 0; ds < C::kSlabs; ++ds)
+      tma_load_2d(base + C::kOffQ + ds * C::kTile, &tmQ, bar_q, ds * 64, q_row0);
+    const int nb_guess = (p.max_keys + kKeyBlock - 1) / kKeyBlock;
+    const int kb_guess = split * nb_guess / S;
+    if (kb_guess < (split + 1) * nb_guess / S) {
+      for (int ds = 0; ds < C::kSlabs; ++ds) {
+        tma_prefetch_l2_4d(&tmK, ds * 64, h, kb_guess * kKeyBlock, b);
+        tma_prefetch_l2_4d(&tmV, ds * 64, h, kb_guess * kKeyBlock, b);
+      }
+    }
+  }
+
+  // This thread's query row and the last slot it may see; the CTA's key end is the maximum.
   const int i = qb * 128 + tid;
   const int nk = min(p.n_keys[b], p.max_keys);
   int last = -1;
   if (i < p.rows_per_group) last = min(p.q_slot[b * p.Nt + i % p.Nt], nk - 1);
-  atomicMax(key_end, last + 1);
+  const int warp_end = __reduce_max_sync(0xFFFFFFFFu, last + 1);
+  if ((tid & 31) == 0) atomicMax(key_end, warp_end);
   __syncthreads();
   const uint32_t tmem = *tmem_slot;
   const uint32_t t_o = tmem + C::kTmemO;
@@ -518,7 +546,6 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
   const int kb0 = split * n_blocks / S, kb1 = (split + 1) * n_blocks / S;
 
   const uint32_t sQ = base + C::kOffQ;
-  const int q_row0 = (b * p.Hq + h * p.G) * p.Nt + qb * 128;
   auto sK = [&](int st) { return base + C::kOffStage + st * C::kStage; };
   auto sV = [&](int st) { return base + C::kOffStage + st * C::kStage + C::kKV; };
   // K or V of block kb0 + j into stage j % NST (thread 0); last_k / last_v: the latest blocks
@@ -558,9 +585,6 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
 
   const int n_mine = kb1 - kb0;
   if (tid == 0 && n_mine > 0) {
-    mbar_arrive_expect_tx(bar_q, C::kKV);
-    for (int ds = 0; ds < C::kSlabs; ++ds)
-      tma_load_2d(sQ + ds * C::kTile, &tmQ, bar_q, ds * 64, q_row0);
     load_k(0);
     load_v(0);
     issue_s(0);
@@ -706,10 +730,11 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
       wait_bounded(bar_k(jj % NST), static_cast<uint32_t>(jj / NST) & 1u, tmo);
     for (int jj = last_v; jj >= 0 && jj > last_v - NST; --jj)
       wait_bounded(bar_v(jj % NST), static_cast<uint32_t>(jj / NST) & 1u, tmo);
-    if (last_k >= 0) wait_bounded(bar_q, 0, tmo);
     umma_commit(bar_drain);
     wait_bounded(bar_drain, 0, tmo);
   }
+  // Q was loaded in every CTA; its memory is reused below.
+  if (tid == 0) wait_bounded(bar_q, 0, tmo);
   __syncthreads();
 
   // Partial (O, m, l) of this CTA's key run -> the CTA that combines each row, by bulk copies
