@@ -181,10 +181,11 @@ int dv_build_visual_memory(dv_plan* plan, const void* x0, int batch, int n_vis, 
  *     used, so its max_batch / max_n_vis do not bound this call.
  *   - Limit: batch * n_vis * (n_layers * r_pad * 2 + n_layers * 4 + 4) bytes (each part
  *     rounded up to 256 bytes, r_pad = rank rounded up to 64, n_layers counting the planned
- *     layers) must fit in 32 MiB; the embedding adapter with r_pad = 64 adds batch * n_vis *
- *     n_layers * r_pad * 4 (the fp32 x0 (2 U_l)^T of the small-token path); the recurrent adapter adds batch * n_vis * (4 d +
- *     n_layers * (2 d + 4 d / 64)) bytes (fp32 state, bf16 M_l of every layer, partial sums
- *     of squares). Larger builds return DV_ERR_UNSUPPORTED_SHAPE and launch nothing.
+ *     layers) must fit in 32 MiB. The embedding adapter with r_pad = 64 adds batch * n_vis *
+ *     n_layers * r_pad * 4 (the fp32 x0 (2 U_l)^T of the small-token path). The recurrent
+ *     adapter adds batch * n_vis * (4 d + n_layers * (2 d + 4 d / 64)) bytes (fp32 state, bf16
+ *     M_l of every layer, partial sums of squares). Larger builds return
+ *     DV_ERR_UNSUPPORTED_SHAPE and launch nothing.
  *   - The first call on a device looks up the array's device address with that device current;
  *     make that first call before any stream capture.
  *   - All calls on a device share the array and find it as the last call left it (nothing in
