@@ -216,7 +216,7 @@ __global__ void __launch_bounds__(kNumThreads, 1)
       } else if constexpr (EPI == EPI_NORM) {
         epi_norm<BN>(p, tbase, l, t);
       } else {
-        epi_resid<BN>(p, tbase, n, t);
+        epi_resid<BN>(p, tbase, n, t, epi_stage + q * kWarpStageFloats);
       }
       tc_fence_before();
       mbar_arrive(tempty_bar(acc));
