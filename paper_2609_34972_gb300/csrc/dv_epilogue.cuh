@@ -68,19 +68,24 @@ __device__ __forceinline__ void warp_store_bf16(float* stage, const uint32_t (&p
   __syncwarp();
 }
 
-// The inverse of warp_store_f32: lane-row gets its 32 values of rows [0, rows) of src (row
-// stride ld floats), read a row segment per instruction through the warp's staging; rows past
-// `rows` read 0.
-__device__ __forceinline__ void warp_load_f32(float* stage, float (&v)[32], const float* src,
-                                              long long ld, int rows) {
+// The inverse of warp_store_f32, in two steps: warp_gather_f32 issues the loads of rows
+// [0, rows) of src (row stride ld floats), a row segment per instruction (rows past `rows` read
+// 0); warp_unstage_f32 then gives lane-row its 32 values through the warp's staging. Loads of
+// the next block can be in flight while the current one is used.
+__device__ __forceinline__ void warp_gather_f32(float4 (&g)[8], const float* src, long long ld,
+                                                int rows) {
   const int lane = threadIdx.x & 31;
-  float4 g[8];
 #pragma unroll
   for (int k = 0; k < 8; ++k) {
     const int row = 4 * k + (lane >> 3), c4 = lane & 7;
     g[k] = row < rows ? reinterpret_cast<const float4*>(src + row * ld)[c4]
                       : make_float4(0.0f, 0.0f, 0.0f, 0.0f);
   }
+}
+
+__device__ __forceinline__ void warp_unstage_f32(float* stage, const float4 (&g)[8],
+                                                 float (&v)[32]) {
+  const int lane = threadIdx.x & 31;
 #pragma unroll
   for (int k = 0; k < 8; ++k) {
     const int row = 4 * k + (lane >> 3), c4 = lane & 7;
@@ -261,16 +266,20 @@ __device__ __forceinline__ void epi_resid(const GemmParams& p, uint32_t tbase, i
   const int rows = p.s.M - t0;         // rows of the warp's block inside the build (may be <= 0)
   const size_t base = static_cast<size_t>(t0) * e.d + static_cast<size_t>(n) * BN;
   float ss = 0.0f;
+  float4 g[8];  // the next chunk of the fp32 state, loading while this chunk is used
+  if (!e.first) warp_gather_f32(g, e.state + base, e.d, rows);
 #pragma unroll 1
   for (int c = 0; c < BN / 32; ++c) {
     uint32_t r[32];
     __syncwarp();
     tmem_ld32(tbase + c * 32, r);  // in flight while the previous M loads
     float mv[32];
-    if (e.first)
+    if (e.first) {
       warp_load_bf16(stage, mv, e.x0 + base + c * 32, e.d, rows);
-    else
-      warp_load_f32(stage, mv, e.state + base + c * 32, e.d, rows);
+    } else {
+      warp_unstage_f32(stage, g, mv);
+      if (c + 1 < BN / 32) warp_gather_f32(g, e.state + base + (c + 1) * 32, e.d, rows);
+    }
     tmem_ld_wait();
     // the accumulator registers are used only past the wait (the empty statement redefines them)
     asm volatile(""
