@@ -68,74 +68,6 @@ __device__ __forceinline__ void warp_store_bf16(float* stage, const uint32_t (&p
   __syncwarp();
 }
 
-// The inverse of warp_store_f32, in two steps: warp_gather_f32 issues the loads of rows
-// [0, rows) of src (row stride ld floats), a row segment per instruction (rows past `rows` read
-// 0); warp_unstage_f32 then gives lane-row its 32 values through the warp's staging. Loads of
-// the next block can be in flight while the current one is used.
-__device__ __forceinline__ void warp_gather_f32(float4 (&g)[8], const float* src, long long ld,
-                                                int rows) {
-  const int lane = threadIdx.x & 31;
-#pragma unroll
-  for (int k = 0; k < 8; ++k) {
-    const int row = 4 * k + (lane >> 3), c4 = lane & 7;
-    g[k] = row < rows ? reinterpret_cast<const float4*>(src + row * ld)[c4]
-                      : make_float4(0.0f, 0.0f, 0.0f, 0.0f);
-  }
-}
-
-__device__ __forceinline__ void warp_unstage_f32(float* stage, const float4 (&g)[8],
-                                                 float (&v)[32]) {
-  const int lane = threadIdx.x & 31;
-#pragma unroll
-  for (int k = 0; k < 8; ++k) {
-    const int row = 4 * k + (lane >> 3), c4 = lane & 7;
-    reinterpret_cast<float4*>(stage + row * kWarpStagePitch)[c4] = g[k];
-  }
-  __syncwarp();
-  const float4* srow = reinterpret_cast<const float4*>(stage + lane * kWarpStagePitch);
-#pragma unroll
-  for (int q = 0; q < 8; ++q) {
-    const float4 x = srow[q];
-    v[4 * q] = x.x;
-    v[4 * q + 1] = x.y;
-    v[4 * q + 2] = x.z;
-    v[4 * q + 3] = x.w;
-  }
-  __syncwarp();
-}
-
-// The same for a bf16 block, widened to fp32.
-__device__ __forceinline__ void warp_load_bf16(float* stage, float (&v)[32], const uint16_t* src,
-                                               long long ld, int rows) {
-  const int lane = threadIdx.x & 31;
-  uint32_t* st = reinterpret_cast<uint32_t*>(stage);
-  constexpr int kPitch = 20;  // words per staged row (16 + 4 pad)
-  uint4 g[4];
-#pragma unroll
-  for (int k = 0; k < 4; ++k) {
-    const int row = 8 * k + (lane >> 2), c4 = lane & 3;
-    g[k] = row < rows ? reinterpret_cast<const uint4*>(src + row * ld)[c4] : make_uint4(0, 0, 0, 0);
-  }
-#pragma unroll
-  for (int k = 0; k < 4; ++k) {
-    const int row = 8 * k + (lane >> 2), c4 = lane & 3;
-    reinterpret_cast<uint4*>(st + row * kPitch)[c4] = g[k];
-  }
-  __syncwarp();
-  const uint4* srow = reinterpret_cast<const uint4*>(st + lane * kPitch);
-#pragma unroll
-  for (int q = 0; q < 4; ++q) {
-    const uint4 w = srow[q];
-    const uint32_t ws[4] = {w.x, w.y, w.z, w.w};
-#pragma unroll
-    for (int u = 0; u < 4; ++u) {
-      v[q * 8 + 2 * u] = bf16_bits_to_float(ws[u] & 0xFFFFu);
-      v[q * 8 + 2 * u + 1] = bf16_bits_to_float(ws[u] >> 16);
-    }
-  }
-  __syncwarp();
-}
-
 // In-register transpose of a warp's 32 x 32 block: on entry lane i holds row i (r[j] = M[i][j]),
 // on exit lane i holds column i (r[j] = M[j][i]). Five butterfly rounds: in the round of bit b,
 // registers j and j + b (j without bit b) of lanes i and i ^ b swap the two off-diagonal
@@ -250,59 +182,6 @@ __device__ __forceinline__ void epi_norm(const GemmParams& p, uint32_t tbase, in
       }
     }
   }
-}
-
-// One step of the recurrent adapter (Sec. 3.1 Eq. 6) for token row t and columns
-// [n*BN, (n+1)*BN): M = prev + h U^T with prev = x0 (first planned layer) or the fp32 state.
-// Writes the new fp32 state, bf16(M) for the K/V GEMM, and the sum of M^2 over the tile. The
-// state moves through the warp's staging a row segment per instruction (whole 128-byte lines),
-// not a 16-byte piece per lane and row.
-template <int BN>
-__device__ __forceinline__ void epi_resid(const GemmParams& p, uint32_t tbase, int n, int t,
-                                          float* stage) {
-  const EpiResid& e = p.resid;
-  const int lane = threadIdx.x & 31;
-  const int t0 = t - lane;             // the warp's first row
-  const int rows = p.s.M - t0;         // rows of the warp's block inside the build (may be <= 0)
-  const size_t base = static_cast<size_t>(t0) * e.d + static_cast<size_t>(n) * BN;
-  float ss = 0.0f;
-  float4 g[8];  // the next chunk of the fp32 state, loading while this chunk is used
-  if (!e.first) warp_gather_f32(g, e.state + base, e.d, rows);
-#pragma unroll 1
-  for (int c = 0; c < BN / 32; ++c) {
-    uint32_t r[32];
-    __syncwarp();
-    tmem_ld32(tbase + c * 32, r);  // in flight while the previous M loads
-    float mv[32];
-    if (e.first) {
-      warp_load_bf16(stage, mv, e.x0 + base + c * 32, e.d, rows);
-    } else {
-      warp_unstage_f32(stage, g, mv);
-      if (c + 1 < BN / 32) warp_gather_f32(g, e.state + base + (c + 1) * 32, e.d, rows);
-    }
-    tmem_ld_wait();
-    // the accumulator registers are used only past the wait (the empty statement redefines them)
-    asm volatile(""
-                 : "+r"(r[0]), "+r"(r[1]), "+r"(r[2]), "+r"(r[3]), "+r"(r[4]), "+r"(r[5]),
-                   "+r"(r[6]), "+r"(r[7]), "+r"(r[8]), "+r"(r[9]), "+r"(r[10]), "+r"(r[11]),
-                   "+r"(r[12]), "+r"(r[13]), "+r"(r[14]), "+r"(r[15]), "+r"(r[16]), "+r"(r[17]),
-                   "+r"(r[18]), "+r"(r[19]), "+r"(r[20]), "+r"(r[21]), "+r"(r[22]), "+r"(r[23]),
-                   "+r"(r[24]), "+r"(r[25]), "+r"(r[26]), "+r"(r[27]), "+r"(r[28]), "+r"(r[29]),
-                   "+r"(r[30]), "+r"(r[31]));
-    uint32_t vb[32], pk[16];
-#pragma unroll
-    for (int u = 0; u < 32; ++u) {
-      const float v = mv[u] + __uint_as_float(r[u]);
-      ss = fmaf(v, v, ss);
-      vb[u] = __float_as_uint(v);
-    }
-#pragma unroll
-    for (int u = 0; u < 16; ++u)
-      pk[u] = pack_bf16x2(__uint_as_float(vb[2 * u]), __uint_as_float(vb[2 * u + 1]));
-    warp_store_f32(stage, vb, e.state + base + c * 32, e.d, rows);
-    warp_store_bf16(stage, pk, e.mem + base + c * 32, e.d, rows);
-  }
-  if (t < p.s.M) e.part[static_cast<size_t>(n) * p.s.M + t] = ss;
 }
 
 // Per-token context of the K/V store: cache row base, positions, rstd of one token.
