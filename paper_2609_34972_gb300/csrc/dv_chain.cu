@@ -9,11 +9,11 @@
 //     operand of its part of the down-projection and the source of the TMA store of M_l.
 // Per layer:
 //   1. down-projection partial: z_s = bf16(M_{l-1})[:, slice] D_l[:, slice]^T (TMEM, fp32);
-//   2. the partial goes to shared memory (a region of its own where shared memory allows, else
-//      over the bf16 slice once its readers are done). CTA s
-//      owns rows [s 128 / S, (s + 1) 128 / S): every CTA sends each peer the peer's rows of its
-//      partial by bulk copies into the peer's D buffer (read by then), completing on the peer's
-//      barrier. CTA s sums its rows over the S partials in the fixed order 0 .. S-1, applies
+//   2. the partial goes to shared memory: a region of its own where shared memory allows (r_pad
+//      64), else the U buffer (r_pad 128; U_l then loads once every peer has acknowledged its z
+//      rows). CTA s owns rows [s 128 / S, (s + 1) 128 / S): every CTA sends each peer the peer's
+//      rows of its partial by bulk copies into the peer's D buffer (read by then), completing
+//      on the peer's barrier. CTA s sums its rows over the S partials in the fixed order 0 .. S-1, applies
 //      SiLU, writes bf16 h into its h tile (A operand of the up-projection) and sends its rows of
 //      h to every peer's h tile the same way;
 //   3. once all h rows have landed: state += h U_l[slice, :]^T (TMEM);
@@ -23,7 +23,8 @@
 // One cluster barrier per layer (arrival once the down MMA has read D_l, wait before sending z)
 // keeps a CTA from sending into a peer's D buffer too early; every other ordering follows from
 // the data: a CTA sends z_{l+1} only after it has all of h_l, so every receiver has finished
-// with z_l, and so on. D_{l+1} loads once the z rows are summed, U_{l+1} after the up MMA.
+// with z_l, and so on. D_{l+1} loads once the z rows are summed; U_{l+1} after the up MMA, or
+// (partial z in the U buffer) once layer l+1's z rows have left it.
 // Only bf16 M_l and the partial sums of squares leave the chip; the state never does. Every
 // wait is bounded; a CTA that gives up keeps passing the cluster barriers and keeps sending (so
 // its peers' waits end and no copy lands after a CTA has exited), stops issuing MMAs and loads,
