@@ -180,6 +180,9 @@ def test_attention_kernel_on_exact_inputs(hd, hq, hkv, nt):
     (64, 2, 32, 32, 64, [700, 650], 768),
     (128, 4, 28, 4, 50, [700, 650, 700, 690], 768),
     (128, 3, 40, 20, 100, [300, 290, 277], 320),
+    # many query blocks per kv head: 28 / 4 GQA, 200 text queries = 1400 rows (11 blocks of
+    # 128, the last ragged), 88 clusters: one stage, S = 2
+    (128, 2, 28, 4, 200, [700, 650], 768),
 ])
 def test_attention_every_cluster_shape(hd, B, hq, hkv, nt, n_keys, S):
     _exact_case(hd, B, hq, hkv, nt, n_keys, S, 500 + hd + B + hq,
