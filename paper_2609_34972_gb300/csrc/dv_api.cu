@@ -781,11 +781,34 @@ static cudaError_t enqueue_recurrent(const PlanView& v, const BuildArgs& a, cuda
   gp.timeout_ns = kTimeoutNs;
   // up-projection step: A = h_i (H columns from i * r_pad), B = U_i ([d][r_pad] rows i * d)
   gp.s = {static_cast<int>(T), 1, d, 0, v.r_pad / 64, v.r_pad, 0, 0, 0, 0};
+  // Large builds at r_pad 256 (one 256-token tile per CTA pair is enough to fill the pairs, so
+  // no K split): the down-projection runs on CTA pairs, each SM staging half of D_l instead of
+  // every CTA reading all of it from L2. Its maps start at the layer's rows: the previous
+  // state (x0 for the first layer) and layer i's rows of the stacked D.
+  const bool down_pairs = v.r_pad == 256 && splits == 1;
+  GemmParams gd;
+  std::memset(&gd, 0, sizeof(gd));
+  gd.status = v.status;
+  gd.timeout_ns = kTimeoutNs;
+  gd.s = {static_cast<int>(T), 1, v.r_pad, d / 64, 0, 0, 0, 0, 0, 0};
+  tm_groups(gd.s, 256, T);
   for (int i = 0; i < L && err == cudaSuccess; ++i) {
-    dp.a_row0 = i == 0 ? 0 : static_cast<int>((i - 1) * T);
-    dp.b_row0 = i * v.r_pad;
-    dp.h_col0 = i * v.r_pad;
-    err = launch_down_split(v.r_pad, splits, i == 0 ? tm_x0 : tm_mem, *v.tm_Dst_rp, dp, st);
+    if (down_pairs) {
+      CUtensorMap tm_a, tm_b;
+      const uint16_t* a_ptr = i == 0 ? static_cast<const uint16_t*>(a.x0)
+                                     : a.mem + static_cast<size_t>(i - 1) * T * d;
+      if (!encode_slabs(&tm_a, a_ptr, d, static_cast<uint64_t>(T), d, kBlockM) ||
+          !encode_slabs(&tm_b, v.Dst + static_cast<size_t>(i) * v.r_pad * v.dst_ld, d, v.r_pad,
+                        v.dst_ld, 128))
+        return cudaErrorInvalidValue;
+      gd.silu = {a.H + static_cast<size_t>(i) * v.r_pad, static_cast<int>(n1), v.r_pad, nullptr, 0};
+      err = launch_pair_tm(EPI_SILU, 256, 0, tm_a, tm_a, tm_b, gd, v.num_sms, st);
+    } else {
+      dp.a_row0 = i == 0 ? 0 : static_cast<int>((i - 1) * T);
+      dp.b_row0 = i * v.r_pad;
+      dp.h_col0 = i * v.r_pad;
+      err = launch_down_split(v.r_pad, splits, i == 0 ? tm_x0 : tm_mem, *v.tm_Dst_rp, dp, st);
+    }
     if (err != cudaSuccess) break;
     gp.s.layer0 = i;
     gp.resid = {static_cast<const uint16_t*>(a.x0), a.state,
@@ -975,6 +998,8 @@ bool plan_view(const dv_plan* p, PlanView* v) {
   v->tm_Dst_rp = &p->tm_Dst_rp;
   v->tm_Uup = &p->tm_Uup;
   v->Uup = p->Uup;
+  v->Dst = p->Dst;
+  v->dst_ld = c.d + 64;  // as the plan allocates Dst
   v->resid_bn = p->resid_bn;
   v->inv_freq = p->inv_freq;
   v->Wkv = p->Wkv;

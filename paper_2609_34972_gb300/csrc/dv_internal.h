@@ -244,6 +244,8 @@ struct PlanView {
   int bn_lpt, bn_rn, bn_groups;    // statistic GEMM: layers per group, their row stride, groups
   const CUtensorMap* tm_Wkv;       // slab map, boxes of 128 rows
   const CUtensorMap* tm_Dst_rp;    // recurrent: boxes of r_pad rows (one layer's D)
+  const uint16_t* Dst;             // stacked D (and 2 U^T): rows of dst_ld elements
+  int dst_ld;
   const CUtensorMap* tm_Uup;       // recurrent: [L*d][r_pad], boxes of resid_bn rows
   const uint16_t* Uup;             // recurrent: U_l as [L*d][r_pad]
   int resid_bn;                    // recurrent: column tile of the up-projection step

@@ -157,7 +157,8 @@ def test_recurrent_noalloc_entry():
     assert torch.equal(k1, k2) and torch.equal(v1, v2)
 
 
-@pytest.mark.parametrize("name", ["llava15_7b", "qwen25vl_7b_image", "llava_next_7b"])
+@pytest.mark.parametrize("name", ["llava15_7b", "qwen25vl_7b_image", "llava_next_7b",
+                                  "qwen25vl_7b_video"])
 def test_recurrent_full_size_sampled(name):
     import torch
     cfg = _rec(synth.CONFIGS[name])
@@ -170,3 +171,20 @@ def test_recurrent_full_size_sampled(name):
     assert bool(torch.isfinite(k).all()) and bool(torch.isfinite(v).all())
     del k, v, plan
     torch.cuda.empty_cache()
+
+
+def test_recurrent_down_projection_on_pairs():
+    # r_pad 256 and 10000 tokens (79 blocks of 128, the last ragged): enough token blocks that the
+    # down-projection needs no K split, so it runs on CTA pairs with per-layer maps of the
+    # previous state and of layer l's rows of D. Sampled tokens against the oracle.
+    import torch
+    cfg = gu.small_config("rec_pairs", d=512, n_layers=3, n_kv_heads=2, n_heads=4, head_dim=128,
+                          rank=200, n_vis=5000, batch=2, x0_sigma=0.5, w_sigma=0.05, seed=171,
+                          pos_start=35, adapter="recurrent")
+    inp = synth.make_inputs(cfg)
+    k, v, plan = gu.run_build(inp)
+    toks = gu.sample_tokens(cfg.tokens, n=48, seed=3)
+    ref = oracle.build_tokens(inp, toks)
+    gk, gv = gu.gather(k, cfg, toks), gu.gather(v, cfg, toks)
+    gu.assert_parity(gk, gv, ref["k"], ref["v"], cfg.head_dim, "recurrent down on pairs")
+    assert bool(torch.isfinite(k).all()) and bool(torch.isfinite(v).all())
