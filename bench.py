@@ -97,8 +97,13 @@ class ClockSampler:
         try:
             out, _ = self.proc.communicate(timeout=5)
         except subprocess.TimeoutExpired:
+            # Every wait here is bounded: an nvidia-smi that does not exit (a driver query that
+            # blocks) must not hold the bench; the line then carries no clock record.
             self.proc.kill()
-            out, _ = self.proc.communicate()
+            try:
+                out, _ = self.proc.communicate(timeout=5)
+            except subprocess.TimeoutExpired:
+                return None
         sm, mx, reasons = [], [], set()
         names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
         for line in out.splitlines():
