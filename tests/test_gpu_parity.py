@@ -211,3 +211,22 @@ def test_layer_modes_tokens_as_m_path():
 def test_layer_modes_noalloc_entry():
     inp = synth.make_inputs(synth.config("tiny", n_vis=64, seed=42))
     _check_layer_modes(inp, [0, 2, 2, 1], "layer modes (no-alloc entry)", noalloc=True)
+
+
+@pytest.mark.parametrize("adapter", ["embedding", "recurrent"])
+def test_single_visual_token_rank_one(adapter):
+    # The degenerate build: one visual token (one ragged row of a 128-row tile) and a rank-1
+    # adapter (r padded to 64), over three layers, in each adapter variant.
+    cfg = gu.small_config(f"one token {adapter}", d=256, n_layers=3, n_kv_heads=2, n_heads=2,
+                          head_dim=128, rank=1, n_vis=1, batch=1, x0_sigma=0.5, seed=21,
+                          pos_start=7, adapter=adapter)
+    _full_check(synth.make_inputs(cfg), f"one token, r = 1, {adapter}")
+
+
+def test_single_token_mrope_grid_batch_three():
+    # A 1x1x1 M-RoPE grid per batch element: every axis sits at the same position.
+    cfg = gu.small_config("one-token grid", d=384, n_layers=2, n_kv_heads=2, n_heads=4,
+                          head_dim=64, rank=8, n_vis=1, batch=3, rope="mrope",
+                          rope_theta=1e6, mrope_section=(8, 12, 12), grid=(1, 1, 1),
+                          x0_sigma=0.5, seed=22, pos_start=40)
+    _full_check(synth.make_inputs(cfg), "one-token M-RoPE grid, batch 3")
