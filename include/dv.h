@@ -245,7 +245,7 @@ const char* dv_error_string(int status);
  *   dv_timing_enable(plan, 1) starts a new record (0 stops recording).
  *   dv_timing_read(plan, ms, n_stages, n_builds) synchronises on the recorded events and
  *   writes the summed milliseconds of each stage into ms[0..n_stages-1] (stage order:
- *   0 row sums of squares of E, 1 stacked down-projection + SiLU, 2 RMS statistics,
+ *   0 stacked down-projection + SiLU, 1 row sums of squares of E, 2 RMS statistics,
  *   3 K/V projection + RoPE + cache store; recurrent adapter: 0 empty, 1 the adapter chain
  *   through all layers, 2 RMS statistics from the chain's partial sums, 3 as above) and the
  *   number of builds into *n_builds.

@@ -47,7 +47,7 @@ EXPORTED = ["dv_memory_plan", "dv_build_visual_memory", "dv_plan_status", "dv_fr
             "dv_debug_wait_timeout", "dv_debug_copy_workspace", "dv_build_visual_memory_noalloc",
             "dv_debug_copy_memory", "dv_kv_engine", "dv_text_attention", "dv_text_attention_status"]
 N_STAGES = 4
-STAGE_NAMES = ["row_sumsq", "down_proj_silu", "rms_stats", "kv_proj_rope_store"]
+STAGE_NAMES = ["down_proj_silu", "row_sumsq", "rms_stats", "kv_proj_rope_store"]
 # Stage names of a recurrent-adapter build (stage 0 is empty there).
 STAGE_NAMES_RECURRENT = ["none", "adapter_chain", "rms_stats", "kv_proj_rope_store"]
 

@@ -489,28 +489,36 @@ __global__ void __launch_bounds__(64) k_rstd_hc(const uint16_t* __restrict__ H, 
 }
 
 // xx[t] = sum_j x0[t][j]^2 (fp32), one warp per token row, 16-byte loads.
+// Launched right after the down-projection and run beside it, on the SMs that its tiles leave
+// free. Its reads of x0 and writes of xx come before its dependency wait. That is safe: a
+// dependent grid starts only once every CTA of the grid before it has triggered, and the
+// down-projection triggers after its own wait, so every earlier writer of x0 and every earlier
+// reader of xx (the previous build's statistic) has finished. The wait comes last, so that this
+// grid completes only after the down-projection has, and the kernel after it, which waits on
+// this grid alone, still sees H.
 __global__ void k_row_sumsq(const uint16_t* __restrict__ x0, int T, int d, float* __restrict__ xx) {
-  dv::pdl_wait();
   dv::pdl_trigger();
   const int warp = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
   const int lane = threadIdx.x & 31;
-  if (warp >= T) return;
-  const uint4* row = reinterpret_cast<const uint4*>(x0 + static_cast<long long>(warp) * d);
-  float s = 0.0f;
+  if (warp < T) {
+    const uint4* row = reinterpret_cast<const uint4*>(x0 + static_cast<long long>(warp) * d);
+    float s = 0.0f;
 #pragma unroll 8
-  for (int c = lane; c < d / 8; c += 32) {
-    const uint4 v = row[c];
-    const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+    for (int c = lane; c < d / 8; c += 32) {
+      const uint4 v = row[c];
+      const uint32_t w[4] = {v.x, v.y, v.z, v.w};
 #pragma unroll
-    for (int e = 0; e < 4; ++e) {
-      const float a = __uint_as_float(w[e] << 16), b = __uint_as_float(w[e] & 0xFFFF0000u);
-      s = fmaf(a, a, s);
-      s = fmaf(b, b, s);
+      for (int e = 0; e < 4; ++e) {
+        const float a = __uint_as_float(w[e] << 16), b = __uint_as_float(w[e] & 0xFFFF0000u);
+        s = fmaf(a, a, s);
+        s = fmaf(b, b, s);
+      }
     }
-  }
 #pragma unroll
-  for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xFFFFFFFFu, s, o);
-  if (lane == 0) xx[warp] = s;
+    for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xFFFFFFFFu, s, o);
+    if (lane == 0) xx[warp] = s;
+  }
+  dv::pdl_wait();
 }
 
 // Failure-detection self-test: waits on a barrier nothing completes; gives up after the limit.
@@ -850,10 +858,13 @@ cudaError_t enqueue_build(const PlanView& v, const BuildArgs& a, cudaStream_t st
   gp.timeout_ns = kTimeoutNs;
   for (int i = 0; i < L; ++i) gp.layer_map[i] = v.active[i];
 
+  // xx = row sums of squares of x0, launched after the down-projection (see k_row_sumsq).
+  auto row_sumsq = [&]() {
+    return launch_pdl(k_row_sumsq, dim3(static_cast<unsigned>((T + 7) / 8)), dim3(256), st,
+                      static_cast<const uint16_t*>(a.x0), static_cast<int>(T), d, a.xx);
+  };
   mark(0);
-  cudaError_t err = launch_pdl(k_row_sumsq, dim3(static_cast<unsigned>((T + 7) / 8)), dim3(256), st,
-                               static_cast<const uint16_t*>(a.x0), static_cast<int>(T), d, a.xx);
-  mark(1);
+  cudaError_t err = cudaSuccess;
 
   // (1) H = SiLU(x0 [D_1 ... D_L]) — one GEMM over all layers' down-projections.
   gp.s = {static_cast<int>(T), 1, static_cast<int>(n1), d / 64, 0, 0, 0, 0, 0, 0};
@@ -874,6 +885,8 @@ cudaError_t enqueue_build(const PlanView& v, const BuildArgs& a, cudaStream_t st
     tm_groups(gp.s, bn, T);
     const CUtensorMap& tmD = v.tm_Dst_half[bn == 64 ? 0 : (bn == 128 ? 1 : 2)];
     if (err == cudaSuccess) err = launch_pair_tm(EPI_SILU, bn, 0, tm_x0_s, tm_x0_s, tmD, gp, v.num_sms, st);
+    mark(1);
+    if (err == cudaSuccess) err = row_sumsq();
     mark(2);
     if (err == cudaSuccess) {
       dim3 grid(static_cast<unsigned>((T + 63) / 64), static_cast<unsigned>(L));
@@ -908,6 +921,8 @@ cudaError_t enqueue_build(const PlanView& v, const BuildArgs& a, cudaStream_t st
     const CUtensorMap& tmD = v.tm_Dst[bn == 64 ? 0 : (bn == 128 ? 1 : 2)];
     if (err == cudaSuccess) err = launch_gemm(EPI_SILU, bn, 0, tm_x0, tm_x0, tmD, gp, v.num_sms, st);
   }
+  mark(1);
+  if (err == cudaSuccess) err = row_sumsq();
   mark(2);
 
   // (2) rstd_l from ||x0||^2 + h_l . ([x0 | h_l] [2 U_l^T ; G_l]): 256-column tiles of lpt
