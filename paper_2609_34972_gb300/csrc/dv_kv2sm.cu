@@ -113,7 +113,11 @@ __global__ void __launch_bounds__(kPairThreads, 1)
   cluster_sync();  // barriers of both CTAs initialised, TMEM allocated in both
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
-  pdl_wait();
+  // Only the epilogue warps wait for the kernel before this one (the RMS statistic): the
+  // producer and MMA warps read x0, H and the weights, which every kernel before the statistic
+  // has finished writing once this grid can start (each trigger follows its kernel's own wait),
+  // so the first tiles' loads and MMAs overlap the statistic's tail. rstd and the cache are
+  // touched only after the epilogue's wait.
   pdl_trigger();
 
   const int tok_tiles = (p.s.M + NT - 1) / NT;
@@ -215,6 +219,7 @@ __global__ void __launch_bounds__(kPairThreads, 1)
     }
   } else {
     // ------------------------------------------------------------------ epilogue warps
+    pdl_wait();
     const int q = warp & 3;  // TMEM lane quarter = block of 32 weight rows of this warp
     const uint32_t leader_tempty0 = map_to_rank(tempty_bar(0), 0);
     int acc = 0;
