@@ -111,7 +111,11 @@ __global__ void __launch_bounds__(kTmThreads, 1)
   cluster_sync();
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
-  pdl_wait();
+  // The K/V epilogue waits for the kernel before it (the RMS statistic) in its epilogue warps
+  // only: its producer reads x0 or M, H and the weights, which every kernel before the statistic
+  // has finished writing once this grid can start (each trigger follows its kernel's own wait).
+  // The down-projection and the statistic wait here, before any access.
+  if (EPI != EPI_KV) pdl_wait();
   pdl_trigger();
 
   const int m_tiles = (p.s.M + 255) / 256;
@@ -214,6 +218,7 @@ __global__ void __launch_bounds__(kTmThreads, 1)
     }
   } else {
     // ------------------------------------------------------------------ epilogue warps
+    if (EPI == EPI_KV) pdl_wait();  // rstd and the cache are touched only after this
     const int q = warp & 3;  // TMEM lane quarter of this warp
     const uint32_t leader_tempty0 = map_to_rank(tempty_bar(0), 0);
     int acc = 0;
