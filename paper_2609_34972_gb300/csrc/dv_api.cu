@@ -140,7 +140,8 @@ bool encode_3d(CUtensorMap* map, const void* ptr, uint64_t cols, uint64_t rows, 
 }
 
 // Launch of a build kernel with programmatic stream serialization (dv::pdl_attribute); the
-// kernel calls dv::pdl_wait() before touching global memory.
+// kernel calls dv::pdl_wait() before touching global memory, except where it states otherwise
+// (k_row_sumsq).
 template <typename... KArgs, typename... Args>
 cudaError_t launch_pdl(void (*kern)(KArgs...), dim3 grid, dim3 block, cudaStream_t st,
                        Args&&... args) {

@@ -83,7 +83,7 @@ struct EpiSilu {
 };
 
 // Launch attribute of the build's kernels: programmatic stream serialization (see pdl_wait in
-// dv_ptx.cuh; every kernel launched with it calls pdl_wait before touching global memory).
+// dv_ptx.cuh for what a kernel launched with it may touch before its wait).
 inline cudaLaunchAttribute pdl_attribute() {
   cudaLaunchAttribute a;
   a.id = cudaLaunchAttributeProgrammaticStreamSerialization;

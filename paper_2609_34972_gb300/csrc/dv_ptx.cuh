@@ -70,10 +70,11 @@ __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, volatil
 // ------------------------------------------------------------------------------ dependent launch
 // The build's kernels are launched with programmatic stream serialization: a kernel may start
 // (and run its prologue: barrier init, TMEM allocation, descriptor prefetch) while the previous
-// kernel of the stream is still running. pdl_wait() returns once every earlier kernel of the
-// stream has completed and its memory operations are visible; no kernel touches global memory
-// before it. pdl_trigger() then lets the next kernel launch early (its CTAs become resident as
-// resources allow and wait in their own pdl_wait()).
+// kernel of the stream is still running. pdl_wait() returns once the previous kernel has
+// completed and its memory operations are visible. A kernel touches global memory before it
+// only where the kernel says why that is safe (data that every trigger before it already
+// implies is written). pdl_trigger() lets the next kernel launch early: its CTAs start once
+// every CTA of this grid has triggered, as resources allow, and wait in their own pdl_wait().
 __device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
 __device__ __forceinline__ void pdl_trigger() {
   asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
