@@ -186,16 +186,72 @@ int dv_build_visual_memory(dv_plan* plan, const void* x0, int batch, int n_vis, 
  *     adapter adds batch * n_vis * (4 d + n_layers * (2 d + 4 d / 64)) bytes (fp32 state, bf16
  *     M_l of every layer, partial sums of squares). Larger builds return
  *     DV_ERR_UNSUPPORTED_SHAPE and launch nothing.
- *   - The first call on a device looks up the array's device address with that device current;
- *     make that first call before any stream capture.
+ *   - dv_memory_plan reserves the array on the plan's device (CUDA loads the module that
+ *     holds it when the plan looks up its address) and loads every kernel a build can launch,
+ *     so this entry point allocates nothing, even on its first call.
  *   - All calls on a device share the array and find it as the last call left it (nothing in
  *     it needs to start at zero). Calls that overlap on the GPU race on it: order them on one
  *     stream.
- * Errors: as dv_build_visual_memory, plus DV_ERR_UNSUPPORTED_SHAPE for builds over the limit.
+ * Errors: as dv_build_visual_memory, plus DV_ERR_UNSUPPORTED_SHAPE for builds over the limit
+ * and DV_ERR_OOM when the array could not be reserved when the plan was made.
  */
 int dv_build_visual_memory_noalloc(dv_plan* plan, const void* x0, int batch, int n_vis,
                                    const int* pos, const int* slot, int slot0,
                                    const dv_kv_cache* out, void* stream);
+
+/*
+ * End-to-end builds from host memory. The visual memory is the K/V entries that text tokens
+ * read (Sec. 3.2 Eq. 7); a caller that keeps E and its KV cache in host memory submits builds
+ * to a pipeline that copies E and the positions in, runs dv_build_visual_memory, and copies the
+ * built K/V out, with the copy-out of one build overlapping the next build.
+ *
+ * dv_host_pipeline_create — device staging for builds of exactly batch x n_vis tokens with
+ * `plan`: `depth` (1..4) sets of E, positions and a dense K/V cache, and three CUDA streams
+ * (copy-in, build, copy-out) on the current device. This call allocates (cudaMalloc) all of
+ * it; builds allocate nothing more. Staging sets are used round-robin: with depth >= 2 the
+ * copy-out of build i overlaps build i + 1. The plan must outlive the pipeline, and no other
+ * build with the same plan may run while the pipeline's builds are in flight (they share the
+ * plan's workspace).
+ * Errors: DV_ERR_INVALID_ARG, DV_ERR_UNSUPPORTED_SHAPE (beyond the plan's max_batch /
+ * max_n_vis), DV_ERR_OOM, DV_ERR_CUDA. On error nothing stays allocated and *out is NULL.
+ */
+typedef struct dv_host_pipeline dv_host_pipeline;
+int dv_host_pipeline_create(dv_plan* plan, int batch, int n_vis, int depth,
+                            dv_host_pipeline** out);
+
+/*
+ * dv_build_visual_memory_host — one end-to-end build, asynchronous. HOST pointers:
+ *   x0_host  bf16 [batch][n_vis][d]   E
+ *   pos_host int32 [batch][P][n_vis]  positions, P = 1 (DV_ROPE_1D) or 3 (M-RoPE modes)
+ *   k_host, v_host  bf16 [n_layers][batch][n_vis][n_kv_heads][head_dim] (dense): receive K and V
+ *            of every built layer; the rows of DV_LAYER_DROP layers are left untouched
+ *   stream   cudaStream_t as void*: the copy-in starts after the work enqueued on it before
+ *            this call (use dv_host_pipeline_join for the other direction)
+ *   ticket   receives the build's sequence number (may be NULL)
+ * The caller must not change x0_host / pos_host, nor read k_host / v_host, until
+ * dv_host_pipeline_wait(ticket) returns. Page-locked host memory (cudaHostAlloc or
+ * cudaHostRegister) lets the copies run asynchronously and overlap the builds; pageable memory
+ * gives the same result, but the driver stages those copies and they do not overlap.
+ * Each build moves batch*n_vis*(2 d + 4 P) bytes in and 2 * n_built * batch*n_vis*kv*2 bytes
+ * out, one cudaMemcpyAsync per contiguous range.
+ * Errors: DV_ERR_INVALID_ARG (NULL pointer, or the pipeline's device is not current),
+ * DV_ERR_ALIGNMENT (pos_host not 4-byte, bf16 buffers not 2-byte aligned), DV_ERR_CUDA.
+ */
+int dv_build_visual_memory_host(dv_host_pipeline* pipe, const void* x0_host, const int* pos_host,
+                                void* k_host, void* v_host, void* stream, long long* ticket);
+
+/* dv_host_pipeline_wait — blocks the calling thread until the host buffers of build `ticket`
+ * hold its K/V. DV_ERR_INVALID_ARG for a ticket not yet issued. Device-side timeouts of the
+ * build are reported by dv_plan_status on the pipeline's plan. */
+int dv_host_pipeline_wait(dv_host_pipeline* pipe, long long ticket);
+
+/* dv_host_pipeline_join — makes work enqueued on `stream` after this call wait until every
+ * build submitted so far has finished its copy-out (stream-ordered, does not block the host). */
+int dv_host_pipeline_join(dv_host_pipeline* pipe, void* stream);
+
+/* dv_host_pipeline_free — waits for the pipeline's builds, then releases its device buffers,
+ * streams and events. NULL is a no-op. */
+void dv_host_pipeline_free(dv_host_pipeline* pipe);
 
 /*
  * dv_plan_status — synchronises the device, reads and clears the plan's device status word.

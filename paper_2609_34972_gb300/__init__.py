@@ -45,7 +45,9 @@ DV_ADAPTER_RECURRENT = 1
 EXPORTED = ["dv_memory_plan", "dv_build_visual_memory", "dv_plan_status", "dv_free",
             "dv_error_string", "dv_timing_enable", "dv_timing_read", "dv_kernels_per_build",
             "dv_debug_wait_timeout", "dv_debug_copy_workspace", "dv_build_visual_memory_noalloc",
-            "dv_debug_copy_memory", "dv_kv_engine", "dv_text_attention", "dv_text_attention_status"]
+            "dv_debug_copy_memory", "dv_kv_engine", "dv_text_attention", "dv_text_attention_status",
+            "dv_host_pipeline_create", "dv_build_visual_memory_host", "dv_host_pipeline_wait",
+            "dv_host_pipeline_join", "dv_host_pipeline_free"]
 N_STAGES = 4
 STAGE_NAMES = ["down_proj_silu", "row_sumsq", "rms_stats", "kv_proj_rope_store"]
 # Stage names of a recurrent-adapter build (stage 0 is empty there).
@@ -107,11 +109,20 @@ def lib() -> ctypes.CDLL:
         L.dv_text_attention.argtypes = [vp, i32, i32, i32, i32, i32, ctypes.POINTER(DvKVCache),
                                         i32, i32, vp, vp, ctypes.c_float, vp, vp]
         L.dv_text_attention_status.argtypes = []
+        L.dv_host_pipeline_create.argtypes = [vp, i32, i32, i32, ctypes.POINTER(vp)]
+        L.dv_build_visual_memory_host.argtypes = [vp, vp, vp, vp, vp, vp,
+                                                  ctypes.POINTER(ctypes.c_longlong)]
+        L.dv_host_pipeline_wait.argtypes = [vp, ctypes.c_longlong]
+        L.dv_host_pipeline_join.argtypes = [vp, vp]
+        L.dv_host_pipeline_free.argtypes = [vp]
+        L.dv_host_pipeline_free.restype = None
         for name in ("dv_memory_plan", "dv_build_visual_memory", "dv_plan_status",
                      "dv_timing_enable", "dv_timing_read", "dv_kernels_per_build",
                      "dv_debug_wait_timeout", "dv_debug_copy_workspace",
                      "dv_build_visual_memory_noalloc", "dv_debug_copy_memory", "dv_kv_engine",
-                     "dv_text_attention", "dv_text_attention_status"):
+                     "dv_text_attention", "dv_text_attention_status", "dv_host_pipeline_create",
+                     "dv_build_visual_memory_host", "dv_host_pipeline_wait",
+                     "dv_host_pipeline_join"):
             getattr(L, name).restype = i32
         _lib = L
     return _lib
@@ -209,10 +220,69 @@ def kv_cache_view(k, v) -> DvKVCache:
     return DvKVCache(k.data_ptr(), v.data_ptr(), s[0], s[1], s[2], s[3])
 
 
+def _n_pos(cfg: DvConfig) -> int:
+    return 1 if cfg.rope == DV_ROPE_1D else 3
+
+
+def _check_tensor(name, t, dtype, device=None, shape=None, contiguous=True):
+    import torch
+    if not isinstance(t, torch.Tensor):
+        raise ValueError(f"{name} must be a torch tensor")
+    if t.dtype != dtype:
+        raise ValueError(f"{name} must be {dtype}, got {t.dtype}")
+    if device is not None and t.device != device:
+        raise ValueError(f"{name} must be on {device}, got {t.device}")
+    if contiguous and not t.is_contiguous():
+        raise ValueError(f"{name} must be contiguous")
+    if shape is not None and tuple(t.shape) != tuple(shape):
+        raise ValueError(f"{name} must have shape {tuple(shape)}, got {tuple(t.shape)}")
+
+
+def validate_build(cfg: DvConfig, x0, pos, k_cache, v_cache, slot=None, slot0: int = 0,
+                   device=None):
+    """Checks of a build's tensors against the plan's configuration, made before the C call.
+    A wrong d or an undersized cache would make the kernels read or write out of bounds, and an
+    int64 position tensor would be read as wrong positions, so they raise ValueError here; the
+    C ABI itself checks pointers, alignment, strides and the plan's token limit. ``device``
+    defaults to the current CUDA device (the one the C ABI builds on). Returns (B, N_v)."""
+    import torch
+    if device is None:
+        device = torch.device("cuda", torch.cuda.current_device())
+    if not isinstance(x0, torch.Tensor) or x0.dim() != 3:
+        raise ValueError("x0 must be a 3-D [B, N_v, d] tensor")
+    B, N = int(x0.shape[0]), int(x0.shape[1])
+    _check_tensor("x0", x0, torch.bfloat16, device, (B, N, cfg.d))
+    _check_tensor("pos", pos, torch.int32, device, (B, _n_pos(cfg), N))
+    for name, c in (("k_cache", k_cache), ("v_cache", v_cache)):
+        _check_tensor(name, c, torch.bfloat16, device, contiguous=False)
+        if c.dim() != 5:
+            raise ValueError(f"{name} must be 5-D [L, B_c, S, H_kv, D_h]")
+        if (c.shape[0] < cfg.n_layers or c.shape[1] < B or c.shape[3] != cfg.n_kv_heads
+                or c.shape[4] != cfg.head_dim):
+            raise ValueError(f"{name} of shape {tuple(c.shape)} cannot hold {cfg.n_layers} layers x "
+                             f"{B} batch rows x {cfg.n_kv_heads} heads x {cfg.head_dim}")
+    if k_cache.shape != v_cache.shape:
+        raise ValueError("k_cache and v_cache must have the same shape")
+    S = int(k_cache.shape[2])
+    if int(slot0) < 0:
+        raise ValueError("slot0 must be >= 0")
+    if slot is None:
+        if B * N > 0 and int(slot0) + N > S:
+            raise ValueError(f"slots {slot0}..{int(slot0) + N - 1} exceed the cache's {S} slots")
+    else:
+        _check_tensor("slot", slot, torch.int32, device, (B, N))
+        if B * N > 0:
+            lo, hi = int(slot.min()), int(slot.max())   # synchronises: slots are checked, not trusted
+            if lo < 0 or hi >= S:
+                raise ValueError(f"slot values {lo}..{hi} outside the cache's {S} slots")
+    return B, N
+
+
 def build_visual_memory(plan: Plan, x0, pos, k_cache, v_cache, slot=None, slot0: int = 0,
                         stream=None) -> None:
-    """Enqueue one build on ``stream`` (default: torch's current stream). Asynchronous."""
-    B, N = int(x0.shape[0]), int(x0.shape[1])
+    """Enqueue one build on ``stream`` (default: torch's current stream). Asynchronous, except
+    that explicit ``slot`` values are range-checked on the host first (a synchronisation)."""
+    B, N = validate_build(plan.cfg, x0, pos, k_cache, v_cache, slot, slot0)
     kvc = kv_cache_view(k_cache, v_cache)
     _check(lib().dv_build_visual_memory(plan.handle, _ptr(x0), B, N, _ptr(pos), _ptr(slot),
                                         int(slot0), ctypes.byref(kvc), _stream_handle(stream)),
@@ -225,7 +295,7 @@ def build_visual_memory_noalloc(plan: Plan, x0, pos, k_cache, v_cache, slot=None
     the intermediates live in the library's static 32 MiB device array, not in the plan's
     workspace. All such calls on a device share that array, so calls must not overlap on the
     GPU; builds whose intermediates exceed 32 MiB raise DvError (unsupported shape)."""
-    B, N = int(x0.shape[0]), int(x0.shape[1])
+    B, N = validate_build(plan.cfg, x0, pos, k_cache, v_cache, slot, slot0)
     kvc = kv_cache_view(k_cache, v_cache)
     _check(lib().dv_build_visual_memory_noalloc(plan.handle, _ptr(x0), B, N, _ptr(pos), _ptr(slot),
                                                 int(slot0), ctypes.byref(kvc),
@@ -327,63 +397,56 @@ def stage_names(plan: Plan):
 
 
 class HostPipeline:
-    """Builds from pinned host buffers with the device-to-host read of one build overlapping the
-    next build (two device buffer sets, a compute stream and a copy stream).
+    """End-to-end builds from host memory through the C ABI (``dv_host_pipeline_*``,
+    ``dv_build_visual_memory_host``): every ``submit`` copies one batch's E and positions to the
+    device, builds, and copies the built K/V back into the caller's host buffers, with the
+    copy-out of one build overlapping the next build (``depth`` device staging sets).
 
-    Every ``submit`` copies that build's E and positions host-to-device, builds (on the compute
-    stream, in submission order: builds share the plan's workspace), and copies the written K/V
-    device-to-host into the caller's pinned buffers. It returns a CUDA event that completes
-    when those host buffers hold the result; the caller must not reuse or read them before.
+    Host tensors (CPU, contiguous; page-locked for the copies to overlap):
+        x0 bf16 [B, N_v, d], pos int32 [B, P, N_v], k / v bf16 [L, B, N_v, H_kv, D_h]
+    ``submit`` returns a ticket; ``wait(ticket)`` blocks until that build's K/V are in its
+    host buffers, ``join(stream)`` orders later work on ``stream`` after every submitted build.
     """
 
-    def __init__(self, plan: Plan, x0_shape, pos_shape, cache_shape, depth: int = 2):
-        import torch
-        dev = torch.device("cuda", torch.cuda.current_device())
+    def __init__(self, plan: Plan, batch: int, n_vis: int, depth: int = 2):
         self.plan = plan
-        self.depth = depth
-        self.compute = torch.cuda.Stream(dev)
-        self.copy = torch.cuda.Stream(dev)
-        self.x0 = [torch.empty(x0_shape, dtype=torch.bfloat16, device=dev) for _ in range(depth)]
-        self.pos = [torch.empty(pos_shape, dtype=torch.int32, device=dev) for _ in range(depth)]
-        self.k = [torch.empty(cache_shape, dtype=torch.bfloat16, device=dev) for _ in range(depth)]
-        self.v = [torch.empty(cache_shape, dtype=torch.bfloat16, device=dev) for _ in range(depth)]
-        self.built = [torch.cuda.Event() for _ in range(depth)]
-        self.read = [torch.cuda.Event() for _ in range(depth)]
-        self.n = 0
+        self.batch, self.n_vis = int(batch), int(n_vis)
+        h = ctypes.c_void_p()
+        _check(lib().dv_host_pipeline_create(plan.handle, self.batch, self.n_vis, int(depth),
+                                             ctypes.byref(h)), "dv_host_pipeline_create")
+        self.handle = h
 
-    def submit(self, x0_host, pos_host, k_host, v_host, slot=None, slot0: int = 0):
+    def _check_host(self, x0, pos, k, v):
         import torch
-        s = self.n % self.depth
-        self.n += 1
-        with torch.cuda.stream(self.compute):
-            self.compute.wait_event(self.read[s])      # this buffer set's last read is done
-            self.x0[s].copy_(x0_host, non_blocking=True)
-            self.pos[s].copy_(pos_host, non_blocking=True)
-            build_visual_memory(self.plan, self.x0[s], self.pos[s], self.k[s], self.v[s], slot=slot,
-                                slot0=slot0, stream=self.compute)
-            self.built[s].record(self.compute)
-        with torch.cuda.stream(self.copy):
-            self.copy.wait_event(self.built[s])
-            k_host.copy_(self.k[s], non_blocking=True)
-            v_host.copy_(self.v[s], non_blocking=True)
-            self.read[s].record(self.copy)
-        return self.read[s]
+        cfg, B, N = self.plan.cfg, self.batch, self.n_vis
+        cpu = torch.device("cpu")
+        _check_tensor("x0", x0, torch.bfloat16, cpu, (B, N, cfg.d))
+        _check_tensor("pos", pos, torch.int32, cpu, (B, _n_pos(cfg), N))
+        shape = (cfg.n_layers, B, N, cfg.n_kv_heads, cfg.head_dim)
+        _check_tensor("k", k, torch.bfloat16, cpu, shape)
+        _check_tensor("v", v, torch.bfloat16, cpu, shape)
 
-    def synchronize(self):
-        self.copy.synchronize()
-        self.compute.synchronize()
+    def submit(self, x0, pos, k, v, stream=None) -> int:
+        self._check_host(x0, pos, k, v)
+        t = ctypes.c_longlong()
+        _check(lib().dv_build_visual_memory_host(self.handle, _ptr(x0), _ptr(pos), _ptr(k), _ptr(v),
+                                                 _stream_handle(stream), ctypes.byref(t)),
+               "dv_build_visual_memory_host")
+        return t.value
 
+    def wait(self, ticket: int) -> None:
+        _check(lib().dv_host_pipeline_wait(self.handle, int(ticket)), "dv_host_pipeline_wait")
 
-def build_visual_memory_from_host(plan: Plan, x0_host, pos_host, k_host, v_host, x0_dev, pos_dev,
-                                  k_dev, v_dev, stream=None) -> None:
-    """End-to-end build from pinned host buffers: copy E and the positions to the device, build,
-    and copy the written K/V entries back, all on one stream. ``*_dev`` are device buffers of the
-    same shapes the caller keeps across calls. Asynchronous like the device-side call."""
-    import torch
-    s = stream or torch.cuda.current_stream()
-    with torch.cuda.stream(s):
-        x0_dev.copy_(x0_host, non_blocking=True)
-        pos_dev.copy_(pos_host, non_blocking=True)
-        build_visual_memory(plan, x0_dev, pos_dev, k_dev, v_dev, stream=s)
-        k_host.copy_(k_dev, non_blocking=True)
-        v_host.copy_(v_dev, non_blocking=True)
+    def join(self, stream=None) -> None:
+        _check(lib().dv_host_pipeline_join(self.handle, _stream_handle(stream)), "dv_host_pipeline_join")
+
+    def close(self) -> None:
+        if self.handle and self.handle.value:
+            lib().dv_host_pipeline_free(self.handle)
+            self.handle = ctypes.c_void_p()
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass

@@ -46,6 +46,7 @@ struct dv_plan {
   void* ws = nullptr;          // workspace of a build of max_tokens tokens (carve_workspace)
   long long last_tokens = 0;   // tokens of the last build (layout of the workspace)
   int* status = nullptr;
+  void* scratch = nullptr;     // static scratch of the no-allocation entry on this device
   CUtensorMap tm_Dst[3];       // boxes of 64, 128, 256 rows
   CUtensorMap tm_Dst_half[3];  // slab maps, boxes of 32, 64, 128 rows (halves for CTA pairs)
   CUtensorMap tm_Bn;           // boxes of 256 rows (one layer group)
@@ -1023,12 +1024,56 @@ bool plan_view(const dv_plan* p, PlanView* v) {
   return true;
 }
 
+const dv_config* plan_config(const dv_plan* p) { return p ? &p->cfg : nullptr; }
+void* plan_scratch(const dv_plan* p) { return p ? p->scratch : nullptr; }
+
 bool encode_bf16_2d(CUtensorMap* map, const void* ptr, uint64_t cols, uint64_t rows, uint64_t ld,
                     uint32_t box_rows) {
   return encode_2d(map, ptr, cols, rows, ld, box_rows);
 }
 
 }  // namespace dv
+
+namespace {
+
+// CUDA loads modules and kernels lazily, on first use, and loading takes device memory for their
+// code. The plan loads every kernel its builds can launch, so that builds allocate nothing (the
+// no-allocation entry relies on this). Each launcher, given no tokens, sets its kernel's
+// attributes (which loads it) and returns without launching; the dispatchers cover every
+// instantiation a build of this plan can pick.
+cudaError_t preload_build_kernels(const dv_plan* p) {
+  GemmParams gp;
+  std::memset(&gp, 0, sizeof(gp));
+  CUtensorMap m;
+  std::memset(&m, 0, sizeof(m));
+  cudaError_t err = cudaSuccess;
+  auto keep = [&](cudaError_t e) {
+    if (err == cudaSuccess) err = e;
+  };
+  const int hd = p->cfg.head_dim;
+  for (int bn : {64, 128, 256}) {
+    keep(dv::launch_gemm(dv::EPI_SILU, bn, 0, m, m, m, gp, 1, nullptr));
+    keep(dv::launch_gemm(dv::EPI_NORM, bn, 0, m, m, m, gp, 1, nullptr));
+    keep(dv::launch_gemm(dv::EPI_RESID, bn, 0, m, m, m, gp, 1, nullptr));
+    keep(dv::launch_pair_tm(dv::EPI_SILU, bn, 0, m, m, m, gp, 1, nullptr));
+    keep(dv::launch_pair_tm(dv::EPI_NORM, bn, 0, m, m, m, gp, 1, nullptr));
+  }
+  keep(dv::launch_pair_tm(dv::EPI_KV, 256, hd, m, m, m, gp, 1, nullptr));
+  for (int nt : {64, 128, 192, 256}) keep(dv::launch_kv_pair(hd, nt, m, m, m, gp, 1, nullptr));
+  if (p->cfg.adapter == DV_ADAPTER_RECURRENT) {
+    dv::DownParams dp;
+    std::memset(&dp, 0, sizeof(dp));
+    dp.k_slabs = 8;
+    for (int s : {1, 2, 4, 8}) keep(dv::launch_down_split(p->r_pad, s, m, m, dp, nullptr));
+    int spc = 0, S = 0;
+    if (dv::chain_shape(p->cfg.d, p->r_pad, &spc, &S))
+      keep(dv::launch_chain(p->r_pad, spc, S, 0, 1, p->cfg.d, m, m, m, m, nullptr, 0, nullptr,
+                            nullptr, 0, nullptr));
+  }
+  return err;
+}
+
+}  // namespace
 
 // ================================================================================== C ABI
 
@@ -1214,6 +1259,18 @@ int dv_memory_plan(const dv_config* cfg, const dv_weights* w, void* stream, dv_p
   }
   for (int j = 0; j < HD / 2; ++j)
     p->inv_freq[j] = std::pow(static_cast<double>(cfg->rope_theta), -2.0 * j / HD);
+  if (preload_build_kernels(p) != cudaSuccess) {
+    cudaGetLastError();
+    free_plan_memory(p);
+    delete p;
+    return DV_ERR_CUDA;
+  }
+  // The no-allocation entry's scratch array: looked up (and so reserved) now. If that fails the
+  // plan still serves the other entry points; dv_build_visual_memory_noalloc then reports it.
+  if (dv::noalloc_scratch(&p->scratch) != DV_OK) {
+    cudaGetLastError();
+    p->scratch = nullptr;
+  }
   *out = p;
   return DV_OK;
 }

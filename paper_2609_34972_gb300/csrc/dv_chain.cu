@@ -504,7 +504,7 @@ cudaError_t launch_t(int S, long long blocks, const CUtensorMap& x, const CUtens
       cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, C::kSmemBytes);
   if (err == cudaSuccess && S > 8)
     err = cudaFuncSetAttribute(kern, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
-  if (err != cudaSuccess) return err;
+  if (err != cudaSuccess || blocks <= 0) return err;
   cudaLaunchConfig_t cfg = {};
   cudaLaunchAttribute attr[2];
   attr[0].id = cudaLaunchAttributeClusterDimension;

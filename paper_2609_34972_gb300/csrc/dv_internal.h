@@ -7,6 +7,7 @@
 
 struct dv_plan;
 struct dv_kv_cache;
+struct dv_config;
 
 namespace dv {
 
@@ -254,6 +255,16 @@ struct PlanView {
   const int16_t* active;      // cache layer of each planned layer
 };
 bool plan_view(const dv_plan* p, PlanView* out);
+
+// The configuration a plan was made with (null for a null plan).
+const ::dv_config* plan_config(const dv_plan* p);
+
+// Device address of the static build scratch of dv_build_visual_memory_noalloc on the current
+// device and context (dv_noalloc.cu). Looking it up loads that file's module, which reserves the
+// array; the plan does this once, so that the entry point itself allocates nothing.
+int noalloc_scratch(void** out);
+// The scratch address the plan looked up when it was made (null if that failed).
+void* plan_scratch(const dv_plan* p);
 
 // Everything one build needs besides the plan: caller tensors and where the intermediates go.
 struct BuildArgs {

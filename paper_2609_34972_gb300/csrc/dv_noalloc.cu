@@ -12,10 +12,12 @@
 // workspace. The plan's repacked weights are still used; nothing here allocates.
 //
 // Behaviour a caller must know:
-//   - The array exists once per device that loads this library and lives until the process
-//     exits, whether or not this entry point is ever called.
-//   - Its device address is looked up (cudaGetSymbolAddress) by the first call on each device,
-//     with that device current; that set-up call should come before any stream capture.
+//   - The array exists once per device (and context) that loads this file's module, and lives
+//     until the process exits. CUDA loads modules lazily, so the array is reserved when the
+//     first plan on a device is made: dv_memory_plan looks up the array's device address
+//     (cudaGetSymbolAddress, with the plan's device current), which loads the module, and also
+//     loads every kernel a build can launch. The entry point therefore allocates nothing, even
+//     on its first call, and needs no set-up step of its own.
 //   - Every call on a device uses the same array. Calls whose kernels overlap on the GPU (on
 //     different streams, or from different threads without ordering) race on it and produce
 //     wrong output; order them on one stream.
@@ -24,40 +26,30 @@
 //     call's token count, so stale rows are never loaded.
 //   - A build that needs more than kScratchBytes of intermediates is rejected with
 //     DV_ERR_UNSUPPORTED_SHAPE before anything is launched.
-#include <mutex>
-
+//   - The address belongs to the CUDA context the plan was made in; cudaDeviceReset ends that
+//     context and invalidates plans and the array alike.
 #include "../../include/dv.h"
 #include "dv_internal.h"
 
 namespace {
 
 constexpr size_t kScratchBytes = 32ull << 20;  // 32 MiB per device
-constexpr int kMaxDevices = 64;
 
 static __device__ __align__(256) unsigned char g_build_scratch[kScratchBytes];
 
-std::mutex g_setup_mutex;
-void* g_scratch_addr[kMaxDevices] = {};
+}  // namespace
 
-// Device address of g_build_scratch on the current device (looked up once per device).
-int scratch_address(void** out) {
-  int dev = 0;
-  if (cudaGetDevice(&dev) != cudaSuccess) return DV_ERR_CUDA;
-  if (dev < 0 || dev >= kMaxDevices) return DV_ERR_UNSUPPORTED_DEVICE;
-  std::lock_guard<std::mutex> lock(g_setup_mutex);
-  if (!g_scratch_addr[dev]) {
-    void* ptr = nullptr;
-    if (cudaGetSymbolAddress(&ptr, g_build_scratch) != cudaSuccess || !ptr) {
-      cudaGetLastError();
-      return DV_ERR_CUDA;
-    }
-    g_scratch_addr[dev] = ptr;
+// In host code g_build_scratch names a host-side stand-in, not device memory: kernels get the
+// address that cudaGetSymbolAddress returns for the current device.
+int dv::noalloc_scratch(void** out) {
+  void* ptr = nullptr;
+  if (cudaGetSymbolAddress(&ptr, g_build_scratch) != cudaSuccess || !ptr) {
+    cudaGetLastError();
+    return DV_ERR_CUDA;
   }
-  *out = g_scratch_addr[dev];
+  *out = ptr;
   return DV_OK;
 }
-
-}  // namespace
 
 extern "C" int dv_build_visual_memory_noalloc(dv_plan* plan, const void* x0, int batch,
                                               int n_vis, const int* pos, const int* slot,
@@ -72,12 +64,15 @@ extern "C" int dv_build_visual_memory_noalloc(dv_plan* plan, const void* x0, int
   // Scratch layout: the build's intermediates as carve_workspace lays them out for T tokens.
   const size_t bytes = dv::carve_workspace(v, T, nullptr, nullptr);
   if (bytes > kScratchBytes || T > (1LL << 24)) return DV_ERR_UNSUPPORTED_SHAPE;
-  if (v.adapter == DV_ADAPTER_RECURRENT && static_cast<long long>(v.n_layers) * T + 128 >= (1LL << 31))
+  // the recurrent K/V GEMM addresses the stacked M_l with 32-bit TMA row coordinates (the
+  // plan applies the same limit to its own workspace)
+  if (v.adapter == DV_ADAPTER_RECURRENT &&
+      static_cast<long long>(v.n_layers) * T + dv::kBlockM >= (1LL << 31))
     return DV_ERR_UNSUPPORTED_SHAPE;
 
-  void* base = nullptr;
-  rc = scratch_address(&base);
-  if (rc != DV_OK) return rc;
+  // looked up when the plan was made (see above); null if the array could not be reserved then
+  void* base = dv::plan_scratch(plan);
+  if (!base) return DV_ERR_OOM;
 
   dv::BuildArgs a;
   a.x0 = x0;

@@ -47,6 +47,14 @@ def test_null_arguments_rejected(dv):
     assert lib.dv_plan_status(None) == dv.DV_ERR_INVALID_ARG
     assert lib.dv_debug_copy_memory(None, 0, None, None) == dv.DV_ERR_INVALID_ARG
     lib.dv_free(None)  # no-op
+    pipe = ctypes.c_void_p(7)
+    assert lib.dv_host_pipeline_create(None, 1, 1, 2, ctypes.byref(pipe)) == dv.DV_ERR_INVALID_ARG
+    assert pipe.value is None                       # set to NULL on error
+    assert lib.dv_host_pipeline_create(None, 1, 1, 2, None) == dv.DV_ERR_INVALID_ARG
+    assert lib.dv_build_visual_memory_host(None, None, None, None, None, None, None) == dv.DV_ERR_INVALID_ARG
+    assert lib.dv_host_pipeline_wait(None, 0) == dv.DV_ERR_INVALID_ARG
+    assert lib.dv_host_pipeline_join(None, None) == dv.DV_ERR_INVALID_ARG
+    lib.dv_host_pipeline_free(None)  # no-op
     with pytest.raises(ValueError):
         dv.make_config(512, 4, 8, 64, 16, adapter="stacked")
 

@@ -111,23 +111,99 @@ def test_gpu_matches_cublas_bf16_sanity(env):
     dv.free(plan)
 
 
+def _host_kv(cfg, torch, fill=0.0, pinned=True):
+    shape = (cfg.n_layers, cfg.batch, cfg.n_vis, cfg.n_kv_heads, cfg.head_dim)
+    k = torch.full(shape, fill, dtype=torch.bfloat16)
+    v = torch.full(shape, fill, dtype=torch.bfloat16)
+    return (k.pin_memory(), v.pin_memory()) if pinned else (k, v)
+
+
 def test_host_pipeline_matches_device_build(env):
-    # The overlapped host path returns, for every submitted build, exactly the device build's K/V.
+    # dv_build_visual_memory_host through the C ABI: every submitted build returns in its host
+    # buffers exactly the K/V of the device build of the same E (bit for bit), with two staging
+    # sets in flight and builds of different E alternating.
     import torch
     dv, inp, plan = env
     cfg = inp.cfg
     k_ref, v_ref, _ = gu.run_build(inp, plan=plan)
+    x0_b = gu.torch_bf16(synth.normal_bf16(77, 0, inp.x0.shape, 0.0, 1.0), "cuda")
+    pos_d = torch.from_numpy(np.ascontiguousarray(inp.pos)).cuda()
+    kb_ref, vb_ref = _cache(cfg, torch)
+    dv.build_visual_memory(plan, x0_b, pos_d, kb_ref, vb_ref)
+    torch.cuda.synchronize()
     x0_h = gu.torch_bf16(inp.x0, "cpu").pin_memory()
+    xb_h = x0_b.cpu().pin_memory()
     pos_h = torch.from_numpy(np.ascontiguousarray(inp.pos)).pin_memory()
-    x0_b = gu.torch_bf16(synth.normal_bf16(77, 0, inp.x0.shape, 0.0, 1.0), "cpu").pin_memory()
-    shape = tuple(k_ref.shape)
-    pipe = dv.HostPipeline(plan, tuple(x0_h.shape), tuple(pos_h.shape), shape)
-    outs = [(torch.empty(shape, dtype=torch.bfloat16).pin_memory(),
-             torch.empty(shape, dtype=torch.bfloat16).pin_memory()) for _ in range(4)]
+    pipe = dv.HostPipeline(plan, cfg.batch, cfg.n_vis, depth=2)
+    outs = [_host_kv(cfg, torch, -9.0) for _ in range(5)]
+    tickets = [pipe.submit(x0_h if i % 2 == 0 else xb_h, pos_h, kh, vh) for i, (kh, vh) in enumerate(outs)]
+    assert tickets == list(range(5))
+    for t in tickets:
+        pipe.wait(t)
     for i, (kh, vh) in enumerate(outs):
-        pipe.submit(x0_h if i % 2 == 0 else x0_b, pos_h, kh, vh)
-    pipe.synchronize()
-    for i in (0, 2):
-        assert torch.equal(outs[i][0], k_ref.cpu()) and torch.equal(outs[i][1], v_ref.cpu())
-    assert not torch.equal(outs[1][0], k_ref.cpu())
-    assert torch.equal(outs[1][0], outs[3][0]) and torch.equal(outs[1][1], outs[3][1])
+        kr, vr = (k_ref, v_ref) if i % 2 == 0 else (kb_ref, vb_ref)
+        assert torch.equal(kh, kr.cpu()) and torch.equal(vh, vr.cpu()), f"build {i}"
+    assert dv.plan_status(plan) == dv.DV_OK
+    with pytest.raises(dv.DvError):
+        pipe.wait(99)                 # not issued yet
+    pipe.close()
+
+
+def test_host_pipeline_join_orders_a_stream(env):
+    # join(stream): work enqueued on the stream afterwards sees the finished copy-out; the copy-in
+    # of a build starts after the stream's earlier work (here: the host buffer the stream wrote).
+    import torch
+    dv, inp, plan = env
+    cfg = inp.cfg
+    k_ref, v_ref, _ = gu.run_build(inp, plan=plan)
+    pos_h = torch.from_numpy(np.ascontiguousarray(inp.pos)).pin_memory()
+    x0_h = torch.zeros((cfg.batch, cfg.n_vis, cfg.d), dtype=torch.bfloat16).pin_memory()
+    x0_d = gu.torch_bf16(inp.x0, "cuda")
+    kh, vh = _host_kv(cfg, torch)
+    side = torch.cuda.Stream()
+    pipe = dv.HostPipeline(plan, cfg.batch, cfg.n_vis, depth=1)
+    with torch.cuda.stream(side):
+        torch.cuda._sleep(2_000_000)                  # keep the stream busy before its copy
+        x0_h.copy_(x0_d, non_blocking=True)           # E reaches the host buffer on the stream
+    pipe.submit(x0_h, pos_h, kh, vh, stream=side)
+    pipe.join(side)
+    done = torch.cuda.Event()
+    done.record(side)
+    done.synchronize()
+    assert torch.equal(kh, k_ref.cpu()) and torch.equal(vh, v_ref.cpu())
+    pipe.close()
+
+
+def test_host_pipeline_dropped_layers_and_pageable_memory():
+    # With DV_LAYER_DROP layers the host rows of those layers stay untouched and the others equal
+    # the device build's; pageable host buffers give the same bytes as page-locked ones.
+    import torch
+    import paper_2609_34972_gb300 as dv
+    cfg = synth.config("tiny", batch=2, n_vis=40, seed=21)
+    inp = synth.make_inputs(cfg)
+    modes = [dv.DV_LAYER_ADAPTER, dv.DV_LAYER_DROP, dv.DV_LAYER_IDENTITY, dv.DV_LAYER_ADAPTER]
+    k_ref, v_ref, plan = gu.run_build(inp, layer_modes=modes, fill=-5.0)
+    x0_h = gu.torch_bf16(inp.x0, "cpu")
+    pos_h = torch.from_numpy(np.ascontiguousarray(inp.pos))
+    pipe = dv.HostPipeline(plan, cfg.batch, cfg.n_vis)
+    for pinned in (True, False):
+        kh, vh = _host_kv(cfg, torch, -5.0, pinned)
+        xh, ph = (x0_h.pin_memory(), pos_h.pin_memory()) if pinned else (x0_h, pos_h)
+        pipe.wait(pipe.submit(xh, ph, kh, vh))
+        assert torch.equal(kh, k_ref.cpu()) and torch.equal(vh, v_ref.cpu()), f"pinned={pinned}"
+        assert bool((kh[1] == -5.0).all()) and bool((vh[1] == -5.0).all())
+    assert dv.plan_status(plan) == dv.DV_OK
+    pipe.close()
+    dv.free(plan)
+
+
+def test_host_pipeline_rejects_shapes_beyond_the_plan(env):
+    dv, inp, plan = env
+    cfg = inp.cfg
+    for b, n, depth, code in [(cfg.batch + 1, cfg.n_vis, 2, dv.DV_ERR_UNSUPPORTED_SHAPE),
+                              (cfg.batch, cfg.n_vis + 1, 2, dv.DV_ERR_UNSUPPORTED_SHAPE),
+                              (cfg.batch, cfg.n_vis, 0, dv.DV_ERR_INVALID_ARG),
+                              (cfg.batch, cfg.n_vis, 5, dv.DV_ERR_INVALID_ARG)]:
+        with pytest.raises(dv.DvError) as e:
+            dv.HostPipeline(plan, b, n, depth=depth)
+        assert e.value.code == code

@@ -45,6 +45,29 @@ def test_tiny_zero_up_projection():
     _full_check(inp, "tiny zero-U")
 
 
+@pytest.mark.parametrize("n_vis,batch,rank", [(64, 1, 16), (256, 2, 64), (300, 1, 128), (576, 1, 64)])
+def test_zero_up_projection_is_bit_identical_to_identity_layers(n_vis, batch, rank):
+    # U = 0 is the paper's initialisation, so A_l starts as the identity (Sec. 3.1). The fold
+    # then multiplies h_l by exact zeros (the rank slab of the K/V weights, 2U and G of the
+    # statistic), so the build must equal, value for value, a build whose layers are all
+    # DV_LAYER_IDENTITY (D = U = 0 packed, M_l = E): the adapter path adds nothing, not even
+    # rounding. Cases: both K/V engines, the small-token statistic and the statistic GEMM.
+    import torch
+    import paper_2609_34972_gb300 as dv
+    cfg = gu.small_config(f"zu_{n_vis}_{batch}_{rank}", d=512, n_layers=3, n_kv_heads=2, n_heads=4,
+                          head_dim=128, rank=rank, n_vis=n_vis, batch=batch, zero_up=True,
+                          x0_sigma=0.5, seed=71, pos_start=35)
+    inp = synth.make_inputs(cfg)
+    k_a, v_a, plan_a = gu.run_build(inp)
+    k_i, v_i, plan_i = gu.run_build(inp, layer_modes=[dv.DV_LAYER_IDENTITY] * cfg.n_layers)
+    assert torch.equal(k_a, k_i) and torch.equal(v_a, v_i)
+    # and it is not vacuous: the adapter's down-projection was live (h_l != 0)
+    H, _, _, _ = dv.debug_workspace(plan_a, cfg.tokens)
+    assert bool((H != 0).any())
+    dv.free(plan_a)
+    dv.free(plan_i)
+
+
 def test_tiny_with_bias():
     inp = synth.make_inputs(synth.config("tiny", bias_sigma=0.02))
     _full_check(inp, "tiny bias")

@@ -5,7 +5,9 @@ the build's intermediates in the library's static device array. This file is col
 so that, if it fails, a run that stops at the first failure has already run every other test.
 It must also pass on its own in a fresh process.
 """
-import ctypes
+import os
+import subprocess
+import sys
 
 import numpy as np
 import pytest
@@ -92,3 +94,41 @@ def test_noalloc_rejects_builds_over_its_limit(dv):
     _check_close(dv, one, k2, v2, k1, v1)
     dv.free(plan)
     dv.free(plan_ref)
+
+
+_FIRST_CALL = r"""
+import sys
+import numpy as np
+import torch
+sys.path.insert(0, sys.argv[1])
+import synth
+import paper_2609_34972_gb300 as dv
+from tests import gpu_util as gu
+torch.cuda.set_device(0)
+cfg = synth.CONFIGS[sys.argv[2]]
+inp = synth.make_inputs(cfg)
+plan = dv.memory_plan(gu.dv_config(cfg), gu.device_weights(inp))
+x0 = gu.torch_bf16(inp.x0, "cuda")
+pos = torch.from_numpy(np.ascontiguousarray(inp.pos)).cuda()
+shape = (cfg.n_layers, cfg.batch, cfg.n_vis, cfg.n_kv_heads, cfg.head_dim)
+k = torch.zeros(shape, dtype=torch.bfloat16, device="cuda")
+v = torch.zeros(shape, dtype=torch.bfloat16, device="cuda")
+torch.cuda.synchronize()
+free_before = torch.cuda.mem_get_info()[0]
+dv.build_visual_memory_noalloc(plan, x0, pos, k, v)   # the first build of this process
+torch.cuda.synchronize()
+free_after = torch.cuda.mem_get_info()[0]
+assert dv.plan_status(plan) == dv.DV_OK
+print("free before", free_before, "after", free_after)
+sys.exit(0 if free_before == free_after else 3)
+"""
+
+
+@pytest.mark.parametrize("name", ["tiny", "llava15_7b"])
+def test_first_call_allocates_nothing(dv, name):
+    # In a fresh process, the first no-allocation build after dv_memory_plan leaves the device's
+    # free memory unchanged: the plan reserved the static array and loaded the build's kernels.
+    root = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+    r = subprocess.run([sys.executable, "-c", _FIRST_CALL, root, name], capture_output=True,
+                       text=True, timeout=600, cwd=root)
+    assert r.returncode == 0, r.stdout[-2000:] + r.stderr[-4000:]
