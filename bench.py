@@ -5,10 +5,18 @@ One step = one build of every layer's visual K/V cache entries for one batch of 
 visual embeddings: row statistics, stacked down-projection + SiLU, RMS statistics, and the
 K/V projection with RoPE and the bf16 cache store, all in the library's CUDA kernels.
 
-    python bench.py [--gpus N] [--steps K] [--warmup W] [--config NAME] [--impl dv|reference]
+The headline workload is the largest synthetic configuration that fits one GPU, the
+LLaVA-NeXT-7B-shaped high-resolution batch (d = 4096, L = 32, 32 x 128 MHA, r = 128,
+8 x 2880 visual tokens). The line also carries ``per_config``: the LLaVA-1.5-7B-shaped and
+both Qwen2.5-VL-7B-shaped workloads, each device-timed with its own roofline.
 
-Prints ONE JSON line on rank 0. Under torchrun (N > 1) every rank builds its own batch of the
-workload (weak scaling, no collective on the data path); timing is the max over ranks.
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--config NAME] [--impl dv|reference]
+                    [--shard replicas|tokens|layers]
+
+Prints ONE JSON line on rank 0. Under torchrun (N > 1) the ranks split the work as --shard
+says: every rank builds its own batch (replicas, weak scaling, no collective on the data path),
+or the ranks split one batch's tokens (no collective) or its layers (x0 broadcast from rank 0
+every step); timing is the max over ranks.
 ``--impl reference`` times the fp64 oracle on the host cores instead (bounded samples).
 """
 from __future__ import annotations
@@ -29,7 +37,9 @@ if ROOT not in sys.path:
 
 METRIC = "visual tokens/sec of layer-wise visual KV-memory build; % of BF16 tensor roofline"
 UNIT = "visual tokens/s"
-DEFAULT_WORKLOAD = "llava15_7b"
+DEFAULT_WORKLOAD = "llava_next_7b"
+# device-timed beside the headline (each with its own roofline)
+PER_CONFIG = ["llava15_7b", "qwen25vl_7b_image", "qwen25vl_7b_video"]
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
 GEMM_SOURCES = ["paper_2609_34972_gb300/csrc/dv_kv2sm.cu", "paper_2609_34972_gb300/csrc/dv_pair_tm.cu",
                 "paper_2609_34972_gb300/csrc/dv_ptx.cuh",
@@ -147,23 +157,47 @@ def weak_scaling_value(world: int, tokens_per_rank: int, steps: int, ms_max: flo
     return world * tokens_per_rank * steps / (ms_max / 1000.0)
 
 
-def time_oracle_sample(inp, budget_s: float, seed: int = 0):
-    """Oracle throughput (tokens/s) on a bounded sample of whole tokens (all layers)."""
+def stratified_tokens(cfg, n: int, seed: int = 0):
+    """n flat token ids spread over every batch element: each element gets its share at evenly
+    spaced positions with a random offset, so the sample covers the whole position range."""
+    import numpy as np
+    rng = np.random.default_rng(seed)
+    n = int(max(1, min(n, cfg.tokens)))
+    per = [n // cfg.batch + (1 if b < n % cfg.batch else 0) for b in range(cfg.batch)]
+    out = []
+    for b, k in enumerate(per):
+        if k == 0:
+            continue
+        step = cfg.n_vis / k
+        idx = np.floor(np.arange(k) * step + rng.uniform(0, step, size=k)).astype(np.int64)
+        out.append(b * cfg.n_vis + np.minimum(idx, cfg.n_vis - 1))
+    return np.unique(np.concatenate(out))
+
+
+def strong_scaling_value(tokens_per_step: int, steps: int, ms_max: float) -> float:
+    """Whole-job visual tokens/s when the ranks split one batch (by tokens or by layers): the
+    job processes the batch's tokens once per step, whatever the rank count."""
+    return tokens_per_step * steps / (ms_max / 1000.0)
+
+
+def time_oracle_sample(inp, budget_s: float, seed: int = 0, min_tokens: int = 0):
+    """Oracle throughput (tokens/s) on a bounded, stratified sample of whole tokens (all
+    layers): at least min_tokens, else as many as about budget_s of oracle time allows."""
     import numpy as np
     import oracle
     cfg = inp.cfg
-    rng = np.random.default_rng(seed)
     t0 = time.perf_counter()
     oracle.build_tokens(inp, np.array([0], dtype=np.int64))
     t1 = time.perf_counter() - t0
-    n = int(max(1, min(cfg.tokens, budget_s / max(t1, 1e-6))))
-    toks = np.sort(rng.choice(cfg.tokens, size=n, replace=False)).astype(np.int64)
+    n = int(max(1, min(cfg.tokens, max(min_tokens, budget_s / max(t1, 1e-6)))))
+    toks = stratified_tokens(cfg, n, seed)
     t0 = time.perf_counter()
     oracle.build_tokens(inp, toks)
     dt = time.perf_counter() - t0
-    return {"value": n / dt, "unit": UNIT, "cores": oracle.num_threads(), "kind": "oracle",
-            "sample": f"{n} of {cfg.tokens} tokens (all {cfg.n_layers} layers each) of the "
-                      f"{cfg.name} workload, fp64, {dt:.1f} s"}
+    return {"value": len(toks) / dt, "unit": UNIT, "cores": oracle.num_threads(), "kind": "oracle",
+            "sample": f"{len(toks)} of {cfg.tokens} tokens (all {cfg.n_layers} layers each), "
+                      f"spread evenly over all {cfg.batch} batch elements, of the {cfg.name} "
+                      f"workload, fp64, {dt:.1f} s; tokens/s = sampled tokens / oracle time"}
 
 
 def workload_config(args):
@@ -231,6 +265,113 @@ def run_reference(args):
     print(json.dumps(out), flush=True)
 
 
+def roofline_of(dv, plan, work, stage_ms, n_timed, ms_total, ms_step, peaks, peak_src, tokens):
+    """Roofline of the dominant kernel (K/V projection + RoPE + store) and of the whole step."""
+    kv_ms = stage_ms[3] / max(n_timed, 1)
+    kv_flops = 4.0 * work.d * work.kv * work.tokens * work.n_layers
+    # The K/V kernel is timed inside a run of back-to-back builds. Once that run lasts as long
+    # as the seconds-long cuBLAS loop behind the sustained figure (the power cap then sets the
+    # clock), its peak is that sustained rate; shorter runs are compared with the burst rate.
+    sustained = ms_total >= 2000.0
+    peak_tf = peaks["bf16_tflops_sustained"] if sustained else peaks["bf16_tflops"]
+    peak_name = "bf16_tflops_sustained" if sustained else "bf16_tflops (burst)"
+    achieved_tf = kv_flops / (kv_ms * 1e-3) / 1e12
+    t_roof_ms = max(work.flops() / (peaks["bf16_tflops"] * 1e12),
+                    work.min_bytes() / (peaks["hbm_gbs"] * 1e9)) * 1e3
+    t_roof_sus = max(work.flops() / (peaks["bf16_tflops_sustained"] * 1e12),
+                     work.min_bytes() / (peaks["hbm_gbs"] * 1e9)) * 1e3
+    roof = {"bound": "tensor", "achieved": achieved_tf, "peak": peak_tf, "unit": "TFLOP/s",
+            "frac": achieved_tf / peak_tf, "traffic": profiled_traffic(work.name),
+            "kernel": dv.kv_kernel(plan, tokens) + ": K/V projection + RoPE + cache store",
+            "peak_source": f"{peak_name} of {peak_src}; timed region {ms_total:.0f} ms of "
+                           f"back-to-back builds",
+            "frac_burst": achieved_tf / peaks["bf16_tflops"],
+            "frac_sustained": achieved_tf / peaks["bf16_tflops_sustained"],
+            "flops_per_launch": kv_flops, "ms_per_launch": kv_ms}
+    step = {"t_roof_ms": t_roof_ms, "frac": t_roof_ms / ms_step, "frac_sustained": t_roof_sus / ms_step,
+            "plain_flops": work.flops(), "min_bytes": work.min_bytes()}
+    return roof, step
+
+
+def time_builds(dv, plan, build, steps, warmup, stream, barrier=None, clocks=None):
+    """Device time (ms) of `steps` back-to-back builds after `warmup` untimed ones, CUDA events
+    on the build stream; then the per-stage times from a second run with the plan's stage events
+    (kept out of the timed run: an event between two kernels stops the next one from starting
+    early)."""
+    import torch
+    for _ in range(warmup):
+        build()
+    torch.cuda.synchronize()
+    st = dv.plan_status(plan)
+    if st != dv.DV_OK:
+        raise RuntimeError(f"device status after warm-up: {dv.error_string(st)}")
+    if barrier:
+        barrier()
+    torch.cuda.synchronize()
+    if clocks:
+        clocks.start()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(steps):
+        build()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    clk = clocks.stop() if clocks else None
+    if barrier:
+        barrier()
+    ms_total = e0.elapsed_time(e1)
+    dv.timing_enable(plan, True)
+    for _ in range(min(steps, 200)):
+        build()
+    torch.cuda.synchronize()
+    stage_ms, n_timed = dv.timing_read(plan)
+    dv.timing_enable(plan, False)
+    st = dv.plan_status(plan)
+    if st != dv.DV_OK:
+        raise RuntimeError(f"device status after timed region: {dv.error_string(st)}")
+    return ms_total, clk, stage_ms, n_timed
+
+
+def gpu_id_of(dev, local):
+    import torch
+    try:
+        return "GPU-" + str(torch.cuda.get_device_properties(dev).uuid)
+    except Exception:
+        return str(local)
+
+
+def measure_config(dv, name, args, dev, peaks, peak_src):
+    """Device-timed build of one more workload (inputs resident), for the per_config block."""
+    import numpy as np
+    import torch
+    import synth
+    from tests import gpu_util as gu
+    cfg = synth.CONFIGS[name]
+    inp = synth.make_inputs(cfg)
+    plan = dv.memory_plan(gu.dv_config(cfg), gu.device_weights(inp, dev))
+    x0 = gu.torch_bf16(inp.x0, dev)
+    pos = torch.from_numpy(np.ascontiguousarray(inp.pos)).to(dev)
+    shape = (cfg.n_layers, cfg.batch, cfg.n_vis, cfg.n_kv_heads, cfg.head_dim)
+    kc = torch.zeros(shape, dtype=torch.bfloat16, device=dev)
+    vc = torch.zeros(shape, dtype=torch.bfloat16, device=dev)
+    stream = torch.cuda.current_stream()
+    build = lambda: dv.build_visual_memory(plan, x0, pos, kc, vc, stream=stream)
+    ms_total, clk, stage_ms, n_timed = time_builds(dv, plan, build, args.steps, args.warmup, stream,
+                                                   clocks=ClockSampler(gpu_id_of(dev, 0)))
+    ms_step = ms_total / args.steps
+    roof, step = roofline_of(dv, plan, cfg, stage_ms, n_timed, ms_total, ms_step, peaks, peak_src,
+                             cfg.tokens)
+    out = {"workload": cfg.name, "description": cfg.description, "tokens_per_step": cfg.tokens,
+           "value": cfg.tokens * args.steps / (ms_total / 1000.0), "unit": UNIT,
+           "ms_per_step": ms_step, "steps": args.steps, "clocks": clk, "roofline": roof,
+           "roofline_step": step,
+           "stage_ms_per_step": dict(zip(dv.stage_names(plan), [x / max(n_timed, 1) for x in stage_ms]))}
+    dv.free(plan)
+    del kc, vc, x0, pos
+    torch.cuda.empty_cache()
+    return out
+
+
 def run_dv(args):
     import numpy as np
     import torch
@@ -238,8 +379,13 @@ def run_dv(args):
     from paper_2609_34972_gb300.build import build_library
     build_library()
     import paper_2609_34972_gb300 as dv
+    from paper_2609_34972_gb300 import shard as sh
+    from tests import gpu_util as gu
 
     rank, world, local = dist_env()
+    if world != args.gpus:
+        raise SystemExit(f"--gpus {args.gpus} but {world} process(es): launch N > 1 under torchrun "
+                         f"with --nproc-per-node N")
     dist = None
     if world > 1:
         import torch.distributed as tdist
@@ -249,27 +395,41 @@ def run_dv(args):
     dev = torch.device("cuda", local)
     cfg = workload_config(args)
     peaks, peak_src = load_peaks()
+    mode = args.shard if world > 1 else "replicas"
+    if mode == "layers" and cfg.adapter == "recurrent":
+        raise SystemExit("the recurrent adapter chains the layers: split it by tokens")
     modes = None
-    layers_built = cfg.n_layers
     if args.skip_layers:
         first, last = (int(x) for x in args.skip_layers.split(","))
         modes = [dv.DV_LAYER_DROP if (l < first or l >= cfg.n_layers - last) else dv.DV_LAYER_ADAPTER
                  for l in range(cfg.n_layers)]
-        layers_built = sum(m != dv.DV_LAYER_DROP for m in modes)
-    from dataclasses import replace as _replace
-    # the algorithmic work counts the layers that get visual memory
-    work = _replace(cfg, n_layers=layers_built,
-                    name=cfg.name + (f"_skip{args.skip_layers.replace(',', '_')}" if modes else ""))
+    if mode == "layers":
+        modes = sh.layer_modes(cfg.n_layers, world, rank, modes)
+    layers_built = cfg.n_layers if modes is None else sum(m != dv.DV_LAYER_DROP for m in modes)
 
     # ---- inputs (host, seeded) -> device; plan once outside the timing
     inp = synth.make_inputs(cfg)
-    from tests import gpu_util as gu
+    x0_full = gu.torch_bf16(inp.x0, "cpu")
+    pos_np = np.ascontiguousarray(inp.pos)
+    if mode == "tokens":
+        part = sh.token_shard(cfg.batch, cfg.n_vis, world, rank)
+        B, N = 1, part.tokens
+        x0_h = x0_full.reshape(cfg.tokens, cfg.d)[part.start:part.stop].reshape(1, N, cfg.d).contiguous()
+        pos_h = torch.from_numpy(sh.shard_positions(pos_np, part))
+    else:
+        B, N = cfg.batch, cfg.n_vis
+        x0_h, pos_h = x0_full, torch.from_numpy(pos_np)
+    T = B * N
+    from dataclasses import replace as _replace
+    # the algorithmic work this rank does: its tokens and the layers that get visual memory
+    work = _replace(cfg, batch=B, n_vis=N, n_layers=layers_built,
+                    name=cfg.name + (f"_skip{args.skip_layers.replace(',', '_')}" if args.skip_layers else ""))
     weights = gu.device_weights(inp, dev)
-    plan = dv.memory_plan(gu.dv_config(cfg), weights, layer_modes=modes)
+    plan = dv.memory_plan(gu.dv_config(cfg, max_batch=B, max_n_vis=N), weights, layer_modes=modes)
     del weights
-    x0 = gu.torch_bf16(inp.x0, dev)
-    pos = torch.from_numpy(np.ascontiguousarray(inp.pos)).to(dev)
-    shape = (cfg.n_layers, cfg.batch, cfg.n_vis, cfg.n_kv_heads, cfg.head_dim)
+    x0 = x0_h.to(dev)
+    pos = pos_h.to(dev)
+    shape = (cfg.n_layers, B, N, cfg.n_kv_heads, cfg.head_dim)
     kc = torch.zeros(shape, dtype=torch.bfloat16, device=dev)
     vc = torch.zeros(shape, dtype=torch.bfloat16, device=dev)
     stream = torch.cuda.current_stream()
@@ -278,135 +438,104 @@ def run_dv(args):
         if dist is not None:
             dist.barrier()
 
-    # ---- warm-up
-    for _ in range(args.warmup):
+    def build():
+        if mode == "layers":
+            dist.broadcast(x0, src=0)   # E from rank 0: the one collective of the layer split
         dv.build_visual_memory(plan, x0, pos, kc, vc, stream=stream)
-    torch.cuda.synchronize()
-    st = dv.plan_status(plan)
-    if st != dv.DV_OK:
-        raise RuntimeError(f"device status after warm-up: {dv.error_string(st)}")
 
     # ---- timed region (device-resident inputs)
-    gpu_id = None
-    try:
-        gpu_id = "GPU-" + str(torch.cuda.get_device_properties(dev).uuid)
-    except Exception:
-        gpu_id = str(local)
-    clocks = ClockSampler(gpu_id)
-    barrier()
-    torch.cuda.synchronize()
-    clocks.start()
-    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    e0.record(stream)
-    for _ in range(args.steps):
-        dv.build_visual_memory(plan, x0, pos, kc, vc, stream=stream)
-    e1.record(stream)
-    torch.cuda.synchronize()
-    clk = clocks.stop()
-    barrier()
-    ms_total = e0.elapsed_time(e1)
-    # Per-stage times come from a second run right after it, with the plan's stage events
-    # between the kernels (kept out of the timed run: an event between two kernels stops the
-    # next one from starting early).
-    dv.timing_enable(plan, True)
-    for _ in range(min(args.steps, 200)):
-        dv.build_visual_memory(plan, x0, pos, kc, vc, stream=stream)
-    torch.cuda.synchronize()
-    stage_ms, n_timed = dv.timing_read(plan)
-    dv.timing_enable(plan, False)
-    st = dv.plan_status(plan)
-    if st != dv.DV_OK:
-        raise RuntimeError(f"device status after timed region: {dv.error_string(st)}")
+    ms_total, clk, stage_ms, n_timed = time_builds(dv, plan, build, args.steps, args.warmup, stream,
+                                                   barrier, ClockSampler(gpu_id_of(dev, local)))
     ms_total = max_over_ranks(ms_total, dist, dev)
     ms_step = ms_total / args.steps
-    value = weak_scaling_value(world, cfg.tokens, args.steps, ms_total)
+    # replicas: every rank builds its own batch; token / layer splits: the ranks build one batch
+    job_tokens = world * T if mode == "replicas" else cfg.tokens
+    value = (weak_scaling_value(world, T, args.steps, ms_total) if mode == "replicas"
+             else strong_scaling_value(cfg.tokens, args.steps, ms_total))
 
-    # ---- end to end through host buffers (pinned), copies inside the timed region: every step
-    #      copies its E and positions host-to-device and reads its K/V back device-to-host; the
-    #      read of one step overlaps the build of the next (dv.HostPipeline)
-    x0_h = gu.torch_bf16(inp.x0, "cpu").pin_memory()
-    pos_h = torch.from_numpy(np.ascontiguousarray(inp.pos)).pin_memory()
-    k_h = [torch.empty(shape, dtype=torch.bfloat16).pin_memory() for _ in range(2)]
-    v_h = [torch.empty(shape, dtype=torch.bfloat16).pin_memory() for _ in range(2)]
+    # ---- end to end through the C ABI from page-locked host buffers: every step copies its E
+    #      and positions host-to-device and its built K/V device-to-host inside the timed region
+    #      (dv_build_visual_memory_host); the copy-out of one step overlaps the next build
+    x0_p = x0_h.pin_memory()
+    pos_p = pos_h.pin_memory()
+    k_p = torch.empty(shape, dtype=torch.bfloat16).pin_memory()
+    v_p = torch.empty(shape, dtype=torch.bfloat16).pin_memory()
     e2e_steps = max(5, min(args.steps, args.e2e_steps))
-    pipe = dv.HostPipeline(plan, tuple(x0.shape), tuple(pos.shape), shape)
-    for i in range(3):
-        pipe.submit(x0_h, pos_h, k_h[i % 2], v_h[i % 2])
-    pipe.synchronize()
+    pipe = dv.HostPipeline(plan, B, N, depth=2)
+    for _ in range(3):
+        pipe.submit(x0_p, pos_p, k_p, v_p, stream=stream)
+    pipe.join(stream)
+    torch.cuda.synchronize()
     barrier()
     s0, s1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    s0.record(pipe.compute)
-    for i in range(e2e_steps):
-        done = pipe.submit(x0_h, pos_h, k_h[i % 2], v_h[i % 2])
-    pipe.compute.wait_event(done)
-    s1.record(pipe.compute)
-    pipe.synchronize()
+    s0.record(stream)
+    for _ in range(e2e_steps):
+        pipe.submit(x0_p, pos_p, k_p, v_p, stream=stream)
+    pipe.join(stream)
+    s1.record(stream)
+    torch.cuda.synchronize()
     barrier()
-    ms_e2e = s0.elapsed_time(s1)
-    ms_e2e = max_over_ranks(ms_e2e, dist, dev)
-    e2e_value = weak_scaling_value(world, cfg.tokens, e2e_steps, ms_e2e)
-    h2d = x0_h.numel() * 2 + pos_h.numel() * 4
-    d2h = (k_h[0].numel() + v_h[0].numel()) * 2
+    ms_e2e = max_over_ranks(s0.elapsed_time(s1), dist, dev)
+    e2e_value = job_tokens * e2e_steps / (ms_e2e / 1000.0)
+    h2d = x0_p.numel() * 2 + pos_p.numel() * 4
+    d2h = 2 * layers_built * T * cfg.kv * 2
     st = dv.plan_status(plan)
     if st != dv.DV_OK:
         raise RuntimeError(f"device status after the end-to-end region: {dv.error_string(st)}")
-    del pipe
+    pipe.close()
+    del pipe, k_p, v_p
 
-    # ---- roofline of the dominant kernel (K/V projection + RoPE + store) and of the step
-    kv_ms = stage_ms[3] / max(n_timed, 1)
-    kv_flops = 4.0 * work.d * work.kv * work.tokens * work.n_layers
-    # The K/V kernel is timed inside a run of back-to-back builds. Once that run lasts long
-    # enough for the power cap to set the clock (about half a second), its peak is the
-    # sustained cuBLAS rate (a seconds-long loop under the same cap); a short run is compared
-    # with the burst rate.
-    sustained = ms_total >= 500.0
-    peak_tf = peaks["bf16_tflops_sustained"] if sustained else peaks["bf16_tflops"]
-    peak_name = "bf16_tflops_sustained" if sustained else "bf16_tflops (burst)"
-    achieved_tf = kv_flops / (kv_ms * 1e-3) / 1e12
-    t_roof_ms = max(work.flops() / (peaks["bf16_tflops"] * 1e12),
-                    work.min_bytes() / (peaks["hbm_gbs"] * 1e9)) * 1e3
-    traffic = profiled_traffic(work.name)
+    roof, roof_step = roofline_of(dv, plan, work, stage_ms, n_timed, ms_total, ms_step, peaks,
+                                  peak_src, T)
+    stage = dict(zip(dv.stage_names(plan), [x / max(n_timed, 1) for x in stage_ms]))
+    launches = args.steps * dv.kernels_per_build(plan)
+    dv.free(plan)
+    del kc, vc
+    torch.cuda.empty_cache()
 
     cpu = None
-    if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        cpu = time_oracle_sample(inp, args.cpu_budget_s)
+    per_config = None
+    if rank == 0 and world == 1:
+        if not args.no_per_config and args.config == DEFAULT_WORKLOAD and not args.layers \
+                and args.adapter == "embedding" and not args.skip_layers:
+            per_config = [measure_config(dv, n, args, dev, peaks, peak_src) for n in PER_CONFIG]
+        if not args.no_cpu_baseline:
+            cpu = time_oracle_sample(inp, args.cpu_budget_s,
+                                     min_tokens=min(cfg.tokens, 512) if cfg.batch > 1 else 0)
 
     if rank == 0:
+        par = {"replicas": "replicas (weak scaling, no collective)",
+               "tokens": "token split of one batch (strong scaling, no collective)",
+               "layers": "layer split of one batch (strong scaling, x0 broadcast per step)"}[mode]
         out = {
             "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": True,
-            "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+            "scaling": "weak" if mode == "replicas" else "strong", "vs_baseline": None,
+            "dtype": "bf16", "data": "synthetic",
             "config": {"workload": work.name, "description": cfg.description,
-                       "layers_with_visual_memory": work.n_layers,
-                       "tokens_per_step_per_gpu": cfg.tokens, "layers": cfg.n_layers,
-                       "l2": f"inputs larger than L2: the {work.n_layers}-layer weight set "
+                       "layers_with_visual_memory": layers_built if mode != "layers" else cfg.n_layers,
+                       "tokens_per_step": job_tokens, "tokens_per_step_per_gpu": T,
+                       "layers": cfg.n_layers,
+                       "l2": f"inputs larger than L2: the {layers_built}-layer weight set "
                              f"({(work.min_bytes() - work.tokens * work.n_layers * 4 * work.kv) / 1e9:.2f} GB "
                              f"incl. x0) is streamed from HBM every step",
-                       "parallelism": "replicas (weak scaling, no collective)" if world > 1 else "1 GPU"},
+                       "parallelism": par if world > 1 else "1 GPU"},
             "clocks": clk,
             "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": h2d,
                     "d2h_bytes_per_step": d2h, "steps": e2e_steps,
                     "ms_per_step": ms_e2e / e2e_steps,
-                    "how": "dv.HostPipeline: per step H2D of E + positions, build, D2H of all K/V "
-                           "written; the D2H of a step overlaps the next build"},
-            "gpu_launches": args.steps * dv.kernels_per_build(plan),
-            "roofline": {"bound": "tensor", "achieved": achieved_tf, "peak": peak_tf,
-                         "unit": "TFLOP/s", "frac": achieved_tf / peak_tf, "traffic": traffic,
-                         "kernel": dv.kv_kernel(plan, cfg.tokens) + ": K/V projection + RoPE + cache store",
-                         "peak_source": f"{peak_name} of {peak_src}; timed region {ms_total:.0f} ms of "
-                                        f"back-to-back builds",
-                         "frac_burst": achieved_tf / peaks["bf16_tflops"],
-                         "frac_sustained": achieved_tf / peaks["bf16_tflops_sustained"],
-                         "flops_per_launch": kv_flops, "ms_per_launch": kv_ms},
-            "roofline_step": {"t_roof_ms": t_roof_ms, "frac": t_roof_ms / ms_step,
-                              "frac_sustained": max(work.flops() / (peaks["bf16_tflops_sustained"] * 1e12),
-                                                    work.min_bytes() / (peaks["hbm_gbs"] * 1e9)) * 1e3 / ms_step,
-                              "plain_flops": work.flops(), "min_bytes": work.min_bytes()},
-            "stage_ms_per_step": dict(zip(dv.stage_names(plan), [s / max(n_timed, 1) for s in stage_ms])),
+                    "how": "C ABI dv_build_visual_memory_host (dv_host_pipeline, 2 staging sets): "
+                           "per step one cudaMemcpyAsync each of E and the positions host-to-device "
+                           "from page-locked memory, the build, and one cudaMemcpyAsync each of K "
+                           "and V device-to-host; the copy-out of a step overlaps the next build"},
+            "gpu_launches": launches,
+            "roofline": roof,
+            "roofline_step": roof_step,
+            "stage_ms_per_step": stage,
             "cpu_baseline": cpu,
+            "per_config": per_config,
         }
         print(json.dumps(out), flush=True)
-    dv.free(plan)
     if dist is not None:
         dist.destroy_process_group()
 
@@ -502,7 +631,7 @@ def run_consumer(args):
 def main():
     ap = argparse.ArgumentParser(description=__doc__, formatter_class=argparse.RawDescriptionHelpFormatter)
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=1000)
+    ap.add_argument("--steps", type=int, default=200)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--config", default=DEFAULT_WORKLOAD)
     ap.add_argument("--layers", type=int, default=0,
@@ -520,6 +649,11 @@ def main():
     ap.add_argument("--consumer-sys", type=int, default=35, help="system-prompt slots before the visual slots")
     ap.add_argument("--consumer-text", type=int, default=64, help="text query tokens after them")
     ap.add_argument("--e2e-steps", type=int, default=100)
+    ap.add_argument("--shard", choices=["replicas", "tokens", "layers"], default="replicas",
+                    help="N > 1: every rank builds its own batch (weak scaling), or the ranks "
+                         "split one batch by tokens or by layers (strong scaling)")
+    ap.add_argument("--no-per-config", action="store_true",
+                    help="skip the per_config block (the other workloads, device-timed)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-budget-s", type=float, default=15.0)
     ap.add_argument("--ref-budget-s", type=float, default=120.0)
