@@ -210,6 +210,9 @@ def workload_config(args):
     if args.adapter == "recurrent":
         cfg = replace(cfg, adapter="recurrent", name=f"{cfg.name}_recurrent",
                       description=cfg.description + "; recurrent adapter (Sec. 3.1 Eq. 6)")
+        if args.split_chain:
+            cfg = replace(cfg, split_chain=True, name=cfg.name + "_split",
+                          description=cfg.description + ", split-bf16 chain")
     return cfg
 
 
@@ -642,6 +645,8 @@ def main():
     ap.add_argument("--adapter", choices=["embedding", "recurrent"], default="embedding",
                     help="embedding adapter (Sec. 3.1 Eq. 5, the default workload) or the "
                          "recurrent adapter (Eq. 6)")
+    ap.add_argument("--split-chain", action="store_true",
+                    help="recurrent adapter: the chain's GEMMs read hi + lo bf16 operands")
     ap.add_argument("--impl", choices=["dv", "reference"], default="dv")
     ap.add_argument("--consumer", action="store_true",
                     help="measure the consumer instead: causal text-query attention over every "

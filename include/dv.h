@@ -68,6 +68,7 @@ enum {
  *   head_dim / 2 (interleaved: the layout must give each axis exactly its section's count);
  *   k_norm in {0, 1}; k_norm_eps >= 0;
  *   adapter in {DV_ADAPTER_EMBEDDING, DV_ADAPTER_RECURRENT};
+ *   split_chain in {0, 1}, and 1 only with DV_ADAPTER_RECURRENT;
  *   max_batch * max_n_vis >= 1 and <= 2^24 (the tokens one build may carry). */
 typedef struct dv_config {
   int d;                 /* hidden size of the language model */
@@ -88,6 +89,12 @@ typedef struct dv_config {
                             dv_weights.k_norm_gamma (the per-head K norm of Qwen3-VL backbones,
                             applied after the bias) */
   float k_norm_eps;      /* epsilon inside that norm's square root */
+  int split_chain;       /* recurrent adapter only (0 otherwise): 1 = each bf16 operand of the
+                            chain's two GEMMs (M_{l-1} into the down-projection, h_l into the
+                            up-projection) is read as a high and a low bf16 part, two MMAs per
+                            product, so the state M_l keeps about fp32 accuracy through deep
+                            chains; the chain then runs as per-layer launches. 0 = one bf16
+                            operand (faster, on chip where it fits). */
 } dv_config;
 
 /* Weights of all L layers, bf16, device pointers. Read only during dv_memory_plan: the plan

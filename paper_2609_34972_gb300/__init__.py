@@ -61,7 +61,8 @@ class DvConfig(ctypes.Structure):
                 ("mrope_section", ctypes.c_int * 3), ("rms_eps", ctypes.c_float),
                 ("max_batch", ctypes.c_int), ("max_n_vis", ctypes.c_int),
                 ("has_kv_bias", ctypes.c_int), ("adapter", ctypes.c_int),
-                ("k_norm", ctypes.c_int), ("k_norm_eps", ctypes.c_float)]
+                ("k_norm", ctypes.c_int), ("k_norm_eps", ctypes.c_float),
+                ("split_chain", ctypes.c_int)]
 
 
 class DvWeights(ctypes.Structure):
@@ -157,10 +158,11 @@ def _ptr(t):
 def make_config(d, n_layers, n_kv_heads, head_dim, rank, rope="1d", rope_theta=10000.0,
                 mrope_section=(0, 0, 0), rms_eps=1e-6, max_batch=1, max_n_vis=1,
                 has_kv_bias=False, adapter="embedding", k_norm=False,
-                k_norm_eps=1e-6) -> DvConfig:
+                k_norm_eps=1e-6, split_chain=False) -> DvConfig:
     """``adapter``: "embedding" (M_l = A_l(E), Sec. 3.1 Eq. 5) or "recurrent"
     (M_l = A_l(M_{l-1}), Sec. 3.1 Eq. 6). ``rope``: "1d", "mrope" (contiguous sections) or
-    "mrope_interleaved". ``k_norm``: per-head RMSNorm of K before RoPE (weights["kgamma"])."""
+    "mrope_interleaved". ``k_norm``: per-head RMSNorm of K before RoPE (weights["kgamma"]).
+    ``split_chain`` (recurrent only): the chain's GEMMs read hi + lo bf16 operands."""
     if adapter not in ("embedding", "recurrent"):
         raise ValueError(f"unknown adapter {adapter!r}")
     if rope not in _ROPE:
@@ -170,7 +172,7 @@ def make_config(d, n_layers, n_kv_heads, head_dim, rank, rope="1d", rope_theta=1
                     float(rope_theta), (ctypes.c_int * 3)(*mrope_section), float(rms_eps),
                     int(max_batch), int(max_n_vis), int(bool(has_kv_bias)),
                     DV_ADAPTER_RECURRENT if adapter == "recurrent" else DV_ADAPTER_EMBEDDING,
-                    int(bool(k_norm)), float(k_norm_eps))
+                    int(bool(k_norm)), float(k_norm_eps), int(bool(split_chain)))
 
 
 class Plan:

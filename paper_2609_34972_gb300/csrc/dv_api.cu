@@ -38,7 +38,8 @@ struct dv_plan {
   uint16_t* Dst = nullptr;
   uint16_t* Bn = nullptr;
   uint16_t* Wkv = nullptr;
-  uint16_t* Uup = nullptr;     // recurrent adapter: U_l as [L*d][r_pad]
+  uint16_t* Uup = nullptr;     // recurrent adapter: U_l as [L*d][uup_ld] (split chain: [U_l | U_l])
+  int uup_ld = 0;              // r_pad, or 2 r_pad with the split chain
   float* bk = nullptr;
   float* bv = nullptr;
   float* kg = nullptr;         // per-head K-norm gain fp32 [L][head_dim] (k_norm)
@@ -351,15 +352,17 @@ __global__ void k_bias_to_f32(const uint16_t* __restrict__ b, float* __restrict_
     out[e] = bf(b[static_cast<long long>(pl.src[e / kv]) * kv + e % kv]);
 }
 
-// Uup[i*d + j][n] = U[src[i]][j][n] for n < r, else 0: the up-projection of the recurrent
-// adapter as a K-major B operand (rows = output channels j, K = bottleneck n).
+// Uup[i*d + j][n] = U[src[i]][j][n mod r_pad] for (n mod r_pad) < r, else 0: the up-projection
+// of the recurrent adapter as a K-major B operand (rows = output channels j, K = bottleneck n),
+// with ld = r_pad, or ld = 2 r_pad for the split chain (U twice: once for the low and once for
+// the high bf16 part of h).
 __global__ void k_pack_up(const uint16_t* __restrict__ U, uint16_t* __restrict__ Uup, int L, int r,
-                          int r_pad, int d, PackLayers pl) {
-  const long long total = static_cast<long long>(L) * d * r_pad;
+                          int r_pad, int d, int ld, PackLayers pl) {
+  const long long total = static_cast<long long>(L) * d * ld;
   for (long long e = blockIdx.x * static_cast<long long>(blockDim.x) + threadIdx.x; e < total;
        e += static_cast<long long>(gridDim.x) * blockDim.x) {
-    const int n = static_cast<int>(e % r_pad);
-    const long long row = e / r_pad;
+    const int n = static_cast<int>(e % ld) % r_pad;
+    const long long row = e / ld;
     const int j = static_cast<int>(row % d), i = static_cast<int>(row / d);
     Uup[e] = (n < r && !pl.zero_du[i]) ? U[(static_cast<long long>(pl.src[i]) * d + j) * r + n] : 0;
   }
@@ -577,6 +580,8 @@ int check_config(const dv_config* c) {
   if (c->has_kv_bias != 0 && c->has_kv_bias != 1) return DV_ERR_INVALID_ARG;
   if (c->adapter != DV_ADAPTER_EMBEDDING && c->adapter != DV_ADAPTER_RECURRENT)
     return DV_ERR_INVALID_ARG;
+  if (c->split_chain != 0 && c->split_chain != 1) return DV_ERR_INVALID_ARG;
+  if (c->split_chain && c->adapter != DV_ADAPTER_RECURRENT) return DV_ERR_INVALID_ARG;
   if (c->d % 64 != 0 || c->d > 16384) return DV_ERR_UNSUPPORTED_SHAPE;
   if (c->rank > 256) return DV_ERR_UNSUPPORTED_SHAPE;
   if (c->head_dim != 64 && c->head_dim != 128) return DV_ERR_UNSUPPORTED_SHAPE;
@@ -756,9 +761,10 @@ static cudaError_t enqueue_recurrent(const PlanView& v, const BuildArgs& a, cuda
   mark(1);
   const long long part_ld = static_cast<long long>(d / 64) * T;
   cudaError_t err = cudaSuccess;
-  // On chip: one cluster per 128-token block runs the whole chain with the state in TMEM.
+  // On chip: one cluster per 128-token block runs the whole chain with the state in TMEM (not
+  // with the split chain, whose low operand parts do not fit beside it).
   int spc = 0, S = 0;
-  if (chain_shape(d, v.r_pad, &spc, &S)) {
+  if (!v.split_chain && chain_shape(d, v.r_pad, &spc, &S)) {
     CUtensorMap tm_u, tm_m3;
     if (!encode_2d(&tm_u, v.Uup, v.r_pad, static_cast<uint64_t>(L) * d, v.r_pad, 64 * spc) ||
         !encode_3d(&tm_m3, a.mem, d, static_cast<uint64_t>(T), L, kBlockM))
@@ -778,6 +784,7 @@ static cudaError_t enqueue_recurrent(const PlanView& v, const BuildArgs& a, cuda
   const long long m_tiles = (T + kBlockM - 1) / kBlockM;
   const int splits = down_splits(m_tiles, d / kBlockK, v.num_sms);
   DownParams dp;
+  std::memset(&dp, 0, sizeof(dp));
   dp.M = static_cast<int>(T);
   dp.k_slabs = d / kBlockK;
   dp.H = a.H;
@@ -789,13 +796,21 @@ static cudaError_t enqueue_recurrent(const PlanView& v, const BuildArgs& a, cuda
   std::memset(&gp, 0, sizeof(gp));
   gp.status = v.status;
   gp.timeout_ns = kTimeoutNs;
-  // up-projection step: A = h_i (H columns from i * r_pad), B = U_i ([d][r_pad] rows i * d)
-  gp.s = {static_cast<int>(T), 1, d, 0, v.r_pad / 64, v.r_pad, 0, 0, 0, 0};
+  // up-projection step: A = h_i (H columns from i * r_pad), B = U_i ([d][r_pad] rows i * d).
+  // Split chain: A = [low part of h_i | h_i] (the low part as A0 through a per-layer map) and
+  // B = [U_i | U_i], so each product reads h_i in two bf16 parts.
+  const bool split = v.split_chain != 0;
+  const int kh = v.r_pad / 64;
+  gp.s = {static_cast<int>(T), 1, d, split ? kh : 0, kh, v.r_pad, 0, 0, 0, 0};
+  CUtensorMap tm_mem_lo = tm_x0;  // split chain: the low part of M_{i-1} (one [T][d] buffer)
+  if (split && !encode_2d(&tm_mem_lo, a.mem_lo, d, static_cast<uint64_t>(T), d, kBlockM))
+    return cudaErrorInvalidValue;
+  dp.Hlo = split ? a.Hlo : nullptr;
   // Large builds at r_pad 256 (one 256-token tile per CTA pair is enough to fill the pairs, so
   // no K split): the down-projection runs on CTA pairs, each SM staging half of D_l instead of
   // every CTA reading all of it from L2. Its maps start at the layer's rows: the previous
   // state (x0 for the first layer) and layer i's rows of the stacked D.
-  const bool down_pairs = v.r_pad == 256 && splits == 1;
+  const bool down_pairs = v.r_pad == 256 && splits == 1 && !split;
   GemmParams gd;
   std::memset(&gd, 0, sizeof(gd));
   gd.status = v.status;
@@ -817,14 +832,20 @@ static cudaError_t enqueue_recurrent(const PlanView& v, const BuildArgs& a, cuda
       dp.a_row0 = i == 0 ? 0 : static_cast<int>((i - 1) * T);
       dp.b_row0 = i * v.r_pad;
       dp.h_col0 = i * v.r_pad;
-      err = launch_down_split(v.r_pad, splits, i == 0 ? tm_x0 : tm_mem, *v.tm_Dst_rp, dp, st);
+      dp.a_lo = split && i > 0 ? 1 : 0;  // E (layer 0) is exact in bf16: no low part
+      err = launch_down_split(v.r_pad, splits, i == 0 ? tm_x0 : tm_mem, tm_mem_lo, *v.tm_Dst_rp,
+                              dp, st);
     }
     if (err != cudaSuccess) break;
     gp.s.layer0 = i;
     gp.resid = {static_cast<const uint16_t*>(a.x0), a.state,
                 a.mem + static_cast<size_t>(i) * T * d, a.part + static_cast<size_t>(i) * part_ld,
-                d, i == 0 ? 1 : 0};
-    err = launch_gemm(EPI_RESID, v.resid_bn, 0, tm_H, tm_H, *v.tm_Uup, gp, v.num_sms, st);
+                d, i == 0 ? 1 : 0, split ? a.mem_lo : nullptr};
+    CUtensorMap tm_a0 = tm_H;
+    if (split && !encode_2d(&tm_a0, a.Hlo + static_cast<size_t>(i) * v.r_pad, v.r_pad,
+                            static_cast<uint64_t>(T), n1, kBlockM))
+      return cudaErrorInvalidValue;
+    err = launch_gemm(EPI_RESID, v.resid_bn, 0, tm_a0, tm_H, *v.tm_Uup, gp, v.num_sms, st);
   }
   mark(2);
   if (err == cudaSuccess) {
@@ -962,7 +983,7 @@ size_t carve_workspace(const PlanView& v, long long T, void* base, BuildArgs* a)
   const size_t L = static_cast<size_t>(v.n_layers), t = static_cast<size_t>(T);
   const size_t d = static_cast<size_t>(v.d);
   const size_t oH = take(t * L * v.r_pad * 2), oR = take(L * t * 4), oX = take(t * 4);
-  size_t oS = 0, oM = 0, oP = 0, oC = 0;
+  size_t oS = 0, oM = 0, oP = 0, oC = 0, oHl = 0, oMl = 0;
   const bool rec = v.adapter == DV_ADAPTER_RECURRENT;
   const bool small_path = !rec && v.r_pad == 64;  // x0 (2 U_l)^T in fp32 (see enqueue_build)
   if (small_path) oC = take(t * L * v.r_pad * 4);
@@ -970,6 +991,10 @@ size_t carve_workspace(const PlanView& v, long long T, void* base, BuildArgs* a)
     oS = take(t * d * 4);
     oM = take(L * t * d * 2);
     oP = take(L * (d / 64) * t * 4);
+    if (v.split_chain) {  // low bf16 parts of h_l (every layer) and of the last M_l
+      oHl = take(t * L * v.r_pad * 2);
+      oMl = take(t * d * 2);
+    }
   }
   if (base && a) {
     unsigned char* b = static_cast<unsigned char*>(base);
@@ -980,6 +1005,9 @@ size_t carve_workspace(const PlanView& v, long long T, void* base, BuildArgs* a)
     a->mem = rec ? reinterpret_cast<uint16_t*>(b + oM) : nullptr;
     a->part = rec ? reinterpret_cast<float*>(b + oP) : nullptr;
     a->c = small_path ? reinterpret_cast<float*>(b + oC) : nullptr;
+    const bool split = rec && v.split_chain;
+    a->Hlo = split ? reinterpret_cast<uint16_t*>(b + oHl) : nullptr;
+    a->mem_lo = split ? reinterpret_cast<uint16_t*>(b + oMl) : nullptr;
   }
   return off;
 }
@@ -1015,6 +1043,7 @@ bool plan_view(const dv_plan* p, PlanView* v) {
   v->tm_Dst_rp = &p->tm_Dst_rp;
   v->tm_Uup = &p->tm_Uup;
   v->Uup = p->Uup;
+  v->split_chain = p->cfg.split_chain;
   v->Dst = p->Dst;
   v->dst_ld = c.d + 64;  // as the plan allocates Dst
   v->resid_bn = p->resid_bn;
@@ -1064,7 +1093,7 @@ cudaError_t preload_build_kernels(const dv_plan* p) {
     dv::DownParams dp;
     std::memset(&dp, 0, sizeof(dp));
     dp.k_slabs = 8;
-    for (int s : {1, 2, 4, 8}) keep(dv::launch_down_split(p->r_pad, s, m, m, dp, nullptr));
+    for (int s : {1, 2, 4, 8}) keep(dv::launch_down_split(p->r_pad, s, m, m, m, dp, nullptr));
     int spc = 0, S = 0;
     if (dv::chain_shape(p->cfg.d, p->r_pad, &spc, &S))
       keep(dv::launch_chain(p->r_pad, spc, S, 0, 1, p->cfg.d, m, m, m, m, nullptr, 0, nullptr,
@@ -1157,6 +1186,7 @@ int dv_memory_plan(const dv_config* cfg, const dv_weights* w, void* stream, dv_p
   p->bn_groups = (L + p->bn_lpt - 1) / p->bn_lpt;
   p->bn_k = d + p->bn_lpt * p->r_pad;
   p->resid_bn = d % 256 == 0 ? 256 : (d % 128 == 0 ? 128 : 64);
+  p->uup_ld = cfg->split_chain ? 2 * p->r_pad : p->r_pad;
   p->max_tokens = cfg->max_batch * cfg->max_n_vis;
   const long long T = p->max_tokens;
   cudaStream_t st = static_cast<cudaStream_t>(stream);
@@ -1176,7 +1206,7 @@ int dv_memory_plan(const dv_config* cfg, const dv_weights* w, void* stream, dv_p
   // 128-row TMA box over the L2 (the K/V weights' d + r_pad stride does the same).
   const int dst_ld = d + 64;
   bool ok = dmalloc(&p->Dst, sizeof(uint16_t) * dst_rows * dst_ld) &&
-            (rec ? dmalloc(&p->Uup, sizeof(uint16_t) * static_cast<size_t>(L) * d * p->r_pad)
+            (rec ? dmalloc(&p->Uup, sizeof(uint16_t) * static_cast<size_t>(L) * d * p->uup_ld)
                  : dmalloc(&p->Bn, sizeof(uint16_t) * p->bn_groups * 256 * p->bn_k)) &&
             dmalloc(&p->Wkv, sizeof(uint16_t) * static_cast<size_t>(L) * 2 * p->kv * p->k_total) &&
             dmalloc(&p->ws, ws_bytes) && dmalloc(&p->status, sizeof(int));
@@ -1207,7 +1237,8 @@ int dv_memory_plan(const dv_config* cfg, const dv_weights* w, void* stream, dv_p
   k_pack_kv<<<grid_for(1LL * L * 2 * p->kv * p->k_total), 256, 0, st>>>(Wk, Wv, G, p->Wkv, L, p->kv,
                                                                         HD, d, p->k_total, pl);
   if (rec) {
-    k_pack_up<<<grid_for(1LL * L * d * p->r_pad), 256, 0, st>>>(U, p->Uup, L, r, p->r_pad, d, pl);
+    k_pack_up<<<grid_for(1LL * L * d * p->uup_ld), 256, 0, st>>>(U, p->Uup, L, r, p->r_pad, d,
+                                                                 p->uup_ld, pl);
   } else {
     k_pack_2u<<<grid_for(1LL * L * p->r_pad * d), 256, 0, st>>>(
         U, p->Dst + static_cast<size_t>(L) * p->r_pad * dst_ld, L, r, p->r_pad, d, dst_ld, pl);
@@ -1247,7 +1278,7 @@ int dv_memory_plan(const dv_config* cfg, const dv_weights* w, void* stream, dv_p
              encode_slabs(&p->tm_Wkv, p->Wkv, p->k_total, 1ull * L * 2 * p->kv, p->k_total, 128);
   if (enc && rec) {
     enc = encode_2d(&p->tm_Dst_rp, p->Dst, d, 1ull * L * p->r_pad, dst_ld, p->r_pad) &&
-          encode_2d(&p->tm_Uup, p->Uup, p->r_pad, 1ull * L * d, p->r_pad, p->resid_bn);
+          encode_2d(&p->tm_Uup, p->Uup, p->uup_ld, 1ull * L * d, p->uup_ld, p->resid_bn);
   } else if (enc) {
     enc = encode_slabs(&p->tm_Bn_half, p->Bn, p->bn_k, 256ull * p->bn_groups, p->bn_k, 128) &&
           encode_2d(&p->tm_Bn, p->Bn, p->bn_k, 256ull * p->bn_groups, p->bn_k, 256);

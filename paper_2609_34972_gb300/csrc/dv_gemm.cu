@@ -126,9 +126,10 @@ __device__ __forceinline__ void warp_load_bf16(float* stage, float (&v)[32], con
 
 // One step of the recurrent adapter (Sec. 3.1 Eq. 6) for token row t and columns
 // [n*BN, (n+1)*BN): M = prev + h U^T with prev = x0 (first planned layer) or the fp32 state.
-// Writes the new fp32 state, bf16(M) for the K/V GEMM, and the sum of M^2 over the tile. The
-// state moves through the warp's staging a row segment per instruction (whole 128-byte lines),
-// not a 16-byte piece per lane and row.
+// Writes the new fp32 state, bf16(M) for the K/V GEMM (with the split chain also the bf16
+// rounding of M - bf16(M), the low part the next down-projection reads), and the sum of M^2 over
+// the tile. The state moves through the warp's staging a row segment per instruction (whole
+// 128-byte lines), not a 16-byte piece per lane and row.
 template <int BN>
 __device__ __forceinline__ void epi_resid(const GemmParams& p, uint32_t tbase, int n, int t,
                                           float* stage) {
@@ -177,6 +178,14 @@ __device__ __forceinline__ void epi_resid(const GemmParams& p, uint32_t tbase, i
       pk[u] = pack_bf16x2(__uint_as_float(vb[2 * u]), __uint_as_float(vb[2 * u + 1]));
     warp_store_f32(stage, vb, e.state + base + c * 32, e.d, rows);
     warp_store_bf16(stage, pk, e.mem + base + c * 32, e.d, rows);
+    if (e.mem_lo) {  // split chain: the remainder M - bf16(M), rounded to bf16
+      uint32_t lo[16];
+#pragma unroll
+      for (int u = 0; u < 16; ++u)
+        lo[u] = pack_bf16x2(__uint_as_float(vb[2 * u]) - __uint_as_float(pk[u] << 16),
+                            __uint_as_float(vb[2 * u + 1]) - __uint_as_float(pk[u] & 0xFFFF0000u));
+      warp_store_bf16(stage, lo, e.mem_lo + base + c * 32, e.d, rows);
+    }
   }
   if (t < p.s.M) e.part[static_cast<size_t>(n) * p.s.M + t] = ss;
 }

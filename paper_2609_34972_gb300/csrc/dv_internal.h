@@ -146,6 +146,7 @@ struct EpiResid {
   float* part;         // fp32 [d / BLOCK_N][M]: this layer's partial sums of squares
   int d;
   int first;           // 1: prev = x0
+  uint16_t* mem_lo;    // split chain: bf16(M - bf16(M)) [M][d], or null
 };
 
 struct GemmParams {
@@ -197,11 +198,13 @@ struct DownParams {
   uint16_t* H;
   int ldh;
   int h_col0;
+  int a_lo;      // split chain: 1 = the second A map holds the low bf16 part of A (rows a_row0..)
+  uint16_t* Hlo; // split chain: bf16(h - bf16(h)) at the same place as H, or null
   int* status;
   unsigned long long timeout_ns;
 };
-cudaError_t launch_down_split(int r_pad, int splits, const CUtensorMap& a, const CUtensorMap& b,
-                              const DownParams& p, cudaStream_t stream);
+cudaError_t launch_down_split(int r_pad, int splits, const CUtensorMap& a, const CUtensorMap& a_lo,
+                              const CUtensorMap& b, const DownParams& p, cudaStream_t stream);
 // K splits (1, 2, 4 or 8) for m_tiles token blocks of 128 rows and k_slabs slabs.
 int down_splits(long long m_tiles, int k_slabs, int num_sms);
 
@@ -248,7 +251,8 @@ struct PlanView {
   const uint16_t* Dst;             // stacked D (and 2 U^T): rows of dst_ld elements
   int dst_ld;
   const CUtensorMap* tm_Uup;       // recurrent: [L*d][r_pad], boxes of resid_bn rows
-  const uint16_t* Uup;             // recurrent: U_l as [L*d][r_pad]
+  const uint16_t* Uup;             // recurrent: U_l as [L*d][r_pad] ([U_l | U_l] when split)
+  int split_chain;                 // recurrent: hi + lo bf16 operands in the chain's GEMMs
   int resid_bn;                    // recurrent: column tile of the up-projection step
   const double* inv_freq;     // head_dim / 2 values
   const uint16_t* Wkv;        // repacked K/V weights [L*2kv][k_total]
@@ -283,6 +287,8 @@ struct BuildArgs {
   float* state;         // recurrent: fp32 [tokens][d]
   uint16_t* mem;        // recurrent: bf16 [L][tokens][d]
   float* part;          // recurrent: fp32 [L][d / 64][tokens]
+  uint16_t* Hlo;        // split chain: low bf16 parts of h, [tokens][L * r_pad]
+  uint16_t* mem_lo;     // split chain: low bf16 part of the last M_l, [tokens][d]
   cudaEvent_t* marks;   // 5 events around the 4 stages, or null
 };
 

@@ -13,6 +13,10 @@
 //     partials through distributed shared memory, in the fixed order 0..S-1 (the result does
 //     not depend on scheduling), applies SiLU and stores bf16 H;
 //   - a second cluster barrier keeps every CTA's shared memory alive until all reads are done.
+// With the split chain the K loop runs twice over the CTA's slabs, first with the high and then
+// with the low bf16 part of M_{l-1} (the second A map), against the same D_l slabs, and h is
+// stored as its bf16 rounding plus the bf16 rounding of the remainder (H and Hlo), so that the
+// up-projection can read it in two parts as well.
 // Every wait is bounded; a CTA that gives up still passes both cluster barriers, flags the
 // plan's status word and returns.
 #include "dv_internal.h"
@@ -65,6 +69,7 @@ __device__ __forceinline__ bool wait_bounded(uint32_t bar, uint32_t parity, uint
 template <int RP>
 __global__ void __launch_bounds__(kDownThreads, 1)
     dv_down_split_kernel(const __grid_constant__ CUtensorMap tmA,
+                         const __grid_constant__ CUtensorMap tmAlo,
                          const __grid_constant__ CUtensorMap tmB,
                          const __grid_constant__ DownParams p) {
   using C = DownCfg<RP>;
@@ -88,7 +93,8 @@ __global__ void __launch_bounds__(kDownThreads, 1)
   const int S = static_cast<int>(cluster_nctarank());
   const int m = static_cast<int>(cluster_id_x());
   const int ks0 = split * p.k_slabs / S;
-  const int n_slabs = (split + 1) * p.k_slabs / S - ks0;
+  const int n_own = (split + 1) * p.k_slabs / S - ks0;  // this CTA's K slabs of A (and of D_l)
+  const int n_slabs = p.a_lo ? 2 * n_own : n_own;       // split chain: high, then low parts
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < NS; ++s) {
@@ -112,6 +118,7 @@ __global__ void __launch_bounds__(kDownThreads, 1)
     if (lane == 0) {
       // ------------------------------------------------------ TMA producer and MMA issuer
       tma_prefetch_desc(&tmA);
+      if (p.a_lo) tma_prefetch_desc(&tmAlo);
       tma_prefetch_desc(&tmB);
       const uint32_t idesc = idesc_bf16_f32(kBlockM, RP);
       const int arow = p.a_row0 + m * kBlockM;
@@ -119,8 +126,13 @@ __global__ void __launch_bounds__(kDownThreads, 1)
         const int s = j % NS;
         const uint32_t a_dst = ring + s * C::kStageBytes;
         mbar_arrive_expect_tx(full_bar(s), C::kStageBytes);
-        tma_load_2d(a_dst, &tmA, full_bar(s), (ks0 + j) * kBlockK, arow);
-        tma_load_2d(a_dst + C::kABytes, &tmB, full_bar(s), (ks0 + j) * kBlockK, p.b_row0);
+        const int kk = ks0 + (j < n_own ? j : j - n_own);
+        if (j < n_own) {
+          tma_load_2d(a_dst, &tmA, full_bar(s), kk * kBlockK, arow);
+        } else {  // the low part of the state: one [M][d] buffer, token rows from 0
+          tma_load_2d(a_dst, &tmAlo, full_bar(s), kk * kBlockK, m * kBlockM);
+        }
+        tma_load_2d(a_dst + C::kABytes, &tmB, full_bar(s), kk * kBlockK, p.b_row0);
       };
       int loaded = 0, consumed = 0;
       for (; loaded < n_slabs && loaded < NS; ++loaded) load(loaded);
@@ -211,10 +223,18 @@ __global__ void __launch_bounds__(kDownThreads, 1)
           z.w += part[s].w;
         }
       }
+      const float h[4] = {silu(z.x), silu(z.y), silu(z.z), silu(z.w)};
       uint2 out;
-      out.x = pack_bf16x2(silu(z.x), silu(z.y));
-      out.y = pack_bf16x2(silu(z.z), silu(z.w));
-      *reinterpret_cast<uint2*>(p.H + static_cast<size_t>(t) * p.ldh + p.h_col0 + c4 * 4) = out;
+      out.x = pack_bf16x2(h[0], h[1]);
+      out.y = pack_bf16x2(h[2], h[3]);
+      const size_t o = static_cast<size_t>(t) * p.ldh + p.h_col0 + c4 * 4;
+      *reinterpret_cast<uint2*>(p.H + o) = out;
+      if (p.Hlo) {  // the remainder h - bf16(h), itself rounded to bf16
+        uint2 lo;
+        lo.x = pack_bf16x2(h[0] - __uint_as_float(out.x << 16), h[1] - __uint_as_float(out.x & 0xFFFF0000u));
+        lo.y = pack_bf16x2(h[2] - __uint_as_float(out.y << 16), h[3] - __uint_as_float(out.y & 0xFFFF0000u));
+        *reinterpret_cast<uint2*>(p.Hlo + o) = lo;
+      }
     }
   }
   __syncwarp();
@@ -228,8 +248,8 @@ __global__ void __launch_bounds__(kDownThreads, 1)
 }
 
 template <int RP>
-cudaError_t launch_t(int splits, const CUtensorMap& a, const CUtensorMap& b, const DownParams& p,
-                     cudaStream_t stream) {
+cudaError_t launch_t(int splits, const CUtensorMap& a, const CUtensorMap& a_lo, const CUtensorMap& b,
+                     const DownParams& p, cudaStream_t stream) {
   using C = DownCfg<RP>;
   auto kern = dv_down_split_kernel<RP>;
   cudaError_t err =
@@ -249,7 +269,7 @@ cudaError_t launch_t(int splits, const CUtensorMap& a, const CUtensorMap& b, con
   cfg.stream = stream;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
-  err = cudaLaunchKernelEx(&cfg, kern, a, b, p);
+  err = cudaLaunchKernelEx(&cfg, kern, a, a_lo, b, p);
   if (err != cudaSuccess) return err;
   return cudaGetLastError();
 }
@@ -273,15 +293,15 @@ int down_splits(long long m_tiles, int k_slabs, int num_sms) {
   return best;
 }
 
-cudaError_t launch_down_split(int r_pad, int splits, const CUtensorMap& a, const CUtensorMap& b,
-                              const DownParams& p, cudaStream_t stream) {
+cudaError_t launch_down_split(int r_pad, int splits, const CUtensorMap& a, const CUtensorMap& a_lo,
+                              const CUtensorMap& b, const DownParams& p, cudaStream_t stream) {
   if (splits != 1 && splits != 2 && splits != 4 && splits != 8) return cudaErrorInvalidValue;
   if (splits > p.k_slabs) return cudaErrorInvalidValue;
   switch (r_pad) {
-    case 64: return launch_t<64>(splits, a, b, p, stream);
-    case 128: return launch_t<128>(splits, a, b, p, stream);
-    case 192: return launch_t<192>(splits, a, b, p, stream);
-    case 256: return launch_t<256>(splits, a, b, p, stream);
+    case 64: return launch_t<64>(splits, a, a_lo, b, p, stream);
+    case 128: return launch_t<128>(splits, a, a_lo, b, p, stream);
+    case 192: return launch_t<192>(splits, a, a_lo, b, p, stream);
+    case 256: return launch_t<256>(splits, a, a_lo, b, p, stream);
     default: return cudaErrorInvalidValue;
   }
 }

@@ -132,6 +132,7 @@ class Config:
     k_norm: bool = False        # per-head RMSNorm of K before RoPE (Qwen3-VL backbones)
     k_norm_eps: float = 1e-6
     k_norm_sigma: float = 0.1   # per-head K-norm gain = 1 + N(0, k_norm_sigma)
+    split_chain: bool = False   # recurrent adapter: hi + lo bf16 operands in the chain's GEMMs
     description: str = ""
 
     @property

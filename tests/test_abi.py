@@ -64,7 +64,7 @@ def test_null_arguments_rejected(dv):
     ("n_layers", -1, 1), ("act", 3, 1), ("rope", 5, 1), ("max_batch", 0, 1),
     ("rope_theta", -1.0, 1), ("rms_eps", -1e-6, 1), ("n_kv_heads", 129, 2),
     ("adapter", 2, 1), ("adapter", -1, 1), ("rope", 3, 1), ("k_norm", 2, 1),
-    ("k_norm_eps", -1.0, 1),
+    ("k_norm_eps", -1.0, 1), ("split_chain", 2, 1), ("split_chain", 1, 1),
 ])
 def test_bad_config_rejected_before_device(dv, field, value, code):
     cfg = dv.make_config(512, 4, 8, 64, 16, max_batch=1, max_n_vis=64)
