@@ -343,13 +343,12 @@ def gpu_id_of(dev, local):
         return str(local)
 
 
-def measure_config(dv, name, args, dev, peaks, peak_src):
+def measure_config(dv, cfg, args, dev, peaks, peak_src):
     """Device-timed build of one more workload (inputs resident), for the per_config block."""
     import numpy as np
     import torch
     import synth
     from tests import gpu_util as gu
-    cfg = synth.CONFIGS[name]
     inp = synth.make_inputs(cfg)
     plan = dv.memory_plan(gu.dv_config(cfg), gu.device_weights(inp, dev))
     x0 = gu.torch_bf16(inp.x0, dev)
@@ -465,7 +464,7 @@ def run_dv(args):
     v_p = torch.empty(shape, dtype=torch.bfloat16).pin_memory()
     e2e_steps = max(5, min(args.steps, args.e2e_steps))
     pipe = dv.HostPipeline(plan, B, N, depth=2)
-    for _ in range(3):
+    for _ in range(max(3, args.warmup)):   # also the first touches of the host pages
         pipe.submit(x0_p, pos_p, k_p, v_p, stream=stream)
     pipe.join(stream)
     torch.cuda.synchronize()
@@ -498,10 +497,22 @@ def run_dv(args):
 
     cpu = None
     per_config = None
+    variants = None
     if rank == 0 and world == 1:
         if not args.no_per_config and args.config == DEFAULT_WORKLOAD and not args.layers \
                 and args.adapter == "embedding" and not args.skip_layers:
-            per_config = [measure_config(dv, n, args, dev, peaks, peak_src) for n in PER_CONFIG]
+            import synth
+            from dataclasses import replace
+            per_config = [measure_config(dv, synth.CONFIGS[n], args, dev, peaks, peak_src)
+                          for n in PER_CONFIG]
+            # the variants of the path beside the embedding adapter, on the LLaVA-1.5 shape:
+            # the recurrent adapter (Sec. 3.1 Eq. 6) and the consumer of the memory (Sec. 3.2)
+            rec = replace(synth.CONFIGS["llava15_7b"], adapter="recurrent",
+                          name="llava15_7b_recurrent",
+                          description=synth.CONFIGS["llava15_7b"].description +
+                          "; recurrent adapter (Sec. 3.1 Eq. 6)")
+            variants = [measure_config(dv, rec, args, dev, peaks, peak_src),
+                        measure_consumer(dv, synth.CONFIGS["llava15_7b"], args, peaks)]
         if not args.no_cpu_baseline:
             cpu = time_oracle_sample(inp, args.cpu_budget_s,
                                      min_tokens=min(cfg.tokens, 512) if cfg.batch > 1 else 0)
@@ -537,33 +548,26 @@ def run_dv(args):
             "stage_ms_per_step": stage,
             "cpu_baseline": cpu,
             "per_config": per_config,
+            "variants": variants,
         }
         print(json.dumps(out), flush=True)
     if dist is not None:
         dist.destroy_process_group()
 
 
-def run_consumer(args):
+def measure_consumer(dv, cfg, args, peaks):
     """The consumer of the visual memory (Sec. 3.2): one step = the causal attention of the
     prefill's text queries over every layer's cache (system-prompt text slots, the visual slots
     written by the build, the text slots), through dv_text_attention, one launch per layer."""
-    import numpy as np
     import torch
     import synth
-    from paper_2609_34972_gb300.build import build_library
-    build_library()
-    import paper_2609_34972_gb300 as dv
     from tests import gpu_util as gu
-    rank, world, local = dist_env()
-    if rank != 0:
-        return
-    torch.cuda.set_device(local)
-    cfg = workload_config(args)
     n_sys, n_text, hq = args.consumer_sys, args.consumer_text, cfg.n_heads
     B, Nv, H, D, L = cfg.batch, cfg.n_vis, cfg.n_kv_heads, cfg.head_dim, cfg.n_layers
     S = n_sys + Nv + n_text
     inp = synth.make_inputs(cfg)
     k, v, plan = gu.run_build(inp, seq_len=S, slot0=n_sys)
+    dv.free(plan)
     gen = torch.Generator(device="cuda").manual_seed(7)
     for l in range(L):
         k[l, :, :n_sys].normal_(generator=gen)
@@ -610,9 +614,10 @@ def run_consumer(args):
     kv_bytes = L * B * H * S * D * 2 * 2
     qo_bytes = L * B * hq * n_text * D * 2 * 2
     flops = sum(4.0 * B * hq * D * (n_sys + Nv + t + 1) for t in range(n_text)) * L
-    peaks, _ = load_peaks()
     gbs = (kv_bytes + qo_bytes) / (ms * 1e-3) / 1e9
-    print(json.dumps({
+    del graph, k, v
+    torch.cuda.empty_cache()
+    return {
         "metric": "text-query attention over the visual memory: text tokens/s (all layers)",
         "value": B * n_text / (ms * 1e-3), "unit": "text tokens/s", "n_gpus": 1,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
@@ -628,7 +633,21 @@ def run_consumer(args):
                      "kernel": "dv_attn_kernel", "bytes_per_step": kv_bytes + qo_bytes,
                      "tflops": flops / (ms * 1e-3) / 1e12},
         "clocks": clocks, "gpu_launches": args.steps * L,
-    }), flush=True)
+    }
+
+
+def run_consumer(args):
+    """``--consumer``: the consumer's own JSON line (see measure_consumer)."""
+    import torch
+    from paper_2609_34972_gb300.build import build_library
+    build_library()
+    import paper_2609_34972_gb300 as dv
+    rank, world, local = dist_env()
+    if rank != 0:
+        return
+    torch.cuda.set_device(local)
+    peaks, _ = load_peaks()
+    print(json.dumps(measure_consumer(dv, workload_config(args), args, peaks)), flush=True)
 
 
 def main():
