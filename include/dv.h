@@ -186,13 +186,16 @@ int dv_build_visual_memory(dv_plan* plan, const void* x0, int batch, int n_vis, 
  *     and the row sums of squares) go to one static device array of 32 MiB that every device
  *     loading this library holds until the process exits. The plan's own workspace is not
  *     used, so its max_batch / max_n_vis do not bound this call.
- *   - Limit: batch * n_vis * (n_layers * r_pad * 2 + n_layers * 4 + 4) bytes (each part
- *     rounded up to 256 bytes, r_pad = rank rounded up to 64, n_layers counting the planned
- *     layers) must fit in 32 MiB. The embedding adapter with r_pad = 64 adds batch * n_vis *
- *     n_layers * r_pad * 4 (the fp32 x0 (2 U_l)^T of the small-token path). The recurrent
- *     adapter adds batch * n_vis * (4 d + n_layers * (2 d + 4 d / 64)) bytes (fp32 state, bf16
- *     M_l of every layer, partial sums of squares). Larger builds return
- *     DV_ERR_UNSUPPORTED_SHAPE and launch nothing.
+ *   - Limit: with T = batch * n_vis, r_pad = rank rounded up to 64 and L the planned layers,
+ *     the intermediates (each part rounded up to 256 bytes) must fit in 32 MiB:
+ *       embedding adapter  T * ((L * r_pad + 64) * 2 + L * 4 + 4 + (d + 64) * 2) bytes (h of
+ *                          every layer, RMS statistics, row sums, a copy of E), plus
+ *                          T * L * r_pad * 4 when r_pad = 64 (the fp32 x0 (2 U_l)^T of the
+ *                          small-token path);
+ *       recurrent adapter  T * (L * r_pad * 2 + L * 4 + 4 + 4 d + L * (2 d + 4 d / 64)) bytes
+ *                          (h, RMS statistics, fp32 state, bf16 M_l of every layer, partial
+ *                          sums of squares), plus T * (L * r_pad + d) * 2 with split_chain.
+ *     Larger builds return DV_ERR_UNSUPPORTED_SHAPE and launch nothing.
  *   - dv_memory_plan reserves the array on the plan's device (CUDA loads the module that
  *     holds it when the plan looks up its address) and loads every kernel a build can launch,
  *     so this entry point allocates nothing, even on its first call.

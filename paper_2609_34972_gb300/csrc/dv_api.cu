@@ -493,24 +493,30 @@ __global__ void __launch_bounds__(64) k_rstd_hc(const uint16_t* __restrict__ H, 
   }
 }
 
-// xx[t] = sum_j x0[t][j]^2 (fp32), one warp per token row, 16-byte loads.
+// xx[t] = sum_j x0[t][j]^2 (fp32), one warp per token row, 16-byte loads; the row also goes to
+// x0p[t] (row pitch ldp elements), the copy of E that the RMS statistic and the K/V GEMM read:
+// a pitch of d + 64 elements is not a power of two, which spreads a TMA box's rows over the L2
+// (the caller's E has pitch d, a power of two on the 7B shapes).
 // Launched right after the down-projection and run beside it, on the SMs that its tiles leave
-// free. Its reads of x0 and writes of xx come before its dependency wait. That is safe: a
-// dependent grid starts only once every CTA of the grid before it has triggered, and the
+// free. Its reads of x0 and its writes of xx and x0p come before its dependency wait. That is
+// safe: a dependent grid starts only once every CTA of the grid before it has triggered, and the
 // down-projection triggers after its own wait, so every earlier writer of x0 and every earlier
-// reader of xx (the previous build's statistic) has finished. The wait comes last, so that this
-// grid completes only after the down-projection has, and the kernel after it, which waits on
-// this grid alone, still sees H.
-__global__ void k_row_sumsq(const uint16_t* __restrict__ x0, int T, int d, float* __restrict__ xx) {
+// reader of xx and x0p (the previous build's statistic and K/V GEMM) has finished. The wait comes
+// last, so that this grid completes only after the down-projection has, and the kernel after it,
+// which waits on this grid alone, still sees H.
+__global__ void k_row_sumsq(const uint16_t* __restrict__ x0, int T, int d, float* __restrict__ xx,
+                            uint16_t* __restrict__ x0p, long long ldp) {
   dv::pdl_trigger();
   const int warp = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
   const int lane = threadIdx.x & 31;
   if (warp < T) {
     const uint4* row = reinterpret_cast<const uint4*>(x0 + static_cast<long long>(warp) * d);
+    uint4* prow = x0p ? reinterpret_cast<uint4*>(x0p + static_cast<long long>(warp) * ldp) : nullptr;
     float s = 0.0f;
 #pragma unroll 8
     for (int c = lane; c < d / 8; c += 32) {
       const uint4 v = row[c];
+      if (prow) prow[c] = v;
       const uint32_t w[4] = {v.x, v.y, v.z, v.w};
 #pragma unroll
       for (int e = 0; e < 4; ++e) {
@@ -703,9 +709,9 @@ static void fill_epi_kv(const PlanView& v, const BuildArgs& a, long long T, EpiK
 // operands are slab maps: a_full / h_full with 128-row boxes, a_half / h_half (made here) with
 // nt / 2-row boxes.
 static cudaError_t launch_kv_stage(const PlanView& v, GemmParams& gp, long long T,
-                                   const void* a_ptr, uint64_t a_rows, const CUtensorMap& a_full,
-                                   const void* h_ptr, uint64_t h_cols, const CUtensorMap& h_full,
-                                   cudaStream_t st) {
+                                   const void* a_ptr, uint64_t a_rows, uint64_t a_ld,
+                                   const CUtensorMap& a_full, const void* h_ptr, uint64_t h_cols,
+                                   uint64_t h_ld, const CUtensorMap& h_full, cudaStream_t st) {
   const int nt = kv_pair_tile_n(T);
   const long long pad256 = (T + 255) / 256 * 256, pad_nt = (T + nt - 1) / nt * nt;
   if (prefer_256(pad256, pad_nt)) {
@@ -713,8 +719,8 @@ static cudaError_t launch_kv_stage(const PlanView& v, GemmParams& gp, long long 
     return launch_pair_tm(EPI_KV, 256, v.head_dim, a_full, h_full, *v.tm_Wkv, gp, v.num_sms, st);
   }
   CUtensorMap a_half, h_half;
-  if (!encode_slabs(&a_half, a_ptr, v.d, a_rows, v.d, nt / 2)) return cudaErrorInvalidValue;
-  if (h_ptr && !encode_slabs(&h_half, h_ptr, h_cols, static_cast<uint64_t>(T), h_cols, nt / 2))
+  if (!encode_slabs(&a_half, a_ptr, v.d, a_rows, a_ld, nt / 2)) return cudaErrorInvalidValue;
+  if (h_ptr && !encode_slabs(&h_half, h_ptr, h_cols, static_cast<uint64_t>(T), h_ld, nt / 2))
     return cudaErrorInvalidValue;
   return launch_kv_pair(v.head_dim, nt, *v.tm_Wkv, a_half, h_ptr ? h_half : a_half, gp, v.num_sms,
                         st);
@@ -733,8 +739,9 @@ static cudaError_t launch_recurrent_kv(const PlanView& v, const BuildArgs& a, lo
   for (int i = 0; i < L; ++i) gp.layer_map[i] = v.active[i];
   gp.s = {static_cast<int>(T), L, 2 * v.kv, d / 64, 0, 0, 0, 0, 0, static_cast<int>(T)};
   fill_epi_kv(v, a, T, gp.kv);
-  const cudaError_t err = launch_kv_stage(v, gp, T, a.mem, static_cast<uint64_t>(L) * T, tm_mem_s,
-                                          nullptr, 0, tm_mem_s, st);
+  const cudaError_t err = launch_kv_stage(v, gp, T, a.mem, static_cast<uint64_t>(L) * T,
+                                          static_cast<uint64_t>(d), tm_mem_s, nullptr, 0, 0,
+                                          tm_mem_s, st);
   mark(4);
   return err;
 }
@@ -867,12 +874,17 @@ cudaError_t enqueue_build(const PlanView& v, const BuildArgs& a, cudaStream_t st
   const long long pad128 = (T + 127) / 128 * 128, pad256 = (T + 255) / 256 * 256;
   const bool rank_pairs = prefer_256(pad256, pad128);
 
-  // 2-D maps for the 1-SM kernel, slab maps (two K slabs per box) for the CTA-pair kernels
-  CUtensorMap tm_x0, tm_H, tm_x0_s, tm_H_s;
+  // 2-D maps for the 1-SM kernel, slab maps (two K slabs per box) for the CTA-pair kernels. The
+  // down-projection reads the caller's E; the statistic and the K/V GEMM read the row sums'
+  // copy of it (x0p, pitch d + 64), and H has pitch hld = L r_pad + 64 (see k_row_sumsq).
+  const long long hld = a.hld, xld = a.x0p_ld;
+  CUtensorMap tm_x0, tm_H, tm_x0_s, tm_H_s, tm_xp, tm_xp_s;
   if (!encode_2d(&tm_x0, a.x0, d, static_cast<uint64_t>(T), d, kBlockM) ||
-      !encode_2d(&tm_H, a.H, n1, static_cast<uint64_t>(T), n1, kBlockM) ||
+      !encode_2d(&tm_H, a.H, n1, static_cast<uint64_t>(T), hld, kBlockM) ||
       !encode_slabs(&tm_x0_s, a.x0, d, static_cast<uint64_t>(T), d, kBlockM) ||
-      !encode_slabs(&tm_H_s, a.H, n1, static_cast<uint64_t>(T), n1, kBlockM))
+      !encode_slabs(&tm_H_s, a.H, n1, static_cast<uint64_t>(T), hld, kBlockM) ||
+      !encode_2d(&tm_xp, a.x0p, d, static_cast<uint64_t>(T), xld, kBlockM) ||
+      !encode_slabs(&tm_xp_s, a.x0p, d, static_cast<uint64_t>(T), xld, kBlockM))
     return cudaErrorInvalidValue;
 
   GemmParams gp;
@@ -884,14 +896,14 @@ cudaError_t enqueue_build(const PlanView& v, const BuildArgs& a, cudaStream_t st
   // xx = row sums of squares of x0, launched after the down-projection (see k_row_sumsq).
   auto row_sumsq = [&]() {
     return launch_pdl(k_row_sumsq, dim3(static_cast<unsigned>((T + 7) / 8)), dim3(256), st,
-                      static_cast<const uint16_t*>(a.x0), static_cast<int>(T), d, a.xx);
+                      static_cast<const uint16_t*>(a.x0), static_cast<int>(T), d, a.xx, a.x0p, xld);
   };
   mark(0);
   cudaError_t err = cudaSuccess;
 
   // (1) H = SiLU(x0 [D_1 ... D_L]) — one GEMM over all layers' down-projections.
   gp.s = {static_cast<int>(T), 1, static_cast<int>(n1), d / 64, 0, 0, 0, 0, 0, 0};
-  gp.silu = {a.H, static_cast<int>(n1), static_cast<int>(n1), nullptr, 0};
+  gp.silu = {a.H, static_cast<int>(hld), static_cast<int>(n1), nullptr, 0};
   if (!rank_pairs && a.c) {
     // Small or awkward token counts: x0 [D_1 .. D_L | 2U_1 .. 2U_L]^T as one GEMM (the
     // down-projections get SiLU, the second half is c_l = x0 (2 U_l)^T in fp32), then the
@@ -904,7 +916,7 @@ cudaError_t enqueue_build(const PlanView& v, const BuildArgs& a, cudaStream_t st
     // a tile is either all down-projection columns or all c columns: bn divides n1
     const int bn = n1 % 256 == 0 ? 256 : (n1 % 128 == 0 ? 128 : 64);
     gp.s = {static_cast<int>(T), 1, static_cast<int>(n2), d / 64, 0, 0, 0, 0, 0, 0};
-    gp.silu = {a.H, static_cast<int>(n1), static_cast<int>(n1), a.c, static_cast<int>(n1)};
+    gp.silu = {a.H, static_cast<int>(hld), static_cast<int>(n1), a.c, static_cast<int>(n1)};
     tm_groups(gp.s, bn, T);
     const CUtensorMap& tmD = v.tm_Dst_half[bn == 64 ? 0 : (bn == 128 ? 1 : 2)];
     if (err == cudaSuccess) err = launch_pair_tm(EPI_SILU, bn, 0, tm_x0_s, tm_x0_s, tmD, gp, v.num_sms, st);
@@ -914,7 +926,7 @@ cudaError_t enqueue_build(const PlanView& v, const BuildArgs& a, cudaStream_t st
     if (err == cudaSuccess) {
       dim3 grid(static_cast<unsigned>((T + 63) / 64), static_cast<unsigned>(L));
       err = launch_pdl(k_rstd_hc<64>, grid, dim3(64), st, static_cast<const uint16_t*>(a.H),
-                       static_cast<int>(n1), static_cast<const float*>(a.c), static_cast<int>(n1),
+                       static_cast<int>(hld), static_cast<const float*>(a.c), static_cast<int>(n1),
                        static_cast<const float*>(a.xx), v.Gf, static_cast<int>(T), 1.0f / d,
                        v.rms_eps, a.rstd);
     }
@@ -954,11 +966,11 @@ cudaError_t enqueue_build(const PlanView& v, const BuildArgs& a, cudaStream_t st
   const int lpt = v.bn_lpt;
   gp.s = {static_cast<int>(T), v.bn_groups, 256, d / 64, lpt * v.r_pad / 64, lpt * v.r_pad, 0, 0, 0, 0};
   if (rank_pairs) tm_groups(gp.s, 256, T);
-  gp.norm = {a.H, static_cast<int>(n1), v.r_pad, lpt, v.bn_rn, L, a.xx, a.rstd,
+  gp.norm = {a.H, static_cast<int>(hld), v.r_pad, lpt, v.bn_rn, L, a.xx, a.rstd,
              static_cast<int>(T), 1.0f / d, v.rms_eps};
   if (err == cudaSuccess) {
-    err = rank_pairs ? launch_pair_tm(EPI_NORM, 256, 0, tm_x0_s, tm_H_s, *v.tm_Bn_half, gp, v.num_sms, st)
-                     : launch_gemm(EPI_NORM, 256, 0, tm_x0, tm_H, *v.tm_Bn, gp, v.num_sms, st);
+    err = rank_pairs ? launch_pair_tm(EPI_NORM, 256, 0, tm_xp_s, tm_H_s, *v.tm_Bn_half, gp, v.num_sms, st)
+                     : launch_gemm(EPI_NORM, 256, 0, tm_xp, tm_H, *v.tm_Bn, gp, v.num_sms, st);
   }
   mark(3);
   }
@@ -967,8 +979,9 @@ cudaError_t enqueue_build(const PlanView& v, const BuildArgs& a, cudaStream_t st
   gp.s = {static_cast<int>(T), L, 2 * v.kv, d / 64, v.r_pad / 64, v.r_pad, 0, 0, 0, 0};
   fill_epi_kv(v, a, T, gp.kv);
   if (err == cudaSuccess)
-    err = launch_kv_stage(v, gp, T, a.x0, static_cast<uint64_t>(T), tm_x0_s, a.H,
-                          static_cast<uint64_t>(n1), tm_H_s, st);
+    err = launch_kv_stage(v, gp, T, a.x0p, static_cast<uint64_t>(T), static_cast<uint64_t>(xld),
+                          tm_xp_s, a.H, static_cast<uint64_t>(n1), static_cast<uint64_t>(hld),
+                          tm_H_s, st);
   mark(4);
   return err;
 }
@@ -982,9 +995,13 @@ size_t carve_workspace(const PlanView& v, long long T, void* base, BuildArgs* a)
   };
   const size_t L = static_cast<size_t>(v.n_layers), t = static_cast<size_t>(T);
   const size_t d = static_cast<size_t>(v.d);
-  const size_t oH = take(t * L * v.r_pad * 2), oR = take(L * t * 4), oX = take(t * 4);
-  size_t oS = 0, oM = 0, oP = 0, oC = 0, oHl = 0, oMl = 0;
   const bool rec = v.adapter == DV_ADAPTER_RECURRENT;
+  // Embedding adapter: H rows and the copy of E get a pitch 64 elements (128 bytes) past their
+  // width, so that no row pitch is a power of two (see k_row_sumsq).
+  const size_t hld = L * v.r_pad + (rec ? 0 : 64), xld = d + 64;
+  const size_t oH = take(t * hld * 2), oR = take(L * t * 4), oX = take(t * 4);
+  const size_t oXp = rec ? 0 : take(t * xld * 2);
+  size_t oS = 0, oM = 0, oP = 0, oC = 0, oHl = 0, oMl = 0;
   const bool small_path = !rec && v.r_pad == 64;  // x0 (2 U_l)^T in fp32 (see enqueue_build)
   if (small_path) oC = take(t * L * v.r_pad * 4);
   if (rec) {
@@ -999,6 +1016,9 @@ size_t carve_workspace(const PlanView& v, long long T, void* base, BuildArgs* a)
   if (base && a) {
     unsigned char* b = static_cast<unsigned char*>(base);
     a->H = reinterpret_cast<uint16_t*>(b + oH);
+    a->hld = static_cast<long long>(hld);
+    a->x0p = rec ? nullptr : reinterpret_cast<uint16_t*>(b + oXp);
+    a->x0p_ld = static_cast<long long>(xld);
     a->rstd = reinterpret_cast<float*>(b + oR);
     a->xx = reinterpret_cast<float*>(b + oX);
     a->state = rec ? reinterpret_cast<float*>(b + oS) : nullptr;
@@ -1417,7 +1437,9 @@ int dv_debug_copy_workspace(dv_plan* p, int tokens, void* H, void* rstd, void* x
   const size_t hrow = static_cast<size_t>(L) * p->r_pad;
   const size_t T = static_cast<size_t>(p->last_tokens);
   cudaError_t err = cudaSuccess;
-  if (H) err = cudaMemcpyAsync(H, a.H, sizeof(uint16_t) * hrow * tokens, cudaMemcpyDeviceToDevice, st);
+  if (H)
+    err = cudaMemcpy2DAsync(H, sizeof(uint16_t) * hrow, a.H, sizeof(uint16_t) * a.hld,
+                            sizeof(uint16_t) * hrow, tokens, cudaMemcpyDeviceToDevice, st);
   if (rstd && err == cudaSuccess)
     err = cudaMemcpy2DAsync(rstd, sizeof(float) * tokens, a.rstd, sizeof(float) * T,
                             sizeof(float) * tokens, L, cudaMemcpyDeviceToDevice, st);

@@ -280,7 +280,10 @@ struct BuildArgs {
   const void* kc;
   const void* vc;
   long long s_layer, s_batch, s_seq, s_head;
-  uint16_t* H;          // [tokens][L * r_pad] bf16
+  uint16_t* H;          // [tokens][hld] bf16, h_l at columns l * r_pad
+  long long hld;        // row pitch of H: L * r_pad (+ 64 for the embedding adapter)
+  uint16_t* x0p;        // embedding adapter: copy of E with row pitch x0p_ld (k_row_sumsq)
+  long long x0p_ld;     // d + 64
   float* rstd;          // [L][tokens]
   float* xx;            // [tokens]
   float* c;             // embedding adapter, small token counts: fp32 [tokens][L * r_pad]

@@ -68,9 +68,10 @@ def test_noalloc_matches_build_on_two_calls(dv, name):
 
 def test_noalloc_rejects_builds_over_its_limit(dv):
     import torch
-    # Qwen-image shape, 28 layers, rank 128: 28 * 128 * 2 + 28 * 4 + 4 = 7284 bytes of
-    # intermediates per token, so its 4 x 1296 = 5184-token batch (37.8 MB) is over the 32 MiB
-    # limit while one image (1296 tokens, 9.4 MB) fits. The plan's own workspace holds 1 token.
+    # Qwen-image shape, 28 layers, rank 128, d = 3584: (28 * 128 + 64) * 2 + 28 * 4 + 4 +
+    # (3584 + 64) * 2 = 14708 bytes of intermediates per token, so its 4 x 1296 = 5184-token
+    # batch (72.7 MiB) is over the 32 MiB limit while one image (1296 tokens, 18.2 MiB) fits.
+    # The plan's own workspace holds 1 token.
     cfg = synth.CONFIGS["qwen25vl_7b_image"]
     inp = synth.make_inputs(cfg)
     plan = dv.memory_plan(gu.dv_config(cfg, max_batch=1, max_n_vis=1), gu.device_weights(inp))
