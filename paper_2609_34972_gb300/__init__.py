@@ -429,6 +429,8 @@ class HostPipeline:
         _check_tensor("v", v, torch.bfloat16, cpu, shape)
 
     def submit(self, x0, pos, k, v, stream=None) -> int:
+        if not self.plan.alive or not (self.handle and self.handle.value):
+            raise ValueError("the pipeline or its plan has been freed")
         self._check_host(x0, pos, k, v)
         t = ctypes.c_longlong()
         _check(lib().dv_build_visual_memory_host(self.handle, _ptr(x0), _ptr(pos), _ptr(k), _ptr(v),
