@@ -505,13 +505,17 @@ def run_dv(args):
             from dataclasses import replace
             per_config = [measure_config(dv, synth.CONFIGS[n], args, dev, peaks, peak_src)
                           for n in PER_CONFIG]
-            # the variants of the path beside the embedding adapter, on the LLaVA-1.5 shape:
-            # the recurrent adapter (Sec. 3.1 Eq. 6) and the consumer of the memory (Sec. 3.2)
+            # the variants of the path beside the embedding adapter: on the LLaVA-1.5 shape the
+            # recurrent adapter (Sec. 3.1 Eq. 6) and the consumer of the memory (Sec. 3.2)
             rec = replace(synth.CONFIGS["llava15_7b"], adapter="recurrent",
                           name="llava15_7b_recurrent",
                           description=synth.CONFIGS["llava15_7b"].description +
                           "; recurrent adapter (Sec. 3.1 Eq. 6)")
+            # and the Qwen3-VL-4B-shaped build (the paper's default backbone: per-head K norm,
+            # interleaved M-RoPE)
             variants = [measure_config(dv, rec, args, dev, peaks, peak_src),
+                        measure_config(dv, synth.CONFIGS["qwen3vl_4b_image"], args, dev, peaks,
+                                       peak_src),
                         measure_consumer(dv, synth.CONFIGS["llava15_7b"], args, peaks)]
         if not args.no_cpu_baseline:
             cpu = time_oracle_sample(inp, args.cpu_budget_s,
