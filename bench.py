@@ -343,14 +343,23 @@ def gpu_id_of(dev, local):
         return str(local)
 
 
-def measure_config(dv, cfg, args, dev, peaks, peak_src):
-    """Device-timed build of one more workload (inputs resident), for the per_config block."""
+def measure_config(dv, cfg, args, dev, peaks, peak_src, skip=None):
+    """Device-timed build of one more workload (inputs resident), for the per_config and
+    variants blocks. ``skip`` = (F, K): no visual memory at the first F and last K layers (App. J
+    adapter skipping, DV_LAYER_DROP); the algorithmic work then counts the built layers."""
     import numpy as np
     import torch
     import synth
+    from dataclasses import replace
     from tests import gpu_util as gu
     inp = synth.make_inputs(cfg)
-    plan = dv.memory_plan(gu.dv_config(cfg), gu.device_weights(inp, dev))
+    modes, work = None, cfg
+    if skip:
+        f, k = skip
+        modes = [dv.DV_LAYER_DROP if (l < f or l >= cfg.n_layers - k) else dv.DV_LAYER_ADAPTER
+                 for l in range(cfg.n_layers)]
+        work = replace(cfg, n_layers=cfg.n_layers - f - k, name=f"{cfg.name}_skip{f}_{k}")
+    plan = dv.memory_plan(gu.dv_config(cfg), gu.device_weights(inp, dev), layer_modes=modes)
     x0 = gu.torch_bf16(inp.x0, dev)
     pos = torch.from_numpy(np.ascontiguousarray(inp.pos)).to(dev)
     shape = (cfg.n_layers, cfg.batch, cfg.n_vis, cfg.n_kv_heads, cfg.head_dim)
@@ -361,9 +370,11 @@ def measure_config(dv, cfg, args, dev, peaks, peak_src):
     ms_total, clk, stage_ms, n_timed = time_builds(dv, plan, build, args.steps, args.warmup, stream,
                                                    clocks=ClockSampler(gpu_id_of(dev, 0)))
     ms_step = ms_total / args.steps
-    roof, step = roofline_of(dv, plan, cfg, stage_ms, n_timed, ms_total, ms_step, peaks, peak_src,
+    roof, step = roofline_of(dv, plan, work, stage_ms, n_timed, ms_total, ms_step, peaks, peak_src,
                              cfg.tokens)
-    out = {"workload": cfg.name, "description": cfg.description, "tokens_per_step": cfg.tokens,
+    out = {"workload": work.name, "description": cfg.description +
+           (f"; no visual memory at the first {skip[0]} and last {skip[1]} layers (App. J)" if skip else ""),
+           "layers_with_visual_memory": work.n_layers, "tokens_per_step": cfg.tokens,
            "value": cfg.tokens * args.steps / (ms_total / 1000.0), "unit": UNIT,
            "ms_per_step": ms_step, "steps": args.steps, "clocks": clk, "roofline": roof,
            "roofline_step": step,
@@ -513,9 +524,11 @@ def run_dv(args):
                           "; recurrent adapter (Sec. 3.1 Eq. 6)")
             # and the Qwen3-VL-4B-shaped build (the paper's default backbone: per-head K norm,
             # interleaved M-RoPE)
+            # with the App. J skipping of its first 5 and last 10 adapters
+            q3 = synth.CONFIGS["qwen3vl_4b_image"]
             variants = [measure_config(dv, rec, args, dev, peaks, peak_src),
-                        measure_config(dv, synth.CONFIGS["qwen3vl_4b_image"], args, dev, peaks,
-                                       peak_src),
+                        measure_config(dv, q3, args, dev, peaks, peak_src),
+                        measure_config(dv, q3, args, dev, peaks, peak_src, skip=(5, 10)),
                         measure_consumer(dv, synth.CONFIGS["llava15_7b"], args, peaks)]
         if not args.no_cpu_baseline:
             cpu = time_oracle_sample(inp, args.cpu_budget_s,
