@@ -768,16 +768,17 @@ static cudaError_t enqueue_recurrent(const PlanView& v, const BuildArgs& a, cuda
   mark(1);
   const long long part_ld = static_cast<long long>(d / 64) * T;
   cudaError_t err = cudaSuccess;
-  // On chip: one cluster per 128-token block runs the whole chain with the state in TMEM (not
-  // with the split chain, whose low operand parts do not fit beside it).
+  // On chip: one cluster per 128-token block runs the whole chain with the state in TMEM. With
+  // the split chain only at r_pad 64: at larger r_pad its low operand parts do not fit beside it.
   int spc = 0, S = 0;
-  if (!v.split_chain && chain_shape(d, v.r_pad, &spc, &S)) {
+  if ((!v.split_chain || v.r_pad == 64) && chain_shape(d, v.r_pad, &spc, &S)) {
     CUtensorMap tm_u, tm_m3;
-    if (!encode_2d(&tm_u, v.Uup, v.r_pad, static_cast<uint64_t>(L) * d, v.r_pad, 64 * spc) ||
+    // U_l as [L d][r_pad] (its first copy when the split chain packs [U_l | U_l])
+    if (!encode_2d(&tm_u, v.Uup, v.r_pad, static_cast<uint64_t>(L) * d, v.uup_ld, 64 * spc) ||
         !encode_3d(&tm_m3, a.mem, d, static_cast<uint64_t>(T), L, kBlockM))
       return cudaErrorInvalidValue;
     err = launch_chain(v.r_pad, spc, S, T, L, d, tm_x0, *v.tm_Dst_rp, tm_u, tm_m3, a.part, part_ld,
-                       a.H, v.status, kTimeoutNs, st);
+                       a.H, v.status, kTimeoutNs, st, v.split_chain != 0);
     if (err == cudaSuccess) {
       mark(2);
       err = launch_pdl(k_rstd_parts, dim3(grid_for(static_cast<long long>(L) * T)), dim3(256), st,
@@ -1063,6 +1064,7 @@ bool plan_view(const dv_plan* p, PlanView* v) {
   v->tm_Dst_rp = &p->tm_Dst_rp;
   v->tm_Uup = &p->tm_Uup;
   v->Uup = p->Uup;
+  v->uup_ld = p->uup_ld;
   v->split_chain = p->cfg.split_chain;
   v->Dst = p->Dst;
   v->dst_ld = c.d + 64;  // as the plan allocates Dst
@@ -1115,9 +1117,9 @@ cudaError_t preload_build_kernels(const dv_plan* p) {
     dp.k_slabs = 8;
     for (int s : {1, 2, 4, 8}) keep(dv::launch_down_split(p->r_pad, s, m, m, m, dp, nullptr));
     int spc = 0, S = 0;
-    if (dv::chain_shape(p->cfg.d, p->r_pad, &spc, &S))
+    if (dv::chain_shape(p->cfg.d, p->r_pad, &spc, &S) && (!p->cfg.split_chain || p->r_pad == 64))
       keep(dv::launch_chain(p->r_pad, spc, S, 0, 1, p->cfg.d, m, m, m, m, nullptr, 0, nullptr,
-                            nullptr, 0, nullptr));
+                            nullptr, 0, nullptr, p->cfg.split_chain != 0));
   }
   return err;
 }

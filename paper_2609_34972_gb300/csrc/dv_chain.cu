@@ -38,12 +38,15 @@ namespace {
 
 constexpr int kChainThreads = 128;
 
-template <int RP, int SPC>
+template <int RP, int SPC, bool SPLIT>
 struct ChainCfg {
   static constexpr int CW = 64 * SPC;             // hidden columns per CTA
   static constexpr int kSlab = 128 * 128;         // [128 rows][64 bf16], 128-byte swizzle
   static constexpr int kA = SPC * kSlab;          // bf16 state slice
   static constexpr int kH = (RP / 64) * kSlab;    // bf16 h
+  // split chain: the low bf16 parts of the state slice and of h, beside their high parts
+  static constexpr int kAlo = SPLIT ? kA : 0;
+  static constexpr int kHlo = SPLIT ? kH : 0;
   static constexpr int kDslab = RP * 128;         // D_l: RP rows x 64 columns
   static constexpr int kD = SPC * kDslab;
   static constexpr int kUslab = CW * 128;         // U_l: CW rows x 64 rank columns
@@ -53,8 +56,10 @@ struct ChainCfg {
   static constexpr int kRecvMax = 130 * RP * 4;
   static constexpr int kDRegion = kD > kRecvMax ? kD : kRecvMax;
   static constexpr int kOffA = 0;
-  static constexpr int kOffH = kOffA + kA;
-  static constexpr int kOffU = kOffH + kH;
+  static constexpr int kOffAlo = kOffA + kA;
+  static constexpr int kOffH = kOffAlo + kAlo;
+  static constexpr int kOffHlo = kOffH + kH;
+  static constexpr int kOffU = kOffHlo + kHlo;
   static constexpr int kOffD = kOffU + kU;
   // The fp32 partial z gets a region of its own where shared memory allows. Otherwise it takes
   // the U buffer: U_l then loads once the peers have acknowledged z (every copy out of the
@@ -158,12 +163,12 @@ __device__ __forceinline__ uint32_t sw128(int row, int c) {
   return static_cast<uint32_t>(row * 128 + ((c ^ (row & 7)) << 4));
 }
 
-template <int RP, int SPC>
+template <int RP, int SPC, bool SPLIT>
 __global__ void __launch_bounds__(kChainThreads, 1)
     dv_chain_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_constant__ CUtensorMap tmD,
                     const __grid_constant__ CUtensorMap tmU, const __grid_constant__ CUtensorMap tmM,
                     const __grid_constant__ ChainParams p) {
-  using C = ChainCfg<RP, SPC>;
+  using C = ChainCfg<RP, SPC, SPLIT>;
   constexpr int CW = C::CW;
   extern __shared__ uint8_t smem_raw[];
   const uint32_t raw = smem_addr(smem_raw);
@@ -186,7 +191,7 @@ __global__ void __launch_bounds__(kChainThreads, 1)
   const int t = row0 + tid;  // this thread's token row
   const int r_lo = chain_row_lo(s, S), n_rows = chain_row_lo(s + 1, S) - r_lo;  // rows summed here
   const uint32_t sA = base + C::kOffA, sH = base + C::kOffH, sD = base + C::kOffD,
-                 sU = base + C::kOffU;
+                 sU = base + C::kOffU, sAlo = base + C::kOffAlo, sHlo = base + C::kOffHlo;
   float* zpart = reinterpret_cast<float*>(base_ptr + C::kOffZ);
   const uint32_t sZ = base + C::kOffZ;
 
@@ -272,7 +277,7 @@ __global__ void __launch_bounds__(kChainThreads, 1)
     const uint32_t ph = static_cast<uint32_t>(l) & 1u;
     if (tid == 0) {  // this layer's transfers into this CTA: the peers' z rows, then h rows
       mbar_arrive_expect_tx(bar_rz, static_cast<uint32_t>((S - 1) * n_rows * RP * 4));
-      mbar_arrive_expect_tx(bar_rh, static_cast<uint32_t>((128 - n_rows) * RP * 2));
+      mbar_arrive_expect_tx(bar_rh, static_cast<uint32_t>((128 - n_rows) * RP * 2 * (SPLIT ? 2 : 1)));
     }
 
     // (1) down-projection partial z = bf16(M_{l-1})[:, slice] D_l[:, slice]^T; store M_{l-1}
@@ -288,6 +293,13 @@ __global__ void __launch_bounds__(kChainThreads, 1)
             umma_bf16(t_z, sdesc_kmajor_sw128(sA + j * C::kSlab + 32u * k),
                       sdesc_kmajor_sw128(sD + j * C::kDslab + 32u * k), idesc,
                       (j | k) != 0 ? 1u : 0u);
+        if (SPLIT && l > 0) {  // the low part of M_{l-1} (E, at l = 0, is exact in bf16)
+          for (int j = 0; j < SPC; ++j)
+#pragma unroll
+            for (int k = 0; k < 4; ++k)
+              umma_bf16(t_z, sdesc_kmajor_sw128(sAlo + j * C::kSlab + 32u * k),
+                        sdesc_kmajor_sw128(sD + j * C::kDslab + 32u * k), idesc, 1u);
+        }
         umma_commit(bar_z);
         mma_open = true;
       }
@@ -375,12 +387,20 @@ __global__ void __launch_bounds__(kChainThreads, 1)
           z.z += v.z;
           z.w += v.w;
         }
+        const float h0 = silu(z.x), h1 = silu(z.y), h2 = silu(z.z), h3 = silu(z.w);
         uint2 hv;
-        hv.x = pack_bf16x2(silu(z.x), silu(z.y));
-        hv.y = pack_bf16x2(silu(z.z), silu(z.w));
+        hv.x = pack_bf16x2(h0, h1);
+        hv.y = pack_bf16x2(h2, h3);
         // columns 4 c4 .. 4 c4 + 3: slab c4 / 16, 16-byte chunk (c4 % 16) / 2, half c4 % 2
-        *reinterpret_cast<uint2*>(base_ptr + C::kOffH + (c4 / 16) * C::kSlab +
-                                  sw128(row, (c4 % 16) / 2) + (c4 % 2) * 8) = hv;
+        const uint32_t hoff = static_cast<uint32_t>((c4 / 16) * C::kSlab + sw128(row, (c4 % 16) / 2) +
+                                                    (c4 % 2) * 8);
+        *reinterpret_cast<uint2*>(base_ptr + C::kOffH + hoff) = hv;
+        if (SPLIT) {  // the remainder h - bf16(h), itself in bf16, at the same place of its tile
+          uint2 lv;
+          lv.x = pack_bf16x2(h0 - __uint_as_float(hv.x << 16), h1 - __uint_as_float(hv.x & 0xFFFF0000u));
+          lv.y = pack_bf16x2(h2 - __uint_as_float(hv.y << 16), h3 - __uint_as_float(hv.y & 0xFFFF0000u));
+          *reinterpret_cast<uint2*>(base_ptr + C::kOffHlo + hoff) = lv;
+        }
         if (row0 + row < p.M)
           *reinterpret_cast<uint2*>(p.H + static_cast<long long>(row0 + row) * p.ldh + l * RP +
                                     c4 * 4) = hv;
@@ -397,6 +417,10 @@ __global__ void __launch_bounds__(kChainThreads, 1)
         for (int j = 0; j < RP / 64; ++j) {
           const uint32_t off = sH + static_cast<uint32_t>(j * C::kSlab + r_lo * 128);
           bulk_copy_to_peer(map_to_rank(off, rank), off, static_cast<uint32_t>(n_rows * 128), cbar);
+          if (SPLIT) {
+            const uint32_t lo = sHlo + static_cast<uint32_t>(j * C::kSlab + r_lo * 128);
+            bulk_copy_to_peer(map_to_rank(lo, rank), lo, static_cast<uint32_t>(n_rows * 128), cbar);
+          }
         }
       }
       if (tid == 0 && ok && !*abort_flag && l + 1 < p.L) load_d(l + 1);  // the z rows are summed
@@ -422,6 +446,12 @@ __global__ void __launch_bounds__(kChainThreads, 1)
             for (int k = 0; k < 4; ++k)
               umma_bf16(t_state, sdesc_kmajor_sw128(sH + j * C::kSlab + 32u * k),
                         sdesc_kmajor_sw128(sU + j * C::kUslab + 32u * k), idesc, 1u);
+          if (SPLIT)  // and the low part of h
+            for (int j = 0; j < RP / 64; ++j)
+#pragma unroll
+              for (int k = 0; k < 4; ++k)
+                umma_bf16(t_state, sdesc_kmajor_sw128(sHlo + j * C::kSlab + 32u * k),
+                          sdesc_kmajor_sw128(sU + j * C::kUslab + 32u * k), idesc, 1u);
           umma_commit(bar_up);
           mma_open = true;
         }
@@ -458,6 +488,18 @@ __global__ void __launch_bounds__(kChainThreads, 1)
           for (int q = 0; q < 4; ++q)
             *reinterpret_cast<uint4*>(slab + sw128(tid, h2 * 4 + q)) =
                 make_uint4(pk[4 * q], pk[4 * q + 1], pk[4 * q + 2], pk[4 * q + 3]);
+          if (SPLIT) {  // the low part M - bf16(M), the next down-projection's second operand
+            uint8_t* lslab = base_ptr + C::kOffAlo + c2 * C::kSlab;
+            uint32_t lo[16];
+#pragma unroll
+            for (int u = 0; u < 16; ++u)
+              lo[u] = pack_bf16x2(__uint_as_float(r[h2][2 * u]) - __uint_as_float(pk[u] << 16),
+                                  __uint_as_float(r[h2][2 * u + 1]) - __uint_as_float(pk[u] & 0xFFFF0000u));
+#pragma unroll
+            for (int q = 0; q < 4; ++q)
+              *reinterpret_cast<uint4*>(lslab + sw128(tid, h2 * 4 + q)) =
+                  make_uint4(lo[4 * q], lo[4 * q + 1], lo[4 * q + 2], lo[4 * q + 3]);
+          }
         }
       }
       if (t < p.M) p.part[l * p.part_ld + static_cast<long long>(s) * p.M + t] = ss;
@@ -494,12 +536,12 @@ __global__ void __launch_bounds__(kChainThreads, 1)
   if (tid == 0 && (!ok || *abort_flag)) atomicExch(p.status, DV_ERR_DEVICE_TIMEOUT);
 }
 
-template <int RP, int SPC>
+template <int RP, int SPC, bool SPLIT = false>
 cudaError_t launch_t(int S, long long blocks, const CUtensorMap& x, const CUtensorMap& dmap,
                      const CUtensorMap& umap, const CUtensorMap& mmap, const ChainParams& p,
                      cudaStream_t stream) {
-  using C = ChainCfg<RP, SPC>;
-  auto kern = dv_chain_kernel<RP, SPC>;
+  using C = ChainCfg<RP, SPC, SPLIT>;
+  auto kern = dv_chain_kernel<RP, SPC, SPLIT>;
   cudaError_t err =
       cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, C::kSmemBytes);
   if (err == cudaSuccess && S > 8)
@@ -549,7 +591,8 @@ bool chain_shape(int d, int r_pad, int* spc_out, int* s_out) {
 cudaError_t launch_chain(int r_pad, int spc, int S, long long tokens, int n_layers, int d,
                          const CUtensorMap& x, const CUtensorMap& dmap, const CUtensorMap& umap,
                          const CUtensorMap& mmap, float* part, long long part_ld, uint16_t* H,
-                         int* status, unsigned long long timeout_ns, cudaStream_t stream) {
+                         int* status, unsigned long long timeout_ns, cudaStream_t stream,
+                         bool split) {
   ChainParams p;
   p.H = H;
   p.ldh = n_layers * r_pad;
@@ -561,6 +604,12 @@ cudaError_t launch_chain(int r_pad, int spc, int S, long long tokens, int n_laye
   p.status = status;
   p.timeout_ns = timeout_ns;
   const long long blocks = (tokens + 127) / 128;
+  if (split) {  // the low parts fit beside the state at r_pad 64 only
+    if (r_pad == 64 && spc == 2) return launch_t<64, 2, true>(S, blocks, x, dmap, umap, mmap, p, stream);
+    if (r_pad == 64 && spc == 3) return launch_t<64, 3, true>(S, blocks, x, dmap, umap, mmap, p, stream);
+    if (r_pad == 64 && spc == 4) return launch_t<64, 4, true>(S, blocks, x, dmap, umap, mmap, p, stream);
+    return cudaErrorInvalidValue;
+  }
   if (r_pad == 64 && spc == 2) return launch_t<64, 2>(S, blocks, x, dmap, umap, mmap, p, stream);
   if (r_pad == 64 && spc == 3) return launch_t<64, 3>(S, blocks, x, dmap, umap, mmap, p, stream);
   if (r_pad == 64 && spc == 4) return launch_t<64, 4>(S, blocks, x, dmap, umap, mmap, p, stream);

@@ -212,13 +212,15 @@ int down_splits(long long m_tiles, int k_slabs, int num_sms);
 // layers with the fp32 state in TMEM. chain_shape gives the slabs per CTA (spc) and S for a
 // hidden size and r_pad, or false when the chain does not fit (then the per-layer launches
 // run). launch_chain returns cudaErrorNotSupported when no cluster of that size can be resident.
+// split: the split chain (hi + lo bf16 operands), available on chip at r_pad 64 only.
 // x: x0 (128-row boxes); dmap: stacked D (r_pad-row boxes); umap: U as [L d][r_pad] (64 spc-row
 // boxes); mmap: the stacked M_l as a 3-D (d, tokens, L) map with (64, 128, 1) boxes.
 bool chain_shape(int d, int r_pad, int* spc_out, int* s_out);
 cudaError_t launch_chain(int r_pad, int spc, int S, long long tokens, int n_layers, int d,
                          const CUtensorMap& x, const CUtensorMap& dmap, const CUtensorMap& umap,
                          const CUtensorMap& mmap, float* part, long long part_ld, uint16_t* H,
-                         int* status, unsigned long long timeout_ns, cudaStream_t stream);
+                         int* status, unsigned long long timeout_ns, cudaStream_t stream,
+                         bool split);
 
 // Token tile (64, 128, 192 or 256) of the pair kernel for a build of `tokens` tokens.
 int kv_pair_tile_n(long long tokens);
@@ -253,6 +255,7 @@ struct PlanView {
   const CUtensorMap* tm_Uup;       // recurrent: [L*d][r_pad], boxes of resid_bn rows
   const uint16_t* Uup;             // recurrent: U_l as [L*d][r_pad] ([U_l | U_l] when split)
   int split_chain;                 // recurrent: hi + lo bf16 operands in the chain's GEMMs
+  int uup_ld;                      // row pitch of Uup: r_pad, or 2 r_pad with the split chain
   int resid_bn;                    // recurrent: column tile of the up-projection step
   const double* inv_freq;     // head_dim / 2 values
   const uint16_t* Wkv;        // repacked K/V weights [L*2kv][k_total]

@@ -4,7 +4,8 @@ The chain M_l = M_{l-1} + SiLU(M_{l-1} D_l) U_l feeds each layer's down-projecti
 previous state, so a bf16 operand there (and for h_l in the up-projection) adds one rounding per
 layer, and the error grows with depth. With split_chain the two GEMMs read each operand as a high
 and a low bf16 part, and the state keeps about fp32 accuracy; only the K/V GEMM reads the bf16
-rounding of M_l. These cases check the build against the fp64 oracle, the chain's state layer by
+rounding of M_l. At r_pad 64 the chain runs on chip (the low parts beside the state in shared
+memory); at larger r_pad as per-layer launches. The small cases cover both. These cases check the build against the fp64 oracle, the chain's state layer by
 layer, and that the split chain stays at the bar where the one-part chain drifts toward it.
 """
 import numpy as np
@@ -104,10 +105,11 @@ def test_split_chain_layer_modes_and_noalloc():
     assert torch.equal(k, k2) and torch.equal(v, v2)
 
 
-@pytest.mark.parametrize("name", ["llava_next_7b", "qwen25vl_7b_video"])
+@pytest.mark.parametrize("name", ["llava15_7b", "llava_next_7b", "qwen25vl_7b_video"])
 def test_split_chain_full_size_sampled(name):
-    # The deepest and the largest recurrent builds at full size, sampled tokens (every token
-    # block's edges, every batch element) against the oracle.
+    # Full-size recurrent builds with the split chain, sampled tokens (every token block's edges,
+    # every batch element) against the oracle: on chip at r_pad 64 (LLaVA-1.5), per layer at
+    # r_pad 128 and 256.
     import torch
     from dataclasses import replace
     cfg = replace(synth.CONFIGS[name], adapter="recurrent", split_chain=True)
