@@ -93,8 +93,9 @@ typedef struct dv_config {
                             chain's two GEMMs (M_{l-1} into the down-projection, h_l into the
                             up-projection) is read as a high and a low bf16 part, two MMAs per
                             product, so the state M_l keeps about fp32 accuracy through deep
-                            chains; the chain runs on chip at rank <= 64 and as per-layer
-                            launches above. 0 = one bf16 operand (faster). */
+                            chains; the chain then runs on chip only at rank <= 64 (where
+                            the on-chip chain fits d at all), else as per-layer launches.
+                            0 = one bf16 operand (faster). */
 } dv_config;
 
 /* Weights of all L layers, bf16, device pointers. Read only during dv_memory_plan: the plan
