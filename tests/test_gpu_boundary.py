@@ -207,3 +207,29 @@ def test_host_pipeline_rejects_shapes_beyond_the_plan(env):
         with pytest.raises(dv.DvError) as e:
             dv.HostPipeline(plan, b, n, depth=depth)
         assert e.value.code == code
+
+
+def test_host_pipeline_mrope_bias_recurrent():
+    # Three position axes (M-RoPE) and K/V bias through the host entry, with the recurrent
+    # adapter: the host buffers equal the device build of the same inputs.
+    import torch
+    import paper_2609_34972_gb300 as dv
+    cfg = gu.small_config("host_mrope", d=512, n_layers=3, n_kv_heads=2, n_heads=4, head_dim=128,
+                          rank=64, n_vis=150, batch=2, rope="mrope", rope_theta=1e6,
+                          mrope_section=(16, 24, 24), grid=(1, 10, 15), x0_sigma=0.5,
+                          bias_sigma=0.02, w_sigma=0.05, seed=131, pos_start=15,
+                          adapter="recurrent")
+    inp = synth.make_inputs(cfg)
+    k_ref, v_ref, plan = gu.run_build(inp)
+    pipe = dv.HostPipeline(plan, cfg.batch, cfg.n_vis, depth=2)
+    x0_h = gu.torch_bf16(inp.x0, "cpu").pin_memory()
+    pos_h = torch.from_numpy(np.ascontiguousarray(inp.pos)).pin_memory()
+    assert tuple(pos_h.shape) == (cfg.batch, 3, cfg.n_vis)
+    kh, vh = _host_kv(cfg, torch, -1.0)
+    for _ in range(2):
+        t = pipe.submit(x0_h, pos_h, kh, vh)
+    pipe.wait(t)
+    assert torch.equal(kh, k_ref.cpu()) and torch.equal(vh, v_ref.cpu())
+    assert dv.plan_status(plan) == dv.DV_OK
+    pipe.close()
+    dv.free(plan)
