@@ -54,6 +54,9 @@ def test_roofline_figures():
     t_roof = max(cfg.flops() / 1888.7e12, cfg.min_bytes() / 6764e9) * 1e3
     assert step["t_roof_ms"] == pytest.approx(t_roof) and step["frac"] == pytest.approx(t_roof / 28.0)
     assert 27.0 < t_roof < 27.1                             # 51.02 TFLOP at the burst peak
+    # beside them, NVIDIA's dense bf16 figure of 2.25 PFLOP/s: 22.7 ms for the same work
+    assert roof["frac_nominal"] == pytest.approx(roof["achieved"] / 2250.0)
+    assert step["frac_nominal"] == pytest.approx(cfg.flops() / 2250e12 * 1e3 / 28.0)
 
 
 def test_scaling_values():
