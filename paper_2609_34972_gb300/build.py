@@ -14,7 +14,7 @@ ROOT = os.path.dirname(HERE)
 CSRC = os.path.join(HERE, "csrc")
 LIB_PATH = os.path.join(HERE, "libdv.so")
 SOURCES = ["dv_api.cu", "dv_gemm.cu", "dv_kv2sm.cu", "dv_pair_tm.cu", "dv_recurrent.cu", "dv_chain.cu", "dv_attention.cu",
-           "dv_noalloc.cu", "dv_host.cu"]
+           "dv_noalloc.cu", "dv_host.cu", "dv_fold.cu"]
 HEADERS = ["dv_internal.h", "dv_ptx.cuh", "dv_epilogue.cuh"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 NVCC_FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-Xptxas", "-v"]

@@ -39,6 +39,10 @@ struct dv_plan {
   uint16_t* Bn = nullptr;
   uint16_t* Wkv = nullptr;
   uint16_t* Uup = nullptr;     // recurrent adapter: U_l as [L*d][uup_ld] (split chain: [U_l | U_l])
+  uint16_t* Pf = nullptr;      // recurrent adapter, refactored chain: [L*r_pad][(L+2)*r_pad]
+                               // (k_fold_identity, k_fold_products), or null
+  bool fold = false;           // recurrent builds may run the refactored chain (dv_fold.cu)
+  int chain_clusters = 0;      // recurrent: clusters of the on-chip chain resident at once
   int uup_ld = 0;              // r_pad, or 2 r_pad with the split chain
   float* bk = nullptr;
   float* bv = nullptr;
@@ -54,6 +58,7 @@ struct dv_plan {
   CUtensorMap tm_Bn_half;      // slab map, boxes of 128 rows (CTA-pair halves)
   CUtensorMap tm_Wkv;          // slab map, boxes of 128 rows
   CUtensorMap tm_Dst_rp, tm_Uup;  // recurrent adapter
+  CUtensorMap tm_Pf;              // recurrent adapter: Pf with r_pad-row boxes
   int resid_bn = 0;
   double inv_freq[dv::kMaxHalfHead];
   unsigned char mode[dv::kMaxLayers];  // DV_LAYER_* per layer
@@ -109,17 +114,16 @@ bool encode_2d(CUtensorMap* map, const void* ptr, uint64_t cols, uint64_t rows, 
 }
 
 // bf16 [rows][cols] (row stride ld elements) viewed as {64 columns, rows, cols / 64 slabs} for
-// the 2-SM kernels: one box = box_rows rows x kSlabsPerStep consecutive K slabs, each slab a
-// 128-byte-swizzled [box_rows][64] tile. cols must be a multiple of 64; slabs past the end of
+// the 2-SM kernels: one box = box_rows rows x box_slabs (default kSlabsPerStep) consecutive K
+// slabs, each slab a 128-byte-swizzled [box_rows][64] tile. cols must be a multiple of 64; slabs past the end of
 // the matrix read as zero.
 bool encode_slabs(CUtensorMap* map, const void* ptr, uint64_t cols, uint64_t rows, uint64_t ld,
-                  uint32_t box_rows) {
+                  uint32_t box_rows, uint32_t box_slabs = dv::kSlabsPerStep) {
   EncodeTiledFn fn = encode_fn();
   if (!fn || cols % dv::kBlockK != 0) return false;
   cuuint64_t dims[3] = {static_cast<cuuint64_t>(dv::kBlockK), rows, cols / dv::kBlockK};
   cuuint64_t strides[2] = {ld * 2, static_cast<cuuint64_t>(dv::kBlockK) * 2};
-  cuuint32_t box[3] = {static_cast<cuuint32_t>(dv::kBlockK), box_rows,
-                       static_cast<cuuint32_t>(dv::kSlabsPerStep)};
+  cuuint32_t box[3] = {static_cast<cuuint32_t>(dv::kBlockK), box_rows, box_slabs};
   cuuint32_t estr[3] = {1, 1, 1};
   return fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(ptr), dims, strides, box,
             estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
@@ -350,6 +354,76 @@ __global__ void k_bias_to_f32(const uint16_t* __restrict__ b, float* __restrict_
   for (long long e = blockIdx.x * static_cast<long long>(blockDim.x) + threadIdx.x; e < n;
        e += static_cast<long long>(gridDim.x) * blockDim.x)
     out[e] = bf(b[static_cast<long long>(pl.src[e / kv]) * kv + e % kv]);
+}
+
+// Recurrent adapter, refactored chain (dv_fold.cu). Pf [L r_pad][pld], pld = (L + 2) r_pad:
+// row i r_pad + a holds, for planned layer i,
+//   columns [0, r_pad) and [r_pad, 2 r_pad): 1 at column a (the identity blocks that add the two
+//   bf16 parts of C_i in the recurrence GEMM);
+//   columns (2 + j) r_pad + b, j < i: bf16 of Q_ij[a][b] = sum_e D_i[a][e] U_j[e][b] (a, b < r;
+//   zero where layer i or j is an identity layer);
+//   everything else 0.
+// The identity entries; the rest is zeroed by the caller before k_fold_products.
+__global__ void k_fold_identity(uint16_t* __restrict__ Pf, int L, int r_pad, long long pld) {
+  const long long n = static_cast<long long>(L) * r_pad;
+  for (long long row = blockIdx.x * static_cast<long long>(blockDim.x) + threadIdx.x; row < n;
+       row += static_cast<long long>(gridDim.x) * blockDim.x) {
+    const int a = static_cast<int>(row % r_pad);
+    Pf[row * pld + a] = 0x3F80;          // 1.0
+    Pf[row * pld + r_pad + a] = 0x3F80;
+  }
+}
+
+// Q_ij blocks: grid (r_pad / 64 b-tiles, (L) * (r_pad / 64) (j, a-tile), L (i)); blocks with
+// j >= i return. 64 x 64 outputs per block, 256 threads with 4 x 4 each, fp32 accumulation
+// over e in steps of 32 (a fixed order).
+__global__ void __launch_bounds__(256) k_fold_products(const uint16_t* __restrict__ D,
+                                                       const uint16_t* __restrict__ U,
+                                                       uint16_t* __restrict__ Pf, int L, int r,
+                                                       int r_pad, int d, long long pld,
+                                                       PackLayers pl) {
+  const int at_n = r_pad / 64;
+  const int i = blockIdx.z, j = blockIdx.y / at_n, at = blockIdx.y % at_n;
+  if (j >= i) return;
+  const bool zero = pl.zero_du[i] || pl.zero_du[j];
+  const int li = pl.src[i], lj = pl.src[j];
+  const int a0 = at * 64, b0 = blockIdx.x * 64;
+  __shared__ float Ds[32][65];
+  __shared__ float Us[32][65];
+  const int tx = threadIdx.x & 15, ty = threadIdx.x >> 4;
+  float acc[4][4] = {};
+  for (int e0 = 0; e0 < d; e0 += 32) {
+    for (int e = threadIdx.x; e < 64 * 32; e += 256) {
+      const int aa = e / 32, ee = e % 32;  // D row a0 + aa, contiguous in e
+      Ds[ee][aa] = (a0 + aa < r && !zero)
+                       ? bf(D[(static_cast<long long>(li) * r + a0 + aa) * d + e0 + ee]) : 0.0f;
+      const int bb = e % 64, ek = e / 64;  // U row e0 + ek, contiguous in b
+      Us[ek][bb] = (b0 + bb < r && !zero)
+                       ? bf(U[(static_cast<long long>(lj) * d + e0 + ek) * r + b0 + bb]) : 0.0f;
+    }
+    __syncthreads();
+#pragma unroll 8
+    for (int ee = 0; ee < 32; ++ee) {
+      float av[4], uv[4];
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        av[q] = Ds[ee][ty * 4 + q];
+        uv[q] = Us[ee][tx * 4 + q];
+      }
+#pragma unroll
+      for (int q = 0; q < 4; ++q)
+#pragma unroll
+        for (int w = 0; w < 4; ++w) acc[q][w] = fmaf(av[q], uv[w], acc[q][w]);
+    }
+    __syncthreads();
+  }
+#pragma unroll
+  for (int q = 0; q < 4; ++q) {
+    const long long row = static_cast<long long>(i) * r_pad + a0 + ty * 4 + q;
+#pragma unroll
+    for (int w = 0; w < 4; ++w)
+      Pf[row * pld + static_cast<long long>(2 + j) * r_pad + b0 + tx * 4 + w] = to_bf16(acc[q][w]);
+  }
 }
 
 // Uup[i*d + j][n] = U[src[i]][j][n mod r_pad] for (n mod r_pad) < r, else 0: the up-projection
@@ -607,7 +681,7 @@ int check_config(const dv_config* c) {
 }
 
 void free_plan_memory(dv_plan* p) {
-  void* ptrs[] = {p->Dst, p->Bn, p->Wkv, p->Uup, p->bk, p->bv, p->kg, p->Gf, p->ws, p->status};
+  void* ptrs[] = {p->Dst, p->Bn, p->Wkv, p->Uup, p->Pf, p->bk, p->bv, p->kg, p->Gf, p->ws, p->status};
   for (void* q : ptrs)
     if (q) cudaFree(q);
   for (cudaEvent_t e : p->ev) cudaEventDestroy(e);
@@ -746,11 +820,97 @@ static cudaError_t launch_recurrent_kv(const PlanView& v, const BuildArgs& a, lo
   return err;
 }
 
+// Recurrent builds of this plan may run the refactored chain (dv_fold.cu): its workspace holds
+// the two parts of E D^T instead of the per-layer path's fp32 state.
+static bool uses_fold(const PlanView& v) { return v.tm_Pf != nullptr; }
+
+// The refactored chain runs a build unless its token blocks fit in one wave of on-chip chain
+// clusters: the chain spreads each block over a cluster of 14-16 SMs, where the refactored
+// recurrence keeps a block on one SM.
+static bool fold_build(const PlanView& v, long long tokens) {
+  return uses_fold(v) && (tokens + kBlockM - 1) / kBlockM > v.chain_clusters;
+}
+
+// Recurrent adapter by the refactored chain (dv_fold.cu): (1) C = E [D_1 .. D_L]^T as two bf16
+// parts, one GEMM on the engine the embedding adapter's down-projection would use; (2) the
+// recurrence h_l = SiLU(C_l + sum_{j<l} h_j Q_lj^T) per 128-token block; (3) the running sum
+// M_l = E + sum_{j<=l} h_j U_j^T with the rows' sums of squares; then the RMS statistics and one
+// K/V launch over all layers, as in the chain below.
+static cudaError_t enqueue_fold(const PlanView& v, const BuildArgs& a, cudaStream_t st) {
+  const long long T = static_cast<long long>(a.batch) * a.n_vis;
+  const int L = v.n_layers, d = v.d;
+  const long long n1 = static_cast<long long>(L) * v.r_pad;
+  const int cw = fold_slice_cols(d);
+  auto mark = [&](int i) {
+    if (a.marks) cudaEventRecord(a.marks[i], st);
+  };
+  const uint32_t ks = static_cast<uint32_t>(hchain_box_slabs(v.r_pad));
+  CUtensorMap tm_x0, tm_x0_s, tm_chi, tm_clo, tm_hs, tm_h, tm_u, tm_m3, tm_mem_s;
+  if (!encode_2d(&tm_x0, a.x0, d, static_cast<uint64_t>(T), d, kBlockM) ||
+      !encode_slabs(&tm_x0_s, a.x0, d, static_cast<uint64_t>(T), d, kBlockM) ||
+      !encode_slabs(&tm_chi, a.Chi, n1, static_cast<uint64_t>(T), n1, kBlockM, ks) ||
+      !encode_slabs(&tm_clo, a.Clo, n1, static_cast<uint64_t>(T), n1, kBlockM, ks) ||
+      !encode_slabs(&tm_hs, a.H, n1, static_cast<uint64_t>(T), a.hld, kBlockM, ks) ||
+      !encode_2d(&tm_h, a.H, n1, static_cast<uint64_t>(T), a.hld, kBlockM) ||
+      !encode_2d(&tm_u, v.Uup, v.r_pad, static_cast<uint64_t>(L) * d, v.uup_ld, cw) ||
+      !encode_3d(&tm_m3, a.mem, d, static_cast<uint64_t>(T), L, kBlockM) ||
+      !encode_slabs(&tm_mem_s, a.mem, d, static_cast<uint64_t>(L) * T, d, kBlockM))
+    return cudaErrorInvalidValue;
+  mark(0);
+  // (1) C = E [D_1 .. D_L]^T, every column into the two bf16 parts
+  GemmParams gp;
+  std::memset(&gp, 0, sizeof(gp));
+  gp.status = v.status;
+  gp.timeout_ns = kTimeoutNs;
+  for (int i = 0; i < L; ++i) gp.layer_map[i] = v.active[i];
+  gp.s = {static_cast<int>(T), 1, static_cast<int>(n1), d / 64, 0, 0, 0, 0, 0, 0};
+  gp.silu = {nullptr, 0, 0, nullptr, static_cast<int>(n1), a.Chi, a.Clo};
+  const long long pad128 = (T + 127) / 128 * 128, pad256 = (T + 255) / 256 * 256;
+  cudaError_t err;
+  if (prefer_256(pad256, pad128)) {
+    const long long pairs = v.num_sms / 2;
+    int bn = 64;
+    for (int cand : {256, 128})
+      if (n1 % cand == 0 && (pad256 / 256) * (n1 / cand) >= pairs) {
+        bn = cand;
+        break;
+      }
+    tm_groups(gp.s, bn, T);
+    err = launch_pair_tm(EPI_SILU, bn, 0, tm_x0_s, tm_x0_s,
+                         v.tm_Dst_half[bn == 64 ? 0 : (bn == 128 ? 1 : 2)], gp, v.num_sms, st);
+  } else {
+    int bn = 64;
+    for (int cand : {256, 128})
+      if (n1 % cand == 0 && (pad128 / 128) * (n1 / cand) >= v.num_sms) {
+        bn = cand;
+        break;
+      }
+    err = launch_gemm(EPI_SILU, bn, 0, tm_x0, tm_x0, v.tm_Dst[bn == 64 ? 0 : (bn == 128 ? 1 : 2)],
+                      gp, v.num_sms, st);
+  }
+  mark(1);
+  // (2) the recurrence over the rank-r vectors, (3) the running sum of the memories
+  const long long part_ld = static_cast<long long>(d / 64) * T;
+  if (err == cudaSuccess)
+    err = launch_hchain(v.r_pad, T, L, tm_chi, tm_clo, tm_hs, *v.tm_Pf, a.H, static_cast<int>(a.hld),
+                        v.status, kTimeoutNs, st);
+  if (err == cudaSuccess)
+    err = launch_accum(v.r_pad, cw, T, L, d, a.x0, tm_h, tm_u, tm_m3, a.part, part_ld, v.status,
+                       kTimeoutNs, st);
+  mark(2);
+  if (err == cudaSuccess)
+    err = launch_pdl(k_rstd_parts, dim3(grid_for(static_cast<long long>(L) * T)), dim3(256), st,
+                     a.part, L, T, d / cw, part_ld, 1.0f / d, v.rms_eps, a.rstd);
+  mark(3);
+  return err == cudaSuccess ? launch_recurrent_kv(v, a, T, tm_mem_s, st, mark) : err;
+}
+
 // Recurrent adapter (Sec. 3.1 Eq. 6): the chain M_i = M_{i-1} + SiLU(M_{i-1} D_i) U_i runs
 // layer by layer (a split-K down-projection, then the up-projection whose epilogue adds the
 // fp32 state and writes bf16 M_i and partial sums of squares); the RMS statistics of all
 // layers follow in one kernel, and one K/V launch covers every layer, reading M_i as A.
 static cudaError_t enqueue_recurrent(const PlanView& v, const BuildArgs& a, cudaStream_t st) {
+  if (fold_build(v, static_cast<long long>(a.batch) * a.n_vis)) return enqueue_fold(v, a, st);
   const long long T = static_cast<long long>(a.batch) * a.n_vis;
   const int L = v.n_layers, d = v.d;
   const long long n1 = static_cast<long long>(L) * v.r_pad;
@@ -787,7 +947,10 @@ static cudaError_t enqueue_recurrent(const PlanView& v, const BuildArgs& a, cuda
       return err == cudaSuccess ? launch_recurrent_kv(v, a, T, tm_mem_s, st, mark) : err;
     }
     if (err != cudaErrorNotSupported) return err;
-    err = cudaSuccess;  // no cluster of that size fits: the per-layer launches below
+    cudaGetLastError();
+    // no cluster of that size fits: the refactored chain, or the per-layer launches below
+    if (uses_fold(v)) return enqueue_fold(v, a, st);
+    err = cudaSuccess;
   }
   const long long m_tiles = (T + kBlockM - 1) / kBlockM;
   const int splits = down_splits(m_tiles, d / kBlockK, v.num_sms);
@@ -1002,11 +1165,18 @@ size_t carve_workspace(const PlanView& v, long long T, void* base, BuildArgs* a)
   const size_t hld = L * v.r_pad + (rec ? 0 : 64), xld = d + 64;
   const size_t oH = take(t * hld * 2), oR = take(L * t * 4), oX = take(t * 4);
   const size_t oXp = rec ? 0 : take(t * xld * 2);
-  size_t oS = 0, oM = 0, oP = 0, oC = 0, oHl = 0, oMl = 0;
+  size_t oS = 0, oM = 0, oP = 0, oC = 0, oHl = 0, oMl = 0, oChi = 0, oClo = 0;
   const bool small_path = !rec && v.r_pad == 64;  // x0 (2 U_l)^T in fp32 (see enqueue_build)
   if (small_path) oC = take(t * L * v.r_pad * 4);
+  // recurrent adapter: E D_l^T in two bf16 parts for the refactored chain, else the fp32 state
+  const bool fold = rec && uses_fold(v);
   if (rec) {
-    oS = take(t * d * 4);
+    if (fold) {
+      oChi = take(t * L * v.r_pad * 2);
+      oClo = take(t * L * v.r_pad * 2);
+    } else {
+      oS = take(t * d * 4);
+    }
     oM = take(L * t * d * 2);
     oP = take(L * (d / 64) * t * 4);
     if (v.split_chain) {  // low bf16 parts of h_l (every layer) and of the last M_l
@@ -1022,7 +1192,9 @@ size_t carve_workspace(const PlanView& v, long long T, void* base, BuildArgs* a)
     a->x0p_ld = static_cast<long long>(xld);
     a->rstd = reinterpret_cast<float*>(b + oR);
     a->xx = reinterpret_cast<float*>(b + oX);
-    a->state = rec ? reinterpret_cast<float*>(b + oS) : nullptr;
+    a->state = rec && !fold ? reinterpret_cast<float*>(b + oS) : nullptr;
+    a->Chi = fold ? reinterpret_cast<uint16_t*>(b + oChi) : nullptr;
+    a->Clo = fold ? reinterpret_cast<uint16_t*>(b + oClo) : nullptr;
     a->mem = rec ? reinterpret_cast<uint16_t*>(b + oM) : nullptr;
     a->part = rec ? reinterpret_cast<float*>(b + oP) : nullptr;
     a->c = small_path ? reinterpret_cast<float*>(b + oC) : nullptr;
@@ -1064,6 +1236,8 @@ bool plan_view(const dv_plan* p, PlanView* v) {
   v->tm_Dst_rp = &p->tm_Dst_rp;
   v->tm_Uup = &p->tm_Uup;
   v->Uup = p->Uup;
+  v->tm_Pf = p->fold ? &p->tm_Pf : nullptr;
+  v->chain_clusters = p->chain_clusters;
   v->uup_ld = p->uup_ld;
   v->split_chain = p->cfg.split_chain;
   v->Dst = p->Dst;
@@ -1111,6 +1285,12 @@ cudaError_t preload_build_kernels(const dv_plan* p) {
   }
   keep(dv::launch_pair_tm(dv::EPI_KV, 256, hd, m, m, m, gp, 1, nullptr));
   for (int nt : {64, 128, 192, 256}) keep(dv::launch_kv_pair(hd, nt, m, m, m, gp, 1, nullptr));
+  if (p->fold) {
+    const int cw = dv::fold_slice_cols(p->cfg.d);
+    keep(dv::launch_hchain(p->r_pad, 0, 1, m, m, m, m, nullptr, 0, nullptr, 0, nullptr));
+    keep(dv::launch_accum(p->r_pad, cw, 0, 1, p->cfg.d, nullptr, m, m, m, nullptr, 0, nullptr, 0,
+                          nullptr));
+  }
   if (p->cfg.adapter == DV_ADAPTER_RECURRENT) {
     dv::DownParams dp;
     std::memset(&dp, 0, sizeof(dp));
@@ -1211,6 +1391,11 @@ int dv_memory_plan(const dv_config* cfg, const dv_weights* w, void* stream, dv_p
   p->uup_ld = cfg->split_chain ? 2 * p->r_pad : p->r_pad;
   p->max_tokens = cfg->max_batch * cfg->max_n_vis;
   const long long T = p->max_tokens;
+  // Recurrent adapter: the refactored chain (dv_fold.cu) unless the split chain is asked for;
+  // builds whose token blocks fit in one wave of on-chip chain clusters take the chain instead.
+  p->fold = rec && !cfg->split_chain && dv::fold_slice_cols(d) > 0;
+  p->chain_clusters = rec ? dv::chain_resident_clusters(d, p->r_pad, cfg->split_chain != 0) : 0;
+  const long long pf_ld = static_cast<long long>(L + 2) * p->r_pad;
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   // The recurrent K/V GEMM addresses the stacked M_l as L * T rows (32-bit TMA coordinates).
   if (rec && static_cast<long long>(L) * T + dv::kBlockM >= (1LL << 31)) {
@@ -1236,6 +1421,8 @@ int dv_memory_plan(const dv_config* cfg, const dv_weights* w, void* stream, dv_p
     ok = dmalloc(&p->bk, sizeof(float) * L * p->kv) && dmalloc(&p->bv, sizeof(float) * L * p->kv);
   if (ok && cfg->k_norm) ok = dmalloc(&p->kg, sizeof(float) * L * HD);
   if (ok && !rec) ok = dmalloc(&p->Gf, sizeof(float) * L * p->r_pad * p->r_pad);
+  const size_t pf_bytes = sizeof(uint16_t) * static_cast<size_t>(L) * p->r_pad * pf_ld;
+  if (ok && p->fold) ok = dmalloc(&p->Pf, pf_bytes);
   if (!ok) {
     free_plan_memory(p);
     delete p;
@@ -1261,6 +1448,14 @@ int dv_memory_plan(const dv_config* cfg, const dv_weights* w, void* stream, dv_p
   if (rec) {
     k_pack_up<<<grid_for(1LL * L * d * p->uup_ld), 256, 0, st>>>(U, p->Uup, L, r, p->r_pad, d,
                                                                  p->uup_ld, pl);
+    if (p->fold) {
+      cudaMemsetAsync(p->Pf, 0, pf_bytes, st);
+      k_fold_identity<<<grid_for(1LL * L * p->r_pad), 256, 0, st>>>(p->Pf, L, p->r_pad, pf_ld);
+      if (L > 1) {
+        const dim3 gq(p->r_pad / 64, L * (p->r_pad / 64), L);
+        k_fold_products<<<gq, 256, 0, st>>>(D, U, p->Pf, L, r, p->r_pad, d, pf_ld, pl);
+      }
+    }
   } else {
     k_pack_2u<<<grid_for(1LL * L * p->r_pad * d), 256, 0, st>>>(
         U, p->Dst + static_cast<size_t>(L) * p->r_pad * dst_ld, L, r, p->r_pad, d, dst_ld, pl);
@@ -1301,6 +1496,9 @@ int dv_memory_plan(const dv_config* cfg, const dv_weights* w, void* stream, dv_p
   if (enc && rec) {
     enc = encode_2d(&p->tm_Dst_rp, p->Dst, d, 1ull * L * p->r_pad, dst_ld, p->r_pad) &&
           encode_2d(&p->tm_Uup, p->Uup, p->uup_ld, 1ull * L * d, p->uup_ld, p->resid_bn);
+    if (enc && p->fold)
+      enc = encode_slabs(&p->tm_Pf, p->Pf, pf_ld, 1ull * L * p->r_pad, pf_ld, p->r_pad,
+                         static_cast<uint32_t>(dv::hchain_box_slabs(p->r_pad)));
   } else if (enc) {
     enc = encode_slabs(&p->tm_Bn_half, p->Bn, p->bn_k, 256ull * p->bn_groups, p->bn_k, 128) &&
           encode_2d(&p->tm_Bn, p->Bn, p->bn_k, 256ull * p->bn_groups, p->bn_k, 256);

@@ -571,7 +571,53 @@ cudaError_t launch_t(int S, long long blocks, const CUtensorMap& x, const CUtens
   return cudaGetLastError();
 }
 
+template <int RP, int SPC, bool SPLIT = false>
+int resident_t(int S) {
+  using C = ChainCfg<RP, SPC, SPLIT>;
+  auto kern = dv_chain_kernel<RP, SPC, SPLIT>;
+  if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, C::kSmemBytes) !=
+          cudaSuccess ||
+      (S > 8 && cudaFuncSetAttribute(kern, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) !=
+                    cudaSuccess)) {
+    cudaGetLastError();
+    return 0;
+  }
+  cudaLaunchConfig_t cfg = {};
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = static_cast<unsigned>(S);
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.gridDim = dim3(static_cast<unsigned>(S), 1, 1);
+  cfg.blockDim = dim3(kChainThreads, 1, 1);
+  cfg.dynamicSmemBytes = C::kSmemBytes;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  int clusters = 0;
+  if (cudaOccupancyMaxActiveClusters(&clusters, kern, &cfg) != cudaSuccess) {
+    cudaGetLastError();
+    return 0;
+  }
+  return clusters;
+}
+
 }  // namespace
+
+int chain_resident_clusters(int d, int r_pad, bool split) {
+  int spc = 0, S = 0;
+  if (!chain_shape(d, r_pad, &spc, &S)) return 0;
+  if (split) {
+    if (r_pad == 64 && spc == 2) return resident_t<64, 2, true>(S);
+    if (r_pad == 64 && spc == 3) return resident_t<64, 3, true>(S);
+    if (r_pad == 64 && spc == 4) return resident_t<64, 4, true>(S);
+    return 0;
+  }
+  if (r_pad == 64 && spc == 2) return resident_t<64, 2>(S);
+  if (r_pad == 64 && spc == 3) return resident_t<64, 3>(S);
+  if (r_pad == 64 && spc == 4) return resident_t<64, 4>(S);
+  if (r_pad == 128 && spc == 4) return resident_t<128, 4>(S);
+  return 0;
+}
 
 bool chain_shape(int d, int r_pad, int* spc_out, int* s_out) {
   if (r_pad != 64 && r_pad != 128) return false;

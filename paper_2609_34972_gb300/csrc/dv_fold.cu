@@ -1,0 +1,678 @@
+// The recurrent adapter (Sec. 3.1 Eq. 6) through an exact rearrangement of its chain. With rows
+// of M, D_l [r][d] and U_l [d][r] (nn.Linear layout):
+//   M_0 = E,   M_l = M_{l-1} + h_l U_l^T,   h_l = SiLU(z_l),   z_l = M_{l-1} D_l^T.
+// Unrolling M_{l-1} = E + sum_{j<l} h_j U_j^T gives
+//   z_l = E D_l^T + sum_{j<l} h_j Q_lj^T,   Q_lj = D_l U_j (r x r, formed once per weight set),
+// so the chain splits into three parts, none of which moves the d-wide state between layers:
+//   (1) C = E [D_1 ... D_L]^T, one GEMM over all layers on the GEMM engines, written as two bf16
+//       parts C = hi + lo (2^-17 relative);
+//   (2) dv_hchain_kernel: per 128-token block, the recurrence over the r-wide vectors,
+//         z_l = [C_l^hi | C_l^lo | h_1 .. h_{l-1}] [I ; I ; Q_l1 .. Q_l,l-1]^T,
+//       one tcgen05 GEMM per layer whose K grows by r_pad each layer, SiLU in its epilogue;
+//   (3) dv_accum_kernel: per 128-token block and hidden slice, M_l = E + sum_{j<=l} h_j U_j^T
+//       as a running sum in TMEM, bf16 M_l stored for the K/V GEMM with its rows' sums of
+//       squares for the RMS statistic.
+// Only (2) runs layer after layer, and each of its layers is a GEMM of N = r_pad with no
+// exchange between CTAs. The sums differ from the chain's only in rounding (the same products,
+// grouped differently).
+#include "../../include/dv.h"
+#include "dv_internal.h"
+#include "dv_ptx.cuh"
+
+namespace dv {
+
+// ------------------------------------------------------------------------------ kernels
+
+namespace {
+
+constexpr int kFoldThreads = 192;  // warp 0 TMA, warp 1 MMA + TMEM, warps 2-5 epilogue
+constexpr int kEpi = 128;
+constexpr int kSlabA = 128 * 128;  // [128 token rows][64] bf16, 128-byte swizzle
+
+// Byte offset of 16-byte chunk `c` (c < 8) of row `row` in a 128-byte-swizzled slab.
+__device__ __forceinline__ uint32_t swz(int row, int c) {
+  return static_cast<uint32_t>(row * 128 + ((c ^ (row & 7)) << 4));
+}
+
+__device__ __forceinline__ bool wait_only(uint32_t bar, uint32_t parity, uint64_t timeout_ns) {
+  int never = 0;
+  return mbar_wait(bar, parity, &never, timeout_ns);
+}
+
+// Registers -> TMEM: lane i of the warp writes TMEM lane (taddr.lane + i), 32 columns.
+__device__ __forceinline__ void tmem_st32x(uint32_t taddr, const uint32_t (&r)[32]) {
+  asm volatile(
+      "tcgen05.st.sync.aligned.32x32b.x32.b32 [%0],"
+      " {%1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, %16,"
+      " %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31, %32};" ::"r"(
+          taddr),
+      "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7]),
+      "r"(r[8]), "r"(r[9]), "r"(r[10]), "r"(r[11]), "r"(r[12]), "r"(r[13]), "r"(r[14]),
+      "r"(r[15]), "r"(r[16]), "r"(r[17]), "r"(r[18]), "r"(r[19]), "r"(r[20]), "r"(r[21]),
+      "r"(r[22]), "r"(r[23]), "r"(r[24]), "r"(r[25]), "r"(r[26]), "r"(r[27]), "r"(r[28]),
+      "r"(r[29]), "r"(r[30]), "r"(r[31])
+      : "memory");
+}
+
+__device__ __forceinline__ void tma_store_3d_x(const CUtensorMap* map, uint32_t src, int c0, int c1,
+                                               int c2) {
+  asm volatile(
+      "cp.async.bulk.tensor.3d.global.shared::cta.bulk_group [%0, {%2, %3, %4}], [%1];" ::"l"(
+          reinterpret_cast<uint64_t>(map)),
+      "r"(src), "r"(c0), "r"(c1), "r"(c2)
+      : "memory");
+}
+
+// ---------------------------------------------------------------- (2) the h recurrence
+
+// 3-D tiled load of a slab-map box {64 columns, rows, slabs} at (0, row, slab).
+__device__ __forceinline__ void tma_load_slabs(uint32_t dst, const CUtensorMap* map, uint32_t bar,
+                                               int row, int slab) {
+  asm volatile(
+      "cp.async.bulk.tensor.3d.shared::cluster.global.mbarrier::complete_tx::bytes"
+      " [%0], [%1, {%3, %4, %5}], [%2];" ::"r"(dst),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(bar), "r"(0), "r"(row), "r"(slab)
+      : "memory");
+}
+
+template <int RP, int KS, int STAGES>
+struct HCfg {
+  static constexpr int R = RP / 64;              // 64-wide K slabs per r_pad
+  static constexpr int kSlabB = RP * 128;        // [RP rows of Pf][64] bf16
+  static constexpr int kA = KS * kSlabA;         // one box of KS slabs of A
+  static constexpr int kB = KS * kSlabB;         // one box of KS slabs of B
+  static constexpr int kStage = kA + kB;
+  static constexpr int kOffH = STAGES * kStage;  // h_{l-1} as the A operand of layer l's last slabs
+  static constexpr int kEnd = kOffH + R * kSlabA;
+  static constexpr int kSmemBytes = kEnd + 1024 + 256;
+  static constexpr int kTmemCols = 2 * RP <= 128 ? 128 : (2 * RP <= 256 ? 256 : 512);
+  static_assert(kSlabB % 1024 == 0, "stage tiles stay 1024-byte aligned");
+  static_assert(kSmemBytes <= 232448, "shared memory of one CTA");
+};
+
+struct HChainParams {
+  int M;        // tokens
+  int L;        // planned layers
+  uint16_t* H;  // bf16 [M][ldh]: h_l at columns l r_pad
+  int ldh;
+  int* status;
+  unsigned long long timeout_ns;
+};
+
+// Segment `seg` of layer l's K loop: n slabs, the first at slab a0 of its A source and at slab
+// b0 of the layer's rows of Pf. 0: C_l^hi (A: Chi), 1: C_l^lo (A: Clo), 2: h_0 .. h_{l-2}
+// (A: H), 3: h_{l-1} (A: the h tile).
+struct HSeg {
+  int n, a0, b0;
+};
+__device__ __forceinline__ HSeg hseg(int l, int seg, int R) {
+  if (seg == 0) return {R, l * R, 0};
+  if (seg == 1) return {R, l * R, R};
+  if (seg == 2) return {l >= 2 ? (l - 1) * R : 0, 0, 2 * R};
+  return {l >= 1 ? R : 0, 0, (l + 1) * R};
+}
+
+// One CTA per 128-token block, all layers. Layer l's GEMM runs over 2R + l R slabs of 64 in the
+// four segments of hseg: the two bf16 parts of C_l against the identity blocks of Pf, then h_j of
+// every earlier layer against the Q_lj blocks. A pipeline step moves KS consecutive slabs of one
+// segment as one TMA box per operand (a TMA instruction has a fixed cost that one 16 KB slab
+// does not amortise); the last step of a segment uses the slabs it needs of its box (the rest is
+// zero fill or data the MMA does not read). Two TMEM accumulators: the MMAs of layer l over C and
+// the older h_j run while the epilogue of layer l - 1 still works. The epilogue applies SiLU,
+// writes bf16 h_l to the h tile (the A operand of layer l + 1's last segment) and to H (read
+// back by TMA from layer l + 2 on, and by the running sum).
+// Barriers (all waits bounded): stage full / empty; accumulator full / free; the h tile written
+// (once per layer); h_l in global memory, alternating between two barriers by layer parity so
+// that the producer, which may run up to two layers ahead of the epilogue, never waits on a
+// phase that has wrapped.
+template <int RP, int KS, int STAGES>
+__global__ void __launch_bounds__(kFoldThreads, 1)
+    dv_hchain_kernel(const __grid_constant__ CUtensorMap tmChi,
+                     const __grid_constant__ CUtensorMap tmClo,
+                     const __grid_constant__ CUtensorMap tmH, const __grid_constant__ CUtensorMap tmP,
+                     const __grid_constant__ HChainParams p) {
+  using C = HCfg<RP, KS, STAGES>;
+  constexpr int R = C::R;
+  extern __shared__ uint8_t smem_raw[];
+  const uint32_t raw = smem_addr(smem_raw);
+  const uint32_t base = (raw + 1023u) & ~1023u;
+  uint8_t* base_ptr = smem_raw + (base - raw);
+  uint64_t* bars = reinterpret_cast<uint64_t*>(base_ptr + C::kEnd);
+  const uint32_t bar0 = smem_addr(bars);
+  auto full_bar = [&](int s) { return bar0 + 8u * s; };
+  auto empty_bar = [&](int s) { return bar0 + 8u * (STAGES + s); };
+  auto accf_bar = [&](int a) { return bar0 + 8u * (2 * STAGES + a); };
+  auto acce_bar = [&](int a) { return bar0 + 8u * (2 * STAGES + 2 + a); };
+  auto hpub_bar = [&](int a) { return bar0 + 8u * (2 * STAGES + 4 + a); };
+  const uint32_t htile_bar = bar0 + 8u * (2 * STAGES + 6);
+  const uint32_t drain_bar = bar0 + 8u * (2 * STAGES + 7);
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 2 * STAGES + 8);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+  const uint32_t ring = base, htile = base + C::kOffH;
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const uint64_t tmo = p.timeout_ns;
+  const int row0 = blockIdx.x * 128;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < STAGES; ++s) {
+      mbar_init(full_bar(s), 1);
+      mbar_init(empty_bar(s), 1);
+    }
+    for (int a = 0; a < 2; ++a) {
+      mbar_init(accf_bar(a), 1);
+      mbar_init(acce_bar(a), kEpi);
+      mbar_init(hpub_bar(a), kEpi);
+    }
+    mbar_init(htile_bar, kEpi);
+    mbar_init(drain_bar, 1);
+    *abort_flag = 0;
+    fence_barrier_init();
+  }
+  if (warp == 0 && lane == 0) {
+    tma_prefetch_desc(&tmChi);
+    tma_prefetch_desc(&tmClo);
+    tma_prefetch_desc(&tmH);
+    tma_prefetch_desc(&tmP);
+  }
+  if (warp == 1) {
+    tmem_alloc(smem_addr(tmem_slot), C::kTmemCols);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+  pdl_wait();
+  pdl_trigger();
+
+  if (warp == 0) {
+    if (lane == 0) {
+      // ---------------------------------------------------------------- TMA producer
+      int stage = 0;
+      uint32_t phase = 0, used = 0, issued_parity = 0;
+      bool ok = true;
+      for (int l = 0; l < p.L && ok; ++l) {
+        for (int seg = 0; seg < 4 && ok; ++seg) {
+          const HSeg g = hseg(l, seg, R);
+          // h_{l-2} is the newest layer segment 2 reads: wait until it is in global memory (the
+          // layers before it were published earlier)
+          if (seg == 2 && g.n > 0 &&
+              !mbar_wait(hpub_bar((l - 2) & 1), static_cast<uint32_t>((l - 2) >> 1) & 1u, abort_flag,
+                         tmo)) {
+            ok = false;
+            break;
+          }
+          for (int s0 = 0; s0 < g.n; s0 += KS) {
+            if (!mbar_wait(empty_bar(stage), phase ^ 1u, abort_flag, tmo)) {
+              ok = false;
+              break;
+            }
+            const uint32_t a_dst = ring + stage * C::kStage, b_dst = a_dst + C::kA;
+            mbar_arrive_expect_tx(full_bar(stage), seg == 3 ? C::kB : C::kStage);
+            if (seg < 3)
+              tma_load_slabs(a_dst, seg == 0 ? &tmChi : (seg == 1 ? &tmClo : &tmH), full_bar(stage),
+                             row0, g.a0 + s0);
+            tma_load_slabs(b_dst, &tmP, full_bar(stage), l * RP, g.b0 + s0);
+            used |= 1u << stage;
+            issued_parity = (issued_parity & ~(1u << stage)) | (phase << stage);
+            if (++stage == STAGES) {
+              stage = 0;
+              phase ^= 1u;
+            }
+          }
+        }
+      }
+      if (*abort_flag) {  // every copy still in flight lands before the CTA exits
+        for (int s = 0; s < STAGES; ++s)
+          if (used & (1u << s)) wait_only(full_bar(s), (issued_parity >> s) & 1u, tmo);
+      }
+    }
+  } else if (warp == 1) {
+    if (lane == 0) {
+      // ---------------------------------------------------------------- MMA issuer
+      const uint32_t idesc = idesc_bf16_f32(128, RP);
+      int stage = 0, acc = 0;
+      uint32_t phase = 0, acc_phase = 0;
+      bool issued_any = false, ok = true;
+      for (int l = 0; l < p.L && ok; ++l) {
+        if (!mbar_wait(acce_bar(acc), acc_phase ^ 1u, abort_flag, tmo)) break;
+        tc_fence_after();
+        const uint32_t d_tmem = tmem + static_cast<uint32_t>(acc * RP);
+        bool first = true;
+        for (int seg = 0; seg < 4 && ok; ++seg) {
+          const HSeg g = hseg(l, seg, R);
+          if (seg == 3 && g.n > 0 &&
+              !mbar_wait(htile_bar, static_cast<uint32_t>(l - 1) & 1u, abort_flag, tmo)) {
+            ok = false;
+            break;
+          }
+          for (int s0 = 0; s0 < g.n; s0 += KS) {
+            if (!mbar_wait(full_bar(stage), phase, abort_flag, tmo)) {
+              ok = false;
+              break;
+            }
+            tc_fence_after();
+            const uint32_t st = ring + stage * C::kStage;
+            const int n_use = g.n - s0 < KS ? g.n - s0 : KS;
+            for (int u = 0; u < n_use; ++u) {
+              const uint32_t a_s = seg == 3 ? htile + static_cast<uint32_t>((s0 + u) * kSlabA)
+                                            : st + static_cast<uint32_t>(u * kSlabA);
+              const uint32_t b_s = st + C::kA + static_cast<uint32_t>(u * C::kSlabB);
+#pragma unroll
+              for (int k = 0; k < 4; ++k) {
+                umma_bf16(d_tmem, sdesc_kmajor_sw128(a_s + 32u * k), sdesc_kmajor_sw128(b_s + 32u * k),
+                          idesc, first ? 0u : 1u);
+                first = false;
+              }
+            }
+            issued_any = true;
+            umma_commit(empty_bar(stage));
+            if (++stage == STAGES) {
+              stage = 0;
+              phase ^= 1u;
+            }
+          }
+        }
+        if (!ok) break;
+        umma_commit(accf_bar(acc));
+        if (++acc == 2) {
+          acc = 0;
+          acc_phase ^= 1u;
+        }
+      }
+      if (*abort_flag && issued_any) {  // no TMEM release while an MMA may still run
+        umma_commit(drain_bar);
+        wait_only(drain_bar, 0, tmo);
+      }
+    }
+  } else {
+    // ------------------------------------------------------------------ epilogue warps
+    const int qq = warp & 3;  // the TMEM lane quarter this warp may access
+    const int row = qq * 32 + lane;
+    const int t = row0 + row;
+    int acc = 0;
+    uint32_t acc_phase = 0;
+    for (int l = 0; l < p.L; ++l) {
+      if (!__all_sync(0xFFFFFFFFu, mbar_wait(accf_bar(acc), acc_phase, abort_flag, tmo))) break;
+      tc_fence_after();
+      const uint32_t tb =
+          tmem + (static_cast<uint32_t>(qq * 32) << 16) + static_cast<uint32_t>(acc * RP);
+#pragma unroll 1
+      for (int c = 0; c < RP / 32; ++c) {
+        uint32_t r[32], pk[16];
+        __syncwarp();
+        tmem_ld32(tb + c * 32, r);
+        tmem_ld_wait();
+#pragma unroll
+        for (int v = 0; v < 16; ++v)
+          pk[v] = pack_bf16x2(silu(__uint_as_float(r[2 * v])), silu(__uint_as_float(r[2 * v + 1])));
+        uint8_t* slab = base_ptr + C::kOffH + (c / 2) * kSlabA;
+#pragma unroll
+        for (int k = 0; k < 4; ++k)
+          *reinterpret_cast<uint4*>(slab + swz(row, (c % 2) * 4 + k)) =
+              make_uint4(pk[4 * k], pk[4 * k + 1], pk[4 * k + 2], pk[4 * k + 3]);
+      }
+      tc_fence_before();
+      mbar_arrive(acce_bar(acc));
+      // The h tile first (the next layer's MMA waits for it; async proxy), then the copy of h_l
+      // in H (TMA loads two or more layers later, and the running sum): read back from the tile.
+      asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+      mbar_arrive(htile_bar);
+      if (t < p.M) {
+        uint4* hg = reinterpret_cast<uint4*>(p.H + static_cast<long long>(t) * p.ldh + l * RP);
+#pragma unroll 1
+        for (int c8 = 0; c8 < RP / 8; ++c8)
+          hg[c8] = *reinterpret_cast<const uint4*>(base_ptr + C::kOffH + (c8 / 8) * kSlabA +
+                                                   swz(row, c8 % 8));
+      }
+      asm volatile("fence.proxy.async.global;" ::: "memory");
+      mbar_arrive(hpub_bar(l & 1));
+      if (++acc == 2) {
+        acc = 0;
+        acc_phase ^= 1u;
+      }
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  if (threadIdx.x == 0 && *abort_flag) atomicExch(p.status, DV_ERR_DEVICE_TIMEOUT);
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem, C::kTmemCols);
+  }
+}
+
+// ---------------------------------------------------------------- (3) the running sum
+
+template <int RP, int CW, int STAGES>
+struct ACfg {
+  static constexpr int R = RP / 64;
+  static constexpr int NS = CW / 64;              // 64-column slabs of the slice
+  static constexpr int kSlabB = CW * 128;         // [CW rows of U_l][64] bf16
+  static constexpr int kStage = kSlabA + kSlabB;
+  static constexpr int kOffOut = STAGES * kStage; // bf16 M_l of the slice, staged for TMA stores
+  static constexpr int kEnd = kOffOut + NS * kSlabA;
+  static constexpr int kSmemBytes = kEnd + 1024 + 256;
+  static constexpr int kTmemCols = CW <= 64 ? 64 : (CW <= 128 ? 128 : 256);
+  static_assert(kSlabB % 1024 == 0, "stage tiles stay 1024-byte aligned");
+  static_assert(kSmemBytes <= 232448, "shared memory of one CTA");
+};
+
+struct AccumParams {
+  int M;               // tokens
+  int L;               // planned layers
+  int d;
+  int S;               // hidden slices (d / CW)
+  const uint16_t* x0;  // bf16 [M][d]
+  float* part;         // fp32 [L][part_ld / M][M]: sums of squares of M_l per slice
+  long long part_ld;
+  int* status;
+  unsigned long long timeout_ns;
+};
+
+// CTA (block b, slice s) of the grid b * S + s: 128 token rows, hidden columns [s CW, (s+1) CW).
+// The accumulator starts as the fp32 widening of E's slice (tcgen05.st); layer l adds
+// h_l U_l^T (K = r_pad) and is read back: bf16 M_l to the stacked memories (TMA store through
+// the staging slabs) and the row's sum of M_l^2 over the slice to part. The next layer's MMA
+// waits until the readback has left TMEM, and runs while the stores go out.
+template <int RP, int CW, int STAGES>
+__global__ void __launch_bounds__(kFoldThreads, 1)
+    dv_accum_kernel(const __grid_constant__ CUtensorMap tmH, const __grid_constant__ CUtensorMap tmU,
+                    const __grid_constant__ CUtensorMap tmM, const __grid_constant__ AccumParams p) {
+  using C = ACfg<RP, CW, STAGES>;
+  constexpr int R = C::R;
+  extern __shared__ uint8_t smem_raw[];
+  const uint32_t raw = smem_addr(smem_raw);
+  const uint32_t base = (raw + 1023u) & ~1023u;
+  uint8_t* base_ptr = smem_raw + (base - raw);
+  uint64_t* bars = reinterpret_cast<uint64_t*>(base_ptr + C::kEnd);
+  const uint32_t bar0 = smem_addr(bars);
+  auto full_bar = [&](int s) { return bar0 + 8u * s; };
+  auto empty_bar = [&](int s) { return bar0 + 8u * (STAGES + s); };
+  const uint32_t accf_bar = bar0 + 8u * (2 * STAGES);
+  const uint32_t accr_bar = bar0 + 8u * (2 * STAGES + 1);
+  const uint32_t drain_bar = bar0 + 8u * (2 * STAGES + 2);
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 2 * STAGES + 3);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+  const uint32_t ring = base, out = base + C::kOffOut;
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const uint64_t tmo = p.timeout_ns;
+  const int blk = blockIdx.x / p.S, sl = blockIdx.x % p.S;
+  const int row0 = blk * 128, col0 = sl * CW;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < STAGES; ++s) {
+      mbar_init(full_bar(s), 1);
+      mbar_init(empty_bar(s), 1);
+    }
+    mbar_init(accf_bar, 1);
+    mbar_init(accr_bar, kEpi);
+    mbar_init(drain_bar, 1);
+    *abort_flag = 0;
+    fence_barrier_init();
+  }
+  if (warp == 0 && lane == 0) {
+    tma_prefetch_desc(&tmH);
+    tma_prefetch_desc(&tmU);
+    tma_prefetch_desc(&tmM);
+  }
+  if (warp == 1) {
+    tmem_alloc(smem_addr(tmem_slot), C::kTmemCols);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+  pdl_wait();
+  pdl_trigger();
+
+  if (warp == 0) {
+    if (lane == 0) {
+      // ---------------------------------------------------------------- TMA producer
+      int stage = 0;
+      uint32_t phase = 0, used = 0, issued_parity = 0;
+      bool ok = true;
+      for (int l = 0; l < p.L && ok; ++l) {
+        for (int q = 0; q < R; ++q) {
+          if (!mbar_wait(empty_bar(stage), phase ^ 1u, abort_flag, tmo)) {
+            ok = false;
+            break;
+          }
+          const uint32_t a_dst = ring + stage * C::kStage, b_dst = a_dst + kSlabA;
+          mbar_arrive_expect_tx(full_bar(stage), C::kStage);
+          tma_load_2d(a_dst, &tmH, full_bar(stage), l * RP + 64 * q, row0);
+          tma_load_2d(b_dst, &tmU, full_bar(stage), 64 * q, l * p.d + col0);
+          used |= 1u << stage;
+          issued_parity = (issued_parity & ~(1u << stage)) | (phase << stage);
+          if (++stage == STAGES) {
+            stage = 0;
+            phase ^= 1u;
+          }
+        }
+      }
+      if (*abort_flag) {
+        for (int s = 0; s < STAGES; ++s)
+          if (used & (1u << s)) wait_only(full_bar(s), (issued_parity >> s) & 1u, tmo);
+      }
+    }
+  } else if (warp == 1) {
+    if (lane == 0) {
+      // ---------------------------------------------------------------- MMA issuer
+      const uint32_t idesc = idesc_bf16_f32(128, CW);
+      int stage = 0;
+      uint32_t phase = 0;
+      bool issued_any = false, ok = true;
+      for (int l = 0; l < p.L && ok; ++l) {
+        // the accumulator holds E (l = 0) or M_{l-1}, and its readback has left TMEM
+        if (!mbar_wait(accr_bar, static_cast<uint32_t>(l) & 1u, abort_flag, tmo)) break;
+        tc_fence_after();
+        for (int q = 0; q < R; ++q) {
+          if (!mbar_wait(full_bar(stage), phase, abort_flag, tmo)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t a_s = ring + stage * C::kStage, b_s = a_s + kSlabA;
+#pragma unroll
+          for (int k = 0; k < 4; ++k)
+            umma_bf16(tmem, sdesc_kmajor_sw128(a_s + 32u * k), sdesc_kmajor_sw128(b_s + 32u * k),
+                      idesc, 1u);
+          issued_any = true;
+          umma_commit(empty_bar(stage));
+          if (++stage == STAGES) {
+            stage = 0;
+            phase ^= 1u;
+          }
+        }
+        if (!ok) break;
+        umma_commit(accf_bar);
+      }
+      if (*abort_flag && issued_any) {
+        umma_commit(drain_bar);
+        wait_only(drain_bar, 0, tmo);
+      }
+    }
+  } else {
+    // ------------------------------------------------------------------ epilogue warps
+    const int qq = warp & 3;
+    const int row = qq * 32 + lane;
+    const int t = row0 + row;
+    const bool issuer = warp == 2 && lane == 0;  // issues the stores of the slice
+    const uint32_t tb = tmem + (static_cast<uint32_t>(qq * 32) << 16);
+    // M_0 = E: the fp32 widening of this row's slice of E into the accumulator
+    {
+      const uint16_t* xr = p.x0 + static_cast<long long>(t) * p.d + col0;
+#pragma unroll 1
+      for (int c = 0; c < CW / 32; ++c) {
+        uint32_t r[32];
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+          const uint4 w = t < p.M ? reinterpret_cast<const uint4*>(xr + c * 32)[k] : make_uint4(0, 0, 0, 0);
+          const uint32_t ws[4] = {w.x, w.y, w.z, w.w};
+#pragma unroll
+          for (int e = 0; e < 4; ++e) {
+            r[k * 8 + 2 * e] = ws[e] << 16;
+            r[k * 8 + 2 * e + 1] = ws[e] & 0xFFFF0000u;
+          }
+        }
+        __syncwarp();
+        tmem_st32x(tb + c * 32, r);
+      }
+      asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
+      tc_fence_before();
+      mbar_arrive(accr_bar);
+    }
+    for (int l = 0; l < p.L; ++l) {
+      bool ok = __all_sync(0xFFFFFFFFu, mbar_wait(accf_bar, static_cast<uint32_t>(l) & 1u, abort_flag, tmo));
+      // the staging slabs are free once the previous layer's stores have read them
+      if (issuer && l > 0) asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory");
+      ok = named_barrier_and(1, kEpi, ok);
+      if (!ok) break;
+      tc_fence_after();
+      float ss = 0.0f;
+#pragma unroll 1
+      for (int c = 0; c < CW / 32; ++c) {
+        uint32_t r[32], pk[16];
+        __syncwarp();
+        tmem_ld32(tb + c * 32, r);
+        tmem_ld_wait();
+#pragma unroll
+        for (int v = 0; v < 16; ++v) {
+          const float a = __uint_as_float(r[2 * v]), b = __uint_as_float(r[2 * v + 1]);
+          ss = fmaf(a, a, ss);
+          ss = fmaf(b, b, ss);
+          pk[v] = pack_bf16x2(a, b);
+        }
+        uint8_t* slab = base_ptr + C::kOffOut + (c / 2) * kSlabA;
+#pragma unroll
+        for (int k = 0; k < 4; ++k)
+          *reinterpret_cast<uint4*>(slab + swz(row, (c % 2) * 4 + k)) =
+              make_uint4(pk[4 * k], pk[4 * k + 1], pk[4 * k + 2], pk[4 * k + 3]);
+      }
+      tc_fence_before();
+      mbar_arrive(accr_bar);  // the readback has left TMEM: the next layer may accumulate
+      if (t < p.M) p.part[l * p.part_ld + static_cast<long long>(sl) * p.M + t] = ss;
+      asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+      named_barrier(1, kEpi);
+      if (issuer) {
+        for (int j = 0; j < C::NS; ++j)
+          tma_store_3d_x(&tmM, out + static_cast<uint32_t>(j * kSlabA), col0 + 64 * j, row0, l);
+        asm volatile("cp.async.bulk.commit_group;" ::: "memory");
+      }
+    }
+    if (issuer) asm volatile("cp.async.bulk.wait_group 0;" ::: "memory");
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  if (threadIdx.x == 0 && *abort_flag) atomicExch(p.status, DV_ERR_DEVICE_TIMEOUT);
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem, C::kTmemCols);
+  }
+}
+
+template <int RP, int KS, int ST>
+cudaError_t hchain_t(long long blocks, const CUtensorMap& chi, const CUtensorMap& clo,
+                     const CUtensorMap& h, const CUtensorMap& pf, const HChainParams& p,
+                     cudaStream_t stream) {
+  using C = HCfg<RP, KS, ST>;
+  auto kern = dv_hchain_kernel<RP, KS, ST>;
+  cudaError_t err = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, C::kSmemBytes);
+  if (err != cudaSuccess || blocks <= 0) return err;
+  cudaLaunchConfig_t cfg = {};
+  cudaLaunchAttribute attr[1] = {pdl_attribute()};
+  cfg.gridDim = dim3(static_cast<unsigned>(blocks), 1, 1);
+  cfg.blockDim = dim3(kFoldThreads, 1, 1);
+  cfg.dynamicSmemBytes = C::kSmemBytes;
+  cfg.stream = stream;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  err = cudaLaunchKernelEx(&cfg, kern, chi, clo, h, pf, p);
+  if (err != cudaSuccess) return err;
+  return cudaGetLastError();
+}
+
+template <int RP, int CW, int ST>
+cudaError_t accum_t(long long ctas, const CUtensorMap& h, const CUtensorMap& u,
+                    const CUtensorMap& m3, const AccumParams& p, cudaStream_t stream) {
+  using C = ACfg<RP, CW, ST>;
+  auto kern = dv_accum_kernel<RP, CW, ST>;
+  cudaError_t err = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, C::kSmemBytes);
+  if (err != cudaSuccess || ctas <= 0) return err;
+  cudaLaunchConfig_t cfg = {};
+  cudaLaunchAttribute attr[1] = {pdl_attribute()};
+  cfg.gridDim = dim3(static_cast<unsigned>(ctas), 1, 1);
+  cfg.blockDim = dim3(kFoldThreads, 1, 1);
+  cfg.dynamicSmemBytes = C::kSmemBytes;
+  cfg.stream = stream;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  err = cudaLaunchKernelEx(&cfg, kern, h, u, m3, p);
+  if (err != cudaSuccess) return err;
+  return cudaGetLastError();
+}
+
+}  // namespace
+
+int hchain_box_slabs(int r_pad) { return r_pad == 256 ? 1 : 2; }
+
+// 128 columns per CTA: with two pipeline stages a CTA takes under half of an SM's shared memory
+// and TMEM, so two run on each SM and one's loads and readback hide behind the other's work.
+int fold_slice_cols(int d) {
+  for (int cw : {128, 64})
+    if (d % cw == 0) return cw;
+  return 0;
+}
+
+cudaError_t launch_hchain(int r_pad, long long tokens, int n_layers, const CUtensorMap& chi,
+                          const CUtensorMap& clo, const CUtensorMap& h, const CUtensorMap& pf,
+                          uint16_t* H, int ldh, int* status, unsigned long long timeout_ns,
+                          cudaStream_t stream) {
+  HChainParams p;
+  p.M = static_cast<int>(tokens);
+  p.L = n_layers;
+  p.H = H;
+  p.ldh = ldh;
+  p.status = status;
+  p.timeout_ns = timeout_ns;
+  const long long blocks = (tokens + 127) / 128;
+  switch (r_pad) {  // slabs per box (hchain_box_slabs) and pipeline stages
+    case 64: return hchain_t<64, 2, 4>(blocks, chi, clo, h, pf, p, stream);
+    case 128: return hchain_t<128, 2, 3>(blocks, chi, clo, h, pf, p, stream);
+    case 192: return hchain_t<192, 2, 2>(blocks, chi, clo, h, pf, p, stream);
+    case 256: return hchain_t<256, 1, 3>(blocks, chi, clo, h, pf, p, stream);
+    default: return cudaErrorInvalidValue;
+  }
+}
+
+cudaError_t launch_accum(int r_pad, int cw, long long tokens, int n_layers, int d,
+                         const void* x0, const CUtensorMap& h, const CUtensorMap& u,
+                         const CUtensorMap& m3, float* part, long long part_ld, int* status,
+                         unsigned long long timeout_ns, cudaStream_t stream) {
+  AccumParams p;
+  p.M = static_cast<int>(tokens);
+  p.L = n_layers;
+  p.d = d;
+  p.S = d / cw;
+  p.x0 = static_cast<const uint16_t*>(x0);
+  p.part = part;
+  p.part_ld = part_ld;
+  p.status = status;
+  p.timeout_ns = timeout_ns;
+  const long long ctas = (tokens + 127) / 128 * p.S;
+#define DV_ACCUM(RPV, CWV, STV) \
+  if (r_pad == RPV && cw == CWV) return accum_t<RPV, CWV, STV>(ctas, h, u, m3, p, stream);
+  DV_ACCUM(64, 256, 3) DV_ACCUM(64, 128, 2) DV_ACCUM(64, 64, 2)
+  DV_ACCUM(128, 256, 3) DV_ACCUM(128, 128, 2) DV_ACCUM(128, 64, 2)
+  DV_ACCUM(192, 256, 3) DV_ACCUM(192, 128, 2) DV_ACCUM(192, 64, 2)
+  DV_ACCUM(256, 256, 3) DV_ACCUM(256, 128, 2) DV_ACCUM(256, 64, 2)
+#undef DV_ACCUM
+  return cudaErrorInvalidValue;
+}
+
+}  // namespace dv

@@ -74,13 +74,17 @@ __host__ __device__ inline KStep k_step(int j, int k0_slabs, int k1_slabs) {
 }
 
 // Columns [0, n_h) of the product are down-projections: H = bf16(SiLU(acc)). Columns from n_h
-// on (x0 (2 U_l)^T when the statistic of M_l is formed outside a GEMM) go to C as fp32.
+// on (x0 (2 U_l)^T when the statistic of M_l is formed outside a GEMM) go to C as fp32, or,
+// when Chi is set (the recurrent adapter's E D_l^T), as two bf16 parts hi = bf16(acc) into Chi
+// and lo = bf16(acc - hi) into Clo, both [M][ldc].
 struct EpiSilu {
   uint16_t* H;   // bf16 [M][ldh]
   int ldh;
   int n_h;       // columns that are down-projections
   float* C;      // fp32 [M][ldc] or null
   int ldc;
+  uint16_t* Chi;
+  uint16_t* Clo;
 };
 
 // Launch attribute of the build's kernels: programmatic stream serialization (see pdl_wait in
@@ -216,11 +220,38 @@ int down_splits(long long m_tiles, int k_slabs, int num_sms);
 // x: x0 (128-row boxes); dmap: stacked D (r_pad-row boxes); umap: U as [L d][r_pad] (64 spc-row
 // boxes); mmap: the stacked M_l as a 3-D (d, tokens, L) map with (64, 128, 1) boxes.
 bool chain_shape(int d, int r_pad, int* spc_out, int* s_out);
+// Clusters of the on-chip chain that can be resident at once on the current device (0: the
+// chain does not fit or does not apply).
+int chain_resident_clusters(int d, int r_pad, bool split);
 cudaError_t launch_chain(int r_pad, int spc, int S, long long tokens, int n_layers, int d,
                          const CUtensorMap& x, const CUtensorMap& dmap, const CUtensorMap& umap,
                          const CUtensorMap& mmap, float* part, long long part_ld, uint16_t* H,
                          int* status, unsigned long long timeout_ns, cudaStream_t stream,
                          bool split);
+
+// The recurrent adapter by the refactored chain (dv_fold.cu). With C = E [D_1 .. D_L]^T given as
+// two bf16 parts (Chi, Clo: [tokens][L r_pad]) and the plan's Pf ([L r_pad][(L + 2) r_pad]:
+// identity blocks, then Q_lj = D_l U_j):
+//   launch_hchain: h_l = SiLU(C_l + sum_{j<l} h_j Q_lj^T) into H ([tokens][ldh], h_l at columns
+//     l r_pad), one CTA per 128-token block. Maps: chi, clo, h: slab maps over [tokens][L r_pad]
+//     with 128-row boxes; pf: slab map over Pf with r_pad-row boxes.
+//   launch_accum: M_l = E + sum_{j<=l} h_j U_j^T, bf16 into the stacked memories (m3: the 3-D
+//     (d, tokens, L) map with (64, 128, 1) boxes) and each row's sum of M_l^2 over each slice of
+//     cw hidden columns into part (d / cw partials per layer). u: U as [L d][r_pad] with cw-row
+//     boxes; x0: E, bf16 [tokens][d].
+// fold_slice_cols: the slice width cw (256, 192, 128 or 64 dividing d), or 0.
+// hchain_box_slabs: K slabs per TMA box of launch_hchain's maps (chi, clo, h and pf are slab maps,
+// encode_slabs, with boxes of that many slabs).
+int fold_slice_cols(int d);
+int hchain_box_slabs(int r_pad);
+cudaError_t launch_hchain(int r_pad, long long tokens, int n_layers, const CUtensorMap& chi,
+                          const CUtensorMap& clo, const CUtensorMap& h, const CUtensorMap& pf,
+                          uint16_t* H, int ldh, int* status, unsigned long long timeout_ns,
+                          cudaStream_t stream);
+cudaError_t launch_accum(int r_pad, int cw, long long tokens, int n_layers, int d,
+                         const void* x0, const CUtensorMap& h, const CUtensorMap& u,
+                         const CUtensorMap& m3, float* part, long long part_ld, int* status,
+                         unsigned long long timeout_ns, cudaStream_t stream);
 
 // Token tile (64, 128, 192 or 256) of the pair kernel for a build of `tokens` tokens.
 int kv_pair_tile_n(long long tokens);
@@ -254,6 +285,8 @@ struct PlanView {
   int dst_ld;
   const CUtensorMap* tm_Uup;       // recurrent: [L*d][r_pad], boxes of resid_bn rows
   const uint16_t* Uup;             // recurrent: U_l as [L*d][r_pad] ([U_l | U_l] when split)
+  const CUtensorMap* tm_Pf;        // recurrent, refactored chain: Pf with r_pad-row boxes, or null
+  int chain_clusters;              // recurrent: resident clusters of the on-chip chain (0: none)
   int split_chain;                 // recurrent: hi + lo bf16 operands in the chain's GEMMs
   int uup_ld;                      // row pitch of Uup: r_pad, or 2 r_pad with the split chain
   int resid_bn;                    // recurrent: column tile of the up-projection step
@@ -295,6 +328,8 @@ struct BuildArgs {
   float* part;          // recurrent: fp32 [L][d / 64][tokens]
   uint16_t* Hlo;        // split chain: low bf16 parts of h, [tokens][L * r_pad]
   uint16_t* mem_lo;     // split chain: low bf16 part of the last M_l, [tokens][d]
+  uint16_t* Chi;        // recurrent, refactored chain: E D_l^T as bf16 hi / lo parts,
+  uint16_t* Clo;        //   [tokens][L * r_pad] each
   cudaEvent_t* marks;   // 5 events around the 4 stages, or null
 };
 
