@@ -95,7 +95,11 @@ typedef struct dv_config {
                             product, so the state M_l keeps about fp32 accuracy through deep
                             chains; the chain then runs on chip only at rank <= 64 (where
                             the on-chip chain fits d at all), else as per-layer launches.
-                            0 = one bf16 operand (faster). */
+                            0 = one bf16 operand (faster): builds whose 128-token blocks fit in
+                            one wave of on-chip chain clusters run the chain, larger ones (and
+                            every build at rank > 128) the rearranged chain, which forms each
+                            layer's down-projection input from E D_l^T and the earlier h_j
+                            through the r x r products D_l U_j (exactly the same sum). */
 } dv_config;
 
 /* Weights of all L layers, bf16, device pointers. Read only during dv_memory_plan: the plan
@@ -159,8 +163,8 @@ int dv_memory_plan(const dv_config* cfg, const dv_weights* w, void* stream, dv_p
 /*
  * dv_build_visual_memory — the hot path. For batch*n_vis visual tokens writes K^v_l and V^v_l
  * of every layer (Sec. 3.1 Eqs. 4-6, Sec. 3.2 Eq. 7) into the cache. With the recurrent
- * adapter the state M_l is carried in fp32 from layer to layer; each layer's K/V read its
- * bf16 rounding.
+ * adapter the state M_l is carried in fp32 from layer to layer (on chip, or as the running sum
+ * E + sum_{j<=l} h_j U_j^T of the rearranged chain); each layer's K/V read its bf16 rounding.
  *   x0     bf16 [batch][n_vis][d]: the visual embeddings E (Sec. 2 Eq. 1); 16-byte aligned
  *   pos    int32 [batch][P][n_vis], P = 1 (DV_ROPE_1D) or 3 (M-RoPE modes: t, h, w): the
  *          original positions of the visual tokens (Sec. 1 and App. H keep them unchanged)
@@ -193,9 +197,11 @@ int dv_build_visual_memory(dv_plan* plan, const void* x0, int batch, int n_vis, 
  *                          every layer, RMS statistics, row sums, a copy of E), plus
  *                          T * L * r_pad * 4 when r_pad = 64 (the fp32 x0 (2 U_l)^T of the
  *                          small-token path);
- *       recurrent adapter  T * (L * r_pad * 2 + L * 4 + 4 + 4 d + L * (2 d + 4 d / 64)) bytes
- *                          (h, RMS statistics, fp32 state, bf16 M_l of every layer, partial
- *                          sums of squares), plus T * (L * r_pad + d) * 2 with split_chain.
+ *       recurrent adapter  T * (L * r_pad * 2 + L * 4 + 4 + L * (2 d + 4 d / 64)) bytes
+ *                          (h, RMS statistics, bf16 M_l of every layer, partial sums of
+ *                          squares), plus T * L * r_pad * 4 (the fp32 E D_l^T of the
+ *                          rearranged chain) without split_chain, or T * 4 d (the fp32 state)
+ *                          and T * (L * r_pad + d) * 2 with it.
  *     Larger builds return DV_ERR_UNSUPPORTED_SHAPE and launch nothing.
  *   - dv_memory_plan reserves the array on the plan's device (CUDA loads the module that
  *     holds it when the plan looks up its address) and loads every kernel a build can launch,
@@ -313,14 +319,15 @@ const char* dv_error_string(int status);
  *   dv_timing_read(plan, ms, n_stages, n_builds) synchronises on the recorded events and
  *   writes the summed milliseconds of each stage into ms[0..n_stages-1] (stage order:
  *   0 stacked down-projection + SiLU, 1 row sums of squares of E, 2 RMS statistics,
- *   3 K/V projection + RoPE + cache store; recurrent adapter: 0 empty, 1 the adapter chain
- *   through all layers, 2 RMS statistics from the chain's partial sums, 3 as above) and the
- *   number of builds into *n_builds.
+ *   3 K/V projection + RoPE + cache store; recurrent adapter: 0 E D^T of every layer (empty
+ *   when the on-chip chain runs), 1 the adapter chain through all layers, 2 RMS statistics from
+ *   the chain's partial sums, 3 as above) and the number of builds into *n_builds.
  */
 int dv_timing_enable(dv_plan* plan, int on);
 int dv_timing_read(dv_plan* plan, double* ms, int n_stages, int* n_builds);
 
-/* Number of kernels one build launches (for launch accounting). */
+/* Number of kernels one build of the plan's full size (max_batch x max_n_vis tokens) launches
+ * (for launch accounting). */
 int dv_kernels_per_build(const dv_plan* plan);
 
 /* Which kernel computes K/V (Sec. 3.2 Eq. 7) in a build of `tokens` tokens, for reporting:

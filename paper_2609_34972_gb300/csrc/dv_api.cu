@@ -39,8 +39,8 @@ struct dv_plan {
   uint16_t* Bn = nullptr;
   uint16_t* Wkv = nullptr;
   uint16_t* Uup = nullptr;     // recurrent adapter: U_l as [L*d][uup_ld] (split chain: [U_l | U_l])
-  uint16_t* Pf = nullptr;      // recurrent adapter, refactored chain: [L*r_pad][(L+2)*r_pad]
-                               // (k_fold_identity, k_fold_products), or null
+  uint16_t* Pf = nullptr;      // recurrent adapter, refactored chain: [L*r_pad][L*r_pad]
+                               // (k_fold_products), or null
   bool fold = false;           // recurrent builds may run the refactored chain (dv_fold.cu)
   int chain_clusters = 0;      // recurrent: clusters of the on-chip chain resident at once
   int uup_ld = 0;              // r_pad, or 2 r_pad with the split chain
@@ -356,24 +356,9 @@ __global__ void k_bias_to_f32(const uint16_t* __restrict__ b, float* __restrict_
     out[e] = bf(b[static_cast<long long>(pl.src[e / kv]) * kv + e % kv]);
 }
 
-// Recurrent adapter, refactored chain (dv_fold.cu). Pf [L r_pad][pld], pld = (L + 2) r_pad:
-// row i r_pad + a holds, for planned layer i,
-//   columns [0, r_pad) and [r_pad, 2 r_pad): 1 at column a (the identity blocks that add the two
-//   bf16 parts of C_i in the recurrence GEMM);
-//   columns (2 + j) r_pad + b, j < i: bf16 of Q_ij[a][b] = sum_e D_i[a][e] U_j[e][b] (a, b < r;
-//   zero where layer i or j is an identity layer);
-//   everything else 0.
-// The identity entries; the rest is zeroed by the caller before k_fold_products.
-__global__ void k_fold_identity(uint16_t* __restrict__ Pf, int L, int r_pad, long long pld) {
-  const long long n = static_cast<long long>(L) * r_pad;
-  for (long long row = blockIdx.x * static_cast<long long>(blockDim.x) + threadIdx.x; row < n;
-       row += static_cast<long long>(gridDim.x) * blockDim.x) {
-    const int a = static_cast<int>(row % r_pad);
-    Pf[row * pld + a] = 0x3F80;          // 1.0
-    Pf[row * pld + r_pad + a] = 0x3F80;
-  }
-}
-
+// Recurrent adapter, refactored chain (dv_fold.cu). Pf [L r_pad][L r_pad]: row i r_pad + a,
+// columns j r_pad + b with j < i hold bf16 of Q_ij[a][b] = sum_e D_i[a][e] U_j[e][b] (a, b < r;
+// zero where layer i or j is an identity layer); the caller zeroes the rest.
 // Q_ij blocks: grid (r_pad / 64 b-tiles, (L) * (r_pad / 64) (j, a-tile), L (i)); blocks with
 // j >= i return. 64 x 64 outputs per block, 256 threads with 4 x 4 each, fp32 accumulation
 // over e in steps of 32 (a fixed order).
@@ -422,7 +407,7 @@ __global__ void __launch_bounds__(256) k_fold_products(const uint16_t* __restric
     const long long row = static_cast<long long>(i) * r_pad + a0 + ty * 4 + q;
 #pragma unroll
     for (int w = 0; w < 4; ++w)
-      Pf[row * pld + static_cast<long long>(2 + j) * r_pad + b0 + tx * 4 + w] = to_bf16(acc[q][w]);
+      Pf[row * pld + static_cast<long long>(j) * r_pad + b0 + tx * 4 + w] = to_bf16(acc[q][w]);
   }
 }
 
@@ -831,8 +816,8 @@ static bool fold_build(const PlanView& v, long long tokens) {
   return uses_fold(v) && (tokens + kBlockM - 1) / kBlockM > v.chain_clusters;
 }
 
-// Recurrent adapter by the refactored chain (dv_fold.cu): (1) C = E [D_1 .. D_L]^T as two bf16
-// parts, one GEMM on the engine the embedding adapter's down-projection would use; (2) the
+// Recurrent adapter by the refactored chain (dv_fold.cu): (1) C = E [D_1 .. D_L]^T in fp32, one
+// GEMM on the engine the embedding adapter's down-projection would use; (2) the
 // recurrence h_l = SiLU(C_l + sum_{j<l} h_j Q_lj^T) per 128-token block; (3) the running sum
 // M_l = E + sum_{j<=l} h_j U_j^T with the rows' sums of squares; then the RMS statistics and one
 // K/V launch over all layers, as in the chain below.
@@ -845,26 +830,23 @@ static cudaError_t enqueue_fold(const PlanView& v, const BuildArgs& a, cudaStrea
     if (a.marks) cudaEventRecord(a.marks[i], st);
   };
   const uint32_t ks = static_cast<uint32_t>(hchain_box_slabs(v.r_pad));
-  CUtensorMap tm_x0, tm_x0_s, tm_chi, tm_clo, tm_hs, tm_h, tm_u, tm_m3, tm_mem_s;
+  CUtensorMap tm_x0, tm_x0_s, tm_hs, tm_h, tm_u, tm_mem_s;
   if (!encode_2d(&tm_x0, a.x0, d, static_cast<uint64_t>(T), d, kBlockM) ||
       !encode_slabs(&tm_x0_s, a.x0, d, static_cast<uint64_t>(T), d, kBlockM) ||
-      !encode_slabs(&tm_chi, a.Chi, n1, static_cast<uint64_t>(T), n1, kBlockM, ks) ||
-      !encode_slabs(&tm_clo, a.Clo, n1, static_cast<uint64_t>(T), n1, kBlockM, ks) ||
       !encode_slabs(&tm_hs, a.H, n1, static_cast<uint64_t>(T), a.hld, kBlockM, ks) ||
       !encode_2d(&tm_h, a.H, n1, static_cast<uint64_t>(T), a.hld, kBlockM) ||
       !encode_2d(&tm_u, v.Uup, v.r_pad, static_cast<uint64_t>(L) * d, v.uup_ld, cw) ||
-      !encode_3d(&tm_m3, a.mem, d, static_cast<uint64_t>(T), L, kBlockM) ||
       !encode_slabs(&tm_mem_s, a.mem, d, static_cast<uint64_t>(L) * T, d, kBlockM))
     return cudaErrorInvalidValue;
   mark(0);
-  // (1) C = E [D_1 .. D_L]^T, every column into the two bf16 parts
+  // (1) C = E [D_1 .. D_L]^T, every column in fp32
   GemmParams gp;
   std::memset(&gp, 0, sizeof(gp));
   gp.status = v.status;
   gp.timeout_ns = kTimeoutNs;
   for (int i = 0; i < L; ++i) gp.layer_map[i] = v.active[i];
   gp.s = {static_cast<int>(T), 1, static_cast<int>(n1), d / 64, 0, 0, 0, 0, 0, 0};
-  gp.silu = {nullptr, 0, 0, nullptr, static_cast<int>(n1), a.Chi, a.Clo};
+  gp.silu = {nullptr, 0, 0, a.c, static_cast<int>(n1)};
   const long long pad128 = (T + 127) / 128 * 128, pad256 = (T + 255) / 256 * 256;
   cudaError_t err;
   if (prefer_256(pad256, pad128)) {
@@ -892,10 +874,10 @@ static cudaError_t enqueue_fold(const PlanView& v, const BuildArgs& a, cudaStrea
   // (2) the recurrence over the rank-r vectors, (3) the running sum of the memories
   const long long part_ld = static_cast<long long>(d / 64) * T;
   if (err == cudaSuccess)
-    err = launch_hchain(v.r_pad, T, L, tm_chi, tm_clo, tm_hs, *v.tm_Pf, a.H, static_cast<int>(a.hld),
-                        v.status, kTimeoutNs, st);
+    err = launch_hchain(v.r_pad, T, L, a.c, static_cast<int>(n1), tm_hs, *v.tm_Pf, a.H,
+                        static_cast<int>(a.hld), v.status, kTimeoutNs, st);
   if (err == cudaSuccess)
-    err = launch_accum(v.r_pad, cw, T, L, d, a.x0, tm_h, tm_u, tm_m3, a.part, part_ld, v.status,
+    err = launch_accum(v.r_pad, cw, T, L, d, a.x0, tm_h, tm_u, a.mem, a.part, part_ld, v.status,
                        kTimeoutNs, st);
   mark(2);
   if (err == cudaSuccess)
@@ -1165,18 +1147,15 @@ size_t carve_workspace(const PlanView& v, long long T, void* base, BuildArgs* a)
   const size_t hld = L * v.r_pad + (rec ? 0 : 64), xld = d + 64;
   const size_t oH = take(t * hld * 2), oR = take(L * t * 4), oX = take(t * 4);
   const size_t oXp = rec ? 0 : take(t * xld * 2);
-  size_t oS = 0, oM = 0, oP = 0, oC = 0, oHl = 0, oMl = 0, oChi = 0, oClo = 0;
-  const bool small_path = !rec && v.r_pad == 64;  // x0 (2 U_l)^T in fp32 (see enqueue_build)
-  if (small_path) oC = take(t * L * v.r_pad * 4);
-  // recurrent adapter: E D_l^T in two bf16 parts for the refactored chain, else the fp32 state
+  size_t oS = 0, oM = 0, oP = 0, oC = 0, oHl = 0, oMl = 0;
+  // fp32 [tokens][L r_pad]: x0 (2 U_l)^T of the embedding adapter at small token counts (see
+  // enqueue_build), or E D_l^T of the recurrent adapter's refactored chain, which needs no fp32
+  // state
   const bool fold = rec && uses_fold(v);
+  const bool small_path = !rec && v.r_pad == 64;
+  if (small_path || fold) oC = take(t * L * v.r_pad * 4);
   if (rec) {
-    if (fold) {
-      oChi = take(t * L * v.r_pad * 2);
-      oClo = take(t * L * v.r_pad * 2);
-    } else {
-      oS = take(t * d * 4);
-    }
+    if (!fold) oS = take(t * d * 4);
     oM = take(L * t * d * 2);
     oP = take(L * (d / 64) * t * 4);
     if (v.split_chain) {  // low bf16 parts of h_l (every layer) and of the last M_l
@@ -1193,11 +1172,9 @@ size_t carve_workspace(const PlanView& v, long long T, void* base, BuildArgs* a)
     a->rstd = reinterpret_cast<float*>(b + oR);
     a->xx = reinterpret_cast<float*>(b + oX);
     a->state = rec && !fold ? reinterpret_cast<float*>(b + oS) : nullptr;
-    a->Chi = fold ? reinterpret_cast<uint16_t*>(b + oChi) : nullptr;
-    a->Clo = fold ? reinterpret_cast<uint16_t*>(b + oClo) : nullptr;
     a->mem = rec ? reinterpret_cast<uint16_t*>(b + oM) : nullptr;
     a->part = rec ? reinterpret_cast<float*>(b + oP) : nullptr;
-    a->c = small_path ? reinterpret_cast<float*>(b + oC) : nullptr;
+    a->c = small_path || fold ? reinterpret_cast<float*>(b + oC) : nullptr;
     const bool split = rec && v.split_chain;
     a->Hlo = split ? reinterpret_cast<uint16_t*>(b + oHl) : nullptr;
     a->mem_lo = split ? reinterpret_cast<uint16_t*>(b + oMl) : nullptr;
@@ -1287,9 +1264,9 @@ cudaError_t preload_build_kernels(const dv_plan* p) {
   for (int nt : {64, 128, 192, 256}) keep(dv::launch_kv_pair(hd, nt, m, m, m, gp, 1, nullptr));
   if (p->fold) {
     const int cw = dv::fold_slice_cols(p->cfg.d);
-    keep(dv::launch_hchain(p->r_pad, 0, 1, m, m, m, m, nullptr, 0, nullptr, 0, nullptr));
-    keep(dv::launch_accum(p->r_pad, cw, 0, 1, p->cfg.d, nullptr, m, m, m, nullptr, 0, nullptr, 0,
-                          nullptr));
+    keep(dv::launch_hchain(p->r_pad, 0, 1, nullptr, 0, m, m, nullptr, 0, nullptr, 0, nullptr));
+    keep(dv::launch_accum(p->r_pad, cw, 0, 1, p->cfg.d, nullptr, m, m, nullptr, nullptr, 0, nullptr,
+                          0, nullptr));
   }
   if (p->cfg.adapter == DV_ADAPTER_RECURRENT) {
     dv::DownParams dp;
@@ -1395,7 +1372,7 @@ int dv_memory_plan(const dv_config* cfg, const dv_weights* w, void* stream, dv_p
   // builds whose token blocks fit in one wave of on-chip chain clusters take the chain instead.
   p->fold = rec && !cfg->split_chain && dv::fold_slice_cols(d) > 0;
   p->chain_clusters = rec ? dv::chain_resident_clusters(d, p->r_pad, cfg->split_chain != 0) : 0;
-  const long long pf_ld = static_cast<long long>(L + 2) * p->r_pad;
+  const long long pf_ld = static_cast<long long>(L) * p->r_pad;
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   // The recurrent K/V GEMM addresses the stacked M_l as L * T rows (32-bit TMA coordinates).
   if (rec && static_cast<long long>(L) * T + dv::kBlockM >= (1LL << 31)) {
@@ -1450,7 +1427,6 @@ int dv_memory_plan(const dv_config* cfg, const dv_weights* w, void* stream, dv_p
                                                                  p->uup_ld, pl);
     if (p->fold) {
       cudaMemsetAsync(p->Pf, 0, pf_bytes, st);
-      k_fold_identity<<<grid_for(1LL * L * p->r_pad), 256, 0, st>>>(p->Pf, L, p->r_pad, pf_ld);
       if (L > 1) {
         const dim3 gq(p->r_pad / 64, L * (p->r_pad / 64), L);
         k_fold_products<<<gq, 256, 0, st>>>(D, U, p->Pf, L, r, p->r_pad, d, pf_ld, pl);
@@ -1537,7 +1513,13 @@ int dv_kv_engine(const dv_plan* p, long long tokens) {
 // launches per planned layer, the RMS statistics and K/V.
 int dv_kernels_per_build(const dv_plan* p) {
   if (!p) return 0;
-  return p->cfg.adapter == DV_ADAPTER_RECURRENT ? 2 * p->n_active + 2 : kStages;
+  if (p->cfg.adapter != DV_ADAPTER_RECURRENT) return kStages;
+  // recurrent, at the plan's full size: the rearranged chain (E D^T, the recurrence, the running
+  // sum, statistics, K/V), the on-chip chain (chain, statistics, K/V) or the per-layer launches
+  const long long blocks = (p->max_tokens + dv::kBlockM - 1) / dv::kBlockM;
+  if (p->fold && blocks > p->chain_clusters) return 5;
+  if (p->chain_clusters > 0) return 3;
+  return p->fold ? 5 : 2 * p->n_active + 2;
 }
 
 int dv_build_visual_memory(dv_plan* p, const void* x0, int batch, int n_vis, const int* pos,

@@ -114,26 +114,7 @@ __device__ __forceinline__ void epi_silu(const GemmParams& p, uint32_t tbase, in
   const int rows = p.s.M - row0;  // valid rows of this warp's block (may be <= 0)
   const int col0 = n * BN;
   if (col0 >= p.silu.n_h) {
-    const size_t coff = static_cast<size_t>(rows > 0 ? row0 : 0) * p.silu.ldc + (col0 - p.silu.n_h);
-    if (p.silu.Chi) {  // the product as two bf16 parts: hi = bf16(c), lo = bf16(c - hi)
-#pragma unroll 1
-      for (int c = 0; c < BN / 32; ++c) {
-        uint32_t r[32], hi[16], lo[16];
-        __syncwarp();
-        tmem_ld32(tbase + c * 32, r);
-        tmem_ld_wait();
-#pragma unroll
-        for (int u = 0; u < 16; ++u) {
-          const float a = __uint_as_float(r[2 * u]), b = __uint_as_float(r[2 * u + 1]);
-          hi[u] = pack_bf16x2(a, b);
-          lo[u] = pack_bf16x2(a - bf16_bits_to_float(hi[u] & 0xFFFFu), b - bf16_bits_to_float(hi[u] >> 16));
-        }
-        warp_store_bf16(wstage, hi, p.silu.Chi + coff + c * 32, p.silu.ldc, rows);
-        warp_store_bf16(wstage, lo, p.silu.Clo + coff + c * 32, p.silu.ldc, rows);
-      }
-      return;
-    }
-    float* c0 = p.silu.C + coff;
+    float* c0 = p.silu.C + static_cast<size_t>(rows > 0 ? row0 : 0) * p.silu.ldc + (col0 - p.silu.n_h);
 #pragma unroll 1
     for (int c = 0; c < BN / 32; ++c) {
       uint32_t r[32];

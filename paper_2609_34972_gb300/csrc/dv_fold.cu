@@ -4,18 +4,19 @@
 // Unrolling M_{l-1} = E + sum_{j<l} h_j U_j^T gives
 //   z_l = E D_l^T + sum_{j<l} h_j Q_lj^T,   Q_lj = D_l U_j (r x r, formed once per weight set),
 // so the chain splits into three parts, none of which moves the d-wide state between layers:
-//   (1) C = E [D_1 ... D_L]^T, one GEMM over all layers on the GEMM engines, written as two bf16
-//       parts C = hi + lo (2^-17 relative);
+//   (1) C = E [D_1 ... D_L]^T, one fp32 GEMM over all layers on the GEMM engines;
 //   (2) dv_hchain_kernel: per 128-token block, the recurrence over the r-wide vectors,
-//         z_l = [C_l^hi | C_l^lo | h_1 .. h_{l-1}] [I ; I ; Q_l1 .. Q_l,l-1]^T,
-//       one tcgen05 GEMM per layer whose K grows by r_pad each layer, SiLU in its epilogue;
-//   (3) dv_accum_kernel: per 128-token block and hidden slice, M_l = E + sum_{j<=l} h_j U_j^T
+//         z_l = C_l + [h_1 .. h_{l-1}] [Q_l1 .. Q_l,l-1]^T,
+//       one tcgen05 GEMM per layer whose accumulator starts at C_l and whose K grows by r_pad
+//       each layer, SiLU in its epilogue;
+//   (3) dv_accum_kernel: per two 128-token blocks and hidden slice, M_l = E + sum_{j<=l} h_j U_j^T
 //       as a running sum in TMEM, bf16 M_l stored for the K/V GEMM with its rows' sums of
 //       squares for the RMS statistic.
 // Only (2) runs layer after layer, and each of its layers is a GEMM of N = r_pad with no
 // exchange between CTAs. The sums differ from the chain's only in rounding (the same products,
 // grouped differently).
 #include "../../include/dv.h"
+#include "dv_epilogue.cuh"
 #include "dv_internal.h"
 #include "dv_ptx.cuh"
 
@@ -54,15 +55,6 @@ __device__ __forceinline__ void tmem_st32x(uint32_t taddr, const uint32_t (&r)[3
       : "memory");
 }
 
-__device__ __forceinline__ void tma_store_3d_x(const CUtensorMap* map, uint32_t src, int c0, int c1,
-                                               int c2) {
-  asm volatile(
-      "cp.async.bulk.tensor.3d.global.shared::cta.bulk_group [%0, {%2, %3, %4}], [%1];" ::"l"(
-          reinterpret_cast<uint64_t>(map)),
-      "r"(src), "r"(c0), "r"(c1), "r"(c2)
-      : "memory");
-}
-
 // ---------------------------------------------------------------- (2) the h recurrence
 
 // 3-D tiled load of a slab-map box {64 columns, rows, slabs} at (0, row, slab).
@@ -91,45 +83,45 @@ struct HCfg {
 };
 
 struct HChainParams {
-  int M;        // tokens
-  int L;        // planned layers
-  uint16_t* H;  // bf16 [M][ldh]: h_l at columns l r_pad
+  int M;           // tokens
+  int L;           // planned layers
+  const float* C;  // fp32 [M][ldc]: E D_l^T at columns l r_pad
+  int ldc;
+  uint16_t* H;     // bf16 [M][ldh]: h_l at columns l r_pad
   int ldh;
   int* status;
   unsigned long long timeout_ns;
 };
 
-// Segment `seg` of layer l's K loop: n slabs, the first at slab a0 of its A source and at slab
-// b0 of the layer's rows of Pf. 0: C_l^hi (A: Chi), 1: C_l^lo (A: Clo), 2: h_0 .. h_{l-2}
-// (A: H), 3: h_{l-1} (A: the h tile).
+// Segment `seg` of layer l's K loop (l >= 1): n slabs, the first at slab a0 of its A source and
+// at slab b0 of the layer's rows of Pf. 0: h_0 .. h_{l-2} (A: H), 1: h_{l-1} (A: the h tile).
 struct HSeg {
   int n, a0, b0;
 };
 __device__ __forceinline__ HSeg hseg(int l, int seg, int R) {
-  if (seg == 0) return {R, l * R, 0};
-  if (seg == 1) return {R, l * R, R};
-  if (seg == 2) return {l >= 2 ? (l - 1) * R : 0, 0, 2 * R};
-  return {l >= 1 ? R : 0, 0, (l + 1) * R};
+  if (seg == 0) return {l >= 2 ? (l - 1) * R : 0, 0, 0};
+  return {R, 0, (l - 1) * R};
 }
 
-// One CTA per 128-token block, all layers. Layer l's GEMM runs over 2R + l R slabs of 64 in the
-// four segments of hseg: the two bf16 parts of C_l against the identity blocks of Pf, then h_j of
-// every earlier layer against the Q_lj blocks. A pipeline step moves KS consecutive slabs of one
-// segment as one TMA box per operand (a TMA instruction has a fixed cost that one 16 KB slab
-// does not amortise); the last step of a segment uses the slabs it needs of its box (the rest is
-// zero fill or data the MMA does not read). Two TMEM accumulators: the MMAs of layer l over C and
-// the older h_j run while the epilogue of layer l - 1 still works. The epilogue applies SiLU,
-// writes bf16 h_l to the h tile (the A operand of layer l + 1's last segment) and to H (read
-// back by TMA from layer l + 2 on, and by the running sum).
-// Barriers (all waits bounded): stage full / empty; accumulator full / free; the h tile written
-// (once per layer); h_l in global memory, alternating between two barriers by layer parity so
-// that the producer, which may run up to two layers ahead of the epilogue, never waits on a
-// phase that has wrapped.
+// One CTA per 128-token block, all layers. Layer l's accumulator starts as C_l, written into TMEM
+// by the epilogue warps (tcgen05.st) while the tensor cores still work on earlier layers; the
+// layer's GEMM then adds h_j Q_lj^T for every j < l over l R slabs of 64 in the two segments of
+// hseg. A pipeline step moves KS consecutive slabs of one segment as one TMA box per operand (a
+// TMA instruction has a fixed cost that one 16 KB slab does not amortise); the last step of a
+// segment uses the slabs it needs of its box (the rest is zero fill or data the MMA does not
+// read). Two accumulators alternate by layer: layer l's MMAs over the older h_j run while the
+// epilogue of layer l - 1 still works. The epilogue applies SiLU (layer 0 straight from C_0),
+// writes bf16 h_l to the h tile (the A operand of layer l + 1's last segment) and to H (read back
+// by TMA from layer l + 2 on, and by the running sum), then loads C_{l+2} into the accumulator it
+// has just read.
+// Barriers (all waits bounded): stage full / empty; accumulator full; accumulator loaded with C;
+// the h tile written (once per layer); h_l in global memory, alternating between two barriers by
+// layer parity so that the producer, which may run up to two layers ahead of the epilogue, never
+// waits on a phase that has wrapped. The accumulator barriers of layer l complete for the
+// ((l - 1) / 2)-th time (integer division) at that layer, on accumulator l mod 2.
 template <int RP, int KS, int STAGES>
 __global__ void __launch_bounds__(kFoldThreads, 1)
-    dv_hchain_kernel(const __grid_constant__ CUtensorMap tmChi,
-                     const __grid_constant__ CUtensorMap tmClo,
-                     const __grid_constant__ CUtensorMap tmH, const __grid_constant__ CUtensorMap tmP,
+    dv_hchain_kernel(const __grid_constant__ CUtensorMap tmH, const __grid_constant__ CUtensorMap tmP,
                      const __grid_constant__ HChainParams p) {
   using C = HCfg<RP, KS, STAGES>;
   constexpr int R = C::R;
@@ -142,7 +134,7 @@ __global__ void __launch_bounds__(kFoldThreads, 1)
   auto full_bar = [&](int s) { return bar0 + 8u * s; };
   auto empty_bar = [&](int s) { return bar0 + 8u * (STAGES + s); };
   auto accf_bar = [&](int a) { return bar0 + 8u * (2 * STAGES + a); };
-  auto acce_bar = [&](int a) { return bar0 + 8u * (2 * STAGES + 2 + a); };
+  auto init_bar = [&](int a) { return bar0 + 8u * (2 * STAGES + 2 + a); };
   auto hpub_bar = [&](int a) { return bar0 + 8u * (2 * STAGES + 4 + a); };
   const uint32_t htile_bar = bar0 + 8u * (2 * STAGES + 6);
   const uint32_t drain_bar = bar0 + 8u * (2 * STAGES + 7);
@@ -161,7 +153,7 @@ __global__ void __launch_bounds__(kFoldThreads, 1)
     }
     for (int a = 0; a < 2; ++a) {
       mbar_init(accf_bar(a), 1);
-      mbar_init(acce_bar(a), kEpi);
+      mbar_init(init_bar(a), kEpi);
       mbar_init(hpub_bar(a), kEpi);
     }
     mbar_init(htile_bar, kEpi);
@@ -170,8 +162,6 @@ __global__ void __launch_bounds__(kFoldThreads, 1)
     fence_barrier_init();
   }
   if (warp == 0 && lane == 0) {
-    tma_prefetch_desc(&tmChi);
-    tma_prefetch_desc(&tmClo);
     tma_prefetch_desc(&tmH);
     tma_prefetch_desc(&tmP);
   }
@@ -192,12 +182,12 @@ __global__ void __launch_bounds__(kFoldThreads, 1)
       int stage = 0;
       uint32_t phase = 0, used = 0, issued_parity = 0;
       bool ok = true;
-      for (int l = 0; l < p.L && ok; ++l) {
-        for (int seg = 0; seg < 4 && ok; ++seg) {
+      for (int l = 1; l < p.L && ok; ++l) {
+        for (int seg = 0; seg < 2 && ok; ++seg) {
           const HSeg g = hseg(l, seg, R);
-          // h_{l-2} is the newest layer segment 2 reads: wait until it is in global memory (the
+          // h_{l-2} is the newest layer segment 0 reads: wait until it is in global memory (the
           // layers before it were published earlier)
-          if (seg == 2 && g.n > 0 &&
+          if (seg == 0 && g.n > 0 &&
               !mbar_wait(hpub_bar((l - 2) & 1), static_cast<uint32_t>((l - 2) >> 1) & 1u, abort_flag,
                          tmo)) {
             ok = false;
@@ -209,10 +199,8 @@ __global__ void __launch_bounds__(kFoldThreads, 1)
               break;
             }
             const uint32_t a_dst = ring + stage * C::kStage, b_dst = a_dst + C::kA;
-            mbar_arrive_expect_tx(full_bar(stage), seg == 3 ? C::kB : C::kStage);
-            if (seg < 3)
-              tma_load_slabs(a_dst, seg == 0 ? &tmChi : (seg == 1 ? &tmClo : &tmH), full_bar(stage),
-                             row0, g.a0 + s0);
+            mbar_arrive_expect_tx(full_bar(stage), seg == 1 ? C::kB : C::kStage);
+            if (seg == 0) tma_load_slabs(a_dst, &tmH, full_bar(stage), row0, g.a0 + s0);
             tma_load_slabs(b_dst, &tmP, full_bar(stage), l * RP, g.b0 + s0);
             used |= 1u << stage;
             issued_parity = (issued_parity & ~(1u << stage)) | (phase << stage);
@@ -232,18 +220,18 @@ __global__ void __launch_bounds__(kFoldThreads, 1)
     if (lane == 0) {
       // ---------------------------------------------------------------- MMA issuer
       const uint32_t idesc = idesc_bf16_f32(128, RP);
-      int stage = 0, acc = 0;
-      uint32_t phase = 0, acc_phase = 0;
+      int stage = 0;
+      uint32_t phase = 0;
       bool issued_any = false, ok = true;
-      for (int l = 0; l < p.L && ok; ++l) {
-        if (!mbar_wait(acce_bar(acc), acc_phase ^ 1u, abort_flag, tmo)) break;
+      for (int l = 1; l < p.L && ok; ++l) {
+        const int acc = l & 1;
+        const uint32_t par = static_cast<uint32_t>((l - 1) >> 1) & 1u;
+        if (!mbar_wait(init_bar(acc), par, abort_flag, tmo)) break;  // C_l is in the accumulator
         tc_fence_after();
         const uint32_t d_tmem = tmem + static_cast<uint32_t>(acc * RP);
-        bool first = true;
-        for (int seg = 0; seg < 4 && ok; ++seg) {
+        for (int seg = 0; seg < 2 && ok; ++seg) {
           const HSeg g = hseg(l, seg, R);
-          if (seg == 3 && g.n > 0 &&
-              !mbar_wait(htile_bar, static_cast<uint32_t>(l - 1) & 1u, abort_flag, tmo)) {
+          if (seg == 1 && !mbar_wait(htile_bar, static_cast<uint32_t>(l - 1) & 1u, abort_flag, tmo)) {
             ok = false;
             break;
           }
@@ -256,15 +244,13 @@ __global__ void __launch_bounds__(kFoldThreads, 1)
             const uint32_t st = ring + stage * C::kStage;
             const int n_use = g.n - s0 < KS ? g.n - s0 : KS;
             for (int u = 0; u < n_use; ++u) {
-              const uint32_t a_s = seg == 3 ? htile + static_cast<uint32_t>((s0 + u) * kSlabA)
+              const uint32_t a_s = seg == 1 ? htile + static_cast<uint32_t>((s0 + u) * kSlabA)
                                             : st + static_cast<uint32_t>(u * kSlabA);
               const uint32_t b_s = st + C::kA + static_cast<uint32_t>(u * C::kSlabB);
 #pragma unroll
-              for (int k = 0; k < 4; ++k) {
+              for (int k = 0; k < 4; ++k)
                 umma_bf16(d_tmem, sdesc_kmajor_sw128(a_s + 32u * k), sdesc_kmajor_sw128(b_s + 32u * k),
-                          idesc, first ? 0u : 1u);
-                first = false;
-              }
+                          idesc, 1u);  // the accumulator starts from C_l
             }
             issued_any = true;
             umma_commit(empty_bar(stage));
@@ -276,10 +262,6 @@ __global__ void __launch_bounds__(kFoldThreads, 1)
         }
         if (!ok) break;
         umma_commit(accf_bar(acc));
-        if (++acc == 2) {
-          acc = 0;
-          acc_phase ^= 1u;
-        }
       }
       if (*abort_flag && issued_any) {  // no TMEM release while an MMA may still run
         umma_commit(drain_bar);
@@ -291,46 +273,88 @@ __global__ void __launch_bounds__(kFoldThreads, 1)
     const int qq = warp & 3;  // the TMEM lane quarter this warp may access
     const int row = qq * 32 + lane;
     const int t = row0 + row;
-    int acc = 0;
-    uint32_t acc_phase = 0;
-    for (int l = 0; l < p.L; ++l) {
-      if (!__all_sync(0xFFFFFFFFu, mbar_wait(accf_bar(acc), acc_phase, abort_flag, tmo))) break;
-      tc_fence_after();
-      const uint32_t tb =
-          tmem + (static_cast<uint32_t>(qq * 32) << 16) + static_cast<uint32_t>(acc * RP);
+    const bool live = t < p.M;
+    const uint32_t tl = tmem + (static_cast<uint32_t>(qq * 32) << 16);
+    const float* crow = p.C + static_cast<long long>(live ? t : 0) * p.ldc;
+    uint8_t* hrow = base_ptr + C::kOffH;
+    // this row's 32 columns c*32 .. of C_lc (zero past the build's tokens)
+    auto load_c = [&](int lc, int c, uint32_t (&r)[32]) {
+      const float4* src = reinterpret_cast<const float4*>(crow + lc * RP + c * 32);
+#pragma unroll
+      for (int k = 0; k < 8; ++k) {
+        const float4 v = live ? src[k] : make_float4(0.0f, 0.0f, 0.0f, 0.0f);
+        r[4 * k] = __float_as_uint(v.x);
+        r[4 * k + 1] = __float_as_uint(v.y);
+        r[4 * k + 2] = __float_as_uint(v.z);
+        r[4 * k + 3] = __float_as_uint(v.w);
+      }
+    };
+    // C_lc into accumulator a, the starting value of layer lc's GEMM
+    auto put_c = [&](int lc, int a) {
 #pragma unroll 1
       for (int c = 0; c < RP / 32; ++c) {
-        uint32_t r[32], pk[16];
+        uint32_t r[32];
+        load_c(lc, c, r);
         __syncwarp();
-        tmem_ld32(tb + c * 32, r);
-        tmem_ld_wait();
-#pragma unroll
-        for (int v = 0; v < 16; ++v)
-          pk[v] = pack_bf16x2(silu(__uint_as_float(r[2 * v])), silu(__uint_as_float(r[2 * v + 1])));
-        uint8_t* slab = base_ptr + C::kOffH + (c / 2) * kSlabA;
-#pragma unroll
-        for (int k = 0; k < 4; ++k)
-          *reinterpret_cast<uint4*>(slab + swz(row, (c % 2) * 4 + k)) =
-              make_uint4(pk[4 * k], pk[4 * k + 1], pk[4 * k + 2], pk[4 * k + 3]);
+        tmem_st32x(tl + static_cast<uint32_t>(a * RP + c * 32), r);
       }
+      asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
       tc_fence_before();
-      mbar_arrive(acce_bar(acc));
+      mbar_arrive(init_bar(a));
+    };
+    // SiLU of the 32 columns c*32 .. of z into the h tile (bf16, swizzled as the MMA reads it)
+    auto put_h = [&](int c, const uint32_t (&r)[32]) {
+      uint32_t pk[16];
+#pragma unroll
+      for (int v = 0; v < 16; ++v)
+        pk[v] = pack_bf16x2(silu(__uint_as_float(r[2 * v])), silu(__uint_as_float(r[2 * v + 1])));
+      uint8_t* slab = hrow + (c / 2) * kSlabA;
+#pragma unroll
+      for (int k = 0; k < 4; ++k)
+        *reinterpret_cast<uint4*>(slab + swz(row, (c % 2) * 4 + k)) =
+            make_uint4(pk[4 * k], pk[4 * k + 1], pk[4 * k + 2], pk[4 * k + 3]);
+    };
+    for (int l = 0; l < p.L; ++l) {
+      if (l == 0) {  // z_0 = C_0
+#pragma unroll 1
+        for (int c = 0; c < RP / 32; ++c) {
+          uint32_t r[32];
+          load_c(0, c, r);
+          put_h(c, r);
+        }
+      } else {
+        const int acc = l & 1;
+        if (!__all_sync(0xFFFFFFFFu, mbar_wait(accf_bar(acc), static_cast<uint32_t>((l - 1) >> 1) & 1u,
+                                               abort_flag, tmo)))
+          break;
+        tc_fence_after();
+#pragma unroll 1
+        for (int c = 0; c < RP / 32; ++c) {
+          uint32_t r[32];
+          __syncwarp();
+          tmem_ld32(tl + static_cast<uint32_t>(acc * RP + c * 32), r);
+          tmem_ld_wait();
+          put_h(c, r);
+        }
+      }
       // The h tile first (the next layer's MMA waits for it; async proxy), then the copy of h_l
       // in H (TMA loads two or more layers later, and the running sum): read back from the tile.
       asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
       mbar_arrive(htile_bar);
-      if (t < p.M) {
+      if (live) {
         uint4* hg = reinterpret_cast<uint4*>(p.H + static_cast<long long>(t) * p.ldh + l * RP);
 #pragma unroll 1
         for (int c8 = 0; c8 < RP / 8; ++c8)
-          hg[c8] = *reinterpret_cast<const uint4*>(base_ptr + C::kOffH + (c8 / 8) * kSlabA +
-                                                   swz(row, c8 % 8));
+          hg[c8] = *reinterpret_cast<const uint4*>(hrow + (c8 / 8) * kSlabA + swz(row, c8 % 8));
       }
       asm volatile("fence.proxy.async.global;" ::: "memory");
       mbar_arrive(hpub_bar(l & 1));
-      if (++acc == 2) {
-        acc = 0;
-        acc_phase ^= 1u;
+      // the accumulator just read starts layer l + 2; before layer 1 both start
+      if (l == 0) {
+        if (p.L > 1) put_c(1, 1);
+        if (p.L > 2) put_c(2, 0);
+      } else if (l + 2 < p.L) {
+        put_c(l + 2, l & 1);
       }
     }
   }
@@ -349,13 +373,12 @@ __global__ void __launch_bounds__(kFoldThreads, 1)
 template <int RP, int CW, int STAGES>
 struct ACfg {
   static constexpr int R = RP / 64;
-  static constexpr int NS = CW / 64;              // 64-column slabs of the slice
-  static constexpr int kSlabB = CW * 128;         // [CW rows of U_l][64] bf16
-  static constexpr int kStage = kSlabA + kSlabB;
-  static constexpr int kOffOut = STAGES * kStage; // bf16 M_l of the slice, staged for TMA stores
-  static constexpr int kEnd = kOffOut + NS * kSlabA;
+  static constexpr int kSlabB = CW * 128;            // [CW rows of U_l][64] bf16
+  static constexpr int kStage = 2 * kSlabA + kSlabB; // h slabs of the two token blocks, U slab
+  static constexpr int kOffWarp = STAGES * kStage;   // per-warp staging of the M_l stores
+  static constexpr int kEnd = kOffWarp + 4 * kWarpStageFloats * 4;
   static constexpr int kSmemBytes = kEnd + 1024 + 256;
-  static constexpr int kTmemCols = CW <= 64 ? 64 : (CW <= 128 ? 128 : 256);
+  static constexpr int kTmemCols = 2 * CW <= 256 ? 256 : 512;
   static_assert(kSlabB % 1024 == 0, "stage tiles stay 1024-byte aligned");
   static_assert(kSmemBytes <= 232448, "shared memory of one CTA");
 };
@@ -366,21 +389,24 @@ struct AccumParams {
   int d;
   int S;               // hidden slices (d / CW)
   const uint16_t* x0;  // bf16 [M][d]
+  uint16_t* mem;       // bf16 [L][M][d]: the stacked M_l
   float* part;         // fp32 [L][part_ld / M][M]: sums of squares of M_l per slice
   long long part_ld;
   int* status;
   unsigned long long timeout_ns;
 };
 
-// CTA (block b, slice s) of the grid b * S + s: 128 token rows, hidden columns [s CW, (s+1) CW).
-// The accumulator starts as the fp32 widening of E's slice (tcgen05.st); layer l adds
-// h_l U_l^T (K = r_pad) and is read back: bf16 M_l to the stacked memories (TMA store through
-// the staging slabs) and the row's sum of M_l^2 over the slice to part. The next layer's MMA
-// waits until the readback has left TMEM, and runs while the stores go out.
+// CTA (pair of token blocks b, slice s) of the grid b * S + s: token blocks 2b and 2b + 1 (128
+// rows each) and hidden columns [s CW, (s+1) CW); one TMEM accumulator per block. Each
+// accumulator starts as the fp32 widening of E's slice (tcgen05.st); layer l adds h_l U_l^T
+// (K = r_pad, the U slab staged once for both blocks) and is read back: bf16 M_l stored through
+// the warp's staging (whole row segments per store instruction) and the row's sum of M_l^2 over
+// the slice to part. Each block has its own barriers, so one block's next MMAs run while the
+// other block's readback and stores go on.
 template <int RP, int CW, int STAGES>
 __global__ void __launch_bounds__(kFoldThreads, 1)
     dv_accum_kernel(const __grid_constant__ CUtensorMap tmH, const __grid_constant__ CUtensorMap tmU,
-                    const __grid_constant__ CUtensorMap tmM, const __grid_constant__ AccumParams p) {
+                    const __grid_constant__ AccumParams p) {
   using C = ACfg<RP, CW, STAGES>;
   constexpr int R = C::R;
   extern __shared__ uint8_t smem_raw[];
@@ -391,25 +417,27 @@ __global__ void __launch_bounds__(kFoldThreads, 1)
   const uint32_t bar0 = smem_addr(bars);
   auto full_bar = [&](int s) { return bar0 + 8u * s; };
   auto empty_bar = [&](int s) { return bar0 + 8u * (STAGES + s); };
-  const uint32_t accf_bar = bar0 + 8u * (2 * STAGES);
-  const uint32_t accr_bar = bar0 + 8u * (2 * STAGES + 1);
-  const uint32_t drain_bar = bar0 + 8u * (2 * STAGES + 2);
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 2 * STAGES + 3);
+  auto accf_bar = [&](int b) { return bar0 + 8u * (2 * STAGES + b); };
+  auto accr_bar = [&](int b) { return bar0 + 8u * (2 * STAGES + 2 + b); };
+  const uint32_t drain_bar = bar0 + 8u * (2 * STAGES + 4);
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 2 * STAGES + 5);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
-  const uint32_t ring = base, out = base + C::kOffOut;
+  const uint32_t ring = base;
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const uint64_t tmo = p.timeout_ns;
-  const int blk = blockIdx.x / p.S, sl = blockIdx.x % p.S;
-  const int row0 = blk * 128, col0 = sl * CW;
+  const int pb = blockIdx.x / p.S, sl = blockIdx.x % p.S;
+  const int row0 = pb * 256, col0 = sl * CW;
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < STAGES; ++s) {
       mbar_init(full_bar(s), 1);
       mbar_init(empty_bar(s), 1);
     }
-    mbar_init(accf_bar, 1);
-    mbar_init(accr_bar, kEpi);
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(accf_bar(b), 1);
+      mbar_init(accr_bar(b), kEpi);
+    }
     mbar_init(drain_bar, 1);
     *abort_flag = 0;
     fence_barrier_init();
@@ -417,7 +445,6 @@ __global__ void __launch_bounds__(kFoldThreads, 1)
   if (warp == 0 && lane == 0) {
     tma_prefetch_desc(&tmH);
     tma_prefetch_desc(&tmU);
-    tma_prefetch_desc(&tmM);
   }
   if (warp == 1) {
     tmem_alloc(smem_addr(tmem_slot), C::kTmemCols);
@@ -442,10 +469,11 @@ __global__ void __launch_bounds__(kFoldThreads, 1)
             ok = false;
             break;
           }
-          const uint32_t a_dst = ring + stage * C::kStage, b_dst = a_dst + kSlabA;
+          const uint32_t dst = ring + stage * C::kStage;
           mbar_arrive_expect_tx(full_bar(stage), C::kStage);
-          tma_load_2d(a_dst, &tmH, full_bar(stage), l * RP + 64 * q, row0);
-          tma_load_2d(b_dst, &tmU, full_bar(stage), 64 * q, l * p.d + col0);
+          tma_load_2d(dst, &tmH, full_bar(stage), l * RP + 64 * q, row0);
+          tma_load_2d(dst + kSlabA, &tmH, full_bar(stage), l * RP + 64 * q, row0 + 128);
+          tma_load_2d(dst + 2 * kSlabA, &tmU, full_bar(stage), 64 * q, l * p.d + col0);
           used |= 1u << stage;
           issued_parity = (issued_parity & ~(1u << stage)) | (phase << stage);
           if (++stage == STAGES) {
@@ -467,29 +495,35 @@ __global__ void __launch_bounds__(kFoldThreads, 1)
       uint32_t phase = 0;
       bool issued_any = false, ok = true;
       for (int l = 0; l < p.L && ok; ++l) {
-        // the accumulator holds E (l = 0) or M_{l-1}, and its readback has left TMEM
-        if (!mbar_wait(accr_bar, static_cast<uint32_t>(l) & 1u, abort_flag, tmo)) break;
-        tc_fence_after();
-        for (int q = 0; q < R; ++q) {
+        for (int q = 0; q < R && ok; ++q) {
           if (!mbar_wait(full_bar(stage), phase, abort_flag, tmo)) {
             ok = false;
             break;
           }
-          tc_fence_after();
-          const uint32_t a_s = ring + stage * C::kStage, b_s = a_s + kSlabA;
+          const uint32_t a0 = ring + stage * C::kStage, b_s = a0 + 2 * kSlabA;
+          for (int b = 0; b < 2; ++b) {
+            // block b's accumulator holds E (l = 0) or M_{l-1}, and its readback has left TMEM
+            if (q == 0 && !mbar_wait(accr_bar(b), static_cast<uint32_t>(l) & 1u, abort_flag, tmo)) {
+              ok = false;
+              break;
+            }
+            tc_fence_after();
+            const uint32_t a_s = a0 + static_cast<uint32_t>(b * kSlabA);
+            const uint32_t d_tmem = tmem + static_cast<uint32_t>(b * CW);
 #pragma unroll
-          for (int k = 0; k < 4; ++k)
-            umma_bf16(tmem, sdesc_kmajor_sw128(a_s + 32u * k), sdesc_kmajor_sw128(b_s + 32u * k),
-                      idesc, 1u);
-          issued_any = true;
+            for (int k = 0; k < 4; ++k)
+              umma_bf16(d_tmem, sdesc_kmajor_sw128(a_s + 32u * k), sdesc_kmajor_sw128(b_s + 32u * k),
+                        idesc, 1u);
+            issued_any = true;
+            if (q == R - 1) umma_commit(accf_bar(b));
+          }
+          if (!ok) break;
           umma_commit(empty_bar(stage));
           if (++stage == STAGES) {
             stage = 0;
             phase ^= 1u;
           }
         }
-        if (!ok) break;
-        umma_commit(accf_bar);
       }
       if (*abort_flag && issued_any) {
         umma_commit(drain_bar);
@@ -498,14 +532,15 @@ __global__ void __launch_bounds__(kFoldThreads, 1)
     }
   } else {
     // ------------------------------------------------------------------ epilogue warps
-    const int qq = warp & 3;
+    const int qq = warp & 3;  // the TMEM lane quarter this warp may access
     const int row = qq * 32 + lane;
-    const int t = row0 + row;
-    const bool issuer = warp == 2 && lane == 0;  // issues the stores of the slice
-    const uint32_t tb = tmem + (static_cast<uint32_t>(qq * 32) << 16);
-    // M_0 = E: the fp32 widening of this row's slice of E into the accumulator
-    {
-      const uint16_t* xr = p.x0 + static_cast<long long>(t) * p.d + col0;
+    const uint32_t tl = tmem + (static_cast<uint32_t>(qq * 32) << 16);
+    float* wstage = reinterpret_cast<float*>(base_ptr + C::kOffWarp) + qq * kWarpStageFloats;
+    // M_0 = E: the fp32 widening of this row's slice of E into both accumulators
+#pragma unroll 1
+    for (int b = 0; b < 2; ++b) {
+      const int t = row0 + b * 128 + row;
+      const uint16_t* xr = p.x0 + static_cast<long long>(t < p.M ? t : 0) * p.d + col0;
 #pragma unroll 1
       for (int c = 0; c < CW / 32; ++c) {
         uint32_t r[32];
@@ -520,51 +555,46 @@ __global__ void __launch_bounds__(kFoldThreads, 1)
           }
         }
         __syncwarp();
-        tmem_st32x(tb + c * 32, r);
+        tmem_st32x(tl + static_cast<uint32_t>(b * CW + c * 32), r);
       }
-      asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
-      tc_fence_before();
-      mbar_arrive(accr_bar);
     }
-    for (int l = 0; l < p.L; ++l) {
-      bool ok = __all_sync(0xFFFFFFFFu, mbar_wait(accf_bar, static_cast<uint32_t>(l) & 1u, abort_flag, tmo));
-      // the staging slabs are free once the previous layer's stores have read them
-      if (issuer && l > 0) asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory");
-      ok = named_barrier_and(1, kEpi, ok);
-      if (!ok) break;
-      tc_fence_after();
-      float ss = 0.0f;
+    asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
+    tc_fence_before();
+    mbar_arrive(accr_bar(0));
+    mbar_arrive(accr_bar(1));
+    bool ok = true;
+    for (int l = 0; l < p.L && ok; ++l) {
 #pragma unroll 1
-      for (int c = 0; c < CW / 32; ++c) {
-        uint32_t r[32], pk[16];
-        __syncwarp();
-        tmem_ld32(tb + c * 32, r);
-        tmem_ld_wait();
+      for (int b = 0; b < 2; ++b) {
+        ok = __all_sync(0xFFFFFFFFu, mbar_wait(accf_bar(b), static_cast<uint32_t>(l) & 1u, abort_flag, tmo));
+        if (!ok) break;
+        tc_fence_after();
+        // the whole row of the slice leaves TMEM first, so the next layer's MMA can start
+        uint32_t pk[CW / 32][16];
+        float ss = 0.0f;
 #pragma unroll
-        for (int v = 0; v < 16; ++v) {
-          const float a = __uint_as_float(r[2 * v]), b = __uint_as_float(r[2 * v + 1]);
-          ss = fmaf(a, a, ss);
-          ss = fmaf(b, b, ss);
-          pk[v] = pack_bf16x2(a, b);
+        for (int c = 0; c < CW / 32; ++c) {
+          uint32_t r[32];
+          __syncwarp();
+          tmem_ld32(tl + static_cast<uint32_t>(b * CW + c * 32), r);
+          tmem_ld_wait();
+#pragma unroll
+          for (int v = 0; v < 16; ++v) {
+            const float x = __uint_as_float(r[2 * v]), y = __uint_as_float(r[2 * v + 1]);
+            ss = fmaf(x, x, ss);
+            ss = fmaf(y, y, ss);
+            pk[c][v] = pack_bf16x2(x, y);
+          }
         }
-        uint8_t* slab = base_ptr + C::kOffOut + (c / 2) * kSlabA;
+        tc_fence_before();
+        mbar_arrive(accr_bar(b));
+        const int t0 = row0 + b * 128 + qq * 32;  // the warp's first row
+        uint16_t* dst = p.mem + (static_cast<long long>(l) * p.M + t0) * p.d + col0;
 #pragma unroll
-        for (int k = 0; k < 4; ++k)
-          *reinterpret_cast<uint4*>(slab + swz(row, (c % 2) * 4 + k)) =
-              make_uint4(pk[4 * k], pk[4 * k + 1], pk[4 * k + 2], pk[4 * k + 3]);
-      }
-      tc_fence_before();
-      mbar_arrive(accr_bar);  // the readback has left TMEM: the next layer may accumulate
-      if (t < p.M) p.part[l * p.part_ld + static_cast<long long>(sl) * p.M + t] = ss;
-      asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-      named_barrier(1, kEpi);
-      if (issuer) {
-        for (int j = 0; j < C::NS; ++j)
-          tma_store_3d_x(&tmM, out + static_cast<uint32_t>(j * kSlabA), col0 + 64 * j, row0, l);
-        asm volatile("cp.async.bulk.commit_group;" ::: "memory");
+        for (int c = 0; c < CW / 32; ++c) warp_store_bf16(wstage, pk[c], dst + c * 32, p.d, p.M - t0);
+        if (t0 + lane < p.M) p.part[l * p.part_ld + static_cast<long long>(sl) * p.M + t0 + lane] = ss;
       }
     }
-    if (issuer) asm volatile("cp.async.bulk.wait_group 0;" ::: "memory");
   }
 
   tc_fence_before();
@@ -577,9 +607,8 @@ __global__ void __launch_bounds__(kFoldThreads, 1)
 }
 
 template <int RP, int KS, int ST>
-cudaError_t hchain_t(long long blocks, const CUtensorMap& chi, const CUtensorMap& clo,
-                     const CUtensorMap& h, const CUtensorMap& pf, const HChainParams& p,
-                     cudaStream_t stream) {
+cudaError_t hchain_t(long long blocks, const CUtensorMap& h, const CUtensorMap& pf,
+                     const HChainParams& p, cudaStream_t stream) {
   using C = HCfg<RP, KS, ST>;
   auto kern = dv_hchain_kernel<RP, KS, ST>;
   cudaError_t err = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, C::kSmemBytes);
@@ -592,14 +621,14 @@ cudaError_t hchain_t(long long blocks, const CUtensorMap& chi, const CUtensorMap
   cfg.stream = stream;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
-  err = cudaLaunchKernelEx(&cfg, kern, chi, clo, h, pf, p);
+  err = cudaLaunchKernelEx(&cfg, kern, h, pf, p);
   if (err != cudaSuccess) return err;
   return cudaGetLastError();
 }
 
 template <int RP, int CW, int ST>
 cudaError_t accum_t(long long ctas, const CUtensorMap& h, const CUtensorMap& u,
-                    const CUtensorMap& m3, const AccumParams& p, cudaStream_t stream) {
+                    const AccumParams& p, cudaStream_t stream) {
   using C = ACfg<RP, CW, ST>;
   auto kern = dv_accum_kernel<RP, CW, ST>;
   cudaError_t err = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, C::kSmemBytes);
@@ -612,7 +641,7 @@ cudaError_t accum_t(long long ctas, const CUtensorMap& h, const CUtensorMap& u,
   cfg.stream = stream;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
-  err = cudaLaunchKernelEx(&cfg, kern, h, u, m3, p);
+  err = cudaLaunchKernelEx(&cfg, kern, h, u, p);
   if (err != cudaSuccess) return err;
   return cudaGetLastError();
 }
@@ -621,38 +650,39 @@ cudaError_t accum_t(long long ctas, const CUtensorMap& h, const CUtensorMap& u,
 
 int hchain_box_slabs(int r_pad) { return r_pad == 256 ? 1 : 2; }
 
-// 128 columns per CTA: with two pipeline stages a CTA takes under half of an SM's shared memory
-// and TMEM, so two run on each SM and one's loads and readback hide behind the other's work.
+// A CTA of the running sum covers two token blocks and 256 hidden columns (128 where d is not a
+// multiple of 256): the U slab it stages serves both blocks, and the two accumulators fill TMEM.
 int fold_slice_cols(int d) {
-  for (int cw : {128, 64})
+  for (int cw : {256, 128})
     if (d % cw == 0) return cw;
   return 0;
 }
 
-cudaError_t launch_hchain(int r_pad, long long tokens, int n_layers, const CUtensorMap& chi,
-                          const CUtensorMap& clo, const CUtensorMap& h, const CUtensorMap& pf,
-                          uint16_t* H, int ldh, int* status, unsigned long long timeout_ns,
-                          cudaStream_t stream) {
+cudaError_t launch_hchain(int r_pad, long long tokens, int n_layers, const float* C, int ldc,
+                          const CUtensorMap& h, const CUtensorMap& pf, uint16_t* H, int ldh,
+                          int* status, unsigned long long timeout_ns, cudaStream_t stream) {
   HChainParams p;
   p.M = static_cast<int>(tokens);
   p.L = n_layers;
+  p.C = C;
+  p.ldc = ldc;
   p.H = H;
   p.ldh = ldh;
   p.status = status;
   p.timeout_ns = timeout_ns;
   const long long blocks = (tokens + 127) / 128;
   switch (r_pad) {  // slabs per box (hchain_box_slabs) and pipeline stages
-    case 64: return hchain_t<64, 2, 4>(blocks, chi, clo, h, pf, p, stream);
-    case 128: return hchain_t<128, 2, 3>(blocks, chi, clo, h, pf, p, stream);
-    case 192: return hchain_t<192, 2, 2>(blocks, chi, clo, h, pf, p, stream);
-    case 256: return hchain_t<256, 1, 3>(blocks, chi, clo, h, pf, p, stream);
+    case 64: return hchain_t<64, 2, 4>(blocks, h, pf, p, stream);
+    case 128: return hchain_t<128, 2, 3>(blocks, h, pf, p, stream);
+    case 192: return hchain_t<192, 2, 2>(blocks, h, pf, p, stream);
+    case 256: return hchain_t<256, 1, 3>(blocks, h, pf, p, stream);
     default: return cudaErrorInvalidValue;
   }
 }
 
 cudaError_t launch_accum(int r_pad, int cw, long long tokens, int n_layers, int d,
-                         const void* x0, const CUtensorMap& h, const CUtensorMap& u,
-                         const CUtensorMap& m3, float* part, long long part_ld, int* status,
+                         const void* x0, const CUtensorMap& h, const CUtensorMap& u, uint16_t* mem,
+                         float* part, long long part_ld, int* status,
                          unsigned long long timeout_ns, cudaStream_t stream) {
   AccumParams p;
   p.M = static_cast<int>(tokens);
@@ -660,17 +690,18 @@ cudaError_t launch_accum(int r_pad, int cw, long long tokens, int n_layers, int 
   p.d = d;
   p.S = d / cw;
   p.x0 = static_cast<const uint16_t*>(x0);
+  p.mem = mem;
   p.part = part;
   p.part_ld = part_ld;
   p.status = status;
   p.timeout_ns = timeout_ns;
-  const long long ctas = (tokens + 127) / 128 * p.S;
+  const long long ctas = (tokens + 255) / 256 * p.S;
 #define DV_ACCUM(RPV, CWV, STV) \
-  if (r_pad == RPV && cw == CWV) return accum_t<RPV, CWV, STV>(ctas, h, u, m3, p, stream);
-  DV_ACCUM(64, 256, 3) DV_ACCUM(64, 128, 2) DV_ACCUM(64, 64, 2)
-  DV_ACCUM(128, 256, 3) DV_ACCUM(128, 128, 2) DV_ACCUM(128, 64, 2)
-  DV_ACCUM(192, 256, 3) DV_ACCUM(192, 128, 2) DV_ACCUM(192, 64, 2)
-  DV_ACCUM(256, 256, 3) DV_ACCUM(256, 128, 2) DV_ACCUM(256, 64, 2)
+  if (r_pad == RPV && cw == CWV) return accum_t<RPV, CWV, STV>(ctas, h, u, p, stream);
+  DV_ACCUM(64, 256, 3) DV_ACCUM(64, 128, 4)
+  DV_ACCUM(128, 256, 3) DV_ACCUM(128, 128, 4)
+  DV_ACCUM(192, 256, 3) DV_ACCUM(192, 128, 4)
+  DV_ACCUM(256, 256, 3) DV_ACCUM(256, 128, 4)
 #undef DV_ACCUM
   return cudaErrorInvalidValue;
 }

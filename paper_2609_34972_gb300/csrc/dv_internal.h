@@ -74,17 +74,13 @@ __host__ __device__ inline KStep k_step(int j, int k0_slabs, int k1_slabs) {
 }
 
 // Columns [0, n_h) of the product are down-projections: H = bf16(SiLU(acc)). Columns from n_h
-// on (x0 (2 U_l)^T when the statistic of M_l is formed outside a GEMM) go to C as fp32, or,
-// when Chi is set (the recurrent adapter's E D_l^T), as two bf16 parts hi = bf16(acc) into Chi
-// and lo = bf16(acc - hi) into Clo, both [M][ldc].
+// on (x0 (2 U_l)^T when the statistic of M_l is formed outside a GEMM) go to C as fp32.
 struct EpiSilu {
   uint16_t* H;   // bf16 [M][ldh]
   int ldh;
   int n_h;       // columns that are down-projections
   float* C;      // fp32 [M][ldc] or null
   int ldc;
-  uint16_t* Chi;
-  uint16_t* Clo;
 };
 
 // Launch attribute of the build's kernels: programmatic stream serialization (see pdl_wait in
@@ -229,28 +225,27 @@ cudaError_t launch_chain(int r_pad, int spc, int S, long long tokens, int n_laye
                          int* status, unsigned long long timeout_ns, cudaStream_t stream,
                          bool split);
 
-// The recurrent adapter by the refactored chain (dv_fold.cu). With C = E [D_1 .. D_L]^T given as
-// two bf16 parts (Chi, Clo: [tokens][L r_pad]) and the plan's Pf ([L r_pad][(L + 2) r_pad]:
-// identity blocks, then Q_lj = D_l U_j):
+// The recurrent adapter by the refactored chain (dv_fold.cu). With C = E [D_1 .. D_L]^T (fp32
+// [tokens][ldc], C_l at columns l r_pad) and the plan's Pf ([L r_pad][L r_pad], block (l, j) =
+// Q_lj = D_l U_j for j < l):
 //   launch_hchain: h_l = SiLU(C_l + sum_{j<l} h_j Q_lj^T) into H ([tokens][ldh], h_l at columns
-//     l r_pad), one CTA per 128-token block. Maps: chi, clo, h: slab maps over [tokens][L r_pad]
-//     with 128-row boxes; pf: slab map over Pf with r_pad-row boxes.
-//   launch_accum: M_l = E + sum_{j<=l} h_j U_j^T, bf16 into the stacked memories (m3: the 3-D
-//     (d, tokens, L) map with (64, 128, 1) boxes) and each row's sum of M_l^2 over each slice of
-//     cw hidden columns into part (d / cw partials per layer). u: U as [L d][r_pad] with cw-row
+//     l r_pad), one CTA per 128-token block. Maps: h: slab map over H with 128-row boxes; pf:
+//     slab map over Pf with r_pad-row boxes.
+//   launch_accum: M_l = E + sum_{j<=l} h_j U_j^T, bf16 into the stacked memories mem
+//     ([L][tokens][d]) and each row's sum of M_l^2 over each slice of cw hidden columns into part
+//     (d / cw partials per layer). h: H with 128-row boxes; u: U as [L d][r_pad] with cw-row
 //     boxes; x0: E, bf16 [tokens][d].
-// fold_slice_cols: the slice width cw (256, 192, 128 or 64 dividing d), or 0.
-// hchain_box_slabs: K slabs per TMA box of launch_hchain's maps (chi, clo, h and pf are slab maps,
+// fold_slice_cols: the slice width cw (256 or 128 dividing d), or 0.
+// hchain_box_slabs: K slabs per TMA box of launch_hchain's maps (h and pf are slab maps,
 // encode_slabs, with boxes of that many slabs).
 int fold_slice_cols(int d);
 int hchain_box_slabs(int r_pad);
-cudaError_t launch_hchain(int r_pad, long long tokens, int n_layers, const CUtensorMap& chi,
-                          const CUtensorMap& clo, const CUtensorMap& h, const CUtensorMap& pf,
-                          uint16_t* H, int ldh, int* status, unsigned long long timeout_ns,
-                          cudaStream_t stream);
+cudaError_t launch_hchain(int r_pad, long long tokens, int n_layers, const float* C, int ldc,
+                          const CUtensorMap& h, const CUtensorMap& pf, uint16_t* H, int ldh,
+                          int* status, unsigned long long timeout_ns, cudaStream_t stream);
 cudaError_t launch_accum(int r_pad, int cw, long long tokens, int n_layers, int d,
-                         const void* x0, const CUtensorMap& h, const CUtensorMap& u,
-                         const CUtensorMap& m3, float* part, long long part_ld, int* status,
+                         const void* x0, const CUtensorMap& h, const CUtensorMap& u, uint16_t* mem,
+                         float* part, long long part_ld, int* status,
                          unsigned long long timeout_ns, cudaStream_t stream);
 
 // Token tile (64, 128, 192 or 256) of the pair kernel for a build of `tokens` tokens.
@@ -322,14 +317,13 @@ struct BuildArgs {
   long long x0p_ld;     // d + 64
   float* rstd;          // [L][tokens]
   float* xx;            // [tokens]
-  float* c;             // embedding adapter, small token counts: fp32 [tokens][L * r_pad]
+  float* c;             // fp32 [tokens][L * r_pad]: embedding adapter at small token counts,
+                        // x0 (2 U_l)^T; recurrent adapter, refactored chain: E D_l^T
   float* state;         // recurrent: fp32 [tokens][d]
   uint16_t* mem;        // recurrent: bf16 [L][tokens][d]
   float* part;          // recurrent: fp32 [L][d / 64][tokens]
   uint16_t* Hlo;        // split chain: low bf16 parts of h, [tokens][L * r_pad]
   uint16_t* mem_lo;     // split chain: low bf16 part of the last M_l, [tokens][d]
-  uint16_t* Chi;        // recurrent, refactored chain: E D_l^T as bf16 hi / lo parts,
-  uint16_t* Clo;        //   [tokens][L * r_pad] each
   cudaEvent_t* marks;   // 5 events around the 4 stages, or null
 };
 
