@@ -529,11 +529,17 @@ def run_dv(args):
                           name="llava15_7b_recurrent",
                           description=synth.CONFIGS["llava15_7b"].description +
                           "; recurrent adapter (Sec. 3.1 Eq. 6)")
+            # on the Qwen2.5-VL video shape (128 token blocks, rank 256) the recurrent adapter
+            # runs the rearranged chain: E D^T, the r-wide recurrence, the running sum of M_l
+            vid = synth.CONFIGS["qwen25vl_7b_video"]
+            rec_v = replace(vid, adapter="recurrent", name="qwen25vl_7b_video_recurrent",
+                            description=vid.description + "; recurrent adapter (Sec. 3.1 Eq. 6)")
             # and the Qwen3-VL-4B-shaped build (the paper's default backbone: per-head K norm,
             # interleaved M-RoPE)
             # with the App. J skipping of its first 5 and last 10 adapters
             q3 = synth.CONFIGS["qwen3vl_4b_image"]
             variants = [measure_config(dv, rec, args, dev, peaks, peak_src),
+                        measure_config(dv, rec_v, args, dev, peaks, peak_src),
                         measure_config(dv, q3, args, dev, peaks, peak_src),
                         measure_config(dv, q3, args, dev, peaks, peak_src, skip=(5, 10)),
                         measure_consumer(dv, synth.CONFIGS["llava15_7b"], args, peaks)]
