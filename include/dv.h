@@ -58,6 +58,17 @@ enum {
   DV_ADAPTER_EMBEDDING = 0,  /* M_l = A_l(E) for every layer (Eq. 5) */
   DV_ADAPTER_RECURRENT = 1   /* M_0 = E, M_l = A_l(M_{l-1}) through the planned layers (Eq. 6) */
 };
+/* How the recurrent adapter's chain is evaluated (the same function either way, Sec. 3.1 Eq. 6):
+ * the chain in the paper's order, z_l = M_{l-1} D_l^T layer after layer (on chip, a cluster of
+ * SMs per 128-token block, where such a cluster fits; else per-layer launches), or rearranged,
+ * z_l = E D_l^T + sum_{j<l} h_j (D_l U_j)^T and M_l = E + sum_{j<=l} h_j U_j^T, whose only
+ * sequential part is r wide. */
+enum {
+  DV_RECURRENT_AUTO = 0,        /* the on-chip chain for builds whose token blocks fit in one
+                                   wave of its clusters, the rearranged chain for larger ones */
+  DV_RECURRENT_CHAIN = 1,       /* the chain in the paper's order for every build */
+  DV_RECURRENT_REARRANGED = 2   /* the rearranged chain for every build */
+};
 
 /* Model shape and build limits. Supported (else DV_ERR_UNSUPPORTED_SHAPE):
  *   d % 64 == 0, 64 <= d <= 16384;  1 <= rank <= 256;  head_dim in {64, 128};
@@ -69,6 +80,8 @@ enum {
  *   k_norm in {0, 1}; k_norm_eps >= 0;
  *   adapter in {DV_ADAPTER_EMBEDDING, DV_ADAPTER_RECURRENT};
  *   split_chain in {0, 1}, and 1 only with DV_ADAPTER_RECURRENT;
+ *   recurrent_path a DV_RECURRENT_* value, not AUTO only with DV_ADAPTER_RECURRENT,
+ *   REARRANGED not with split_chain (DV_ERR_INVALID_ARG) and only with d % 128 == 0;
  *   max_batch * max_n_vis >= 1 and <= 2^24 (the tokens one build may carry). */
 typedef struct dv_config {
   int d;                 /* hidden size of the language model */
@@ -100,6 +113,8 @@ typedef struct dv_config {
                             every build at rank > 128) the rearranged chain, which forms each
                             layer's down-projection input from E D_l^T and the earlier h_j
                             through the r x r products D_l U_j (exactly the same sum). */
+  int recurrent_path;    /* recurrent adapter only: DV_RECURRENT_AUTO (0), _CHAIN or
+                            _REARRANGED; the split chain always takes the chain's path */
 } dv_config;
 
 /* Weights of all L layers, bf16, device pointers. Read only during dv_memory_plan: the plan

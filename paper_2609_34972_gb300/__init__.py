@@ -41,6 +41,11 @@ DV_LAYER_IDENTITY = 1
 DV_LAYER_DROP = 2
 DV_ADAPTER_EMBEDDING = 0
 DV_ADAPTER_RECURRENT = 1
+DV_RECURRENT_AUTO = 0
+DV_RECURRENT_CHAIN = 1
+DV_RECURRENT_REARRANGED = 2
+_RECURRENT_PATH = {"auto": DV_RECURRENT_AUTO, "chain": DV_RECURRENT_CHAIN,
+                   "rearranged": DV_RECURRENT_REARRANGED}
 
 EXPORTED = ["dv_memory_plan", "dv_build_visual_memory", "dv_plan_status", "dv_free",
             "dv_error_string", "dv_timing_enable", "dv_timing_read", "dv_kernels_per_build",
@@ -62,7 +67,7 @@ class DvConfig(ctypes.Structure):
                 ("max_batch", ctypes.c_int), ("max_n_vis", ctypes.c_int),
                 ("has_kv_bias", ctypes.c_int), ("adapter", ctypes.c_int),
                 ("k_norm", ctypes.c_int), ("k_norm_eps", ctypes.c_float),
-                ("split_chain", ctypes.c_int)]
+                ("split_chain", ctypes.c_int), ("recurrent_path", ctypes.c_int)]
 
 
 class DvWeights(ctypes.Structure):
@@ -158,21 +163,25 @@ def _ptr(t):
 def make_config(d, n_layers, n_kv_heads, head_dim, rank, rope="1d", rope_theta=10000.0,
                 mrope_section=(0, 0, 0), rms_eps=1e-6, max_batch=1, max_n_vis=1,
                 has_kv_bias=False, adapter="embedding", k_norm=False,
-                k_norm_eps=1e-6, split_chain=False) -> DvConfig:
+                k_norm_eps=1e-6, split_chain=False, recurrent_path="auto") -> DvConfig:
     """``adapter``: "embedding" (M_l = A_l(E), Sec. 3.1 Eq. 5) or "recurrent"
     (M_l = A_l(M_{l-1}), Sec. 3.1 Eq. 6). ``rope``: "1d", "mrope" (contiguous sections) or
     "mrope_interleaved". ``k_norm``: per-head RMSNorm of K before RoPE (weights["kgamma"]).
-    ``split_chain`` (recurrent only): the chain's GEMMs read hi + lo bf16 operands."""
+    ``split_chain`` (recurrent only): the chain's GEMMs read hi + lo bf16 operands.
+    ``recurrent_path`` (recurrent only): "auto", "chain" (the paper's order) or "rearranged"."""
     if adapter not in ("embedding", "recurrent"):
         raise ValueError(f"unknown adapter {adapter!r}")
     if rope not in _ROPE:
         raise ValueError(f"unknown rope {rope!r}")
+    if recurrent_path not in _RECURRENT_PATH:
+        raise ValueError(f"unknown recurrent_path {recurrent_path!r}")
     return DvConfig(int(d), int(n_layers), int(n_kv_heads), int(head_dim), int(rank),
                     DV_ACT_SILU, _ROPE[rope],
                     float(rope_theta), (ctypes.c_int * 3)(*mrope_section), float(rms_eps),
                     int(max_batch), int(max_n_vis), int(bool(has_kv_bias)),
                     DV_ADAPTER_RECURRENT if adapter == "recurrent" else DV_ADAPTER_EMBEDDING,
-                    int(bool(k_norm)), float(k_norm_eps), int(bool(split_chain)))
+                    int(bool(k_norm)), float(k_norm_eps), int(bool(split_chain)),
+                    _RECURRENT_PATH[recurrent_path])
 
 
 class Plan:

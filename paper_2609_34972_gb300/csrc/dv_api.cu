@@ -647,6 +647,14 @@ int check_config(const dv_config* c) {
     return DV_ERR_INVALID_ARG;
   if (c->split_chain != 0 && c->split_chain != 1) return DV_ERR_INVALID_ARG;
   if (c->split_chain && c->adapter != DV_ADAPTER_RECURRENT) return DV_ERR_INVALID_ARG;
+  if (c->recurrent_path != DV_RECURRENT_AUTO && c->recurrent_path != DV_RECURRENT_CHAIN &&
+      c->recurrent_path != DV_RECURRENT_REARRANGED)
+    return DV_ERR_INVALID_ARG;
+  if (c->recurrent_path != DV_RECURRENT_AUTO && c->adapter != DV_ADAPTER_RECURRENT)
+    return DV_ERR_INVALID_ARG;
+  if (c->recurrent_path == DV_RECURRENT_REARRANGED && c->split_chain) return DV_ERR_INVALID_ARG;
+  if (c->recurrent_path == DV_RECURRENT_REARRANGED && dv::fold_slice_cols(c->d) == 0)
+    return DV_ERR_UNSUPPORTED_SHAPE;
   if (c->d % 64 != 0 || c->d > 16384) return DV_ERR_UNSUPPORTED_SHAPE;
   if (c->rank > 256) return DV_ERR_UNSUPPORTED_SHAPE;
   if (c->head_dim != 64 && c->head_dim != 128) return DV_ERR_UNSUPPORTED_SHAPE;
@@ -1370,8 +1378,11 @@ int dv_memory_plan(const dv_config* cfg, const dv_weights* w, void* stream, dv_p
   const long long T = p->max_tokens;
   // Recurrent adapter: the refactored chain (dv_fold.cu) unless the split chain is asked for;
   // builds whose token blocks fit in one wave of on-chip chain clusters take the chain instead.
-  p->fold = rec && !cfg->split_chain && dv::fold_slice_cols(d) > 0;
-  p->chain_clusters = rec ? dv::chain_resident_clusters(d, p->r_pad, cfg->split_chain != 0) : 0;
+  p->fold = rec && !cfg->split_chain && dv::fold_slice_cols(d) > 0 &&
+            cfg->recurrent_path != DV_RECURRENT_CHAIN;
+  p->chain_clusters = rec && cfg->recurrent_path != DV_RECURRENT_REARRANGED
+                          ? dv::chain_resident_clusters(d, p->r_pad, cfg->split_chain != 0)
+                          : 0;
   const long long pf_ld = static_cast<long long>(L) * p->r_pad;
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   // The recurrent K/V GEMM addresses the stacked M_l as L * T rows (32-bit TMA coordinates).

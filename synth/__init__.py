@@ -133,6 +133,7 @@ class Config:
     k_norm_eps: float = 1e-6
     k_norm_sigma: float = 0.1   # per-head K-norm gain = 1 + N(0, k_norm_sigma)
     split_chain: bool = False   # recurrent adapter: hi + lo bf16 operands in the chain's GEMMs
+    recurrent_path: str = "auto"  # recurrent adapter: "auto", "chain" or "rearranged"
     description: str = ""
 
     @property

@@ -44,7 +44,8 @@ def dv_config(cfg, max_batch=None, max_n_vis=None):
                           max_batch=max_batch or cfg.batch, max_n_vis=max_n_vis or cfg.n_vis,
                           has_kv_bias=cfg.bias_sigma > 0, adapter=cfg.adapter,
                           k_norm=cfg.k_norm, k_norm_eps=cfg.k_norm_eps,
-                          split_chain=getattr(cfg, "split_chain", False))
+                          split_chain=getattr(cfg, "split_chain", False),
+                          recurrent_path=getattr(cfg, "recurrent_path", "auto"))
 
 
 def run_build(inp, plan=None, seq_len=None, batch_cache=None, slot=None, slot0=0, fill=0.0,

@@ -65,10 +65,29 @@ def test_null_arguments_rejected(dv):
     ("rope_theta", -1.0, 1), ("rms_eps", -1e-6, 1), ("n_kv_heads", 129, 2),
     ("adapter", 2, 1), ("adapter", -1, 1), ("rope", 3, 1), ("k_norm", 2, 1),
     ("k_norm_eps", -1.0, 1), ("split_chain", 2, 1), ("split_chain", 1, 1),
+    ("recurrent_path", 3, 1), ("recurrent_path", -1, 1), ("recurrent_path", 2, 1),
 ])
 def test_bad_config_rejected_before_device(dv, field, value, code):
     cfg = dv.make_config(512, 4, 8, 64, 16, max_batch=1, max_n_vis=64)
     setattr(cfg, field, value)
+    w = dv.DvWeights(*([ctypes.c_void_p(256)] * 5 + [None, None, None]))
+    h = ctypes.c_void_p()
+    assert dv.lib().dv_memory_plan(ctypes.byref(cfg), ctypes.byref(w), None, ctypes.byref(h)) == code
+    assert not h.value
+
+
+@pytest.mark.parametrize("d,split,path,code", [
+    (512, 1, "rearranged", 1),   # the split chain has only the chain's path
+    (576, 0, "rearranged", 2),   # the rearranged chain's slices need d % 128 == 0
+    (512, 0, "bogus", None),     # refused by the binding
+])
+def test_recurrent_path_rules(dv, d, split, path, code):
+    if code is None:
+        with pytest.raises(ValueError):
+            dv.make_config(d, 4, 8, 64, 16, adapter="recurrent", recurrent_path=path)
+        return
+    cfg = dv.make_config(d, 4, 8, 64, 16, max_batch=1, max_n_vis=64, adapter="recurrent",
+                         split_chain=bool(split), recurrent_path=path)
     w = dv.DvWeights(*([ctypes.c_void_p(256)] * 5 + [None, None, None]))
     h = ctypes.c_void_p()
     assert dv.lib().dv_memory_plan(ctypes.byref(cfg), ctypes.byref(w), None, ctypes.byref(h)) == code

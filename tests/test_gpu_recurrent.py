@@ -1,11 +1,12 @@
 """GPU parity of the recurrent adapter (Sec. 3.1 Eq. 6): M_0 = E, M_l = M_{l-1} +
 SiLU(M_{l-1} D_l) U_l, then the same norm, projections, rotation and cache store as the
-embedding adapter. The CUDA build (split-K down-projection per layer, fp32 state carried by the
-up-projection epilogue, one K/V launch over every layer) is compared with the fp64 oracle's
-recurrent variant on the same inputs: element by element on small cases (every r_pad, both
-K/V engines, ragged tails, M-RoPE and bias, layer modes, the no-alloc entry) and on sampled
-tokens at full size. The chain's intermediates (SiLU(M_{l-1} D_l), bf16 M_l, the RMS statistic)
-are checked stage by stage.
+embedding adapter. Both ways the library evaluates the chain are compared with the fp64 oracle's
+recurrent variant on the same inputs: the chain in the paper's order (on chip, or per-layer
+launches where no cluster fits) and the rearranged chain (E D^T, the r-wide recurrence through
+the products D_l U_j, the running sum of M_l), element by element on small cases (every r_pad,
+both K/V engines, ragged tails, M-RoPE and bias, layer modes, the no-alloc entry) and, with the
+automatic choice, on sampled tokens at full size. The intermediates (SiLU(M_{l-1} D_l), bf16 M_l,
+the RMS statistic) are checked stage by stage.
 """
 import numpy as np
 import pytest
@@ -40,8 +41,13 @@ def _full_check(inp, label, **kw):
     return gu.assert_parity(gk, gv, ref["k"], ref["v"], cfg.head_dim, label), (k, v, plan)
 
 
-def test_recurrent_tiny():
-    _full_check(synth.make_inputs(_rec(synth.CONFIGS["tiny"])), "recurrent tiny")
+PATHS = ["chain", "rearranged"]
+
+
+@pytest.mark.parametrize("path", PATHS)
+def test_recurrent_tiny(path):
+    _full_check(synth.make_inputs(_rec(synth.CONFIGS["tiny"], recurrent_path=path)),
+                f"recurrent tiny, {path}")
 
 
 def test_recurrent_zero_up_equals_embedding_build():
@@ -59,44 +65,51 @@ def test_recurrent_zero_up_equals_embedding_build():
     assert float((vr.float() - ve.float()).abs().max()) <= 2e-2 * float(ve.float().abs().max())
 
 
+@pytest.mark.parametrize("path", PATHS)
 @pytest.mark.parametrize("rank,d,splits_hint", [(16, 512, "r_pad 64"), (80, 1024, "r_pad 128"),
                                                 (150, 768, "r_pad 192"), (256, 512, "r_pad 256")])
-def test_recurrent_every_rank_padding(rank, d, splits_hint):
+def test_recurrent_every_rank_padding(rank, d, splits_hint, path):
     # 300 tokens in 2 batch elements: 3 token blocks (ragged), K split over the cluster.
     cfg = gu.small_config(f"rec_r{rank}", d=d, n_layers=3, n_kv_heads=2, n_heads=4, head_dim=128,
                           rank=rank, n_vis=150, batch=2, x0_sigma=0.5, w_sigma=0.05, seed=50 + rank,
                           pos_start=35, adapter="recurrent")
-    _full_check(synth.make_inputs(cfg), f"recurrent {splits_hint}")
+    _full_check(synth.make_inputs(_rec(cfg, recurrent_path=path)), f"recurrent {splits_hint}, {path}")
 
 
-def test_recurrent_tokens_as_m_mrope_bias():
+@pytest.mark.parametrize("path", PATHS)
+def test_recurrent_tokens_as_m_mrope_bias(path):
     # T = 2 x 256: the K/V launch takes the tokens-as-M engine over the stacked M_l.
     cfg = gu.small_config("rec_tm", d=512, n_layers=3, n_kv_heads=2, n_heads=8, head_dim=128,
                           rank=64, n_vis=256, batch=2, rope="mrope", rope_theta=1e6,
                           mrope_section=(16, 24, 24), grid=(1, 16, 16), x0_sigma=0.5,
                           bias_sigma=0.02, w_sigma=0.05, seed=61, pos_start=15,
                           adapter="recurrent")
-    _full_check(synth.make_inputs(cfg), "recurrent tokens-as-M")
+    _full_check(synth.make_inputs(_rec(cfg, recurrent_path=path)), f"recurrent tokens-as-M, {path}")
 
 
-def test_recurrent_long_chain_head64():
+@pytest.mark.parametrize("path", PATHS)
+def test_recurrent_long_chain_head64(path):
     # 12 layers of 8 x 64 heads: the state passes through many steps.
-    cfg = synth.config("tiny", n_layers=12, n_vis=200, w_sigma=0.05, seed=62, adapter="recurrent")
-    _full_check(synth.make_inputs(cfg), "recurrent 12 layers")
+    cfg = synth.config("tiny", n_layers=12, n_vis=200, w_sigma=0.05, seed=62, adapter="recurrent",
+                       recurrent_path=path)
+    _full_check(synth.make_inputs(cfg), f"recurrent 12 layers, {path}")
 
 
-def test_recurrent_rebuild_is_deterministic():
-    # The split-K partials are summed in a fixed order: two builds agree bit for bit.
+@pytest.mark.parametrize("path", PATHS)
+def test_recurrent_rebuild_is_deterministic(path):
+    # Every sum runs in a fixed order: two builds agree bit for bit.
     import torch
     cfg = gu.small_config("rec_det", d=1024, n_layers=2, n_kv_heads=2, n_heads=4, head_dim=128,
                           rank=64, n_vis=200, batch=1, x0_sigma=0.5, seed=63, adapter="recurrent")
+    cfg = _rec(cfg, recurrent_path=path)
     inp = synth.make_inputs(cfg)
     k1, v1, plan = gu.run_build(inp)
     k2, v2, _ = gu.run_build(inp, plan=plan)
     assert torch.equal(k1, k2) and torch.equal(v1, v2)
 
 
-def test_recurrent_stages():
+@pytest.mark.parametrize("path", PATHS)
+def test_recurrent_stages(path):
     # H_l = bf16(SiLU(M_{l-1} D_l)), bf16 M_l and rstd_l = 1 / sqrt(mean(M_l^2) + eps) of the
     # chain against the oracle's fp64 chain.
     import torch
@@ -104,6 +117,7 @@ def test_recurrent_stages():
     cfg = gu.small_config("rec_stage", d=1024, n_layers=3, n_kv_heads=2, n_heads=4, head_dim=128,
                           rank=80, n_vis=300, batch=1, x0_sigma=0.5, w_sigma=0.05, seed=64,
                           adapter="recurrent")
+    cfg = _rec(cfg, recurrent_path=path)
     inp = synth.make_inputs(cfg)
     k, v, plan = gu.run_build(inp)
     H, rstd, _, r_pad = dv.debug_workspace(plan, cfg.tokens)
@@ -126,11 +140,12 @@ def test_recurrent_stages():
     dv.free(plan)
 
 
-def test_recurrent_layer_modes():
+@pytest.mark.parametrize("path", PATHS)
+def test_recurrent_layer_modes(path):
     # IDENTITY and DROP both pass the state on unchanged (M_l = M_{l-1}); DROP writes no K/V.
     # The oracle sees zero D_l, U_l at those layers and is compared on the kept ones.
     import torch
-    cfg = _rec(synth.config("tiny", n_vis=100, w_sigma=0.05, seed=65))
+    cfg = _rec(synth.config("tiny", n_vis=100, w_sigma=0.05, seed=65), recurrent_path=path)
     inp = synth.make_inputs(cfg)
     modes = [1, 0, 2, 0]
     k, v, plan = gu.run_build(inp, fill=-5.0, layer_modes=modes)
@@ -149,9 +164,10 @@ def test_recurrent_layer_modes():
     assert bool((k[2] == -5.0).all()) and bool((v[2] == -5.0).all())
 
 
-def test_recurrent_noalloc_entry():
+@pytest.mark.parametrize("path", PATHS)
+def test_recurrent_noalloc_entry(path):
     import torch
-    inp = synth.make_inputs(_rec(synth.config("tiny", n_vis=64, seed=66)))
+    inp = synth.make_inputs(_rec(synth.config("tiny", n_vis=64, seed=66), recurrent_path=path))
     k1, v1, plan = gu.run_build(inp)
     k2, v2, _ = gu.run_build(inp, plan=plan, noalloc=True)
     assert torch.equal(k1, k2) and torch.equal(v1, v2)
