@@ -173,17 +173,19 @@ def test_recurrent_noalloc_entry(path):
     assert torch.equal(k1, k2) and torch.equal(v1, v2)
 
 
+@pytest.mark.parametrize("path", ["auto", "chain"])
 @pytest.mark.parametrize("name", ["llava15_7b", "qwen25vl_7b_image", "llava_next_7b",
                                   "qwen25vl_7b_video"])
-def test_recurrent_full_size_sampled(name):
+def test_recurrent_full_size_sampled(name, path):
+    # "auto" takes the rearranged chain for all but the LLaVA-1.5 shape; "chain" the paper's order
     import torch
-    cfg = _rec(synth.CONFIGS[name])
+    cfg = _rec(synth.CONFIGS[name], recurrent_path=path)
     inp = synth.make_inputs(cfg)
     k, v, plan = gu.run_build(inp)
     toks = gu.sample_tokens(cfg.tokens, n=24, seed=2)
     ref = oracle.build_tokens(inp, toks)
     gk, gv = gu.gather(k, cfg, toks), gu.gather(v, cfg, toks)
-    gu.assert_parity(gk, gv, ref["k"], ref["v"], cfg.head_dim, name + " recurrent")
+    gu.assert_parity(gk, gv, ref["k"], ref["v"], cfg.head_dim, f"{name} recurrent, {path}")
     assert bool(torch.isfinite(k).all()) and bool(torch.isfinite(v).all())
     del k, v, plan
     torch.cuda.empty_cache()
