@@ -81,7 +81,7 @@ enum {
  *   adapter in {DV_ADAPTER_EMBEDDING, DV_ADAPTER_RECURRENT};
  *   split_chain in {0, 1}, and 1 only with DV_ADAPTER_RECURRENT;
  *   recurrent_path a DV_RECURRENT_* value, not AUTO only with DV_ADAPTER_RECURRENT,
- *   REARRANGED not with split_chain (DV_ERR_INVALID_ARG) and only with d % 128 == 0;
+ *   REARRANGED only with d % 128 == 0;
  *   max_batch * max_n_vis >= 1 and <= 2^24 (the tokens one build may carry). */
 typedef struct dv_config {
   int d;                 /* hidden size of the language model */
@@ -106,15 +106,17 @@ typedef struct dv_config {
                             chain's two GEMMs (M_{l-1} into the down-projection, h_l into the
                             up-projection) is read as a high and a low bf16 part, two MMAs per
                             product, so the state M_l keeps about fp32 accuracy through deep
-                            chains; the chain then runs on chip only at rank <= 64 (where
-                            the on-chip chain fits d at all), else as per-layer launches.
-                            0 = one bf16 operand (faster): builds whose 128-token blocks fit in
-                            one wave of on-chip chain clusters run the chain, larger ones (and
-                            every build at rank > 128) the rearranged chain, which forms each
-                            layer's down-projection input from E D_l^T and the earlier h_j
-                            through the r x r products D_l U_j (exactly the same sum). */
+                            chains (in the rearranged chain: h_j and the products D_l U_j in two
+                            parts each); the chain in the paper's order then runs on chip only
+                            at rank <= 64, else as per-layer launches.
+                            0 = one bf16 operand (faster).
+                            Either way, with DV_RECURRENT_AUTO, builds whose 128-token blocks fit
+                            in one wave of on-chip chain clusters run the chain, larger ones (and
+                            every build the on-chip chain does not fit) the rearranged chain,
+                            which forms each layer's down-projection input from E D_l^T and the
+                            earlier h_j through the r x r products D_l U_j (the same sum). */
   int recurrent_path;    /* recurrent adapter only: DV_RECURRENT_AUTO (0), _CHAIN or
-                            _REARRANGED; the split chain always takes the chain's path */
+                            _REARRANGED */
 } dv_config;
 
 /* Weights of all L layers, bf16, device pointers. Read only during dv_memory_plan: the plan

@@ -41,6 +41,7 @@ struct dv_plan {
   uint16_t* Uup = nullptr;     // recurrent adapter: U_l as [L*d][uup_ld] (split chain: [U_l | U_l])
   uint16_t* Pf = nullptr;      // recurrent adapter, refactored chain: [L*r_pad][L*r_pad]
                                // (k_fold_products), or null
+  uint16_t* Pf_lo = nullptr;   // its low bf16 part with split_chain, or null
   bool fold = false;           // recurrent builds may run the refactored chain (dv_fold.cu)
   int chain_clusters = 0;      // recurrent: clusters of the on-chip chain resident at once
   int uup_ld = 0;              // r_pad, or 2 r_pad with the split chain
@@ -58,7 +59,7 @@ struct dv_plan {
   CUtensorMap tm_Bn_half;      // slab map, boxes of 128 rows (CTA-pair halves)
   CUtensorMap tm_Wkv;          // slab map, boxes of 128 rows
   CUtensorMap tm_Dst_rp, tm_Uup;  // recurrent adapter
-  CUtensorMap tm_Pf;              // recurrent adapter: Pf with r_pad-row boxes
+  CUtensorMap tm_Pf, tm_Pf_lo;    // recurrent adapter: Pf (and Pf_lo) with r_pad-row boxes
   int resid_bn = 0;
   double inv_freq[dv::kMaxHalfHead];
   unsigned char mode[dv::kMaxLayers];  // DV_LAYER_* per layer
@@ -358,13 +359,15 @@ __global__ void k_bias_to_f32(const uint16_t* __restrict__ b, float* __restrict_
 
 // Recurrent adapter, refactored chain (dv_fold.cu). Pf [L r_pad][L r_pad]: row i r_pad + a,
 // columns j r_pad + b with j < i hold bf16 of Q_ij[a][b] = sum_e D_i[a][e] U_j[e][b] (a, b < r;
-// zero where layer i or j is an identity layer); the caller zeroes the rest.
+// zero where layer i or j is an identity layer), and Pf_lo (split chain, or null) the bf16 of
+// Q_ij - bf16(Q_ij); the caller zeroes the rest.
 // Q_ij blocks: grid (r_pad / 64 b-tiles, (L) * (r_pad / 64) (j, a-tile), L (i)); blocks with
 // j >= i return. 64 x 64 outputs per block, 256 threads with 4 x 4 each, fp32 accumulation
 // over e in steps of 32 (a fixed order).
 __global__ void __launch_bounds__(256) k_fold_products(const uint16_t* __restrict__ D,
                                                        const uint16_t* __restrict__ U,
-                                                       uint16_t* __restrict__ Pf, int L, int r,
+                                                       uint16_t* __restrict__ Pf,
+                                                       uint16_t* __restrict__ Pf_lo, int L, int r,
                                                        int r_pad, int d, long long pld,
                                                        PackLayers pl) {
   const int at_n = r_pad / 64;
@@ -406,8 +409,12 @@ __global__ void __launch_bounds__(256) k_fold_products(const uint16_t* __restric
   for (int q = 0; q < 4; ++q) {
     const long long row = static_cast<long long>(i) * r_pad + a0 + ty * 4 + q;
 #pragma unroll
-    for (int w = 0; w < 4; ++w)
-      Pf[row * pld + static_cast<long long>(j) * r_pad + b0 + tx * 4 + w] = to_bf16(acc[q][w]);
+    for (int w = 0; w < 4; ++w) {
+      const long long e = row * pld + static_cast<long long>(j) * r_pad + b0 + tx * 4 + w;
+      const uint16_t hi = to_bf16(acc[q][w]);
+      Pf[e] = hi;
+      if (Pf_lo) Pf_lo[e] = to_bf16(acc[q][w] - bf(hi));  // split: the remainder, in bf16
+    }
   }
 }
 
@@ -652,7 +659,6 @@ int check_config(const dv_config* c) {
     return DV_ERR_INVALID_ARG;
   if (c->recurrent_path != DV_RECURRENT_AUTO && c->adapter != DV_ADAPTER_RECURRENT)
     return DV_ERR_INVALID_ARG;
-  if (c->recurrent_path == DV_RECURRENT_REARRANGED && c->split_chain) return DV_ERR_INVALID_ARG;
   if (c->recurrent_path == DV_RECURRENT_REARRANGED && dv::fold_slice_cols(c->d) == 0)
     return DV_ERR_UNSUPPORTED_SHAPE;
   if (c->d % 64 != 0 || c->d > 16384) return DV_ERR_UNSUPPORTED_SHAPE;
@@ -674,7 +680,8 @@ int check_config(const dv_config* c) {
 }
 
 void free_plan_memory(dv_plan* p) {
-  void* ptrs[] = {p->Dst, p->Bn, p->Wkv, p->Uup, p->Pf, p->bk, p->bv, p->kg, p->Gf, p->ws, p->status};
+  void* ptrs[] = {p->Dst, p->Bn, p->Wkv, p->Uup, p->Pf, p->Pf_lo, p->bk, p->bv, p->kg, p->Gf,
+                  p->ws, p->status};
   for (void* q : ptrs)
     if (q) cudaFree(q);
   for (cudaEvent_t e : p->ev) cudaEventDestroy(e);
@@ -837,7 +844,8 @@ static cudaError_t enqueue_fold(const PlanView& v, const BuildArgs& a, cudaStrea
   auto mark = [&](int i) {
     if (a.marks) cudaEventRecord(a.marks[i], st);
   };
-  const uint32_t ks = static_cast<uint32_t>(hchain_box_slabs(v.r_pad));
+  const bool split = v.split_chain != 0;
+  const uint32_t ks = static_cast<uint32_t>(hchain_box_slabs(v.r_pad, split));
   CUtensorMap tm_x0, tm_x0_s, tm_hs, tm_h, tm_u, tm_mem_s;
   if (!encode_2d(&tm_x0, a.x0, d, static_cast<uint64_t>(T), d, kBlockM) ||
       !encode_slabs(&tm_x0_s, a.x0, d, static_cast<uint64_t>(T), d, kBlockM) ||
@@ -846,6 +854,12 @@ static cudaError_t enqueue_fold(const PlanView& v, const BuildArgs& a, cudaStrea
       !encode_2d(&tm_u, v.Uup, v.r_pad, static_cast<uint64_t>(L) * d, v.uup_ld, cw) ||
       !encode_slabs(&tm_mem_s, a.mem, d, static_cast<uint64_t>(L) * T, d, kBlockM))
     return cudaErrorInvalidValue;
+  // split chain: the low parts of h (its own buffer, H's pitch) and of the products
+  CUtensorMap tm_hlo_s = tm_hs, tm_hlo = tm_h;
+  if (split && (!encode_slabs(&tm_hlo_s, a.Hlo, n1, static_cast<uint64_t>(T), a.hld, kBlockM, ks) ||
+                !encode_2d(&tm_hlo, a.Hlo, n1, static_cast<uint64_t>(T), a.hld, kBlockM)))
+    return cudaErrorInvalidValue;
+  const CUtensorMap& tm_pf_lo = split ? *v.tm_Pf_lo : *v.tm_Pf;
   mark(0);
   // (1) C = E [D_1 .. D_L]^T, every column in fp32
   GemmParams gp;
@@ -882,11 +896,12 @@ static cudaError_t enqueue_fold(const PlanView& v, const BuildArgs& a, cudaStrea
   // (2) the recurrence over the rank-r vectors, (3) the running sum of the memories
   const long long part_ld = static_cast<long long>(d / 64) * T;
   if (err == cudaSuccess)
-    err = launch_hchain(v.r_pad, T, L, a.c, static_cast<int>(n1), tm_hs, *v.tm_Pf, a.H,
-                        static_cast<int>(a.hld), v.status, kTimeoutNs, st);
+    err = launch_hchain(v.r_pad, split, T, L, a.c, static_cast<int>(n1), tm_hs, tm_hlo_s, *v.tm_Pf,
+                        tm_pf_lo, a.H, split ? a.Hlo : nullptr, static_cast<int>(a.hld), v.status,
+                        kTimeoutNs, st);
   if (err == cudaSuccess)
-    err = launch_accum(v.r_pad, cw, T, L, d, a.x0, tm_h, tm_u, a.mem, a.part, part_ld, v.status,
-                       kTimeoutNs, st);
+    err = launch_accum(v.r_pad, cw, T, L, d, a.x0, tm_h, tm_hlo, split, tm_u, a.mem, a.part, part_ld,
+                       v.status, kTimeoutNs, st);
   mark(2);
   if (err == cudaSuccess)
     err = launch_pdl(k_rstd_parts, dim3(grid_for(static_cast<long long>(L) * T)), dim3(256), st,
@@ -1222,6 +1237,7 @@ bool plan_view(const dv_plan* p, PlanView* v) {
   v->tm_Uup = &p->tm_Uup;
   v->Uup = p->Uup;
   v->tm_Pf = p->fold ? &p->tm_Pf : nullptr;
+  v->tm_Pf_lo = p->fold && c.split_chain ? &p->tm_Pf_lo : nullptr;
   v->chain_clusters = p->chain_clusters;
   v->uup_ld = p->uup_ld;
   v->split_chain = p->cfg.split_chain;
@@ -1272,9 +1288,10 @@ cudaError_t preload_build_kernels(const dv_plan* p) {
   for (int nt : {64, 128, 192, 256}) keep(dv::launch_kv_pair(hd, nt, m, m, m, gp, 1, nullptr));
   if (p->fold) {
     const int cw = dv::fold_slice_cols(p->cfg.d);
-    keep(dv::launch_hchain(p->r_pad, 0, 1, nullptr, 0, m, m, nullptr, 0, nullptr, 0, nullptr));
-    keep(dv::launch_accum(p->r_pad, cw, 0, 1, p->cfg.d, nullptr, m, m, nullptr, nullptr, 0, nullptr,
-                          0, nullptr));
+    keep(dv::launch_hchain(p->r_pad, p->cfg.split_chain != 0, 0, 1, nullptr, 0, m, m, m, m, nullptr,
+                           nullptr, 0, nullptr, 0, nullptr));
+    keep(dv::launch_accum(p->r_pad, cw, 0, 1, p->cfg.d, nullptr, m, m, false, m, nullptr, nullptr, 0,
+                          nullptr, 0, nullptr));
   }
   if (p->cfg.adapter == DV_ADAPTER_RECURRENT) {
     dv::DownParams dp;
@@ -1376,10 +1393,9 @@ int dv_memory_plan(const dv_config* cfg, const dv_weights* w, void* stream, dv_p
   p->uup_ld = cfg->split_chain ? 2 * p->r_pad : p->r_pad;
   p->max_tokens = cfg->max_batch * cfg->max_n_vis;
   const long long T = p->max_tokens;
-  // Recurrent adapter: the refactored chain (dv_fold.cu) unless the split chain is asked for;
-  // builds whose token blocks fit in one wave of on-chip chain clusters take the chain instead.
-  p->fold = rec && !cfg->split_chain && dv::fold_slice_cols(d) > 0 &&
-            cfg->recurrent_path != DV_RECURRENT_CHAIN;
+  // Recurrent adapter: the refactored chain (dv_fold.cu); builds whose token blocks fit in one
+  // wave of on-chip chain clusters take the chain instead (DV_RECURRENT_AUTO).
+  p->fold = rec && dv::fold_slice_cols(d) > 0 && cfg->recurrent_path != DV_RECURRENT_CHAIN;
   p->chain_clusters = rec && cfg->recurrent_path != DV_RECURRENT_REARRANGED
                           ? dv::chain_resident_clusters(d, p->r_pad, cfg->split_chain != 0)
                           : 0;
@@ -1411,6 +1427,7 @@ int dv_memory_plan(const dv_config* cfg, const dv_weights* w, void* stream, dv_p
   if (ok && !rec) ok = dmalloc(&p->Gf, sizeof(float) * L * p->r_pad * p->r_pad);
   const size_t pf_bytes = sizeof(uint16_t) * static_cast<size_t>(L) * p->r_pad * pf_ld;
   if (ok && p->fold) ok = dmalloc(&p->Pf, pf_bytes);
+  if (ok && p->fold && cfg->split_chain) ok = dmalloc(&p->Pf_lo, pf_bytes);
   if (!ok) {
     free_plan_memory(p);
     delete p;
@@ -1438,9 +1455,10 @@ int dv_memory_plan(const dv_config* cfg, const dv_weights* w, void* stream, dv_p
                                                                  p->uup_ld, pl);
     if (p->fold) {
       cudaMemsetAsync(p->Pf, 0, pf_bytes, st);
+      if (p->Pf_lo) cudaMemsetAsync(p->Pf_lo, 0, pf_bytes, st);
       if (L > 1) {
         const dim3 gq(p->r_pad / 64, L * (p->r_pad / 64), L);
-        k_fold_products<<<gq, 256, 0, st>>>(D, U, p->Pf, L, r, p->r_pad, d, pf_ld, pl);
+        k_fold_products<<<gq, 256, 0, st>>>(D, U, p->Pf, p->Pf_lo, L, r, p->r_pad, d, pf_ld, pl);
       }
     }
   } else {
@@ -1485,7 +1503,10 @@ int dv_memory_plan(const dv_config* cfg, const dv_weights* w, void* stream, dv_p
           encode_2d(&p->tm_Uup, p->Uup, p->uup_ld, 1ull * L * d, p->uup_ld, p->resid_bn);
     if (enc && p->fold)
       enc = encode_slabs(&p->tm_Pf, p->Pf, pf_ld, 1ull * L * p->r_pad, pf_ld, p->r_pad,
-                         static_cast<uint32_t>(dv::hchain_box_slabs(p->r_pad)));
+                         static_cast<uint32_t>(dv::hchain_box_slabs(p->r_pad, cfg->split_chain)));
+    if (enc && p->Pf_lo)
+      enc = encode_slabs(&p->tm_Pf_lo, p->Pf_lo, pf_ld, 1ull * L * p->r_pad, pf_ld, p->r_pad,
+                         static_cast<uint32_t>(dv::hchain_box_slabs(p->r_pad, true)));
   } else if (enc) {
     enc = encode_slabs(&p->tm_Bn_half, p->Bn, p->bn_k, 256ull * p->bn_groups, p->bn_k, 128) &&
           encode_2d(&p->tm_Bn, p->Bn, p->bn_k, 256ull * p->bn_groups, p->bn_k, 256);

@@ -67,7 +67,7 @@ __device__ __forceinline__ void tma_load_slabs(uint32_t dst, const CUtensorMap* 
       : "memory");
 }
 
-template <int RP, int KS, int STAGES>
+template <int RP, int KS, int STAGES, bool SPLIT>
 struct HCfg {
   static constexpr int R = RP / 64;              // 64-wide K slabs per r_pad
   static constexpr int kSlabB = RP * 128;        // [RP rows of Pf][64] bf16
@@ -75,7 +75,8 @@ struct HCfg {
   static constexpr int kB = KS * kSlabB;         // one box of KS slabs of B
   static constexpr int kStage = kA + kB;
   static constexpr int kOffH = STAGES * kStage;  // h_{l-1} as the A operand of layer l's last slabs
-  static constexpr int kEnd = kOffH + R * kSlabA;
+  static constexpr int kOffL = kOffH + R * kSlabA;  // split: the low part of h_{l-1}
+  static constexpr int kEnd = kOffL + (SPLIT ? R * kSlabA : 0);
   static constexpr int kSmemBytes = kEnd + 1024 + 256;
   static constexpr int kTmemCols = 2 * RP <= 128 ? 128 : (2 * RP <= 256 ? 256 : 512);
   static_assert(kSlabB % 1024 == 0, "stage tiles stay 1024-byte aligned");
@@ -88,19 +89,32 @@ struct HChainParams {
   const float* C;  // fp32 [M][ldc]: E D_l^T at columns l r_pad
   int ldc;
   uint16_t* H;     // bf16 [M][ldh]: h_l at columns l r_pad
+  uint16_t* Hlo;   // split: bf16(h_l - bf16(h_l)), the same layout; else null
   int ldh;
   int* status;
   unsigned long long timeout_ns;
 };
 
 // Segment `seg` of layer l's K loop (l >= 1): n slabs, the first at slab a0 of its A source and
-// at slab b0 of the layer's rows of Pf. 0: h_0 .. h_{l-2} (A: H), 1: h_{l-1} (A: the h tile).
+// at slab b0 of the layer's rows of its B source. A: 0 H, 1 Hlo, 2 the h tile, 3 the low h tile;
+// B: 0 Pf, 1 Pf_lo. h_0 .. h_{l-2} come from global memory (A 0 / 1), h_{l-1} from the tiles the
+// epilogue has just written (A 2 / 3). Without the split: (H, Pf), (h tile, Pf). With it, each
+// product in three parts, h_hi Q_hi + h_lo Q_hi + h_hi Q_lo, for the older h_j and for h_{l-1}.
 struct HSeg {
-  int n, a0, b0;
+  int n, a0, b0, asrc, bsrc;
 };
+template <bool SPLIT>
 __device__ __forceinline__ HSeg hseg(int l, int seg, int R) {
-  if (seg == 0) return {l >= 2 ? (l - 1) * R : 0, 0, 0};
-  return {R, 0, (l - 1) * R};
+  const int n_old = l >= 2 ? (l - 1) * R : 0, b_new = (l - 1) * R;
+  if (!SPLIT) return seg == 0 ? HSeg{n_old, 0, 0, 0, 0} : HSeg{R, 0, b_new, 2, 0};
+  switch (seg) {
+    case 0: return {n_old, 0, 0, 0, 0};
+    case 1: return {n_old, 0, 0, 1, 0};
+    case 2: return {n_old, 0, 0, 0, 1};
+    case 3: return {R, 0, b_new, 2, 0};
+    case 4: return {R, 0, b_new, 3, 0};
+    default: return {R, 0, b_new, 2, 1};
+  }
 }
 
 // One CTA per 128-token block, all layers. Layer l's accumulator starts as C_l, written into TMEM
@@ -119,11 +133,14 @@ __device__ __forceinline__ HSeg hseg(int l, int seg, int R) {
 // layer parity so that the producer, which may run up to two layers ahead of the epilogue, never
 // waits on a phase that has wrapped. The accumulator barriers of layer l complete for the
 // ((l - 1) / 2)-th time (integer division) at that layer, on accumulator l mod 2.
-template <int RP, int KS, int STAGES>
+template <int RP, int KS, int STAGES, bool SPLIT>
 __global__ void __launch_bounds__(kFoldThreads, 1)
-    dv_hchain_kernel(const __grid_constant__ CUtensorMap tmH, const __grid_constant__ CUtensorMap tmP,
+    dv_hchain_kernel(const __grid_constant__ CUtensorMap tmH, const __grid_constant__ CUtensorMap tmHlo,
+                     const __grid_constant__ CUtensorMap tmP, const __grid_constant__ CUtensorMap tmPlo,
                      const __grid_constant__ HChainParams p) {
-  using C = HCfg<RP, KS, STAGES>;
+  using C = HCfg<RP, KS, STAGES, SPLIT>;
+  constexpr int kSegs = SPLIT ? 6 : 2;
+  constexpr int kFirstNew = SPLIT ? 3 : 1;  // the first segment that reads the h tiles
   constexpr int R = C::R;
   extern __shared__ uint8_t smem_raw[];
   const uint32_t raw = smem_addr(smem_raw);
@@ -140,7 +157,7 @@ __global__ void __launch_bounds__(kFoldThreads, 1)
   const uint32_t drain_bar = bar0 + 8u * (2 * STAGES + 7);
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 2 * STAGES + 8);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
-  const uint32_t ring = base, htile = base + C::kOffH;
+  const uint32_t ring = base, htile = base + C::kOffH, ltile = base + C::kOffL;
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const uint64_t tmo = p.timeout_ns;
@@ -164,6 +181,10 @@ __global__ void __launch_bounds__(kFoldThreads, 1)
   if (warp == 0 && lane == 0) {
     tma_prefetch_desc(&tmH);
     tma_prefetch_desc(&tmP);
+    if (SPLIT) {
+      tma_prefetch_desc(&tmHlo);
+      tma_prefetch_desc(&tmPlo);
+    }
   }
   if (warp == 1) {
     tmem_alloc(smem_addr(tmem_slot), C::kTmemCols);
@@ -183,10 +204,10 @@ __global__ void __launch_bounds__(kFoldThreads, 1)
       uint32_t phase = 0, used = 0, issued_parity = 0;
       bool ok = true;
       for (int l = 1; l < p.L && ok; ++l) {
-        for (int seg = 0; seg < 2 && ok; ++seg) {
-          const HSeg g = hseg(l, seg, R);
-          // h_{l-2} is the newest layer segment 0 reads: wait until it is in global memory (the
-          // layers before it were published earlier)
+        for (int seg = 0; seg < kSegs && ok; ++seg) {
+          const HSeg g = hseg<SPLIT>(l, seg, R);
+          // h_{l-2} is the newest layer the older segments read: wait until it is in global
+          // memory (the layers before it were published earlier)
           if (seg == 0 && g.n > 0 &&
               !mbar_wait(hpub_bar((l - 2) & 1), static_cast<uint32_t>((l - 2) >> 1) & 1u, abort_flag,
                          tmo)) {
@@ -199,9 +220,10 @@ __global__ void __launch_bounds__(kFoldThreads, 1)
               break;
             }
             const uint32_t a_dst = ring + stage * C::kStage, b_dst = a_dst + C::kA;
-            mbar_arrive_expect_tx(full_bar(stage), seg == 1 ? C::kB : C::kStage);
-            if (seg == 0) tma_load_slabs(a_dst, &tmH, full_bar(stage), row0, g.a0 + s0);
-            tma_load_slabs(b_dst, &tmP, full_bar(stage), l * RP, g.b0 + s0);
+            mbar_arrive_expect_tx(full_bar(stage), g.asrc >= 2 ? C::kB : C::kStage);
+            if (g.asrc < 2)
+              tma_load_slabs(a_dst, g.asrc == 0 ? &tmH : &tmHlo, full_bar(stage), row0, g.a0 + s0);
+            tma_load_slabs(b_dst, g.bsrc == 0 ? &tmP : &tmPlo, full_bar(stage), l * RP, g.b0 + s0);
             used |= 1u << stage;
             issued_parity = (issued_parity & ~(1u << stage)) | (phase << stage);
             if (++stage == STAGES) {
@@ -229,9 +251,10 @@ __global__ void __launch_bounds__(kFoldThreads, 1)
         if (!mbar_wait(init_bar(acc), par, abort_flag, tmo)) break;  // C_l is in the accumulator
         tc_fence_after();
         const uint32_t d_tmem = tmem + static_cast<uint32_t>(acc * RP);
-        for (int seg = 0; seg < 2 && ok; ++seg) {
-          const HSeg g = hseg(l, seg, R);
-          if (seg == 1 && !mbar_wait(htile_bar, static_cast<uint32_t>(l - 1) & 1u, abort_flag, tmo)) {
+        for (int seg = 0; seg < kSegs && ok; ++seg) {
+          const HSeg g = hseg<SPLIT>(l, seg, R);
+          if (seg == kFirstNew &&
+              !mbar_wait(htile_bar, static_cast<uint32_t>(l - 1) & 1u, abort_flag, tmo)) {
             ok = false;
             break;
           }
@@ -244,8 +267,9 @@ __global__ void __launch_bounds__(kFoldThreads, 1)
             const uint32_t st = ring + stage * C::kStage;
             const int n_use = g.n - s0 < KS ? g.n - s0 : KS;
             for (int u = 0; u < n_use; ++u) {
-              const uint32_t a_s = seg == 1 ? htile + static_cast<uint32_t>((s0 + u) * kSlabA)
-                                            : st + static_cast<uint32_t>(u * kSlabA);
+              const uint32_t a_s =
+                  g.asrc >= 2 ? (g.asrc == 2 ? htile : ltile) + static_cast<uint32_t>((s0 + u) * kSlabA)
+                              : st + static_cast<uint32_t>(u * kSlabA);
               const uint32_t b_s = st + C::kA + static_cast<uint32_t>(u * C::kSlabB);
 #pragma unroll
               for (int k = 0; k < 4; ++k)
@@ -277,6 +301,7 @@ __global__ void __launch_bounds__(kFoldThreads, 1)
     const uint32_t tl = tmem + (static_cast<uint32_t>(qq * 32) << 16);
     const float* crow = p.C + static_cast<long long>(live ? t : 0) * p.ldc;
     uint8_t* hrow = base_ptr + C::kOffH;
+    uint8_t* lrow = base_ptr + C::kOffL;
     // this row's 32 columns c*32 .. of C_lc (zero past the build's tokens)
     auto load_c = [&](int lc, int c, uint32_t (&r)[32]) {
       const float4* src = reinterpret_cast<const float4*>(crow + lc * RP + c * 32);
@@ -302,17 +327,24 @@ __global__ void __launch_bounds__(kFoldThreads, 1)
       tc_fence_before();
       mbar_arrive(init_bar(a));
     };
-    // SiLU of the 32 columns c*32 .. of z into the h tile (bf16, swizzled as the MMA reads it)
+    // SiLU of the 32 columns c*32 .. of z into the h tile (bf16, swizzled as the MMA reads it);
+    // split: the remainder h - bf16(h), itself in bf16, into the low tile
     auto put_h = [&](int c, const uint32_t (&r)[32]) {
-      uint32_t pk[16];
+      uint32_t pk[16], lo[16];
 #pragma unroll
-      for (int v = 0; v < 16; ++v)
-        pk[v] = pack_bf16x2(silu(__uint_as_float(r[2 * v])), silu(__uint_as_float(r[2 * v + 1])));
-      uint8_t* slab = hrow + (c / 2) * kSlabA;
+      for (int v = 0; v < 16; ++v) {
+        const float a = silu(__uint_as_float(r[2 * v])), b = silu(__uint_as_float(r[2 * v + 1]));
+        pk[v] = pack_bf16x2(a, b);
+        if (SPLIT)
+          lo[v] = pack_bf16x2(a - __uint_as_float(pk[v] << 16), b - __uint_as_float(pk[v] & 0xFFFF0000u));
+      }
 #pragma unroll
-      for (int k = 0; k < 4; ++k)
-        *reinterpret_cast<uint4*>(slab + swz(row, (c % 2) * 4 + k)) =
-            make_uint4(pk[4 * k], pk[4 * k + 1], pk[4 * k + 2], pk[4 * k + 3]);
+      for (int k = 0; k < 4; ++k) {
+        const uint32_t off = static_cast<uint32_t>((c / 2) * kSlabA) + swz(row, (c % 2) * 4 + k);
+        *reinterpret_cast<uint4*>(hrow + off) = make_uint4(pk[4 * k], pk[4 * k + 1], pk[4 * k + 2], pk[4 * k + 3]);
+        if (SPLIT)
+          *reinterpret_cast<uint4*>(lrow + off) = make_uint4(lo[4 * k], lo[4 * k + 1], lo[4 * k + 2], lo[4 * k + 3]);
+      }
     };
     for (int l = 0; l < p.L; ++l) {
       if (l == 0) {  // z_0 = C_0
@@ -342,10 +374,17 @@ __global__ void __launch_bounds__(kFoldThreads, 1)
       asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
       mbar_arrive(htile_bar);
       if (live) {
-        uint4* hg = reinterpret_cast<uint4*>(p.H + static_cast<long long>(t) * p.ldh + l * RP);
+        const long long go = static_cast<long long>(t) * p.ldh + l * RP;
+        uint4* hg = reinterpret_cast<uint4*>(p.H + go);
 #pragma unroll 1
         for (int c8 = 0; c8 < RP / 8; ++c8)
           hg[c8] = *reinterpret_cast<const uint4*>(hrow + (c8 / 8) * kSlabA + swz(row, c8 % 8));
+        if (SPLIT) {
+          uint4* lg = reinterpret_cast<uint4*>(p.Hlo + go);
+#pragma unroll 1
+          for (int c8 = 0; c8 < RP / 8; ++c8)
+            lg[c8] = *reinterpret_cast<const uint4*>(lrow + (c8 / 8) * kSlabA + swz(row, c8 % 8));
+        }
       }
       asm volatile("fence.proxy.async.global;" ::: "memory");
       mbar_arrive(hpub_bar(l & 1));
@@ -392,6 +431,7 @@ struct AccumParams {
   uint16_t* mem;       // bf16 [L][M][d]: the stacked M_l
   float* part;         // fp32 [L][part_ld / M][M]: sums of squares of M_l per slice
   long long part_ld;
+  int split;           // 1: h_l in two bf16 parts (H, then Hlo), both against U_l
   int* status;
   unsigned long long timeout_ns;
 };
@@ -405,10 +445,11 @@ struct AccumParams {
 // other block's readback and stores go on.
 template <int RP, int CW, int STAGES>
 __global__ void __launch_bounds__(kFoldThreads, 1)
-    dv_accum_kernel(const __grid_constant__ CUtensorMap tmH, const __grid_constant__ CUtensorMap tmU,
-                    const __grid_constant__ AccumParams p) {
+    dv_accum_kernel(const __grid_constant__ CUtensorMap tmH, const __grid_constant__ CUtensorMap tmHlo,
+                    const __grid_constant__ CUtensorMap tmU, const __grid_constant__ AccumParams p) {
   using C = ACfg<RP, CW, STAGES>;
   constexpr int R = C::R;
+  const int nq = p.split ? 2 * R : R;  // K slabs per layer: h_l (and its low part), 64 wide
   extern __shared__ uint8_t smem_raw[];
   const uint32_t raw = smem_addr(smem_raw);
   const uint32_t base = (raw + 1023u) & ~1023u;
@@ -445,6 +486,7 @@ __global__ void __launch_bounds__(kFoldThreads, 1)
   if (warp == 0 && lane == 0) {
     tma_prefetch_desc(&tmH);
     tma_prefetch_desc(&tmU);
+    if (p.split) tma_prefetch_desc(&tmHlo);
   }
   if (warp == 1) {
     tmem_alloc(smem_addr(tmem_slot), C::kTmemCols);
@@ -464,16 +506,18 @@ __global__ void __launch_bounds__(kFoldThreads, 1)
       uint32_t phase = 0, used = 0, issued_parity = 0;
       bool ok = true;
       for (int l = 0; l < p.L && ok; ++l) {
-        for (int q = 0; q < R; ++q) {
+        for (int q = 0; q < nq; ++q) {
           if (!mbar_wait(empty_bar(stage), phase ^ 1u, abort_flag, tmo)) {
             ok = false;
             break;
           }
           const uint32_t dst = ring + stage * C::kStage;
+          const CUtensorMap* ha = q < R ? &tmH : &tmHlo;
+          const int kq = q % R;
           mbar_arrive_expect_tx(full_bar(stage), C::kStage);
-          tma_load_2d(dst, &tmH, full_bar(stage), l * RP + 64 * q, row0);
-          tma_load_2d(dst + kSlabA, &tmH, full_bar(stage), l * RP + 64 * q, row0 + 128);
-          tma_load_2d(dst + 2 * kSlabA, &tmU, full_bar(stage), 64 * q, l * p.d + col0);
+          tma_load_2d(dst, ha, full_bar(stage), l * RP + 64 * kq, row0);
+          tma_load_2d(dst + kSlabA, ha, full_bar(stage), l * RP + 64 * kq, row0 + 128);
+          tma_load_2d(dst + 2 * kSlabA, &tmU, full_bar(stage), 64 * kq, l * p.d + col0);
           used |= 1u << stage;
           issued_parity = (issued_parity & ~(1u << stage)) | (phase << stage);
           if (++stage == STAGES) {
@@ -495,7 +539,7 @@ __global__ void __launch_bounds__(kFoldThreads, 1)
       uint32_t phase = 0;
       bool issued_any = false, ok = true;
       for (int l = 0; l < p.L && ok; ++l) {
-        for (int q = 0; q < R && ok; ++q) {
+        for (int q = 0; q < nq && ok; ++q) {
           if (!mbar_wait(full_bar(stage), phase, abort_flag, tmo)) {
             ok = false;
             break;
@@ -515,7 +559,7 @@ __global__ void __launch_bounds__(kFoldThreads, 1)
               umma_bf16(d_tmem, sdesc_kmajor_sw128(a_s + 32u * k), sdesc_kmajor_sw128(b_s + 32u * k),
                         idesc, 1u);
             issued_any = true;
-            if (q == R - 1) umma_commit(accf_bar(b));
+            if (q == nq - 1) umma_commit(accf_bar(b));
           }
           if (!ok) break;
           umma_commit(empty_bar(stage));
@@ -606,11 +650,12 @@ __global__ void __launch_bounds__(kFoldThreads, 1)
   }
 }
 
-template <int RP, int KS, int ST>
-cudaError_t hchain_t(long long blocks, const CUtensorMap& h, const CUtensorMap& pf,
-                     const HChainParams& p, cudaStream_t stream) {
-  using C = HCfg<RP, KS, ST>;
-  auto kern = dv_hchain_kernel<RP, KS, ST>;
+template <int RP, int KS, int ST, bool SPLIT>
+cudaError_t hchain_t(long long blocks, const CUtensorMap& h, const CUtensorMap& hlo,
+                     const CUtensorMap& pf, const CUtensorMap& pflo, const HChainParams& p,
+                     cudaStream_t stream) {
+  using C = HCfg<RP, KS, ST, SPLIT>;
+  auto kern = dv_hchain_kernel<RP, KS, ST, SPLIT>;
   cudaError_t err = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, C::kSmemBytes);
   if (err != cudaSuccess || blocks <= 0) return err;
   cudaLaunchConfig_t cfg = {};
@@ -621,14 +666,14 @@ cudaError_t hchain_t(long long blocks, const CUtensorMap& h, const CUtensorMap& 
   cfg.stream = stream;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
-  err = cudaLaunchKernelEx(&cfg, kern, h, pf, p);
+  err = cudaLaunchKernelEx(&cfg, kern, h, hlo, pf, pflo, p);
   if (err != cudaSuccess) return err;
   return cudaGetLastError();
 }
 
 template <int RP, int CW, int ST>
-cudaError_t accum_t(long long ctas, const CUtensorMap& h, const CUtensorMap& u,
-                    const AccumParams& p, cudaStream_t stream) {
+cudaError_t accum_t(long long ctas, const CUtensorMap& h, const CUtensorMap& hlo,
+                    const CUtensorMap& u, const AccumParams& p, cudaStream_t stream) {
   using C = ACfg<RP, CW, ST>;
   auto kern = dv_accum_kernel<RP, CW, ST>;
   cudaError_t err = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, C::kSmemBytes);
@@ -641,14 +686,16 @@ cudaError_t accum_t(long long ctas, const CUtensorMap& h, const CUtensorMap& u,
   cfg.stream = stream;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
-  err = cudaLaunchKernelEx(&cfg, kern, h, u, p);
+  err = cudaLaunchKernelEx(&cfg, kern, h, hlo, u, p);
   if (err != cudaSuccess) return err;
   return cudaGetLastError();
 }
 
 }  // namespace
 
-int hchain_box_slabs(int r_pad) { return r_pad == 256 ? 1 : 2; }
+int hchain_box_slabs(int r_pad, bool split) {
+  return r_pad == 256 || (split && r_pad == 192) ? 1 : 2;
+}
 
 // A CTA of the running sum covers two token blocks and 256 hidden columns (128 where d is not a
 // multiple of 256): the U slab it stages serves both blocks, and the two accumulators fill TMEM.
@@ -658,32 +705,45 @@ int fold_slice_cols(int d) {
   return 0;
 }
 
-cudaError_t launch_hchain(int r_pad, long long tokens, int n_layers, const float* C, int ldc,
-                          const CUtensorMap& h, const CUtensorMap& pf, uint16_t* H, int ldh,
-                          int* status, unsigned long long timeout_ns, cudaStream_t stream) {
+cudaError_t launch_hchain(int r_pad, bool split, long long tokens, int n_layers, const float* C,
+                          int ldc, const CUtensorMap& h, const CUtensorMap& hlo,
+                          const CUtensorMap& pf, const CUtensorMap& pflo, uint16_t* H, uint16_t* Hlo,
+                          int ldh, int* status, unsigned long long timeout_ns, cudaStream_t stream) {
   HChainParams p;
   p.M = static_cast<int>(tokens);
   p.L = n_layers;
   p.C = C;
   p.ldc = ldc;
   p.H = H;
+  p.Hlo = Hlo;
   p.ldh = ldh;
   p.status = status;
   p.timeout_ns = timeout_ns;
   const long long blocks = (tokens + 127) / 128;
-  switch (r_pad) {  // slabs per box (hchain_box_slabs) and pipeline stages
-    case 64: return hchain_t<64, 2, 4>(blocks, h, pf, p, stream);
-    case 128: return hchain_t<128, 2, 3>(blocks, h, pf, p, stream);
-    case 192: return hchain_t<192, 2, 2>(blocks, h, pf, p, stream);
-    case 256: return hchain_t<256, 1, 3>(blocks, h, pf, p, stream);
+  // slabs per box (hchain_box_slabs) and pipeline stages; the split keeps a low h tile beside
+  // the high one
+  if (split) {
+    switch (r_pad) {
+      case 64: return hchain_t<64, 2, 4, true>(blocks, h, hlo, pf, pflo, p, stream);
+      case 128: return hchain_t<128, 2, 2, true>(blocks, h, hlo, pf, pflo, p, stream);
+      case 192: return hchain_t<192, 1, 3, true>(blocks, h, hlo, pf, pflo, p, stream);
+      case 256: return hchain_t<256, 1, 2, true>(blocks, h, hlo, pf, pflo, p, stream);
+      default: return cudaErrorInvalidValue;
+    }
+  }
+  switch (r_pad) {
+    case 64: return hchain_t<64, 2, 4, false>(blocks, h, hlo, pf, pflo, p, stream);
+    case 128: return hchain_t<128, 2, 3, false>(blocks, h, hlo, pf, pflo, p, stream);
+    case 192: return hchain_t<192, 2, 2, false>(blocks, h, hlo, pf, pflo, p, stream);
+    case 256: return hchain_t<256, 1, 3, false>(blocks, h, hlo, pf, pflo, p, stream);
     default: return cudaErrorInvalidValue;
   }
 }
 
 cudaError_t launch_accum(int r_pad, int cw, long long tokens, int n_layers, int d,
-                         const void* x0, const CUtensorMap& h, const CUtensorMap& u, uint16_t* mem,
-                         float* part, long long part_ld, int* status,
-                         unsigned long long timeout_ns, cudaStream_t stream) {
+                         const void* x0, const CUtensorMap& h, const CUtensorMap& hlo, bool split,
+                         const CUtensorMap& u, uint16_t* mem, float* part, long long part_ld,
+                         int* status, unsigned long long timeout_ns, cudaStream_t stream) {
   AccumParams p;
   p.M = static_cast<int>(tokens);
   p.L = n_layers;
@@ -693,11 +753,12 @@ cudaError_t launch_accum(int r_pad, int cw, long long tokens, int n_layers, int 
   p.mem = mem;
   p.part = part;
   p.part_ld = part_ld;
+  p.split = split ? 1 : 0;
   p.status = status;
   p.timeout_ns = timeout_ns;
   const long long ctas = (tokens + 255) / 256 * p.S;
 #define DV_ACCUM(RPV, CWV, STV) \
-  if (r_pad == RPV && cw == CWV) return accum_t<RPV, CWV, STV>(ctas, h, u, p, stream);
+  if (r_pad == RPV && cw == CWV) return accum_t<RPV, CWV, STV>(ctas, h, hlo, u, p, stream);
   DV_ACCUM(64, 256, 3) DV_ACCUM(64, 128, 4)
   DV_ACCUM(128, 256, 3) DV_ACCUM(128, 128, 4)
   DV_ACCUM(192, 256, 3) DV_ACCUM(192, 128, 4)

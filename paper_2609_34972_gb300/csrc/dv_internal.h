@@ -238,15 +238,20 @@ cudaError_t launch_chain(int r_pad, int spc, int S, long long tokens, int n_laye
 // fold_slice_cols: the slice width cw (256 or 128 dividing d), or 0.
 // hchain_box_slabs: K slabs per TMA box of launch_hchain's maps (h and pf are slab maps,
 // encode_slabs, with boxes of that many slabs).
+// split (split_chain): h_l also as its low bf16 part Hlo (hlo: its maps, as h's), and Pf_lo
+// (pflo: its map, as pf's), the low part of the products: each product is taken in three parts,
+// h_hi Q_hi + h_lo Q_hi + h_hi Q_lo, and the running sum adds h_hi U + h_lo U. Without the split
+// hlo and pflo are not read.
 int fold_slice_cols(int d);
-int hchain_box_slabs(int r_pad);
-cudaError_t launch_hchain(int r_pad, long long tokens, int n_layers, const float* C, int ldc,
-                          const CUtensorMap& h, const CUtensorMap& pf, uint16_t* H, int ldh,
-                          int* status, unsigned long long timeout_ns, cudaStream_t stream);
+int hchain_box_slabs(int r_pad, bool split);
+cudaError_t launch_hchain(int r_pad, bool split, long long tokens, int n_layers, const float* C,
+                          int ldc, const CUtensorMap& h, const CUtensorMap& hlo,
+                          const CUtensorMap& pf, const CUtensorMap& pflo, uint16_t* H, uint16_t* Hlo,
+                          int ldh, int* status, unsigned long long timeout_ns, cudaStream_t stream);
 cudaError_t launch_accum(int r_pad, int cw, long long tokens, int n_layers, int d,
-                         const void* x0, const CUtensorMap& h, const CUtensorMap& u, uint16_t* mem,
-                         float* part, long long part_ld, int* status,
-                         unsigned long long timeout_ns, cudaStream_t stream);
+                         const void* x0, const CUtensorMap& h, const CUtensorMap& hlo, bool split,
+                         const CUtensorMap& u, uint16_t* mem, float* part, long long part_ld,
+                         int* status, unsigned long long timeout_ns, cudaStream_t stream);
 
 // Token tile (64, 128, 192 or 256) of the pair kernel for a build of `tokens` tokens.
 int kv_pair_tile_n(long long tokens);
@@ -281,6 +286,7 @@ struct PlanView {
   const CUtensorMap* tm_Uup;       // recurrent: [L*d][r_pad], boxes of resid_bn rows
   const uint16_t* Uup;             // recurrent: U_l as [L*d][r_pad] ([U_l | U_l] when split)
   const CUtensorMap* tm_Pf;        // recurrent, refactored chain: Pf with r_pad-row boxes, or null
+  const CUtensorMap* tm_Pf_lo;     // the same for Pf_lo (split chain), or null
   int chain_clusters;              // recurrent: resident clusters of the on-chip chain (0: none)
   int split_chain;                 // recurrent: hi + lo bf16 operands in the chain's GEMMs
   int uup_ld;                      // row pitch of Uup: r_pad, or 2 r_pad with the split chain

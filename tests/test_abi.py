@@ -77,7 +77,6 @@ def test_bad_config_rejected_before_device(dv, field, value, code):
 
 
 @pytest.mark.parametrize("d,split,path,code", [
-    (512, 1, "rearranged", 1),   # the split chain has only the chain's path
     (576, 0, "rearranged", 2),   # the rearranged chain's slices need d % 128 == 0
     (512, 0, "bogus", None),     # refused by the binding
 ])
