@@ -7,8 +7,9 @@
 // batch is not acceptable, and code that must not risk the implicit device synchronisation
 // of cudaMalloc / cudaFree in its latency-critical path. For them this file keeps the build's
 // intermediate buffers (SiLU(E D_l) for every layer, the RMS statistics and the row sums of
-// squares; for the recurrent adapter also the fp32 state, M_l of every layer and partial sums of
-// squares) in one file-scope static device array of kScratchBytes instead of the plan's
+// squares; for the recurrent adapter also M_l of every layer, partial sums of squares, and the
+// fp32 state or, for the rearranged chain, the fp32 E D_l^T) in one file-scope static device
+// array of kScratchBytes instead of the plan's
 // workspace. The plan's repacked weights are still used; nothing here allocates.
 //
 // Behaviour a caller must know:
