@@ -209,16 +209,20 @@ def test_host_pipeline_rejects_shapes_beyond_the_plan(env):
         assert e.value.code == code
 
 
-def test_host_pipeline_mrope_bias_recurrent():
+@pytest.mark.parametrize("path", ["chain", "rearranged"])
+def test_host_pipeline_mrope_bias_recurrent(path):
     # Three position axes (M-RoPE) and K/V bias through the host entry, with the recurrent
-    # adapter: the host buffers equal the device build of the same inputs.
+    # adapter (either evaluation of its chain): the host buffers equal the device build of the
+    # same inputs.
     import torch
+    from dataclasses import replace
     import paper_2609_34972_gb300 as dv
     cfg = gu.small_config("host_mrope", d=512, n_layers=3, n_kv_heads=2, n_heads=4, head_dim=128,
                           rank=64, n_vis=150, batch=2, rope="mrope", rope_theta=1e6,
                           mrope_section=(16, 24, 24), grid=(1, 10, 15), x0_sigma=0.5,
                           bias_sigma=0.02, w_sigma=0.05, seed=131, pos_start=15,
                           adapter="recurrent")
+    cfg = replace(cfg, recurrent_path=path)
     inp = synth.make_inputs(cfg)
     k_ref, v_ref, plan = gu.run_build(inp)
     pipe = dv.HostPipeline(plan, cfg.batch, cfg.n_vis, depth=2)
