@@ -14,7 +14,8 @@
 //       squares for the RMS statistic.
 // Only (2) runs layer after layer, and each of its layers is a GEMM of N = r_pad with no
 // exchange between CTAs. The sums differ from the chain's only in rounding (the same products,
-// grouped differently).
+// grouped differently). With the split chain, h_j and Q_lj are each read as a high and a low
+// bf16 part in (2), and h_j in both parts in (3).
 #include "../../include/dv.h"
 #include "dv_epilogue.cuh"
 #include "dv_internal.h"
@@ -119,15 +120,15 @@ __device__ __forceinline__ HSeg hseg(int l, int seg, int R) {
 
 // One CTA per 128-token block, all layers. Layer l's accumulator starts as C_l, written into TMEM
 // by the epilogue warps (tcgen05.st) while the tensor cores still work on earlier layers; the
-// layer's GEMM then adds h_j Q_lj^T for every j < l over l R slabs of 64 in the two segments of
-// hseg. A pipeline step moves KS consecutive slabs of one segment as one TMA box per operand (a
+// layer's GEMM then adds h_j Q_lj^T for every j < l over l R slabs of 64 in the segments of hseg
+// (two; six with the split). A pipeline step moves KS consecutive slabs of one segment as one TMA box per operand (a
 // TMA instruction has a fixed cost that one 16 KB slab does not amortise); the last step of a
 // segment uses the slabs it needs of its box (the rest is zero fill or data the MMA does not
 // read). Two accumulators alternate by layer: layer l's MMAs over the older h_j run while the
 // epilogue of layer l - 1 still works. The epilogue applies SiLU (layer 0 straight from C_0),
-// writes bf16 h_l to the h tile (the A operand of layer l + 1's last segment) and to H (read back
-// by TMA from layer l + 2 on, and by the running sum), then loads C_{l+2} into the accumulator it
-// has just read.
+// writes bf16 h_l to the h tile (the A operand of layer l + 1's last segments; with the split, its
+// low part to a second tile) and to H (read back by TMA from layer l + 2 on, and by the running
+// sum), then loads C_{l+2} into the accumulator it has just read.
 // Barriers (all waits bounded): stage full / empty; accumulator full; accumulator loaded with C;
 // the h tile written (once per layer); h_l in global memory, alternating between two barriers by
 // layer parity so that the producer, which may run up to two layers ahead of the epilogue, never
