@@ -77,6 +77,17 @@ def test_recurrent_every_rank_padding(rank, d, splits_hint, path):
 
 
 @pytest.mark.parametrize("path", PATHS)
+@pytest.mark.parametrize("n_layers,n_vis,batch", [(1, 1, 1), (2, 129, 1), (3, 257, 1), (4, 193, 2)])
+def test_recurrent_edge_shapes(n_layers, n_vis, batch, path):
+    # One layer (no recurrence), two layers (nothing loaded two layers ahead), a single token,
+    # and odd token-block counts (the running sum takes two blocks per CTA; the last pair has
+    # one block past the build) with ragged tails.
+    cfg = synth.config("tiny", n_layers=n_layers, n_vis=n_vis, batch=batch, w_sigma=0.05,
+                       seed=70 + n_layers, adapter="recurrent", recurrent_path=path)
+    _full_check(synth.make_inputs(cfg), f"recurrent L{n_layers} T{n_vis * batch}, {path}")
+
+
+@pytest.mark.parametrize("path", PATHS)
 def test_recurrent_tokens_as_m_mrope_bias(path):
     # T = 2 x 256: the K/V launch takes the tokens-as-M engine over the stacked M_l.
     cfg = gu.small_config("rec_tm", d=512, n_layers=3, n_kv_heads=2, n_heads=8, head_dim=128,
