@@ -1502,10 +1502,11 @@ int dv_memory_plan(const dv_config* cfg, const dv_weights* w, void* stream, dv_p
     enc = encode_2d(&p->tm_Dst_rp, p->Dst, d, 1ull * L * p->r_pad, dst_ld, p->r_pad) &&
           encode_2d(&p->tm_Uup, p->Uup, p->uup_ld, 1ull * L * d, p->uup_ld, p->resid_bn);
     if (enc && p->fold)
-      enc = encode_slabs(&p->tm_Pf, p->Pf, pf_ld, 1ull * L * p->r_pad, pf_ld, p->r_pad,
+      // boxes of r_pad / 2 rows: each CTA of a recurrence pair stages half of a layer's rows
+      enc = encode_slabs(&p->tm_Pf, p->Pf, pf_ld, 1ull * L * p->r_pad, pf_ld, p->r_pad / 2,
                          static_cast<uint32_t>(dv::hchain_box_slabs(p->r_pad, cfg->split_chain)));
     if (enc && p->Pf_lo)
-      enc = encode_slabs(&p->tm_Pf_lo, p->Pf_lo, pf_ld, 1ull * L * p->r_pad, pf_ld, p->r_pad,
+      enc = encode_slabs(&p->tm_Pf_lo, p->Pf_lo, pf_ld, 1ull * L * p->r_pad, pf_ld, p->r_pad / 2,
                          static_cast<uint32_t>(dv::hchain_box_slabs(p->r_pad, true)));
   } else if (enc) {
     enc = encode_slabs(&p->tm_Bn_half, p->Bn, p->bn_k, 256ull * p->bn_groups, p->bn_k, 128) &&

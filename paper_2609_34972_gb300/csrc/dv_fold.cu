@@ -68,10 +68,11 @@ __device__ __forceinline__ void tma_load_slabs(uint32_t dst, const CUtensorMap* 
       : "memory");
 }
 
-template <int RP, int KS, int STAGES, bool SPLIT>
+template <int RP, int KS, int STAGES, bool SPLIT, bool PAIR>
 struct HCfg {
   static constexpr int R = RP / 64;              // 64-wide K slabs per r_pad
-  static constexpr int kSlabB = RP * 128;        // [RP rows of Pf][64] bf16
+  // [RP rows of Pf][64] bf16; on CTA pairs each CTA stages its half of the rows
+  static constexpr int kSlabB = (PAIR ? RP / 2 : RP) * 128;
   static constexpr int kA = KS * kSlabA;         // one box of KS slabs of A
   static constexpr int kB = KS * kSlabB;         // one box of KS slabs of B
   static constexpr int kStage = kA + kB;
@@ -134,12 +135,18 @@ __device__ __forceinline__ HSeg hseg(int l, int seg, int R) {
 // layer parity so that the producer, which may run up to two layers ahead of the epilogue, never
 // waits on a phase that has wrapped. The accumulator barriers of layer l complete for the
 // ((l - 1) / 2)-th time (integer division) at that layer, on accumulator l mod 2.
-template <int RP, int KS, int STAGES, bool SPLIT>
+// PAIR: a cluster of two CTAs (token blocks 2c and 2c + 1) runs each layer's GEMM as one 2-SM
+// MMA (M = 256, tcgen05 cta_group::2) issued by the leader: each CTA stages its own 128 rows of
+// h and half of the layer's rows of Pf, so an SM moves half the B bytes per MMA through shared
+// memory. The leader's stage-full barrier counts both CTAs' bytes; its commits arrive on both
+// CTAs' stage-empty and accumulator-full barriers; both CTAs' epilogue warps arrive on the
+// leader's accumulator-loaded and h-tile barriers (one lane per warp, 8 arrivals).
+template <int RP, int KS, int STAGES, bool SPLIT, bool PAIR>
 __global__ void __launch_bounds__(kFoldThreads, 1)
     dv_hchain_kernel(const __grid_constant__ CUtensorMap tmH, const __grid_constant__ CUtensorMap tmHlo,
                      const __grid_constant__ CUtensorMap tmP, const __grid_constant__ CUtensorMap tmPlo,
                      const __grid_constant__ HChainParams p) {
-  using C = HCfg<RP, KS, STAGES, SPLIT>;
+  using C = HCfg<RP, KS, STAGES, SPLIT, PAIR>;
   constexpr int kSegs = SPLIT ? 6 : 2;
   constexpr int kFirstNew = SPLIT ? 3 : 1;  // the first segment that reads the h tiles
   constexpr int R = C::R;
@@ -162,7 +169,11 @@ __global__ void __launch_bounds__(kFoldThreads, 1)
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const uint64_t tmo = p.timeout_ns;
-  const int row0 = blockIdx.x * 128;
+  const int row0 = blockIdx.x * 128;  // with pairs: cluster c, rank r -> block 2c + r
+  const uint32_t rank = PAIR ? cluster_ctarank() : 0u;
+  // arrivals on the accumulator-loaded and h-tile barriers: every epilogue thread, or with pairs
+  // one lane per epilogue warp of both CTAs on the leader's
+  constexpr int kEpiArrivals = PAIR ? 8 : kEpi;
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < STAGES; ++s) {
@@ -171,10 +182,10 @@ __global__ void __launch_bounds__(kFoldThreads, 1)
     }
     for (int a = 0; a < 2; ++a) {
       mbar_init(accf_bar(a), 1);
-      mbar_init(init_bar(a), kEpi);
+      mbar_init(init_bar(a), kEpiArrivals);
       mbar_init(hpub_bar(a), kEpi);
     }
-    mbar_init(htile_bar, kEpi);
+    mbar_init(htile_bar, kEpiArrivals);
     mbar_init(drain_bar, 1);
     *abort_flag = 0;
     fence_barrier_init();
@@ -188,11 +199,19 @@ __global__ void __launch_bounds__(kFoldThreads, 1)
     }
   }
   if (warp == 1) {
-    tmem_alloc(smem_addr(tmem_slot), C::kTmemCols);
-    tmem_relinquish();
+    if (PAIR) {
+      tmem_alloc_pair(smem_addr(tmem_slot), C::kTmemCols);
+      tmem_relinquish_pair();
+    } else {
+      tmem_alloc(smem_addr(tmem_slot), C::kTmemCols);
+      tmem_relinquish();
+    }
   }
   tc_fence_before();
-  __syncthreads();
+  if (PAIR)
+    cluster_sync();  // both CTAs' barriers exist before any remote arrival or pair load
+  else
+    __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
   pdl_wait();
@@ -201,6 +220,7 @@ __global__ void __launch_bounds__(kFoldThreads, 1)
   if (warp == 0) {
     if (lane == 0) {
       // ---------------------------------------------------------------- TMA producer
+      const uint32_t leader_full0 = PAIR ? map_to_rank(full_bar(0), 0) : full_bar(0);
       int stage = 0;
       uint32_t phase = 0, used = 0, issued_parity = 0;
       bool ok = true;
@@ -221,10 +241,20 @@ __global__ void __launch_bounds__(kFoldThreads, 1)
               break;
             }
             const uint32_t a_dst = ring + stage * C::kStage, b_dst = a_dst + C::kA;
-            mbar_arrive_expect_tx(full_bar(stage), g.asrc >= 2 ? C::kB : C::kStage);
-            if (g.asrc < 2)
-              tma_load_slabs(a_dst, g.asrc == 0 ? &tmH : &tmHlo, full_bar(stage), row0, g.a0 + s0);
-            tma_load_slabs(b_dst, g.bsrc == 0 ? &tmP : &tmPlo, full_bar(stage), l * RP, g.b0 + s0);
+            const uint32_t bytes = g.asrc >= 2 ? C::kB : C::kStage;
+            const CUtensorMap* am = g.asrc == 0 ? &tmH : &tmHlo;
+            const CUtensorMap* bm = g.bsrc == 0 ? &tmP : &tmPlo;
+            if (PAIR) {
+              // both CTAs' copies complete on the leader's barrier, which expects both
+              const uint32_t fb = leader_full0 + 8u * stage;
+              if (rank == 0) mbar_arrive_expect_tx(full_bar(stage), 2 * bytes);
+              if (g.asrc < 2) tma_load_3d_pair(a_dst, am, fb, row0, g.a0 + s0);
+              tma_load_3d_pair(b_dst, bm, fb, l * RP + static_cast<int>(rank) * (RP / 2), g.b0 + s0);
+            } else {
+              mbar_arrive_expect_tx(full_bar(stage), bytes);
+              if (g.asrc < 2) tma_load_slabs(a_dst, am, full_bar(stage), row0, g.a0 + s0);
+              tma_load_slabs(b_dst, bm, full_bar(stage), l * RP, g.b0 + s0);
+            }
             used |= 1u << stage;
             issued_parity = (issued_parity & ~(1u << stage)) | (phase << stage);
             if (++stage == STAGES) {
@@ -234,15 +264,17 @@ __global__ void __launch_bounds__(kFoldThreads, 1)
           }
         }
       }
-      if (*abort_flag) {  // every copy still in flight lands before the CTA exits
+      // every copy still in flight lands before the CTA exits (pairs: their copies complete on
+      // the leader's barriers; the teardown waits instead)
+      if (!PAIR && *abort_flag) {
         for (int s = 0; s < STAGES; ++s)
           if (used & (1u << s)) wait_only(full_bar(s), (issued_parity >> s) & 1u, tmo);
       }
     }
   } else if (warp == 1) {
-    if (lane == 0) {
-      // ---------------------------------------------------------------- MMA issuer
-      const uint32_t idesc = idesc_bf16_f32(128, RP);
+    if (lane == 0 && rank == 0) {
+      // ---------------------------------------------------------------- MMA issuer (the leader)
+      const uint32_t idesc = idesc_bf16_f32(PAIR ? 256 : 128, RP);
       int stage = 0;
       uint32_t phase = 0;
       bool issued_any = false, ok = true;
@@ -273,12 +305,20 @@ __global__ void __launch_bounds__(kFoldThreads, 1)
                               : st + static_cast<uint32_t>(u * kSlabA);
               const uint32_t b_s = st + C::kA + static_cast<uint32_t>(u * C::kSlabB);
 #pragma unroll
-              for (int k = 0; k < 4; ++k)
-                umma_bf16(d_tmem, sdesc_kmajor_sw128(a_s + 32u * k), sdesc_kmajor_sw128(b_s + 32u * k),
-                          idesc, 1u);  // the accumulator starts from C_l
+              for (int k = 0; k < 4; ++k) {  // the accumulator starts from C_l
+                if (PAIR)
+                  umma_bf16_pair(d_tmem, sdesc_kmajor_sw128(a_s + 32u * k),
+                                 sdesc_kmajor_sw128(b_s + 32u * k), idesc, 1u);
+                else
+                  umma_bf16(d_tmem, sdesc_kmajor_sw128(a_s + 32u * k),
+                            sdesc_kmajor_sw128(b_s + 32u * k), idesc, 1u);
+              }
             }
             issued_any = true;
-            umma_commit(empty_bar(stage));
+            if (PAIR)
+              umma_commit_pair(empty_bar(stage), 0x3);
+            else
+              umma_commit(empty_bar(stage));
             if (++stage == STAGES) {
               stage = 0;
               phase ^= 1u;
@@ -286,10 +326,16 @@ __global__ void __launch_bounds__(kFoldThreads, 1)
           }
         }
         if (!ok) break;
-        umma_commit(accf_bar(acc));
+        if (PAIR)
+          umma_commit_pair(accf_bar(acc), 0x3);
+        else
+          umma_commit(accf_bar(acc));
       }
       if (*abort_flag && issued_any) {  // no TMEM release while an MMA may still run
-        umma_commit(drain_bar);
+        if (PAIR)
+          umma_commit_pair(drain_bar, 0x1);
+        else
+          umma_commit(drain_bar);
         wait_only(drain_bar, 0, tmo);
       }
     }
@@ -326,7 +372,12 @@ __global__ void __launch_bounds__(kFoldThreads, 1)
       }
       asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
       tc_fence_before();
-      mbar_arrive(init_bar(a));
+      if (PAIR) {  // one lane per warp on the leader's barrier, for the warp's 32 rows
+        __syncwarp();
+        if (lane == 0) mbar_arrive_cluster(map_to_rank(init_bar(a), 0));
+      } else {
+        mbar_arrive(init_bar(a));
+      }
     };
     // SiLU of the 32 columns c*32 .. of z into the h tile (bf16, swizzled as the MMA reads it);
     // split: the remainder h - bf16(h), itself in bf16, into the low tile
@@ -373,7 +424,12 @@ __global__ void __launch_bounds__(kFoldThreads, 1)
       // The h tile first (the next layer's MMA waits for it; async proxy), then the copy of h_l
       // in H (TMA loads two or more layers later, and the running sum): read back from the tile.
       asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-      mbar_arrive(htile_bar);
+      if (PAIR) {
+        __syncwarp();
+        if (lane == 0) mbar_arrive_cluster(map_to_rank(htile_bar, 0));
+      } else {
+        mbar_arrive(htile_bar);
+      }
       if (live) {
         const long long go = static_cast<long long>(t) * p.ldh + l * RP;
         uint4* hg = reinterpret_cast<uint4*>(p.H + go);
@@ -401,10 +457,21 @@ __global__ void __launch_bounds__(kFoldThreads, 1)
 
   tc_fence_before();
   __syncthreads();
-  if (threadIdx.x == 0 && *abort_flag) atomicExch(p.status, DV_ERR_DEVICE_TIMEOUT);
+  if (threadIdx.x == 0 && *abort_flag) {
+    if (PAIR) {  // this CTA's own copies still in flight land before the pair is torn down
+      const uint64_t t0 = globaltimer_ns();
+      while (globaltimer_ns() - t0 < 200000ull) {
+      }
+    }
+    atomicExch(p.status, DV_ERR_DEVICE_TIMEOUT);
+  }
+  if (PAIR) cluster_sync();
   if (warp == 1) {
     tc_fence_after();
-    tmem_dealloc(tmem, C::kTmemCols);
+    if (PAIR)
+      tmem_dealloc_pair(tmem, C::kTmemCols);
+    else
+      tmem_dealloc(tmem, C::kTmemCols);
   }
 }
 
@@ -655,18 +722,24 @@ template <int RP, int KS, int ST, bool SPLIT>
 cudaError_t hchain_t(long long blocks, const CUtensorMap& h, const CUtensorMap& hlo,
                      const CUtensorMap& pf, const CUtensorMap& pflo, const HChainParams& p,
                      cudaStream_t stream) {
-  using C = HCfg<RP, KS, ST, SPLIT>;
-  auto kern = dv_hchain_kernel<RP, KS, ST, SPLIT>;
+  // CTA pairs: two token blocks per cluster (the last pair may hold a block past the build)
+  using C = HCfg<RP, KS, ST, SPLIT, true>;
+  auto kern = dv_hchain_kernel<RP, KS, ST, SPLIT, true>;
   cudaError_t err = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, C::kSmemBytes);
   if (err != cudaSuccess || blocks <= 0) return err;
   cudaLaunchConfig_t cfg = {};
-  cudaLaunchAttribute attr[1] = {pdl_attribute()};
-  cfg.gridDim = dim3(static_cast<unsigned>(blocks), 1, 1);
+  cudaLaunchAttribute attr[2];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = 2;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  attr[1] = pdl_attribute();
+  cfg.gridDim = dim3(static_cast<unsigned>((blocks + 1) / 2 * 2), 1, 1);
   cfg.blockDim = dim3(kFoldThreads, 1, 1);
   cfg.dynamicSmemBytes = C::kSmemBytes;
   cfg.stream = stream;
   cfg.attrs = attr;
-  cfg.numAttrs = 1;
+  cfg.numAttrs = 2;
   err = cudaLaunchKernelEx(&cfg, kern, h, hlo, pf, pflo, p);
   if (err != cudaSuccess) return err;
   return cudaGetLastError();
@@ -726,17 +799,17 @@ cudaError_t launch_hchain(int r_pad, bool split, long long tokens, int n_layers,
   if (split) {
     switch (r_pad) {
       case 64: return hchain_t<64, 2, 4, true>(blocks, h, hlo, pf, pflo, p, stream);
-      case 128: return hchain_t<128, 2, 2, true>(blocks, h, hlo, pf, pflo, p, stream);
-      case 192: return hchain_t<192, 1, 3, true>(blocks, h, hlo, pf, pflo, p, stream);
-      case 256: return hchain_t<256, 1, 2, true>(blocks, h, hlo, pf, pflo, p, stream);
+      case 128: return hchain_t<128, 2, 3, true>(blocks, h, hlo, pf, pflo, p, stream);
+      case 192: return hchain_t<192, 1, 4, true>(blocks, h, hlo, pf, pflo, p, stream);
+      case 256: return hchain_t<256, 1, 3, true>(blocks, h, hlo, pf, pflo, p, stream);
       default: return cudaErrorInvalidValue;
     }
   }
   switch (r_pad) {
-    case 64: return hchain_t<64, 2, 4, false>(blocks, h, hlo, pf, pflo, p, stream);
-    case 128: return hchain_t<128, 2, 3, false>(blocks, h, hlo, pf, pflo, p, stream);
-    case 192: return hchain_t<192, 2, 2, false>(blocks, h, hlo, pf, pflo, p, stream);
-    case 256: return hchain_t<256, 1, 3, false>(blocks, h, hlo, pf, pflo, p, stream);
+    case 64: return hchain_t<64, 2, 5, false>(blocks, h, hlo, pf, pflo, p, stream);
+    case 128: return hchain_t<128, 2, 4, false>(blocks, h, hlo, pf, pflo, p, stream);
+    case 192: return hchain_t<192, 2, 3, false>(blocks, h, hlo, pf, pflo, p, stream);
+    case 256: return hchain_t<256, 1, 5, false>(blocks, h, hlo, pf, pflo, p, stream);
     default: return cudaErrorInvalidValue;
   }
 }
