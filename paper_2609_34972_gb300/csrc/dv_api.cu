@@ -905,7 +905,7 @@ static cudaError_t enqueue_fold(const PlanView& v, const BuildArgs& a, cudaStrea
   mark(2);
   if (err == cudaSuccess)
     err = launch_pdl(k_rstd_parts, dim3(grid_for(static_cast<long long>(L) * T)), dim3(256), st,
-                     a.part, L, T, d / cw, part_ld, 1.0f / d, v.rms_eps, a.rstd);
+                     a.part, L, T, fold_sum_parts(d), part_ld, 1.0f / d, v.rms_eps, a.rstd);
   mark(3);
   return err == cudaSuccess ? launch_recurrent_kv(v, a, T, tm_mem_s, st, mark) : err;
 }

@@ -29,6 +29,7 @@ namespace {
 
 constexpr int kFoldThreads = 192;  // warp 0 TMA, warp 1 MMA + TMEM, warps 2-5 epilogue
 constexpr int kEpi = 128;
+constexpr int kAccumWarps = 2;     // epilogue warps per TMEM lane quarter of the running sum
 constexpr int kSlabA = 128 * 128;  // [128 token rows][64] bf16, 128-byte swizzle
 
 // Byte offset of 16-byte chunk `c` (c < 8) of row `row` in a 128-byte-swizzled slab.
@@ -477,13 +478,20 @@ __global__ void __launch_bounds__(kFoldThreads, 1)
 
 // ---------------------------------------------------------------- (3) the running sum
 
-template <int RP, int CW, int STAGES>
+// Shared staging of one warp's bf16 stores (warp_store_bf16: 32 rows of 20 words).
+constexpr int kBf16StageFloats = 32 * 20;
+
+template <int RP, int CW, int STAGES, int EW>
 struct ACfg {
   static constexpr int R = RP / 64;
+  static constexpr int kThreads = 64 + 128 * EW;     // TMA warp, MMA warp, EW warps per lane quarter
+  static constexpr int kEpiThreads = 128 * EW;
+  static constexpr int kCols = CW / EW;              // hidden columns of one epilogue warp
   static constexpr int kSlabB = CW * 128;            // [CW rows of U_l][64] bf16
   static constexpr int kStage = 2 * kSlabA + kSlabB; // h slabs of the two token blocks, U slab
   static constexpr int kOffWarp = STAGES * kStage;   // per-warp staging of the M_l stores
-  static constexpr int kEnd = kOffWarp + 4 * kWarpStageFloats * 4;
+  static constexpr int kEnd = kOffWarp + 4 * EW * kBf16StageFloats * 4;
+  static_assert(kCols % 32 == 0 && CW / 64 >= EW, "whole 32-column chunks; parts fit d / 64");
   static constexpr int kSmemBytes = kEnd + 1024 + 256;
   static constexpr int kTmemCols = 2 * CW <= 256 ? 256 : 512;
   static_assert(kSlabB % 1024 == 0, "stage tiles stay 1024-byte aligned");
@@ -497,7 +505,7 @@ struct AccumParams {
   int S;               // hidden slices (d / CW)
   const uint16_t* x0;  // bf16 [M][d]
   uint16_t* mem;       // bf16 [L][M][d]: the stacked M_l
-  float* part;         // fp32 [L][part_ld / M][M]: sums of squares of M_l per slice
+  float* part;         // fp32 [L][part_ld / M][M]: sums of squares of M_l per CW / EW columns
   long long part_ld;
   int split;           // 1: h_l in two bf16 parts (H, then Hlo), both against U_l
   int* status;
@@ -509,13 +517,15 @@ struct AccumParams {
 // accumulator starts as the fp32 widening of E's slice (tcgen05.st); layer l adds h_l U_l^T
 // (K = r_pad, the U slab staged once for both blocks) and is read back: bf16 M_l stored through
 // the warp's staging (whole row segments per store instruction) and the row's sum of M_l^2 over
-// the slice to part. Each block has its own barriers, so one block's next MMAs run while the
-// other block's readback and stores go on.
-template <int RP, int CW, int STAGES>
-__global__ void __launch_bounds__(kFoldThreads, 1)
+// the warp's CW / EW columns to part (slot s EW + e). EW warps share each TMEM lane quarter,
+// each with its own columns, so that the loads, conversions and stores of several warps overlap
+// on every SM sub-partition. Each block has its own barriers, so one block's next MMAs run while
+// the other block's readback and stores go on.
+template <int RP, int CW, int STAGES, int EW>
+__global__ void __launch_bounds__(ACfg<RP, CW, STAGES, EW>::kThreads, 1)
     dv_accum_kernel(const __grid_constant__ CUtensorMap tmH, const __grid_constant__ CUtensorMap tmHlo,
                     const __grid_constant__ CUtensorMap tmU, const __grid_constant__ AccumParams p) {
-  using C = ACfg<RP, CW, STAGES>;
+  using C = ACfg<RP, CW, STAGES, EW>;
   constexpr int R = C::R;
   const int nq = p.split ? 2 * R : R;  // K slabs per layer: h_l (and its low part), 64 wide
   extern __shared__ uint8_t smem_raw[];
@@ -545,7 +555,7 @@ __global__ void __launch_bounds__(kFoldThreads, 1)
     }
     for (int b = 0; b < 2; ++b) {
       mbar_init(accf_bar(b), 1);
-      mbar_init(accr_bar(b), kEpi);
+      mbar_init(accr_bar(b), C::kEpiThreads);
     }
     mbar_init(drain_bar, 1);
     *abort_flag = 0;
@@ -644,17 +654,19 @@ __global__ void __launch_bounds__(kFoldThreads, 1)
     }
   } else {
     // ------------------------------------------------------------------ epilogue warps
-    const int qq = warp & 3;  // the TMEM lane quarter this warp may access
+    const int qq = warp & 3;          // the TMEM lane quarter this warp may access
+    const int eh = (warp - 2) >> 2;   // which CW / EW columns of the quarter's rows
     const int row = qq * 32 + lane;
-    const uint32_t tl = tmem + (static_cast<uint32_t>(qq * 32) << 16);
-    float* wstage = reinterpret_cast<float*>(base_ptr + C::kOffWarp) + qq * kWarpStageFloats;
-    // M_0 = E: the fp32 widening of this row's slice of E into both accumulators
+    const int cw0 = eh * C::kCols;    // the warp's first column in the slice
+    const uint32_t tl = tmem + (static_cast<uint32_t>(qq * 32) << 16) + static_cast<uint32_t>(cw0);
+    float* wstage = reinterpret_cast<float*>(base_ptr + C::kOffWarp) + (warp - 2) * kBf16StageFloats;
+    // M_0 = E: the fp32 widening of this row's columns of E into both accumulators
 #pragma unroll 1
     for (int b = 0; b < 2; ++b) {
       const int t = row0 + b * 128 + row;
-      const uint16_t* xr = p.x0 + static_cast<long long>(t < p.M ? t : 0) * p.d + col0;
+      const uint16_t* xr = p.x0 + static_cast<long long>(t < p.M ? t : 0) * p.d + col0 + cw0;
 #pragma unroll 1
-      for (int c = 0; c < CW / 32; ++c) {
+      for (int c = 0; c < C::kCols / 32; ++c) {
         uint32_t r[32];
 #pragma unroll
         for (int k = 0; k < 4; ++k) {
@@ -681,11 +693,11 @@ __global__ void __launch_bounds__(kFoldThreads, 1)
         ok = __all_sync(0xFFFFFFFFu, mbar_wait(accf_bar(b), static_cast<uint32_t>(l) & 1u, abort_flag, tmo));
         if (!ok) break;
         tc_fence_after();
-        // the whole row of the slice leaves TMEM first, so the next layer's MMA can start
-        uint32_t pk[CW / 32][16];
+        // the warp's whole row segment leaves TMEM first, so the next layer's MMA can start
+        uint32_t pk[C::kCols / 32][16];
         float ss = 0.0f;
 #pragma unroll
-        for (int c = 0; c < CW / 32; ++c) {
+        for (int c = 0; c < C::kCols / 32; ++c) {
           uint32_t r[32];
           __syncwarp();
           tmem_ld32(tl + static_cast<uint32_t>(b * CW + c * 32), r);
@@ -701,10 +713,11 @@ __global__ void __launch_bounds__(kFoldThreads, 1)
         tc_fence_before();
         mbar_arrive(accr_bar(b));
         const int t0 = row0 + b * 128 + qq * 32;  // the warp's first row
-        uint16_t* dst = p.mem + (static_cast<long long>(l) * p.M + t0) * p.d + col0;
+        uint16_t* dst = p.mem + (static_cast<long long>(l) * p.M + t0) * p.d + col0 + cw0;
 #pragma unroll
-        for (int c = 0; c < CW / 32; ++c) warp_store_bf16(wstage, pk[c], dst + c * 32, p.d, p.M - t0);
-        if (t0 + lane < p.M) p.part[l * p.part_ld + static_cast<long long>(sl) * p.M + t0 + lane] = ss;
+        for (int c = 0; c < C::kCols / 32; ++c) warp_store_bf16(wstage, pk[c], dst + c * 32, p.d, p.M - t0);
+        if (t0 + lane < p.M)
+          p.part[l * p.part_ld + static_cast<long long>(sl * EW + eh) * p.M + t0 + lane] = ss;
       }
     }
   }
@@ -745,17 +758,17 @@ cudaError_t hchain_t(long long blocks, const CUtensorMap& h, const CUtensorMap& 
   return cudaGetLastError();
 }
 
-template <int RP, int CW, int ST>
+template <int RP, int CW, int ST, int EW>
 cudaError_t accum_t(long long ctas, const CUtensorMap& h, const CUtensorMap& hlo,
                     const CUtensorMap& u, const AccumParams& p, cudaStream_t stream) {
-  using C = ACfg<RP, CW, ST>;
-  auto kern = dv_accum_kernel<RP, CW, ST>;
+  using C = ACfg<RP, CW, ST, EW>;
+  auto kern = dv_accum_kernel<RP, CW, ST, EW>;
   cudaError_t err = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, C::kSmemBytes);
   if (err != cudaSuccess || ctas <= 0) return err;
   cudaLaunchConfig_t cfg = {};
   cudaLaunchAttribute attr[1] = {pdl_attribute()};
   cfg.gridDim = dim3(static_cast<unsigned>(ctas), 1, 1);
-  cfg.blockDim = dim3(kFoldThreads, 1, 1);
+  cfg.blockDim = dim3(C::kThreads, 1, 1);
   cfg.dynamicSmemBytes = C::kSmemBytes;
   cfg.stream = stream;
   cfg.attrs = attr;
@@ -777,6 +790,13 @@ int fold_slice_cols(int d) {
   for (int cw : {256, 128})
     if (d % cw == 0) return cw;
   return 0;
+}
+
+// Two epilogue warps share each TMEM lane quarter of the running sum, each with half of the
+// slice's columns and its own sum-of-squares slot: d / CW * 2 slots per layer.
+int fold_sum_parts(int d) {
+  const int cw = fold_slice_cols(d);
+  return cw > 0 ? d / cw * kAccumWarps : 0;
 }
 
 cudaError_t launch_hchain(int r_pad, bool split, long long tokens, int n_layers, const float* C,
@@ -832,7 +852,7 @@ cudaError_t launch_accum(int r_pad, int cw, long long tokens, int n_layers, int 
   p.timeout_ns = timeout_ns;
   const long long ctas = (tokens + 255) / 256 * p.S;
 #define DV_ACCUM(RPV, CWV, STV) \
-  if (r_pad == RPV && cw == CWV) return accum_t<RPV, CWV, STV>(ctas, h, hlo, u, p, stream);
+  if (r_pad == RPV && cw == CWV) return accum_t<RPV, CWV, STV, kAccumWarps>(ctas, h, hlo, u, p, stream);
   DV_ACCUM(64, 256, 3) DV_ACCUM(64, 128, 4)
   DV_ACCUM(128, 256, 3) DV_ACCUM(128, 128, 4)
   DV_ACCUM(192, 256, 3) DV_ACCUM(192, 128, 4)

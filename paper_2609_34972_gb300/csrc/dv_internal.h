@@ -232,10 +232,11 @@ cudaError_t launch_chain(int r_pad, int spc, int S, long long tokens, int n_laye
 //     l r_pad), one CTA per 128-token block. Maps: h: slab map over H with 128-row boxes; pf:
 //     slab map over Pf with r_pad-row boxes.
 //   launch_accum: M_l = E + sum_{j<=l} h_j U_j^T, bf16 into the stacked memories mem
-//     ([L][tokens][d]) and each row's sum of M_l^2 over each slice of cw hidden columns into part
-//     (d / cw partials per layer). h: H with 128-row boxes; u: U as [L d][r_pad] with cw-row
-//     boxes; x0: E, bf16 [tokens][d].
+//     ([L][tokens][d]) and each row's partial sums of M_l^2 into part (fold_sum_parts(d)
+//     partials per layer, at most d / 64). h: H with 128-row boxes; u: U as [L d][r_pad] with
+//     cw-row boxes; x0: E, bf16 [tokens][d].
 // fold_slice_cols: the slice width cw (256 or 128 dividing d), or 0.
+// fold_sum_parts: the partial sums of squares per token and layer that launch_accum writes.
 // hchain_box_slabs: K slabs per TMA box of launch_hchain's maps (h and pf are slab maps,
 // encode_slabs, with boxes of that many slabs).
 // split (split_chain): h_l also as its low bf16 part Hlo (hlo: its maps, as h's), and Pf_lo
@@ -243,6 +244,7 @@ cudaError_t launch_chain(int r_pad, int spc, int S, long long tokens, int n_laye
 // h_hi Q_hi + h_lo Q_hi + h_hi Q_lo, and the running sum adds h_hi U + h_lo U. Without the split
 // hlo and pflo are not read.
 int fold_slice_cols(int d);
+int fold_sum_parts(int d);
 int hchain_box_slabs(int r_pad, bool split);
 cudaError_t launch_hchain(int r_pad, bool split, long long tokens, int n_layers, const float* C,
                           int ldc, const CUtensorMap& h, const CUtensorMap& hlo,
