@@ -846,18 +846,21 @@ static cudaError_t enqueue_fold(const PlanView& v, const BuildArgs& a, cudaStrea
   };
   const bool split = v.split_chain != 0;
   const uint32_t ks = static_cast<uint32_t>(hchain_box_slabs(v.r_pad, split));
-  CUtensorMap tm_x0, tm_x0_s, tm_hs, tm_h, tm_u, tm_mem_s;
+  // tm_hst: the recurrence's stores of h_l, 32 rows (one epilogue warp) per box
+  CUtensorMap tm_x0, tm_x0_s, tm_hs, tm_h, tm_hst, tm_u, tm_mem_s;
   if (!encode_2d(&tm_x0, a.x0, d, static_cast<uint64_t>(T), d, kBlockM) ||
       !encode_slabs(&tm_x0_s, a.x0, d, static_cast<uint64_t>(T), d, kBlockM) ||
       !encode_slabs(&tm_hs, a.H, n1, static_cast<uint64_t>(T), a.hld, kBlockM, ks) ||
       !encode_2d(&tm_h, a.H, n1, static_cast<uint64_t>(T), a.hld, kBlockM) ||
+      !encode_2d(&tm_hst, a.H, n1, static_cast<uint64_t>(T), a.hld, 32) ||
       !encode_2d(&tm_u, v.Uup, v.r_pad, static_cast<uint64_t>(L) * d, v.uup_ld, cw) ||
       !encode_slabs(&tm_mem_s, a.mem, d, static_cast<uint64_t>(L) * T, d, kBlockM))
     return cudaErrorInvalidValue;
   // split chain: the low parts of h (its own buffer, H's pitch) and of the products
-  CUtensorMap tm_hlo_s = tm_hs, tm_hlo = tm_h;
+  CUtensorMap tm_hlo_s = tm_hs, tm_hlo = tm_h, tm_hlo_st = tm_hst;
   if (split && (!encode_slabs(&tm_hlo_s, a.Hlo, n1, static_cast<uint64_t>(T), a.hld, kBlockM, ks) ||
-                !encode_2d(&tm_hlo, a.Hlo, n1, static_cast<uint64_t>(T), a.hld, kBlockM)))
+                !encode_2d(&tm_hlo, a.Hlo, n1, static_cast<uint64_t>(T), a.hld, kBlockM) ||
+                !encode_2d(&tm_hlo_st, a.Hlo, n1, static_cast<uint64_t>(T), a.hld, 32)))
     return cudaErrorInvalidValue;
   const CUtensorMap& tm_pf_lo = split ? *v.tm_Pf_lo : *v.tm_Pf;
   mark(0);
@@ -897,8 +900,8 @@ static cudaError_t enqueue_fold(const PlanView& v, const BuildArgs& a, cudaStrea
   const long long part_ld = static_cast<long long>(d / 64) * T;
   if (err == cudaSuccess)
     err = launch_hchain(v.r_pad, split, T, L, a.c, static_cast<int>(n1), tm_hs, tm_hlo_s, *v.tm_Pf,
-                        tm_pf_lo, a.H, split ? a.Hlo : nullptr, static_cast<int>(a.hld), v.status,
-                        kTimeoutNs, st);
+                        tm_pf_lo, tm_hst, tm_hlo_st, a.H, split ? a.Hlo : nullptr,
+                        static_cast<int>(a.hld), v.status, kTimeoutNs, st);
   if (err == cudaSuccess)
     err = launch_accum(v.r_pad, cw, T, L, d, a.x0, tm_h, tm_hlo, split, tm_u, a.mem, a.part, part_ld,
                        v.status, kTimeoutNs, st);
@@ -1288,8 +1291,8 @@ cudaError_t preload_build_kernels(const dv_plan* p) {
   for (int nt : {64, 128, 192, 256}) keep(dv::launch_kv_pair(hd, nt, m, m, m, gp, 1, nullptr));
   if (p->fold) {
     const int cw = dv::fold_slice_cols(p->cfg.d);
-    keep(dv::launch_hchain(p->r_pad, p->cfg.split_chain != 0, 0, 1, nullptr, 0, m, m, m, m, nullptr,
-                           nullptr, 0, nullptr, 0, nullptr));
+    keep(dv::launch_hchain(p->r_pad, p->cfg.split_chain != 0, 0, 1, nullptr, 0, m, m, m, m, m, m,
+                           nullptr, nullptr, 0, nullptr, 0, nullptr));
     keep(dv::launch_accum(p->r_pad, cw, 0, 1, p->cfg.d, nullptr, m, m, false, m, nullptr, nullptr, 0,
                           nullptr, 0, nullptr));
   }

@@ -69,6 +69,19 @@ __device__ __forceinline__ void tma_load_slabs(uint32_t dst, const CUtensorMap* 
       : "memory");
 }
 
+// 2-D tiled store of a shared-memory box to global memory (bulk-group completion), and the
+// group's commit and wait (writes complete: the source may be rewritten and the data is in
+// global memory).
+__device__ __forceinline__ void tma_store_2d(const CUtensorMap* map, uint32_t src, int x, int y) {
+  asm volatile("cp.async.bulk.tensor.2d.global.shared::cta.bulk_group [%0, {%2, %3}], [%1];" ::"l"(
+                   reinterpret_cast<uint64_t>(map)),
+               "r"(src), "r"(x), "r"(y)
+               : "memory");
+}
+__device__ __forceinline__ void bulk_commit_wait() {
+  asm volatile("cp.async.bulk.commit_group;\n\tcp.async.bulk.wait_group 0;" ::: "memory");
+}
+
 template <int RP, int KS, int STAGES, bool SPLIT, bool PAIR>
 struct HCfg {
   static constexpr int R = RP / 64;              // 64-wide K slabs per r_pad
@@ -129,8 +142,12 @@ __device__ __forceinline__ HSeg hseg(int l, int seg, int R) {
 // read). Two accumulators alternate by layer: layer l's MMAs over the older h_j run while the
 // epilogue of layer l - 1 still works. The epilogue applies SiLU (layer 0 straight from C_0),
 // writes bf16 h_l to the h tile (the A operand of layer l + 1's last segments; with the split, its
-// low part to a second tile) and to H (read back by TMA from layer l + 2 on, and by the running
-// sum), then loads C_{l+2} into the accumulator it has just read.
+// low part to a second tile), loads C_{l+2} into the accumulator it has just read, and stores
+// its rows of the tiles to H by TMA (read back by TMA from layer l + 2 on, and by the running
+// sum). The per-layer chain (accumulator full -> readback -> h tile -> layer l + 1's last MMAs)
+// sets the pace, so everything else stays off it: at r_pad <= 128 C_{l+2} is fetched into
+// registers a layer ahead, and the producer waits for h_{l-2} in H only before the box that
+// reads it, the last of the older segment.
 // Barriers (all waits bounded): stage full / empty; accumulator full; accumulator loaded with C;
 // the h tile written (once per layer); h_l in global memory, alternating between two barriers by
 // layer parity so that the producer, which may run up to two layers ahead of the epilogue, never
@@ -146,6 +163,7 @@ template <int RP, int KS, int STAGES, bool SPLIT, bool PAIR>
 __global__ void __launch_bounds__(kFoldThreads, 1)
     dv_hchain_kernel(const __grid_constant__ CUtensorMap tmH, const __grid_constant__ CUtensorMap tmHlo,
                      const __grid_constant__ CUtensorMap tmP, const __grid_constant__ CUtensorMap tmPlo,
+                     const __grid_constant__ CUtensorMap tmHst, const __grid_constant__ CUtensorMap tmHlost,
                      const __grid_constant__ HChainParams p) {
   using C = HCfg<RP, KS, STAGES, SPLIT, PAIR>;
   constexpr int kSegs = SPLIT ? 6 : 2;
@@ -226,17 +244,21 @@ __global__ void __launch_bounds__(kFoldThreads, 1)
       uint32_t phase = 0, used = 0, issued_parity = 0;
       bool ok = true;
       for (int l = 1; l < p.L && ok; ++l) {
+        bool newest_in_h = false;
         for (int seg = 0; seg < kSegs && ok; ++seg) {
           const HSeg g = hseg<SPLIT>(l, seg, R);
-          // h_{l-2} is the newest layer the older segments read: wait until it is in global
-          // memory (the layers before it were published earlier)
-          if (seg == 0 && g.n > 0 &&
-              !mbar_wait(hpub_bar((l - 2) & 1), static_cast<uint32_t>((l - 2) >> 1) & 1u, abort_flag,
-                         tmo)) {
-            ok = false;
-            break;
-          }
           for (int s0 = 0; s0 < g.n; s0 += KS) {
+            // h_{l-2}, the newest layer the older segments read, fills their last R slabs: wait
+            // until it is in global memory before the first box that covers one of them (the
+            // layers before it were published earlier)
+            if (g.asrc < 2 && !newest_in_h && s0 + KS > (l - 2) * R) {
+              if (!mbar_wait(hpub_bar((l - 2) & 1), static_cast<uint32_t>((l - 2) >> 1) & 1u,
+                             abort_flag, tmo)) {
+                ok = false;
+                break;
+              }
+              newest_in_h = true;
+            }
             if (!mbar_wait(empty_bar(stage), phase ^ 1u, abort_flag, tmo)) {
               ok = false;
               break;
@@ -350,6 +372,10 @@ __global__ void __launch_bounds__(kFoldThreads, 1)
     const float* crow = p.C + static_cast<long long>(live ? t : 0) * p.ldc;
     uint8_t* hrow = base_ptr + C::kOffH;
     uint8_t* lrow = base_ptr + C::kOffL;
+    // At r_pad <= 128 a row of C_{l+2} (r_pad fp32) is fetched into registers one layer before it
+    // goes into TMEM, so its global-memory latency is not on the per-layer chain.
+    constexpr bool kAhead = RP <= 128;
+    uint32_t cnext[kAhead ? RP / 32 : 1][32];
     // this row's 32 columns c*32 .. of C_lc (zero past the build's tokens)
     auto load_c = [&](int lc, int c, uint32_t (&r)[32]) {
       const float4* src = reinterpret_cast<const float4*>(crow + lc * RP + c * 32);
@@ -362,15 +388,13 @@ __global__ void __launch_bounds__(kFoldThreads, 1)
         r[4 * k + 3] = __float_as_uint(v.w);
       }
     };
-    // C_lc into accumulator a, the starting value of layer lc's GEMM
-    auto put_c = [&](int lc, int a) {
-#pragma unroll 1
-      for (int c = 0; c < RP / 32; ++c) {
-        uint32_t r[32];
-        load_c(lc, c, r);
-        __syncwarp();
-        tmem_st32x(tl + static_cast<uint32_t>(a * RP + c * 32), r);
+    auto fetch_c = [&](int lc) {
+      if constexpr (kAhead) {
+#pragma unroll
+        for (int c = 0; c < RP / 32; ++c) load_c(lc, c, cnext[c]);
       }
+    };
+    auto loaded = [&](int a) {  // accumulator a holds its C
       asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
       tc_fence_before();
       if (PAIR) {  // one lane per warp on the leader's barrier, for the warp's 32 rows
@@ -379,6 +403,27 @@ __global__ void __launch_bounds__(kFoldThreads, 1)
       } else {
         mbar_arrive(init_bar(a));
       }
+    };
+    // C_lc into accumulator a, the starting value of layer lc's GEMM: from the registers fetched
+    // a layer ahead, else straight from global memory
+    auto put_c = [&](int lc, int a) {
+      if constexpr (kAhead) {
+        (void)lc;
+#pragma unroll
+        for (int c = 0; c < RP / 32; ++c) {
+          __syncwarp();
+          tmem_st32x(tl + static_cast<uint32_t>(a * RP + c * 32), cnext[c]);
+        }
+      } else {
+#pragma unroll 1
+        for (int c = 0; c < RP / 32; ++c) {
+          uint32_t r[32];
+          load_c(lc, c, r);
+          __syncwarp();
+          tmem_st32x(tl + static_cast<uint32_t>(a * RP + c * 32), r);
+        }
+      }
+      loaded(a);
     };
     // SiLU of the 32 columns c*32 .. of z into the h tile (bf16, swizzled as the MMA reads it);
     // split: the remainder h - bf16(h), itself in bf16, into the low tile
@@ -422,8 +467,7 @@ __global__ void __launch_bounds__(kFoldThreads, 1)
           put_h(c, r);
         }
       }
-      // The h tile first (the next layer's MMA waits for it; async proxy), then the copy of h_l
-      // in H (TMA loads two or more layers later, and the running sum): read back from the tile.
+      // The h tile first: layer l + 1's last MMAs wait for it (async proxy reads).
       asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
       if (PAIR) {
         __syncwarp();
@@ -431,28 +475,42 @@ __global__ void __launch_bounds__(kFoldThreads, 1)
       } else {
         mbar_arrive(htile_bar);
       }
-      if (live) {
-        const long long go = static_cast<long long>(t) * p.ldh + l * RP;
-        uint4* hg = reinterpret_cast<uint4*>(p.H + go);
-#pragma unroll 1
-        for (int c8 = 0; c8 < RP / 8; ++c8)
-          hg[c8] = *reinterpret_cast<const uint4*>(hrow + (c8 / 8) * kSlabA + swz(row, c8 % 8));
-        if (SPLIT) {
-          uint4* lg = reinterpret_cast<uint4*>(p.Hlo + go);
-#pragma unroll 1
-          for (int c8 = 0; c8 < RP / 8; ++c8)
-            lg[c8] = *reinterpret_cast<const uint4*>(lrow + (c8 / 8) * kSlabA + swz(row, c8 % 8));
-        }
-      }
-      asm volatile("fence.proxy.async.global;" ::: "memory");
-      mbar_arrive(hpub_bar(l & 1));
-      // the accumulator just read starts layer l + 2; before layer 1 both start
+      // Then the accumulator just read starts layer l + 2 (before layer 1 both start), and the
+      // C of the layer after that is fetched.
       if (l == 0) {
-        if (p.L > 1) put_c(1, 1);
-        if (p.L > 2) put_c(2, 0);
-      } else if (l + 2 < p.L) {
-        put_c(l + 2, l & 1);
+        if constexpr (kAhead) {
+          if (p.L > 1) {
+            fetch_c(1);
+            put_c(1, 1);
+          }
+          if (p.L > 2) {
+            fetch_c(2);
+            put_c(2, 0);
+          }
+        } else {
+          if (p.L > 1) put_c(1, 1);
+          if (p.L > 2) put_c(2, 0);
+        }
+        if (p.L > 3) fetch_c(3);
+      } else {
+        if (l + 2 < p.L) put_c(l + 2, l & 1);
+        if (l + 3 < p.L) fetch_c(l + 3);
       }
+      // Last, the warp's 32 rows of h_l (and of its low part) go from the tiles to H by TMA;
+      // complete before the tiles are rewritten and before the producer may read them back.
+      // Rows past the build's tokens are clipped; a warp with none of them stores nothing.
+      __syncwarp();
+      if (lane == 0 && row0 + qq * 32 < p.M) {
+#pragma unroll
+        for (int sl = 0; sl < R; ++sl) {
+          const uint32_t src = static_cast<uint32_t>(sl * kSlabA + qq * 32 * 128);
+          tma_store_2d(&tmHst, htile + src, l * RP + 64 * sl, row0 + qq * 32);
+          if (SPLIT) tma_store_2d(&tmHlost, ltile + src, l * RP + 64 * sl, row0 + qq * 32);
+        }
+        bulk_commit_wait();
+      }
+      __syncwarp();
+      mbar_arrive(hpub_bar(l & 1));
     }
   }
 
@@ -733,8 +791,8 @@ __global__ void __launch_bounds__(ACfg<RP, CW, STAGES, EW>::kThreads, 1)
 
 template <int RP, int KS, int ST, bool SPLIT>
 cudaError_t hchain_t(long long blocks, const CUtensorMap& h, const CUtensorMap& hlo,
-                     const CUtensorMap& pf, const CUtensorMap& pflo, const HChainParams& p,
-                     cudaStream_t stream) {
+                     const CUtensorMap& pf, const CUtensorMap& pflo, const CUtensorMap& hst,
+                     const CUtensorMap& hlost, const HChainParams& p, cudaStream_t stream) {
   // CTA pairs: two token blocks per cluster (the last pair may hold a block past the build)
   using C = HCfg<RP, KS, ST, SPLIT, true>;
   auto kern = dv_hchain_kernel<RP, KS, ST, SPLIT, true>;
@@ -753,7 +811,7 @@ cudaError_t hchain_t(long long blocks, const CUtensorMap& h, const CUtensorMap& 
   cfg.stream = stream;
   cfg.attrs = attr;
   cfg.numAttrs = 2;
-  err = cudaLaunchKernelEx(&cfg, kern, h, hlo, pf, pflo, p);
+  err = cudaLaunchKernelEx(&cfg, kern, h, hlo, pf, pflo, hst, hlost, p);
   if (err != cudaSuccess) return err;
   return cudaGetLastError();
 }
@@ -801,8 +859,9 @@ int fold_sum_parts(int d) {
 
 cudaError_t launch_hchain(int r_pad, bool split, long long tokens, int n_layers, const float* C,
                           int ldc, const CUtensorMap& h, const CUtensorMap& hlo,
-                          const CUtensorMap& pf, const CUtensorMap& pflo, uint16_t* H, uint16_t* Hlo,
-                          int ldh, int* status, unsigned long long timeout_ns, cudaStream_t stream) {
+                          const CUtensorMap& pf, const CUtensorMap& pflo, const CUtensorMap& hst,
+                          const CUtensorMap& hlost, uint16_t* H, uint16_t* Hlo, int ldh, int* status,
+                          unsigned long long timeout_ns, cudaStream_t stream) {
   HChainParams p;
   p.M = static_cast<int>(tokens);
   p.L = n_layers;
@@ -818,18 +877,18 @@ cudaError_t launch_hchain(int r_pad, bool split, long long tokens, int n_layers,
   // the high one
   if (split) {
     switch (r_pad) {
-      case 64: return hchain_t<64, 2, 4, true>(blocks, h, hlo, pf, pflo, p, stream);
-      case 128: return hchain_t<128, 2, 3, true>(blocks, h, hlo, pf, pflo, p, stream);
-      case 192: return hchain_t<192, 1, 4, true>(blocks, h, hlo, pf, pflo, p, stream);
-      case 256: return hchain_t<256, 1, 3, true>(blocks, h, hlo, pf, pflo, p, stream);
+      case 64: return hchain_t<64, 2, 4, true>(blocks, h, hlo, pf, pflo, hst, hlost, p, stream);
+      case 128: return hchain_t<128, 2, 3, true>(blocks, h, hlo, pf, pflo, hst, hlost, p, stream);
+      case 192: return hchain_t<192, 1, 4, true>(blocks, h, hlo, pf, pflo, hst, hlost, p, stream);
+      case 256: return hchain_t<256, 1, 3, true>(blocks, h, hlo, pf, pflo, hst, hlost, p, stream);
       default: return cudaErrorInvalidValue;
     }
   }
   switch (r_pad) {
-    case 64: return hchain_t<64, 2, 5, false>(blocks, h, hlo, pf, pflo, p, stream);
-    case 128: return hchain_t<128, 2, 4, false>(blocks, h, hlo, pf, pflo, p, stream);
-    case 192: return hchain_t<192, 2, 3, false>(blocks, h, hlo, pf, pflo, p, stream);
-    case 256: return hchain_t<256, 1, 5, false>(blocks, h, hlo, pf, pflo, p, stream);
+    case 64: return hchain_t<64, 2, 5, false>(blocks, h, hlo, pf, pflo, hst, hlost, p, stream);
+    case 128: return hchain_t<128, 2, 4, false>(blocks, h, hlo, pf, pflo, hst, hlost, p, stream);
+    case 192: return hchain_t<192, 2, 3, false>(blocks, h, hlo, pf, pflo, hst, hlost, p, stream);
+    case 256: return hchain_t<256, 1, 5, false>(blocks, h, hlo, pf, pflo, hst, hlost, p, stream);
     default: return cudaErrorInvalidValue;
   }
 }

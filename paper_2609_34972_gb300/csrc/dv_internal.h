@@ -230,7 +230,8 @@ cudaError_t launch_chain(int r_pad, int spc, int S, long long tokens, int n_laye
 // Q_lj = D_l U_j for j < l):
 //   launch_hchain: h_l = SiLU(C_l + sum_{j<l} h_j Q_lj^T) into H ([tokens][ldh], h_l at columns
 //     l r_pad), one CTA per 128-token block. Maps: h: slab map over H with 128-row boxes; pf:
-//     slab map over Pf with r_pad-row boxes.
+//     slab map over Pf with r_pad-row boxes; hst: H as a 2-D map with 32-row boxes (the
+//     stores of h_l).
 //   launch_accum: M_l = E + sum_{j<=l} h_j U_j^T, bf16 into the stacked memories mem
 //     ([L][tokens][d]) and each row's partial sums of M_l^2 into part (fold_sum_parts(d)
 //     partials per layer, at most d / 64). h: H with 128-row boxes; u: U as [L d][r_pad] with
@@ -239,17 +240,18 @@ cudaError_t launch_chain(int r_pad, int spc, int S, long long tokens, int n_laye
 // fold_sum_parts: the partial sums of squares per token and layer that launch_accum writes.
 // hchain_box_slabs: K slabs per TMA box of launch_hchain's maps (h and pf are slab maps,
 // encode_slabs, with boxes of that many slabs).
-// split (split_chain): h_l also as its low bf16 part Hlo (hlo: its maps, as h's), and Pf_lo
+// split (split_chain): h_l also as its low bf16 part Hlo (hlo, hlost: its maps, as h's and hst's), and Pf_lo
 // (pflo: its map, as pf's), the low part of the products: each product is taken in three parts,
 // h_hi Q_hi + h_lo Q_hi + h_hi Q_lo, and the running sum adds h_hi U + h_lo U. Without the split
-// hlo and pflo are not read.
+// hlo, hlost and pflo are not used.
 int fold_slice_cols(int d);
 int fold_sum_parts(int d);
 int hchain_box_slabs(int r_pad, bool split);
 cudaError_t launch_hchain(int r_pad, bool split, long long tokens, int n_layers, const float* C,
                           int ldc, const CUtensorMap& h, const CUtensorMap& hlo,
-                          const CUtensorMap& pf, const CUtensorMap& pflo, uint16_t* H, uint16_t* Hlo,
-                          int ldh, int* status, unsigned long long timeout_ns, cudaStream_t stream);
+                          const CUtensorMap& pf, const CUtensorMap& pflo, const CUtensorMap& hst,
+                          const CUtensorMap& hlost, uint16_t* H, uint16_t* Hlo, int ldh, int* status,
+                          unsigned long long timeout_ns, cudaStream_t stream);
 cudaError_t launch_accum(int r_pad, int cw, long long tokens, int n_layers, int d,
                          const void* x0, const CUtensorMap& h, const CUtensorMap& hlo, bool split,
                          const CUtensorMap& u, uint16_t* mem, float* part, long long part_ld,
