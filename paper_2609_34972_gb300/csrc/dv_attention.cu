@@ -197,7 +197,7 @@ __device__ __forceinline__ void tmem_st_wait() {
 
 __device__ __forceinline__ bool wait_bounded(uint32_t bar, uint32_t parity, uint64_t timeout_ns) {
   int never = 0;
-  return mbar_wait(bar, parity, &never, timeout_ns);
+  return mbar_wait<false>(bar, parity, &never, timeout_ns);
 }
 
 // Partial rows travel between the CTAs of a cluster as fp32 rows of HD / 4 16-byte chunks,
@@ -567,8 +567,8 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
   };
   auto issue_s = [&](int j) {  // thread 0: S_j = Q K_j^T into score buffer j % kSBuf
     const int st = j % NST;
-    if (mbar_wait(bar_q, 0, abort_flag, tmo) &&
-        mbar_wait(bar_k(st), static_cast<uint32_t>(j / NST) & 1u, abort_flag, tmo)) {
+    if (mbar_wait<false>(bar_q, 0, abort_flag, tmo) &&
+        mbar_wait<false>(bar_k(st), static_cast<uint32_t>(j / NST) & 1u, abort_flag, tmo)) {
       tc_fence_after();
       const uint32_t idesc = idesc_bf16_f32(128, kKeyBlock);
       for (int ds = 0; ds < C::kSlabs; ++ds)
@@ -604,7 +604,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
     }
 
     // Scores -> probabilities (this thread: query row tid).
-    ok = mbar_wait(bar_s, ph, abort_flag, tmo);
+    ok = mbar_wait<false>(bar_s, ph, abort_flag, tmo);
     if (NST == 1 && tid == 0 && ok && j + 1 < n_mine) load_k(j + 1);  // K slot read
     if (__all_sync(0xFFFFFFFFu, ok)) {
       tc_fence_after();
@@ -684,7 +684,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
 
     // O (+)= P V in TMEM; the CTA's first block initialises O. V is read as it lies ([keys]
     // [channels], an MN-major B operand); P (A, K-major) from TMEM, 16 keys = 8 columns.
-    if (ok && tid == 0 && mbar_wait(bar_v(st), sph, abort_flag, tmo)) {
+    if (ok && tid == 0 && mbar_wait<false>(bar_v(st), sph, abort_flag, tmo)) {
       tc_fence_after();
       const uint32_t idesc = idesc_bf16_f32(128, HD) | (1u << 16);
 #pragma unroll
@@ -697,7 +697,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
       // P V, which has completed).
       if (C::kSBuf == 2 && j + 1 < n_mine) issue_s(j + 1);
     }
-    ok = ok && mbar_wait(bar_o, ph, abort_flag, tmo);
+    ok = ok && mbar_wait<false>(bar_o, ph, abort_flag, tmo);
     if (NST == 1 && tid == 0 && ok && j + 1 < n_mine) {
       load_v(j + 1);  // V slot read
       issue_s(j + 1);  // P_j (in the one score buffer) read
