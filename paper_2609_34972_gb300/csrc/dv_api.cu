@@ -146,6 +146,22 @@ bool encode_3d(CUtensorMap* map, const void* ptr, uint64_t cols, uint64_t rows, 
             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+// The same [L][rows][cols] bf16 tensor for stores of one warp's 32 x 32 block: boxes of 32
+// columns x 32 rows x 1 layer with 64-byte swizzle (a 16-byte chunk q of staged row r sits at
+// chunk q ^ ((r / 2) mod 4) of its 64-byte row); a store past `rows` is clipped per layer.
+bool encode_3d_warp_store(CUtensorMap* map, const void* ptr, uint64_t cols, uint64_t rows,
+                          uint64_t layers) {
+  EncodeTiledFn fn = encode_fn();
+  if (!fn) return false;
+  cuuint64_t dims[3] = {cols, rows, layers};
+  cuuint64_t strides[2] = {cols * 2, cols * rows * 2};
+  cuuint32_t box[3] = {32, 32, 1};
+  cuuint32_t estr[3] = {1, 1, 1};
+  return fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(ptr), dims, strides, box,
+            estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_64B,
+            CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
 // Launch of a build kernel with programmatic stream serialization (dv::pdl_attribute); the
 // kernel calls dv::pdl_wait() before touching global memory, except where it states otherwise
 // (k_row_sumsq).
@@ -846,15 +862,17 @@ static cudaError_t enqueue_fold(const PlanView& v, const BuildArgs& a, cudaStrea
   };
   const bool split = v.split_chain != 0;
   const uint32_t ks = static_cast<uint32_t>(hchain_box_slabs(v.r_pad, split));
-  // tm_hst: the recurrence's stores of h_l, 32 rows (one epilogue warp) per box
-  CUtensorMap tm_x0, tm_x0_s, tm_hs, tm_h, tm_hst, tm_u, tm_mem_s;
+  // tm_hst: the recurrence's stores of h_l, 32 rows (one epilogue warp) per box; tm_mem_w: the
+  // running sum's stores of M_l, one warp's 32 x 32 block per box
+  CUtensorMap tm_x0, tm_x0_s, tm_hs, tm_h, tm_hst, tm_u, tm_mem_s, tm_mem_w;
   if (!encode_2d(&tm_x0, a.x0, d, static_cast<uint64_t>(T), d, kBlockM) ||
       !encode_slabs(&tm_x0_s, a.x0, d, static_cast<uint64_t>(T), d, kBlockM) ||
       !encode_slabs(&tm_hs, a.H, n1, static_cast<uint64_t>(T), a.hld, kBlockM, ks) ||
       !encode_2d(&tm_h, a.H, n1, static_cast<uint64_t>(T), a.hld, kBlockM) ||
       !encode_2d(&tm_hst, a.H, n1, static_cast<uint64_t>(T), a.hld, 32) ||
       !encode_2d(&tm_u, v.Uup, v.r_pad, static_cast<uint64_t>(L) * d, v.uup_ld, cw) ||
-      !encode_slabs(&tm_mem_s, a.mem, d, static_cast<uint64_t>(L) * T, d, kBlockM))
+      !encode_slabs(&tm_mem_s, a.mem, d, static_cast<uint64_t>(L) * T, d, kBlockM) ||
+      !encode_3d_warp_store(&tm_mem_w, a.mem, d, static_cast<uint64_t>(T), L))
     return cudaErrorInvalidValue;
   // split chain: the low parts of h (its own buffer, H's pitch) and of the products
   CUtensorMap tm_hlo_s = tm_hs, tm_hlo = tm_h, tm_hlo_st = tm_hst;
@@ -903,7 +921,7 @@ static cudaError_t enqueue_fold(const PlanView& v, const BuildArgs& a, cudaStrea
                         tm_pf_lo, tm_hst, tm_hlo_st, a.H, split ? a.Hlo : nullptr,
                         static_cast<int>(a.hld), v.status, kTimeoutNs, st);
   if (err == cudaSuccess)
-    err = launch_accum(v.r_pad, cw, T, L, d, a.x0, tm_h, tm_hlo, split, tm_u, a.mem, a.part, part_ld,
+    err = launch_accum(v.r_pad, cw, T, L, d, a.x0, tm_h, tm_hlo, split, tm_u, tm_mem_w, a.part, part_ld,
                        v.status, kTimeoutNs, st);
   mark(2);
   if (err == cudaSuccess)
@@ -1293,7 +1311,7 @@ cudaError_t preload_build_kernels(const dv_plan* p) {
     const int cw = dv::fold_slice_cols(p->cfg.d);
     keep(dv::launch_hchain(p->r_pad, p->cfg.split_chain != 0, 0, 1, nullptr, 0, m, m, m, m, m, m,
                            nullptr, nullptr, 0, nullptr, 0, nullptr));
-    keep(dv::launch_accum(p->r_pad, cw, 0, 1, p->cfg.d, nullptr, m, m, false, m, nullptr, nullptr, 0,
+    keep(dv::launch_accum(p->r_pad, cw, 0, 1, p->cfg.d, nullptr, m, m, false, m, m, nullptr, 0,
                           nullptr, 0, nullptr));
   }
   if (p->cfg.adapter == DV_ADAPTER_RECURRENT) {

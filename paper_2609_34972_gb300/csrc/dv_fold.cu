@@ -536,8 +536,10 @@ __global__ void __launch_bounds__(kFoldThreads, 1)
 
 // ---------------------------------------------------------------- (3) the running sum
 
-// Shared staging of one warp's bf16 stores (warp_store_bf16: 32 rows of 20 words).
-constexpr int kBf16StageFloats = 32 * 20;
+// Shared staging of one warp's 32 x 32 bf16 block for its TMA store: 32 rows of 64 bytes, the
+// 16-byte chunk q of row r at chunk q ^ ((r / 2) mod 4) (the tensor map's 64-byte swizzle). Two
+// per warp, alternating, so that a block is staged while the previous one is still being read.
+constexpr int kStageBytes = 32 * 64;
 
 template <int RP, int CW, int STAGES, int EW>
 struct ACfg {
@@ -548,7 +550,7 @@ struct ACfg {
   static constexpr int kSlabB = CW * 128;            // [CW rows of U_l][64] bf16
   static constexpr int kStage = 2 * kSlabA + kSlabB; // h slabs of the two token blocks, U slab
   static constexpr int kOffWarp = STAGES * kStage;   // per-warp staging of the M_l stores
-  static constexpr int kEnd = kOffWarp + 4 * EW * kBf16StageFloats * 4;
+  static constexpr int kEnd = kOffWarp + 4 * EW * 2 * kStageBytes;
   static_assert(kCols % 32 == 0 && CW / 64 >= EW, "whole 32-column chunks; parts fit d / 64");
   static constexpr int kSmemBytes = kEnd + 1024 + 256;
   static constexpr int kTmemCols = 2 * CW <= 256 ? 256 : 512;
@@ -562,7 +564,6 @@ struct AccumParams {
   int d;
   int S;               // hidden slices (d / CW)
   const uint16_t* x0;  // bf16 [M][d]
-  uint16_t* mem;       // bf16 [L][M][d]: the stacked M_l
   float* part;         // fp32 [L][part_ld / M][M]: sums of squares of M_l per CW / EW columns
   long long part_ld;
   int split;           // 1: h_l in two bf16 parts (H, then Hlo), both against U_l
@@ -582,7 +583,8 @@ struct AccumParams {
 template <int RP, int CW, int STAGES, int EW>
 __global__ void __launch_bounds__(ACfg<RP, CW, STAGES, EW>::kThreads, 1)
     dv_accum_kernel(const __grid_constant__ CUtensorMap tmH, const __grid_constant__ CUtensorMap tmHlo,
-                    const __grid_constant__ CUtensorMap tmU, const __grid_constant__ AccumParams p) {
+                    const __grid_constant__ CUtensorMap tmU, const __grid_constant__ CUtensorMap tmM,
+                    const __grid_constant__ AccumParams p) {
   using C = ACfg<RP, CW, STAGES, EW>;
   constexpr int R = C::R;
   const int nq = p.split ? 2 * R : R;  // K slabs per layer: h_l (and its low part), 64 wide
@@ -717,7 +719,9 @@ __global__ void __launch_bounds__(ACfg<RP, CW, STAGES, EW>::kThreads, 1)
     const int row = qq * 32 + lane;
     const int cw0 = eh * C::kCols;    // the warp's first column in the slice
     const uint32_t tl = tmem + (static_cast<uint32_t>(qq * 32) << 16) + static_cast<uint32_t>(cw0);
-    float* wstage = reinterpret_cast<float*>(base_ptr + C::kOffWarp) + (warp - 2) * kBf16StageFloats;
+    const uint32_t wstage = base + static_cast<uint32_t>(C::kOffWarp + (warp - 2) * 2 * kStageBytes);
+    uint8_t* wstage_ptr = base_ptr + C::kOffWarp + (warp - 2) * 2 * kStageBytes;
+    int nstored = 0;  // blocks this warp has stored: the staging buffer alternates with it
     // M_0 = E: the fp32 widening of this row's columns of E into both accumulators
 #pragma unroll 1
     for (int b = 0; b < 2; ++b) {
@@ -771,13 +775,37 @@ __global__ void __launch_bounds__(ACfg<RP, CW, STAGES, EW>::kThreads, 1)
         tc_fence_before();
         mbar_arrive(accr_bar(b));
         const int t0 = row0 + b * 128 + qq * 32;  // the warp's first row
-        uint16_t* dst = p.mem + (static_cast<long long>(l) * p.M + t0) * p.d + col0 + cw0;
+        // each 32 x 32 block: staged (lane i's row i, swizzled), then one TMA store by lane 0
+        // (rows past the build's tokens are clipped by the map); before a buffer is restaged,
+        // the store issued from it two blocks earlier has finished reading it
 #pragma unroll
-        for (int c = 0; c < C::kCols / 32; ++c) warp_store_bf16(wstage, pk[c], dst + c * 32, p.d, p.M - t0);
+        for (int c = 0; c < C::kCols / 32; ++c, ++nstored) {
+          const int sb = nstored & 1;
+          if (lane == 0 && nstored >= 2) asm volatile("cp.async.bulk.wait_group.read 1;" ::: "memory");
+          __syncwarp();
+          uint8_t* st = wstage_ptr + sb * kStageBytes;
+#pragma unroll
+          for (int q = 0; q < 4; ++q)
+            *reinterpret_cast<uint4*>(st + lane * 64 + ((q ^ ((lane >> 1) & 3)) << 4)) =
+                make_uint4(pk[c][4 * q], pk[c][4 * q + 1], pk[c][4 * q + 2], pk[c][4 * q + 3]);
+          asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+          __syncwarp();
+          if (lane == 0 && t0 < p.M) {
+            asm volatile(
+                "cp.async.bulk.tensor.3d.global.shared::cta.bulk_group [%0, {%2, %3, %4}], [%1];" ::"l"(
+                    reinterpret_cast<uint64_t>(&tmM)),
+                "r"(wstage + static_cast<uint32_t>(sb * kStageBytes)), "r"(col0 + cw0 + c * 32), "r"(t0), "r"(l)
+                : "memory");
+          }
+          if (lane == 0) asm volatile("cp.async.bulk.commit_group;" ::: "memory");
+        }
         if (t0 + lane < p.M)
           p.part[l * p.part_ld + static_cast<long long>(sl * EW + eh) * p.M + t0 + lane] = ss;
       }
     }
+    // every store has left shared memory and reached global memory before the CTA exits
+    if (lane == 0) asm volatile("cp.async.bulk.wait_group 0;" ::: "memory");
+    __syncwarp();
   }
 
   tc_fence_before();
@@ -818,7 +846,8 @@ cudaError_t hchain_t(long long blocks, const CUtensorMap& h, const CUtensorMap& 
 
 template <int RP, int CW, int ST, int EW>
 cudaError_t accum_t(long long ctas, const CUtensorMap& h, const CUtensorMap& hlo,
-                    const CUtensorMap& u, const AccumParams& p, cudaStream_t stream) {
+                    const CUtensorMap& u, const CUtensorMap& m, const AccumParams& p,
+                    cudaStream_t stream) {
   using C = ACfg<RP, CW, ST, EW>;
   auto kern = dv_accum_kernel<RP, CW, ST, EW>;
   cudaError_t err = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, C::kSmemBytes);
@@ -831,7 +860,7 @@ cudaError_t accum_t(long long ctas, const CUtensorMap& h, const CUtensorMap& hlo
   cfg.stream = stream;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
-  err = cudaLaunchKernelEx(&cfg, kern, h, hlo, u, p);
+  err = cudaLaunchKernelEx(&cfg, kern, h, hlo, u, m, p);
   if (err != cudaSuccess) return err;
   return cudaGetLastError();
 }
@@ -895,7 +924,7 @@ cudaError_t launch_hchain(int r_pad, bool split, long long tokens, int n_layers,
 
 cudaError_t launch_accum(int r_pad, int cw, long long tokens, int n_layers, int d,
                          const void* x0, const CUtensorMap& h, const CUtensorMap& hlo, bool split,
-                         const CUtensorMap& u, uint16_t* mem, float* part, long long part_ld,
+                         const CUtensorMap& u, const CUtensorMap& mem, float* part, long long part_ld,
                          int* status, unsigned long long timeout_ns, cudaStream_t stream) {
   AccumParams p;
   p.M = static_cast<int>(tokens);
@@ -903,7 +932,6 @@ cudaError_t launch_accum(int r_pad, int cw, long long tokens, int n_layers, int 
   p.d = d;
   p.S = d / cw;
   p.x0 = static_cast<const uint16_t*>(x0);
-  p.mem = mem;
   p.part = part;
   p.part_ld = part_ld;
   p.split = split ? 1 : 0;
@@ -911,7 +939,7 @@ cudaError_t launch_accum(int r_pad, int cw, long long tokens, int n_layers, int 
   p.timeout_ns = timeout_ns;
   const long long ctas = (tokens + 255) / 256 * p.S;
 #define DV_ACCUM(RPV, CWV, STV) \
-  if (r_pad == RPV && cw == CWV) return accum_t<RPV, CWV, STV, kAccumWarps>(ctas, h, hlo, u, p, stream);
+  if (r_pad == RPV && cw == CWV) return accum_t<RPV, CWV, STV, kAccumWarps>(ctas, h, hlo, u, mem, p, stream);
   DV_ACCUM(64, 256, 3) DV_ACCUM(64, 128, 4)
   DV_ACCUM(128, 256, 3) DV_ACCUM(128, 128, 4)
   DV_ACCUM(192, 256, 3) DV_ACCUM(192, 128, 4)

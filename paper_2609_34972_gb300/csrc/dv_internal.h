@@ -232,10 +232,11 @@ cudaError_t launch_chain(int r_pad, int spc, int S, long long tokens, int n_laye
 //     l r_pad), one CTA per 128-token block. Maps: h: slab map over H with 128-row boxes; pf:
 //     slab map over Pf with r_pad-row boxes; hst: H as a 2-D map with 32-row boxes (the
 //     stores of h_l).
-//   launch_accum: M_l = E + sum_{j<=l} h_j U_j^T, bf16 into the stacked memories mem
-//     ([L][tokens][d]) and each row's partial sums of M_l^2 into part (fold_sum_parts(d)
-//     partials per layer, at most d / 64). h: H with 128-row boxes; u: U as [L d][r_pad] with
-//     cw-row boxes; x0: E, bf16 [tokens][d].
+//   launch_accum: M_l = E + sum_{j<=l} h_j U_j^T, bf16 into the stacked memories ([L][tokens][d],
+//     stored through mem: a 3-D map over them with 32 x 32 boxes and 64-byte swizzle) and each
+//     row's partial sums of M_l^2 into part (fold_sum_parts(d) partials per layer, at most
+//     d / 64). h: H with 128-row boxes; u: U as [L d][r_pad] with cw-row boxes; x0: E, bf16
+//     [tokens][d].
 // fold_slice_cols: the slice width cw (256 or 128 dividing d), or 0.
 // fold_sum_parts: the partial sums of squares per token and layer that launch_accum writes.
 // hchain_box_slabs: K slabs per TMA box of launch_hchain's maps (h and pf are slab maps,
@@ -254,7 +255,7 @@ cudaError_t launch_hchain(int r_pad, bool split, long long tokens, int n_layers,
                           unsigned long long timeout_ns, cudaStream_t stream);
 cudaError_t launch_accum(int r_pad, int cw, long long tokens, int n_layers, int d,
                          const void* x0, const CUtensorMap& h, const CUtensorMap& hlo, bool split,
-                         const CUtensorMap& u, uint16_t* mem, float* part, long long part_ld,
+                         const CUtensorMap& u, const CUtensorMap& mem, float* part, long long part_ld,
                          int* status, unsigned long long timeout_ns, cudaStream_t stream);
 
 // Token tile (64, 128, 192 or 256) of the pair kernel for a build of `tokens` tokens.
