@@ -88,6 +88,18 @@ def test_recurrent_edge_shapes(n_layers, n_vis, batch, path):
 
 
 @pytest.mark.parametrize("path", PATHS)
+@pytest.mark.parametrize("d,rank", [(384, 80), (640, 200)])
+def test_recurrent_narrow_slices(d, rank, path):
+    # d not a multiple of 256: the running sum takes 128-column slices (its second kernel
+    # shape: four stages, two epilogue warps per lane quarter), at r_pad 128 and 256, with a
+    # ragged tail and an odd number of token blocks.
+    cfg = gu.small_config(f"rec_d{d}", d=d, n_layers=3, n_kv_heads=2, n_heads=4, head_dim=128,
+                          rank=rank, n_vis=330, batch=1, x0_sigma=0.5, w_sigma=0.05,
+                          seed=90 + rank, pos_start=7, adapter="recurrent")
+    _full_check(synth.make_inputs(_rec(cfg, recurrent_path=path)), f"recurrent d {d} r {rank}, {path}")
+
+
+@pytest.mark.parametrize("path", PATHS)
 def test_recurrent_tokens_as_m_mrope_bias(path):
     # T = 2 x 256: the K/V launch takes the tokens-as-M engine over the stacked M_l.
     cfg = gu.small_config("rec_tm", d=512, n_layers=3, n_kv_heads=2, n_heads=8, head_dim=128,
