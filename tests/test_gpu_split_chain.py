@@ -42,7 +42,8 @@ PATHS = ["chain", "rearranged"]
 
 
 @pytest.mark.parametrize("path", PATHS)
-@pytest.mark.parametrize("rank,d", [(16, 512), (80, 1024), (150, 768), (256, 512)])
+@pytest.mark.parametrize("rank,d", [(16, 512), (80, 1024), (150, 768), (256, 512), (80, 384),
+                                    (200, 640)])
 def test_split_chain_every_rank_padding(rank, d, path):
     from dataclasses import replace
     cfg = gu.small_config(f"split_r{rank}", d=d, n_layers=3, n_kv_heads=2, n_heads=4, head_dim=128,
